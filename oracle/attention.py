@@ -1,0 +1,183 @@
+"""Oracle: per-segment compact attention, forward and backward, in float64.
+
+TEST INFRASTRUCTURE ONLY (see ``oracle/__init__``).
+
+This is the LogitTree formulation (§4.1; App. E.2 "The five methods"): split
+the rollout at its junctions, materialise each segment's live view as its own
+compact sequence, and run ordinary causal softmax attention on it alone. The
+segment's rows are the tail of that compact sequence, so each row attends to
+the compact prefix up to and including itself. Theorem "materialization
+equivalence" (§4.3, proof in App. C.3) states that the packed 4D-masked
+computation gives the same outputs and gradients; the CUDA path is checked
+against this file.
+
+Layouts (token-major, trajectories packed back to back):
+``Q, O``: ``[T_total, Hq, Dh]``; ``K, V``: ``[T_total, Hkv, Dh]``;
+``LSE``: ``[Hq, T_total]`` (natural log). Query head ``h`` reads KV head
+``h // (Hq // Hkv)`` (contiguous GQA groups).
+"""
+
+import numpy as np
+
+from .visibility import live_views
+
+_ROW_CHUNK = 512
+
+
+def _segments(seqlens, edits_per_traj):
+    """Yield ``(global_rows, global_view_positions, n_before)`` per segment."""
+    base = 0
+    for T, edits in zip(seqlens, edits_per_traj):
+        for lo, hi, view in live_views(T, edits):
+            idx = np.asarray(view, dtype=np.int64) + base
+            yield np.arange(lo, hi, dtype=np.int64) + base, idx, len(view) - (hi - lo)
+        base += T
+
+
+def _scores(q, k, scale, compact_rows):
+    """Scaled scores of compact rows against the compact keys, causal.
+
+    ``compact_rows[r]`` is the compact index of row r of ``q``; that row may
+    see compact keys ``0 .. compact_rows[r]`` and nothing after.
+    """
+    s = (q @ k.T) * scale
+    c = np.arange(k.shape[0])[None, :]
+    s[c > np.asarray(compact_rows)[:, None]] = -np.inf
+    return s
+
+
+def attn_fwd(seqlens, edits_per_traj, Q, K, V, scale, rows=None, heads=None):
+    """Masked GQA attention forward via per-segment compact sequences.
+
+    Returns ``(O_sel, LSE_sel)`` for the selected global rows (default: all)
+    and query heads (default: all): ``O_sel[r, h_i, :]``, ``LSE_sel[h_i, r]``.
+    Softmax over each row's visible keys exactly (no large-negative fill).
+    """
+    Q = np.asarray(Q, dtype=np.float64)
+    K = np.asarray(K, dtype=np.float64)
+    V = np.asarray(V, dtype=np.float64)
+    Ttot, Hq, Dh = Q.shape
+    Hkv = K.shape[1]
+    grp = Hq // Hkv
+    heads = list(range(Hq)) if heads is None else list(heads)
+    rows = np.arange(Ttot) if rows is None else np.asarray(rows, dtype=np.int64)
+    pos_of = {int(r): n for n, r in enumerate(rows)}
+    O = np.full((len(rows), len(heads), Dh), np.nan)
+    L = np.full((len(heads), len(rows)), np.nan)
+    want = np.zeros(Ttot, dtype=bool)
+    want[rows] = True
+    for seg_rows, idx, n_before in _segments(seqlens, edits_per_traj):
+        sel = np.nonzero(want[seg_rows])[0]
+        if sel.size == 0:
+            continue
+        for c0 in range(0, sel.size, _ROW_CHUNK):
+            part = sel[c0 : c0 + _ROW_CHUNK]
+            # compact index of each selected row = n_before + local offset
+            grows = seg_rows[part]
+            out_pos = [pos_of[int(r)] for r in grows]
+            for hi, h in enumerate(heads):
+                g = h // grp
+                k = K[idx, g]
+                v = V[idx, g]
+                q = Q[grows, h]
+                s = _scores(q, k, scale, n_before + part)
+                m = s.max(axis=1, keepdims=True)
+                p = np.exp(s - m)
+                l = p.sum(axis=1, keepdims=True)
+                O[out_pos, hi] = (p @ v) / l
+                L[hi, out_pos] = (m + np.log(l))[:, 0]
+    return O, L
+
+
+def attn_bwd(seqlens, edits_per_traj, Q, K, V, dO, scale, groups=None):
+    """Textbook softmax-attention backward on every segment's compact sequence.
+
+    For one segment and head (compact rows r, compact keys c):
+    ``P = softmax(S)``, ``dP = dO V^T``, ``dS = P * (dP - rowsum(P * dP))``,
+    ``dQ = scale dS K``, ``dK += scale dS^T Q``, ``dV += P^T dO``; dK and dV
+    are scatter-added to the physical key rows across every segment and every
+    query head of the KV group.
+
+    ``groups`` restricts the computation to some KV groups (all their query
+    heads); returns full-size ``(dQ, dK, dV)`` with NaN outside the selection.
+    """
+    Q = np.asarray(Q, dtype=np.float64)
+    K = np.asarray(K, dtype=np.float64)
+    V = np.asarray(V, dtype=np.float64)
+    dO = np.asarray(dO, dtype=np.float64)
+    Ttot, Hq, Dh = Q.shape
+    Hkv = K.shape[1]
+    grp = Hq // Hkv
+    groups = list(range(Hkv)) if groups is None else list(groups)
+    dQ = np.full_like(Q, np.nan)
+    dK = np.full_like(K, np.nan)
+    dV = np.full_like(V, np.nan)
+    for g in groups:
+        dQ[:, g * grp : (g + 1) * grp] = 0.0
+        dK[:, g] = 0.0
+        dV[:, g] = 0.0
+    for seg_rows, idx, n_before in _segments(seqlens, edits_per_traj):
+        for c0 in range(0, seg_rows.size, _ROW_CHUNK):
+            grows = seg_rows[c0 : c0 + _ROW_CHUNK]
+            for g in groups:
+                k = K[idx, g]
+                v = V[idx, g]
+                dk = np.zeros_like(k)
+                dv = np.zeros_like(v)
+                for h in range(g * grp, (g + 1) * grp):
+                    q = Q[grows, h]
+                    do = dO[grows, h]
+                    s = _scores(q, k, scale, n_before + c0 + np.arange(grows.size))
+                    m = s.max(axis=1, keepdims=True)
+                    p = np.exp(s - m)
+                    p /= p.sum(axis=1, keepdims=True)
+                    dp = do @ v.T
+                    ds = p * (dp - (p * dp).sum(axis=1, keepdims=True))
+                    dQ[grows, h] = scale * (ds @ k)
+                    dk += scale * (ds.T @ q)
+                    dv += p.T @ do
+                np.add.at(dK[:, g], idx, dk)
+                np.add.at(dV[:, g], idx, dv)
+    return dQ, dK, dV
+
+
+def attn_bwd_keys(seqlens, edits_per_traj, Q, K, V, dO, scale, g, keys):
+    """dK, dV of KV group ``g`` for a few physical key rows only.
+
+    Same textbook formulas as ``attn_bwd``; only the columns of the selected
+    keys of each segment's ``dS`` and ``P`` are accumulated, but every row's
+    softmax is still normalised over its full live view. Used for sampled
+    checks on workloads too large for the full backward.
+    """
+    Q = np.asarray(Q, dtype=np.float64)
+    K = np.asarray(K, dtype=np.float64)
+    V = np.asarray(V, dtype=np.float64)
+    dO = np.asarray(dO, dtype=np.float64)
+    Hq = Q.shape[1]
+    grp = Hq // K.shape[1]
+    keys = np.asarray(keys, dtype=np.int64)
+    dk_out = np.zeros((keys.size, K.shape[2]))
+    dv_out = np.zeros((keys.size, K.shape[2]))
+    for seg_rows, idx, n_before in _segments(seqlens, edits_per_traj):
+        where = {int(p): c for c, p in enumerate(idx)}
+        cols = [(n, where[int(kk)]) for n, kk in enumerate(keys) if int(kk) in where]
+        if not cols:
+            continue
+        kn = np.asarray([a for a, _ in cols])
+        kc = np.asarray([b for _, b in cols])
+        k = K[idx, g]
+        v = V[idx, g]
+        for c0 in range(0, seg_rows.size, _ROW_CHUNK):
+            grows = seg_rows[c0 : c0 + _ROW_CHUNK]
+            for h in range(g * grp, (g + 1) * grp):
+                q = Q[grows, h]
+                do = dO[grows, h]
+                s = _scores(q, k, scale, n_before + c0 + np.arange(grows.size))
+                m = s.max(axis=1, keepdims=True)
+                p = np.exp(s - m)
+                p /= p.sum(axis=1, keepdims=True)
+                dp = do @ v.T
+                ds = p * (dp - (p * dp).sum(axis=1, keepdims=True))
+                np.add.at(dk_out, kn, scale * (ds[:, kc].T @ q))
+                np.add.at(dv_out, kn, p[:, kc].T @ do)
+    return dk_out, dv_out

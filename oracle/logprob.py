@@ -1,0 +1,115 @@
+"""Oracle: LM-head log-probabilities and the clipped policy loss, in float64.
+
+TEST INFRASTRUCTURE ONLY (see ``oracle/__init__``).
+
+The importance ratio of App. B.4 ("Pitfall A, RL view") is
+``rho_t = pi_theta(a_t | view) / pi_old(a_t | view)``, both under the live
+view; the paper trains with GRPO/PPO clipping (§6.1 "Optimization"; App. F.1:
+clip range 0.2 low / 0.28 high). The per-token surrogate is PPO's
+``-min(rho A, clip(rho, 1-eps_lo, 1+eps_hi) A)``, averaged over the M
+loss-carrying tokens (the logdiff average of Eq. 1 runs over the same set).
+
+Layouts: ``H [N, d]`` hidden rows, ``W [V, d]`` LM-head weight (torch Linear
+layout), ``targets [N]`` next-token ids by physical row, ``rows [M]`` the
+physical rows that carry loss (distinct), ``lp_old, adv [M]``.
+"""
+
+import numpy as np
+
+_ROW_CHUNK = 256
+
+
+def logits(H, W, rows):
+    """``z[m, v] = sum_d H[rows[m], d] W[v, d]`` (small problems only)."""
+    H = np.asarray(H, dtype=np.float64)
+    W = np.asarray(W, dtype=np.float64)
+    return H[np.asarray(rows)] @ W.T
+
+
+def logprob(H, W, targets, rows):
+    """Per loss row: ``lse = log sum_v exp(z_v)``, ``lp = z_target - lse``.
+
+    Rows are processed in chunks; each row is independent.
+    """
+    H = np.asarray(H, dtype=np.float64)
+    W = np.asarray(W, dtype=np.float64)
+    rows = np.asarray(rows, dtype=np.int64)
+    tgt = np.asarray(targets, dtype=np.int64)[rows]
+    lse = np.empty(rows.size)
+    lp = np.empty(rows.size)
+    for c0 in range(0, rows.size, _ROW_CHUNK):
+        r = rows[c0 : c0 + _ROW_CHUNK]
+        z = H[r] @ W.T
+        m = z.max(axis=1, keepdims=True)
+        l = m[:, 0] + np.log(np.exp(z - m).sum(axis=1))
+        lse[c0 : c0 + r.size] = l
+        lp[c0 : c0 + r.size] = z[np.arange(r.size), tgt[c0 : c0 + r.size]] - l
+    return lp, lse
+
+
+def policy_loss(lp, lp_old, adv, eps_lo, eps_hi, dloss=1.0):
+    """Ratio, clipped surrogate, mean loss and ``g_t = dL/dlp_t``.
+
+    ``rho = exp(lp - lp_old)``; ``l_t = -min(rho A, clip(rho) A)``;
+    ``L = mean_t l_t``. Differentiating the min case by case: the unclipped
+    term is selected (gradient ``-A rho / M``) unless the clipped term is
+    strictly smaller, which happens exactly when ``A > 0, rho > 1 + eps_hi``
+    or ``A < 0, rho < 1 - eps_lo``; there the surrogate is flat in lp and the
+    gradient is 0. At equality both terms coincide and the unclipped branch
+    is used. ``dloss`` scales the gradient (upstream dL).
+    """
+    lp = np.asarray(lp, dtype=np.float64)
+    lp_old = np.asarray(lp_old, dtype=np.float64)
+    adv = np.asarray(adv, dtype=np.float64)
+    M = lp.size
+    ratio = np.exp(lp - lp_old)
+    unclipped = ratio * adv
+    clipped = np.clip(ratio, 1.0 - eps_lo, 1.0 + eps_hi) * adv
+    per_tok = -np.minimum(unclipped, clipped)
+    loss = per_tok.mean() if M else 0.0
+    flat = clipped < unclipped
+    g = np.where(flat, 0.0, -adv * ratio) / max(M, 1) * dloss
+    return ratio, per_tok, loss, g
+
+
+def logprob_loss_bwd(H, W, targets, rows, lse, g):
+    """Gradients of ``L`` with respect to ``H`` and ``W``.
+
+    With ``lp_t = z_{t,tgt} - lse_t``, ``dlp_t/dz_{t,v} = 1[v = tgt] - p_{t,v}``
+    where ``p = softmax(z_t)``, so ``dz_{t,v} = g_t (1[v = tgt] - p_{t,v})``;
+    ``dH_t = sum_v dz_{t,v} W_v`` (zero on rows outside the loss) and
+    ``dW_v = sum_t dz_{t,v} H_t``.
+    """
+    H = np.asarray(H, dtype=np.float64)
+    W = np.asarray(W, dtype=np.float64)
+    rows = np.asarray(rows, dtype=np.int64)
+    tgt = np.asarray(targets, dtype=np.int64)[rows]
+    lse = np.asarray(lse, dtype=np.float64)
+    g = np.asarray(g, dtype=np.float64)
+    dH = np.zeros_like(H)
+    dW = np.zeros_like(W)
+    for c0 in range(0, rows.size, _ROW_CHUNK):
+        r = rows[c0 : c0 + _ROW_CHUNK]
+        sl = slice(c0, c0 + r.size)
+        z = H[r] @ W.T
+        p = np.exp(z - lse[sl, None])
+        onehot = np.zeros_like(p)
+        onehot[np.arange(r.size), tgt[sl]] = 1.0
+        dz = g[sl, None] * (onehot - p)
+        dH[r] = dz @ W
+        dW += dz.T @ H[r]
+    return dH, dW
+
+
+def logprob_loss_bwd_vocab(H, W, targets, rows, lse, g, vocab):
+    """``dW`` for a few vocabulary rows only (sampled checks on big heads)."""
+    H = np.asarray(H, dtype=np.float64)
+    Wv = np.asarray(W, dtype=np.float64)[np.asarray(vocab)]
+    rows = np.asarray(rows, dtype=np.int64)
+    tgt = np.asarray(targets, dtype=np.int64)[rows]
+    vocab = np.asarray(vocab, dtype=np.int64)
+    z = H[rows] @ Wv.T
+    p = np.exp(z - np.asarray(lse, dtype=np.float64)[:, None])
+    onehot = (tgt[:, None] == vocab[None, :]).astype(np.float64)
+    dz = np.asarray(g, dtype=np.float64)[:, None] * (onehot - p)
+    return dz.T @ H[rows]
