@@ -1,0 +1,212 @@
+/*
+ * mw.h -- C ABI of libmw: view-consistent scoring of compressed agent rollouts
+ * on one GB300 (sm_103a).
+ *
+ * Method: MemoryWalker (arXiv 2609.00865). Every generated token of an edited
+ * (compressed) rollout is scored under the live context view the policy held
+ * when it decoded that token (§3.2 live-view equation; §3.3 conditioning
+ * invariant), using the packed 4D-mask form of §4.2 on the physical union of
+ * all tokens, which Theorem "materialization equivalence" (§4.3) equates with
+ * per-branch LogitTree forwards (§4.1).
+ *
+ * Conventions shared by every entry point
+ * ----------------------------------------
+ *  - Trajectories are packed back to back. cu_seqlens[n_traj+1] (host int32)
+ *    holds their token offsets; T_b = cu_seqlens[b+1] - cu_seqlens[b].
+ *  - Positions inside a trajectory are 0-based (the prompt starts at 0). The
+ *    k-th edit of a trajectory fires at junction J_k = the physical index of
+ *    the last token that existed before the edit; every row i >= J_k is scored
+ *    under the post-edit view (App. B.4 Table "running-prefixes" pins this).
+ *    Row i predicts token i+1.
+ *  - Key j is visible to row i iff j <= i < omega(j), where omega(j) is the
+ *    smallest junction whose evicted set contains j (never evicted: INT32_MAX)
+ *    (§4.2, the M = M^causal (+) M^logical equation with lifetime [j, omega(j))).
+ *    Inserted summary tokens are ordinary physical tokens placed after their
+ *    junction, so causality alone hides them from earlier rows.
+ *  - Tiles are 128 x 128, trajectory-local, the last one ragged. Class EMPTY
+ *    (no visible in-range pair), FULL (all in-range pairs visible) or PARTIAL.
+ *    Tile-list entries are int32 (tile << 2) | class.
+ *  - Every device pointer is caller-owned device memory (the library never
+ *    allocates device memory, never frees, never synchronises a stream except
+ *    where stated). Host pointers are read during the call only.
+ *  - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
+ *  - Errors are returned as mw_status; nothing is thrown across the ABI. All
+ *    argument checks run on the host before any launch; on error nothing is
+ *    launched. MW_ECUDA reports a failed launch or copy (the CUDA error is
+ *    available through mw_last_cuda_error()).
+ */
+#ifndef MW_H_
+#define MW_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum mw_status {
+    MW_OK = 0,
+    MW_EINVAL = 1,    /* null pointer, negative size or bad scalar */
+    MW_EEDITS = 2,    /* record breaks the junction / span conventions */
+    MW_ESHAPE = 3,    /* unsupported or inconsistent shape */
+    MW_EDTYPE = 4,    /* unsupported dtype code */
+    MW_ECUDA = 5,     /* a CUDA runtime call failed */
+    MW_ETIMEOUT = 6,  /* a bounded device-side wait gave up (status word) */
+    MW_EDEVICE = 7,   /* a device-side consistency check failed (status word) */
+    MW_ENOSPACE = 8   /* request exceeds a fixed capacity */
+} mw_status;
+
+enum { MW_F32 = 0, MW_BF16 = 1 };
+enum { MW_TILE = 128 };
+enum { MW_TILE_EMPTY = 0, MW_TILE_PARTIAL = 1, MW_TILE_FULL = 2 };
+
+/* Human-readable name of a status code (static string). */
+const char* mw_status_str(int status);
+/* Last CUDA error code seen by the library on this host thread (0 if none). */
+int mw_last_cuda_error(void);
+/* ABI version of this header (bumped on any signature change). */
+int mw_abi_version(void);
+
+/*
+ * Visibility layout: sizes and byte offsets of every array inside the
+ * caller-allocated device buffer `vis` (vis_bytes) and of the build
+ * workspace `ws` (ws_bytes). All offsets are multiples of 256.
+ */
+typedef struct mw_vis_layout {
+    int32_t n_traj;
+    int32_t n_junc;
+    int32_t n_spans;
+    int32_t max_tiles;      /* max over trajectories of ceil(T_b / 128) */
+    int64_t total_tokens;   /* sum T_b */
+    int64_t n_tiles;        /* sum ceil(T_b / 128): q-tiles == k-tiles */
+    int64_t n_tri;          /* sum nt_b (nt_b + 1) / 2: tile pairs kt <= qt */
+    int64_t n_segs;         /* n_traj + n_junc */
+    int64_t n_keymask;      /* sum (1 + K_b) nt_b keymask entries */
+    /* --- arrays in `vis` (byte offsets) --- */
+    int64_t off_omega;      /* int32 [total_tokens] lifetime end, traj-local */
+    int64_t off_seg;        /* int32 [total_tokens] segment id of each row */
+    int64_t off_traj_tok;   /* int32 [n_traj + 1] token offset of each traj */
+    int64_t off_traj_tile;  /* int32 [n_traj + 1] first global tile of each traj */
+    int64_t off_traj_seg;   /* int32 [n_traj + 1] first global segment of each traj */
+    int64_t off_traj_tri;   /* int64 [n_traj + 1] first triangle entry of each traj */
+    int64_t off_traj_km;    /* int64 [n_traj + 1] first keymask entry of each traj */
+    int64_t off_seg_start;  /* int32 [n_segs] first row of each segment (0, J_1..J_K per traj) */
+    int64_t off_tile_traj;  /* int32 [n_tiles] trajectory of each global tile */
+    int64_t off_cls;        /* uint8 [n_tri] class of (qt, kt), index qt(qt+1)/2 + kt */
+    int64_t off_fwd_ptr;    /* int32 [n_tiles + 1] per global q-tile */
+    int64_t off_fwd_idx;    /* int32 [n_tri] ascending k-tiles (capacity n_tri) */
+    int64_t off_bwd_ptr;    /* int32 [n_tiles + 1] per global k-tile */
+    int64_t off_bwd_idx;    /* int32 [n_tri] ascending q-tiles (capacity n_tri) */
+    int64_t off_pairs;      /* int64 [n_traj + 1] visible pairs per traj, then total */
+    int64_t off_keymask;    /* uint32 [n_keymask][4] per (segment, k-tile) view bits */
+    int64_t off_status;     /* int32 [8] device status words (0 = ok) */
+    int64_t vis_bytes;
+    /* --- arrays in `ws` (build workspace; byte offsets) --- */
+    int64_t ws_off_spans;   /* int32 [n_spans][3] (global a, global b, J) */
+    int64_t ws_off_tstat;   /* int32 [n_tiles][2] per k-tile min / max lifetime */
+    int64_t ws_off_cnt;     /* int32 [2][n_tiles] fwd / bwd list lengths */
+    int64_t ws_bytes;
+} mw_vis_layout;
+
+/*
+ * Fill `out` for a record shape. Host-only; launches nothing.
+ *   n_traj >= 0; cu_seqlens[n_traj+1] non-decreasing from 0;
+ *   junc_traj[n_junc] non-decreasing in [0, n_traj); n_spans >= 0.
+ * Returns MW_EINVAL / MW_EEDITS on malformed input.
+ */
+mw_status mw_visibility_layout(int n_traj, const int32_t* cu_seqlens, int n_junc,
+                               const int32_t* junc_traj, int n_spans, mw_vis_layout* out);
+
+/*
+ * Build every visibility artefact of a record (§4.2 lifetimes; App. B.1
+ * segments) into `vis` (layout->vis_bytes, device) using `ws`
+ * (layout->ws_bytes, device).
+ *   junctions[n_junc]      host int32, traj-local J_k, strictly ascending
+ *                          within a trajectory, 1 <= J_k <= T_b - 1
+ *   junc_traj[n_junc]      host int32, owning trajectory, non-decreasing
+ *   junc_span_off[n_junc+1] host int32 CSR offsets into spans
+ *   spans[n_spans][2]      host int32 half-open [a, b), 0 <= a < b <= J_k
+ * The record is validated on the host (MW_EEDITS), packed and copied to `ws`
+ * with one cudaMemcpyAsync from pageable memory (the runtime may order that
+ * copy after earlier work on `stream`); everything else runs asynchronously.
+ */
+mw_status mw_build_visibility(const mw_vis_layout* layout, const int32_t* cu_seqlens,
+                              int n_junc, const int32_t* junctions, const int32_t* junc_traj,
+                              const int32_t* junc_span_off, const int32_t* spans,
+                              void* ws, void* vis, void* stream);
+
+/*
+ * Eviction-aware masked GQA attention forward (§4.2 mask; §4.3 equivalence).
+ *   Q, O  [total_tokens, Hq, Dh]   K, V [total_tokens, Hkv, Dh]   (dtype)
+ *   LSE   [Hq, total_tokens] float32, natural-log row log-sum-exp (saved for bwd)
+ *   O_i = sum_{j visible} softmax_j(scale q_i . k_j) v_j;  q-head h reads
+ *   kv-head h / (Hq / Hkv). Only non-EMPTY tiles are visited.
+ * dtype MW_BF16 requires Dh == 128 (tensor-core path); MW_F32 accepts Dh 64
+ * or 128 (exact-fp32 SIMT path). Hq % Hkv == 0.
+ */
+mw_status mw_masked_attn_fwd(const mw_vis_layout* layout, const void* vis,
+                             const void* Q, const void* K, const void* V, void* O, float* LSE,
+                             int Hq, int Hkv, int Dh, int dtype, float scale, void* stream);
+
+/* Bytes of device workspace mw_masked_attn_bwd needs for these sizes. */
+mw_status mw_masked_attn_bwd_ws(const mw_vis_layout* layout, int Hq, int Dh, int dtype,
+                                size_t* ws_bytes);
+
+/*
+ * Backward of mw_masked_attn_fwd for upstream dO (same layout as O).
+ * Writes dQ (like Q), dK, dV (like K, V), all in `dtype`, overwriting them.
+ * Delta_i = rowsum(dO_i * O_i) and, for bf16, a float32 dQ accumulator live
+ * in `ws` (mw_masked_attn_bwd_ws bytes).
+ */
+mw_status mw_masked_attn_bwd(const mw_vis_layout* layout, const void* vis,
+                             const void* Q, const void* K, const void* V, const void* O,
+                             const void* dO, const float* LSE, void* dQ, void* dK, void* dV,
+                             int Hq, int Hkv, int Dh, int dtype, float scale,
+                             void* ws, void* stream);
+
+/* Bytes of device workspace the log-prob loss forward/backward pair needs. */
+mw_status mw_logprob_ws(int N, int M, int d, int Vocab, int dtype, size_t* ws_bytes);
+
+/*
+ * Fused LM-head log-prob + clipped policy loss, forward. No logits tensor is
+ * materialised. For loss row m (physical row t = rows[m]):
+ *   z_v = H_t . W_v,  lse_m = log sum_v exp z_v,  lp_m = z_{targets[t]} - lse_m,
+ *   ratio_m = exp(lp_m - lp_old_m),
+ *   loss = (1/M) sum_m -min(ratio_m A_m, clip(ratio_m, 1-eps_lo, 1+eps_hi) A_m)
+ * (App. B.4 "Pitfall A, RL view" ratio; PPO/GRPO clipping, App. F.1).
+ *   H [N, d], W [Vocab, d] (dtype; W in torch Linear layout); targets[N],
+ *   rows[M] distinct physical rows (int32, device); lp_old, adv [M] float32.
+ *   Outputs lp, ratio, lse [M] float32, loss: one float32 (device).
+ * `ws` (mw_logprob_ws bytes) keeps dL/dlp per row for the backward.
+ * dtype MW_BF16 requires d % 64 == 0; MW_F32 requires d <= 256.
+ */
+mw_status mw_logprob_loss_fwd(const void* H, const void* W, const int32_t* targets,
+                              const int32_t* rows, int M, const float* lp_old, const float* adv,
+                              float eps_lo, float eps_hi, int N, int d, int Vocab, int dtype,
+                              float* lp, float* ratio, float* lse, float* loss,
+                              void* ws, void* stream);
+
+/*
+ * Backward of mw_logprob_loss_fwd, scaled by the upstream gradient dloss:
+ *   dz_{m,v} = dloss * g_m * (1[v = target] - softmax_v(z_m)),
+ *   dH_t = sum_v dz_{m,v} W_v (rows outside `rows` get 0),
+ *   dW_v = sum_m dz_{m,v} H_{rows[m]}.
+ * Needs the forward's lse and `ws`. dH [N, d] in dtype; dW [Vocab, d] float32.
+ * Both are overwritten.
+ */
+mw_status mw_logprob_loss_bwd(const void* H, const void* W, const int32_t* targets,
+                              const int32_t* rows, int M, int N, int d, int Vocab, int dtype,
+                              const float* lse, const void* ws, float dloss,
+                              void* dH, float* dW, void* stream);
+
+/*
+ * Copy the device status words of a visibility buffer to the host after
+ * synchronising `stream`; returns MW_OK, MW_ETIMEOUT or MW_EDEVICE.
+ */
+mw_status mw_check_status(const mw_vis_layout* layout, const void* vis, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* MW_H_ */

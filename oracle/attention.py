@@ -141,6 +141,40 @@ def attn_bwd(seqlens, edits_per_traj, Q, K, V, dO, scale, groups=None):
     return dQ, dK, dV
 
 
+def attn_bwd_rows(seqlens, edits_per_traj, Q, K, V, dO, scale, rows, heads):
+    """dQ of a few physical rows and query heads (same formulas as
+    ``attn_bwd``; a row's dQ needs only its own segment's compact view).
+    Returns ``dQ_sel[r, h_i, :]``."""
+    Q = np.asarray(Q, dtype=np.float64)
+    K = np.asarray(K, dtype=np.float64)
+    V = np.asarray(V, dtype=np.float64)
+    dO = np.asarray(dO, dtype=np.float64)
+    Hq = Q.shape[1]
+    grp = Hq // K.shape[1]
+    rows = np.asarray(rows, dtype=np.int64)
+    pos_of = {int(r): n for n, r in enumerate(rows)}
+    out = np.full((rows.size, len(heads), Q.shape[2]), np.nan)
+    want = np.zeros(Q.shape[0], dtype=bool)
+    want[rows] = True
+    for seg_rows, idx, n_before in _segments(seqlens, edits_per_traj):
+        part = np.nonzero(want[seg_rows])[0]
+        if part.size == 0:
+            continue
+        grows = seg_rows[part]
+        outp = [pos_of[int(r)] for r in grows]
+        for hi, h in enumerate(heads):
+            k = K[idx, h // grp]
+            v = V[idx, h // grp]
+            s = _scores(Q[grows, h], k, scale, n_before + part)
+            m = s.max(axis=1, keepdims=True)
+            p = np.exp(s - m)
+            p /= p.sum(axis=1, keepdims=True)
+            dp = dO[grows, h] @ v.T
+            ds = p * (dp - (p * dp).sum(axis=1, keepdims=True))
+            out[outp, hi] = scale * (ds @ k)
+    return out
+
+
 def attn_bwd_keys(seqlens, edits_per_traj, Q, K, V, dO, scale, g, keys):
     """dK, dV of KV group ``g`` for a few physical key rows only.
 

@@ -41,8 +41,8 @@ def validate_edits(T, edits):
     App. B Def. "trajectory tree": compressions fire at increasing physical
     positions and each evicts positions before its junction.
     """
-    if T < 1:
-        raise RecordError("empty trajectory")
+    if T < 0:
+        raise RecordError("negative trajectory length")
     prev = 0
     for J, spans in edits:
         if not (1 <= J <= T - 1):
@@ -226,16 +226,15 @@ def build(seqlens, edits_per_traj, tile=TILE):
         seg.append(segment_ids(T, edits))
         qtraj.append(np.full(nt, b, dtype=np.int32))
         classes.append(cls)
-        for qt in range(nt):
-            for kt in range(qt + 1):
-                if cls[qt, kt] != EMPTY:
-                    fwd_idx.append((kt << 2) | int(cls[qt, kt]))
-            fwd_ptr.append(len(fwd_idx))
-        for kt in range(nt):
-            for qt in range(kt, nt):
-                if cls[qt, kt] != EMPTY:
-                    bwd_idx.append((qt << 2) | int(cls[qt, kt]))
-            bwd_ptr.append(len(bwd_idx))
+        # fwd list of q-tile qt: its non-EMPTY k-tiles in ascending order
+        # (row-major scan of the class matrix); bwd list of k-tile kt: its
+        # non-EMPTY q-tiles in ascending order (scan of the transpose).
+        q_nz, k_nz = np.nonzero(cls != EMPTY)
+        fwd_idx.extend(((k_nz << 2) | cls[q_nz, k_nz]).tolist())
+        fwd_ptr.extend((fwd_ptr[-1] + np.cumsum(np.bincount(q_nz, minlength=nt))).tolist())
+        k_nz2, q_nz2 = np.nonzero(cls.T != EMPTY)
+        bwd_idx.extend(((q_nz2 << 2) | cls[q_nz2, k_nz2]).tolist())
+        bwd_ptr.extend((bwd_ptr[-1] + np.cumsum(np.bincount(k_nz2, minlength=nt))).tolist())
         pairs.append(int(counts.sum()))
         keymask.append(segment_keymask(T, edits, tile).reshape(-1, tile // 32))
     return {

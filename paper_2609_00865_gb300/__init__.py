@@ -1,0 +1,30 @@
+"""libmw Python binding: view-consistent scoring of compressed rollouts on GB300.
+
+The compute path lives in ``libmw.so`` (hand-written CUDA for sm_103a behind
+the C ABI of ``include/mw.h``); this package only marshals arguments. Import
+fails loudly on first use when the library has not been built.
+"""
+
+from ._lib import (  # noqa: F401
+    MW_BF16,
+    MW_F32,
+    MWError,
+    TILE,
+    Visibility,
+    VisLayout,
+    build_visibility,
+    exported_names,
+    flatten_record,
+    logprob_loss_bwd,
+    logprob_loss_fwd,
+    masked_attn_bwd,
+    masked_attn_fwd,
+    mw_build_visibility,
+    mw_logprob_loss_bwd,
+    mw_logprob_loss_fwd,
+    mw_logprob_ws,
+    mw_masked_attn_bwd,
+    mw_masked_attn_bwd_ws,
+    mw_masked_attn_fwd,
+    mw_visibility_layout,
+)

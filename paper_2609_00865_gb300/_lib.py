@@ -1,0 +1,330 @@
+"""ctypes binding of libmw (include/mw.h): argument marshalling only.
+
+Every step of the path runs inside libmw's CUDA kernels; this module converts
+torch tensors to pointers, allocates outputs with torch (device memory and
+streams are torch's), and raises ``MWError`` on a non-OK status. It fails
+loudly when libmw.so is missing: there is no CPU fallback.
+"""
+
+import ctypes
+import os
+
+import numpy as np
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libmw.so")
+
+MW_F32, MW_BF16 = 0, 1
+TILE = 128
+STATUS = ["MW_OK", "MW_EINVAL", "MW_EEDITS", "MW_ESHAPE", "MW_EDTYPE", "MW_ECUDA",
+          "MW_ETIMEOUT", "MW_EDEVICE", "MW_ENOSPACE"]
+
+
+class MWError(RuntimeError):
+    def __init__(self, status, where):
+        self.status = status
+        name = STATUS[status] if 0 <= status < len(STATUS) else str(status)
+        super().__init__(f"{where}: {name} ({_lib().mw_status_str(status).decode()})")
+
+
+class VisLayout(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in ("n_traj", "n_junc", "n_spans", "max_tiles")] + \
+               [(n, ctypes.c_int64) for n in (
+                   "total_tokens", "n_tiles", "n_tri", "n_segs", "n_keymask",
+                   "off_omega", "off_seg", "off_traj_tok", "off_traj_tile", "off_traj_seg",
+                   "off_traj_tri", "off_traj_km", "off_seg_start", "off_tile_traj", "off_cls",
+                   "off_fwd_ptr", "off_fwd_idx", "off_bwd_ptr", "off_bwd_idx", "off_pairs",
+                   "off_keymask", "off_status", "vis_bytes",
+                   "ws_off_spans", "ws_off_tstat", "ws_off_cnt", "ws_bytes")]
+
+
+_P = ctypes.c_void_p
+_I = ctypes.c_int
+_F = ctypes.c_float
+_LP = ctypes.POINTER(VisLayout)
+_IP = ctypes.POINTER(ctypes.c_int32)
+
+_SIGS = {
+    "mw_status_str": (ctypes.c_char_p, [_I]),
+    "mw_last_cuda_error": (_I, []),
+    "mw_abi_version": (_I, []),
+    "mw_visibility_layout": (_I, [_I, _IP, _I, _IP, _I, _LP]),
+    "mw_build_visibility": (_I, [_LP, _IP, _I, _IP, _IP, _IP, _IP, _P, _P, _P]),
+    "mw_masked_attn_fwd": (_I, [_LP, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _F, _P]),
+    "mw_masked_attn_bwd_ws": (_I, [_LP, _I, _I, _I, ctypes.POINTER(ctypes.c_size_t)]),
+    "mw_masked_attn_bwd": (_I, [_LP, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _F, _P, _P]),
+    "mw_logprob_ws": (_I, [_I, _I, _I, _I, _I, ctypes.POINTER(ctypes.c_size_t)]),
+    "mw_logprob_loss_fwd": (_I, [_P, _P, _P, _P, _I, _P, _P, _F, _F, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P]),
+    "mw_logprob_loss_bwd": (_I, [_P, _P, _P, _P, _I, _I, _I, _I, _I, _P, _P, _F, _P, _P, _P]),
+    "mw_check_status": (_I, [_LP, _P, _P]),
+}
+
+_handle = None
+
+
+def _lib():
+    global _handle
+    if _handle is None:
+        if not os.path.exists(LIB_PATH):
+            raise ImportError(f"libmw.so not built at {LIB_PATH}; run __graft_entry__.build()")
+        h = ctypes.CDLL(LIB_PATH)
+        for name, (res, args) in _SIGS.items():
+            fn = getattr(h, name)
+            fn.restype = res
+            fn.argtypes = args
+        _handle = h
+    return _handle
+
+
+def exported_names():
+    return list(_SIGS)
+
+
+def _check(st, where):
+    if st != 0:
+        raise MWError(st, where)
+
+
+def _i32(a):
+    a = np.ascontiguousarray(np.asarray(a, dtype=np.int32))
+    return a, a.ctypes.data_as(_IP)
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    import torch
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _dtype_code(t):
+    import torch
+    if t.dtype == torch.float32:
+        return MW_F32
+    if t.dtype == torch.bfloat16:
+        return MW_BF16
+    raise MWError(4, f"dtype {t.dtype}")
+
+
+def _need(t, name, dtype=None, device=None):
+    import torch
+    if not t.is_cuda or not t.is_contiguous():
+        raise MWError(1, f"{name} must be a contiguous CUDA tensor")
+    if dtype is not None and t.dtype != dtype:
+        raise MWError(4, f"{name} dtype {t.dtype}")
+    return t
+
+
+# --- records ------------------------------------------------------------------
+
+def flatten_record(seqlens, edits_per_traj):
+    """Record -> (cu_seqlens, junctions, junc_traj, junc_span_off, spans) arrays."""
+    cu = np.zeros(len(seqlens) + 1, dtype=np.int32)
+    cu[1:] = np.cumsum(seqlens)
+    J, jt, off, spans = [], [], [0], []
+    for b, edits in enumerate(edits_per_traj):
+        for j, sp in edits:
+            J.append(j)
+            jt.append(b)
+            for a, e in sp:
+                spans.append((a, e))
+            off.append(len(spans))
+    return (cu, np.asarray(J, np.int32), np.asarray(jt, np.int32), np.asarray(off, np.int32),
+            np.asarray(spans, np.int32).reshape(-1, 2))
+
+
+def mw_visibility_layout(cu_seqlens, junc_traj, n_spans):
+    L = VisLayout()
+    cu, cup = _i32(cu_seqlens)
+    jt, jtp = _i32(junc_traj)
+    _check(_lib().mw_visibility_layout(len(cu) - 1, cup, len(jt), jtp, int(n_spans), ctypes.byref(L)),
+           "mw_visibility_layout")
+    return L
+
+
+def mw_build_visibility(layout, cu_seqlens, junctions, junc_traj, junc_span_off, spans, ws, vis, stream=None):
+    cu, cup = _i32(cu_seqlens)
+    J, Jp = _i32(junctions)
+    jt, jtp = _i32(junc_traj)
+    off, offp = _i32(junc_span_off)
+    sp, spp = _i32(np.asarray(spans).reshape(-1))
+    _check(_lib().mw_build_visibility(ctypes.byref(layout), cup, len(J), Jp, jtp, offp, spp,
+                                      _ptr(ws), _ptr(vis), _stream(stream)), "mw_build_visibility")
+
+
+class Visibility:
+    """Device visibility buffer of one packed record plus its layout."""
+
+    def __init__(self, layout, vis, ws):
+        self.layout = layout
+        self.vis = vis
+        self.ws = ws
+
+    def _arr(self, off, count, dtype):
+        import torch
+        nbytes = int(count) * np.dtype(dtype).itemsize
+        t = self.vis[off: off + nbytes].cpu().numpy()
+        return t.view(dtype).copy()
+
+    def arrays(self):
+        """Copy every artefact to the host in the oracle's ``build`` format."""
+        L = self.layout
+        n = L.n_tiles
+        fwd_ptr = self._arr(L.off_fwd_ptr, n + 1, np.int32)
+        bwd_ptr = self._arr(L.off_bwd_ptr, n + 1, np.int32)
+        tok = self._arr(L.off_traj_tok, L.n_traj + 1, np.int32)
+        tile = self._arr(L.off_traj_tile, L.n_traj + 1, np.int32)
+        tri = self._arr(L.off_traj_tri, L.n_traj + 1, np.int64)
+        cls_flat = self._arr(L.off_cls, L.n_tri, np.uint8)
+        classes = []
+        for b in range(L.n_traj):
+            nt = int(tile[b + 1] - tile[b])
+            c = np.zeros((nt, nt), dtype=np.int32)
+            base = int(tri[b])
+            for q in range(nt):
+                c[q, : q + 1] = cls_flat[base + q * (q + 1) // 2: base + q * (q + 1) // 2 + q + 1]
+            classes.append(c)
+        pairs = self._arr(L.off_pairs, L.n_traj + 1, np.int64)
+        return {
+            "omega": self._arr(L.off_omega, L.total_tokens, np.int32),
+            "seg": self._arr(L.off_seg, L.total_tokens, np.int32),
+            "qtile_traj": self._arr(L.off_tile_traj, n, np.int32),
+            "cls": classes,
+            "fwd_ptr": fwd_ptr,
+            "fwd_idx": self._arr(L.off_fwd_idx, int(fwd_ptr[-1]), np.int32),
+            "bwd_ptr": bwd_ptr,
+            "bwd_idx": self._arr(L.off_bwd_idx, int(bwd_ptr[-1]), np.int32),
+            "pairs": pairs[:-1],
+            "pairs_total": int(pairs[-1]),
+            "keymask": self._arr(L.off_keymask, L.n_keymask * 4, np.uint32).reshape(-1, 4),
+            "traj_tok": tok,
+        }
+
+    @property
+    def pairs_total(self):
+        L = self.layout
+        return int(self._arr(L.off_pairs + 8 * L.n_traj, 1, np.int64)[0])
+
+    def check_status(self, stream=None):
+        _check(_lib().mw_check_status(ctypes.byref(self.layout), _ptr(self.vis), _stream(stream)),
+               "mw_check_status")
+
+
+def build_visibility(seqlens, edits_per_traj, device="cuda", stream=None):
+    """Flatten a record, allocate its buffers with torch, run the builder."""
+    import torch
+    cu, J, jt, off, spans = flatten_record(seqlens, edits_per_traj)
+    L = mw_visibility_layout(cu, jt, len(spans))
+    vis = torch.empty(max(int(L.vis_bytes), 1), dtype=torch.uint8, device=device)
+    ws = torch.empty(max(int(L.ws_bytes), 1), dtype=torch.uint8, device=device)
+    mw_build_visibility(L, cu, J, jt, off, spans, ws, vis, stream)
+    return Visibility(L, vis, ws)
+
+
+# --- attention ----------------------------------------------------------------
+
+def mw_masked_attn_fwd(vis, Q, K, V, O, LSE, scale, stream=None):
+    Hq, Dh = Q.shape[1], Q.shape[2]
+    Hkv = K.shape[1]
+    _check(_lib().mw_masked_attn_fwd(ctypes.byref(vis.layout), _ptr(vis.vis), _ptr(Q), _ptr(K), _ptr(V),
+                                     _ptr(O), _ptr(LSE), Hq, Hkv, Dh, _dtype_code(Q), float(scale),
+                                     _stream(stream)), "mw_masked_attn_fwd")
+
+
+def masked_attn_fwd(vis, Q, K, V, scale=None, stream=None):
+    """Allocate O [T, Hq, Dh] and LSE [Hq, T] and run the forward."""
+    import torch
+    for t, n in ((Q, "Q"), (K, "K"), (V, "V")):
+        _need(t, n, dtype=Q.dtype)
+    scale = float(Q.shape[2]) ** -0.5 if scale is None else scale
+    O = torch.empty_like(Q)
+    LSE = torch.empty(Q.shape[1], Q.shape[0], dtype=torch.float32, device=Q.device)
+    mw_masked_attn_fwd(vis, Q, K, V, O, LSE, scale, stream)
+    return O, LSE
+
+
+def mw_masked_attn_bwd_ws(vis, Hq, Dh, dtype):
+    n = ctypes.c_size_t()
+    _check(_lib().mw_masked_attn_bwd_ws(ctypes.byref(vis.layout), Hq, Dh, dtype, ctypes.byref(n)),
+           "mw_masked_attn_bwd_ws")
+    return int(n.value)
+
+
+def mw_masked_attn_bwd(vis, Q, K, V, O, dO, LSE, dQ, dK, dV, scale, ws, stream=None):
+    Hq, Dh = Q.shape[1], Q.shape[2]
+    Hkv = K.shape[1]
+    _check(_lib().mw_masked_attn_bwd(ctypes.byref(vis.layout), _ptr(vis.vis), _ptr(Q), _ptr(K), _ptr(V), _ptr(O),
+                                     _ptr(dO), _ptr(LSE), _ptr(dQ), _ptr(dK), _ptr(dV), Hq, Hkv, Dh,
+                                     _dtype_code(Q), float(scale), _ptr(ws), _stream(stream)),
+           "mw_masked_attn_bwd")
+
+
+def masked_attn_bwd(vis, Q, K, V, O, dO, LSE, scale=None, ws=None, stream=None):
+    """Allocate dQ, dK, dV (and the workspace) and run the backward."""
+    import torch
+    for t, n in ((Q, "Q"), (K, "K"), (V, "V"), (O, "O"), (dO, "dO")):
+        _need(t, n, dtype=Q.dtype)
+    _need(LSE, "LSE", dtype=torch.float32)
+    scale = float(Q.shape[2]) ** -0.5 if scale is None else scale
+    if ws is None:
+        nbytes = mw_masked_attn_bwd_ws(vis, Q.shape[1], Q.shape[2], _dtype_code(Q))
+        ws = torch.empty(max(nbytes, 1), dtype=torch.uint8, device=Q.device)
+    dQ, dK, dV = torch.empty_like(Q), torch.empty_like(K), torch.empty_like(V)
+    mw_masked_attn_bwd(vis, Q, K, V, O, dO, LSE, dQ, dK, dV, scale, ws, stream)
+    return dQ, dK, dV
+
+
+# --- LM head ------------------------------------------------------------------
+
+def mw_logprob_ws(N, M, d, Vocab, dtype):
+    n = ctypes.c_size_t()
+    _check(_lib().mw_logprob_ws(N, M, d, Vocab, dtype, ctypes.byref(n)), "mw_logprob_ws")
+    return int(n.value)
+
+
+def mw_logprob_loss_fwd(H, W, targets, rows, lp_old, adv, eps_lo, eps_hi, lp, ratio, lse, loss, ws, stream=None):
+    N, d = H.shape
+    _check(_lib().mw_logprob_loss_fwd(_ptr(H), _ptr(W), _ptr(targets), _ptr(rows), int(rows.numel()),
+                                      _ptr(lp_old), _ptr(adv), float(eps_lo), float(eps_hi), N, d, W.shape[0],
+                                      _dtype_code(H), _ptr(lp), _ptr(ratio), _ptr(lse), _ptr(loss), _ptr(ws),
+                                      _stream(stream)), "mw_logprob_loss_fwd")
+
+
+def logprob_loss_fwd(H, W, targets, rows, lp_old, adv, eps_lo=0.2, eps_hi=0.2, stream=None):
+    """Allocate outputs + workspace; returns dict(lp, ratio, lse, loss, ws)."""
+    import torch
+    _need(H, "H")
+    _need(W, "W", dtype=H.dtype)
+    _need(targets, "targets", dtype=torch.int32)
+    _need(rows, "rows", dtype=torch.int32)
+    _need(lp_old, "lp_old", dtype=torch.float32)
+    _need(adv, "adv", dtype=torch.float32)
+    M = rows.numel()
+    dev = H.device
+    ws = torch.empty(max(mw_logprob_ws(H.shape[0], M, H.shape[1], W.shape[0], _dtype_code(H)), 1),
+                     dtype=torch.uint8, device=dev)
+    out = {k: torch.empty(M, dtype=torch.float32, device=dev) for k in ("lp", "ratio", "lse")}
+    out["loss"] = torch.empty(1, dtype=torch.float32, device=dev)
+    mw_logprob_loss_fwd(H, W, targets, rows, lp_old, adv, eps_lo, eps_hi, out["lp"], out["ratio"], out["lse"],
+                        out["loss"], ws, stream)
+    out["ws"] = ws
+    return out
+
+
+def mw_logprob_loss_bwd(H, W, targets, rows, lse, ws, dloss, dH, dW, stream=None):
+    N, d = H.shape
+    _check(_lib().mw_logprob_loss_bwd(_ptr(H), _ptr(W), _ptr(targets), _ptr(rows), int(rows.numel()), N, d,
+                                      W.shape[0], _dtype_code(H), _ptr(lse), _ptr(ws), float(dloss), _ptr(dH),
+                                      _ptr(dW), _stream(stream)), "mw_logprob_loss_bwd")
+
+
+def logprob_loss_bwd(H, W, targets, rows, lse, ws, dloss=1.0, stream=None):
+    """Allocate dH (H's dtype) and dW (float32) and run the backward."""
+    import torch
+    dH = torch.empty_like(H)
+    dW = torch.empty(W.shape, dtype=torch.float32, device=W.device)
+    mw_logprob_loss_bwd(H, W, targets, rows, lse, ws, dloss, dH, dW, stream)
+    return dH, dW

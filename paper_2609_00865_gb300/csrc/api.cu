@@ -1,0 +1,123 @@
+// extern "C" entry points of libmw: host-side argument checks and dispatch.
+// See include/mw.h for the contract of every function.
+
+#include <math.h>
+
+#include "common.cuh"
+
+namespace mw {
+mw_status attn_fwd_simt(const mw_vis_layout*, const void*, const void*, const void*, const void*, void*, float*,
+                        int, int, int, int, float, cudaStream_t);
+mw_status attn_bwd_simt(const mw_vis_layout*, const void*, const void*, const void*, const void*, const void*,
+                        const void*, const float*, void*, void*, void*, int, int, int, int, float, float*,
+                        cudaStream_t);
+mw_status lm_fwd_simt(const void*, const void*, const int32_t*, const int32_t*, int, int, int, int, float*, float*,
+                      float*, cudaStream_t);
+mw_status lm_bwd_simt(const void*, const void*, const int32_t*, const int32_t*, int, int, int, int, int,
+                      const float*, const float*, float, void*, float*, cudaStream_t);
+__global__ void k_loss_epilogue(int, const float*, const float*, const float*, float, float, float*, float*, float*);
+
+// Byte offsets inside the log-prob workspace.
+struct LmWs {
+    int64_t g, zt, bytes;
+};
+static LmWs lm_ws_layout(int N, int M, int d, int V, int dtype) {
+    (void)N; (void)d; (void)V; (void)dtype;
+    LmWs w;
+    int64_t o = 0;
+    w.g = o; o = align256(o + 4 * (int64_t)M);
+    w.zt = o; o = align256(o + 4 * (int64_t)M);
+    w.bytes = o;
+    return w;
+}
+
+static mw_status attn_args(const mw_vis_layout* L, const void* vis, int Hq, int Hkv, int Dh, int dtype,
+                           float scale) {
+    if (!L) return MW_EINVAL;
+    if (L->total_tokens > 0 && !vis) return MW_EINVAL;
+    if (dtype != MW_F32 && dtype != MW_BF16) return MW_EDTYPE;
+    if (Hq <= 0 || Hkv <= 0 || Hq % Hkv != 0) return MW_ESHAPE;
+    if (!(Dh == 64 || Dh == 128)) return MW_ESHAPE;
+    if (!(scale > 0.f) || !isfinite(scale)) return MW_EINVAL;
+    return MW_OK;
+}
+
+}  // namespace mw
+
+using namespace mw;
+
+extern "C" mw_status mw_masked_attn_fwd(const mw_vis_layout* L, const void* vis, const void* Q, const void* K,
+                                        const void* V, void* O, float* LSE, int Hq, int Hkv, int Dh, int dtype,
+                                        float scale, void* stream) {
+    mw_status st = attn_args(L, vis, Hq, Hkv, Dh, dtype, scale);
+    if (st != MW_OK) return st;
+    if (L->total_tokens == 0) return MW_OK;
+    if (!Q || !K || !V || !O || !LSE) return MW_EINVAL;
+    return attn_fwd_simt(L, vis, Q, K, V, O, LSE, Hq, Hkv, Dh, dtype, scale, (cudaStream_t)stream);
+}
+
+extern "C" mw_status mw_masked_attn_bwd_ws(const mw_vis_layout* L, int Hq, int Dh, int dtype, size_t* bytes) {
+    if (!L || !bytes) return MW_EINVAL;
+    (void)Dh; (void)dtype;
+    *bytes = (size_t)align256(4 * L->total_tokens * (int64_t)Hq);
+    return MW_OK;
+}
+
+extern "C" mw_status mw_masked_attn_bwd(const mw_vis_layout* L, const void* vis, const void* Q, const void* K,
+                                        const void* V, const void* O, const void* dO, const float* LSE, void* dQ,
+                                        void* dK, void* dV, int Hq, int Hkv, int Dh, int dtype, float scale,
+                                        void* ws, void* stream) {
+    mw_status st = attn_args(L, vis, Hq, Hkv, Dh, dtype, scale);
+    if (st != MW_OK) return st;
+    if (L->total_tokens == 0) return MW_OK;
+    if (!Q || !K || !V || !O || !dO || !LSE || !dQ || !dK || !dV || !ws) return MW_EINVAL;
+    return attn_bwd_simt(L, vis, Q, K, V, O, dO, LSE, dQ, dK, dV, Hq, Hkv, Dh, dtype, scale, (float*)ws,
+                         (cudaStream_t)stream);
+}
+
+static mw_status lm_args(int N, int M, int d, int V, int dtype) {
+    if (N < 0 || M < 0 || d <= 0 || V <= 0) return MW_ESHAPE;
+    if (M > N) return MW_ESHAPE;
+    if (dtype != MW_F32 && dtype != MW_BF16) return MW_EDTYPE;
+    if (d > 256) return MW_ESHAPE;
+    return MW_OK;
+}
+
+extern "C" mw_status mw_logprob_ws(int N, int M, int d, int V, int dtype, size_t* bytes) {
+    if (!bytes) return MW_EINVAL;
+    mw_status st = lm_args(N, M, d, V, dtype);
+    if (st != MW_OK) return st;
+    *bytes = (size_t)lm_ws_layout(N, M, d, V, dtype).bytes;
+    return MW_OK;
+}
+
+extern "C" mw_status mw_logprob_loss_fwd(const void* H, const void* W, const int32_t* targets, const int32_t* rows,
+                                         int M, const float* lp_old, const float* adv, float eps_lo, float eps_hi,
+                                         int N, int d, int V, int dtype, float* lp, float* ratio, float* lse,
+                                         float* loss, void* ws, void* stream) {
+    mw_status st = lm_args(N, M, d, V, dtype);
+    if (st != MW_OK) return st;
+    if (!(eps_lo >= 0.f && eps_lo < 1.f && eps_hi >= 0.f && isfinite(eps_hi))) return MW_EINVAL;
+    if (!loss || !ws) return MW_EINVAL;
+    if (M > 0 && (!H || !W || !targets || !rows || !lp_old || !adv || !lp || !ratio || !lse)) return MW_EINVAL;
+    cudaStream_t s = (cudaStream_t)stream;
+    LmWs w = lm_ws_layout(N, M, d, V, dtype);
+    float* g = at<float>(ws, w.g);
+    float* zt = at<float>(ws, w.zt);
+    if ((st = lm_fwd_simt(H, W, targets, rows, M, d, V, dtype, lse, zt, lp, s)) != MW_OK) return st;
+    k_loss_epilogue<<<1, 1024, 0, s>>>(M, lp, lp_old, adv, eps_lo, eps_hi, ratio, g, loss);
+    return launch_status();
+}
+
+extern "C" mw_status mw_logprob_loss_bwd(const void* H, const void* W, const int32_t* targets, const int32_t* rows,
+                                         int M, int N, int d, int V, int dtype, const float* lse, const void* ws,
+                                         float dloss, void* dH, float* dW, void* stream) {
+    mw_status st = lm_args(N, M, d, V, dtype);
+    if (st != MW_OK) return st;
+    if (!isfinite(dloss)) return MW_EINVAL;
+    if (!ws || !dW || (N > 0 && !dH)) return MW_EINVAL;
+    if (M > 0 && (!H || !W || !targets || !rows || !lse)) return MW_EINVAL;
+    LmWs w = lm_ws_layout(N, M, d, V, dtype);
+    return lm_bwd_simt(H, W, targets, rows, M, N, d, V, dtype, lse, at<float>(ws, w.g), dloss, dH, dW,
+                       (cudaStream_t)stream);
+}

@@ -1,0 +1,94 @@
+// Shared device/host helpers for libmw (no method arithmetic here).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include "mw.h"
+
+namespace mw {
+
+// Record the CUDA error (if any) in the thread-local slot and map to status.
+mw_status cuda_status(cudaError_t e);
+mw_status launch_status();
+
+inline int64_t align256(int64_t x) { return (x + 255) & ~int64_t(255); }
+inline int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
+
+template <typename T>
+__host__ __device__ inline T* at(void* base, int64_t off) {
+    return reinterpret_cast<T*>(reinterpret_cast<char*>(base) + off);
+}
+template <typename T>
+__host__ __device__ inline const T* at(const void* base, int64_t off) {
+    return reinterpret_cast<const T*>(reinterpret_cast<const char*>(base) + off);
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+    return v;
+}
+__device__ __forceinline__ int warp_sum_i(int v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+// Element loads that widen to float (the inputs are float32 or bfloat16).
+__device__ __forceinline__ float ld_f(const float* p) { return *p; }
+__device__ __forceinline__ float ld_f(const __nv_bfloat16* p) { return __bfloat162float(*p); }
+__device__ __forceinline__ void st_f(float* p, float v) { *p = v; }
+__device__ __forceinline__ void st_f(__nv_bfloat16* p, float v) { *p = __float2bfloat16_rn(v); }
+
+// Visibility context for one launch: base pointers into the `vis` buffer.
+struct VisView {
+    const int32_t* omega;
+    const int32_t* seg;
+    const int32_t* traj_tok;
+    const int32_t* traj_tile;
+    const int32_t* traj_seg;
+    const int64_t* traj_tri;
+    const int64_t* traj_km;
+    const int32_t* seg_start;
+    const int32_t* tile_traj;
+    const uint8_t* cls;
+    const int32_t* fwd_ptr;
+    const int32_t* fwd_idx;
+    const int32_t* bwd_ptr;
+    const int32_t* bwd_idx;
+    const uint32_t* keymask;
+    int32_t* status;
+};
+
+inline VisView make_view(const mw_vis_layout* L, const void* vis) {
+    VisView v;
+    v.omega = at<int32_t>(vis, L->off_omega);
+    v.seg = at<int32_t>(vis, L->off_seg);
+    v.traj_tok = at<int32_t>(vis, L->off_traj_tok);
+    v.traj_tile = at<int32_t>(vis, L->off_traj_tile);
+    v.traj_seg = at<int32_t>(vis, L->off_traj_seg);
+    v.traj_tri = at<int64_t>(vis, L->off_traj_tri);
+    v.traj_km = at<int64_t>(vis, L->off_traj_km);
+    v.seg_start = at<int32_t>(vis, L->off_seg_start);
+    v.tile_traj = at<int32_t>(vis, L->off_tile_traj);
+    v.cls = at<uint8_t>(vis, L->off_cls);
+    v.fwd_ptr = at<int32_t>(vis, L->off_fwd_ptr);
+    v.fwd_idx = at<int32_t>(vis, L->off_fwd_idx);
+    v.bwd_ptr = at<int32_t>(vis, L->off_bwd_ptr);
+    v.bwd_idx = at<int32_t>(vis, L->off_bwd_idx);
+    v.keymask = at<uint32_t>(vis, L->off_keymask);
+    v.status = const_cast<int32_t*>(at<int32_t>(vis, L->off_status));
+    return v;
+}
+
+// Status-word slots written by device code.
+enum { ST_BOUNDS = 0, ST_TIMEOUT = 1, ST_WHERE = 2 };
+
+}  // namespace mw

@@ -1,0 +1,505 @@
+// Visibility builder: record -> lifetimes, segments, tile classes, tile lists.
+//
+// Lifetimes follow the 4D mask of §4.2: key j is visible to row i iff
+// j <= i < omega(j), omega(j) = min{J_k : j in E_k}. Segments are the branch
+// layers of App. B.1 (rows [J_k, J_{k+1})). Everything here is O(T + tiles):
+// a tile's class follows from the min / max lifetime of its keys, because on an
+// off-diagonal tile (keys all before the rows) visibility depends on the row
+// only through i < omega(j).
+
+#include <stdio.h>
+#include <stdlib.h>
+#include <string.h>
+
+#include <vector>
+
+#include "common.cuh"
+
+namespace mw {
+
+static thread_local int g_last_cuda_error = 0;
+
+mw_status cuda_status(cudaError_t e) {
+    if (e == cudaSuccess) return MW_OK;
+    g_last_cuda_error = (int)e;
+    return MW_ECUDA;
+}
+mw_status launch_status() { return cuda_status(cudaGetLastError()); }
+
+}  // namespace mw
+
+using namespace mw;
+
+extern "C" const char* mw_status_str(int s) {
+    switch (s) {
+        case MW_OK: return "ok";
+        case MW_EINVAL: return "invalid argument";
+        case MW_EEDITS: return "record breaks the junction/span conventions";
+        case MW_ESHAPE: return "unsupported or inconsistent shape";
+        case MW_EDTYPE: return "unsupported dtype";
+        case MW_ECUDA: return "CUDA runtime error";
+        case MW_ETIMEOUT: return "bounded device wait timed out";
+        case MW_EDEVICE: return "device-side check failed";
+        case MW_ENOSPACE: return "request exceeds a fixed capacity";
+        default: return "unknown status";
+    }
+}
+
+extern "C" int mw_last_cuda_error(void) { return g_last_cuda_error; }
+extern "C" int mw_abi_version(void) { return 1; }
+
+static mw_status check_shape(int n_traj, const int32_t* cu, int n_junc, const int32_t* jt,
+                             int n_spans) {
+    if (n_traj < 0 || n_junc < 0 || n_spans < 0) return MW_EINVAL;
+    if (n_traj > 0 && !cu) return MW_EINVAL;
+    if (n_junc > 0 && !jt) return MW_EINVAL;
+    if (n_traj > 0 && cu[0] != 0) return MW_EEDITS;
+    for (int b = 0; b < n_traj; ++b)
+        if (cu[b + 1] < cu[b]) return MW_EEDITS;
+    for (int k = 0; k < n_junc; ++k) {
+        if (jt[k] < 0 || jt[k] >= n_traj) return MW_EEDITS;
+        if (k > 0 && jt[k] < jt[k - 1]) return MW_EEDITS;
+    }
+    return MW_OK;
+}
+
+extern "C" mw_status mw_visibility_layout(int n_traj, const int32_t* cu, int n_junc,
+                                          const int32_t* jt, int n_spans, mw_vis_layout* L) {
+    if (!L) return MW_EINVAL;
+    mw_status st = check_shape(n_traj, cu, n_junc, jt, n_spans);
+    if (st != MW_OK) return st;
+    memset(L, 0, sizeof(*L));
+    L->n_traj = n_traj;
+    L->n_junc = n_junc;
+    L->n_spans = n_spans;
+    int64_t tiles = 0, tri = 0, km = 0;
+    int max_tiles = 0;
+    int k = 0;
+    for (int b = 0; b < n_traj; ++b) {
+        int64_t T = cu[b + 1] - cu[b];
+        int64_t nt = ceil_div(T, MW_TILE);
+        int Kb = 0;
+        while (k < n_junc && jt[k] == b) { ++Kb; ++k; }
+        tiles += nt;
+        tri += nt * (nt + 1) / 2;
+        km += (1 + Kb) * nt;
+        if (nt > max_tiles) max_tiles = (int)nt;
+    }
+    L->max_tiles = max_tiles;
+    L->total_tokens = n_traj > 0 ? cu[n_traj] : 0;
+    L->n_tiles = tiles;
+    L->n_tri = tri;
+    L->n_segs = (int64_t)n_traj + n_junc;
+    L->n_keymask = km;
+    int64_t o = 0;
+    auto take = [&](int64_t bytes) { int64_t r = o; o = align256(o + bytes); return r; };
+    L->off_omega = take(4 * L->total_tokens);
+    L->off_seg = take(4 * L->total_tokens);
+    L->off_traj_tok = take(4 * (n_traj + 1));
+    L->off_traj_tile = take(4 * (n_traj + 1));
+    L->off_traj_seg = take(4 * (n_traj + 1));
+    L->off_traj_tri = take(8 * (n_traj + 1));
+    L->off_traj_km = take(8 * (n_traj + 1));
+    L->off_seg_start = take(4 * L->n_segs);
+    L->off_tile_traj = take(4 * tiles);
+    L->off_cls = take(tri);
+    L->off_fwd_ptr = take(4 * (tiles + 1));
+    L->off_fwd_idx = take(4 * tri);
+    L->off_bwd_ptr = take(4 * (tiles + 1));
+    L->off_bwd_idx = take(4 * tri);
+    L->off_pairs = take(8 * (n_traj + 1));
+    L->off_keymask = take(16 * km);
+    L->off_status = take(4 * 8);
+    L->vis_bytes = o;
+    o = 0;
+    L->ws_off_spans = take(12 * (int64_t)n_spans);
+    L->ws_off_tstat = take(8 * tiles);
+    L->ws_off_cnt = take(8 * tiles);
+    L->ws_bytes = o;
+    return MW_OK;
+}
+
+// ---------------------------------------------------------------------------
+// kernels
+
+namespace {
+
+struct BuildArgs {
+    int n_traj;
+    int64_t total;
+    int64_t n_tiles;
+    int n_spans;
+    int32_t* omega;
+    int32_t* seg;
+    const int32_t* traj_tok;
+    const int32_t* traj_tile;
+    const int32_t* traj_seg;
+    const int64_t* traj_tri;
+    const int64_t* traj_km;
+    const int32_t* seg_start;
+    const int32_t* tile_traj;
+    uint8_t* cls;
+    int32_t* fwd_ptr;
+    int32_t* fwd_idx;
+    int32_t* bwd_ptr;
+    int32_t* bwd_idx;
+    unsigned long long* pairs;
+    uint32_t* keymask;
+    const int32_t* spans;   // [n_spans][3]
+    int32_t* tstat;         // [n_tiles][2]
+    int32_t* fwd_cnt;       // [n_tiles]
+    int32_t* bwd_cnt;       // [n_tiles]
+};
+
+__device__ __forceinline__ int find_traj(const int32_t* off, int n, int64_t t) {
+    int lo = 0, hi = n;  // off[lo] <= t < off[hi]
+    while (hi - lo > 1) {
+        int mid = (lo + hi) >> 1;
+        if (off[mid] <= t) lo = mid; else hi = mid;
+    }
+    return lo;
+}
+
+// omega = never; seg = number of junctions <= local row.
+__global__ void k_init_tokens(BuildArgs a) {
+    for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < a.total;
+         t += (int64_t)gridDim.x * blockDim.x) {
+        int b = find_traj(a.traj_tok, a.n_traj, t);
+        int i = (int)(t - a.traj_tok[b]);
+        int s0 = a.traj_seg[b], s1 = a.traj_seg[b + 1];
+        int lo = s0, hi = s1;  // seg_start[lo] <= i (seg_start[s0] = 0)
+        while (hi - lo > 1) {
+            int mid = (lo + hi) >> 1;
+            if (a.seg_start[mid] <= i) lo = mid; else hi = mid;
+        }
+        a.omega[t] = INT32_MAX;
+        a.seg[t] = lo - s0;
+    }
+}
+
+// One block per evicted span: omega(j) = min over the junctions evicting j.
+__global__ void k_scatter_spans(BuildArgs a) {
+    for (int s = blockIdx.x; s < a.n_spans; s += gridDim.x) {
+        int ga = a.spans[3 * s], gb = a.spans[3 * s + 1], J = a.spans[3 * s + 2];
+        for (int t = ga + threadIdx.x; t < gb; t += blockDim.x) atomicMin(&a.omega[t], J);
+    }
+}
+
+// One block (128 threads) per global k-tile: min / max lifetime over its keys,
+// visible pairs sum_j (min(omega_j, T) - j), and the per-segment view bits.
+__global__ void k_tile_stats(BuildArgs a) {
+    int64_t g = blockIdx.x;
+    int b = a.tile_traj[g];
+    int kt = (int)(g - a.traj_tile[b]);
+    int T = a.traj_tok[b + 1] - a.traj_tok[b];
+    int j = kt * MW_TILE + threadIdx.x;
+    bool in = j < T;
+    int om = in ? a.omega[a.traj_tok[b] + j] : 0;
+    int omc = in ? min(om, T) : 0;
+    int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+    __shared__ int smin[4], smax[4];
+    __shared__ unsigned long long spair[4];
+    int vmin = in ? om : INT32_MAX, vmax = in ? om : INT32_MIN;
+    unsigned long long pr = in ? (unsigned long long)(omc - j) : 0ull;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        vmin = min(vmin, __shfl_xor_sync(0xffffffffu, vmin, o));
+        vmax = max(vmax, __shfl_xor_sync(0xffffffffu, vmax, o));
+        pr += __shfl_xor_sync(0xffffffffu, pr, o);
+    }
+    if (lane == 0) { smin[w] = vmin; smax[w] = vmax; spair[w] = pr; }
+    // view bits: key j is in segment s's view iff omega(j) > J_s and j < J_{s+1}
+    int s0 = a.traj_seg[b], nseg = a.traj_seg[b + 1] - s0;
+    for (int s = 0; s < nseg; ++s) {
+        int Js = a.seg_start[s0 + s];
+        int Jn = (s + 1 < nseg) ? a.seg_start[s0 + s + 1] : T;
+        bool bit = in && om > Js && j < Jn;
+        uint32_t word = __ballot_sync(0xffffffffu, bit);
+        if (lane == 0) a.keymask[(a.traj_km[b] + (int64_t)s * (a.traj_tile[b + 1] - a.traj_tile[b]) + kt) * 4 + w] = word;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int mn = min(min(smin[0], smin[1]), min(smin[2], smin[3]));
+        int mx = max(max(smax[0], smax[1]), max(smax[2], smax[3]));
+        a.tstat[2 * g] = mn;
+        a.tstat[2 * g + 1] = mx;
+        unsigned long long p = spair[0] + spair[1] + spair[2] + spair[3];
+        atomicAdd(&a.pairs[b], p);
+        atomicAdd(&a.pairs[a.n_traj], p);
+    }
+}
+
+__device__ __forceinline__ int tile_class(int qt, int kt, int T, int kmin, int kmax) {
+    int q0 = qt * MW_TILE, q1 = min(q0 + MW_TILE, T);
+    if (kt == qt) return (q1 - q0 == 1) ? MW_TILE_FULL : MW_TILE_PARTIAL;
+    if (kmin >= q1) return MW_TILE_FULL;
+    if (kmax <= q0) return MW_TILE_EMPTY;
+    return MW_TILE_PARTIAL;
+}
+
+// One warp per global q-tile: classes of (qt, 0..qt) and the fwd list length.
+__global__ void k_classify(BuildArgs a) {
+    int64_t g = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+    int lane = threadIdx.x & 31;
+    if (g >= a.n_tiles) return;
+    int b = a.tile_traj[g];
+    int tb = a.traj_tile[b];
+    int qt = (int)(g - tb);
+    int T = a.traj_tok[b + 1] - a.traj_tok[b];
+    uint8_t* row = a.cls + a.traj_tri[b] + (int64_t)qt * (qt + 1) / 2;
+    int cnt = 0;
+    for (int kt = lane; kt <= qt; kt += 32) {
+        int c = tile_class(qt, kt, T, a.tstat[2 * (tb + kt)], a.tstat[2 * (tb + kt) + 1]);
+        row[kt] = (uint8_t)c;
+        cnt += c != MW_TILE_EMPTY;
+    }
+    cnt = warp_sum_i(cnt);
+    if (lane == 0) a.fwd_cnt[g] = cnt;
+}
+
+// One warp per global k-tile: bwd list length (column of the class triangle).
+__global__ void k_bwd_count(BuildArgs a) {
+    int64_t g = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+    int lane = threadIdx.x & 31;
+    if (g >= a.n_tiles) return;
+    int b = a.tile_traj[g];
+    int tb = a.traj_tile[b], nt = a.traj_tile[b + 1] - tb;
+    int kt = (int)(g - tb);
+    const uint8_t* tri = a.cls + a.traj_tri[b];
+    int cnt = 0;
+    for (int qt = kt + lane; qt < nt; qt += 32) cnt += tri[(int64_t)qt * (qt + 1) / 2 + kt] != MW_TILE_EMPTY;
+    cnt = warp_sum_i(cnt);
+    if (lane == 0) a.bwd_cnt[g] = cnt;
+}
+
+// Single block: exclusive scans of both count arrays into the list pointers.
+__global__ void k_scan(BuildArgs a) {
+    __shared__ int carry[2];
+    __shared__ int wsum[2][32];
+    int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    if (threadIdx.x < 2) carry[threadIdx.x] = 0;
+    __syncthreads();
+    for (int64_t c0 = 0; c0 < a.n_tiles; c0 += blockDim.x) {
+        int64_t i = c0 + threadIdx.x;
+        int v[2];
+        v[0] = i < a.n_tiles ? a.fwd_cnt[i] : 0;
+        v[1] = i < a.n_tiles ? a.bwd_cnt[i] : 0;
+        int inc[2];
+        for (int q = 0; q < 2; ++q) {
+            int x = v[q];
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                int y = __shfl_up_sync(0xffffffffu, x, o);
+                if (lane >= o) x += y;
+            }
+            inc[q] = x;
+            if (lane == 31) wsum[q][w] = x;
+        }
+        __syncthreads();
+        if (w == 0) {
+            for (int q = 0; q < 2; ++q) {
+                int x = lane < nw ? wsum[q][lane] : 0;
+#pragma unroll
+                for (int o = 1; o < 32; o <<= 1) {
+                    int y = __shfl_up_sync(0xffffffffu, x, o);
+                    if (lane >= o) x += y;
+                }
+                if (lane < nw) wsum[q][lane] = x;  // inclusive over warps
+            }
+        }
+        __syncthreads();
+        for (int q = 0; q < 2; ++q) {
+            int before = carry[q] + (w > 0 ? wsum[q][w - 1] : 0) + inc[q] - v[q];
+            int32_t* ptr = q == 0 ? a.fwd_ptr : a.bwd_ptr;
+            if (i < a.n_tiles) ptr[i] = before;
+        }
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            carry[0] += wsum[0][nw - 1];
+            carry[1] += wsum[1][nw - 1];
+        }
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) {
+        a.fwd_ptr[a.n_tiles] = carry[0];
+        a.bwd_ptr[a.n_tiles] = carry[1];
+    }
+}
+
+// One warp per global q-tile (fwd) or k-tile (bwd): ordered compaction.
+__global__ void k_fill(BuildArgs a) {
+    int64_t g = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+    int lane = threadIdx.x & 31;
+    if (g >= a.n_tiles) return;
+    int b = a.tile_traj[g];
+    int tb = a.traj_tile[b], nt = a.traj_tile[b + 1] - tb;
+    int t = (int)(g - tb);
+    const uint8_t* tri = a.cls + a.traj_tri[b];
+    uint32_t lt = (1u << lane) - 1u;
+    int base = a.fwd_ptr[g];
+    for (int k0 = 0; k0 <= t; k0 += 32) {
+        int kt = k0 + lane;
+        int c = kt <= t ? tri[(int64_t)t * (t + 1) / 2 + kt] : MW_TILE_EMPTY;
+        uint32_t m = __ballot_sync(0xffffffffu, c != MW_TILE_EMPTY);
+        if (c != MW_TILE_EMPTY) a.fwd_idx[base + __popc(m & lt)] = (kt << 2) | c;
+        base += __popc(m);
+    }
+    base = a.bwd_ptr[g];
+    for (int q0 = t; q0 < nt; q0 += 32) {
+        int qt = q0 + lane;
+        int c = qt < nt ? tri[(int64_t)qt * (qt + 1) / 2 + t] : MW_TILE_EMPTY;
+        uint32_t m = __ballot_sync(0xffffffffu, c != MW_TILE_EMPTY);
+        if (c != MW_TILE_EMPTY) a.bwd_idx[base + __popc(m & lt)] = (qt << 2) | c;
+        base += __popc(m);
+    }
+}
+
+}  // namespace
+
+// ---------------------------------------------------------------------------
+
+extern "C" mw_status mw_build_visibility(const mw_vis_layout* L, const int32_t* cu, int n_junc,
+                                         const int32_t* J, const int32_t* jt,
+                                         const int32_t* span_off, const int32_t* spans,
+                                         void* ws, void* vis, void* stream_) {
+    if (!L) return MW_EINVAL;
+    if (n_junc != L->n_junc) return MW_EINVAL;
+    mw_status st = check_shape(L->n_traj, cu, n_junc, jt, L->n_spans);
+    if (st != MW_OK) return st;
+    const int n_traj = L->n_traj;
+    if (n_traj > 0 && cu[n_traj] != L->total_tokens) return MW_EINVAL;
+    if (n_junc > 0 && (!J || !span_off)) return MW_EINVAL;
+    if (L->n_spans > 0 && !spans) return MW_EINVAL;
+    if (L->vis_bytes > 0 && !vis) return MW_EINVAL;
+    if (L->ws_bytes > 0 && !ws) return MW_EINVAL;
+    if (n_junc > 0 && (span_off[0] != 0 || span_off[n_junc] != L->n_spans)) return MW_EEDITS;
+    // validate junctions and spans (App. B Def. "trajectory tree")
+    for (int k = 0; k < n_junc; ++k) {
+        int b = jt[k];
+        int T = cu[b + 1] - cu[b];
+        if (J[k] < 1 || J[k] > T - 1) return MW_EEDITS;
+        if (k > 0 && jt[k - 1] == b && J[k] <= J[k - 1]) return MW_EEDITS;
+        if (span_off[k + 1] < span_off[k]) return MW_EEDITS;
+        for (int s = span_off[k]; s < span_off[k + 1]; ++s) {
+            int a0 = spans[2 * s], b0 = spans[2 * s + 1];
+            if (!(0 <= a0 && a0 < b0 && b0 <= J[k])) return MW_EEDITS;
+        }
+    }
+    cudaStream_t stream = (cudaStream_t)stream_;
+    if (L->vis_bytes == 0) return MW_OK;
+
+    // host-side packing of the small per-trajectory tables
+    const int64_t n_tiles = L->n_tiles;
+    std::vector<int32_t> traj_tile(n_traj + 1), traj_seg(n_traj + 1), seg_start(L->n_segs),
+        tile_traj(n_tiles);
+    std::vector<int64_t> traj_tri(n_traj + 1), traj_km(n_traj + 1);
+    {
+        int k = 0;
+        int64_t tiles = 0, tri = 0, km = 0;
+        int segs = 0;
+        for (int b = 0; b < n_traj; ++b) {
+            int64_t nt = ceil_div(cu[b + 1] - cu[b], MW_TILE);
+            traj_tile[b] = (int32_t)tiles;
+            traj_tri[b] = tri;
+            traj_km[b] = km;
+            traj_seg[b] = segs;
+            seg_start[segs++] = 0;
+            int Kb = 0;
+            while (k < n_junc && jt[k] == b) { seg_start[segs++] = J[k]; ++k; ++Kb; }
+            for (int64_t t = 0; t < nt; ++t) tile_traj[tiles + t] = b;
+            tiles += nt;
+            tri += nt * (nt + 1) / 2;
+            km += (1 + Kb) * nt;
+        }
+        traj_tile[n_traj] = (int32_t)tiles;
+        traj_tri[n_traj] = tri;
+        traj_km[n_traj] = km;
+        traj_seg[n_traj] = segs;
+    }
+    std::vector<int32_t> span3(3 * (size_t)L->n_spans);
+    for (int k = 0; k < n_junc; ++k)
+        for (int s = span_off[k]; s < span_off[k + 1]; ++s) {
+            span3[3 * s] = cu[jt[k]] + spans[2 * s];
+            span3[3 * s + 1] = cu[jt[k]] + spans[2 * s + 1];
+            span3[3 * s + 2] = J[k];
+        }
+
+    // one contiguous host image of the metadata region [off_traj_tok, off_cls)
+    // plus the span table; two copies.
+    const int64_t meta0 = L->off_traj_tok, meta1 = L->off_cls;
+    std::vector<char> img(meta1 - meta0, 0);
+    auto put = [&](int64_t off, const void* src, size_t bytes) {
+        if (bytes) memcpy(img.data() + (off - meta0), src, bytes);
+    };
+    put(L->off_traj_tok, cu, 4 * (size_t)(n_traj + 1));
+    put(L->off_traj_tile, traj_tile.data(), 4 * traj_tile.size());
+    put(L->off_traj_seg, traj_seg.data(), 4 * traj_seg.size());
+    put(L->off_traj_tri, traj_tri.data(), 8 * traj_tri.size());
+    put(L->off_traj_km, traj_km.data(), 8 * traj_km.size());
+    put(L->off_seg_start, seg_start.data(), 4 * seg_start.size());
+    put(L->off_tile_traj, tile_traj.data(), 4 * tile_traj.size());
+    if ((st = cuda_status(cudaMemcpyAsync(at<char>(vis, meta0), img.data(), img.size(),
+                                          cudaMemcpyHostToDevice, stream))) != MW_OK)
+        return st;
+    if (L->n_spans > 0 &&
+        (st = cuda_status(cudaMemcpyAsync(at<char>(ws, L->ws_off_spans), span3.data(),
+                                          span3.size() * 4, cudaMemcpyHostToDevice, stream))) != MW_OK)
+        return st;
+    if ((st = cuda_status(cudaMemsetAsync(at<char>(vis, L->off_pairs), 0, 8 * (n_traj + 1), stream))) != MW_OK)
+        return st;
+    if ((st = cuda_status(cudaMemsetAsync(at<char>(vis, L->off_status), 0, 32, stream))) != MW_OK)
+        return st;
+
+    BuildArgs a;
+    a.n_traj = n_traj;
+    a.total = L->total_tokens;
+    a.n_tiles = n_tiles;
+    a.n_spans = L->n_spans;
+    a.omega = at<int32_t>(vis, L->off_omega);
+    a.seg = at<int32_t>(vis, L->off_seg);
+    a.traj_tok = at<int32_t>(vis, L->off_traj_tok);
+    a.traj_tile = at<int32_t>(vis, L->off_traj_tile);
+    a.traj_seg = at<int32_t>(vis, L->off_traj_seg);
+    a.traj_tri = at<int64_t>(vis, L->off_traj_tri);
+    a.traj_km = at<int64_t>(vis, L->off_traj_km);
+    a.seg_start = at<int32_t>(vis, L->off_seg_start);
+    a.tile_traj = at<int32_t>(vis, L->off_tile_traj);
+    a.cls = at<uint8_t>(vis, L->off_cls);
+    a.fwd_ptr = at<int32_t>(vis, L->off_fwd_ptr);
+    a.fwd_idx = at<int32_t>(vis, L->off_fwd_idx);
+    a.bwd_ptr = at<int32_t>(vis, L->off_bwd_ptr);
+    a.bwd_idx = at<int32_t>(vis, L->off_bwd_idx);
+    a.pairs = at<unsigned long long>(vis, L->off_pairs);
+    a.keymask = at<uint32_t>(vis, L->off_keymask);
+    a.spans = at<int32_t>(ws, L->ws_off_spans);
+    a.tstat = at<int32_t>(ws, L->ws_off_tstat);
+    a.fwd_cnt = at<int32_t>(ws, L->ws_off_cnt);
+    a.bwd_cnt = at<int32_t>(ws, L->ws_off_cnt) + n_tiles;
+
+    if (a.total > 0) {
+        int grid = (int)std::min<int64_t>(ceil_div(a.total, 256), 152 * 16);
+        k_init_tokens<<<grid, 256, 0, stream>>>(a);
+        if (L->n_spans > 0) k_scatter_spans<<<(int)std::min<int64_t>(L->n_spans, 152 * 8), 256, 0, stream>>>(a);
+    }
+    if (n_tiles > 0) {
+        k_tile_stats<<<(unsigned)n_tiles, MW_TILE, 0, stream>>>(a);
+        unsigned wgrid = (unsigned)ceil_div(n_tiles * 32, 256);
+        k_classify<<<wgrid, 256, 0, stream>>>(a);
+        k_bwd_count<<<wgrid, 256, 0, stream>>>(a);
+    }
+    k_scan<<<1, 1024, 0, stream>>>(a);
+    if (n_tiles > 0) k_fill<<<(unsigned)ceil_div(n_tiles * 32, 256), 256, 0, stream>>>(a);
+    return launch_status();
+}
+
+extern "C" mw_status mw_check_status(const mw_vis_layout* L, const void* vis, void* stream) {
+    if (!L || !vis) return MW_EINVAL;
+    int32_t h[8];
+    mw_status st = cuda_status(cudaMemcpyAsync(h, at<char>(vis, L->off_status), sizeof(h),
+                                               cudaMemcpyDeviceToHost, (cudaStream_t)stream));
+    if (st != MW_OK) return st;
+    if ((st = cuda_status(cudaStreamSynchronize((cudaStream_t)stream))) != MW_OK) return st;
+    if (h[ST_TIMEOUT]) return MW_ETIMEOUT;
+    if (h[ST_BOUNDS]) return MW_EDEVICE;
+    return MW_OK;
+}

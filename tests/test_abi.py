@@ -1,0 +1,113 @@
+"""C-ABI checks that need no GPU: the library loads, exports every symbol the
+header declares, and rejects malformed calls on the host before any launch."""
+
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _lib():
+    mw = pytest.importorskip("paper_2609_00865_gb300")
+    from paper_2609_00865_gb300 import _lib as L
+    if not os.path.exists(L.LIB_PATH):
+        from paper_2609_00865_gb300 import build as B
+        B.build()
+    return L, L._lib()
+
+
+def _declared():
+    names = set()
+    for f in os.listdir(os.path.join(ROOT, "include")):
+        if f.endswith(".h"):
+            src = open(os.path.join(ROOT, "include", f)).read()
+            names |= set(re.findall(r"^\s*(?:const\s+)?\w+\s*\*?\s*(mw_\w+)\s*\(", src, re.M))
+    return names
+
+
+def test_header_symbols_exported():
+    L, h = _lib()
+    declared = _declared()
+    assert {"mw_build_visibility", "mw_masked_attn_fwd", "mw_masked_attn_bwd",
+            "mw_logprob_loss_fwd", "mw_logprob_loss_bwd"} <= declared
+    for name in declared:
+        assert hasattr(h, name), name
+    assert declared <= set(L.exported_names())
+
+
+def test_status_strings_and_version():
+    L, h = _lib()
+    assert h.mw_status_str(0) == b"ok"
+    assert b"junction" in h.mw_status_str(2)
+    assert h.mw_abi_version() >= 1
+
+
+def test_layout_is_host_only_and_consistent():
+    L, h = _lib()
+    cu = np.array([0, 300, 300, 1000], np.int32)   # includes an empty trajectory
+    lay = L.mw_visibility_layout(cu, np.array([0, 2, 2], np.int32), 5)
+    assert lay.n_traj == 3 and lay.total_tokens == 1000
+    assert lay.n_tiles == 3 + 0 + 6
+    assert lay.n_tri == 6 + 0 + 21
+    assert lay.n_keymask == 2 * 3 + 1 * 0 + 3 * 6
+    offs = sorted(getattr(lay, f) for f, _ in L.VisLayout._fields_ if f.startswith("off_"))
+    assert all(o % 256 == 0 for o in offs) and offs == sorted(set(offs))
+    assert lay.vis_bytes >= offs[-1]
+
+
+@pytest.mark.parametrize("cu,jt,err", [
+    ([5, 10], [], 2),          # cu_seqlens must start at 0
+    ([0, 10, 5], [], 2),       # decreasing offsets
+    ([0, 10], [1], 2),         # junction names a missing trajectory
+    ([0, 10, 20], [1, 0], 2),  # junctions not grouped by trajectory
+])
+def test_layout_rejects_bad_shapes(cu, jt, err):
+    L, h = _lib()
+    with pytest.raises(L.MWError) as e:
+        L.mw_visibility_layout(np.array(cu, np.int32), np.array(jt, np.int32), 0)
+    assert e.value.status == err
+
+
+@pytest.mark.parametrize("J,spans,off", [
+    ([0], [], [0, 0]),              # junction at 0
+    ([10], [], [0, 0]),             # junction at T
+    ([5, 5], [], [0, 0, 0]),        # not ascending
+    ([5], [[2, 7]], [0, 1]),        # span past J
+    ([5], [[3, 3]], [0, 1]),        # empty span
+    ([5], [[-1, 2]], [0, 1]),       # negative start
+])
+def test_build_rejects_bad_records_before_launch(J, spans, off):
+    """Validation runs on the host; with null device buffers nothing could
+    be launched, so an MW_EEDITS here proves the check precedes any launch."""
+    L, h = _lib()
+    cu = np.array([0, 10], np.int32)
+    jt = np.zeros(len(J), np.int32)
+    lay = L.mw_visibility_layout(cu, jt, len(spans))
+    sp = np.array(spans, np.int32).reshape(-1)
+    st = h.mw_build_visibility(ctypes.byref(lay), cu.ctypes.data_as(L._IP), len(J),
+                               np.array(J, np.int32).ctypes.data_as(L._IP), jt.ctypes.data_as(L._IP),
+                               np.array(off, np.int32).ctypes.data_as(L._IP),
+                               sp.ctypes.data_as(L._IP) if sp.size else None,
+                               ctypes.c_void_p(16), ctypes.c_void_p(16), None)
+    assert st == 2
+
+
+def test_attention_and_lmhead_reject_bad_args_on_host():
+    L, h = _lib()
+    lay = L.mw_visibility_layout(np.array([0, 10], np.int32), np.zeros(0, np.int32), 0)
+    P = ctypes.c_void_p(16)
+    # Hq not a multiple of Hkv
+    assert h.mw_masked_attn_fwd(ctypes.byref(lay), P, P, P, P, P, P, 6, 4, 128, 1, 0.1, None) == 3
+    # bad dtype, bad head dim, bad scale
+    assert h.mw_masked_attn_fwd(ctypes.byref(lay), P, P, P, P, P, P, 4, 4, 128, 7, 0.1, None) == 4
+    assert h.mw_masked_attn_fwd(ctypes.byref(lay), P, P, P, P, P, P, 4, 4, 96, 1, 0.1, None) == 3
+    assert h.mw_masked_attn_fwd(ctypes.byref(lay), P, P, P, P, P, P, 4, 4, 128, 1, -1.0, None) == 1
+    # log-prob: M > N, bad eps, null loss
+    n = ctypes.c_size_t()
+    assert h.mw_logprob_ws(10, 11, 128, 100, 0, ctypes.byref(n)) == 3
+    assert h.mw_logprob_loss_fwd(P, P, P, P, 4, P, P, 1.5, 0.2, 10, 128, 100, 0, P, P, P, P, P, None) == 1
+    assert h.mw_logprob_loss_fwd(P, P, P, P, 4, P, P, 0.2, 0.2, 10, 128, 100, 0, P, P, P, None, P, None) == 1

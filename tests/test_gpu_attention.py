@@ -1,0 +1,103 @@
+"""GPU masked attention (fwd + bwd) vs the per-segment oracle."""
+
+import numpy as np
+import pytest
+import torch
+
+import synth
+from helpers import assert_grad_bf16, assert_maxabs, assert_rel, np64
+from oracle import attention as OA
+
+pytestmark = pytest.mark.gpu
+
+
+def _tensors(T, Hq, Hkv, Dh, seed, dtype):
+    Q = synth.normal((T, Hq, Dh), seed).to(dtype)
+    K = synth.normal((T, Hkv, Dh), seed + 1).to(dtype)
+    V = synth.normal((T, Hkv, Dh), seed + 2).to(dtype)
+    dO = synth.normal((T, Hq, Dh), seed + 3).to(dtype)
+    return Q, K, V, dO
+
+
+def _run(seqlens, edits, Q, K, V, dO, scale):
+    import paper_2609_00865_gb300 as mw
+    vis = mw.build_visibility(seqlens, edits)
+    q, k, v, do = (t.cuda() for t in (Q, K, V, dO))
+    O, LSE = mw.masked_attn_fwd(vis, q, k, v, scale)
+    dQ, dK, dV = mw.masked_attn_bwd(vis, q, k, v, O, do, LSE, scale)
+    torch.cuda.synchronize()
+    return O, LSE, dQ, dK, dV
+
+
+def _medium_record(seed):
+    rng = np.random.default_rng(seed)
+    seqlens = [700, 1000, 333]
+    edits = []
+    for T in seqlens:
+        Js = sorted(rng.choice(np.arange(64, T), size=3, replace=False).tolist())
+        e = []
+        for J in Js:
+            sp = []
+            for _ in range(3):
+                a = int(rng.integers(0, J - 1))
+                sp.append((a, min(J, a + int(rng.integers(1, 120)))))
+            e.append((J, sp))
+        edits.append(e)
+    return seqlens, edits
+
+
+def test_config1_fp32_full():
+    """Config 1 (tiny fp32): every output within 1e-4 relative."""
+    c = synth.CONFIGS[1]
+    r = synth.config_record(1)
+    Q, K, V, dO = _tensors(r.total, c["Hq"], c["Hkv"], c["Dh"], 11, torch.float32)
+    scale = c["Dh"] ** -0.5
+    O, LSE, dQ, dK, dV = _run(r.seqlens, r.edits, Q, K, V, dO, scale)
+    Or, Lr = OA.attn_fwd(r.seqlens, r.edits, np64(Q), np64(K), np64(V), scale)
+    assert_rel(np64(O), Or, 1e-4, "O")
+    assert_rel(np64(LSE), Lr, 1e-4, "LSE")
+    dQr, dKr, dVr = OA.attn_bwd(r.seqlens, r.edits, np64(Q), np64(K), np64(V), np64(dO), scale)
+    assert_rel(np64(dQ), dQr, 1e-4, "dQ")
+    assert_rel(np64(dK), dKr, 1e-4, "dK")
+    assert_rel(np64(dV), dVr, 1e-4, "dV")
+
+
+@pytest.mark.parametrize("Dh", [64, 128])
+def test_medium_fp32_gqa(Dh):
+    seqlens, edits = _medium_record(5)
+    Q, K, V, dO = _tensors(sum(seqlens), 8, 2, Dh, 21, torch.float32)
+    scale = Dh ** -0.5
+    O, LSE, dQ, dK, dV = _run(seqlens, edits, Q, K, V, dO, scale)
+    Or, Lr = OA.attn_fwd(seqlens, edits, np64(Q), np64(K), np64(V), scale)
+    assert_rel(np64(O), Or, 1e-4, "O")
+    assert_rel(np64(LSE), Lr, 1e-4, "LSE")
+    dQr, dKr, dVr = OA.attn_bwd(seqlens, edits, np64(Q), np64(K), np64(V), np64(dO), scale)
+    assert_rel(np64(dQ), dQr, 1e-4, "dQ")
+    assert_rel(np64(dK), dKr, 1e-4, "dK")
+    assert_rel(np64(dV), dVr, 1e-4, "dV")
+
+
+def test_medium_bf16_gqa():
+    seqlens, edits = _medium_record(6)
+    Q, K, V, dO = _tensors(sum(seqlens), 8, 2, 128, 31, torch.bfloat16)
+    scale = 128 ** -0.5
+    O, LSE, dQ, dK, dV = _run(seqlens, edits, Q, K, V, dO, scale)
+    Or, Lr = OA.attn_fwd(seqlens, edits, np64(Q), np64(K), np64(V), scale)
+    assert_maxabs(np64(O), Or, 2e-2, "O")
+    assert_maxabs(np64(LSE), Lr, 2e-2, "LSE")
+    dQr, dKr, dVr = OA.attn_bwd(seqlens, edits, np64(Q), np64(K), np64(V), np64(dO), scale)
+    assert_grad_bf16(np64(dQ), dQr, "dQ")
+    assert_grad_bf16(np64(dK), dKr, "dK")
+    assert_grad_bf16(np64(dV), dVr, "dV")
+
+
+def test_no_edits_is_causal_attention():
+    """K = 0 reduces to ordinary causal attention (library SDPA on the GPU
+    output's inputs, float64 on the CPU)."""
+    T, H, Dh = 300, 2, 64
+    Q, K, V, dO = _tensors(T, H, H, Dh, 41, torch.float32)
+    O, LSE, *_ = _run([T], [[]], Q, K, V, dO, 0.125)
+    ref = torch.nn.functional.scaled_dot_product_attention(
+        Q.double().permute(1, 0, 2), K.double().permute(1, 0, 2), V.double().permute(1, 0, 2),
+        is_causal=True, scale=0.125).permute(1, 0, 2).numpy()
+    assert_rel(np64(O), ref, 1e-4, "O")

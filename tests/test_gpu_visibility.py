@@ -1,0 +1,94 @@
+"""GPU visibility builder vs the oracle, bit for bit (every array)."""
+
+import json
+import os
+
+import numpy as np
+import pytest
+
+import synth
+from oracle import visibility as OV
+
+pytestmark = pytest.mark.gpu
+
+
+def _gpu(seqlens, edits):
+    import torch
+    import paper_2609_00865_gb300 as mw
+    vis = mw.build_visibility(seqlens, edits)
+    torch.cuda.synchronize()
+    vis.check_status()
+    return vis.arrays()
+
+
+def _compare(seqlens, edits):
+    got = _gpu(seqlens, edits)
+    want = OV.build(seqlens, edits)
+    for key in ("omega", "seg", "qtile_traj", "fwd_ptr", "fwd_idx", "bwd_ptr", "bwd_idx", "pairs", "keymask"):
+        np.testing.assert_array_equal(got[key], want[key], err_msg=key)
+    assert got["pairs_total"] == want["pairs_total"]
+    assert len(got["cls"]) == len(want["cls"])
+    for a, b in zip(got["cls"], want["cls"]):
+        np.testing.assert_array_equal(np.tril(a), np.tril(b), err_msg="cls")
+    return got
+
+
+def test_running_example():
+    g = json.load(open(os.path.join(os.path.dirname(__file__), "golden", "running_example.json")))
+    edits = [(J, [tuple(s) for s in sp]) for J, sp in g["edits"]]
+    got = _compare([14], [edits])
+    assert list(got["omega"][[5, 8, 11]]) == [7, 10, 12]
+
+
+def _rand_record(rng, n_traj):
+    seqlens, edits = [], []
+    for _ in range(n_traj):
+        T = int(rng.choice([1, 2, 127, 128, 129, 300, 777, 1024, 1500]))
+        K = int(rng.integers(0, min(6, T - 1) + 1)) if T > 1 else 0
+        Js = sorted(rng.choice(np.arange(1, T), size=K, replace=False).tolist()) if K else []
+        e = []
+        for J in Js:
+            sp = []
+            for _ in range(int(rng.integers(0, 5))):
+                a = int(rng.integers(0, J))
+                sp.append((a, int(rng.integers(a + 1, J + 1))))
+            e.append((J, sp))
+        seqlens.append(T)
+        edits.append(e)
+    return seqlens, edits
+
+
+@pytest.mark.parametrize("seed", range(10))
+def test_random_records(seed):
+    rng = np.random.default_rng(seed)
+    _compare(*_rand_record(rng, int(rng.integers(1, 6))))
+
+
+def test_empty_trajectory_inside_record():
+    _compare([300, 0, 129], [[(100, [(0, 50)])], [], [(5, [(1, 3)])]])
+
+
+def test_empty_record():
+    import paper_2609_00865_gb300 as mw
+    vis = mw.build_visibility([], [])
+    assert vis.layout.n_tiles == 0 and vis.pairs_total == 0
+
+
+@pytest.mark.parametrize("cfg", [1, 2, 4])
+def test_config_records(cfg):
+    r = synth.config_record(cfg)
+    _compare(r.seqlens, r.edits)
+
+
+@pytest.mark.parametrize("K", synth.CONFIGS[5]["sweep_K"])
+@pytest.mark.parametrize("f", synth.CONFIGS[5]["sweep_f"])
+def test_sweep_records(K, f):
+    r = synth.config_record(5, K=K, f=f)
+    _compare(r.seqlens, r.edits)
+
+
+def test_bad_record_raises():
+    import paper_2609_00865_gb300 as mw
+    with pytest.raises(mw.MWError) as e:
+        mw.build_visibility([50], [[(10, [(5, 12)])]])
+    assert e.value.status == 2

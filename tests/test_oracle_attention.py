@@ -146,3 +146,13 @@ def test_backward_finite_differences():
         args2 = [a2 if arr is x else x for x in (Q, K, V_)]
         fd = (f(*args1) - f(*args2)) / (2 * eps)
         assert abs(fd - grad[idx]) < 1e-6 * max(1.0, abs(fd))
+
+
+def test_row_sampled_dq_matches_full():
+    T, Hq, Hkv, Dh = 64, 4, 2, 8
+    edits = _edits(T, 30, 3)
+    Q, K, V_, dO = _inputs(T, Hq, Hkv, Dh, 30)
+    dQ, _, _ = A.attn_bwd([T], [edits], Q, K, V_, dO, 0.4)
+    rows = [0, 63, 20, 41]
+    got = A.attn_bwd_rows([T], [edits], Q, K, V_, dO, 0.4, rows, [0, 3])
+    np.testing.assert_allclose(got, dQ[rows][:, [0, 3]], rtol=1e-11, atol=1e-13)
