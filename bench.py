@@ -1,0 +1,486 @@
+"""Benchmark: view-consistent scored tokens/s (fwd+bwd) of the whole hot path.
+
+Default workload (N=1): the 7B-shaped layer step -- 2 x 65,536 tokens, 8
+junctions per trajectory at 70% eviction with 1,024-token summaries, masked
+GQA attention 28/4 heads Dh 128 fwd+bwd chained into the fused LM-head
+log-prob + clipped loss (d = 3,584, V = 152,064) fwd+bwd. One step runs every
+step of the path: visibility build, attention fwd, LM-head fwd + loss,
+LM-head bwd, attention bwd (dO = dH). Scored tokens are the loss rows.
+Other workloads: ``--config 2`` (attention op, 8 x 16,384), ``--config 3``
+(log-prob loss, N = 32,768), ``--config 5 --K k --f f`` (one sweep point).
+
+``--impl reference`` times the CPU oracle (the only reference this method has)
+on a bounded sample of the same workload. Under torchrun every rank runs its
+own replica (trajectories are independent): weak scaling, no collective on
+the data path; rank 0 prints one JSON line.
+"""
+
+import argparse
+import json
+import os
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "view-consistent scored tokens/sec (fwd+bwd)"
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["bf16_tflops"]), float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 1900.0, 6800.0, "fallback"
+
+
+class Clocks:
+    """nvidia-smi sampler running while the timed region runs."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.path = tempfile.mktemp(suffix=".csv")
+
+    def start(self):
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.f.close()
+        sm, mx, reasons = [], 0.0, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            p = [x.strip() for x in line.split(",")]
+            if len(p) < 9:
+                continue
+            try:
+                sm.append(float(p[1]))
+                mx = max(mx, float(p[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, p[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        os.unlink(self.path)
+        if not sm:
+            return None
+        sm.sort()
+        return {"sm_mhz": sm[len(sm) // 2], "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ----------------------------------------------------------------------------- workloads
+
+def make_workload(cfg, K=None, f=None, seed_offset=0):
+    """Host-side inputs of one workload (pinned CPU tensors + record)."""
+    import numpy as np
+    import torch
+
+    import synth
+    c = synth.CONFIGS[cfg]
+    g = torch.Generator().manual_seed(1000 * cfg + 17 + seed_offset)
+    w = {"cfg": cfg}
+    bf = torch.bfloat16
+
+    def randn(*shape, std=1.0):
+        t = torch.randn(*shape, generator=g, dtype=torch.float32)
+        if std != 1.0:
+            t.mul_(std)
+        return t.to(bf).pin_memory()
+
+    if cfg in (2, 4, 5):
+        rec = synth.config_record(cfg, K=K, f=f)
+        w["record"] = rec
+        T = rec.total
+        w["Q"] = randn(T, c["Hq"], c["Dh"])
+        w["K"] = randn(T, c["Hkv"], c["Dh"])
+        w["V"] = randn(T, c["Hkv"], c["Dh"])
+        w["heads"] = (c["Hq"], c["Hkv"], c["Dh"])
+        if cfg != 4:
+            w["dO"] = randn(T, c["Hq"], c["Dh"])
+    if cfg in (3, 4):
+        if cfg == 3:
+            N, d = c["N"], c["d"]
+            rows = synth.loss_rows_fraction(N, c["loss_frac"], 3000)
+            w["H"] = randn(N, d)
+        else:
+            N, d = w["record"].total, c["Hq"] * c["Dh"]
+            rows = w["record"].loss_rows()
+        w["N"], w["d"], w["Vocab"] = N, d, c["V"]
+        w["W"] = randn(c["V"], d, std=0.02)
+        w["targets"] = torch.randint(0, c["V"], (N,), generator=g, dtype=torch.int32).pin_memory()
+        w["rows"] = torch.tensor(rows, dtype=torch.int32).pin_memory()
+        M = len(rows)
+        w["adv"] = torch.randn(M, generator=g).pin_memory()
+        w["noise"] = (0.05 * torch.randn(M, generator=g)).pin_memory()
+    return w
+
+
+def describe(w):
+    import synth
+    c = synth.CONFIGS[w["cfg"]]
+    d = {"workload": c["name"]}
+    if "record" in w:
+        r = w["record"]
+        d.update(trajectories=len(r.trajs), tokens=r.total,
+                 junctions=sum(len(e) for e in r.edits), heads=f"{w['heads'][0]}/{w['heads'][1]}",
+                 head_dim=w["heads"][2])
+    if "rows" in w:
+        d.update(loss_rows=int(w["rows"].numel()), hidden=w["d"], vocab=w["Vocab"])
+    d["l2"] = "inputs larger than L2 (129 MB); no flush"
+    return d
+
+
+class Step:
+    """Device buffers and one pass of the hot path through the public API."""
+
+    def __init__(self, w, device):
+        import torch
+
+        import paper_2609_00865_gb300 as mw
+        self.mw = mw
+        self.w = w
+        self.dev = device
+        self.stream = torch.cuda.current_stream(device)
+        self.d = {k: v.to(device, non_blocking=True) for k, v in w.items() if isinstance(v, torch.Tensor)}
+        self.events = {}
+        self.timing = False
+        if "record" in w:
+            r = w["record"]
+            self.flat = mw.flatten_record(r.seqlens, r.edits)
+            cu, J, jt, off, spans = self.flat
+            self.L = mw.mw_visibility_layout(cu, jt, len(spans))
+            self.vis = mw.Visibility(self.L, torch.empty(self.L.vis_bytes, dtype=torch.uint8, device=device),
+                                     torch.empty(max(self.L.ws_bytes, 1), dtype=torch.uint8, device=device))
+            Hq, Hkv, Dh = w["heads"]
+            self.scale = Dh ** -0.5
+            T = r.total
+            self.O = torch.empty(T, Hq, Dh, dtype=torch.bfloat16, device=device)
+            self.LSE = torch.empty(Hq, T, dtype=torch.float32, device=device)
+            self.dQ = torch.empty_like(self.O)
+            self.dK = torch.empty(T, Hkv, Dh, dtype=torch.bfloat16, device=device)
+            self.dV = torch.empty_like(self.dK)
+            nb = mw.mw_masked_attn_bwd_ws(self.vis, Hq, Dh, mw.MW_BF16)
+            self.attn_ws = torch.empty(max(nb, 1), dtype=torch.uint8, device=device)
+        if "rows" in w:
+            M = int(w["rows"].numel())
+            N, d, V = w["N"], w["d"], w["Vocab"]
+            self.lm_ws = torch.empty(max(mw.mw_logprob_ws(N, M, d, V, mw.MW_BF16), 1), dtype=torch.uint8,
+                                     device=device)
+            self.lp = torch.empty(M, dtype=torch.float32, device=device)
+            self.ratio = torch.empty_like(self.lp)
+            self.lse = torch.empty_like(self.lp)
+            self.loss = torch.empty(1, dtype=torch.float32, device=device)
+            self.dH = torch.empty(N, d, dtype=torch.bfloat16, device=device)
+            self.dW = torch.empty(V, d, dtype=torch.float32, device=device)
+            self.lp_old = torch.empty(M, dtype=torch.float32, device=device)
+
+    def _ev(self, name, fn):
+        import torch
+        if not self.timing:
+            return fn()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(self.stream)
+        r = fn()
+        b.record(self.stream)
+        self.events.setdefault(name, []).append((a, b))
+        return r
+
+    def H(self):
+        return self.O.view(self.O.shape[0], -1) if self.w["cfg"] == 4 else self.d["H"]
+
+    def prime(self):
+        """lp_old = current log-prob + N(0, 0.05) (computed once, untimed)."""
+        if "rows" not in self.w:
+            return
+        if "record" in self.w:
+            self.build()
+            self.attn_fwd()
+        self.d["lp_old"] = self.lp_old
+        self.lp_old.zero_()
+        self.lm_fwd()
+        self.lp_old.copy_(self.lp + self.d["noise"])
+
+    def build(self):
+        cu, J, jt, off, spans = self.flat
+        self._ev("mw_build_visibility", lambda: self.mw.mw_build_visibility(
+            self.L, cu, J, jt, off, spans, self.vis.ws, self.vis.vis, self.stream))
+
+    def attn_fwd(self):
+        self._ev("mw_masked_attn_fwd", lambda: self.mw.mw_masked_attn_fwd(
+            self.vis, self.d["Q"], self.d["K"], self.d["V"], self.O, self.LSE, self.scale, self.stream))
+
+    def attn_bwd(self, dO):
+        self._ev("mw_masked_attn_bwd", lambda: self.mw.mw_masked_attn_bwd(
+            self.vis, self.d["Q"], self.d["K"], self.d["V"], self.O, dO, self.LSE, self.dQ, self.dK, self.dV,
+            self.scale, self.attn_ws, self.stream))
+
+    def lm_fwd(self):
+        self._ev("mw_logprob_loss_fwd", lambda: self.mw.mw_logprob_loss_fwd(
+            self.H(), self.d["W"], self.d["targets"], self.d["rows"], self.lp_old, self.d["adv"], 0.2, 0.2,
+            self.lp, self.ratio, self.lse, self.loss, self.lm_ws, self.stream))
+
+    def lm_bwd(self):
+        self._ev("mw_logprob_loss_bwd", lambda: self.mw.mw_logprob_loss_bwd(
+            self.H(), self.d["W"], self.d["targets"], self.d["rows"], self.lse, self.lm_ws, 1.0, self.dH, self.dW,
+            self.stream))
+
+    def run(self):
+        cfg = self.w["cfg"]
+        if cfg in (2, 5):
+            self.build()
+            self.attn_fwd()
+            self.attn_bwd(self.d["dO"])
+        elif cfg == 3:
+            self.lm_fwd()
+            self.lm_bwd()
+        else:
+            self.build()
+            self.attn_fwd()
+            self.lm_fwd()
+            self.lm_bwd()
+            self.attn_bwd(self.dH.view_as(self.O))
+
+    def upload(self, host):
+        """e2e: copy this step's inputs from pinned host memory."""
+        for k, v in host.items():
+            if k in self.d:
+                self.d[k].copy_(v, non_blocking=True)
+
+    def scored(self):
+        return int(self.w["rows"].numel()) if "rows" in self.w else self.w["record"].total
+
+    def flops(self):
+        """Visible FLOPs per step: attention 14 P Dh Hq, LM head 8 M d V."""
+        f = {}
+        if "record" in self.w:
+            Hq, _, Dh = self.w["heads"]
+            f["attn"] = 14.0 * self.vis.pairs_total * Dh * Hq
+        if "rows" in self.w:
+            f["lm"] = 8.0 * self.w["rows"].numel() * self.w["d"] * self.w["Vocab"]
+        return f
+
+
+# ----------------------------------------------------------------------------- reference arm (CPU oracle)
+
+def cpu_sample(w, budget_s=15.0):
+    """Time the oracle on a bounded sample of loss rows of this workload.
+
+    Per sampled row: attention fwd + dQ over all query heads (its segment's
+    compact view), LM-head log-prob over the full vocabulary and the dH/dW
+    contributions of that row. Returns (tokens/s, cores, description).
+    """
+    import numpy as np
+    import torch
+
+    from oracle import attention as OA
+    from oracle import logprob as OL
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    if "_f64" not in w:   # exact float64 copies of the bf16 inputs, made once
+        w["_f64"] = {k: w[k].to(torch.float64).numpy() for k in ("Q", "K", "V", "dO", "H", "W") if k in w}
+    x = w["_f64"]
+    rng = np.random.default_rng(5)
+    if "rows" in w:
+        pool = w["rows"].numpy().astype(np.int64)
+    else:
+        pool = np.arange(w["record"].total)
+    done, t0 = 0, time.perf_counter()
+    batch = 8
+    parts = []
+    while time.perf_counter() - t0 < budget_s and done < 4096:
+        rows = np.sort(rng.choice(pool, size=batch, replace=False))
+        parts = []
+        O = None
+        if "record" in w:
+            r = w["record"]
+            Hq, Hkv, Dh = w["heads"]
+            parts.append("attention fwd+dQ, all heads")
+            O, _ = OA.attn_fwd(r.seqlens, r.edits, x["Q"], x["K"], x["V"], Dh ** -0.5, rows=rows)
+            OA.attn_bwd_rows(r.seqlens, r.edits, x["Q"], x["K"], x["V"], x.get("dO", x["Q"]), Dh ** -0.5,
+                             rows, list(range(Hq)))
+        if "rows" in w:
+            parts.append("LM-head fwd over the full vocabulary + dH/dW")
+            if "H" in x:
+                H = x["H"]
+            else:       # chained: H rows are the oracle's own attention outputs
+                H = np.zeros((w["N"], w["d"]))
+                H[rows] = O.reshape(len(rows), -1)
+            lp, lse = OL.logprob(H, x["W"], w["targets"].numpy(), rows)
+            g = OL.policy_loss(lp, lp + 0.01, np.ones_like(lp), 0.2, 0.2)[3]
+            OL.logprob_loss_bwd(H, x["W"], w["targets"].numpy(), rows, lse, g)
+        done += batch
+    dt = time.perf_counter() - t0
+    return done / dt, cores, f"{done} sampled scored tokens ({' + '.join(parts)}), {dt:.1f} s"
+
+
+def run_reference(args, rank, world):
+    if rank != 0:
+        return
+    w = make_workload(args.config, args.K, args.f)
+    vals = []
+    for i in range(args.warmup + args.steps):
+        v, cores, desc = cpu_sample(w, budget_s=args.cpu_seconds / max(1, args.steps))
+        if i >= args.warmup:
+            vals.append(v)
+    v = sorted(vals)[len(vals) // 2]
+    line = {"impl": "reference", "metric": METRIC, "value": v, "unit": "tokens/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 / v, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": describe(w),
+            "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": cores, "kind": "oracle", "sample": desc},
+            "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ----------------------------------------------------------------------------- GPU arm
+
+def run_gpu(args, rank, world, local_rank):
+    import torch
+    import torch.distributed as dist
+
+    import paper_2609_00865_gb300 as mw
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    w = make_workload(args.config, args.K, args.f, seed_offset=rank)
+    step = Step(w, dev)
+    step.prime()
+    for _ in range(args.warmup):
+        step.run()
+    torch.cuda.synchronize()
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    clocks = Clocks(local_rank)
+    barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    step.timing = True
+    n0 = mw.kernel_launches()
+    ev0 = torch.cuda.Event(enable_timing=True)
+    ev1 = torch.cuda.Event(enable_timing=True)
+    ev0.record(step.stream)
+    for _ in range(args.steps):
+        step.run()
+    ev1.record(step.stream)
+    torch.cuda.synchronize()
+    launches = mw.kernel_launches() - n0
+    step.timing = False
+    ms = ev0.elapsed_time(ev1) / args.steps
+    clk = clocks.stop()
+    barrier()
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    per_call = {k: sum(a.elapsed_time(b) for a, b in v) / len(v) for k, v in step.events.items()}
+
+    # e2e: pinned host inputs -> device, step, loss/metric read back
+    host = {k: v for k, v in w.items() if isinstance(v, torch.Tensor) and k in step.d}
+    h2d = sum(v.numel() * v.element_size() for v in host.values())
+    out = step.loss if hasattr(step, "loss") else step.LSE[0, :1]
+    d2h = out.numel() * out.element_size()
+    pinned_out = torch.empty(out.shape, dtype=out.dtype).pin_memory()
+    barrier()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(step.stream)
+    for _ in range(args.steps):
+        step.upload(host)
+        step.run()
+        pinned_out.copy_(out, non_blocking=True)
+    e1.record(step.stream)
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1) / args.steps
+    if world > 1:
+        t = torch.tensor([e2e_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_ms = float(t.item())
+
+    if rank != 0:
+        return
+    scored = step.scored() * world
+    flops = step.flops()
+    peak_tf, hbm, peak_kind = _peaks()
+    dom = max(per_call, key=per_call.get)
+    dom_flops = {"mw_masked_attn_fwd": 4.0 / 14.0 * flops.get("attn", 0),
+                 "mw_masked_attn_bwd": 10.0 / 14.0 * flops.get("attn", 0),
+                 "mw_logprob_loss_fwd": 2.0 / 8.0 * flops.get("lm", 0),
+                 "mw_logprob_loss_bwd": 6.0 / 8.0 * flops.get("lm", 0)}.get(dom, 0.0)
+    achieved = dom_flops / (per_call[dom] * 1e-3) / 1e12
+    total_tf = sum(flops.values()) / (ms * 1e-3) / 1e12
+    cpu = None
+    if world == 1 and not args.no_cpu:
+        v, cores, desc = cpu_sample(w, budget_s=args.cpu_seconds)
+        cpu = {"value": v, "unit": "tokens/s", "cores": cores, "kind": "oracle", "sample": desc}
+    line = {
+        "metric": METRIC, "value": scored / (ms * 1e-3), "unit": "tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": describe(w),
+        "visible_tflops": total_tf, "visible_frac_of_peak": total_tf / peak_tf,
+        "roofline": {"bound": "tensor", "kernel": dom, "achieved": achieved, "peak": peak_tf,
+                     "unit": "TFLOP/s", "frac": achieved / peak_tf, "traffic": None,
+                     "peak_kind": f"bf16 dense burst, {peak_kind}"},
+        "per_call_ms": per_call,
+        "cpu_baseline": cpu,
+        "e2e": {"value": scored / (e2e_ms * 1e-3), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
+        "gpu_launches": launches,
+        "clocks": clk,
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="mw", choices=["mw", "reference"])
+    ap.add_argument("--config", type=int, default=4, choices=[2, 3, 4, 5])
+    ap.add_argument("--K", type=int, default=8)
+    ap.add_argument("--f", type=float, default=0.6)
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--no-cpu", action="store_true")
+    args = ap.parse_args()
+    rank = int(os.environ.get("RANK", 0))
+    world = int(os.environ.get("WORLD_SIZE", args.gpus if args.gpus == 1 else 1))
+    local_rank = int(os.environ.get("LOCAL_RANK", 0))
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl" if args.impl == "mw" else "gloo")
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+    else:
+        run_gpu(args, rank, world, local_rank)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -67,6 +67,9 @@ const char* mw_status_str(int status);
 int mw_last_cuda_error(void);
 /* ABI version of this header (bumped on any signature change). */
 int mw_abi_version(void);
+/* Number of CUDA kernels this library has launched in this process so far
+ * (all threads, all devices); lets callers count launches in a timed region. */
+uint64_t mw_kernel_launches(void);
 
 /*
  * Visibility layout: sizes and byte offsets of every array inside the

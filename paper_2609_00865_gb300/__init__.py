@@ -15,6 +15,7 @@ from ._lib import (  # noqa: F401
     build_visibility,
     exported_names,
     flatten_record,
+    kernel_launches,
     logprob_loss_bwd,
     logprob_loss_fwd,
     masked_attn_bwd,

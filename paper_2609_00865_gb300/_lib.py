@@ -48,6 +48,7 @@ _SIGS = {
     "mw_status_str": (ctypes.c_char_p, [_I]),
     "mw_last_cuda_error": (_I, []),
     "mw_abi_version": (_I, []),
+    "mw_kernel_launches": (ctypes.c_uint64, []),
     "mw_visibility_layout": (_I, [_I, _IP, _I, _IP, _I, _LP]),
     "mw_build_visibility": (_I, [_LP, _IP, _I, _IP, _IP, _IP, _IP, _P, _P, _P]),
     "mw_masked_attn_fwd": (_I, [_LP, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _F, _P]),
@@ -74,6 +75,11 @@ def _lib():
             fn.argtypes = args
         _handle = h
     return _handle
+
+
+def kernel_launches():
+    """Kernels libmw has launched in this process so far."""
+    return int(_lib().mw_kernel_launches())
 
 
 def exported_names():

@@ -15,6 +15,8 @@ mw_status lm_fwd_simt(const void*, const void*, const int32_t*, const int32_t*, 
                       float*, cudaStream_t);
 mw_status lm_bwd_simt(const void*, const void*, const int32_t*, const int32_t*, int, int, int, int, int,
                       const float*, const float*, float, void*, float*, cudaStream_t);
+mw_status attn_fwd_tc(const mw_vis_layout*, const void*, const void*, const void*, const void*, void*, float*, int,
+                      int, float, cudaStream_t);
 __global__ void k_loss_epilogue(int, const float*, const float*, const float*, float, float, float*, float*, float*);
 
 // Byte offsets inside the log-prob workspace.
@@ -53,6 +55,8 @@ extern "C" mw_status mw_masked_attn_fwd(const mw_vis_layout* L, const void* vis,
     if (st != MW_OK) return st;
     if (L->total_tokens == 0) return MW_OK;
     if (!Q || !K || !V || !O || !LSE) return MW_EINVAL;
+    if (dtype == MW_BF16 && Dh == 128)
+        return attn_fwd_tc(L, vis, Q, K, V, O, LSE, Hq, Hkv, scale, (cudaStream_t)stream);
     return attn_fwd_simt(L, vis, Q, K, V, O, LSE, Hq, Hkv, Dh, dtype, scale, (cudaStream_t)stream);
 }
 
@@ -105,6 +109,7 @@ extern "C" mw_status mw_logprob_loss_fwd(const void* H, const void* W, const int
     float* g = at<float>(ws, w.g);
     float* zt = at<float>(ws, w.zt);
     if ((st = lm_fwd_simt(H, W, targets, rows, M, d, V, dtype, lse, zt, lp, s)) != MW_OK) return st;
+    count_launches(1);
     k_loss_epilogue<<<1, 1024, 0, s>>>(M, lp, lp_old, adv, eps_lo, eps_hi, ratio, g, loss);
     return launch_status();
 }

@@ -241,6 +241,7 @@ mw_status fwd_impl(const mw_vis_layout* L, const void* vis, const void* Q, const
     if (L->n_tiles == 0 || Hq == 0) return MW_OK;
     VisView v = make_view(L, vis);
     dim3 grid((unsigned)L->n_tiles, (unsigned)Hq);
+    count_launches(1);
     k_attn_fwd_simt<Tin, DH><<<grid, 128, 0, s>>>(v, L->total_tokens, (const Tin*)Q, (const Tin*)K,
                                                   (const Tin*)V, (Tin*)O, LSE, Hq, Hkv, scale);
     return launch_status();
@@ -253,6 +254,7 @@ mw_status bwd_impl(const mw_vis_layout* L, const void* vis, const void* Q, const
     if (L->n_tiles == 0 || Hq == 0) return MW_OK;
     VisView v = make_view(L, vis);
     const int64_t warps = L->total_tokens * Hq;
+    count_launches(3);
     k_attn_delta<Tin, DH><<<(unsigned)std::min<int64_t>(ceil_div(warps, 8), 152 * 64), 256, 0, s>>>(
         L->total_tokens, Hq, (const Tin*)O, (const Tin*)dO, delta);
     dim3 gq((unsigned)L->n_tiles, (unsigned)Hq);

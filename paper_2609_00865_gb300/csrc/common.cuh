@@ -12,6 +12,8 @@ namespace mw {
 // Record the CUDA error (if any) in the thread-local slot and map to status.
 mw_status cuda_status(cudaError_t e);
 mw_status launch_status();
+// Count `n` kernel launches issued by the library (see mw_kernel_launches).
+void count_launches(int n);
 
 inline int64_t align256(int64_t x) { return (x + 255) & ~int64_t(255); }
 inline int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }

@@ -244,6 +244,7 @@ template <typename Tin>
 mw_status fwd_t(const void* H, const void* W, const int32_t* targets, const int32_t* rows, int M, int d, int Vocab,
                 float* lse, float* zt, float* lp, cudaStream_t s) {
     const size_t smem = sizeof(float) * FR * d;
+    count_launches(2);
     cudaFuncSetAttribute(k_lm_fwd_simt<Tin>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     k_lm_fwd_simt<Tin><<<(unsigned)ceil_div(M, FR), 256, smem, s>>>(M, d, Vocab, (const Tin*)H, (const Tin*)W,
                                                                     targets, rows, lse, zt);
@@ -257,6 +258,7 @@ mw_status bwd_t(const void* H, const void* W, const int32_t* targets, const int3
     mw_status st = cuda_status(cudaMemsetAsync(dH, 0, sizeof(Tin) * (size_t)N * d, s));
     if (st != MW_OK) return st;
     if (M == 0) return cuda_status(cudaMemsetAsync(dW, 0, sizeof(float) * (size_t)Vocab * d, s));
+    count_launches(2);
     const size_t smem_h = sizeof(float) * (FR * d + FR * 256);
     cudaFuncSetAttribute(k_lm_dh_simt<Tin>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_h);
     k_lm_dh_simt<Tin><<<(unsigned)ceil_div(M, FR), 256, smem_h, s>>>(M, d, Vocab, (const Tin*)H, (const Tin*)W,

@@ -11,6 +11,8 @@
 #include <stdlib.h>
 #include <string.h>
 
+#include <algorithm>
+#include <atomic>
 #include <vector>
 
 #include "common.cuh"
@@ -25,6 +27,9 @@ mw_status cuda_status(cudaError_t e) {
     return MW_ECUDA;
 }
 mw_status launch_status() { return cuda_status(cudaGetLastError()); }
+
+static std::atomic<unsigned long long> g_launches{0};
+void count_launches(int n) { g_launches.fetch_add((unsigned long long)n, std::memory_order_relaxed); }
 
 }  // namespace mw
 
@@ -47,6 +52,7 @@ extern "C" const char* mw_status_str(int s) {
 
 extern "C" int mw_last_cuda_error(void) { return g_last_cuda_error; }
 extern "C" int mw_abi_version(void) { return 1; }
+extern "C" uint64_t mw_kernel_launches(void) { return (uint64_t)g_launches.load(std::memory_order_relaxed); }
 
 static mw_status check_shape(int n_traj, const int32_t* cu, int n_junc, const int32_t* jt,
                              int n_spans) {
@@ -476,6 +482,7 @@ extern "C" mw_status mw_build_visibility(const mw_vis_layout* L, const int32_t* 
     a.fwd_cnt = at<int32_t>(ws, L->ws_off_cnt);
     a.bwd_cnt = at<int32_t>(ws, L->ws_off_cnt) + n_tiles;
 
+    count_launches((a.total > 0 ? 1 + (L->n_spans > 0) : 0) + (n_tiles > 0 ? 3 : 0) + 1 + (n_tiles > 0));
     if (a.total > 0) {
         int grid = (int)std::min<int64_t>(ceil_div(a.total, 256), 152 * 16);
         k_init_tokens<<<grid, 256, 0, stream>>>(a);
