@@ -101,3 +101,47 @@ def test_no_edits_is_causal_attention():
         Q.double().permute(1, 0, 2), K.double().permute(1, 0, 2), V.double().permute(1, 0, 2),
         is_causal=True, scale=0.125).permute(1, 0, 2).numpy()
     assert_rel(np64(O), ref, 1e-4, "O")
+
+
+def _sample_rows(rec, rng, n_random=24):
+    """Rows around every junction, trajectory ends, and random rows."""
+    rows, base = set(), 0
+    for t in rec.trajs:
+        rows.update({base, base + t.T - 1, base + min(127, t.T - 1), base + min(128, t.T - 1)})
+        for J, _ in t.edits[:3]:
+            rows.update({base + J - 1, base + J, base + min(J + 1, t.T - 1)})
+        base += t.T
+    rows.update(rng.integers(0, base, n_random).tolist())
+    return np.array(sorted(rows))
+
+
+def _full_size_fwd(rec, c, seed):
+    import paper_2609_00865_gb300 as mw
+    T = rec.total
+    g = torch.Generator(device="cuda").manual_seed(seed)
+    q = torch.randn(T, c["Hq"], c["Dh"], device="cuda", generator=g).to(torch.bfloat16)
+    k = torch.randn(T, c["Hkv"], c["Dh"], device="cuda", generator=g).to(torch.bfloat16)
+    v = torch.randn(T, c["Hkv"], c["Dh"], device="cuda", generator=g).to(torch.bfloat16)
+    vis = mw.build_visibility(rec.seqlens, rec.edits)
+    scale = c["Dh"] ** -0.5
+    O, LSE = mw.masked_attn_fwd(vis, q, k, v, scale)
+    torch.cuda.synchronize()
+    vis.check_status()
+    rng = np.random.default_rng(seed)
+    rows = _sample_rows(rec, rng)
+    heads = sorted(set(rng.integers(0, c["Hq"], 3).tolist()) | {0, c["Hq"] - 1})
+    Or, Lr = OA.attn_fwd(rec.seqlens, rec.edits, np64(q), np64(k), np64(v), scale, rows=rows, heads=heads)
+    assert_maxabs(np64(O[rows][:, heads]), Or, 2e-2, "O")
+    assert_maxabs(np64(LSE[heads][:, rows]), Lr, 2e-2, "LSE")
+
+
+@pytest.mark.parametrize("cfg", [2, 4])
+def test_full_size_forward_sampled(cfg):
+    """Full-size workloads in the bench's launch configuration; the oracle
+    recomputes sampled rows (every head's compact view) one by one."""
+    _full_size_fwd(synth.config_record(cfg), synth.CONFIGS[cfg], 100 + cfg)
+
+
+@pytest.mark.parametrize("K,f", [(1, 0.3), (32, 0.9)])
+def test_sweep_forward_sampled(K, f):
+    _full_size_fwd(synth.config_record(5, K=K, f=f), synth.CONFIGS[5], 200 + K)
