@@ -140,6 +140,28 @@ mw_status mw_build_visibility(const mw_vis_layout* layout, const int32_t* cu_seq
                               void* ws, void* vis, void* stream);
 
 /*
+ * Same result as mw_build_visibility, but allocation-free: for callers that
+ * are handed their input and output buffers and may not allocate device
+ * memory (e.g. a plugin inside a host framework that owns all device memory
+ * through its own pool, where cudaMalloc would synchronise the device or
+ * bypass the pool's accounting). The paper has no counterpart; this is a
+ * library convenience.
+ *   The build workspace is a fixed 1 MiB device array inside libmw, resident
+ *   on every GPU that loads the library until process exit. Records whose
+ *   layout->ws_bytes exceeds 1 MiB are rejected with MW_ENOSPACE (nothing is
+ *   launched). The first call on a device looks up the array's address with
+ *   that device current; make that first call before any stream capture.
+ *   All calls on a device share the array: calls whose GPU work overlaps
+ *   (other streams or threads) race and must be serialised by the caller.
+ *   The caller still provides `vis` (layout->vis_bytes, device). No device
+ *   memory is allocated or freed.
+ */
+mw_status mw_build_visibility_noalloc(const mw_vis_layout* layout, const int32_t* cu_seqlens,
+                                      int n_junc, const int32_t* junctions, const int32_t* junc_traj,
+                                      const int32_t* junc_span_off, const int32_t* spans,
+                                      void* vis, void* stream);
+
+/*
  * Eviction-aware masked GQA attention forward (§4.2 mask; §4.3 equivalence).
  *   Q, O  [total_tokens, Hq, Dh]   K, V [total_tokens, Hkv, Dh]   (dtype)
  *   LSE   [Hq, total_tokens] float32, natural-log row log-sum-exp (saved for bwd)

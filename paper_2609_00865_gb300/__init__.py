@@ -21,6 +21,7 @@ from ._lib import (  # noqa: F401
     masked_attn_bwd,
     masked_attn_fwd,
     mw_build_visibility,
+    mw_build_visibility_noalloc,
     mw_logprob_loss_bwd,
     mw_logprob_loss_fwd,
     mw_logprob_ws,

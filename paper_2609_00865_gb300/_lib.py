@@ -51,6 +51,7 @@ _SIGS = {
     "mw_kernel_launches": (ctypes.c_uint64, []),
     "mw_visibility_layout": (_I, [_I, _IP, _I, _IP, _I, _LP]),
     "mw_build_visibility": (_I, [_LP, _IP, _I, _IP, _IP, _IP, _IP, _P, _P, _P]),
+    "mw_build_visibility_noalloc": (_I, [_LP, _IP, _I, _IP, _IP, _IP, _IP, _P, _P]),
     "mw_masked_attn_fwd": (_I, [_LP, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _F, _P]),
     "mw_masked_attn_bwd_ws": (_I, [_LP, _I, _I, _I, ctypes.POINTER(ctypes.c_size_t)]),
     "mw_masked_attn_bwd": (_I, [_LP, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _F, _P, _P]),
@@ -159,6 +160,18 @@ def mw_build_visibility(layout, cu_seqlens, junctions, junc_traj, junc_span_off,
     sp, spp = _i32(np.asarray(spans).reshape(-1))
     _check(_lib().mw_build_visibility(ctypes.byref(layout), cup, len(J), Jp, jtp, offp, spp,
                                       _ptr(ws), _ptr(vis), _stream(stream)), "mw_build_visibility")
+
+
+def mw_build_visibility_noalloc(layout, cu_seqlens, junctions, junc_traj, junc_span_off, spans, vis, stream=None):
+    """Allocation-free build: the workspace is libmw's fixed device array
+    (for callers that may not allocate; see include/mw.h)."""
+    cu, cup = _i32(cu_seqlens)
+    J, Jp = _i32(junctions)
+    jt, jtp = _i32(junc_traj)
+    off, offp = _i32(junc_span_off)
+    sp, spp = _i32(np.asarray(spans).reshape(-1))
+    _check(_lib().mw_build_visibility_noalloc(ctypes.byref(layout), cup, len(J), Jp, jtp, offp, spp,
+                                              _ptr(vis), _stream(stream)), "mw_build_visibility_noalloc")
 
 
 class Visibility:
