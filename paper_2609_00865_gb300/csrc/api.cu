@@ -17,6 +17,8 @@ mw_status lm_bwd_simt(const void*, const void*, const int32_t*, const int32_t*, 
                       const float*, const float*, float, void*, float*, cudaStream_t);
 mw_status attn_fwd_tc(const mw_vis_layout*, const void*, const void*, const void*, const void*, void*, float*, int,
                       int, float, cudaStream_t);
+mw_status attn_bwd_tc(const mw_vis_layout*, const void*, const void*, const void*, const void*, const void*,
+                      const void*, const float*, void*, void*, void*, int, int, float, float*, cudaStream_t);
 __global__ void k_loss_epilogue(int, const float*, const float*, const float*, float, float, float*, float*, float*);
 
 // Byte offsets inside the log-prob workspace.
@@ -75,6 +77,8 @@ extern "C" mw_status mw_masked_attn_bwd(const mw_vis_layout* L, const void* vis,
     if (st != MW_OK) return st;
     if (L->total_tokens == 0) return MW_OK;
     if (!Q || !K || !V || !O || !dO || !LSE || !dQ || !dK || !dV || !ws) return MW_EINVAL;
+    if (dtype == MW_BF16 && Dh == 128)
+        return attn_bwd_tc(L, vis, Q, K, V, O, dO, LSE, dQ, dK, dV, Hq, Hkv, scale, (float*)ws, (cudaStream_t)stream);
     return attn_bwd_simt(L, vis, Q, K, V, O, dO, LSE, dQ, dK, dV, Hq, Hkv, Dh, dtype, scale, (float*)ws,
                          (cudaStream_t)stream);
 }

@@ -268,6 +268,28 @@ mw_status bwd_impl(const mw_vis_layout* L, const void* vis, const void* Q, const
 
 }  // namespace
 
+// Delta_i = rowsum(dO_i * O_i) for every (row, head); HBM-bound, shared by
+// both backward paths.
+mw_status attn_delta(const mw_vis_layout* L, const void* O, const void* dO, int Hq, int Dh, int dtype, float* delta,
+                     cudaStream_t s) {
+    const int64_t warps = L->total_tokens * Hq;
+    if (warps == 0) return MW_OK;
+    const unsigned grid = (unsigned)std::min<int64_t>(ceil_div(warps, 8), 152 * 64);
+    count_launches(1);
+    if (dtype == MW_F32) {
+        if (Dh == 64) k_attn_delta<float, 64><<<grid, 256, 0, s>>>(L->total_tokens, Hq, (const float*)O, (const float*)dO, delta);
+        else k_attn_delta<float, 128><<<grid, 256, 0, s>>>(L->total_tokens, Hq, (const float*)O, (const float*)dO, delta);
+    } else {
+        if (Dh == 64)
+            k_attn_delta<__nv_bfloat16, 64><<<grid, 256, 0, s>>>(L->total_tokens, Hq, (const __nv_bfloat16*)O,
+                                                                 (const __nv_bfloat16*)dO, delta);
+        else
+            k_attn_delta<__nv_bfloat16, 128><<<grid, 256, 0, s>>>(L->total_tokens, Hq, (const __nv_bfloat16*)O,
+                                                                  (const __nv_bfloat16*)dO, delta);
+    }
+    return launch_status();
+}
+
 mw_status attn_fwd_simt(const mw_vis_layout* L, const void* vis, const void* Q, const void* K, const void* V,
                         void* O, float* LSE, int Hq, int Hkv, int Dh, int dtype, float scale, cudaStream_t s) {
     if (dtype == MW_F32) {

@@ -318,6 +318,531 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     }
 }
 
+// ----------------------------------------------------------------------------
+// dQ kernel (Q-stationary, one CTA per (q-tile, q-head), same item order as the
+// forward). Per listed k-tile j:
+//   S_j = Q K_j^T (TMEM, double-buffered), dP_j = dO V_j^T (TMEM, single),
+//   P = exp2(S c - LSE2) on visible pairs, dS = P (dP - Delta) -> bf16 smem,
+//   dQ += dS K_j (TMEM accumulator; K_j read as an MN-major operand).
+// dQ = scale * accumulator, written as bf16. No atomics: each dQ row is owned
+// by one CTA.
+constexpr uint32_t DQ_Q = 0;
+constexpr uint32_t DQ_DO = DQ_Q + TILE_B;
+constexpr uint32_t DQ_K = DQ_DO + TILE_B;
+constexpr uint32_t DQ_V = DQ_K + 2 * TILE_B;
+constexpr uint32_t DQ_DS = DQ_V + 2 * TILE_B;
+constexpr uint32_t SMEM_DQ = DQ_DS + TILE_B + 1024;
+constexpr uint32_t TM_DP = 256, TM_DQ = 384;
+
+struct BwdParams {
+    VisView v;
+    int64_t total;
+    int n_traj, max_tiles, Hq, Hkv;
+    float scale, scale_log2;
+    const float* LSE;
+    const float* delta;
+    __nv_bfloat16* dQ;
+    __nv_bfloat16* dK;
+    __nv_bfloat16* dV;
+};
+
+__global__ void __launch_bounds__(NTHREADS, 1)
+    k_attn_dq_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmDO,
+                 const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, BwdParams p) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* sm = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~uintptr_t(1023));
+    __shared__ __align__(8) uint64_t q_full, k_full[2], k_empty[2], v_full[2], v_empty[2], s_full[2], s_free[2],
+        dp_full, dp_free, ds_full, dq_done;
+    __shared__ uint32_t tmem_base;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int h = blockIdx.x % p.Hq;
+    const int r = blockIdx.x / p.Hq;
+    const int qt = p.max_tiles - 1 - r / p.n_traj;
+    const int b = r % p.n_traj;
+    const VisView& v = p.v;
+    const int nt = v.traj_tile[b + 1] - v.traj_tile[b];
+    if (qt >= nt) return;
+    const int64_t g = v.traj_tile[b] + qt;
+    const int64_t tok0 = v.traj_tok[b];
+    const int T = v.traj_tok[b + 1] - (int)tok0;
+    const int kvh = h / (p.Hq / p.Hkv);
+    const int p0 = v.fwd_ptr[g];
+    const int n = v.fwd_ptr[g + 1] - p0;
+    int32_t* status = v.status;
+    if (*(volatile int32_t*)&status[1]) return;
+
+    if (threadIdx.x == 0) {
+        mbar_init(&q_full, 1);
+        for (int s = 0; s < 2; ++s) {
+            mbar_init(&k_full[s], 1);
+            mbar_init(&k_empty[s], 1);
+            mbar_init(&v_full[s], 1);
+            mbar_init(&v_empty[s], 1);
+            mbar_init(&s_full[s], 1);
+            mbar_init(&s_free[s], 128);
+        }
+        mbar_init(&dp_full, 1);
+        mbar_init(&dp_free, 128);
+        mbar_init(&ds_full, 128);
+        mbar_init(&dq_done, 1);
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(&tmem_base, 512);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_base;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            prefetch_tmap(&tmQ);
+            prefetch_tmap(&tmDO);
+            prefetch_tmap(&tmK);
+            prefetch_tmap(&tmV);
+            const int row0 = (int)(tok0 + qt * 128);
+            mbar_expect_tx(&q_full, 2 * TILE_B);
+            load_tile(sm + DQ_Q, &tmQ, &q_full, h, row0);
+            load_tile(sm + DQ_DO, &tmDO, &q_full, h, row0);
+            for (int j = 0; j < n; ++j) {
+                const int kt = v.fwd_idx[p0 + j] >> 2;
+                const int s = j & 1;
+                const int row = (int)(tok0 + kt * 128);
+                if (j >= 2 && !mbar_wait(&v_empty[s], ((j - 2) >> 1) & 1, status, 111)) break;
+                mbar_expect_tx(&v_full[s], TILE_B);
+                load_tile(sm + DQ_V + s * TILE_B, &tmV, &v_full[s], kvh, row);
+                if (j >= 2 && !mbar_wait(&k_empty[s], ((j - 2) >> 1) & 1, status, 112)) break;
+                mbar_expect_tx(&k_full[s], TILE_B);
+                load_tile(sm + DQ_K + s * TILE_B, &tmK, &k_full[s], kvh, row);
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            const uint32_t iKK = idesc_bf16(128, 128, 0, 0);  // both operands K-major
+            const uint32_t iMN = idesc_bf16(128, 128, 0, 1);  // B MN-major
+            const uint32_t sq = smem_u32(sm + DQ_Q), sdo = smem_u32(sm + DQ_DO), sk = smem_u32(sm + DQ_K),
+                           sv = smem_u32(sm + DQ_V), sds = smem_u32(sm + DQ_DS);
+            bool ok = mbar_wait(&q_full, 0, status, 211);
+            // S_j (needs K_j and a free S buffer)
+            auto issue_s = [&](int j) -> bool {
+                const int s = j & 1;
+                if (!mbar_wait(&k_full[s], (j >> 1) & 1, status, 212)) return false;
+                if (j >= 2 && !mbar_wait(&s_free[s], ((j - 2) >> 1) & 1, status, 213)) return false;
+                tc_fence_after();
+#pragma unroll
+                for (int ks = 0; ks < 8; ++ks)
+                    mma_ss(tmem + TM_S0 + s * 128, kmaj(sq, ks), kmaj(sk + s * TILE_B, ks), iKK, ks > 0);
+                mma_commit(&s_full[s]);
+                return true;
+            };
+            // dP_j (needs V_j and the softmax to have read dP_{j-1})
+            auto issue_dp = [&](int j) -> bool {
+                const int s = j & 1;
+                if (!mbar_wait(&v_full[s], (j >> 1) & 1, status, 214)) return false;
+                if (j >= 1 && !mbar_wait(&dp_free, (j - 1) & 1, status, 215)) return false;
+                tc_fence_after();
+#pragma unroll
+                for (int ks = 0; ks < 8; ++ks)
+                    mma_ss(tmem + TM_DP, kmaj(sdo, ks), kmaj(sv + s * TILE_B, ks), iKK, ks > 0);
+                mma_commit(&v_empty[s]);
+                mma_commit(&dp_full);
+                return true;
+            };
+            // dQ += dS_t K_t
+            auto issue_dq = [&](int t) -> bool {
+                if (!mbar_wait(&ds_full, t & 1, status, 216)) return false;
+                tc_fence_after();
+#pragma unroll
+                for (int ks = 0; ks < 8; ++ks)
+                    mma_ss(tmem + TM_DQ, kmaj(sds, ks), mnmaj(sk + (t & 1) * TILE_B, ks), iMN, (t > 0 || ks > 0));
+                mma_commit(&k_empty[t & 1]);
+                mma_commit(&dq_done);
+                return true;
+            };
+            if (ok && n > 0) ok = issue_s(0) && issue_dp(0);
+            for (int j = 0; ok && j < n; ++j) {
+                if (j + 1 < n && !issue_s(j + 1)) { ok = false; break; }
+                if (!issue_dq(j)) { ok = false; break; }
+                if (j + 1 < n && !issue_dp(j + 1)) { ok = false; break; }
+            }
+        }
+    } else {
+        const int qw = warp & 3;
+        const int rl = qw * 32 + lane;
+        const int i = qt * 128 + rl;
+        const int ie = min(i, T - 1);
+        const int seg = v.seg[tok0 + ie];
+        const uint4* km = reinterpret_cast<const uint4*>(v.keymask) + v.traj_km[b] + (int64_t)seg * nt;
+        const uint32_t lane_base = tmem + ((uint32_t)(qw * 32) << 16);
+        uint8_t* dsrow = sm + DQ_DS;
+        const float lse2 = p.LSE[(int64_t)h * p.total + tok0 + ie] * LOG2E;
+        const float dl = p.delta[(int64_t)h * p.total + tok0 + ie];
+        bool ok = true;
+        for (int j = 0; j < n; ++j) {
+            const int e = v.fwd_idx[p0 + j];
+            const int kt = e >> 2, cls = e & 3;
+            if (!mbar_wait(&s_full[j & 1], (j >> 1) & 1, status, 311)) { ok = false; break; }
+            tc_fence_after();
+            float s[128];
+            {
+                uint32_t rr[32];
+#pragma unroll
+                for (int c = 0; c < 4; ++c) {
+                    tmem_ld32(lane_base + TM_S0 + (j & 1) * 128 + c * 32, rr);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int x = 0; x < 32; ++x) s[c * 32 + x] = __uint_as_float(rr[x]);
+                }
+            }
+            tc_fence_before();
+            mbar_arrive(&s_free[j & 1]);
+            uint32_t wd[4] = {0xffffffffu, 0xffffffffu, 0xffffffffu, 0xffffffffu};
+            if (cls != MW_TILE_FULL || kt == qt) {
+                uint4 w = km[kt];
+                wd[0] = w.x; wd[1] = w.y; wd[2] = w.z; wd[3] = w.w;
+                if (kt == qt) {
+                    const int lim = ie - kt * 128;
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        const int hi = lim - 32 * q;
+                        wd[q] &= hi >= 31 ? 0xffffffffu : (hi < 0 ? 0u : ((2u << hi) - 1u));
+                    }
+                }
+            }
+#pragma unroll
+            for (int c = 0; c < 128; ++c)
+                s[c] = ((wd[c >> 5] >> (c & 31)) & 1u) ? ex2(fmaf(s[c], p.scale_log2, -lse2)) : 0.f;
+            if (!mbar_wait(&dp_full, j & 1, status, 312)) { ok = false; break; }
+            tc_fence_after();
+            // dS_j overwrites dS_{j-1}: wait until dQ += dS_{j-1} K_{j-1} is done
+            if (j >= 1 && !mbar_wait(&dq_done, (j - 1) & 1, status, 313)) { ok = false; break; }
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                uint32_t dp[32];
+                tmem_ld32(lane_base + TM_DP + c * 32, dp);
+                tmem_wait_ld();
+                if (c == 3) {
+                    tc_fence_before();
+                    mbar_arrive(&dp_free);
+                }
+#pragma unroll
+                for (int x = 0; x < 4; ++x) {
+                    uint4 pk;
+                    const int c0 = c * 32 + 8 * x;
+                    pk.x = pack_bf16(s[c0 + 0] * (__uint_as_float(dp[8 * x + 0]) - dl),
+                                     s[c0 + 1] * (__uint_as_float(dp[8 * x + 1]) - dl));
+                    pk.y = pack_bf16(s[c0 + 2] * (__uint_as_float(dp[8 * x + 2]) - dl),
+                                     s[c0 + 3] * (__uint_as_float(dp[8 * x + 3]) - dl));
+                    pk.z = pack_bf16(s[c0 + 4] * (__uint_as_float(dp[8 * x + 4]) - dl),
+                                     s[c0 + 5] * (__uint_as_float(dp[8 * x + 5]) - dl));
+                    pk.w = pack_bf16(s[c0 + 6] * (__uint_as_float(dp[8 * x + 6]) - dl),
+                                     s[c0 + 7] * (__uint_as_float(dp[8 * x + 7]) - dl));
+                    const int chunk = c * 4 + x;   // 16-byte chunk 0..15 of the row
+                    *reinterpret_cast<uint4*>(dsrow + (chunk >> 3) * HALF_B + sw128_off(rl, chunk & 7)) = pk;
+                }
+            }
+            fence_async_smem();
+            tc_fence_before();
+            mbar_arrive(&ds_full);
+        }
+        if (ok && n > 0 && mbar_wait(&dq_done, (n - 1) & 1, status, 314)) {
+            tc_fence_after();
+            __nv_bfloat16* qrow = p.dQ + ((tok0 + ie) * p.Hq + h) * DH;
+            uint32_t o[32];
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                tmem_ld32(lane_base + TM_DQ + c * 32, o);
+                tmem_wait_ld();
+                if (i < T) {
+#pragma unroll
+                    for (int x = 0; x < 4; ++x) {
+                        uint4 pk;
+                        pk.x = pack_bf16(__uint_as_float(o[8 * x + 0]) * p.scale, __uint_as_float(o[8 * x + 1]) * p.scale);
+                        pk.y = pack_bf16(__uint_as_float(o[8 * x + 2]) * p.scale, __uint_as_float(o[8 * x + 3]) * p.scale);
+                        pk.z = pack_bf16(__uint_as_float(o[8 * x + 4]) * p.scale, __uint_as_float(o[8 * x + 5]) * p.scale);
+                        pk.w = pack_bf16(__uint_as_float(o[8 * x + 6]) * p.scale, __uint_as_float(o[8 * x + 7]) * p.scale);
+                        *reinterpret_cast<uint4*>(qrow + c * 32 + 8 * x) = pk;
+                    }
+                }
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, 512);
+    }
+}
+
+// ----------------------------------------------------------------------------
+// dK / dV kernel (KV-stationary, one CTA per (k-tile, kv-head), smallest
+// k-tiles -- the longest lists -- first). Steps run over the k-tile's bwd list
+// x the group's query heads x two 64-row halves of each q-tile:
+//   S^T = K Q^T, dP^T = V dO^T   (M=128 keys, N=64 rows; TMEM, double-buffered)
+//   P^T = exp2(S^T c - LSE2_i), dS^T = P^T (dP^T - Delta_i) on visible pairs,
+//   written as bf16 [128 keys][64 rows] (double-buffered smem)
+//   dV += P^T dO, dK += dS^T Q   (dO, Q read as MN-major operands)
+// The rows that see key j form the interval [j, min(omega(j), T)), so the mask
+// is two compares per element.
+constexpr uint32_t HT_B = 64 * DH * 2;     // 64-row half tile: two [64][64] swizzled halves
+constexpr uint32_t HT_HALF = HT_B / 2;
+constexpr uint32_t PT_B = 128 * 64 * 2;    // [128 keys][64 rows] bf16
+constexpr uint32_t KV_K = 0;
+constexpr uint32_t KV_V = KV_K + TILE_B;
+constexpr uint32_t KV_Q = KV_V + TILE_B;           // 2 stages of (Q half, dO half)
+constexpr uint32_t KV_P = KV_Q + 2 * 2 * HT_B;     // 2 buffers of P^T
+constexpr uint32_t KV_DS = KV_P + 2 * PT_B;        // 2 buffers of dS^T
+constexpr uint32_t SMEM_KV = KV_DS + 2 * PT_B + 1024;
+constexpr uint32_t TM_ST = 0, TM_DPT = 128, TM_DV = 256, TM_DK = 384;
+
+// K-major descriptor, k-step ks, of a 64-row half tile ([64][128] as two [64][64]).
+__device__ __forceinline__ uint64_t kmaj_ht(uint32_t base, int ks) {
+    return sdesc_sw128(base + (ks >> 2) * HT_HALF + (ks & 3) * 32, 16, 1024);
+}
+// MN-major descriptor, k-step ks (16 rows), of a 64-row half tile.
+__device__ __forceinline__ uint64_t mnmaj_ht(uint32_t base, int ks) {
+    return sdesc_sw128(base + ks * 2048, HT_HALF, 1024);
+}
+
+__global__ void __launch_bounds__(NTHREADS, 1)
+    k_attn_dkdv_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmDO,
+                   const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, BwdParams p) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* sm = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~uintptr_t(1023));
+    __shared__ __align__(8) uint64_t kv_full, qd_full[2], qd_empty[2], sd_full[2], sd_free[2], pd_full[2],
+        pd_free[2], ls_full[2], ls_free[2];
+    __shared__ uint32_t tmem_base;
+    __shared__ float lsd[2][128];   // per step: LSE2 of the 64 rows, then Delta of the 64 rows
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int grp = p.Hq / p.Hkv;
+    const int kvh = blockIdx.x % p.Hkv;
+    const int r = blockIdx.x / p.Hkv;
+    const int kt = r / p.n_traj;
+    const int b = r % p.n_traj;
+    const VisView& v = p.v;
+    const int nt = v.traj_tile[b + 1] - v.traj_tile[b];
+    if (kt >= nt) return;
+    const int64_t gk = v.traj_tile[b] + kt;
+    const int64_t tok0 = v.traj_tok[b];
+    const int T = v.traj_tok[b + 1] - (int)tok0;
+    const int p0 = v.bwd_ptr[gk];
+    const int nlist = v.bwd_ptr[gk + 1] - p0;
+    const int nsteps = nlist * grp * 2;
+    int32_t* status = v.status;
+    if (*(volatile int32_t*)&status[1]) return;
+
+    if (threadIdx.x == 0) {
+        mbar_init(&kv_full, 1);
+        for (int s = 0; s < 2; ++s) {
+            mbar_init(&qd_full[s], 1);
+            mbar_init(&qd_empty[s], 1);
+            mbar_init(&sd_full[s], 1);
+            mbar_init(&sd_free[s], 128);
+            mbar_init(&pd_full[s], 128);
+            mbar_init(&pd_free[s], 1);
+            mbar_init(&ls_full[s], 128);
+            mbar_init(&ls_free[s], 128);
+        }
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(&tmem_base, 512);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_base;
+    // step t -> (list entry, head in group, half)
+    auto step_q0 = [&](int t, int& hq) -> int {
+        const int e = t / (grp * 2);
+        const int rem = t % (grp * 2);
+        hq = kvh * grp + rem / 2;
+        return (v.bwd_idx[p0 + e] >> 2) * 128 + (rem & 1) * 64;
+    };
+
+    if (warp == 0) {
+        if (lane == 0) {
+            prefetch_tmap(&tmQ);
+            prefetch_tmap(&tmDO);
+            prefetch_tmap(&tmK);
+            prefetch_tmap(&tmV);
+            mbar_expect_tx(&kv_full, 2 * TILE_B);
+            load_tile(sm + KV_K, &tmK, &kv_full, kvh, (int)(tok0 + kt * 128));
+            load_tile(sm + KV_V, &tmV, &kv_full, kvh, (int)(tok0 + kt * 128));
+            for (int t = 0; t < nsteps; ++t) {
+                const int s = t & 1;
+                int hq;
+                const int q0 = step_q0(t, hq);
+                if (t >= 2 && !mbar_wait(&qd_empty[s], ((t - 2) >> 1) & 1, status, 121)) break;
+                mbar_expect_tx(&qd_full[s], 2 * HT_B);
+                uint8_t* dst = sm + KV_Q + s * 2 * HT_B;
+                tma_load_3d(dst, &tmQ, &qd_full[s], 0, hq, (int)(tok0 + q0));
+                tma_load_3d(dst + HT_HALF, &tmQ, &qd_full[s], 64, hq, (int)(tok0 + q0));
+                tma_load_3d(dst + HT_B, &tmDO, &qd_full[s], 0, hq, (int)(tok0 + q0));
+                tma_load_3d(dst + HT_B + HT_HALF, &tmDO, &qd_full[s], 64, hq, (int)(tok0 + q0));
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            const uint32_t iSD = idesc_bf16(128, 64, 0, 0);
+            const uint32_t iAC = idesc_bf16(128, 128, 0, 1);
+            const uint32_t sk = smem_u32(sm + KV_K), sv = smem_u32(sm + KV_V), sq = smem_u32(sm + KV_Q),
+                           spb = smem_u32(sm + KV_P), sdb = smem_u32(sm + KV_DS);
+            bool ok = mbar_wait(&kv_full, 0, status, 221);
+            auto issue_sd = [&](int t) -> bool {
+                const int s = t & 1;
+                if (!mbar_wait(&qd_full[s], (t >> 1) & 1, status, 222)) return false;
+                if (t >= 2 && !mbar_wait(&sd_free[s], ((t - 2) >> 1) & 1, status, 223)) return false;
+                tc_fence_after();
+                const uint32_t qb = sq + s * 2 * HT_B, db = qb + HT_B;
+#pragma unroll
+                for (int ks = 0; ks < 8; ++ks) mma_ss(tmem + TM_ST + s * 64, kmaj(sk, ks), kmaj_ht(qb, ks), iSD, ks > 0);
+#pragma unroll
+                for (int ks = 0; ks < 8; ++ks) mma_ss(tmem + TM_DPT + s * 64, kmaj(sv, ks), kmaj_ht(db, ks), iSD, ks > 0);
+                mma_commit(&sd_full[s]);
+                return true;
+            };
+            auto issue_acc = [&](int t) -> bool {
+                const int s = t & 1;
+                if (!mbar_wait(&pd_full[s], (t >> 1) & 1, status, 224)) return false;
+                tc_fence_after();
+                const uint32_t qb = sq + s * 2 * HT_B, db = qb + HT_B;
+                const uint32_t pb = spb + s * PT_B, dsb = sdb + s * PT_B;
+#pragma unroll
+                for (int ks = 0; ks < 4; ++ks)
+                    mma_ss(tmem + TM_DV, sdesc_sw128(pb + ks * 32, 16, 1024), mnmaj_ht(db, ks), iAC, (t > 0 || ks > 0));
+#pragma unroll
+                for (int ks = 0; ks < 4; ++ks)
+                    mma_ss(tmem + TM_DK, sdesc_sw128(dsb + ks * 32, 16, 1024), mnmaj_ht(qb, ks), iAC, (t > 0 || ks > 0));
+                mma_commit(&qd_empty[s]);
+                mma_commit(&pd_free[s]);
+                return true;
+            };
+            if (ok && nsteps > 0) ok = issue_sd(0);
+            for (int t = 0; ok && t < nsteps; ++t) {
+                if (t + 1 < nsteps && !issue_sd(t + 1)) { ok = false; break; }
+                if (!issue_acc(t)) { ok = false; break; }
+            }
+        }
+    } else {
+        const int qw = warp & 3;
+        const int rl = qw * 32 + lane;               // key row inside the k-tile = TMEM lane
+        const int jk = kt * 128 + rl;
+        const int je = min(jk, T - 1);
+        const int iend = jk < T ? min(v.omega[tok0 + je], T) : 0;   // rows [jk, iend) see this key
+        const uint32_t lane_base = tmem + ((uint32_t)(qw * 32) << 16);
+        const int tid = threadIdx.x - 64;            // 0..127 among the softmax threads
+        bool ok = true;
+        for (int t = 0; t < nsteps; ++t) {
+            const int s = t & 1;
+            int hq;
+            const int q0 = step_q0(t, hq);
+            {   // this step's LSE2 (threads 0..63) and Delta (64..127) of rows q0 .. q0+63
+                if (t >= 2 && !mbar_wait(&ls_free[s], ((t - 2) >> 1) & 1, status, 324)) { ok = false; break; }
+                const int row = min(q0 + (tid & 63), T - 1);
+                const int64_t at = (int64_t)hq * p.total + tok0 + row;
+                lsd[s][tid] = tid < 64 ? p.LSE[at] * LOG2E : p.delta[at];
+                mbar_arrive(&ls_full[s]);
+                if (!mbar_wait(&ls_full[s], (t >> 1) & 1, status, 325)) { ok = false; break; }
+            }
+            if (!mbar_wait(&sd_full[s], (t >> 1) & 1, status, 321)) { ok = false; break; }
+            tc_fence_after();
+            float sv[64], dp[64];
+            {
+                uint32_t rr[32];
+#pragma unroll
+                for (int c = 0; c < 2; ++c) {
+                    tmem_ld32(lane_base + TM_ST + s * 64 + c * 32, rr);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int x = 0; x < 32; ++x) sv[c * 32 + x] = __uint_as_float(rr[x]);
+                    tmem_ld32(lane_base + TM_DPT + s * 64 + c * 32, rr);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int x = 0; x < 32; ++x) dp[c * 32 + x] = __uint_as_float(rr[x]);
+                }
+            }
+            tc_fence_before();
+            mbar_arrive(&sd_free[s]);
+            const int lo = max(jk, q0) - q0, hi = min(iend, q0 + 64) - q0;   // visible columns [lo, hi)
+#pragma unroll
+            for (int c = 0; c < 64; ++c) {
+                const bool vis = c >= lo && c < hi;
+                const float pr = vis ? ex2(fmaf(sv[c], p.scale_log2, -lsd[s][c])) : 0.f;
+                sv[c] = pr;
+                dp[c] = pr * (dp[c] - lsd[s][64 + c]);
+            }
+            mbar_arrive(&ls_free[s]);
+            if (t >= 2 && !mbar_wait(&pd_free[s], ((t - 2) >> 1) & 1, status, 322)) { ok = false; break; }
+            uint8_t* pbuf = sm + KV_P + s * PT_B;
+            uint8_t* dbuf = sm + KV_DS + s * PT_B;
+#pragma unroll
+            for (int c = 0; c < 8; ++c) {
+                uint4 a, d;
+                a.x = pack_bf16(sv[8 * c + 0], sv[8 * c + 1]);
+                a.y = pack_bf16(sv[8 * c + 2], sv[8 * c + 3]);
+                a.z = pack_bf16(sv[8 * c + 4], sv[8 * c + 5]);
+                a.w = pack_bf16(sv[8 * c + 6], sv[8 * c + 7]);
+                d.x = pack_bf16(dp[8 * c + 0], dp[8 * c + 1]);
+                d.y = pack_bf16(dp[8 * c + 2], dp[8 * c + 3]);
+                d.z = pack_bf16(dp[8 * c + 4], dp[8 * c + 5]);
+                d.w = pack_bf16(dp[8 * c + 6], dp[8 * c + 7]);
+                *reinterpret_cast<uint4*>(pbuf + sw128_off(rl, c)) = a;
+                *reinterpret_cast<uint4*>(dbuf + sw128_off(rl, c)) = d;
+            }
+            fence_async_smem();
+            tc_fence_before();
+            mbar_arrive(&pd_full[s]);
+        }
+        if (ok && nsteps > 0 && mbar_wait(&pd_free[(nsteps - 1) & 1], ((nsteps - 1) >> 1) & 1, status, 323)) {
+            tc_fence_after();
+            const int64_t row = ((tok0 + je) * p.Hkv + kvh) * DH;
+            uint32_t o[32];
+#pragma unroll
+            for (int pass = 0; pass < 2; ++pass) {
+                __nv_bfloat16* dst = (pass == 0 ? p.dV : p.dK) + row;
+                const float mul = pass == 0 ? 1.f : p.scale;
+                const uint32_t col = pass == 0 ? TM_DV : TM_DK;
+#pragma unroll
+                for (int c = 0; c < 4; ++c) {
+                    tmem_ld32(lane_base + col + c * 32, o);
+                    tmem_wait_ld();
+                    if (jk < T) {
+#pragma unroll
+                        for (int x = 0; x < 4; ++x) {
+                            uint4 pk;
+                            pk.x = pack_bf16(__uint_as_float(o[8 * x + 0]) * mul, __uint_as_float(o[8 * x + 1]) * mul);
+                            pk.y = pack_bf16(__uint_as_float(o[8 * x + 2]) * mul, __uint_as_float(o[8 * x + 3]) * mul);
+                            pk.z = pack_bf16(__uint_as_float(o[8 * x + 4]) * mul, __uint_as_float(o[8 * x + 5]) * mul);
+                            pk.w = pack_bf16(__uint_as_float(o[8 * x + 6]) * mul, __uint_as_float(o[8 * x + 7]) * mul);
+                            *reinterpret_cast<uint4*>(dst + c * 32 + 8 * x) = pk;
+                        }
+                    }
+                }
+            }
+        } else if (jk < T) {
+            // no listed q-tile (cannot happen: the diagonal tile is always listed)
+            const int64_t row = ((tok0 + je) * p.Hkv + kvh) * DH;
+            for (int c = 0; c < DH; ++c) {
+                p.dK[row + c] = __float2bfloat16(0.f);
+                p.dV[row + c] = __float2bfloat16(0.f);
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, 512);
+    }
+}
+
 }  // namespace
 
 mw_status attn_fwd_tc(const mw_vis_layout* L, const void* vis, const void* Q, const void* K, const void* V,
@@ -344,6 +869,47 @@ mw_status attn_fwd_tc(const mw_vis_layout* L, const void* vis, const void* Q, co
     const unsigned grid = (unsigned)((int64_t)L->max_tiles * L->n_traj * Hq);
     count_launches(1);
     k_attn_fwd_tc<<<grid, NTHREADS, SMEM_FWD, s>>>(tq, tk, tv, p);
+    return launch_status();
+}
+
+mw_status attn_delta(const mw_vis_layout*, const void*, const void*, int, int, int, float*, cudaStream_t);
+
+mw_status attn_bwd_tc(const mw_vis_layout* L, const void* vis, const void* Q, const void* K, const void* V,
+                      const void* O, const void* dO, const float* LSE, void* dQ, void* dK, void* dV, int Hq, int Hkv,
+                      float scale, float* delta, cudaStream_t s) {
+    if (L->n_tiles == 0) return MW_OK;
+    mw_status st = attn_delta(L, O, dO, Hq, DH, MW_BF16, delta, s);
+    if (st != MW_OK) return st;
+    const uint64_t T = (uint64_t)L->total_tokens;
+    CUtensorMap tq, tdo, tk, tv, tq64, tdo64;
+    if (!tmap_bf16_3d(&tq, Q, T, Hq, DH, 128, 64) || !tmap_bf16_3d(&tdo, dO, T, Hq, DH, 128, 64) ||
+        !tmap_bf16_3d(&tk, K, T, Hkv, DH, 128, 64) || !tmap_bf16_3d(&tv, V, T, Hkv, DH, 128, 64) ||
+        !tmap_bf16_3d(&tq64, Q, T, Hq, DH, 64, 64) || !tmap_bf16_3d(&tdo64, dO, T, Hq, DH, 64, 64))
+        return MW_ECUDA;
+    BwdParams p;
+    p.v = make_view(L, vis);
+    p.total = L->total_tokens;
+    p.n_traj = L->n_traj;
+    p.max_tiles = L->max_tiles;
+    p.Hq = Hq;
+    p.Hkv = Hkv;
+    p.scale = scale;
+    p.scale_log2 = scale * LOG2E;
+    p.LSE = LSE;
+    p.delta = delta;
+    p.dQ = (__nv_bfloat16*)dQ;
+    p.dK = (__nv_bfloat16*)dK;
+    p.dV = (__nv_bfloat16*)dV;
+    if ((st = cuda_status(cudaFuncSetAttribute(k_attn_dq_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               (int)SMEM_DQ))) != MW_OK)
+        return st;
+    if ((st = cuda_status(cudaFuncSetAttribute(k_attn_dkdv_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               (int)SMEM_KV))) != MW_OK)
+        return st;
+    count_launches(2);
+    k_attn_dq_tc<<<(unsigned)((int64_t)L->max_tiles * L->n_traj * Hq), NTHREADS, SMEM_DQ, s>>>(tq, tdo, tk, tv, p);
+    k_attn_dkdv_tc<<<(unsigned)((int64_t)L->max_tiles * L->n_traj * Hkv), NTHREADS, SMEM_KV, s>>>(tq64, tdo64, tk,
+                                                                                                   tv, p);
     return launch_status();
 }
 

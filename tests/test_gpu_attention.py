@@ -145,3 +145,50 @@ def test_full_size_forward_sampled(cfg):
 @pytest.mark.parametrize("K,f", [(1, 0.3), (32, 0.9)])
 def test_sweep_forward_sampled(K, f):
     _full_size_fwd(synth.config_record(5, K=K, f=f), synth.CONFIGS[5], 200 + K)
+
+
+def _full_size_bwd(rec, c, seed, keys_mode):
+    import paper_2609_00865_gb300 as mw
+    T = rec.total
+    g = torch.Generator(device="cuda").manual_seed(seed)
+    q = torch.randn(T, c["Hq"], c["Dh"], device="cuda", generator=g).to(torch.bfloat16)
+    k = torch.randn(T, c["Hkv"], c["Dh"], device="cuda", generator=g).to(torch.bfloat16)
+    v = torch.randn(T, c["Hkv"], c["Dh"], device="cuda", generator=g).to(torch.bfloat16)
+    do = torch.randn(T, c["Hq"], c["Dh"], device="cuda", generator=g).to(torch.bfloat16)
+    vis = mw.build_visibility(rec.seqlens, rec.edits)
+    scale = c["Dh"] ** -0.5
+    O, LSE = mw.masked_attn_fwd(vis, q, k, v, scale)
+    dQ, dK, dV = mw.masked_attn_bwd(vis, q, k, v, O, do, LSE, scale)
+    torch.cuda.synchronize()
+    vis.check_status()
+    rng = np.random.default_rng(seed)
+    Q64, K64, V64, dO64 = np64(q), np64(k), np64(v), np64(do)
+    rows = _sample_rows(rec, rng, n_random=12)
+    heads = sorted(set(rng.integers(0, c["Hq"], 2).tolist()) | {c["Hq"] - 1})
+    dQr = OA.attn_bwd_rows(rec.seqlens, rec.edits, Q64, K64, V64, dO64, scale, rows, heads)
+    assert_grad_bf16(np64(dQ[rows][:, heads]), dQr, "dQ (sampled rows)")
+    grp = int(rng.integers(0, c["Hkv"]))
+    t0 = rec.trajs[0]
+    if keys_mode == "all":        # keys across every segment of trajectory 0
+        keys = np.unique(np.concatenate([[0, 1, 127, 128, t0.T - 1],
+                                         [a for J, sp in t0.edits for a, _ in sp[:2]],
+                                         rng.integers(0, t0.T, 10)]))
+    else:                          # keys of the last segment only (cheap oracle)
+        J_last = t0.edits[-1][0] if t0.edits else 0
+        keys = np.unique(np.concatenate([[J_last, t0.T - 1], rng.integers(J_last, t0.T, 10)]))
+    dkr, dvr = OA.attn_bwd_keys(rec.seqlens[:1], rec.edits[:1], Q64[: t0.T], K64[: t0.T], V64[: t0.T],
+                                dO64[: t0.T], scale, grp, keys)
+    assert_grad_bf16(np64(dK[keys, grp]), dkr, "dK (sampled keys)")
+    assert_grad_bf16(np64(dV[keys, grp]), dvr, "dV (sampled keys)")
+
+
+def test_full_size_backward_config2():
+    _full_size_bwd(synth.config_record(2), synth.CONFIGS[2], 302, "all")
+
+
+def test_full_size_backward_config4():
+    _full_size_bwd(synth.config_record(4), synth.CONFIGS[4], 304, "last")
+
+
+def test_sweep_backward_sampled():
+    _full_size_bwd(synth.config_record(5, K=8, f=0.6), synth.CONFIGS[5], 305, "last")
