@@ -91,8 +91,11 @@ class Clocks:
 
 # ----------------------------------------------------------------------------- workloads
 
-def make_workload(cfg, K=None, f=None, seed_offset=0):
-    """Host-side inputs of one workload (pinned CPU tensors + record)."""
+def make_workload(cfg, K=None, f=None, seed_offset=0, n_traj=None):
+    """Host-side inputs of one workload (pinned CPU tensors + record).
+
+    ``n_traj`` keeps only the first trajectories of the record (a smaller
+    case of the same kernels, for profiler captures)."""
     import numpy as np
     import torch
 
@@ -110,6 +113,8 @@ def make_workload(cfg, K=None, f=None, seed_offset=0):
 
     if cfg in (2, 4, 5):
         rec = synth.config_record(cfg, K=K, f=f)
+        if n_traj:
+            rec = synth.Record(rec.trajs[:n_traj])
         w["record"] = rec
         T = rec.total
         w["Q"] = randn(T, c["Hq"], c["Dh"])
@@ -337,7 +342,7 @@ def cpu_sample(w, budget_s=15.0):
 def run_reference(args, rank, world):
     if rank != 0:
         return
-    w = make_workload(args.config, args.K, args.f)
+    w = make_workload(args.config, args.K, args.f, n_traj=args.n_traj)
     vals = []
     for i in range(args.warmup + args.steps):
         v, cores, desc = cpu_sample(w, budget_s=args.cpu_seconds / max(1, args.steps))
@@ -362,7 +367,7 @@ def run_gpu(args, rank, world, local_rank):
     import paper_2609_00865_gb300 as mw
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
-    w = make_workload(args.config, args.K, args.f, seed_offset=rank)
+    w = make_workload(args.config, args.K, args.f, seed_offset=rank, n_traj=args.n_traj)
     step = Step(w, dev)
     step.prime()
     for _ in range(args.warmup):
@@ -464,6 +469,8 @@ def main():
     ap.add_argument("--config", type=int, default=4, choices=[2, 3, 4, 5])
     ap.add_argument("--K", type=int, default=8)
     ap.add_argument("--f", type=float, default=0.6)
+    ap.add_argument("--n-traj", type=int, default=None,
+                    help="keep only the first trajectories (smaller case for profiler captures)")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu", action="store_true")
     args = ap.parse_args()

@@ -581,7 +581,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
 // ----------------------------------------------------------------------------
 // dK / dV kernel (KV-stationary, one CTA per (k-tile, kv-head), smallest
 // k-tiles -- the longest lists -- first). Steps run over the k-tile's bwd list
-// x the group's query heads x two 64-row halves of each q-tile:
+// (last q-tile first) x the group's query heads x two 64-row halves:
 //   S^T = K Q^T, dP^T = V dO^T   (M=128 keys, N=64 rows; TMEM, double-buffered)
 //   P^T = exp2(S^T c - LSE2_i), dS^T = P^T (dP^T - Delta_i) on visible pairs,
 //   written as bf16 [128 keys][64 rows] (double-buffered smem)
@@ -658,9 +658,11 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = tmem_base;
-    // step t -> (list entry, head in group, half)
+    // step t -> (list entry, head in group, half). The list is walked from its
+    // last q-tile down, so CTAs of one KV head that started together stream the
+    // same Q / dO tiles at the same time (L2 reuse across k-tiles).
     auto step_q0 = [&](int t, int& hq) -> int {
-        const int e = t / (grp * 2);
+        const int e = nlist - 1 - t / (grp * 2);
         const int rem = t % (grp * 2);
         hq = kvh * grp + rem / 2;
         return (v.bwd_idx[p0 + e] >> 2) * 128 + (rem & 1) * 64;
