@@ -21,16 +21,39 @@ mw_status attn_bwd_tc(const mw_vis_layout*, const void*, const void*, const void
                       const void*, const float*, void*, void*, void*, int, int, float, float*, cudaStream_t);
 __global__ void k_loss_epilogue(int, const float*, const float*, const float*, float, float, float*, float*, float*);
 
+struct LmPlan {
+    int M_pad, R, NV, C, NVC, grid;
+};
+LmPlan lm_plan(int M, int V);
+mw_status lm_fwd_tc(const void*, const void*, const int32_t*, const int32_t*, int, int, int, void*, int32_t*,
+                    float2*, float*, float*, float*, int32_t*, cudaStream_t);
+
+bool lm_bwd_tc_supported(int d);
+mw_status lm_bwd_tc(const void*, int, int, int, int, const int32_t*, const void*, const int32_t*, const float*,
+                    const float*, float, void*, float*, int32_t*, cudaStream_t);
+
+// Tensor-core LM-head path: bf16 with d a multiple of 64 that the clustered
+// backward can split (d / C <= 448 for a cluster of C <= 8 CTAs).
+static bool lm_tc(int d, int dtype) { return dtype == MW_BF16 && d % 64 == 0 && lm_bwd_tc_supported(d); }
+
 // Byte offsets inside the log-prob workspace.
 struct LmWs {
-    int64_t g, zt, bytes;
+    int64_t g, zt, hg, tg, part, status, bytes;
 };
 static LmWs lm_ws_layout(int N, int M, int d, int V, int dtype) {
-    (void)N; (void)d; (void)V; (void)dtype;
+    (void)N; (void)V;
     LmWs w;
     int64_t o = 0;
+    const int64_t M_pad = ceil_div(M, 128) * 128;
     w.g = o; o = align256(o + 4 * (int64_t)M);
     w.zt = o; o = align256(o + 4 * (int64_t)M);
+    w.status = o; o = align256(o + 32);
+    w.hg = w.tg = w.part = o;
+    if (lm_tc(d, dtype)) {
+        w.hg = o; o = align256(o + 2 * M_pad * d);
+        w.tg = o; o = align256(o + 4 * M_pad);
+        w.part = o; o = align256(o + 8 * 64 * M_pad);
+    }
     w.bytes = o;
     return w;
 }
@@ -87,7 +110,7 @@ static mw_status lm_args(int N, int M, int d, int V, int dtype) {
     if (N < 0 || M < 0 || d <= 0 || V <= 0) return MW_ESHAPE;
     if (M > N) return MW_ESHAPE;
     if (dtype != MW_F32 && dtype != MW_BF16) return MW_EDTYPE;
-    if (d > 256) return MW_ESHAPE;
+    if (!lm_tc(d, dtype) && d > 256) return MW_ESHAPE;
     return MW_OK;
 }
 
@@ -112,7 +135,14 @@ extern "C" mw_status mw_logprob_loss_fwd(const void* H, const void* W, const int
     LmWs w = lm_ws_layout(N, M, d, V, dtype);
     float* g = at<float>(ws, w.g);
     float* zt = at<float>(ws, w.zt);
-    if ((st = lm_fwd_simt(H, W, targets, rows, M, d, V, dtype, lse, zt, lp, s)) != MW_OK) return st;
+    if (lm_tc(d, dtype)) {
+        if ((st = cuda_status(cudaMemsetAsync(at<char>(ws, w.status), 0, 32, s))) != MW_OK) return st;
+        st = lm_fwd_tc(H, W, targets, rows, M, d, V, at<char>(ws, w.hg), at<int32_t>(ws, w.tg),
+                       at<float2>(ws, w.part), zt, lse, lp, at<int32_t>(ws, w.status), s);
+    } else {
+        st = lm_fwd_simt(H, W, targets, rows, M, d, V, dtype, lse, zt, lp, s);
+    }
+    if (st != MW_OK) return st;
     count_launches(1);
     k_loss_epilogue<<<1, 1024, 0, s>>>(M, lp, lp_old, adv, eps_lo, eps_hi, ratio, g, loss);
     return launch_status();
@@ -127,6 +157,15 @@ extern "C" mw_status mw_logprob_loss_bwd(const void* H, const void* W, const int
     if (!ws || !dW || (N > 0 && !dH)) return MW_EINVAL;
     if (M > 0 && (!H || !W || !targets || !rows || !lse)) return MW_EINVAL;
     LmWs w = lm_ws_layout(N, M, d, V, dtype);
+    if (lm_tc(d, dtype)) {
+        // the backward reads the forward's gathered rows and g, and writes
+        // only the status words of the workspace
+        void* wsm = const_cast<void*>(ws);
+        if ((st = cuda_status(cudaMemsetAsync(at<char>(wsm, w.status), 0, 32, (cudaStream_t)stream))) != MW_OK)
+            return st;
+        return lm_bwd_tc(W, M, N, d, V, rows, at<char>(wsm, w.hg), at<int32_t>(wsm, w.tg), lse,
+                         at<float>(wsm, w.g), dloss, dH, dW, at<int32_t>(wsm, w.status), (cudaStream_t)stream);
+    }
     return lm_bwd_simt(H, W, targets, rows, M, N, d, V, dtype, lse, at<float>(ws, w.g), dloss, dH, dW,
                        (cudaStream_t)stream);
 }

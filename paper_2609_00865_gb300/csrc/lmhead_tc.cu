@@ -1,0 +1,282 @@
+// Tensor-core fused LM-head log-prob (bf16 in, fp32 accumulate): no logits
+// tensor is stored.
+//
+//   gather   Hg[m] = H[rows[m]] (bf16, zero-padded to a multiple of 128 rows),
+//            tg[m] = targets[rows[m]]
+//   forward  persistent CTAs over (vocab chunk, 128-row tile) items; per item
+//            the chunk's 256-wide vocab tiles are computed as
+//            Z = Hg_tile W_tile^T with tcgen05.mma into one of two TMEM
+//            accumulators (128 x 256 fp32 each) fed by a 4-stage TMA ring, while
+//            four epilogue warps fold the previous tile into a running
+//            (max, sum 2^(z log2 e - max)) per row and pick out the target
+//            logit. Each item writes one (max, sum) partial per row.
+//   combine  lse = ln 2 (M + log2 sum_c l_c 2^(m_c - M)), lp = z_target - lse.
+// Concurrent CTAs work on the same vocab chunk, so each W tile is read from
+// HBM about once per wave and shared through L2.
+
+#include <math.h>
+
+#include "common.cuh"
+#include "tc.cuh"
+#include "tmap.cuh"
+
+namespace mw {
+
+namespace {
+
+using namespace tc;
+
+constexpr int NT = 192;
+constexpr int BM = 128, BN = 256, BK = 64;
+constexpr uint32_t A_B = BM * BK * 2;   // 16 KB
+constexpr uint32_t B_B = BN * BK * 2;   // 32 KB
+constexpr uint32_t ST_B = A_B + B_B;
+constexpr int NSTAGE = 4;
+constexpr uint32_t SMEM_LMF = NSTAGE * ST_B + 1024;
+constexpr float LOG2E_F = 1.4426950408889634f;
+
+struct LmFwdParams {
+    int M, M_pad, d, V;
+    int R, NV, C, NVC;        // row tiles, vocab tiles, chunks, vocab tiles per chunk
+    const int32_t* tg;        // [M_pad]
+    float2* part;             // [C][M_pad] (max2, sum)
+    float* zt;                // [M]
+    int32_t* status;
+};
+
+__global__ void __launch_bounds__(NT, 1)
+    k_lm_fwd_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, LmFwdParams p) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* sm = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~uintptr_t(1023));
+    __shared__ __align__(8) uint64_t full[NSTAGE], empty[NSTAGE], acc_full[2], acc_empty[2];
+    __shared__ uint32_t tmem_base;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int n_items = p.R * p.C;
+    const int KC = p.d / BK;
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < NSTAGE; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        for (int s = 0; s < 2; ++s) {
+            mbar_init(&acc_full[s], 1);
+            mbar_init(&acc_empty[s], 128);
+        }
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(&tmem_base, 512);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_base;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            prefetch_tmap(&tmA);
+            prefetch_tmap(&tmB);
+            uint32_t it = 0;
+            bool ok = true;
+            for (int w = blockIdx.x; ok && w < n_items; w += gridDim.x) {
+                const int c = w / p.R, r = w % p.R;
+                const int v0 = c * p.NVC, v1 = min(v0 + p.NVC, p.NV);
+                for (int vt = v0; ok && vt < v1; ++vt)
+                    for (int kc = 0; kc < KC; ++kc, ++it) {
+                        const int s = it % NSTAGE;
+                        if (it >= NSTAGE && !mbar_wait(&empty[s], ((it / NSTAGE) - 1) & 1, p.status, 401)) {
+                            ok = false;
+                            break;
+                        }
+                        mbar_expect_tx(&full[s], ST_B);
+                        tma_load_2d(sm + s * ST_B, &tmA, &full[s], kc * BK, r * BM);
+                        tma_load_2d(sm + s * ST_B + A_B, &tmB, &full[s], kc * BK, vt * BN);
+                    }
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            const uint32_t idesc = idesc_bf16(BM, BN, 0, 0);
+            const uint32_t base = smem_u32(sm);
+            uint32_t it = 0, tile = 0;
+            bool ok = true;
+            for (int w = blockIdx.x; ok && w < n_items; w += gridDim.x) {
+                const int c = w / p.R;
+                const int v0 = c * p.NVC, v1 = min(v0 + p.NVC, p.NV);
+                for (int vt = v0; ok && vt < v1; ++vt, ++tile) {
+                    const int ab = tile & 1;
+                    if (tile >= 2 && !mbar_wait(&acc_empty[ab], ((tile >> 1) - 1) & 1, p.status, 402)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    for (int kc = 0; kc < KC; ++kc, ++it) {
+                        const int s = it % NSTAGE;
+                        if (!mbar_wait(&full[s], (it / NSTAGE) & 1, p.status, 403)) { ok = false; break; }
+                        tc_fence_after();
+                        const uint32_t a = base + s * ST_B, b = a + A_B;
+#pragma unroll
+                        for (int ks = 0; ks < 4; ++ks)
+                            mma_ss(tmem + ab * BN, sdesc_sw128(a + ks * 32, 16, 1024), sdesc_sw128(b + ks * 32, 16, 1024),
+                                   idesc, (kc | ks) != 0);
+                        mma_commit(&empty[s]);
+                    }
+                    if (ok) mma_commit(&acc_full[ab]);
+                }
+            }
+        }
+    } else {
+        const int qw = warp & 3;
+        const int rl = qw * 32 + lane;
+        const uint32_t lane_base = tmem + ((uint32_t)(qw * 32) << 16);
+        uint32_t tile = 0;
+        bool ok = true;
+        for (int w = blockIdx.x; ok && w < n_items; w += gridDim.x) {
+            const int c = w / p.R, r = w % p.R;
+            const int v0 = c * p.NVC, v1 = min(v0 + p.NVC, p.NV);
+            const int m = r * BM + rl;
+            const int tgt = p.tg[m];
+            float mx = -INFINITY, l = 0.f;
+            for (int vt = v0; vt < v1; ++vt, ++tile) {
+                const int ab = tile & 1;
+                if (!mbar_wait(&acc_full[ab], (tile >> 1) & 1, p.status, 404)) { ok = false; break; }
+                tc_fence_after();
+#pragma unroll 1
+                for (int cc = 0; cc < BN / 32; ++cc) {
+                    uint32_t z[32];
+                    tmem_ld32(lane_base + ab * BN + cc * 32, z);
+                    tmem_wait_ld();
+                    const int vb = vt * BN + cc * 32;
+                    const int nvalid = min(32, p.V - vb);
+                    if (tgt >= vb && tgt < vb + 32 && m < p.M) {
+#pragma unroll
+                        for (int x = 0; x < 32; ++x)
+                            if (tgt == vb + x) p.zt[m] = __uint_as_float(z[x]);
+                    }
+                    float cm = -INFINITY;
+#pragma unroll
+                    for (int x = 0; x < 32; ++x)
+                        if (x < nvalid) cm = fmaxf(cm, __uint_as_float(z[x]));
+                    const float cm2 = cm * LOG2E_F;
+                    if (cm2 > mx) {
+                        l *= ex2f_approx(mx - cm2);
+                        mx = cm2;
+                    }
+                    float s = 0.f;
+#pragma unroll
+                    for (int x = 0; x < 32; ++x)
+                        if (x < nvalid) s += ex2f_approx(fmaf(__uint_as_float(z[x]), LOG2E_F, -mx));
+                    l += s;
+                }
+                tc_fence_before();
+                mbar_arrive(&acc_empty[ab]);
+            }
+            if (ok) p.part[(int64_t)c * p.M_pad + m] = make_float2(mx, l);
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, 512);
+    }
+}
+
+__global__ void k_lm_gather(int M, int M_pad, int d, const __nv_bfloat16* __restrict__ H,
+                            const int32_t* __restrict__ targets, const int32_t* __restrict__ rows,
+                            __nv_bfloat16* __restrict__ Hg, int32_t* __restrict__ tg) {
+    const int vec = d / 8;   // 16-byte vectors per row
+    const int64_t total = (int64_t)M_pad * vec;
+    for (int64_t x = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; x < total; x += (int64_t)gridDim.x * blockDim.x) {
+        const int m = (int)(x / vec), k = (int)(x % vec);
+        uint4 val = make_uint4(0, 0, 0, 0);
+        if (m < M) val = reinterpret_cast<const uint4*>(H + (int64_t)rows[m] * d)[k];
+        reinterpret_cast<uint4*>(Hg + (int64_t)m * d)[k] = val;
+        if (k == 0) tg[m] = m < M ? targets[rows[m]] : -1;
+    }
+}
+
+__global__ void k_lm_combine(int M, int M_pad, int C, const float2* __restrict__ part, const float* __restrict__ zt,
+                             float* __restrict__ lse, float* __restrict__ lp) {
+    const int m = blockIdx.x * blockDim.x + threadIdx.x;
+    if (m >= M) return;
+    float mx = -INFINITY;
+    for (int c = 0; c < C; ++c) mx = fmaxf(mx, part[(int64_t)c * M_pad + m].x);
+    float l = 0.f;
+    for (int c = 0; c < C; ++c) {
+        const float2 q = part[(int64_t)c * M_pad + m];
+        if (q.y > 0.f) l += q.y * exp2f(q.x - mx);
+    }
+    const float v = (mx + log2f(l)) * 0.6931471805599453f;
+    lse[m] = v;
+    lp[m] = zt[m] - v;
+}
+
+}  // namespace
+
+// Shapes of the bf16 LM-head work split, shared with the workspace layout.
+struct LmPlan {
+    int M_pad, R, NV, C, NVC, grid;
+};
+
+static int num_sms() {
+    int dev = 0, n = 152;
+    if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    return n > 0 ? n : 152;
+}
+
+LmPlan lm_plan(int M, int V) {
+    LmPlan q;
+    q.M_pad = (int)ceil_div(M, BM) * BM;
+    q.R = q.M_pad / BM;
+    q.NV = (int)ceil_div(V, BN);
+    const int G = num_sms();
+    // choose the number of vocab chunks C minimising waves x tiles-per-item
+    long best = -1;
+    q.C = 1;
+    for (int C = 1; C <= 64; ++C) {
+        const long items = (long)q.R * C;
+        const long waves = (items + G - 1) / G;
+        const long cost = waves * ceil_div(q.NV, C);
+        if (best < 0 || cost < best) { best = cost; q.C = C; }
+    }
+    q.NVC = (int)ceil_div(q.NV, q.C);
+    q.C = (int)ceil_div(q.NV, q.NVC);
+    q.grid = (int)std::min<long>((long)q.R * q.C, G);
+    return q;
+}
+
+mw_status lm_fwd_tc(const void* H, const void* W, const int32_t* targets, const int32_t* rows, int M, int d, int V,
+                    void* Hg, int32_t* tg, float2* part, float* zt, float* lse, float* lp, int32_t* status,
+                    cudaStream_t s) {
+    if (M == 0) return MW_OK;
+    const LmPlan q = lm_plan(M, V);
+    count_launches(3);
+    const int64_t vec = (int64_t)q.M_pad * (d / 8);
+    k_lm_gather<<<(unsigned)std::min<int64_t>(ceil_div(vec, 256), 152 * 32), 256, 0, s>>>(
+        M, q.M_pad, d, (const __nv_bfloat16*)H, targets, rows, (__nv_bfloat16*)Hg, tg);
+    CUtensorMap ta, tb;
+    if (!tmap_bf16_2d(&ta, Hg, q.M_pad, d, d, BM, BK) || !tmap_bf16_2d(&tb, W, V, d, d, BN, BK)) return MW_ECUDA;
+    LmFwdParams p;
+    p.M = M;
+    p.M_pad = q.M_pad;
+    p.d = d;
+    p.V = V;
+    p.R = q.R;
+    p.NV = q.NV;
+    p.C = q.C;
+    p.NVC = q.NVC;
+    p.tg = tg;
+    p.part = part;
+    p.zt = zt;
+    p.status = status;
+    mw_status st = cuda_status(cudaFuncSetAttribute(k_lm_fwd_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                    (int)SMEM_LMF));
+    if (st != MW_OK) return st;
+    k_lm_fwd_tc<<<q.grid, NT, SMEM_LMF, s>>>(ta, tb, p);
+    k_lm_combine<<<(unsigned)ceil_div(M, 256), 256, 0, s>>>(M, q.M_pad, q.C, part, zt, lse, lp);
+    return launch_status();
+}
+
+}  // namespace mw

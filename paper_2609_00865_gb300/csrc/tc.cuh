@@ -194,6 +194,13 @@ __device__ __forceinline__ uint32_t sw128_off(uint32_t row, uint32_t chunk16) {
     return row * 128u + ((chunk16 ^ (row & 7u)) << 4);
 }
 
+// 2^x on the MUFU unit (approximate; flushes denormals).
+__device__ __forceinline__ float ex2f_approx(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
     uint32_t r;
     asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));

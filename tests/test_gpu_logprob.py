@@ -82,3 +82,52 @@ def test_zero_weights_uniform():
     M = len(rows)
     out, dH, dW = _run(H, W, t, torch.tensor(rows, dtype=torch.int32), torch.zeros(M), torch.ones(M), 0.2, 0.2)
     np.testing.assert_allclose(np64(out["lp"]), -np.log(V), rtol=1e-6)
+
+
+@pytest.mark.parametrize("N,M,d,V", [
+    (700, 450, 512, 3001),      # 2-CTA cluster split of d, ragged vocab tail
+    (600, 300, 1536, 2999),     # the config-3 hidden size (4-CTA cluster)
+    (1200, 700, 3584, 152064),  # the config-4 hidden size and vocabulary (8-CTA cluster)
+])
+def test_tensor_core_shapes(N, M, d, V):
+    rows = np.sort(np.random.default_rng(N).permutation(N)[:M])
+    args = _case(N, d, V, rows, 70 + d, torch.bfloat16)
+    out, dH, dW = _run(*args[:6], 0.2, 0.28, dloss=0.7)
+    _check(*args, out, dH, dW, 0.2, 0.28, fp32=False, dloss=0.7)
+
+
+def test_config3_full_size_sampled():
+    """N = 32,768, d = 1,536, V = 151,936, 70% loss rows, in the bench's launch
+    configuration. lp / dH are checked on sampled rows, dW on sampled vocab
+    rows (the oracle's lse covers every loss row)."""
+    import paper_2609_00865_gb300 as mw
+    c = synth.CONFIGS[3]
+    N, d, V = c["N"], c["d"], c["V"]
+    rows = synth.loss_rows_fraction(N, c["loss_frac"], 3000)
+    M = len(rows)
+    g = torch.Generator(device="cuda").manual_seed(33)
+    H = torch.randn(N, d, device="cuda", generator=g).to(torch.bfloat16)
+    W = (0.02 * torch.randn(V, d, device="cuda", generator=g)).to(torch.bfloat16)
+    tg = torch.randint(0, V, (N,), device="cuda", generator=g, dtype=torch.int32)
+    adv = torch.randn(M, device="cuda", generator=g)
+    r_dev = torch.tensor(rows, dtype=torch.int32, device="cuda")
+    H64, W64, t_np = np64(H), np64(W), tg.cpu().numpy()
+    lp_ref, lse_ref = OL.logprob(H64, W64, t_np, rows)
+    lp_old = torch.tensor(lp_ref + 0.05 * np.random.default_rng(3).standard_normal(M), dtype=torch.float32,
+                          device="cuda")
+    out = mw.logprob_loss_fwd(H, W, tg, r_dev, lp_old, adv, 0.2, 0.2)
+    dH, dW = mw.logprob_loss_bwd(H, W, tg, r_dev, out["lse"], out["ws"])
+    torch.cuda.synchronize()
+    assert_maxabs(np64(out["lp"]), lp_ref, 1e-2, "lp")
+    ratio_r, _, loss_r, g_r = OL.policy_loss(lp_ref, np64(lp_old), np64(adv), 0.2, 0.2)
+    loss = float(out["loss"].item())
+    assert abs(loss - loss_r) <= 1e-3 * max(abs(loss_r), np.mean(np.abs(ratio_r * np64(adv))))
+    rng = np.random.default_rng(4)
+    pick = np.sort(rng.choice(M, 48, replace=False))
+    dHr, _ = OL.logprob_loss_bwd(H64, W64, t_np, rows[pick], lse_ref[pick], g_r[pick])
+    assert_grad_bf16(np64(dH)[rows[pick]], dHr[rows[pick]], "dH (sampled rows)")
+    notloss = np.setdiff1d(np.arange(N), rows)[:64]
+    assert (np64(dH)[notloss] == 0).all()
+    vocab = np.unique(np.concatenate([rng.integers(0, V, 40), t_np[rows[:8]], [0, V - 1]]))
+    dWr = OL.logprob_loss_bwd_vocab(H64, W64, t_np, rows, lse_ref, g_r, vocab)
+    assert_grad_bf16(np64(dW)[vocab], dWr, "dW (sampled vocab rows)")
