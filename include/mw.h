@@ -218,11 +218,13 @@ mw_status mw_logprob_loss_fwd(const void* H, const void* W, const int32_t* targe
  *   dH_t = sum_v dz_{m,v} W_v (rows outside `rows` get 0),
  *   dW_v = sum_m dz_{m,v} H_{rows[m]}.
  * Needs the forward's lse and `ws`. dH [N, d] in dtype; dW [Vocab, d] float32.
- * Both are overwritten.
+ * Both are overwritten. The backward keeps the forward's part of `ws` intact
+ * (it may run again with another dloss) and uses the rest as scratch, so two
+ * backward calls on one `ws` must not overlap in time.
  */
 mw_status mw_logprob_loss_bwd(const void* H, const void* W, const int32_t* targets,
                               const int32_t* rows, int M, int N, int d, int Vocab, int dtype,
-                              const float* lse, const void* ws, float dloss,
+                              const float* lse, void* ws, float dloss,
                               void* dH, float* dW, void* stream);
 
 /*

@@ -29,8 +29,9 @@ mw_status lm_fwd_tc(const void*, const void*, const int32_t*, const int32_t*, in
                     float2*, float*, float*, float*, int32_t*, cudaStream_t);
 
 bool lm_bwd_tc_supported(int d);
+int64_t lm_bwd_tc_scratch(int M, int d);
 mw_status lm_bwd_tc(const void*, int, int, int, int, const int32_t*, const void*, const int32_t*, const float*,
-                    const float*, float, void*, float*, int32_t*, cudaStream_t);
+                    const float*, float, void*, float*, int32_t*, void*, cudaStream_t);
 
 // Tensor-core LM-head path: bf16 with d a multiple of 64 that the clustered
 // backward can split (d / C <= 448 for a cluster of C <= 8 CTAs).
@@ -38,7 +39,7 @@ static bool lm_tc(int d, int dtype) { return dtype == MW_BF16 && d % 64 == 0 && 
 
 // Byte offsets inside the log-prob workspace.
 struct LmWs {
-    int64_t g, zt, hg, tg, part, status, bytes;
+    int64_t g, zt, hg, tg, part, bwd, status, bytes;
 };
 static LmWs lm_ws_layout(int N, int M, int d, int V, int dtype) {
     (void)N; (void)V;
@@ -48,11 +49,12 @@ static LmWs lm_ws_layout(int N, int M, int d, int V, int dtype) {
     w.g = o; o = align256(o + 4 * (int64_t)M);
     w.zt = o; o = align256(o + 4 * (int64_t)M);
     w.status = o; o = align256(o + 32);
-    w.hg = w.tg = w.part = o;
+    w.hg = w.tg = w.part = w.bwd = o;
     if (lm_tc(d, dtype)) {
         w.hg = o; o = align256(o + 2 * M_pad * d);
         w.tg = o; o = align256(o + 4 * M_pad);
         w.part = o; o = align256(o + 8 * 64 * M_pad);
+        w.bwd = o; o = align256(o + lm_bwd_tc_scratch(M, d));
     }
     w.bytes = o;
     return w;
@@ -149,7 +151,7 @@ extern "C" mw_status mw_logprob_loss_fwd(const void* H, const void* W, const int
 }
 
 extern "C" mw_status mw_logprob_loss_bwd(const void* H, const void* W, const int32_t* targets, const int32_t* rows,
-                                         int M, int N, int d, int V, int dtype, const float* lse, const void* ws,
+                                         int M, int N, int d, int V, int dtype, const float* lse, void* ws,
                                          float dloss, void* dH, float* dW, void* stream) {
     mw_status st = lm_args(N, M, d, V, dtype);
     if (st != MW_OK) return st;
@@ -158,13 +160,12 @@ extern "C" mw_status mw_logprob_loss_bwd(const void* H, const void* W, const int
     if (M > 0 && (!H || !W || !targets || !rows || !lse)) return MW_EINVAL;
     LmWs w = lm_ws_layout(N, M, d, V, dtype);
     if (lm_tc(d, dtype)) {
-        // the backward reads the forward's gathered rows and g, and writes
-        // only the status words of the workspace
-        void* wsm = const_cast<void*>(ws);
-        if ((st = cuda_status(cudaMemsetAsync(at<char>(wsm, w.status), 0, 32, (cudaStream_t)stream))) != MW_OK)
+        // the backward reads the forward's gathered rows and g; it writes the
+        // status words and its own scratch region of the workspace
+        if ((st = cuda_status(cudaMemsetAsync(at<char>(ws, w.status), 0, 32, (cudaStream_t)stream))) != MW_OK)
             return st;
-        return lm_bwd_tc(W, M, N, d, V, rows, at<char>(wsm, w.hg), at<int32_t>(wsm, w.tg), lse,
-                         at<float>(wsm, w.g), dloss, dH, dW, at<int32_t>(wsm, w.status), (cudaStream_t)stream);
+        return lm_bwd_tc(W, M, N, d, V, rows, at<char>(ws, w.hg), at<int32_t>(ws, w.tg), lse, at<float>(ws, w.g),
+                         dloss, dH, dW, at<int32_t>(ws, w.status), at<char>(ws, w.bwd), (cudaStream_t)stream);
     }
     return lm_bwd_simt(H, W, targets, rows, M, N, d, V, dtype, lse, at<float>(ws, w.g), dloss, dH, dW,
                        (cudaStream_t)stream);
