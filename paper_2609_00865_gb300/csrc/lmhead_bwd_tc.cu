@@ -7,22 +7,27 @@
 // A pass holds a 128-row tile X of the stationary operand and streams the
 // other operand Y. The tile's accumulator over the whole hidden size (128 x d
 // fp32) is larger than one SM's tensor memory, so a cluster of C CTAs shares
-// the tile: CTA r accumulates hidden columns [r ds, (r+1) ds), ds = d / C.
-// Step t of the cluster covers C NY streamed rows; CTA r
+// the tile: CTA r accumulates hidden columns [r ds, (r+1) ds), ds = d / C <=
+// 256. Step t of the cluster covers C NY streamed rows (NY = 256); CTA r
 //   1. computes the logits of its own NY streamed rows over the full hidden
 //      size, Z_r = X Y_{t,r}^T (TMEM; X and Y k-slices streamed by TMA),
 //   2. forms dz_r (bf16, 128 x NY) in the epilogue, writes it into its slot
-//      of a per-cluster ring in global memory (R = L + 1 steps deep, a few
+//      of a per-cluster ring in global memory (R = L + 2 steps deep, tens of
 //      MB in all, so it stays in L2) and signals every CTA of the cluster,
 //   3. accumulates Acc_r += sum_q dz_q Y_{t,q}[:, slice r] over the C dz
-//      tiles of the step (dz tiles and Y slices loaded by TMA).
+//      tiles of the step (dz k-chunks and Y slices loaded by TMA).
 // Only bf16 dz tiles cross CTAs, once per step. The accumulation of step t
 // is issued after the logits of step t + L, so the exchange has L steps of
 // tensor work to complete in. Clusters are persistent (as many as fit on the
-// GPU at once), so each owns a fixed ring region. One operand ring in shared
-// memory carries the stages in the order the MMA thread consumes them: the
-// k-slices of Z(t), then the Y slices of Acc(t - L). Every wait is bounded in
-// time.
+// GPU at once), so each owns a fixed ring region. One ring of 48 KB stages in
+// shared memory carries the operands in the order the MMA thread consumes
+// them: the k-slices of Z(t) (X 16 KB + Y 32 KB), then the stages of
+// Acc(t - L) (a 64-column chunk of one dz tile + the matching 64 Y rows).
+//
+// Every stage feeds at least 384 cycles of tensor work (N >= 192, K = 64):
+// one thread issues about one tcgen05.mma per 60 cycles and pays a few
+// hundred cycles per wait/commit, so narrower stages leave the tensor pipe
+// idle. Every wait is bounded in time.
 
 #include <math.h>
 
@@ -37,22 +42,24 @@ namespace {
 using namespace tc;
 
 constexpr int NT = 224;              // warp 0 TMA, warp 1 MMA, warp 2 signals, warps 3..6 epilogue
-constexpr int MAX_S = 8, MAX_DS = 2, MAX_R = 4;
-constexpr uint32_t SLOT = 32768;     // bytes per operand stage
+constexpr int NY = 256;              // streamed rows per CTA and step
+constexpr int S = 4;                 // operand stages
+constexpr uint32_t SLOT = 49152;     // bytes per operand stage
+constexpr uint32_t SMEM = S * SLOT + 1024;
+constexpr int MAX_R = 4;             // ring depth
 constexpr int RING_CTAS = 160;       // ring capacity, in CTAs
 constexpr float LOG2E_B = 1.4426950408889634f;
 
 struct LmBwdParams {
     int mode;            // 0: dH pass, 1: dW pass
-    int C, ds;           // cluster size, d-slice
-    int S, DS;           // operand stages, dz-tile stages
-    int L, R;            // accumulation lag in steps, ring depth R = L + 1
+    int C, ds;           // cluster size, d-slice (<= 256)
+    int L, R;            // accumulation lag in steps, ring depth R = L + 2
     int KD;              // 64-wide k-slices of d
     int NS;              // steps per tile
     int tiles, nclus;    // stationary tiles, clusters in the grid
     int M, M_pad, V;
     const int32_t* rows;   // [M]
-    const float4* par;     // [M_pad] per loss row: (dloss g, lse log2 e, target bits, valid)
+    const float4* par;     // [M_pad] per loss row: (dloss g, lse log2 e, target bits, -)
     __nv_bfloat16* dH;     // [N, d]
     float* dW;             // [V, d]
     __nv_bfloat16* ring;   // [nclus][R][C][128][NY] dz exchange ring
@@ -69,12 +76,23 @@ __device__ __forceinline__ uint32_t mapa(uint32_t addr, uint32_t rank) {
     asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
     return r;
 }
-__device__ __forceinline__ void arrive_remote(uint32_t cluster_addr) {
-    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+// Remote arrive without its own release; the caller issues one cluster-scope
+// fence before a batch of these.
+__device__ __forceinline__ void arrive_remote_relaxed(uint32_t cluster_addr) {
+    asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
 }
+__device__ __forceinline__ void fence_acq_rel_cluster() { asm volatile("fence.acq_rel.cluster;" ::: "memory"); }
 // Orders this thread's generic global accesses with the async proxy (TMA).
 __device__ __forceinline__ void fence_proxy_async_global() {
     asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+// Arrive on the mbarrier at the same shared-memory offset in every CTA of
+// `mask` once this thread's issued MMAs have completed.
+__device__ __forceinline__ void commit_multicast(uint64_t* bar, uint16_t mask) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::
+                     "r"(smem_u32(bar)),
+                 "h"(mask)
+                 : "memory");
 }
 // Non-suspending poll: the arrivals on these barriers come from other CTAs.
 __device__ __forceinline__ bool try_wait_cluster(uint32_t addr, uint32_t parity) {
@@ -106,25 +124,21 @@ __device__ __forceinline__ bool wait_cluster(uint64_t* bar, uint32_t parity, int
     return false;
 }
 
-template <int NY>
 __global__ void __launch_bounds__(NT, 1)
     k_lm_bwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmYz,
                 const __grid_constant__ CUtensorMap tmYa, const __grid_constant__ CUtensorMap tmD, LmBwdParams p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~uintptr_t(1023));
-    __shared__ __align__(8) uint64_t op_full[MAX_S], op_empty[MAX_S], dz_full[MAX_DS], dz_empty[MAX_DS], zt_full,
-        zt_free, acc_full, acc_free, epi_done[MAX_R], dz_ready[MAX_R], dz_free[MAX_R];
+    __shared__ __align__(8) uint64_t op_full[S], op_empty[S], zt_full, zt_free, acc_full, acc_free, epi_done[MAX_R],
+        dz_ready[MAX_R], dz_free[MAX_R];
     __shared__ uint32_t tmem_base;
 
-    constexpr int KA = NY / 64;                 // 64-row k-chunks of a dz tile
-    constexpr uint32_t dzb = NY * 256;          // bytes of one dz tile
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int C = p.C, ds = p.ds, S = p.S, DS = p.DS, KD = p.KD, NS = p.NS, L = p.L, R = p.R;
+    const int C = p.C, ds = p.ds, KD = p.KD, NS = p.NS, L = p.L, R = p.R;
     const int rank = (int)cluster_rank();
     const int cid = blockIdx.x / C;
     const int col0 = rank * ds;                 // this CTA's hidden-column slice
-    const int NB = ds / 64;                     // 64-column boxes of the slice
-    const int NG = (NB + 3) / 4;                // accumulation MMAs (N <= 256) per k-chunk
+    const int NB = (ds + 63) / 64;              // 64-column Y boxes covering the slice
     const int my_tiles = cid < p.tiles ? (p.tiles - 1 - cid) / p.nclus + 1 : 0;
     const int G = my_tiles * NS;                // steps of this cluster
     const uint32_t TM_ACC = 0, TM_Z = (uint32_t)ds;
@@ -134,10 +148,6 @@ __global__ void __launch_bounds__(NT, 1)
         for (int s = 0; s < S; ++s) {
             mbar_init(&op_full[s], 1);
             mbar_init(&op_empty[s], 1);
-        }
-        for (int s = 0; s < DS; ++s) {
-            mbar_init(&dz_full[s], 1);
-            mbar_init(&dz_empty[s], 2);   // the MMA's completion and the signaller
         }
         mbar_init(&zt_full, 1);
         mbar_init(&zt_free, 128);
@@ -160,7 +170,6 @@ __global__ void __launch_bounds__(NT, 1)
     tc_fence_after();
     const uint32_t tmem = tmem_base;
     const uint32_t base = smem_u32(sm);
-    const uint32_t dz_base = base + (uint32_t)S * SLOT;   // dz stages follow the operand stages
 
     // first ring row of writer q's tile in ring slot `slot`
     auto ring_row = [&](int slot, int q) { return ((cid * R + slot) * C + q) * 128; };
@@ -175,9 +184,9 @@ __global__ void __launch_bounds__(NT, 1)
             prefetch_tmap(&tmYz);
             prefetch_tmap(&tmYa);
             prefetch_tmap(&tmD);
-            int s = 0, dsl = 0;
-            uint32_t ph = 0, dph = 0;
-            bool filled = false, dfilled = false;
+            int s = 0;
+            uint32_t ph = 0;
+            bool filled = false;
             int zt = 0, ztile = cid;               // Z stream: step in tile, tile
             int at = 0, aslot = 0;                 // accumulation stream: step in tile, ring slot
             uint32_t aph = 0;
@@ -215,8 +224,8 @@ __global__ void __launch_bounds__(NT, 1)
                     }
                 }
                 if (gt >= L) {
-                    // Acc(gt - L): the C dz tiles of the step and, for each, the
-                    // matching Y rows restricted to this CTA's column slice
+                    // Acc(gt - L): for each writer q and 64-row k-chunk, the dz
+                    // chunk (128 x 64) and Y rows restricted to this CTA's slice
                     if (!wait_cluster(&dz_ready[aslot], aph, status, 602)) {
                         ok = false;
                         break;
@@ -224,31 +233,19 @@ __global__ void __launch_bounds__(NT, 1)
                     fence_proxy_async_global();
                     const int yb = at * C * NY;
                     for (int q = 0; ok && q < C; ++q) {
-                        if (dfilled && !mbar_wait(&dz_empty[dsl], dph ^ 1u, status, 603)) {
-                            ok = false;
-                            break;
-                        }
-                        mbar_expect_tx(&dz_full[dsl], dzb);
                         const int rr = ring_row(aslot, q);
-                        for (int kc = 0; kc < KA; ++kc)
-                            tma_load_2d(sm + S * SLOT + dsl * dzb + kc * 16384, &tmD, &dz_full[dsl], kc * 64, rr);
-                        if (++dsl == DS) {
-                            dsl = 0;
-                            dph ^= 1u;
-                            dfilled = true;
-                        }
-                        for (int kc = 0; ok && kc < KA; ++kc)
-                            for (int g = 0; g < NG; ++g) {
-                                const int nb = min(4, NB - 4 * g);
-                                const int slot = acquire((uint32_t)nb * 8192u);
-                                if (slot < 0) {
-                                    ok = false;
-                                    break;
-                                }
-                                for (int j = 0; j < nb; ++j)
-                                    tma_load_2d(sm + slot * SLOT + j * 8192, &tmYa, &op_full[slot],
-                                                col0 + (4 * g + j) * 64, yb + q * NY + kc * 64);
+                        for (int kc = 0; kc < NY / 64; ++kc) {
+                            const int slot = acquire(16384u + (uint32_t)NB * 8192u);
+                            if (slot < 0) {
+                                ok = false;
+                                break;
                             }
+                            uint8_t* dst = sm + slot * SLOT;
+                            tma_load_2d(dst, &tmD, &op_full[slot], kc * 64, rr);
+                            for (int j = 0; j < NB; ++j)
+                                tma_load_2d(dst + 16384 + j * 8192, &tmYa, &op_full[slot], col0 + j * 64,
+                                            yb + q * NY + kc * 64);
+                        }
                     }
                     if (++at == NS) at = 0;
                     if (++aslot == R) {
@@ -262,16 +259,14 @@ __global__ void __launch_bounds__(NT, 1)
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0) {
             const uint32_t iZ = idesc_bf16(128, NY, 0, 0);
-            const uint32_t iA0 = idesc_bf16(128, min(4, NB) * 64, 0, 1);
-            const uint32_t iA1 = idesc_bf16(128, NB > 4 ? (NB - 4) * 64 : 64, 0, 1);
-            // descriptors of byte 0 of the operand ring (K-major / MN-major with
-            // 64-row boxes) and of the dz stages; a byte offset b adds b >> 4
+            const uint32_t iA = idesc_bf16(128, ds, 0, 1);
+            // descriptors of byte 0 of the ring (K-major) and of byte 16384 of
+            // the ring (MN-major, 64-row boxes); a byte offset b adds b >> 4
             const uint64_t dK0 = sdesc_sw128(base, 16, 1024);
-            const uint64_t dM0 = sdesc_sw128(base, 8192, 1024);
-            const uint64_t dD0 = sdesc_sw128(dz_base, 16, 1024);
-            int s = 0, dsl = 0;
-            uint32_t ph = 0, dph = 0;
-            int at = 0, an = 0;                    // accumulation stream: step in tile, tiles done
+            const uint64_t dM0 = sdesc_sw128(base + 16384, 8192, 1024);
+            int s = 0;
+            uint32_t ph = 0;
+            int at = 0, an = 0, aslot = 0;         // accumulation stream: step in tile, tiles done, ring slot
             bool ok = true;
             for (int gt = 0; ok && gt < G + L; ++gt) {
                 if (gt < G) {
@@ -308,84 +303,50 @@ __global__ void __launch_bounds__(NT, 1)
                     }
                     tc_fence_after();
                     for (int q = 0; ok && q < C; ++q) {
-                        if (!mbar_wait(&dz_full[dsl], dph, status, 614)) {
-                            ok = false;
-                            break;
-                        }
-                        tc_fence_after();
-                        const uint64_t dzd = dD0 + (uint64_t)((dsl * dzb) >> 4);
-                        for (int kc = 0; ok && kc < KA; ++kc)
-                            for (int g = 0; g < NG; ++g) {
-                                if (!mbar_wait(&op_full[s], ph, status, 615)) {
-                                    ok = false;
-                                    break;
-                                }
-                                tc_fence_after();
-                                // B: 64 streamed rows (K) x nb 64-column boxes (N), MN-major
-                                const uint64_t da = dzd + (uint64_t)(kc * (16384 >> 4));
-                                const uint64_t db = dM0 + (uint64_t)((s * SLOT) >> 4);
-                                const uint32_t iA = g ? iA1 : iA0;
-#pragma unroll
-                                for (int ks = 0; ks < 4; ++ks)
-                                    mma_ss(tmem + TM_ACC + g * 256, da + 2 * ks, db + 128 * ks, iA,
-                                           (at | q | kc | ks) != 0);
-                                mma_commit(&op_empty[s]);
-                                if (++s == S) {
-                                    s = 0;
-                                    ph ^= 1u;
-                                }
+                        for (int kc = 0; kc < NY / 64; ++kc) {
+                            if (!mbar_wait(&op_full[s], ph, status, 615)) {
+                                ok = false;
+                                break;
                             }
-                        mma_commit(&dz_empty[dsl]);
-                        if (++dsl == DS) {
-                            dsl = 0;
-                            dph ^= 1u;
+                            tc_fence_after();
+                            const uint64_t da = dK0 + (uint64_t)((s * SLOT) >> 4);
+                            const uint64_t db = dM0 + (uint64_t)((s * SLOT) >> 4);
+#pragma unroll
+                            for (int ks = 0; ks < 4; ++ks)
+                                mma_ss(tmem + TM_ACC, da + 2 * ks, db + 128 * ks, iA, (at | q | kc | ks) != 0);
+                            mma_commit(&op_empty[s]);
+                            if (++s == S) {
+                                s = 0;
+                                ph ^= 1u;
+                            }
                         }
+                        // writer q may reuse its ring slot once these MMAs (and
+                        // so the loads of its tile) have completed
+                        if (ok) commit_multicast(&dz_free[aslot], (uint16_t)(1u << q));
                     }
                     if (ok && at == NS - 1) mma_commit(&acc_full);
                     if (++at == NS) {
                         at = 0;
                         ++an;
                     }
+                    if (++aslot == R) aslot = 0;
                 }
             }
         }
     } else if (warp == 2) {
         // ------------------------------------------------------------ signaller
-        // remote arrivals, kept off the MMA thread: dz tile of step gt
-        // published (to every CTA), dz tiles of step gt - L read (to their writers)
+        // the dz tile of step gt is published: tell every CTA of the cluster
         if (lane == 0) {
-            int slot = 0, aslot = 0, dsl = 0;
-            uint32_t sph = 0, dph = 0;
-            bool ok = true;
-            for (int gt = 0; ok && gt < G + L; ++gt) {
-                if (gt < G) {
-                    if (!mbar_wait(&epi_done[slot], sph, status, 631)) {
-                        ok = false;
-                        break;
-                    }
-                    const uint32_t a = smem_u32(&dz_ready[slot]);
-                    for (int q = 0; q < C; ++q) arrive_remote(mapa(a, (uint32_t)q));
-                    if (++slot == R) {
-                        slot = 0;
-                        sph ^= 1u;
-                    }
-                }
-                if (gt >= L) {
-                    const uint32_t a = smem_u32(&dz_free[aslot]);
-                    for (int q = 0; q < C; ++q) {
-                        // writer q's tile is in shared memory: q may reuse its ring slot
-                        if (!mbar_wait(&dz_full[dsl], dph, status, 632)) {
-                            ok = false;
-                            break;
-                        }
-                        arrive_remote(mapa(a, (uint32_t)q));
-                        mbar_arrive(&dz_empty[dsl]);
-                        if (++dsl == DS) {
-                            dsl = 0;
-                            dph ^= 1u;
-                        }
-                    }
-                    if (++aslot == R) aslot = 0;
+            int slot = 0;
+            uint32_t sph = 0;
+            for (int gt = 0; gt < G; ++gt) {
+                if (!mbar_wait(&epi_done[slot], sph, status, 631)) break;
+                fence_acq_rel_cluster();
+                const uint32_t a = smem_u32(&dz_ready[slot]);
+                for (int q = 0; q < C; ++q) arrive_remote_relaxed(mapa(a, (uint32_t)q));
+                if (++slot == R) {
+                    slot = 0;
+                    sph ^= 1u;
                 }
             }
         }
@@ -438,6 +399,7 @@ __global__ void __launch_bounds__(NT, 1)
         // zero-filled by TMA, so their dz contributes nothing.
         float4 rp = make_float4(0.f, 0.f, __int_as_float(-1), 0.f);
         int t = 0, tile = cid, slot = 0, drained = 0;
+        uint32_t sph = 0;                       // phase of ring slot `slot`
         int next_drain = NS + L - 1;            // step after which tile `drained` is complete
         for (int gt = 0; ok && gt < G; ++gt) {
             if (p.mode == 0 && t == 0) rp = p.par[tile * 128 + rl];
@@ -450,33 +412,33 @@ __global__ void __launch_bounds__(NT, 1)
                     cpar[j] = c < p.M_pad ? __ldg(&p.par[c]) : make_float4(0.f, 0.f, __int_as_float(-1), 0.f);
                 }
             }
+            if (!mbar_wait(&zt_full, (uint32_t)gt & 1u, status, 623)) {
+                ok = false;
+                break;
+            }
+            tc_fence_after();
             // every CTA has loaded this ring slot's previous tile (step gt - R)
             if (gt >= R) {
                 bool w = true;
-                if (lane == 0) w = wait_cluster(&dz_free[slot], (uint32_t)((gt - R) / R) & 1u, status, 622);
+                if (lane == 0) w = wait_cluster(&dz_free[slot], sph ^ 1u, status, 622);
                 w = __shfl_sync(0xffffffffu, w, 0);
                 if (!w) {
                     ok = false;
                     break;
                 }
             }
-            if (!mbar_wait(&zt_full, (uint32_t)gt & 1u, status, 623)) {
-                ok = false;
-                break;
-            }
-            tc_fence_after();
-            uint32_t z[NY];
-#pragma unroll
-            for (int j = 0; j < NY / 32; ++j)
-                tmem_ld32(lane_base + TM_Z + 32 * j, *reinterpret_cast<uint32_t(*)[32]>(z + 32 * j));
-            tmem_wait_ld();
-            tc_fence_before();
-            mbar_arrive(&zt_free);   // the MMA may overwrite Z now
             __nv_bfloat16* dst = p.ring + (int64_t)(ring_row(slot, rank) + rl) * NY;
             const int vrow = tile * 128 + rl;        // pass 1: this row's vocabulary entry
             const int tj = __float_as_int(rp.z) - cb;   // pass 0: target column inside the tile
 #pragma unroll
             for (int j = 0; j < NY / 32; ++j) {
+                uint32_t z[32];
+                tmem_ld32(lane_base + TM_Z + 32 * j, z);
+                tmem_wait_ld();
+                if (j == NY / 32 - 1) {
+                    tc_fence_before();
+                    mbar_arrive(&zt_free);   // the MMA may overwrite Z now
+                }
                 uint32_t pk[16];
 #pragma unroll
                 for (int x = 0; x < 32; x += 2) {
@@ -484,7 +446,7 @@ __global__ void __launch_bounds__(NT, 1)
 #pragma unroll
                     for (int y = 0; y < 2; ++y) {
                         const int c = 32 * j + x + y;
-                        const float zv = __uint_as_float(z[c]);
+                        const float zv = __uint_as_float(z[x + y]);
                         if (p.mode == 0) {
                             const float pr = ex2f_approx(fmaf(zv, LOG2E_B, -rp.y));
                             dz[y] = rp.x * ((c == tj ? 1.f : 0.f) - pr);
@@ -505,7 +467,10 @@ __global__ void __launch_bounds__(NT, 1)
             // publish: the tile is in global memory before any CTA's TMA reads it
             fence_proxy_async_global();
             mbar_arrive(&epi_done[slot]);
-            if (++slot == R) slot = 0;
+            if (++slot == R) {
+                slot = 0;
+                sph ^= 1u;
+            }
             if (++t == NS) {
                 t = 0;
                 tile += p.nclus;
@@ -543,52 +508,32 @@ __global__ void k_lm_bwd_par(int M, int M_pad, const float* __restrict__ g, cons
                    : make_float4(0.f, 0.f, __int_as_float(-1), 0.f);
 }
 
-struct BwdCfg {
-    int C, ds, NY, S, DS, L;
-    uint32_t smem;
-};
-
-// Smallest cluster whose d-slice leaves TMEM room for a logit tile of at
-// least 64 columns (ds + NY <= 512 columns); 128 columns when they fit. The
-// operand ring takes what two dz stages leave of the shared memory.
-bool choose_cfg(int d, BwdCfg& c) {
-    const uint32_t limit = 224 * 1024;
-    for (int C : {1, 2, 4, 8}) {
-        if (d % C) continue;
-        const int ds = d / C;
-        if (ds % 64 || ds > 448) continue;
-        const int NY = ds + 128 <= 512 ? 128 : 64;
-        const int DS = 2;
-        const uint32_t dzb = (uint32_t)NY * 256u;
-        const int S = std::min<int>(MAX_S, (int)((limit - DS * dzb) / SLOT));
-        if (S < 3) continue;
-        c = {C, ds, NY, S, DS, 2, (uint32_t)S * SLOT + DS * dzb + 1024};
-        return true;
-    }
-    return false;
-}
+// Cluster sizes whose d-slice fits beside a 256-column logit tile in TMEM
+// (ds <= 256) and keeps 32-column output chunks (ds % 32 == 0).
+bool slice_ok(int d, int C) { return d % C == 0 && d / C <= 256 && (d / C) % 32 == 0; }
+constexpr int kClusterSizes[] = {1, 2, 3, 4, 5, 6, 7, 8, 10, 12, 14, 16};
 
 }  // namespace
 
 bool lm_bwd_tc_supported(int d) {
-    BwdCfg c;
-    return choose_cfg(d, c);
+    if (d % 64) return false;
+    for (int C : kClusterSizes)
+        if (slice_ok(d, C)) return true;
+    return false;
 }
 
 // Scratch of the backward inside the log-prob workspace: the per-row
 // parameters and the dz exchange ring.
 int64_t lm_bwd_tc_scratch(int M, int d) {
-    BwdCfg c;
-    if (!choose_cfg(d, c)) return 0;
+    if (!lm_bwd_tc_supported(d)) return 0;
     const int64_t M_pad = ceil_div(M, 128) * 128;
-    return align256(16 * M_pad) + (int64_t)RING_CTAS * MAX_R * 128 * c.NY * 2;
+    return align256(16 * M_pad) + (int64_t)RING_CTAS * MAX_R * 128 * NY * 2;
 }
 
 mw_status lm_bwd_tc(const void* W, int M, int N, int d, int V, const int32_t* rows, const void* Hg, const int32_t* tg,
                     const float* lse, const float* g, float dloss, void* dH, float* dW, int32_t* status, void* scratch,
                     cudaStream_t s) {
-    BwdCfg c;
-    if (!choose_cfg(d, c)) return MW_ESHAPE;
+    if (!lm_bwd_tc_supported(d)) return MW_ESHAPE;
     mw_status st = cuda_status(cudaMemsetAsync(dH, 0, (size_t)N * d * 2, s));
     if (st != MW_OK) return st;
     if (M == 0) return cuda_status(cudaMemsetAsync(dW, 0, (size_t)V * d * 4, s));
@@ -599,41 +544,55 @@ mw_status lm_bwd_tc(const void* W, int M, int N, int d, int V, const int32_t* ro
     k_lm_bwd_par<<<(unsigned)ceil_div(M_pad, 256), 256, 0, s>>>(M, M_pad, g, lse, tg, dloss, par);
     if ((st = launch_status()) != MW_OK) return st;
 
-    const int ring_rows = RING_CTAS * MAX_R * 128;
-    CUtensorMap hx, hyz, hya, wx, wyz, wya, dm;
-    if (!tmap_bf16_2d(&hx, Hg, M_pad, d, d, 128, 64) || !tmap_bf16_2d(&hyz, Hg, M_pad, d, d, c.NY, 64) ||
-        !tmap_bf16_2d(&hya, Hg, M_pad, d, d, 64, 64) || !tmap_bf16_2d(&wx, W, V, d, d, 128, 64) ||
-        !tmap_bf16_2d(&wyz, W, V, d, d, c.NY, 64) || !tmap_bf16_2d(&wya, W, V, d, d, 64, 64) ||
-        !tmap_bf16_2d(&dm, ring, ring_rows, c.NY, c.NY, 128, 64))
-        return MW_ECUDA;
-    auto kern = c.NY == 128 ? k_lm_bwd_tc<128> : k_lm_bwd_tc<64>;
-    if ((st = cuda_status(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                               (int)c.smem))) != MW_OK)
+    if ((st = cuda_status(cudaFuncSetAttribute(k_lm_bwd_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               (int)SMEM))) != MW_OK ||
+        (st = cuda_status(cudaFuncSetAttribute(k_lm_bwd_tc, cudaFuncAttributeNonPortableClusterSizeAllowed, 1))) !=
+            MW_OK)
         return st;
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = c.C;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
     cfg.blockDim = dim3(NT);
-    cfg.dynamicSmemBytes = c.smem;
+    cfg.dynamicSmemBytes = SMEM;
     cfg.stream = s;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    cfg.gridDim = dim3((unsigned)c.C);
-    int max_clusters = 0;
-    if ((st = cuda_status(cudaOccupancyMaxActiveClusters(&max_clusters, kern, &cfg))) != MW_OK) return st;
-    if (max_clusters < 1) return MW_EDEVICE;
-    max_clusters = std::min(max_clusters, RING_CTAS / c.C);
+    // the cluster size that keeps the most CTAs resident (smaller on ties)
+    int C = 0, max_clusters = 0, best = 0;
+    for (int c : kClusterSizes) {
+        if (!slice_ok(d, c)) continue;
+        attr[0].val.clusterDim.x = (unsigned)c;
+        cfg.gridDim = dim3((unsigned)c);
+        int n = 0;
+        if (cudaOccupancyMaxActiveClusters(&n, k_lm_bwd_tc, &cfg) != cudaSuccess) {
+            (void)cudaGetLastError();
+            continue;
+        }
+        n = std::min(n, RING_CTAS / c);
+        if (n * c > best) {
+            best = n * c;
+            C = c;
+            max_clusters = n;
+        }
+    }
+    if (C == 0) return MW_EDEVICE;
+    attr[0].val.clusterDim.x = (unsigned)C;
+
+    const int ring_rows = RING_CTAS * MAX_R * 128;
+    CUtensorMap hx, hyz, hya, wx, wyz, wya, dm;
+    if (!tmap_bf16_2d(&hx, Hg, M_pad, d, d, 128, 64) || !tmap_bf16_2d(&hyz, Hg, M_pad, d, d, NY, 64) ||
+        !tmap_bf16_2d(&hya, Hg, M_pad, d, d, 64, 64) || !tmap_bf16_2d(&wx, W, V, d, d, 128, 64) ||
+        !tmap_bf16_2d(&wyz, W, V, d, d, NY, 64) || !tmap_bf16_2d(&wya, W, V, d, d, 64, 64) ||
+        !tmap_bf16_2d(&dm, ring, ring_rows, NY, NY, 128, 64))
+        return MW_ECUDA;
 
     LmBwdParams p;
-    p.C = c.C;
-    p.ds = c.ds;
-    p.S = c.S;
-    p.DS = c.DS;
-    p.L = c.L;
-    p.R = c.L + 1;
+    p.C = C;
+    p.ds = d / C;
+    p.L = 2;
+    p.R = p.L + 2;
     p.KD = d / 64;
     p.M = M;
     p.M_pad = M_pad;
@@ -647,11 +606,11 @@ mw_status lm_bwd_tc(const void* W, int M, int N, int d, int V, const int32_t* ro
     for (int mode = 0; mode < 2; ++mode) {
         p.mode = mode;
         p.tiles = mode == 0 ? M_pad / 128 : (int)ceil_div(V, 128);
-        p.NS = (int)ceil_div(mode == 0 ? V : M_pad, (int64_t)c.C * c.NY);
+        p.NS = (int)ceil_div(mode == 0 ? V : M_pad, (int64_t)C * NY);
         p.nclus = std::min(p.tiles, max_clusters);
-        cfg.gridDim = dim3((unsigned)(p.nclus * c.C));
+        cfg.gridDim = dim3((unsigned)(p.nclus * C));
         count_launches(1);
-        if ((st = cuda_status(cudaLaunchKernelEx(&cfg, kern, mode == 0 ? hx : wx, mode == 0 ? wyz : hyz,
+        if ((st = cuda_status(cudaLaunchKernelEx(&cfg, k_lm_bwd_tc, mode == 0 ? hx : wx, mode == 0 ? wyz : hyz,
                                                  mode == 0 ? wya : hya, dm, p))) != MW_OK)
             return st;
     }
