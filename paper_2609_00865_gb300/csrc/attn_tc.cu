@@ -36,6 +36,11 @@ constexpr int DH = 128;
 constexpr uint32_t TILE_B = 128 * DH * 2;  // one 128 x 128 bf16 tile: two [128][64] swizzled halves
 constexpr uint32_t HALF_B = TILE_B / 2;
 constexpr int NTHREADS = 192;
+// Backward kernels: warp 0 TMA, warp 1 MMA, warps 2..9 elementwise; two warps
+// per TMEM lane quarter split each row's columns, which hides the latency of
+// the exp / scale / pack chains that bound the kernels with one warp per quarter.
+constexpr int NT_BWD = 320;
+constexpr int NEW = 256;   // elementwise threads
 constexpr float LOG2E = 1.4426950408889634f;
 constexpr float RESCALE_T = 8.0f;          // lazy-rescale threshold (log2 units)
 
@@ -346,7 +351,7 @@ struct BwdParams {
     __nv_bfloat16* dV;
 };
 
-__global__ void __launch_bounds__(NTHREADS, 1)
+__global__ void __launch_bounds__(NT_BWD, 1)
     k_attn_dq_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmDO,
                  const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, BwdParams p) {
     extern __shared__ uint8_t smem_raw[];
@@ -380,11 +385,11 @@ __global__ void __launch_bounds__(NTHREADS, 1)
             mbar_init(&v_full[s], 1);
             mbar_init(&v_empty[s], 1);
             mbar_init(&s_full[s], 1);
-            mbar_init(&s_free[s], 128);
+            mbar_init(&s_free[s], NEW);
         }
         mbar_init(&dp_full, 1);
-        mbar_init(&dp_free, 128);
-        mbar_init(&ds_full, 128);
+        mbar_init(&dp_free, NEW);
+        mbar_init(&ds_full, NEW);
         mbar_init(&dq_done, 1);
         fence_mbar_init();
     }
@@ -470,7 +475,9 @@ __global__ void __launch_bounds__(NTHREADS, 1)
             }
         }
     } else {
+        // row rl = TMEM lane; this warp's 64 of the 128 key columns: [64 ch, 64 ch + 64)
         const int qw = warp & 3;
+        const int ch = (warp - 2) >> 2;
         const int rl = qw * 32 + lane;
         const int i = qt * 128 + rl;
         const int ie = min(i, T - 1);
@@ -486,12 +493,12 @@ __global__ void __launch_bounds__(NTHREADS, 1)
             const int kt = e >> 2, cls = e & 3;
             if (!mbar_wait(&s_full[j & 1], (j >> 1) & 1, status, 311)) { ok = false; break; }
             tc_fence_after();
-            float s[128];
+            float s[64];
             {
                 uint32_t rr[32];
 #pragma unroll
-                for (int c = 0; c < 4; ++c) {
-                    tmem_ld32(lane_base + TM_S0 + (j & 1) * 128 + c * 32, rr);
+                for (int c = 0; c < 2; ++c) {
+                    tmem_ld32(lane_base + TM_S0 + (j & 1) * 128 + (2 * ch + c) * 32, rr);
                     tmem_wait_ld();
 #pragma unroll
                     for (int x = 0; x < 32; ++x) s[c * 32 + x] = __uint_as_float(rr[x]);
@@ -512,26 +519,28 @@ __global__ void __launch_bounds__(NTHREADS, 1)
                     }
                 }
             }
+            const uint32_t w0 = ch ? wd[2] : wd[0], w1 = ch ? wd[3] : wd[1];
 #pragma unroll
-            for (int c = 0; c < 128; ++c)
-                s[c] = ((wd[c >> 5] >> (c & 31)) & 1u) ? ex2(fmaf(s[c], p.scale_log2, -lse2)) : 0.f;
+            for (int c = 0; c < 64; ++c)
+                s[c] = (((c < 32 ? w0 : w1) >> (c & 31)) & 1u) ? ex2(fmaf(s[c], p.scale_log2, -lse2)) : 0.f;
             if (!mbar_wait(&dp_full, j & 1, status, 312)) { ok = false; break; }
             tc_fence_after();
             // dS_j overwrites dS_{j-1}: wait until dQ += dS_{j-1} K_{j-1} is done
             if (j >= 1 && !mbar_wait(&dq_done, (j - 1) & 1, status, 313)) { ok = false; break; }
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
+            for (int cc = 0; cc < 2; ++cc) {
+                const int c = 2 * ch + cc;   // 32-column chunk of the row
                 uint32_t dp[32];
                 tmem_ld32(lane_base + TM_DP + c * 32, dp);
                 tmem_wait_ld();
-                if (c == 3) {
+                if (cc == 1) {
                     tc_fence_before();
                     mbar_arrive(&dp_free);
                 }
 #pragma unroll
                 for (int x = 0; x < 4; ++x) {
                     uint4 pk;
-                    const int c0 = c * 32 + 8 * x;
+                    const int c0 = cc * 32 + 8 * x;
                     pk.x = pack_bf16(s[c0 + 0] * (__uint_as_float(dp[8 * x + 0]) - dl),
                                      s[c0 + 1] * (__uint_as_float(dp[8 * x + 1]) - dl));
                     pk.y = pack_bf16(s[c0 + 2] * (__uint_as_float(dp[8 * x + 2]) - dl),
@@ -553,7 +562,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
             __nv_bfloat16* qrow = p.dQ + ((tok0 + ie) * p.Hq + h) * DH;
             uint32_t o[32];
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
+            for (int cc = 0; cc < 2; ++cc) {
+                const int c = 2 * ch + cc;
                 tmem_ld32(lane_base + TM_DQ + c * 32, o);
                 tmem_wait_ld();
                 if (i < T) {
@@ -593,8 +603,9 @@ constexpr uint32_t HT_HALF = HT_B / 2;
 constexpr uint32_t PT_B = 128 * 64 * 2;    // [128 keys][64 rows] bf16
 constexpr uint32_t KV_K = 0;
 constexpr uint32_t KV_V = KV_K + TILE_B;
-constexpr uint32_t KV_Q = KV_V + TILE_B;           // 2 stages of (Q half, dO half)
-constexpr uint32_t KV_P = KV_Q + 2 * 2 * HT_B;     // 2 buffers of P^T
+constexpr int QD_ST = 3;                           // (Q half, dO half) stages
+constexpr uint32_t KV_Q = KV_V + TILE_B;
+constexpr uint32_t KV_P = KV_Q + QD_ST * 2 * HT_B; // 2 buffers of P^T
 constexpr uint32_t KV_DS = KV_P + 2 * PT_B;        // 2 buffers of dS^T
 constexpr uint32_t SMEM_KV = KV_DS + 2 * PT_B + 1024;
 constexpr uint32_t TM_ST = 0, TM_DPT = 128, TM_DV = 256, TM_DK = 384;
@@ -608,12 +619,12 @@ __device__ __forceinline__ uint64_t mnmaj_ht(uint32_t base, int ks) {
     return sdesc_sw128(base + ks * 2048, HT_HALF, 1024);
 }
 
-__global__ void __launch_bounds__(NTHREADS, 1)
+__global__ void __launch_bounds__(NT_BWD, 1)
     k_attn_dkdv_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmDO,
                    const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, BwdParams p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~uintptr_t(1023));
-    __shared__ __align__(8) uint64_t kv_full, qd_full[2], qd_empty[2], sd_full[2], sd_free[2], pd_full[2],
+    __shared__ __align__(8) uint64_t kv_full, qd_full[QD_ST], qd_empty[QD_ST], sd_full[2], sd_free[2], pd_full[2],
         pd_free[2], ls_full[2], ls_free[2];
     __shared__ uint32_t tmem_base;
     __shared__ float lsd[2][128];   // per step: LSE2 of the 64 rows, then Delta of the 64 rows
@@ -638,15 +649,17 @@ __global__ void __launch_bounds__(NTHREADS, 1)
 
     if (threadIdx.x == 0) {
         mbar_init(&kv_full, 1);
-        for (int s = 0; s < 2; ++s) {
+        for (int s = 0; s < QD_ST; ++s) {
             mbar_init(&qd_full[s], 1);
             mbar_init(&qd_empty[s], 1);
+        }
+        for (int s = 0; s < 2; ++s) {
             mbar_init(&sd_full[s], 1);
-            mbar_init(&sd_free[s], 128);
-            mbar_init(&pd_full[s], 128);
+            mbar_init(&sd_free[s], NEW);
+            mbar_init(&pd_full[s], NEW);
             mbar_init(&pd_free[s], 1);
-            mbar_init(&ls_full[s], 128);
-            mbar_init(&ls_free[s], 128);
+            mbar_init(&ls_full[s], NEW);
+            mbar_init(&ls_free[s], NEW);
         }
         fence_mbar_init();
     }
@@ -678,10 +691,10 @@ __global__ void __launch_bounds__(NTHREADS, 1)
             load_tile(sm + KV_K, &tmK, &kv_full, kvh, (int)(tok0 + kt * 128));
             load_tile(sm + KV_V, &tmV, &kv_full, kvh, (int)(tok0 + kt * 128));
             for (int t = 0; t < nsteps; ++t) {
-                const int s = t & 1;
+                const int s = t % QD_ST;
                 int hq;
                 const int q0 = step_q0(t, hq);
-                if (t >= 2 && !mbar_wait(&qd_empty[s], ((t - 2) >> 1) & 1, status, 121)) break;
+                if (t >= QD_ST && !mbar_wait(&qd_empty[s], ((t / QD_ST) - 1) & 1, status, 121)) break;
                 mbar_expect_tx(&qd_full[s], 2 * HT_B);
                 uint8_t* dst = sm + KV_Q + s * 2 * HT_B;
                 tma_load_3d(dst, &tmQ, &qd_full[s], 0, hq, (int)(tok0 + q0));
@@ -698,11 +711,11 @@ __global__ void __launch_bounds__(NTHREADS, 1)
                            spb = smem_u32(sm + KV_P), sdb = smem_u32(sm + KV_DS);
             bool ok = mbar_wait(&kv_full, 0, status, 221);
             auto issue_sd = [&](int t) -> bool {
-                const int s = t & 1;
-                if (!mbar_wait(&qd_full[s], (t >> 1) & 1, status, 222)) return false;
+                const int s = t & 1, qs = t % QD_ST;
+                if (!mbar_wait(&qd_full[qs], (t / QD_ST) & 1, status, 222)) return false;
                 if (t >= 2 && !mbar_wait(&sd_free[s], ((t - 2) >> 1) & 1, status, 223)) return false;
                 tc_fence_after();
-                const uint32_t qb = sq + s * 2 * HT_B, db = qb + HT_B;
+                const uint32_t qb = sq + qs * 2 * HT_B, db = qb + HT_B;
 #pragma unroll
                 for (int ks = 0; ks < 8; ++ks) mma_ss(tmem + TM_ST + s * 64, kmaj(sk, ks), kmaj_ht(qb, ks), iSD, ks > 0);
 #pragma unroll
@@ -711,10 +724,10 @@ __global__ void __launch_bounds__(NTHREADS, 1)
                 return true;
             };
             auto issue_acc = [&](int t) -> bool {
-                const int s = t & 1;
+                const int s = t & 1, qs = t % QD_ST;
                 if (!mbar_wait(&pd_full[s], (t >> 1) & 1, status, 224)) return false;
                 tc_fence_after();
-                const uint32_t qb = sq + s * 2 * HT_B, db = qb + HT_B;
+                const uint32_t qb = sq + qs * 2 * HT_B, db = qb + HT_B;
                 const uint32_t pb = spb + s * PT_B, dsb = sdb + s * PT_B;
 #pragma unroll
                 for (int ks = 0; ks < 4; ++ks)
@@ -722,7 +735,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
 #pragma unroll
                 for (int ks = 0; ks < 4; ++ks)
                     mma_ss(tmem + TM_DK, sdesc_sw128(dsb + ks * 32, 16, 1024), mnmaj_ht(qb, ks), iAC, (t > 0 || ks > 0));
-                mma_commit(&qd_empty[s]);
+                mma_commit(&qd_empty[qs]);
                 mma_commit(&pd_free[s]);
                 return true;
             };
@@ -733,13 +746,16 @@ __global__ void __launch_bounds__(NTHREADS, 1)
             }
         }
     } else {
+        // key row rl = TMEM lane; this warp's 32 of a half-step's 64 query
+        // columns: [32 ch, 32 ch + 32)
         const int qw = warp & 3;
+        const int ch = (warp - 2) >> 2;
         const int rl = qw * 32 + lane;               // key row inside the k-tile = TMEM lane
         const int jk = kt * 128 + rl;
         const int je = min(jk, T - 1);
         const int iend = jk < T ? min(v.omega[tok0 + je], T) : 0;   // rows [jk, iend) see this key
         const uint32_t lane_base = tmem + ((uint32_t)(qw * 32) << 16);
-        const int tid = threadIdx.x - 64;            // 0..127 among the softmax threads
+        const int tid = threadIdx.x - 64;            // 0..255 among the elementwise threads
         bool ok = true;
         for (int t = 0; t < nsteps; ++t) {
             const int s = t & 1;
@@ -747,45 +763,47 @@ __global__ void __launch_bounds__(NTHREADS, 1)
             const int q0 = step_q0(t, hq);
             {   // this step's LSE2 (threads 0..63) and Delta (64..127) of rows q0 .. q0+63
                 if (t >= 2 && !mbar_wait(&ls_free[s], ((t - 2) >> 1) & 1, status, 324)) { ok = false; break; }
-                const int row = min(q0 + (tid & 63), T - 1);
-                const int64_t at = (int64_t)hq * p.total + tok0 + row;
-                lsd[s][tid] = tid < 64 ? p.LSE[at] * LOG2E : p.delta[at];
+                if (tid < 128) {
+                    const int row = min(q0 + (tid & 63), T - 1);
+                    const int64_t at = (int64_t)hq * p.total + tok0 + row;
+                    lsd[s][tid] = tid < 64 ? p.LSE[at] * LOG2E : p.delta[at];
+                }
                 mbar_arrive(&ls_full[s]);
                 if (!mbar_wait(&ls_full[s], (t >> 1) & 1, status, 325)) { ok = false; break; }
             }
             if (!mbar_wait(&sd_full[s], (t >> 1) & 1, status, 321)) { ok = false; break; }
             tc_fence_after();
-            float sv[64], dp[64];
+            float sv[32], dp[32];
             {
                 uint32_t rr[32];
+                tmem_ld32(lane_base + TM_ST + s * 64 + ch * 32, rr);
+                tmem_wait_ld();
 #pragma unroll
-                for (int c = 0; c < 2; ++c) {
-                    tmem_ld32(lane_base + TM_ST + s * 64 + c * 32, rr);
-                    tmem_wait_ld();
+                for (int x = 0; x < 32; ++x) sv[x] = __uint_as_float(rr[x]);
+                tmem_ld32(lane_base + TM_DPT + s * 64 + ch * 32, rr);
+                tmem_wait_ld();
 #pragma unroll
-                    for (int x = 0; x < 32; ++x) sv[c * 32 + x] = __uint_as_float(rr[x]);
-                    tmem_ld32(lane_base + TM_DPT + s * 64 + c * 32, rr);
-                    tmem_wait_ld();
-#pragma unroll
-                    for (int x = 0; x < 32; ++x) dp[c * 32 + x] = __uint_as_float(rr[x]);
-                }
+                for (int x = 0; x < 32; ++x) dp[x] = __uint_as_float(rr[x]);
             }
             tc_fence_before();
             mbar_arrive(&sd_free[s]);
-            const int lo = max(jk, q0) - q0, hi = min(iend, q0 + 64) - q0;   // visible columns [lo, hi)
+            // visible columns [lo, hi) of this warp's 32
+            const int lo = max(jk, q0 + 32 * ch) - q0 - 32 * ch, hi = min(iend, q0 + 64) - q0 - 32 * ch;
+            const float* lse_c = lsd[s] + 32 * ch;
+            const float* del_c = lsd[s] + 64 + 32 * ch;
 #pragma unroll
-            for (int c = 0; c < 64; ++c) {
+            for (int c = 0; c < 32; ++c) {
                 const bool vis = c >= lo && c < hi;
-                const float pr = vis ? ex2(fmaf(sv[c], p.scale_log2, -lsd[s][c])) : 0.f;
+                const float pr = vis ? ex2(fmaf(sv[c], p.scale_log2, -lse_c[c])) : 0.f;
                 sv[c] = pr;
-                dp[c] = pr * (dp[c] - lsd[s][64 + c]);
+                dp[c] = pr * (dp[c] - del_c[c]);
             }
             mbar_arrive(&ls_free[s]);
             if (t >= 2 && !mbar_wait(&pd_free[s], ((t - 2) >> 1) & 1, status, 322)) { ok = false; break; }
             uint8_t* pbuf = sm + KV_P + s * PT_B;
             uint8_t* dbuf = sm + KV_DS + s * PT_B;
 #pragma unroll
-            for (int c = 0; c < 8; ++c) {
+            for (int c = 0; c < 4; ++c) {
                 uint4 a, d;
                 a.x = pack_bf16(sv[8 * c + 0], sv[8 * c + 1]);
                 a.y = pack_bf16(sv[8 * c + 2], sv[8 * c + 3]);
@@ -795,8 +813,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
                 d.y = pack_bf16(dp[8 * c + 2], dp[8 * c + 3]);
                 d.z = pack_bf16(dp[8 * c + 4], dp[8 * c + 5]);
                 d.w = pack_bf16(dp[8 * c + 6], dp[8 * c + 7]);
-                *reinterpret_cast<uint4*>(pbuf + sw128_off(rl, c)) = a;
-                *reinterpret_cast<uint4*>(dbuf + sw128_off(rl, c)) = d;
+                *reinterpret_cast<uint4*>(pbuf + sw128_off(rl, 4 * ch + c)) = a;
+                *reinterpret_cast<uint4*>(dbuf + sw128_off(rl, 4 * ch + c)) = d;
             }
             fence_async_smem();
             tc_fence_before();
@@ -812,7 +830,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
                 const float mul = pass == 0 ? 1.f : p.scale;
                 const uint32_t col = pass == 0 ? TM_DV : TM_DK;
 #pragma unroll
-                for (int c = 0; c < 4; ++c) {
+                for (int cc = 0; cc < 2; ++cc) {
+                    const int c = 2 * ch + cc;
                     tmem_ld32(lane_base + col + c * 32, o);
                     tmem_wait_ld();
                     if (jk < T) {
@@ -909,8 +928,8 @@ mw_status attn_bwd_tc(const mw_vis_layout* L, const void* vis, const void* Q, co
                                                (int)SMEM_KV))) != MW_OK)
         return st;
     count_launches(2);
-    k_attn_dq_tc<<<(unsigned)((int64_t)L->max_tiles * L->n_traj * Hq), NTHREADS, SMEM_DQ, s>>>(tq, tdo, tk, tv, p);
-    k_attn_dkdv_tc<<<(unsigned)((int64_t)L->max_tiles * L->n_traj * Hkv), NTHREADS, SMEM_KV, s>>>(tq64, tdo64, tk,
+    k_attn_dq_tc<<<(unsigned)((int64_t)L->max_tiles * L->n_traj * Hq), NT_BWD, SMEM_DQ, s>>>(tq, tdo, tk, tv, p);
+    k_attn_dkdv_tc<<<(unsigned)((int64_t)L->max_tiles * L->n_traj * Hkv), NT_BWD, SMEM_KV, s>>>(tq64, tdo64, tk,
                                                                                                    tv, p);
     return launch_status();
 }
