@@ -35,7 +35,8 @@ using namespace tc;
 constexpr int DH = 128;
 constexpr uint32_t TILE_B = 128 * DH * 2;  // one 128 x 128 bf16 tile: two [128][64] swizzled halves
 constexpr uint32_t HALF_B = TILE_B / 2;
-constexpr int NTHREADS = 192;
+// Forward: warp 0 TMA, warp 1 MMA, warps 2..5 softmax (one row per thread).
+constexpr int NT_FWD = 192;
 // Backward kernels: warp 0 TMA, warp 1 MMA, warps 2..9 elementwise; two warps
 // per TMEM lane quarter split each row's columns, which hides the latency of
 // the exp / scale / pack chains that bound the kernels with one warp per quarter.
@@ -85,7 +86,7 @@ __device__ __forceinline__ uint64_t mnmaj(uint32_t base, int ks) {
     return sdesc_sw128(base + ks * 2048, HALF_B, 1024);
 }
 
-__global__ void __launch_bounds__(NTHREADS, 1)
+__global__ void __launch_bounds__(NT_FWD, 1)
     k_attn_fwd_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                   const __grid_constant__ CUtensorMap tmV, FwdParams p) {
     extern __shared__ uint8_t smem_raw[];
@@ -757,20 +758,25 @@ __global__ void __launch_bounds__(NT_BWD, 1)
         const uint32_t lane_base = tmem + ((uint32_t)(qw * 32) << 16);
         const int tid = threadIdx.x - 64;            // 0..255 among the elementwise threads
         bool ok = true;
+        // LSE2 (threads 0..63) and Delta (64..127) of step t's rows q0 .. q0+63; a
+        // step's values are loaded during the previous step and published at its end
+        auto ls_load = [&](int t) -> float {
+            int hq;
+            const int q0 = step_q0(t, hq);
+            const int row = min(q0 + (tid & 63), T - 1);
+            const int64_t at = (int64_t)hq * p.total + tok0 + row;
+            return tid < 64 ? p.LSE[at] * LOG2E : p.delta[at];
+        };
+        if (nsteps > 0) {
+            if (tid < 128) lsd[0][tid] = ls_load(0);
+            mbar_arrive(&ls_full[0]);
+        }
         for (int t = 0; t < nsteps; ++t) {
             const int s = t & 1;
             int hq;
             const int q0 = step_q0(t, hq);
-            {   // this step's LSE2 (threads 0..63) and Delta (64..127) of rows q0 .. q0+63
-                if (t >= 2 && !mbar_wait(&ls_free[s], ((t - 2) >> 1) & 1, status, 324)) { ok = false; break; }
-                if (tid < 128) {
-                    const int row = min(q0 + (tid & 63), T - 1);
-                    const int64_t at = (int64_t)hq * p.total + tok0 + row;
-                    lsd[s][tid] = tid < 64 ? p.LSE[at] * LOG2E : p.delta[at];
-                }
-                mbar_arrive(&ls_full[s]);
-                if (!mbar_wait(&ls_full[s], (t >> 1) & 1, status, 325)) { ok = false; break; }
-            }
+            const float ls_next = (tid < 128 && t + 1 < nsteps) ? ls_load(t + 1) : 0.f;
+            if (!mbar_wait(&ls_full[s], (t >> 1) & 1, status, 325)) { ok = false; break; }
             if (!mbar_wait(&sd_full[s], (t >> 1) & 1, status, 321)) { ok = false; break; }
             tc_fence_after();
             float sv[32], dp[32];
@@ -799,6 +805,12 @@ __global__ void __launch_bounds__(NT_BWD, 1)
                 dp[c] = pr * (dp[c] - del_c[c]);
             }
             mbar_arrive(&ls_free[s]);
+            if (t + 1 < nsteps) {
+                // buffer s ^ 1 was last read in step t - 1
+                if (t >= 1 && !mbar_wait(&ls_free[s ^ 1], ((t - 1) >> 1) & 1, status, 324)) { ok = false; break; }
+                if (tid < 128) lsd[s ^ 1][tid] = ls_next;
+                mbar_arrive(&ls_full[s ^ 1]);
+            }
             if (t >= 2 && !mbar_wait(&pd_free[s], ((t - 2) >> 1) & 1, status, 322)) { ok = false; break; }
             uint8_t* pbuf = sm + KV_P + s * PT_B;
             uint8_t* dbuf = sm + KV_DS + s * PT_B;
@@ -889,7 +901,7 @@ mw_status attn_fwd_tc(const mw_vis_layout* L, const void* vis, const void* Q, co
     if (st != MW_OK) return st;
     const unsigned grid = (unsigned)((int64_t)L->max_tiles * L->n_traj * Hq);
     count_launches(1);
-    k_attn_fwd_tc<<<grid, NTHREADS, SMEM_FWD, s>>>(tq, tk, tv, p);
+    k_attn_fwd_tc<<<grid, NT_FWD, SMEM_FWD, s>>>(tq, tk, tv, p);
     return launch_status();
 }
 
