@@ -91,6 +91,29 @@ class Clocks:
 
 # ----------------------------------------------------------------------------- workloads
 
+def replica_seed(cfg, rank):
+    """Seed of rank ``rank``'s replica: every rank scores its own independent
+    synthetic batch (weak scaling)."""
+    return 1000 * cfg + 17 + rank
+
+
+def reduce_max(x, world, device=None):
+    """Max of ``x`` over the ranks of the default process group (identity at
+    world 1): the job's time is its slowest rank's."""
+    if world <= 1:
+        return float(x)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_value(scored_per_rank, world, ms):
+    """Whole-job throughput: the units all ranks processed over the job's time."""
+    return scored_per_rank * world / (ms * 1e-3)
+
+
 def make_workload(cfg, K=None, f=None, seed_offset=0, n_traj=None):
     """Host-side inputs of one workload (pinned CPU tensors + record).
 
@@ -101,7 +124,7 @@ def make_workload(cfg, K=None, f=None, seed_offset=0, n_traj=None):
 
     import synth
     c = synth.CONFIGS[cfg]
-    g = torch.Generator().manual_seed(1000 * cfg + 17 + seed_offset)
+    g = torch.Generator().manual_seed(replica_seed(cfg, seed_offset))
     w = {"cfg": cfg}
     bf = torch.bfloat16
 
@@ -396,10 +419,7 @@ def run_gpu(args, rank, world, local_rank):
     ms = ev0.elapsed_time(ev1) / args.steps
     clk = clocks.stop()
     barrier()
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = reduce_max(ms, world, dev)
     per_call = {k: sum(a.elapsed_time(b) for a, b in v) / len(v) for k, v in step.events.items()}
 
     # e2e: pinned host inputs -> device, step, loss/metric read back
@@ -419,15 +439,11 @@ def run_gpu(args, rank, world, local_rank):
         pinned_out.copy_(out, non_blocking=True)
     e1.record(step.stream)
     torch.cuda.synchronize()
-    e2e_ms = e0.elapsed_time(e1) / args.steps
-    if world > 1:
-        t = torch.tensor([e2e_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_ms = float(t.item())
+    e2e_ms = reduce_max(e0.elapsed_time(e1) / args.steps, world, dev)
 
     if rank != 0:
         return
-    scored = step.scored() * world
+    scored = step.scored()
     flops = step.flops()
     peak_tf, hbm, peak_kind = _peaks()
     dom = max(per_call, key=per_call.get)
@@ -442,7 +458,7 @@ def run_gpu(args, rank, world, local_rank):
         v, cores, desc = cpu_sample(w, budget_s=args.cpu_seconds)
         cpu = {"value": v, "unit": "tokens/s", "cores": cores, "kind": "oracle", "sample": desc}
     line = {
-        "metric": METRIC, "value": scored / (ms * 1e-3), "unit": "tokens/s", "n_gpus": world,
+        "metric": METRIC, "value": job_value(scored, world, ms), "unit": "tokens/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": describe(w),
@@ -452,7 +468,7 @@ def run_gpu(args, rank, world, local_rank):
                      "peak_kind": f"bf16 dense burst, {peak_kind}"},
         "per_call_ms": per_call,
         "cpu_baseline": cpu,
-        "e2e": {"value": scored / (e2e_ms * 1e-3), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
+        "e2e": {"value": job_value(scored, world, e2e_ms), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
         "gpu_launches": launches,
         "clocks": clk,
