@@ -299,6 +299,21 @@ class Step:
     def scored(self):
         return int(self.w["rows"].numel()) if "rows" in self.w else self.w["record"].total
 
+    def tile_stats(self):
+        """Attention work skipped by the visibility structure, against plain
+        causal attention of the same trajectory lengths: 128x128 tiles listed
+        (non-empty) vs causal tiles, visible pairs vs causal pairs."""
+        if "record" not in self.w:
+            return None
+        import numpy as np
+        L = self.vis.layout
+        listed = int(self.vis._arr(L.off_fwd_ptr + 4 * L.n_tiles, 1, np.int32)[0])
+        causal_pairs = sum(t * (t + 1) // 2 for t in self.w["record"].seqlens)
+        return {"tiles_listed": listed, "tiles_causal": int(L.n_tri),
+                "skipped_tile_frac": 1.0 - listed / max(1, int(L.n_tri)),
+                "visible_pairs": int(self.vis.pairs_total), "causal_pairs": int(causal_pairs),
+                "visible_pair_frac": int(self.vis.pairs_total) / max(1, causal_pairs)}
+
     def flops(self):
         """Visible FLOPs per step: attention 14 P Dh Hq, LM head 8 M d V."""
         f = {}
@@ -473,6 +488,9 @@ def run_gpu(args, rank, world, local_rank):
         "gpu_launches": launches,
         "clocks": clk,
     }
+    ts = step.tile_stats()
+    if ts is not None:
+        line["attention_tiles"] = ts
     print(json.dumps(line), flush=True)
 
 
