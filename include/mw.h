@@ -233,6 +233,24 @@ mw_status mw_logprob_loss_bwd(const void* H, const void* W, const int32_t* targe
  */
 mw_status mw_check_status(const mw_vis_layout* layout, const void* vis, void* stream);
 
+/*
+ * Status of the last mw_logprob_loss_fwd / mw_logprob_loss_bwd on `ws` (same
+ * shape arguments): synchronises `stream`, then returns MW_ETIMEOUT if a
+ * tensor-core kernel gave up a bounded wait, else MW_OK. No counterpart in the
+ * paper: failure detection of this implementation.
+ */
+mw_status mw_logprob_check_status(int N, int M, int d, int Vocab, int dtype, const void* ws, void* stream);
+
+/*
+ * Self-test of the bounded-wait failure path (no counterpart in the paper):
+ * launches one kernel that waits on an mbarrier nothing arrives on, gives up
+ * after `limit_ns` (0 < limit_ns <= 1e9), records the timeout in `status`
+ * (device int32[8], overwritten) and returns. Synchronises `stream` and
+ * returns MW_ETIMEOUT when the timeout was recorded (the expected outcome);
+ * the CUDA context stays usable.
+ */
+mw_status mw_selftest_wait_timeout(int64_t limit_ns, int32_t* status, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

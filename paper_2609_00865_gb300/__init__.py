@@ -22,11 +22,13 @@ from ._lib import (  # noqa: F401
     masked_attn_fwd,
     mw_build_visibility,
     mw_build_visibility_noalloc,
+    mw_logprob_check_status,
     mw_logprob_loss_bwd,
     mw_logprob_loss_fwd,
     mw_logprob_ws,
     mw_masked_attn_bwd,
     mw_masked_attn_bwd_ws,
     mw_masked_attn_fwd,
+    mw_selftest_wait_timeout,
     mw_visibility_layout,
 )

@@ -59,6 +59,8 @@ _SIGS = {
     "mw_logprob_loss_fwd": (_I, [_P, _P, _P, _P, _I, _P, _P, _F, _F, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P]),
     "mw_logprob_loss_bwd": (_I, [_P, _P, _P, _P, _I, _I, _I, _I, _I, _P, _P, _F, _P, _P, _P]),
     "mw_check_status": (_I, [_LP, _P, _P]),
+    "mw_logprob_check_status": (_I, [_I, _I, _I, _I, _I, _P, _P]),
+    "mw_selftest_wait_timeout": (_I, [ctypes.c_int64, _P, _P]),
 }
 
 _handle = None
@@ -338,6 +340,20 @@ def mw_logprob_loss_bwd(H, W, targets, rows, lse, ws, dloss, dH, dW, stream=None
     _check(_lib().mw_logprob_loss_bwd(_ptr(H), _ptr(W), _ptr(targets), _ptr(rows), int(rows.numel()), N, d,
                                       W.shape[0], _dtype_code(H), _ptr(lse), _ptr(ws), float(dloss), _ptr(dH),
                                       _ptr(dW), _stream(stream)), "mw_logprob_loss_bwd")
+
+
+def mw_logprob_check_status(H, W, rows, ws, stream=None):
+    """Raise MWError (MW_ETIMEOUT) if a tensor-core LM-head kernel that last
+    ran on ``ws`` gave up a bounded wait; synchronises the stream."""
+    N, d = H.shape
+    _check(_lib().mw_logprob_check_status(N, int(rows.numel()), d, W.shape[0], _dtype_code(H), _ptr(ws),
+                                          _stream(stream)), "mw_logprob_check_status")
+
+
+def mw_selftest_wait_timeout(limit_ns, status, stream=None):
+    """Run the bounded-wait self-test; returns the raw status code
+    (MW_ETIMEOUT = 6 is the expected outcome). ``status``: device int32[8]."""
+    return int(_lib().mw_selftest_wait_timeout(int(limit_ns), _ptr(status), _stream(stream)))
 
 
 def logprob_loss_bwd(H, W, targets, rows, lse, ws, dloss=1.0, stream=None):

@@ -170,3 +170,18 @@ extern "C" mw_status mw_logprob_loss_bwd(const void* H, const void* W, const int
     return lm_bwd_simt(H, W, targets, rows, M, N, d, V, dtype, lse, at<float>(ws, w.g), dloss, dH, dW,
                        (cudaStream_t)stream);
 }
+
+extern "C" mw_status mw_logprob_check_status(int N, int M, int d, int V, int dtype, const void* ws, void* stream) {
+    mw_status st = lm_args(N, M, d, V, dtype);
+    if (st != MW_OK) return st;
+    if (!ws) return MW_EINVAL;
+    // only the tensor-core kernels wait on barriers; the SIMT path has no status words
+    if (!lm_tc(d, dtype)) return cuda_status(cudaStreamSynchronize((cudaStream_t)stream));
+    LmWs w = lm_ws_layout(N, M, d, V, dtype);
+    int32_t h[8];
+    if ((st = cuda_status(cudaMemcpyAsync(h, at<char>(ws, w.status), sizeof(h), cudaMemcpyDeviceToHost,
+                                          (cudaStream_t)stream))) != MW_OK)
+        return st;
+    if ((st = cuda_status(cudaStreamSynchronize((cudaStream_t)stream))) != MW_OK) return st;
+    return h[1] ? MW_ETIMEOUT : MW_OK;
+}
