@@ -38,6 +38,33 @@ def _peaks():
         return 1900.0, 6800.0, "fallback"
 
 
+# DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) per call of a
+# dominant C-ABI call, from one ncu capture of the same bench command (summaries
+# in profiles/). Reported only while the kernel source still hashes to the
+# value it had when the counters were taken.
+TRAFFIC = {
+    (4, "mw_logprob_loss_bwd"): {
+        "bytes": 121432050944 + 12028077056 + 122184046080 + 14604399872,   # dH pass + dW pass
+        "source": "paper_2609_00865_gb300/csrc/lmhead_bwd_tc.cu",
+        "sha256": "3e7fabc08aa4485f57d0fa6e95f540c317bc119f2c81ba5111a68f59b8ec7cc7",
+    },
+}
+
+
+def _traffic(cfg, call):
+    import hashlib
+    t = TRAFFIC.get((cfg, call))
+    if t is None:
+        return None
+    try:
+        with open(os.path.join(ROOT, t["source"]), "rb") as f:
+            if hashlib.sha256(f.read()).hexdigest() != t["sha256"]:
+                return None
+    except OSError:
+        return None
+    return t["bytes"]
+
+
 class Clocks:
     """nvidia-smi sampler running while the timed region runs."""
 
@@ -479,7 +506,7 @@ def run_gpu(args, rank, world, local_rank):
         "config": describe(w),
         "visible_tflops": total_tf, "visible_frac_of_peak": total_tf / peak_tf,
         "roofline": {"bound": "tensor", "kernel": dom, "achieved": achieved, "peak": peak_tf,
-                     "unit": "TFLOP/s", "frac": achieved / peak_tf, "traffic": None,
+                     "unit": "TFLOP/s", "frac": achieved / peak_tf, "traffic": _traffic(w["cfg"], dom),
                      "peak_kind": f"bf16 dense burst, {peak_kind}"},
         "per_call_ms": per_call,
         "cpu_baseline": cpu,
