@@ -239,9 +239,15 @@ __global__ void __launch_bounds__(NT_FWD, 1)
                 for (int c = 0; c < 128; ++c)
                     if (!((wd[c >> 5] >> (c & 31)) & 1u)) s[c] = -INFINITY;
             }
-            float mx = -INFINITY;
+            // row max and row sum as 8 independent partial chains (a single
+            // 128-long dependency chain per reduction bounds the warp's latency)
+            float pm[8];
 #pragma unroll
-            for (int c = 0; c < 128; ++c) mx = fmaxf(mx, s[c]);
+            for (int k = 0; k < 8; ++k) pm[k] = s[k];
+#pragma unroll
+            for (int c = 8; c < 128; ++c) pm[c & 7] = fmaxf(pm[c & 7], s[c]);
+            const float mx = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
+                                   fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
             const float mx2 = mx * p.scale_log2;
             float alpha = 1.f;
             if (mx2 > m + RESCALE_T) {
@@ -249,12 +255,13 @@ __global__ void __launch_bounds__(NT_FWD, 1)
                 m = mx2;
             }
             const float mu = (m == -INFINITY) ? 0.f : m;
-            float rs = 0.f;
+            float ps[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
             for (int c = 0; c < 128; ++c) {
                 s[c] = ex2(fmaf(s[c], p.scale_log2, -mu));
-                rs += s[c];
+                ps[c & 7] += s[c];
             }
+            const float rs = ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
             l = l * alpha + rs;
             // P_j overwrites P_{j-1}: wait for O += P_{j-1} V_{j-1} to finish
             if (j >= 1 && !mbar_wait(&o_done, (j - 1) & 1, status, 302)) { ok = false; break; }
