@@ -35,12 +35,21 @@ using namespace tc;
 constexpr int DH = 128;
 constexpr uint32_t TILE_B = 128 * DH * 2;  // one 128 x 128 bf16 tile: two [128][64] swizzled halves
 constexpr uint32_t HALF_B = TILE_B / 2;
-// Forward: warp 0 TMA, warp 1 MMA, warps 2..5 softmax (one row per thread).
-constexpr int NT_FWD = 192;
-// Backward kernels: warp 0 TMA, warp 1 MMA, warps 2..9 elementwise; two warps
-// per TMEM lane quarter split each row's columns, which hides the latency of
-// the exp / scale / pack chains that bound the kernels with one warp per quarter.
-constexpr int NT_BWD = 320;
+// Each kernel issues its tensor-core work from two threads in two warps: one
+// thread issues about one tcgen05.mma per 57-114 cycles, and a 128 x 128 x 16
+// MMA is only 64 cycles of work, so a single issuer leaves the tensor pipe idle
+// (measured: two issuing warps double the issue rate, reaching the MMA's own rate
+// at N = 128). The two streams are independent except through the barriers.
+// Forward: warp 0 TMA, warp 1 S = Q K^T, warps 2..5 softmax (one row per thread),
+// warp 6 O += P V.
+constexpr int NT_FWD = 224;
+constexpr int FWD_PV_WARP = 6;
+// Backward kernels: warp 0 TMA, warp 1 the recomputed products, warps 2..9
+// elementwise, warp 10 the gradient accumulation. Two elementwise warps per TMEM
+// lane quarter split each row's columns, which hides the latency of the exp /
+// scale / pack chains that bound the kernels with one warp per quarter.
+constexpr int NT_BWD = 352;
+constexpr int BWD_ACC_WARP = 10;
 constexpr int NEW = 256;   // elementwise threads
 constexpr float LOG2E = 1.4426950408889634f;
 constexpr float RESCALE_T = 8.0f;          // lazy-rescale threshold (log2 units)
@@ -159,8 +168,9 @@ __global__ void __launch_bounds__(NT_FWD, 1)
                 if (*(volatile int*)&abort_flag) break;
             }
         }
-    } else if (warp == 1) {
-        // ------------------------------------------------------------ MMA issuer
+    } else if (warp == 1 || warp == FWD_PV_WARP) {
+        // ------------------------------------------------------------ MMA issuers
+        // warp 1: S_j = Q K_j^T; warp FWD_PV_WARP: O += P_t V_t
         if (lane == 0) {
             const uint32_t iS = idesc_bf16(128, 128, 0, 0);   // S = Q K^T: both K-major
             const uint32_t iO = idesc_bf16(128, 128, 0, 1);   // O += P V: V is MN-major
@@ -178,19 +188,22 @@ __global__ void __launch_bounds__(NT_FWD, 1)
                 mma_commit(&o_done);
                 return true;
             };
-            for (int j = 0; ok && j < n; ++j) {
-                const int s = j & 1;
-                if (!mbar_wait(&k_full[s], (j >> 1) & 1, status, 204)) { ok = false; break; }
-                if (j >= 2 && !mbar_wait(&s_free[s], ((j - 2) >> 1) & 1, status, 205)) { ok = false; break; }
-                tc_fence_after();
-                const uint32_t kb = sk + s * TILE_B;
+            if (warp == 1) {
+                for (int j = 0; ok && j < n; ++j) {
+                    const int s = j & 1;
+                    if (!mbar_wait(&k_full[s], (j >> 1) & 1, status, 204)) { ok = false; break; }
+                    if (j >= 2 && !mbar_wait(&s_free[s], ((j - 2) >> 1) & 1, status, 205)) { ok = false; break; }
+                    tc_fence_after();
+                    const uint32_t kb = sk + s * TILE_B;
 #pragma unroll
-                for (int ks = 0; ks < 8; ++ks) mma_ss(tmem + TM_S0 + s * 128, kmaj(sq, ks), kmaj(kb, ks), iS, ks > 0);
-                mma_commit(&k_empty[s]);
-                mma_commit(&s_full[s]);
-                if (j >= 1 && !pv(j - 1)) { ok = false; break; }
+                    for (int ks = 0; ks < 8; ++ks)
+                        mma_ss(tmem + TM_S0 + s * 128, kmaj(sq, ks), kmaj(kb, ks), iS, ks > 0);
+                    mma_commit(&k_empty[s]);
+                    mma_commit(&s_full[s]);
+                }
+            } else {
+                for (int t = 0; ok && t < n; ++t) ok = pv(t);
             }
-            if (ok && n > 0) ok = pv(n - 1);
             if (!ok) abort_flag = 1;
         }
     } else {
@@ -432,7 +445,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
                 load_tile(sm + DQ_K + s * TILE_B, &tmK, &k_full[s], kvh, row);
             }
         }
-    } else if (warp == 1) {
+    } else if (warp == 1 || warp == BWD_ACC_WARP) {
         if (lane == 0) {
             const uint32_t iKK = idesc_bf16(128, 128, 0, 0);  // both operands K-major
             const uint32_t iMN = idesc_bf16(128, 128, 0, 1);  // B MN-major
@@ -475,11 +488,11 @@ __global__ void __launch_bounds__(NT_BWD, 1)
                 mma_commit(&dq_done);
                 return true;
             };
-            if (ok && n > 0) ok = issue_s(0) && issue_dp(0);
-            for (int j = 0; ok && j < n; ++j) {
-                if (j + 1 < n && !issue_s(j + 1)) { ok = false; break; }
-                if (!issue_dq(j)) { ok = false; break; }
-                if (j + 1 < n && !issue_dp(j + 1)) { ok = false; break; }
+            if (warp == 1) {
+                for (int j = 0; ok && j < n; ++j) ok = issue_s(j) && issue_dp(j);
+            } else {
+                // dQ's K-stage release also covers S_j: dS_j exists only once S_j is done
+                for (int j = 0; ok && j < n; ++j) ok = issue_dq(j);
             }
         }
     } else {
@@ -711,7 +724,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
                 tma_load_3d(dst + HT_B + HT_HALF, &tmDO, &qd_full[s], 64, hq, (int)(tok0 + q0));
             }
         }
-    } else if (warp == 1) {
+    } else if (warp == 1 || warp == BWD_ACC_WARP) {
         if (lane == 0) {
             const uint32_t iSD = idesc_bf16(128, 64, 0, 0);
             const uint32_t iAC = idesc_bf16(128, 128, 0, 1);
@@ -747,10 +760,12 @@ __global__ void __launch_bounds__(NT_BWD, 1)
                 mma_commit(&pd_free[s]);
                 return true;
             };
-            if (ok && nsteps > 0) ok = issue_sd(0);
-            for (int t = 0; ok && t < nsteps; ++t) {
-                if (t + 1 < nsteps && !issue_sd(t + 1)) { ok = false; break; }
-                if (!issue_acc(t)) { ok = false; break; }
+            if (warp == 1) {
+                for (int t = 0; ok && t < nsteps; ++t) ok = issue_sd(t);
+            } else {
+                // the Q/dO stage release also covers S^T_t, dP^T_t: P^T_t, dS^T_t
+                // exist only once those are done
+                for (int t = 0; ok && t < nsteps; ++t) ok = issue_acc(t);
             }
         }
     } else {
