@@ -224,15 +224,15 @@ __global__ void __launch_bounds__(NT_FWD, 1)
             if (!mbar_wait(&s_full[j & 1], (j >> 1) & 1, status, 301)) { ok = false; break; }
             tc_fence_after();
             float s[128];
-            {
-                uint32_t rr[32];
+            {   // all four loads in flight before one wait
+                uint32_t rr[4][32];
 #pragma unroll
-                for (int c = 0; c < 4; ++c) {
-                    tmem_ld32(lane_base + TM_S0 + (j & 1) * 128 + c * 32, rr);
-                    tmem_wait_ld();
+                for (int c = 0; c < 4; ++c) tmem_ld32(lane_base + TM_S0 + (j & 1) * 128 + c * 32, rr[c]);
+                tmem_wait_ld();
 #pragma unroll
-                    for (int x = 0; x < 32; ++x) s[c * 32 + x] = __uint_as_float(rr[x]);
-                }
+                for (int c = 0; c < 4; ++c)
+#pragma unroll
+                    for (int x = 0; x < 32; ++x) s[c * 32 + x] = __uint_as_float(rr[c][x]);
             }
             tc_fence_before();
             mbar_arrive(&s_free[j & 1]);
@@ -515,15 +515,15 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             if (!mbar_wait(&s_full[j & 1], (j >> 1) & 1, status, 311)) { ok = false; break; }
             tc_fence_after();
             float s[64];
-            {
-                uint32_t rr[32];
+            {   // both loads in flight before one wait
+                uint32_t rr[2][32];
 #pragma unroll
-                for (int c = 0; c < 2; ++c) {
-                    tmem_ld32(lane_base + TM_S0 + (j & 1) * 128 + (2 * ch + c) * 32, rr);
-                    tmem_wait_ld();
+                for (int c = 0; c < 2; ++c) tmem_ld32(lane_base + TM_S0 + (j & 1) * 128 + (2 * ch + c) * 32, rr[c]);
+                tmem_wait_ld();
 #pragma unroll
-                    for (int x = 0; x < 32; ++x) s[c * 32 + x] = __uint_as_float(rr[x]);
-                }
+                for (int c = 0; c < 2; ++c)
+#pragma unroll
+                    for (int x = 0; x < 32; ++x) s[c * 32 + x] = __uint_as_float(rr[c][x]);
             }
             tc_fence_before();
             mbar_arrive(&s_free[j & 1]);
@@ -548,16 +548,16 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             tc_fence_after();
             // dS_j overwrites dS_{j-1}: wait until dQ += dS_{j-1} K_{j-1} is done
             if (j >= 1 && !mbar_wait(&dq_done, (j - 1) & 1, status, 313)) { ok = false; break; }
+            uint32_t dpr[2][32];   // both dP loads in flight before one wait
+#pragma unroll
+            for (int cc = 0; cc < 2; ++cc) tmem_ld32(lane_base + TM_DP + (2 * ch + cc) * 32, dpr[cc]);
+            tmem_wait_ld();
+            tc_fence_before();
+            mbar_arrive(&dp_free);
 #pragma unroll
             for (int cc = 0; cc < 2; ++cc) {
                 const int c = 2 * ch + cc;   // 32-column chunk of the row
-                uint32_t dp[32];
-                tmem_ld32(lane_base + TM_DP + c * 32, dp);
-                tmem_wait_ld();
-                if (cc == 1) {
-                    tc_fence_before();
-                    mbar_arrive(&dp_free);
-                }
+                const uint32_t* dp = dpr[cc];
 #pragma unroll
                 for (int x = 0; x < 4; ++x) {
                     uint4 pk;
@@ -802,16 +802,16 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             if (!mbar_wait(&sd_full[s], (t >> 1) & 1, status, 321)) { ok = false; break; }
             tc_fence_after();
             float sv[32], dp[32];
-            {
-                uint32_t rr[32];
-                tmem_ld32(lane_base + TM_ST + s * 64 + ch * 32, rr);
+            {   // both loads in flight before one wait
+                uint32_t ra[32], rb[32];
+                tmem_ld32(lane_base + TM_ST + s * 64 + ch * 32, ra);
+                tmem_ld32(lane_base + TM_DPT + s * 64 + ch * 32, rb);
                 tmem_wait_ld();
 #pragma unroll
-                for (int x = 0; x < 32; ++x) sv[x] = __uint_as_float(rr[x]);
-                tmem_ld32(lane_base + TM_DPT + s * 64 + ch * 32, rr);
-                tmem_wait_ld();
-#pragma unroll
-                for (int x = 0; x < 32; ++x) dp[x] = __uint_as_float(rr[x]);
+                for (int x = 0; x < 32; ++x) {
+                    sv[x] = __uint_as_float(ra[x]);
+                    dp[x] = __uint_as_float(rb[x]);
+                }
             }
             tc_fence_before();
             mbar_arrive(&sd_free[s]);
