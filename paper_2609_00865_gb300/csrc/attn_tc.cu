@@ -648,12 +648,14 @@ __global__ void __launch_bounds__(NT_BWD, 1)
     __shared__ __align__(8) uint64_t kv_full, qd_full[QD_ST], qd_empty[QD_ST], sd_full[2], sd_free[2], pd_full[2],
         pd_free[2], ls_full[2], ls_free[2];
     __shared__ uint32_t tmem_base;
-    __shared__ float lsd[2][128];   // per step: LSE2 of the 64 rows, then Delta of the 64 rows
+    __shared__ __align__(16) float lsd[2][128];   // per step: LSE2 of the 64 rows, then Delta of the 64 rows
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int grp = p.Hq / p.Hkv;
-    const int kvh = blockIdx.x % p.Hkv;
-    const int r = blockIdx.x / p.Hkv;
+    // KV head outermost: the CTAs resident at one time share one head's Q / dO
+    // (whose working set then fits in L2)
+    const int kvh = blockIdx.x / (p.max_tiles * p.n_traj);
+    const int r = blockIdx.x % (p.max_tiles * p.n_traj);
     const int kt = r / p.n_traj;
     const int b = r % p.n_traj;
     const VisView& v = p.v;
@@ -817,8 +819,19 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             mbar_arrive(&sd_free[s]);
             // visible columns [lo, hi) of this warp's 32
             const int lo = max(jk, q0 + 32 * ch) - q0 - 32 * ch, hi = min(iend, q0 + 64) - q0 - 32 * ch;
-            const float* lse_c = lsd[s] + 32 * ch;
-            const float* del_c = lsd[s] + 64 + 32 * ch;
+            // this warp's 32 LSE2 and Delta values: broadcast 16-byte loads into registers
+            float lse_c[32], del_c[32];
+            {
+                const float4* l4 = reinterpret_cast<const float4*>(lsd[s] + 32 * ch);
+                const float4* d4 = reinterpret_cast<const float4*>(lsd[s] + 64 + 32 * ch);
+#pragma unroll
+                for (int q = 0; q < 8; ++q) {
+                    const float4 a = l4[q], d = d4[q];
+                    lse_c[4 * q] = a.x; lse_c[4 * q + 1] = a.y; lse_c[4 * q + 2] = a.z; lse_c[4 * q + 3] = a.w;
+                    del_c[4 * q] = d.x; del_c[4 * q + 1] = d.y; del_c[4 * q + 2] = d.z; del_c[4 * q + 3] = d.w;
+                }
+            }
+            mbar_arrive(&ls_free[s]);
 #pragma unroll
             for (int c = 0; c < 32; ++c) {
                 const bool vis = c >= lo && c < hi;
@@ -826,7 +839,6 @@ __global__ void __launch_bounds__(NT_BWD, 1)
                 sv[c] = pr;
                 dp[c] = pr * (dp[c] - del_c[c]);
             }
-            mbar_arrive(&ls_free[s]);
             if (t + 1 < nsteps) {
                 // buffer s ^ 1 was last read in step t - 1
                 if (t >= 1 && !mbar_wait(&ls_free[s ^ 1], ((t - 1) >> 1) & 1, status, 324)) { ok = false; break; }
