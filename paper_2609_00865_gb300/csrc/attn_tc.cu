@@ -58,8 +58,7 @@ constexpr float RESCALE_T = 8.0f;          // lazy-rescale threshold (log2 units
 constexpr uint32_t SM_Q = 0;
 constexpr uint32_t SM_K = SM_Q + TILE_B;
 constexpr uint32_t SM_V = SM_K + 2 * TILE_B;
-constexpr uint32_t SM_P = SM_V + 2 * TILE_B;
-constexpr uint32_t SM_TOTAL = SM_P + TILE_B;
+constexpr uint32_t SM_TOTAL = SM_V + 2 * TILE_B;   // P lives in TMEM
 constexpr uint32_t SMEM_FWD = SM_TOTAL + 1024;
 
 // TMEM columns
@@ -101,7 +100,7 @@ __global__ void __launch_bounds__(NT_FWD, 1)
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~uintptr_t(1023));
     __shared__ __align__(8) uint64_t q_full, k_full[2], k_empty[2], v_full[2], v_empty[2], s_full[2], s_free[2],
-        p_full, o_done;
+        p_full[2], o_done;
     __shared__ uint32_t tmem_base;
     __shared__ int abort_flag;
 
@@ -131,9 +130,9 @@ __global__ void __launch_bounds__(NT_FWD, 1)
             mbar_init(&v_full[s], 1);
             mbar_init(&v_empty[s], 1);
             mbar_init(&s_full[s], 1);
-            mbar_init(&s_free[s], 128);
+            mbar_init(&s_free[s], 1);     // PV's completion: P lives in the S buffer until then
+            mbar_init(&p_full[s], 128);   // per S buffer
         }
-        mbar_init(&p_full, 128);
         mbar_init(&o_done, 1);
         abort_flag = 0;
         fence_mbar_init();
@@ -174,17 +173,20 @@ __global__ void __launch_bounds__(NT_FWD, 1)
         if (lane == 0) {
             const uint32_t iS = idesc_bf16(128, 128, 0, 0);   // S = Q K^T: both K-major
             const uint32_t iO = idesc_bf16(128, 128, 0, 1);   // O += P V: V is MN-major
-            const uint32_t sq = smem_u32(sm + SM_Q), sk = smem_u32(sm + SM_K), sv = smem_u32(sm + SM_V),
-                           sp = smem_u32(sm + SM_P);
+            const uint32_t sq = smem_u32(sm + SM_Q), sk = smem_u32(sm + SM_K), sv = smem_u32(sm + SM_V);
             bool ok = mbar_wait(&q_full, 0, status, 201);
+            // O += P_t V_t with P_t (bf16, two keys per 32-bit column) read from
+            // the first 64 columns of S buffer t & 1
             auto pv = [&](int t) -> bool {
-                if (!mbar_wait(&p_full, t & 1, status, 202)) return false;
+                if (!mbar_wait(&p_full[t & 1], (t >> 1) & 1, status, 202)) return false;
                 if (!mbar_wait(&v_full[t & 1], (t >> 1) & 1, status, 203)) return false;
                 tc_fence_after();
                 const uint32_t vb = sv + (t & 1) * TILE_B;
+                const uint32_t pa = tmem + TM_S0 + (t & 1) * 128;
 #pragma unroll
-                for (int ks = 0; ks < 8; ++ks) mma_ss(tmem + TM_O, kmaj(sp, ks), mnmaj(vb, ks), iO, (t > 0 || ks > 0));
+                for (int ks = 0; ks < 8; ++ks) mma_ts(tmem + TM_O, pa + 8 * ks, mnmaj(vb, ks), iO, (t > 0 || ks > 0));
                 mma_commit(&v_empty[t & 1]);
+                mma_commit(&s_free[t & 1]);
                 mma_commit(&o_done);
                 return true;
             };
@@ -215,7 +217,6 @@ __global__ void __launch_bounds__(NT_FWD, 1)
         const int seg = v.seg[tok0 + ie];
         const uint4* km = reinterpret_cast<const uint4*>(v.keymask) + v.traj_km[b] + (int64_t)seg * nt;
         const uint32_t lane_base = tmem + ((uint32_t)(qw * 32) << 16);
-        uint8_t* prow = sm + SM_P;
         float m = -INFINITY, l = 0.f;
         bool ok = true;
         for (int j = 0; j < n; ++j) {
@@ -234,8 +235,6 @@ __global__ void __launch_bounds__(NT_FWD, 1)
 #pragma unroll
                     for (int x = 0; x < 32; ++x) s[c * 32 + x] = __uint_as_float(rr[c][x]);
             }
-            tc_fence_before();
-            mbar_arrive(&s_free[j & 1]);
             if (cls != MW_TILE_FULL || kt == qt) {
                 uint4 w = km[kt];
                 uint32_t wd[4] = {w.x, w.y, w.z, w.w};
@@ -276,20 +275,23 @@ __global__ void __launch_bounds__(NT_FWD, 1)
             }
             const float rs = ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
             l = l * alpha + rs;
-            // P_j overwrites P_{j-1}: wait for O += P_{j-1} V_{j-1} to finish
-            if (j >= 1 && !mbar_wait(&o_done, (j - 1) & 1, status, 302)) { ok = false; break; }
-            tc_fence_after();
+            // P_j (bf16 pairs) over the first 64 columns of its own S buffer; the
+            // PV MMA reads it from there, so P never touches shared memory
+            {
+                const uint32_t pt = lane_base + TM_S0 + (j & 1) * 128;
 #pragma unroll
-            for (int c = 0; c < 16; ++c) {
-                uint4 pk;
-                pk.x = pack_bf16(s[8 * c + 0], s[8 * c + 1]);
-                pk.y = pack_bf16(s[8 * c + 2], s[8 * c + 3]);
-                pk.z = pack_bf16(s[8 * c + 4], s[8 * c + 5]);
-                pk.w = pack_bf16(s[8 * c + 6], s[8 * c + 7]);
-                *reinterpret_cast<uint4*>(prow + (c >> 3) * HALF_B + sw128_off(rl, c & 7)) = pk;
+                for (int q = 0; q < 4; ++q) {
+                    uint32_t pk[16];
+#pragma unroll
+                    for (int x = 0; x < 16; ++x) pk[x] = pack_bf16(s[32 * q + 2 * x], s[32 * q + 2 * x + 1]);
+                    tmem_st16(pt + 16 * q, pk);
+                }
+                tmem_wait_st();
             }
             // O was last written by PV_{j-1}; rescale it when the max moved
             if (j >= 1 && __any_sync(0xffffffffu, alpha != 1.f)) {
+                if (!mbar_wait(&o_done, (j - 1) & 1, status, 302)) { ok = false; break; }
+                tc_fence_after();
                 uint32_t o[32];
 #pragma unroll
                 for (int c = 0; c < 4; ++c) {
@@ -305,9 +307,8 @@ __global__ void __launch_bounds__(NT_FWD, 1)
                 }
                 tmem_wait_st();
             }
-            fence_async_smem();
             tc_fence_before();
-            mbar_arrive(&p_full);
+            mbar_arrive(&p_full[j & 1]);
         }
         // epilogue: O / l, LSE (natural log)
         if (ok && n > 0 && mbar_wait(&o_done, (n - 1) & 1, status, 303)) {
