@@ -358,7 +358,7 @@ constexpr uint32_t DQ_DO = DQ_Q + TILE_B;
 constexpr uint32_t DQ_K = DQ_DO + TILE_B;
 constexpr uint32_t DQ_V = DQ_K + 2 * TILE_B;
 constexpr uint32_t DQ_DS = DQ_V + 2 * TILE_B;
-constexpr uint32_t SMEM_DQ = DQ_DS + TILE_B + 1024;
+constexpr uint32_t SMEM_DQ = DQ_DS + 1024;   // dS lives in TMEM
 constexpr uint32_t TM_DP = 256, TM_DQ = 384;
 
 struct BwdParams {
@@ -379,7 +379,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~uintptr_t(1023));
     __shared__ __align__(8) uint64_t q_full, k_full[2], k_empty[2], v_full[2], v_empty[2], s_full[2], s_free[2],
-        dp_full, dp_free, ds_full, dq_done;
+        dp_full, dp_free, ds_full[2], dq_done;
     __shared__ uint32_t tmem_base;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -407,11 +407,11 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             mbar_init(&v_full[s], 1);
             mbar_init(&v_empty[s], 1);
             mbar_init(&s_full[s], 1);
-            mbar_init(&s_free[s], NEW);
+            mbar_init(&s_free[s], 1);     // dQ's completion: dS lives in the S buffer until then
+            mbar_init(&ds_full[s], NEW);  // per S buffer
         }
         mbar_init(&dp_full, 1);
         mbar_init(&dp_free, NEW);
-        mbar_init(&ds_full, NEW);
         mbar_init(&dq_done, 1);
         fence_mbar_init();
     }
@@ -451,7 +451,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             const uint32_t iKK = idesc_bf16(128, 128, 0, 0);  // both operands K-major
             const uint32_t iMN = idesc_bf16(128, 128, 0, 1);  // B MN-major
             const uint32_t sq = smem_u32(sm + DQ_Q), sdo = smem_u32(sm + DQ_DO), sk = smem_u32(sm + DQ_K),
-                           sv = smem_u32(sm + DQ_V), sds = smem_u32(sm + DQ_DS);
+                           sv = smem_u32(sm + DQ_V);
             bool ok = mbar_wait(&q_full, 0, status, 211);
             // S_j (needs K_j and a free S buffer)
             auto issue_s = [&](int j) -> bool {
@@ -478,14 +478,18 @@ __global__ void __launch_bounds__(NT_BWD, 1)
                 mma_commit(&dp_full);
                 return true;
             };
-            // dQ += dS_t K_t
+            // dQ += dS_t K_t, dS_t (bf16 pairs) read from TMEM: keys 0..63 in
+            // columns 0..31 and keys 64..127 in columns 64..95 of S buffer t & 1
             auto issue_dq = [&](int t) -> bool {
-                if (!mbar_wait(&ds_full, t & 1, status, 216)) return false;
+                if (!mbar_wait(&ds_full[t & 1], (t >> 1) & 1, status, 216)) return false;
                 tc_fence_after();
+                const uint32_t da = tmem + TM_S0 + (t & 1) * 128;
 #pragma unroll
                 for (int ks = 0; ks < 8; ++ks)
-                    mma_ss(tmem + TM_DQ, kmaj(sds, ks), mnmaj(sk + (t & 1) * TILE_B, ks), iMN, (t > 0 || ks > 0));
+                    mma_ts(tmem + TM_DQ, da + (ks < 4 ? 8 * ks : 64 + 8 * (ks - 4)), mnmaj(sk + (t & 1) * TILE_B, ks),
+                           iMN, (t > 0 || ks > 0));
                 mma_commit(&k_empty[t & 1]);
+                mma_commit(&s_free[t & 1]);
                 mma_commit(&dq_done);
                 return true;
             };
@@ -506,7 +510,6 @@ __global__ void __launch_bounds__(NT_BWD, 1)
         const int seg = v.seg[tok0 + ie];
         const uint4* km = reinterpret_cast<const uint4*>(v.keymask) + v.traj_km[b] + (int64_t)seg * nt;
         const uint32_t lane_base = tmem + ((uint32_t)(qw * 32) << 16);
-        uint8_t* dsrow = sm + DQ_DS;
         const float lse2 = p.LSE[(int64_t)h * p.total + tok0 + ie] * LOG2E;
         const float dl = p.delta[(int64_t)h * p.total + tok0 + ie];
         bool ok = true;
@@ -526,8 +529,6 @@ __global__ void __launch_bounds__(NT_BWD, 1)
 #pragma unroll
                     for (int x = 0; x < 32; ++x) s[c * 32 + x] = __uint_as_float(rr[c][x]);
             }
-            tc_fence_before();
-            mbar_arrive(&s_free[j & 1]);
             uint32_t wd[4] = {0xffffffffu, 0xffffffffu, 0xffffffffu, 0xffffffffu};
             if (cls != MW_TILE_FULL || kt == qt) {
                 uint4 w = km[kt];
@@ -547,37 +548,30 @@ __global__ void __launch_bounds__(NT_BWD, 1)
                 s[c] = (((c < 32 ? w0 : w1) >> (c & 31)) & 1u) ? ex2(fmaf(s[c], p.scale_log2, -lse2)) : 0.f;
             if (!mbar_wait(&dp_full, j & 1, status, 312)) { ok = false; break; }
             tc_fence_after();
-            // dS_j overwrites dS_{j-1}: wait until dQ += dS_{j-1} K_{j-1} is done
-            if (j >= 1 && !mbar_wait(&dq_done, (j - 1) & 1, status, 313)) { ok = false; break; }
             uint32_t dpr[2][32];   // both dP loads in flight before one wait
 #pragma unroll
             for (int cc = 0; cc < 2; ++cc) tmem_ld32(lane_base + TM_DP + (2 * ch + cc) * 32, dpr[cc]);
             tmem_wait_ld();
             tc_fence_before();
             mbar_arrive(&dp_free);
+            // dS (bf16 pairs) over the first 32 of this warp's own 64 S columns,
+            // which only this thread has read
+            const uint32_t dst = lane_base + TM_S0 + (j & 1) * 128 + 64 * ch;
 #pragma unroll
             for (int cc = 0; cc < 2; ++cc) {
-                const int c = 2 * ch + cc;   // 32-column chunk of the row
                 const uint32_t* dp = dpr[cc];
+                uint32_t pk[16];
 #pragma unroll
-                for (int x = 0; x < 4; ++x) {
-                    uint4 pk;
-                    const int c0 = cc * 32 + 8 * x;
-                    pk.x = pack_bf16(s[c0 + 0] * (__uint_as_float(dp[8 * x + 0]) - dl),
-                                     s[c0 + 1] * (__uint_as_float(dp[8 * x + 1]) - dl));
-                    pk.y = pack_bf16(s[c0 + 2] * (__uint_as_float(dp[8 * x + 2]) - dl),
-                                     s[c0 + 3] * (__uint_as_float(dp[8 * x + 3]) - dl));
-                    pk.z = pack_bf16(s[c0 + 4] * (__uint_as_float(dp[8 * x + 4]) - dl),
-                                     s[c0 + 5] * (__uint_as_float(dp[8 * x + 5]) - dl));
-                    pk.w = pack_bf16(s[c0 + 6] * (__uint_as_float(dp[8 * x + 6]) - dl),
-                                     s[c0 + 7] * (__uint_as_float(dp[8 * x + 7]) - dl));
-                    const int chunk = c * 4 + x;   // 16-byte chunk 0..15 of the row
-                    *reinterpret_cast<uint4*>(dsrow + (chunk >> 3) * HALF_B + sw128_off(rl, chunk & 7)) = pk;
+                for (int x = 0; x < 16; ++x) {
+                    const int c0 = cc * 32 + 2 * x;
+                    pk[x] = pack_bf16(s[c0] * (__uint_as_float(dp[2 * x]) - dl),
+                                      s[c0 + 1] * (__uint_as_float(dp[2 * x + 1]) - dl));
                 }
+                tmem_st16(dst + 16 * cc, pk);
             }
-            fence_async_smem();
+            tmem_wait_st();
             tc_fence_before();
-            mbar_arrive(&ds_full);
+            mbar_arrive(&ds_full[j & 1]);
         }
         if (ok && n > 0 && mbar_wait(&dq_done, (n - 1) & 1, status, 314)) {
             tc_fence_after();
