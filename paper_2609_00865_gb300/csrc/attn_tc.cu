@@ -349,8 +349,9 @@ __global__ void __launch_bounds__(NT_FWD, 1)
 // dQ kernel (Q-stationary, one CTA per (q-tile, q-head), same item order as the
 // forward). Per listed k-tile j:
 //   S_j = Q K_j^T (TMEM, double-buffered), dP_j = dO V_j^T (TMEM, single),
-//   P = exp2(S c - LSE2) on visible pairs, dS = P (dP - Delta) -> bf16 smem,
-//   dQ += dS K_j (TMEM accumulator; K_j read as an MN-major operand).
+//   P = exp2(S c - LSE2) on visible pairs, dS = P (dP - Delta) -> bf16 over
+//   its own S buffer in TMEM, dQ += dS K_j (dS a TMEM operand, K_j MN-major in
+//   smem; TMEM accumulator).
 // dQ = scale * accumulator, written as bf16. No atomics: each dQ row is owned
 // by one CTA.
 constexpr uint32_t DQ_Q = 0;
@@ -610,20 +611,17 @@ __global__ void __launch_bounds__(NT_BWD, 1)
 // (last q-tile first) x the group's query heads x two 64-row halves:
 //   S^T = K Q^T, dP^T = V dO^T   (M=128 keys, N=64 rows; TMEM, double-buffered)
 //   P^T = exp2(S^T c - LSE2_i), dS^T = P^T (dP^T - Delta_i) on visible pairs,
-//   written as bf16 [128 keys][64 rows] (double-buffered smem)
-//   dV += P^T dO, dK += dS^T Q   (dO, Q read as MN-major operands)
+//   written as bf16 over their own S^T / dP^T TMEM buffers
+//   dV += P^T dO, dK += dS^T Q   (P^T, dS^T TMEM operands; dO, Q MN-major in smem)
 // The rows that see key j form the interval [j, min(omega(j), T)), so the mask
 // is two compares per element.
 constexpr uint32_t HT_B = 64 * DH * 2;     // 64-row half tile: two [64][64] swizzled halves
 constexpr uint32_t HT_HALF = HT_B / 2;
-constexpr uint32_t PT_B = 128 * 64 * 2;    // [128 keys][64 rows] bf16
 constexpr uint32_t KV_K = 0;
 constexpr uint32_t KV_V = KV_K + TILE_B;
-constexpr int QD_ST = 3;                           // (Q half, dO half) stages
+constexpr int QD_ST = 5;                           // (Q half, dO half) stages
 constexpr uint32_t KV_Q = KV_V + TILE_B;
-constexpr uint32_t KV_P = KV_Q + QD_ST * 2 * HT_B; // 2 buffers of P^T
-constexpr uint32_t KV_DS = KV_P + 2 * PT_B;        // 2 buffers of dS^T
-constexpr uint32_t SMEM_KV = KV_DS + 2 * PT_B + 1024;
+constexpr uint32_t SMEM_KV = KV_Q + QD_ST * 2 * HT_B + 1024;   // P^T, dS^T live in TMEM
 constexpr uint32_t TM_ST = 0, TM_DPT = 128, TM_DV = 256, TM_DK = 384;
 
 // K-major descriptor, k-step ks, of a 64-row half tile ([64][128] as two [64][64]).
@@ -641,7 +639,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~uintptr_t(1023));
     __shared__ __align__(8) uint64_t kv_full, qd_full[QD_ST], qd_empty[QD_ST], sd_full[2], sd_free[2], pd_full[2],
-        pd_free[2], ls_full[2], ls_free[2];
+        ls_full[2], ls_free[2];
     __shared__ uint32_t tmem_base;
     __shared__ __align__(16) float lsd[2][128];   // per step: LSE2 of the 64 rows, then Delta of the 64 rows
 
@@ -673,9 +671,8 @@ __global__ void __launch_bounds__(NT_BWD, 1)
         }
         for (int s = 0; s < 2; ++s) {
             mbar_init(&sd_full[s], 1);
-            mbar_init(&sd_free[s], NEW);
+            mbar_init(&sd_free[s], 1);     // the accumulation's completion: P^T / dS^T live there until then
             mbar_init(&pd_full[s], NEW);
-            mbar_init(&pd_free[s], 1);
             mbar_init(&ls_full[s], NEW);
             mbar_init(&ls_free[s], NEW);
         }
@@ -725,8 +722,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
         if (lane == 0) {
             const uint32_t iSD = idesc_bf16(128, 64, 0, 0);
             const uint32_t iAC = idesc_bf16(128, 128, 0, 1);
-            const uint32_t sk = smem_u32(sm + KV_K), sv = smem_u32(sm + KV_V), sq = smem_u32(sm + KV_Q),
-                           spb = smem_u32(sm + KV_P), sdb = smem_u32(sm + KV_DS);
+            const uint32_t sk = smem_u32(sm + KV_K), sv = smem_u32(sm + KV_V), sq = smem_u32(sm + KV_Q);
             bool ok = mbar_wait(&kv_full, 0, status, 221);
             auto issue_sd = [&](int t) -> bool {
                 const int s = t & 1, qs = t % QD_ST;
@@ -746,15 +742,19 @@ __global__ void __launch_bounds__(NT_BWD, 1)
                 if (!mbar_wait(&pd_full[s], (t >> 1) & 1, status, 224)) return false;
                 tc_fence_after();
                 const uint32_t qb = sq + qs * 2 * HT_B, db = qb + HT_B;
-                const uint32_t pb = spb + s * PT_B, dsb = sdb + s * PT_B;
+                // P^T, dS^T (bf16 pairs of query rows) in TMEM: rows 0..31 of the
+                // half-step in columns 0..15, rows 32..63 in columns 32..47 of
+                // their S^T / dP^T buffer
 #pragma unroll
                 for (int ks = 0; ks < 4; ++ks)
-                    mma_ss(tmem + TM_DV, sdesc_sw128(pb + ks * 32, 16, 1024), mnmaj_ht(db, ks), iAC, (t > 0 || ks > 0));
+                    mma_ts(tmem + TM_DV, tmem + TM_ST + s * 64 + 32 * (ks >> 1) + 8 * (ks & 1), mnmaj_ht(db, ks), iAC,
+                           (t > 0 || ks > 0));
 #pragma unroll
                 for (int ks = 0; ks < 4; ++ks)
-                    mma_ss(tmem + TM_DK, sdesc_sw128(dsb + ks * 32, 16, 1024), mnmaj_ht(qb, ks), iAC, (t > 0 || ks > 0));
+                    mma_ts(tmem + TM_DK, tmem + TM_DPT + s * 64 + 32 * (ks >> 1) + 8 * (ks & 1), mnmaj_ht(qb, ks), iAC,
+                           (t > 0 || ks > 0));
                 mma_commit(&qd_empty[qs]);
-                mma_commit(&pd_free[s]);
+                mma_commit(&sd_free[s]);
                 return true;
             };
             if (warp == 1) {
@@ -810,8 +810,6 @@ __global__ void __launch_bounds__(NT_BWD, 1)
                     dp[x] = __uint_as_float(rb[x]);
                 }
             }
-            tc_fence_before();
-            mbar_arrive(&sd_free[s]);
             // visible columns [lo, hi) of this warp's 32
             const int lo = max(jk, q0 + 32 * ch) - q0 - 32 * ch, hi = min(iend, q0 + 64) - q0 - 32 * ch;
             // this warp's 32 LSE2 and Delta values: broadcast 16-byte loads into registers
@@ -840,28 +838,22 @@ __global__ void __launch_bounds__(NT_BWD, 1)
                 if (tid < 128) lsd[s ^ 1][tid] = ls_next;
                 mbar_arrive(&ls_full[s ^ 1]);
             }
-            if (t >= 2 && !mbar_wait(&pd_free[s], ((t - 2) >> 1) & 1, status, 322)) { ok = false; break; }
-            uint8_t* pbuf = sm + KV_P + s * PT_B;
-            uint8_t* dbuf = sm + KV_DS + s * PT_B;
+            {   // P^T, dS^T (bf16 pairs) over the first 16 of this warp's own 32
+                // columns of the S^T / dP^T buffers, which only this thread has read
+                uint32_t pa[16], pd[16];
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                uint4 a, d;
-                a.x = pack_bf16(sv[8 * c + 0], sv[8 * c + 1]);
-                a.y = pack_bf16(sv[8 * c + 2], sv[8 * c + 3]);
-                a.z = pack_bf16(sv[8 * c + 4], sv[8 * c + 5]);
-                a.w = pack_bf16(sv[8 * c + 6], sv[8 * c + 7]);
-                d.x = pack_bf16(dp[8 * c + 0], dp[8 * c + 1]);
-                d.y = pack_bf16(dp[8 * c + 2], dp[8 * c + 3]);
-                d.z = pack_bf16(dp[8 * c + 4], dp[8 * c + 5]);
-                d.w = pack_bf16(dp[8 * c + 6], dp[8 * c + 7]);
-                *reinterpret_cast<uint4*>(pbuf + sw128_off(rl, 4 * ch + c)) = a;
-                *reinterpret_cast<uint4*>(dbuf + sw128_off(rl, 4 * ch + c)) = d;
+                for (int x = 0; x < 16; ++x) {
+                    pa[x] = pack_bf16(sv[2 * x], sv[2 * x + 1]);
+                    pd[x] = pack_bf16(dp[2 * x], dp[2 * x + 1]);
+                }
+                tmem_st16(lane_base + TM_ST + s * 64 + 32 * ch, pa);
+                tmem_st16(lane_base + TM_DPT + s * 64 + 32 * ch, pd);
+                tmem_wait_st();
             }
-            fence_async_smem();
             tc_fence_before();
             mbar_arrive(&pd_full[s]);
         }
-        if (ok && nsteps > 0 && mbar_wait(&pd_free[(nsteps - 1) & 1], ((nsteps - 1) >> 1) & 1, status, 323)) {
+        if (ok && nsteps > 0 && mbar_wait(&sd_free[(nsteps - 1) & 1], ((nsteps - 1) >> 1) & 1, status, 323)) {
             tc_fence_after();
             const int64_t row = ((tok0 + je) * p.Hkv + kvh) * DH;
             uint32_t o[32];
