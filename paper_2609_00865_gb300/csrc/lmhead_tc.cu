@@ -38,11 +38,24 @@ constexpr float LOG2E_F = 1.4426950408889634f;
 struct LmFwdParams {
     int M, M_pad, d, V;
     int R, NV, C, NVC;        // row tiles, vocab tiles, chunks, vocab tiles per chunk
+    int GR;                   // row tiles per item group
     const int32_t* tg;        // [M_pad]
     float2* part;             // [C][M_pad] (max2, sum)
     float* zt;                // [M]
     int32_t* status;
 };
+
+// Item w -> (vocab chunk c, row tile r). Items run in groups of GR row tiles:
+// within a group chunk-major, rows fastest. The CTAs resident at one time then
+// cover at most GR row tiles, whose hidden-state tiles stay in L2 (GR is sized
+// from d on the host), and the W tiles of their chunks are shared in step.
+__device__ __forceinline__ void item_rc(int w, int R, int C, int GR, int& c, int& r) {
+    const int rg = w / (GR * C);
+    const int rem = w - rg * (GR * C);
+    const int gr = min(GR, R - rg * GR);   // rows in this (possibly ragged last) group
+    c = rem / gr;
+    r = rg * GR + rem % gr;
+}
 
 __global__ void __launch_bounds__(NT, 1)
     k_lm_fwd_tc(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, LmFwdParams p) {
@@ -80,7 +93,8 @@ __global__ void __launch_bounds__(NT, 1)
             uint32_t it = 0;
             bool ok = true;
             for (int w = blockIdx.x; ok && w < n_items; w += gridDim.x) {
-                const int c = w / p.R, r = w % p.R;
+                int c, r;
+                item_rc(w, p.R, p.C, p.GR, c, r);
                 const int v0 = c * p.NVC, v1 = min(v0 + p.NVC, p.NV);
                 for (int vt = v0; ok && vt < v1; ++vt)
                     for (int kc = 0; kc < KC; ++kc, ++it) {
@@ -102,7 +116,8 @@ __global__ void __launch_bounds__(NT, 1)
             uint32_t it = 0, tile = 0;
             bool ok = true;
             for (int w = blockIdx.x; ok && w < n_items; w += gridDim.x) {
-                const int c = w / p.R;
+                int c, r_unused;
+                item_rc(w, p.R, p.C, p.GR, c, r_unused);
                 const int v0 = c * p.NVC, v1 = min(v0 + p.NVC, p.NV);
                 for (int vt = v0; ok && vt < v1; ++vt, ++tile) {
                     const int ab = tile & 1;
@@ -133,7 +148,8 @@ __global__ void __launch_bounds__(NT, 1)
         uint32_t tile = 0;
         bool ok = true;
         for (int w = blockIdx.x; ok && w < n_items; w += gridDim.x) {
-            const int c = w / p.R, r = w % p.R;
+            int c, r;
+            item_rc(w, p.R, p.C, p.GR, c, r);
             const int v0 = c * p.NVC, v1 = min(v0 + p.NVC, p.NV);
             const int m = r * BM + rl;
             const int tgt = p.tg[m];
@@ -267,6 +283,8 @@ mw_status lm_fwd_tc(const void* H, const void* W, const int32_t* targets, const 
     p.NV = q.NV;
     p.C = q.C;
     p.NVC = q.NVC;
+    // row tiles whose bf16 hidden-state tiles fill about 30 MB of L2 (32 at d = 3584)
+    p.GR = (int)std::max<int64_t>(8, std::min<int64_t>(q.R, (30ll << 20) / ((int64_t)BM * d * 2)));
     p.tg = tg;
     p.part = part;
     p.zt = zt;
