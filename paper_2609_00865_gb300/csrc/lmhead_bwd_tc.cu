@@ -6,20 +6,27 @@
 //
 // A pass holds a 128-row tile X of the stationary operand and streams the
 // other operand Y. The tile's accumulator over the whole hidden size (128 x d
-// fp32) is larger than one SM's tensor memory, so a cluster of C CTAs shares
+// fp32) is larger than one SM's tensor memory, so a group of C CTAs shares
 // the tile: CTA r accumulates hidden columns [r ds, (r+1) ds), ds = d / C <=
-// 256. Step t of the cluster covers C NY streamed rows (NY = 256); CTA r
+// 256. Step t of the group covers C NY streamed rows (NY = 256); CTA r
 //   1. computes the logits of its own NY streamed rows over the full hidden
 //      size, Z_r = X Y_{t,r}^T (TMEM; X and Y k-slices streamed by TMA),
 //   2. forms dz_r (bf16, 128 x NY) in the epilogue, writes it into its slot
-//      of a per-cluster ring in global memory (R = L + 2 steps deep, tens of
-//      MB in all, so it stays in L2) and signals every CTA of the cluster,
+//      of a per-group ring in global memory (R = L + 2 steps deep, tens of
+//      MB in all, so it stays in L2) and counts it on the slot's "ready"
+//      counter,
 //   3. accumulates Acc_r += sum_q dz_q Y_{t,q}[:, slice r] over the C dz
-//      tiles of the step (dz k-chunks and Y slices loaded by TMA).
+//      tiles of the step (dz k-chunks and Y slices loaded by TMA) and then
+//      counts the slot on its "freed" counter.
 // Only bf16 dz tiles cross CTAs, once per step. The accumulation of step t
 // is issued after the logits of step t + L, so the exchange has L steps of
-// tensor work to complete in. Clusters are persistent (as many as fit on the
-// GPU at once), so each owns a fixed ring region. One ring of 48 KB stages in
+// tensor work to complete in. The two counters per ring slot live in global
+// memory and only grow (release adds, acquire polls): a group is not a
+// hardware cluster, so any C co-resident CTAs can form one. The launch is
+// cooperative (every CTA resident at once, as the counters' waits require)
+// and the groups are persistent, each owning a fixed ring region. Hardware
+// clusters of 14 or 16 CTAs fit only 7 at a time (98 or 112 SMs); software
+// groups of 14 fill 140 SMs. One ring of 48 KB stages in
 // shared memory carries the operands in the order the MMA thread consumes
 // them: the k-slices of Z(t) (X 16 KB + Y 32 KB), then the stages of
 // Acc(t - L) (a 64-column chunk of one dz tile + the matching 64 Y rows).
@@ -41,7 +48,10 @@ namespace {
 
 using namespace tc;
 
-constexpr int NT = 224;              // warp 0 TMA, warp 1 MMA, warp 2 signals, warps 3..6 epilogue
+// warp 0 TMA, warp 1 MMA, warp 2 counts published dz tiles, warps 3..6
+// epilogue, warp 7 counts consumed ring slots
+constexpr int NT = 256;
+constexpr int FREE_WARP = 7;
 constexpr int NY = 256;              // streamed rows per CTA and step
 constexpr int S = 4;                 // operand stages
 constexpr uint32_t SLOT = 49152;     // bytes per operand stage
@@ -63,57 +73,33 @@ struct LmBwdParams {
     __nv_bfloat16* dH;     // [N, d]
     float* dW;             // [V, d]
     __nv_bfloat16* ring;   // [nclus][R][C][128][NY] dz exchange ring
+    uint32_t* ready;       // [nclus][R] dz tiles published into the slot, all uses
+    uint32_t* freed;       // [nclus][R] CTAs done reading the slot, all uses
     int32_t* status;
 };
 
-__device__ __forceinline__ uint32_t cluster_rank() {
-    uint32_t r;
-    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-    return r;
+// Counters of the ring slots, in global memory. A group's CTAs are not a
+// hardware cluster: they synchronise through gpu-scope release / acquire.
+__device__ __forceinline__ void count_release_gpu(uint32_t* ctr) {
+    asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(ctr) : "memory");
 }
-__device__ __forceinline__ uint32_t mapa(uint32_t addr, uint32_t rank) {
-    uint32_t r;
-    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
-    return r;
+__device__ __forceinline__ uint32_t load_acquire_gpu(const uint32_t* ctr) {
+    uint32_t v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(ctr) : "memory");
+    return v;
 }
-// Remote arrive without its own release; the caller issues one cluster-scope
-// fence before a batch of these.
-__device__ __forceinline__ void arrive_remote_relaxed(uint32_t cluster_addr) {
-    asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
-}
-__device__ __forceinline__ void fence_acq_rel_cluster() { asm volatile("fence.acq_rel.cluster;" ::: "memory"); }
 // Orders this thread's generic global accesses with the async proxy (TMA).
 __device__ __forceinline__ void fence_proxy_async_global() {
     asm volatile("fence.proxy.async.global;" ::: "memory");
 }
-// Arrive on the mbarrier at the same shared-memory offset in every CTA of
-// `mask` once this thread's issued MMAs have completed.
-__device__ __forceinline__ void commit_multicast(uint64_t* bar, uint16_t mask) {
-    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::
-                     "r"(smem_u32(bar)),
-                 "h"(mask)
-                 : "memory");
-}
-// Non-suspending poll: the arrivals on these barriers come from other CTAs.
-__device__ __forceinline__ bool try_wait_cluster(uint32_t addr, uint32_t parity) {
-    uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.test_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(ok)
-        : "r"(addr), "r"(parity)
-        : "memory");
-    return ok != 0;
-}
-// Bounded acquire-at-cluster-scope wait (for barriers that other CTAs arrive on).
-__device__ __forceinline__ bool wait_cluster(uint64_t* bar, uint32_t parity, int32_t* status, int where) {
-    const uint32_t a = smem_u32(bar);
-    if (try_wait_cluster(a, parity)) return true;
+// Bounded wait until *ctr >= target; the counters only grow during a launch.
+__device__ __forceinline__ bool wait_count(const uint32_t* ctr, uint32_t target, int32_t* status, int where) {
+    if (load_acquire_gpu(ctr) >= target) return true;
     const uint64_t t0 = globaltimer_ns();
     for (uint32_t i = 1;; ++i) {
-        if (try_wait_cluster(a, parity)) return true;
-        if ((i & 255u) == 0 &&
+        __nanosleep(32);
+        if (load_acquire_gpu(ctr) >= target) return true;
+        if ((i & 63u) == 0 &&
             ((status && *(volatile int32_t*)&status[1]) || globaltimer_ns() - t0 > kWaitLimitNs))
             break;
     }
@@ -130,12 +116,12 @@ __global__ void __launch_bounds__(NT, 1)
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~uintptr_t(1023));
     __shared__ __align__(8) uint64_t op_full[S], op_empty[S], zt_full, zt_free, acc_full, acc_free, epi_done[MAX_R],
-        dz_ready[MAX_R], dz_free[MAX_R];
+        acc_done[MAX_R];
     __shared__ uint32_t tmem_base;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int C = p.C, ds = p.ds, KD = p.KD, NS = p.NS, L = p.L, R = p.R;
-    const int rank = (int)cluster_rank();
+    const int rank = (int)(blockIdx.x % C);
     const int cid = blockIdx.x / C;
     const int col0 = rank * ds;                 // this CTA's hidden-column slice
     const int NB = (ds + 63) / 64;              // 64-column Y boxes covering the slice
@@ -155,8 +141,7 @@ __global__ void __launch_bounds__(NT, 1)
         mbar_init(&acc_free, 128);
         for (int s = 0; s < R; ++s) {
             mbar_init(&epi_done[s], 128);
-            mbar_init(&dz_ready[s], C);   // one arrive per writer CTA and step
-            mbar_init(&dz_free[s], C);    // one arrive per reader CTA and step
+            mbar_init(&acc_done[s], 1);   // this CTA's accumulation of the slot's step completed
         }
         fence_mbar_init();
     }
@@ -165,8 +150,7 @@ __global__ void __launch_bounds__(NT, 1)
         tmem_relinquish();
     }
     tc_fence_before();
-    // every CTA's barriers are initialised before any remote arrive
-    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+    __syncthreads();
     tc_fence_after();
     const uint32_t tmem = tmem_base;
     const uint32_t base = smem_u32(sm);
@@ -189,7 +173,7 @@ __global__ void __launch_bounds__(NT, 1)
             bool filled = false;
             int zt = 0, ztile = cid;               // Z stream: step in tile, tile
             int at = 0, aslot = 0;                 // accumulation stream: step in tile, ring slot
-            uint32_t aph = 0;
+            uint32_t ause = 0;                     // earlier uses of ring slot `aslot`
             bool ok = true;
             auto acquire = [&](uint32_t bytes) -> int {
                 const int slot = s;
@@ -226,7 +210,7 @@ __global__ void __launch_bounds__(NT, 1)
                 if (gt >= L) {
                     // Acc(gt - L): for each writer q and 64-row k-chunk, the dz
                     // chunk (128 x 64) and Y rows restricted to this CTA's slice
-                    if (!wait_cluster(&dz_ready[aslot], aph, status, 602)) {
+                    if (!wait_count(&p.ready[cid * R + aslot], (uint32_t)C * (ause + 1u), status, 602)) {
                         ok = false;
                         break;
                     }
@@ -250,7 +234,7 @@ __global__ void __launch_bounds__(NT, 1)
                     if (++at == NS) at = 0;
                     if (++aslot == R) {
                         aslot = 0;
-                        aph ^= 1u;
+                        ++ause;
                     }
                 }
             }
@@ -320,10 +304,10 @@ __global__ void __launch_bounds__(NT, 1)
                                 ph ^= 1u;
                             }
                         }
-                        // writer q may reuse its ring slot once these MMAs (and
-                        // so the loads of its tile) have completed
-                        if (ok) commit_multicast(&dz_free[aslot], (uint16_t)(1u << q));
                     }
+                    // the writers may reuse the slot once these MMAs (and so
+                    // the loads of its tiles) have completed
+                    if (ok) mma_commit(&acc_done[aslot]);
                     if (ok && at == NS - 1) mma_commit(&acc_full);
                     if (++at == NS) {
                         at = 0;
@@ -333,17 +317,19 @@ __global__ void __launch_bounds__(NT, 1)
                 }
             }
         }
-    } else if (warp == 2) {
-        // ------------------------------------------------------------ signaller
-        // the dz tile of step gt is published: tell every CTA of the cluster
+    } else if (warp == 2 || warp == FREE_WARP) {
+        // ------------------------------------------------------------ counters
+        // warp 2: this CTA's dz tile of step gt is in the ring (epilogue done);
+        // warp FREE_WARP: this CTA's accumulation of step gt has completed
         if (lane == 0) {
             int slot = 0;
             uint32_t sph = 0;
+            uint64_t* bars = warp == 2 ? epi_done : acc_done;
+            uint32_t* ctr = (warp == 2 ? p.ready : p.freed) + cid * R;
             for (int gt = 0; gt < G; ++gt) {
-                if (!mbar_wait(&epi_done[slot], sph, status, 631)) break;
-                fence_acq_rel_cluster();
-                const uint32_t a = smem_u32(&dz_ready[slot]);
-                for (int q = 0; q < C; ++q) arrive_remote_relaxed(mapa(a, (uint32_t)q));
+                if (!mbar_wait(&bars[slot], sph, status, warp == 2 ? 631 : 632)) break;
+                __threadfence();
+                count_release_gpu(&ctr[slot]);
                 if (++slot == R) {
                     slot = 0;
                     sph ^= 1u;
@@ -355,7 +341,6 @@ __global__ void __launch_bounds__(NT, 1)
         // warps 3..6: thread = stationary row rl = TMEM lane
         const int qw = warp & 3;
         const int rl = qw * 32 + lane;
-        const int et = threadIdx.x - 96;
         const uint32_t lane_base = tmem + ((uint32_t)(qw * 32) << 16);
         bool ok = true;
         // drain the accumulator of tile `tile` (its `n`-th) into dH / dW
@@ -399,7 +384,7 @@ __global__ void __launch_bounds__(NT, 1)
         // zero-filled by TMA, so their dz contributes nothing.
         float4 rp = make_float4(0.f, 0.f, __int_as_float(-1), 0.f);
         int t = 0, tile = cid, slot = 0, drained = 0;
-        uint32_t sph = 0;                       // phase of ring slot `slot`
+        uint32_t uses = 0;                      // earlier uses of ring slot `slot`
         int next_drain = NS + L - 1;            // step after which tile `drained` is complete
         for (int gt = 0; ok && gt < G; ++gt) {
             if (p.mode == 0 && t == 0) rp = p.par[tile * 128 + rl];
@@ -417,10 +402,11 @@ __global__ void __launch_bounds__(NT, 1)
                 break;
             }
             tc_fence_after();
-            // every CTA has loaded this ring slot's previous tile (step gt - R)
+            // every CTA of the group has consumed this ring slot's previous
+            // tiles (step gt - R)
             if (gt >= R) {
                 bool w = true;
-                if (lane == 0) w = wait_cluster(&dz_free[slot], sph ^ 1u, status, 622);
+                if (lane == 0) w = wait_count(&p.freed[cid * R + slot], (uint32_t)C * uses, status, 622);
                 w = __shfl_sync(0xffffffffu, w, 0);
                 if (!w) {
                     ok = false;
@@ -469,7 +455,7 @@ __global__ void __launch_bounds__(NT, 1)
             mbar_arrive(&epi_done[slot]);
             if (++slot == R) {
                 slot = 0;
-                sph ^= 1u;
+                ++uses;
             }
             if (++t == NS) {
                 t = 0;
@@ -487,10 +473,6 @@ __global__ void __launch_bounds__(NT, 1)
             }
         }
         for (; ok && drained < my_tiles; ++drained) ok = output(cid + drained * p.nclus, drained);
-        // the last R steps' slot-free signals from the readers aim here
-        if (et == 0)
-            for (int gt = max(0, G - R); ok && gt < G; ++gt)
-                if (!wait_cluster(&dz_free[gt % R], (uint32_t)(gt / R) & 1u, status, 625)) ok = false;
     }
     tc_fence_before();
     __syncthreads();
@@ -508,26 +490,27 @@ __global__ void k_lm_bwd_par(int M, int M_pad, const float* __restrict__ g, cons
                    : make_float4(0.f, 0.f, __int_as_float(-1), 0.f);
 }
 
-// Cluster sizes whose d-slice fits beside a 256-column logit tile in TMEM
+// Group sizes whose d-slice fits beside a 256-column logit tile in TMEM
 // (ds <= 256) and keeps 32-column output chunks (ds % 32 == 0).
 bool slice_ok(int d, int C) { return d % C == 0 && d / C <= 256 && (d / C) % 32 == 0; }
-constexpr int kClusterSizes[] = {1, 2, 3, 4, 5, 6, 7, 8, 10, 12, 14, 16};
+constexpr int kGroupSizes[] = {1, 2, 3, 4, 5, 6, 7, 8, 10, 12, 14, 16};
+constexpr int64_t kCounterBytes = 2 * 2 * RING_CTAS * MAX_R * 4;   // per pass: ready, freed
 
 }  // namespace
 
 bool lm_bwd_tc_supported(int d) {
     if (d % 64) return false;
-    for (int C : kClusterSizes)
+    for (int C : kGroupSizes)
         if (slice_ok(d, C)) return true;
     return false;
 }
 
 // Scratch of the backward inside the log-prob workspace: the per-row
-// parameters and the dz exchange ring.
+// parameters, the dz exchange ring and the ring slots' counters.
 int64_t lm_bwd_tc_scratch(int M, int d) {
     if (!lm_bwd_tc_supported(d)) return 0;
     const int64_t M_pad = ceil_div(M, 128) * 128;
-    return align256(16 * M_pad) + (int64_t)RING_CTAS * MAX_R * 128 * NY * 2;
+    return align256(16 * M_pad) + (int64_t)RING_CTAS * MAX_R * 128 * NY * 2 + kCounterBytes;
 }
 
 mw_status lm_bwd_tc(const void* W, int M, int N, int d, int V, const int32_t* rows, const void* Hg, const int32_t* tg,
@@ -540,45 +523,45 @@ mw_status lm_bwd_tc(const void* W, int M, int N, int d, int V, const int32_t* ro
     const int M_pad = (int)ceil_div(M, 128) * 128;
     float4* par = (float4*)scratch;
     __nv_bfloat16* ring = at<__nv_bfloat16>(scratch, align256(16 * (int64_t)M_pad));
+    uint32_t* counters = at<uint32_t>(ring, (int64_t)RING_CTAS * MAX_R * 128 * NY * 2);
+    if ((st = cuda_status(cudaMemsetAsync(counters, 0, kCounterBytes, s))) != MW_OK) return st;
     count_launches(1);
     k_lm_bwd_par<<<(unsigned)ceil_div(M_pad, 256), 256, 0, s>>>(M, M_pad, g, lse, tg, dloss, par);
     if ((st = launch_status()) != MW_OK) return st;
 
     if ((st = cuda_status(cudaFuncSetAttribute(k_lm_bwd_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                               (int)SMEM))) != MW_OK ||
-        (st = cuda_status(cudaFuncSetAttribute(k_lm_bwd_tc, cudaFuncAttributeNonPortableClusterSizeAllowed, 1))) !=
-            MW_OK)
+                                               (int)SMEM))) != MW_OK)
         return st;
+    // The CTAs of a group wait on one another's counters, so every CTA must be
+    // resident at once: the launch is cooperative (it fails rather than run
+    // CTAs in waves) and the grid never exceeds what fits.
+    int dev = 0, sms = 0, per_sm = 0;
+    if ((st = cuda_status(cudaGetDevice(&dev))) != MW_OK ||
+        (st = cuda_status(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev))) != MW_OK ||
+        (st = cuda_status(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_lm_bwd_tc, NT, SMEM))) != MW_OK)
+        return st;
+    const int resident = std::min(per_sm * sms, RING_CTAS);
+    // The fewest CTAs per group (the widest slice): a CTA's tensor work per
+    // step is 2 * 128 * NY * d FLOP for any C, but its dz chunk loads, stages
+    // and waits per step grow with C (d = 3584 measured: C = 14, 140 CTAs,
+    // 114 ms; C = 16, 144 CTAs, 127 ms; d = 1536: C = 6 beats C = 8 and 12).
+    int C = 0;
+    for (int c : kGroupSizes)
+        if (slice_ok(d, c)) {
+            C = c;
+            break;
+        }
+    const int max_groups = C > 0 ? resident / C : 0;
+    if (max_groups == 0) return MW_EDEVICE;
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
+    attr[0].id = cudaLaunchAttributeCooperative;
+    attr[0].val.cooperative = 1;
     cfg.blockDim = dim3(NT);
     cfg.dynamicSmemBytes = SMEM;
     cfg.stream = s;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    // the cluster size that keeps the most CTAs resident (smaller on ties)
-    int C = 0, max_clusters = 0, best = 0;
-    for (int c : kClusterSizes) {
-        if (!slice_ok(d, c)) continue;
-        attr[0].val.clusterDim.x = (unsigned)c;
-        cfg.gridDim = dim3((unsigned)c);
-        int n = 0;
-        if (cudaOccupancyMaxActiveClusters(&n, k_lm_bwd_tc, &cfg) != cudaSuccess) {
-            (void)cudaGetLastError();
-            continue;
-        }
-        n = std::min(n, RING_CTAS / c);
-        if (n * c > best) {
-            best = n * c;
-            C = c;
-            max_clusters = n;
-        }
-    }
-    if (C == 0) return MW_EDEVICE;
-    attr[0].val.clusterDim.x = (unsigned)C;
 
     const int ring_rows = RING_CTAS * MAX_R * 128;
     CUtensorMap hx, hyz, hya, wx, wyz, wya, dm;
@@ -605,9 +588,11 @@ mw_status lm_bwd_tc(const void* W, int M, int N, int d, int V, const int32_t* ro
     p.status = status;
     for (int mode = 0; mode < 2; ++mode) {
         p.mode = mode;
+        p.ready = counters + mode * 2 * RING_CTAS * MAX_R;
+        p.freed = p.ready + RING_CTAS * MAX_R;
         p.tiles = mode == 0 ? M_pad / 128 : (int)ceil_div(V, 128);
         p.NS = (int)ceil_div(mode == 0 ? V : M_pad, (int64_t)C * NY);
-        p.nclus = std::min(p.tiles, max_clusters);
+        p.nclus = std::min(p.tiles, max_groups);
         cfg.gridDim = dim3((unsigned)(p.nclus * C));
         count_launches(1);
         if ((st = cuda_status(cudaLaunchKernelEx(&cfg, k_lm_bwd_tc, mode == 0 ? hx : wx, mode == 0 ? wyz : hyz,

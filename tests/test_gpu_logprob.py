@@ -85,9 +85,13 @@ def test_zero_weights_uniform():
 
 
 @pytest.mark.parametrize("N,M,d,V", [
-    (700, 450, 512, 3001),      # 2-CTA cluster split of d, ragged vocab tail
-    (600, 300, 1536, 2999),     # the config-3 hidden size (4-CTA cluster)
-    (1200, 700, 3584, 152064),  # the config-4 hidden size and vocabulary (8-CTA cluster)
+    # the backward splits d over a group of C CTAs, each owning a d-slice of at
+    # most 256 columns (the fewest CTAs per group)
+    (300, 200, 256, 4097),      # one CTA per group (C = 1)
+    (700, 450, 512, 3001),      # ragged vocab tail (C = 2)
+    (500, 260, 960, 5003),      # C = 5, d-slice 192
+    (600, 300, 1536, 2999),     # the config-3 hidden size (C = 6)
+    (1200, 700, 3584, 152064),  # the config-4 hidden size and vocabulary (C = 14)
 ])
 def test_tensor_core_shapes(N, M, d, V):
     rows = np.sort(np.random.default_rng(N).permutation(N)[:M])
