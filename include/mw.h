@@ -181,8 +181,9 @@ mw_status mw_masked_attn_bwd_ws(const mw_vis_layout* layout, int Hq, int Dh, int
 /*
  * Backward of mw_masked_attn_fwd for upstream dO (same layout as O).
  * Writes dQ (like Q), dK, dV (like K, V), all in `dtype`, overwriting them.
- * Delta_i = rowsum(dO_i * O_i) and, for bf16, a float32 dQ accumulator live
- * in `ws` (mw_masked_attn_bwd_ws bytes).
+ * Delta_i = rowsum(dO_i * O_i) (for bf16 with Dh 128: the pair (LSE_i log2 e,
+ * Delta_i) per row, rows padded to whole 128-row tiles) lives in `ws`
+ * (mw_masked_attn_bwd_ws bytes).
  */
 mw_status mw_masked_attn_bwd(const mw_vis_layout* layout, const void* vis,
                              const void* Q, const void* K, const void* V, const void* O,

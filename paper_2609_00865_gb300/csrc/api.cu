@@ -1,6 +1,7 @@
 // extern "C" entry points of libmw: host-side argument checks and dispatch.
 // See include/mw.h for the contract of every function.
 
+#include <algorithm>
 #include <math.h>
 
 #include "common.cuh"
@@ -19,6 +20,7 @@ mw_status attn_fwd_tc(const mw_vis_layout*, const void*, const void*, const void
                       int, float, cudaStream_t);
 mw_status attn_bwd_tc(const mw_vis_layout*, const void*, const void*, const void*, const void*, const void*,
                       const void*, const float*, void*, void*, void*, int, int, float, float*, cudaStream_t);
+int64_t attn_bwd_tc_ws(const mw_vis_layout*, int);
 __global__ void k_loss_epilogue(int, const float*, const float*, const float*, float, float, float*, float*, float*);
 
 struct LmPlan {
@@ -89,8 +91,9 @@ extern "C" mw_status mw_masked_attn_fwd(const mw_vis_layout* L, const void* vis,
 
 extern "C" mw_status mw_masked_attn_bwd_ws(const mw_vis_layout* L, int Hq, int Dh, int dtype, size_t* bytes) {
     if (!L || !bytes) return MW_EINVAL;
-    (void)Dh; (void)dtype;
-    *bytes = (size_t)align256(4 * L->total_tokens * (int64_t)Hq);
+    int64_t b = 4 * L->total_tokens * (int64_t)Hq;   // Delta per (head, row)
+    if (dtype == MW_BF16 && Dh == 128) b = std::max(b, attn_bwd_tc_ws(L, Hq));
+    *bytes = (size_t)align256(b);
     return MW_OK;
 }
 

@@ -367,8 +367,8 @@ struct BwdParams {
     int64_t total;
     int n_traj, max_tiles, Hq, Hkv;
     float scale, scale_log2;
-    const float* LSE;
-    const float* delta;
+    const float2* lsd;     // [Hq][n_tiles * 128] (LSE_i log2 e, Delta_i), rows padded to whole tiles
+    int64_t n_rows;        // n_tiles * 128
     __nv_bfloat16* dQ;
     __nv_bfloat16* dK;
     __nv_bfloat16* dV;
@@ -511,8 +511,8 @@ __global__ void __launch_bounds__(NT_BWD, 1)
         const int seg = v.seg[tok0 + ie];
         const uint4* km = reinterpret_cast<const uint4*>(v.keymask) + v.traj_km[b] + (int64_t)seg * nt;
         const uint32_t lane_base = tmem + ((uint32_t)(qw * 32) << 16);
-        const float lse2 = p.LSE[(int64_t)h * p.total + tok0 + ie] * LOG2E;
-        const float dl = p.delta[(int64_t)h * p.total + tok0 + ie];
+        const float2 ld = p.lsd[(int64_t)h * p.n_rows + g * 128 + rl];
+        const float lse2 = ld.x, dl = ld.y;
         bool ok = true;
         for (int j = 0; j < n; ++j) {
             const int e = v.fwd_idx[p0 + j];
@@ -638,10 +638,8 @@ __global__ void __launch_bounds__(NT_BWD, 1)
                    const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, BwdParams p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~uintptr_t(1023));
-    __shared__ __align__(8) uint64_t kv_full, qd_full[QD_ST], qd_empty[QD_ST], sd_full[2], sd_free[2], pd_full[2],
-        ls_full[2], ls_free[2];
+    __shared__ __align__(8) uint64_t kv_full, qd_full[QD_ST], qd_empty[QD_ST], sd_full[2], sd_free[2], pd_full[2];
     __shared__ uint32_t tmem_base;
-    __shared__ __align__(16) float lsd[2][128];   // per step: LSE2 of the 64 rows, then Delta of the 64 rows
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int grp = p.Hq / p.Hkv;
@@ -673,8 +671,6 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             mbar_init(&sd_full[s], 1);
             mbar_init(&sd_free[s], 1);     // the accumulation's completion: P^T / dS^T live there until then
             mbar_init(&pd_full[s], NEW);
-            mbar_init(&ls_full[s], NEW);
-            mbar_init(&ls_free[s], NEW);
         }
         fence_mbar_init();
     }
@@ -686,14 +682,24 @@ __global__ void __launch_bounds__(NT_BWD, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = tmem_base;
-    // step t -> (list entry, head in group, half). The list is walked from its
-    // last q-tile down, so CTAs of one KV head that started together stream the
-    // same Q / dO tiles at the same time (L2 reuse across k-tiles).
-    auto step_q0 = [&](int t, int& hq) -> int {
-        const int e = nlist - 1 - t / (grp * 2);
-        const int rem = t % (grp * 2);
-        hq = kvh * grp + rem / 2;
-        return (v.bwd_idx[p0 + e] >> 2) * 128 + (rem & 1) * 64;
+    // step t -> (list entry e, head in group, half), kept as a running cursor
+    // (integer division on these threads costs more than a step's work). The
+    // list is walked from its last q-tile down, so CTAs of one KV head that
+    // started together stream the same Q / dO tiles at the same time (L2 reuse
+    // across k-tiles); rem = 2 * (head in group) + half.
+    struct Cursor {
+        int e, rem;
+    };
+    const Cursor first{nlist - 1, 0};
+    auto advance = [&](Cursor& c) {
+        if (++c.rem == 2 * grp) {
+            c.rem = 0;
+            --c.e;
+        }
+    };
+    auto cur_q0 = [&](const Cursor& c, int& hq) -> int {
+        hq = kvh * grp + (c.rem >> 1);
+        return (v.bwd_idx[p0 + c.e] >> 2) * 128 + (c.rem & 1) * 64;
     };
 
     if (warp == 0) {
@@ -705,17 +711,23 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             mbar_expect_tx(&kv_full, 2 * TILE_B);
             load_tile(sm + KV_K, &tmK, &kv_full, kvh, (int)(tok0 + kt * 128));
             load_tile(sm + KV_V, &tmV, &kv_full, kvh, (int)(tok0 + kt * 128));
-            for (int t = 0; t < nsteps; ++t) {
-                const int s = t % QD_ST;
+            Cursor c = first;
+            int s = 0;
+            uint32_t ph = 0;
+            for (int t = 0; t < nsteps; ++t, advance(c)) {
                 int hq;
-                const int q0 = step_q0(t, hq);
-                if (t >= QD_ST && !mbar_wait(&qd_empty[s], ((t / QD_ST) - 1) & 1, status, 121)) break;
+                const int q0 = cur_q0(c, hq);
+                if (t >= QD_ST && !mbar_wait(&qd_empty[s], ph ^ 1u, status, 121)) break;
                 mbar_expect_tx(&qd_full[s], 2 * HT_B);
                 uint8_t* dst = sm + KV_Q + s * 2 * HT_B;
                 tma_load_3d(dst, &tmQ, &qd_full[s], 0, hq, (int)(tok0 + q0));
                 tma_load_3d(dst + HT_HALF, &tmQ, &qd_full[s], 64, hq, (int)(tok0 + q0));
                 tma_load_3d(dst + HT_B, &tmDO, &qd_full[s], 0, hq, (int)(tok0 + q0));
                 tma_load_3d(dst + HT_B + HT_HALF, &tmDO, &qd_full[s], 64, hq, (int)(tok0 + q0));
+                if (++s == QD_ST) {
+                    s = 0;
+                    ph ^= 1u;
+                }
             }
         }
     } else if (warp == 1 || warp == BWD_ACC_WARP) {
@@ -775,27 +787,28 @@ __global__ void __launch_bounds__(NT_BWD, 1)
         const int je = min(jk, T - 1);
         const int iend = jk < T ? min(v.omega[tok0 + je], T) : 0;   // rows [jk, iend) see this key
         const uint32_t lane_base = tmem + ((uint32_t)(qw * 32) << 16);
-        const int tid = threadIdx.x - 64;            // 0..255 among the elementwise threads
         bool ok = true;
-        // LSE2 (threads 0..63) and Delta (64..127) of step t's rows q0 .. q0+63; a
-        // step's values are loaded during the previous step and published at its end
-        auto ls_load = [&](int t) -> float {
+        // (LSE2, Delta) of this warp's 32 query rows of a step: 256 contiguous
+        // bytes of the tile-padded pair array, read by every lane (broadcast);
+        // the next step's two lines are prefetched into L1 a step ahead
+        const float2* lsd_k = p.lsd + (int64_t)v.traj_tile[b] * 128 + 32 * ch;
+        auto lsd_row = [&](const Cursor& c) -> const float4* {
             int hq;
-            const int q0 = step_q0(t, hq);
-            const int row = min(q0 + (tid & 63), T - 1);
-            const int64_t at = (int64_t)hq * p.total + tok0 + row;
-            return tid < 64 ? p.LSE[at] * LOG2E : p.delta[at];
+            const int q0 = cur_q0(c, hq);
+            return reinterpret_cast<const float4*>(lsd_k + (int64_t)hq * p.n_rows + q0);
         };
-        if (nsteps > 0) {
-            if (tid < 128) lsd[0][tid] = ls_load(0);
-            mbar_arrive(&ls_full[0]);
-        }
+        Cursor cur = first;
         for (int t = 0; t < nsteps; ++t) {
             const int s = t & 1;
             int hq;
-            const int q0 = step_q0(t, hq);
-            const float ls_next = (tid < 128 && t + 1 < nsteps) ? ls_load(t + 1) : 0.f;
-            if (!mbar_wait(&ls_full[s], (t >> 1) & 1, status, 325)) { ok = false; break; }
+            const int q0 = cur_q0(cur, hq);
+            const float4* l4 = reinterpret_cast<const float4*>(lsd_k + (int64_t)hq * p.n_rows + q0);
+            float4 lv[16];
+#pragma unroll
+            for (int q = 0; q < 16; ++q) lv[q] = l4[q];
+            advance(cur);
+            if (t + 1 < nsteps && lane < 2)
+                asm volatile("prefetch.global.L1 [%0];" ::"l"(reinterpret_cast<const char*>(lsd_row(cur)) + 128 * lane));
             if (!mbar_wait(&sd_full[s], (t >> 1) & 1, status, 321)) { ok = false; break; }
             tc_fence_after();
             float sv[32], dp[32];
@@ -812,31 +825,20 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             }
             // visible columns [lo, hi) of this warp's 32
             const int lo = max(jk, q0 + 32 * ch) - q0 - 32 * ch, hi = min(iend, q0 + 64) - q0 - 32 * ch;
-            // this warp's 32 LSE2 and Delta values: broadcast 16-byte loads into registers
             float lse_c[32], del_c[32];
-            {
-                const float4* l4 = reinterpret_cast<const float4*>(lsd[s] + 32 * ch);
-                const float4* d4 = reinterpret_cast<const float4*>(lsd[s] + 64 + 32 * ch);
 #pragma unroll
-                for (int q = 0; q < 8; ++q) {
-                    const float4 a = l4[q], d = d4[q];
-                    lse_c[4 * q] = a.x; lse_c[4 * q + 1] = a.y; lse_c[4 * q + 2] = a.z; lse_c[4 * q + 3] = a.w;
-                    del_c[4 * q] = d.x; del_c[4 * q + 1] = d.y; del_c[4 * q + 2] = d.z; del_c[4 * q + 3] = d.w;
-                }
+            for (int q = 0; q < 16; ++q) {
+                lse_c[2 * q] = lv[q].x;
+                del_c[2 * q] = lv[q].y;
+                lse_c[2 * q + 1] = lv[q].z;
+                del_c[2 * q + 1] = lv[q].w;
             }
-            mbar_arrive(&ls_free[s]);
 #pragma unroll
             for (int c = 0; c < 32; ++c) {
                 const bool vis = c >= lo && c < hi;
                 const float pr = vis ? ex2(fmaf(sv[c], p.scale_log2, -lse_c[c])) : 0.f;
                 sv[c] = pr;
                 dp[c] = pr * (dp[c] - del_c[c]);
-            }
-            if (t + 1 < nsteps) {
-                // buffer s ^ 1 was last read in step t - 1
-                if (t >= 1 && !mbar_wait(&ls_free[s ^ 1], ((t - 1) >> 1) & 1, status, 324)) { ok = false; break; }
-                if (tid < 128) lsd[s ^ 1][tid] = ls_next;
-                mbar_arrive(&ls_full[s ^ 1]);
             }
             {   // P^T, dS^T (bf16 pairs) over the first 16 of this warp's own 32
                 // columns of the S^T / dP^T buffers, which only this thread has read
@@ -926,13 +928,54 @@ mw_status attn_fwd_tc(const mw_vis_layout* L, const void* vis, const void* Q, co
     return launch_status();
 }
 
-mw_status attn_delta(const mw_vis_layout*, const void*, const void*, int, int, int, float*, cudaStream_t);
+namespace {
+
+// (LSE_i log2 e, Delta_i = rowsum(dO_i * O_i)) per (head, row) in the
+// tile-padded layout [Hq][n_tiles * 128]: row r of global tile g sits at
+// g * 128 + r, so any 32 rows of a tile are 256 contiguous, 16-byte aligned
+// bytes. Rows past a trajectory's end hold zeros. One warp per (row, head).
+__global__ void k_attn_lsd(VisView v, int64_t total, int64_t n_rows, int Hq, const __nv_bfloat16* __restrict__ O,
+                           const __nv_bfloat16* __restrict__ dO, const float* __restrict__ LSE,
+                           float2* __restrict__ lsd) {
+    const int lane = threadIdx.x & 31;
+    const int64_t nw = (int64_t)gridDim.x * (blockDim.x >> 5);
+    for (int64_t w = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5; w < n_rows * Hq; w += nw) {
+        const int64_t gr = w / Hq;
+        const int h = (int)(w - gr * Hq);
+        const int g = (int)(gr >> 7);
+        const int b = v.tile_traj[g];
+        const int64_t tok0 = v.traj_tok[b];
+        const int i = (g - v.traj_tile[b]) * 128 + (int)(gr & 127);
+        float2 out = make_float2(0.f, 0.f);
+        if (i < v.traj_tok[b + 1] - (int)tok0) {
+            const int64_t row = ((tok0 + i) * Hq + h) * DH + 4 * lane;
+            const uint2 o = *reinterpret_cast<const uint2*>(O + row), d = *reinterpret_cast<const uint2*>(dO + row);
+            const float2 o0 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&o.x));
+            const float2 o1 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&o.y));
+            const float2 d0 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&d.x));
+            const float2 d1 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&d.y));
+            const float acc = warp_sum(fmaf(o0.x, d0.x, fmaf(o0.y, d0.y, fmaf(o1.x, d1.x, o1.y * d1.y))));
+            out = make_float2(LSE[(int64_t)h * total + tok0 + i] * LOG2E, acc);
+        }
+        if (lane == 0) lsd[(int64_t)h * n_rows + gr] = out;
+    }
+}
+
+}  // namespace
+
+int64_t attn_bwd_tc_ws(const mw_vis_layout* L, int Hq) { return 8 * L->n_tiles * 128 * (int64_t)Hq; }
 
 mw_status attn_bwd_tc(const mw_vis_layout* L, const void* vis, const void* Q, const void* K, const void* V,
                       const void* O, const void* dO, const float* LSE, void* dQ, void* dK, void* dV, int Hq, int Hkv,
-                      float scale, float* delta, cudaStream_t s) {
+                      float scale, float* ws, cudaStream_t s) {
     if (L->n_tiles == 0) return MW_OK;
-    mw_status st = attn_delta(L, O, dO, Hq, DH, MW_BF16, delta, s);
+    const int64_t n_rows = L->n_tiles * 128;
+    float2* lsd = reinterpret_cast<float2*>(ws);
+    const VisView view = make_view(L, vis);
+    count_launches(1);
+    k_attn_lsd<<<(unsigned)std::min<int64_t>(ceil_div(n_rows * Hq, 8), 152 * 64), 256, 0, s>>>(
+        view, L->total_tokens, n_rows, Hq, (const __nv_bfloat16*)O, (const __nv_bfloat16*)dO, LSE, lsd);
+    mw_status st = launch_status();
     if (st != MW_OK) return st;
     const uint64_t T = (uint64_t)L->total_tokens;
     CUtensorMap tq, tdo, tk, tv, tq64, tdo64;
@@ -949,8 +992,8 @@ mw_status attn_bwd_tc(const mw_vis_layout* L, const void* vis, const void* Q, co
     p.Hkv = Hkv;
     p.scale = scale;
     p.scale_log2 = scale * LOG2E;
-    p.LSE = LSE;
-    p.delta = delta;
+    p.lsd = lsd;
+    p.n_rows = n_rows;
     p.dQ = (__nv_bfloat16*)dQ;
     p.dK = (__nv_bfloat16*)dK;
     p.dV = (__nv_bfloat16*)dV;
