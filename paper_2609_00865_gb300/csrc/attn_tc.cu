@@ -79,6 +79,25 @@ __device__ __forceinline__ float ex2(float x) {
     return y;
 }
 
+// Softmax-gradient elements of the backward, two at a time: p = 2^(s c + n)
+// with n = -LSE_i log2 e, masked pairs (bit clear in vm) entering the exp2 as
+// -inf (so p = +0, no branch); ds = p (dp - Delta_i). MASKED = false when the
+// caller knows every pair is visible.
+template <bool MASKED>
+__device__ __forceinline__ void soft_pair(float s0, float s1, float dp0, float dp1, uint64_t c2, uint64_t n2,
+                                          uint64_t dl2, uint32_t vm, int bit, uint32_t& p_pk, uint32_t& ds_pk) {
+    const uint64_t a = fma2(f2(s0, s1), c2, n2);
+    float a0 = f2_lo(a), a1 = f2_hi(a);
+    if (MASKED) {
+        a0 = ((vm >> bit) & 1u) ? a0 : -INFINITY;
+        a1 = ((vm >> (bit + 1)) & 1u) ? a1 : -INFINITY;
+    }
+    const float p0 = ex2(a0), p1 = ex2(a1);
+    const uint64_t d = mul2(f2(p0, p1), sub2(f2(dp0, dp1), dl2));
+    p_pk = pack_bf16(p0, p1);
+    ds_pk = pack_bf16(f2_lo(d), f2_hi(d));
+}
+
 __device__ __forceinline__ void load_tile(uint8_t* dst, const CUtensorMap* map, uint64_t* bar, int head, int row) {
     tma_load_3d(dst, map, bar, 0, head, row);
     tma_load_3d(dst + HALF_B, map, bar, 64, head, row);
@@ -367,7 +386,7 @@ struct BwdParams {
     int64_t total;
     int n_traj, max_tiles, Hq, Hkv;
     float scale, scale_log2;
-    const float2* lsd;     // [Hq][n_tiles * 128] (LSE_i log2 e, Delta_i), rows padded to whole tiles
+    const float2* lsd;     // [Hq][n_tiles * 128] (-LSE_i log2 e, Delta_i), rows padded to whole tiles
     int64_t n_rows;        // n_tiles * 128
     __nv_bfloat16* dQ;
     __nv_bfloat16* dK;
@@ -512,7 +531,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
         const uint4* km = reinterpret_cast<const uint4*>(v.keymask) + v.traj_km[b] + (int64_t)seg * nt;
         const uint32_t lane_base = tmem + ((uint32_t)(qw * 32) << 16);
         const float2 ld = p.lsd[(int64_t)h * p.n_rows + g * 128 + rl];
-        const float lse2 = ld.x, dl = ld.y;
+        const uint64_t c2 = f2(p.scale_log2, p.scale_log2), n2 = f2(ld.x, ld.x), dl2 = f2(ld.y, ld.y);
         bool ok = true;
         for (int j = 0; j < n; ++j) {
             const int e = v.fwd_idx[p0 + j];
@@ -544,9 +563,25 @@ __global__ void __launch_bounds__(NT_BWD, 1)
                 }
             }
             const uint32_t w0 = ch ? wd[2] : wd[0], w1 = ch ? wd[3] : wd[1];
+            // P = 2^(S c - LSE2), two elements per instruction; masked pairs
+            // enter the exp2 as -inf (P = +0) instead of branching around it
+            if (__all_sync(0xffffffffu, (w0 & w1) == 0xffffffffu)) {
 #pragma unroll
-            for (int c = 0; c < 64; ++c)
-                s[c] = (((c < 32 ? w0 : w1) >> (c & 31)) & 1u) ? ex2(fmaf(s[c], p.scale_log2, -lse2)) : 0.f;
+                for (int x = 0; x < 32; ++x) {
+                    const uint64_t a = fma2(f2(s[2 * x], s[2 * x + 1]), c2, n2);
+                    s[2 * x] = ex2(f2_lo(a));
+                    s[2 * x + 1] = ex2(f2_hi(a));
+                }
+            } else {
+#pragma unroll
+                for (int x = 0; x < 32; ++x) {
+                    const uint32_t wm = x < 16 ? w0 : w1;
+                    const int bit = (2 * x) & 31;
+                    const uint64_t a = fma2(f2(s[2 * x], s[2 * x + 1]), c2, n2);
+                    s[2 * x] = ex2(((wm >> bit) & 1u) ? f2_lo(a) : -INFINITY);
+                    s[2 * x + 1] = ex2(((wm >> (bit + 1)) & 1u) ? f2_hi(a) : -INFINITY);
+                }
+            }
             if (!mbar_wait(&dp_full, j & 1, status, 312)) { ok = false; break; }
             tc_fence_after();
             uint32_t dpr[2][32];   // both dP loads in flight before one wait
@@ -555,8 +590,8 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             tmem_wait_ld();
             tc_fence_before();
             mbar_arrive(&dp_free);
-            // dS (bf16 pairs) over the first 32 of this warp's own 64 S columns,
-            // which only this thread has read
+            // dS = P (dP - Delta) as bf16 pairs over the first 32 of this warp's
+            // own 64 S columns, which only this thread has read
             const uint32_t dst = lane_base + TM_S0 + (j & 1) * 128 + 64 * ch;
 #pragma unroll
             for (int cc = 0; cc < 2; ++cc) {
@@ -565,8 +600,9 @@ __global__ void __launch_bounds__(NT_BWD, 1)
 #pragma unroll
                 for (int x = 0; x < 16; ++x) {
                     const int c0 = cc * 32 + 2 * x;
-                    pk[x] = pack_bf16(s[c0] * (__uint_as_float(dp[2 * x]) - dl),
-                                      s[c0 + 1] * (__uint_as_float(dp[2 * x + 1]) - dl));
+                    const uint64_t d = mul2(f2(s[c0], s[c0 + 1]),
+                                            sub2(f2(__uint_as_float(dp[2 * x]), __uint_as_float(dp[2 * x + 1])), dl2));
+                    pk[x] = pack_bf16(f2_lo(d), f2_hi(d));
                 }
                 tmem_st16(dst + 16 * cc, pk);
             }
@@ -687,19 +723,24 @@ __global__ void __launch_bounds__(NT_BWD, 1)
     // list is walked from its last q-tile down, so CTAs of one KV head that
     // started together stream the same Q / dO tiles at the same time (L2 reuse
     // across k-tiles); rem = 2 * (head in group) + half.
+    // The q-tiles of the current and the next list entry are cached, so that
+    // no step waits on a load of the list.
     struct Cursor {
-        int e, rem;
+        int e, rem, qt, qt_next;
     };
-    const Cursor first{nlist - 1, 0};
+    auto list_qt = [&](int e) -> int { return e >= 0 ? v.bwd_idx[p0 + e] >> 2 : 0; };
+    const Cursor first{nlist - 1, 0, list_qt(nlist - 1), list_qt(nlist - 2)};
     auto advance = [&](Cursor& c) {
         if (++c.rem == 2 * grp) {
             c.rem = 0;
             --c.e;
+            c.qt = c.qt_next;
+            c.qt_next = list_qt(c.e - 1);
         }
     };
     auto cur_q0 = [&](const Cursor& c, int& hq) -> int {
         hq = kvh * grp + (c.rem >> 1);
-        return (v.bwd_idx[p0 + c.e] >> 2) * 128 + (c.rem & 1) * 64;
+        return c.qt * 128 + (c.rem & 1) * 64;
     };
 
     if (warp == 0) {
@@ -788,27 +829,29 @@ __global__ void __launch_bounds__(NT_BWD, 1)
         const int iend = jk < T ? min(v.omega[tok0 + je], T) : 0;   // rows [jk, iend) see this key
         const uint32_t lane_base = tmem + ((uint32_t)(qw * 32) << 16);
         bool ok = true;
-        // (LSE2, Delta) of this warp's 32 query rows of a step: 256 contiguous
-        // bytes of the tile-padded pair array, read by every lane (broadcast);
-        // the next step's two lines are prefetched into L1 a step ahead
+        // (-LSE2, Delta) of this warp's 32 query rows of a step: 256 contiguous
+        // bytes of the tile-padded pair array, read by every lane (broadcast)
+        // at the start of the step, after a prefetch into L1 one step earlier.
         const float2* lsd_k = p.lsd + (int64_t)v.traj_tile[b] * 128 + 32 * ch;
         auto lsd_row = [&](const Cursor& c) -> const float4* {
             int hq;
             const int q0 = cur_q0(c, hq);
             return reinterpret_cast<const float4*>(lsd_k + (int64_t)hq * p.n_rows + q0);
         };
-        Cursor cur = first;
+        Cursor cur = first, nxt = first;   // steps t and t + 1
+        advance(nxt);
         for (int t = 0; t < nsteps; ++t) {
             const int s = t & 1;
             int hq;
             const int q0 = cur_q0(cur, hq);
-            const float4* l4 = reinterpret_cast<const float4*>(lsd_k + (int64_t)hq * p.n_rows + q0);
             float4 lv[16];
+            {
+                const float4* l4 = lsd_row(cur);
 #pragma unroll
-            for (int q = 0; q < 16; ++q) lv[q] = l4[q];
-            advance(cur);
+                for (int q = 0; q < 16; ++q) lv[q] = l4[q];
+            }
             if (t + 1 < nsteps && lane < 2)
-                asm volatile("prefetch.global.L1 [%0];" ::"l"(reinterpret_cast<const char*>(lsd_row(cur)) + 128 * lane));
+                asm volatile("prefetch.global.L1 [%0];" ::"l"(reinterpret_cast<const char*>(lsd_row(nxt)) + 128 * lane));
             if (!mbar_wait(&sd_full[s], (t >> 1) & 1, status, 321)) { ok = false; break; }
             tc_fence_after();
             float sv[32], dp[32];
@@ -823,30 +866,24 @@ __global__ void __launch_bounds__(NT_BWD, 1)
                     dp[x] = __uint_as_float(rb[x]);
                 }
             }
-            // visible columns [lo, hi) of this warp's 32
-            const int lo = max(jk, q0 + 32 * ch) - q0 - 32 * ch, hi = min(iend, q0 + 64) - q0 - 32 * ch;
-            float lse_c[32], del_c[32];
-#pragma unroll
-            for (int q = 0; q < 16; ++q) {
-                lse_c[2 * q] = lv[q].x;
-                del_c[2 * q] = lv[q].y;
-                lse_c[2 * q + 1] = lv[q].z;
-                del_c[2 * q + 1] = lv[q].w;
-            }
-#pragma unroll
-            for (int c = 0; c < 32; ++c) {
-                const bool vis = c >= lo && c < hi;
-                const float pr = vis ? ex2(fmaf(sv[c], p.scale_log2, -lse_c[c])) : 0.f;
-                sv[c] = pr;
-                dp[c] = pr * (dp[c] - del_c[c]);
-            }
+            // visible columns [lo, hi) of this warp's 32, as a bit mask
+            const int lo = min(max(jk, q0 + 32 * ch) - q0 - 32 * ch, 32);
+            const int hi = max(min(min(iend, q0 + 64) - q0 - 32 * ch, 32), lo);
+            const uint32_t vm = (hi >= 32 ? 0xffffffffu : ((1u << hi) - 1u)) & ~(lo >= 32 ? 0xffffffffu : ((1u << lo) - 1u));
             {   // P^T, dS^T (bf16 pairs) over the first 16 of this warp's own 32
                 // columns of the S^T / dP^T buffers, which only this thread has read
                 uint32_t pa[16], pd[16];
+                const uint64_t c2 = f2(p.scale_log2, p.scale_log2);
+                if (__all_sync(0xffffffffu, vm == 0xffffffffu)) {
 #pragma unroll
-                for (int x = 0; x < 16; ++x) {
-                    pa[x] = pack_bf16(sv[2 * x], sv[2 * x + 1]);
-                    pd[x] = pack_bf16(dp[2 * x], dp[2 * x + 1]);
+                    for (int x = 0; x < 16; ++x)
+                        soft_pair<false>(sv[2 * x], sv[2 * x + 1], dp[2 * x], dp[2 * x + 1], c2, f2(lv[x].x, lv[x].z),
+                                         f2(lv[x].y, lv[x].w), vm, 2 * x, pa[x], pd[x]);
+                } else {
+#pragma unroll
+                    for (int x = 0; x < 16; ++x)
+                        soft_pair<true>(sv[2 * x], sv[2 * x + 1], dp[2 * x], dp[2 * x + 1], c2, f2(lv[x].x, lv[x].z),
+                                        f2(lv[x].y, lv[x].w), vm, 2 * x, pa[x], pd[x]);
                 }
                 tmem_st16(lane_base + TM_ST + s * 64 + 32 * ch, pa);
                 tmem_st16(lane_base + TM_DPT + s * 64 + 32 * ch, pd);
@@ -854,6 +891,8 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             }
             tc_fence_before();
             mbar_arrive(&pd_full[s]);
+            cur = nxt;
+            advance(nxt);
         }
         if (ok && nsteps > 0 && mbar_wait(&sd_free[(nsteps - 1) & 1], ((nsteps - 1) >> 1) & 1, status, 323)) {
             tc_fence_after();
@@ -930,7 +969,7 @@ mw_status attn_fwd_tc(const mw_vis_layout* L, const void* vis, const void* Q, co
 
 namespace {
 
-// (LSE_i log2 e, Delta_i = rowsum(dO_i * O_i)) per (head, row) in the
+// (-LSE_i log2 e, Delta_i = rowsum(dO_i * O_i)) per (head, row) in the
 // tile-padded layout [Hq][n_tiles * 128]: row r of global tile g sits at
 // g * 128 + r, so any 32 rows of a tile are 256 contiguous, 16-byte aligned
 // bytes. Rows past a trajectory's end hold zeros. One warp per (row, head).
@@ -955,7 +994,7 @@ __global__ void k_attn_lsd(VisView v, int64_t total, int64_t n_rows, int Hq, con
             const float2 d0 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&d.x));
             const float2 d1 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&d.y));
             const float acc = warp_sum(fmaf(o0.x, d0.x, fmaf(o0.y, d0.y, fmaf(o1.x, d1.x, o1.y * d1.y))));
-            out = make_float2(LSE[(int64_t)h * total + tok0 + i] * LOG2E, acc);
+            out = make_float2(-LSE[(int64_t)h * total + tok0 + i] * LOG2E, acc);
         }
         if (lane == 0) lsd[(int64_t)h * n_rows + gr] = out;
     }
