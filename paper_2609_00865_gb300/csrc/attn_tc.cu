@@ -271,14 +271,16 @@ __global__ void __launch_bounds__(NT_FWD, 1)
                     if (!((wd[c >> 5] >> (c & 31)) & 1u)) s[c] = -INFINITY;
             }
             // row max and row sum as 8 independent partial chains (a single
-            // 128-long dependency chain per reduction bounds the warp's latency)
+            // 128-long dependency chain per reduction bounds the warp's latency);
+            // the max folds two new elements per instruction
             float pm[8];
 #pragma unroll
             for (int k = 0; k < 8; ++k) pm[k] = s[k];
 #pragma unroll
-            for (int c = 8; c < 128; ++c) pm[c & 7] = fmaxf(pm[c & 7], s[c]);
-            const float mx = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
-                                   fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
+            for (int c = 8; c < 128; c += 16)
+#pragma unroll
+                for (int k = 0; k < 8; ++k) pm[k] = max3(pm[k], s[c + k], s[c + 8 + k]);
+            const float mx = max3(max3(pm[0], pm[1], pm[2]), max3(pm[3], pm[4], pm[5]), fmaxf(pm[6], pm[7]));
             const float mx2 = mx * p.scale_log2;
             float alpha = 1.f;
             if (mx2 > m + RESCALE_T) {
@@ -286,13 +288,18 @@ __global__ void __launch_bounds__(NT_FWD, 1)
                 m = mx2;
             }
             const float mu = (m == -INFINITY) ? 0.f : m;
-            float ps[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+            // P = 2^(S c - mu) and its row sum, two elements per FMA / add
+            const uint64_t c2 = f2(p.scale_log2, p.scale_log2), n2 = f2(-mu, -mu);
+            uint64_t ps[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
-            for (int c = 0; c < 128; ++c) {
-                s[c] = ex2(fmaf(s[c], p.scale_log2, -mu));
-                ps[c & 7] += s[c];
+            for (int c = 0; c < 128; c += 2) {
+                const uint64_t a = fma2(f2(s[c], s[c + 1]), c2, n2);
+                s[c] = ex2(f2_lo(a));
+                s[c + 1] = ex2(f2_hi(a));
+                ps[(c >> 1) & 3] = add2(ps[(c >> 1) & 3], f2(s[c], s[c + 1]));
             }
-            const float rs = ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
+            const uint64_t ps2 = add2(add2(ps[0], ps[1]), add2(ps[2], ps[3]));
+            const float rs = f2_lo(ps2) + f2_hi(ps2);
             l = l * alpha + rs;
             // P_j (bf16 pairs) over the first 64 columns of its own S buffer; the
             // PV MMA reads it from there, so P never touches shared memory
