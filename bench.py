@@ -44,9 +44,14 @@ def _peaks():
 # value it had when the counters were taken.
 TRAFFIC = {
     (4, "mw_logprob_loss_bwd"): {
-        "bytes": 121432050944 + 12028077056 + 122184046080 + 14604399872,   # dH pass + dW pass
+        "bytes": 79358121984 + 11882540288 + 86699048960 + 14107458304,   # dH pass + dW pass
         "source": "paper_2609_00865_gb300/csrc/lmhead_bwd_tc.cu",
-        "sha256": "3e7fabc08aa4485f57d0fa6e95f540c317bc119f2c81ba5111a68f59b8ec7cc7",
+        "sha256": "5657c62c221bfbecae71d0954adb5970de2d73155845e6fa0d1761f9c1df110e",
+    },
+    (4, "mw_masked_attn_bwd"): {
+        "bytes": (1894422272 + 28065792) + (30600770560 + 908907264) + (63477532416 + 263952896),   # lsd, dQ, dK/dV
+        "source": "paper_2609_00865_gb300/csrc/attn_tc.cu",
+        "sha256": "e5b85e37e292919afdef3229f3f80edc0e1bcb77282b62adcab6eb45c08821d1",
     },
 }
 
