@@ -30,12 +30,13 @@ METRIC = "view-consistent scored tokens/sec (fwd+bwd)"
 
 
 def _peaks():
+    """(bf16 burst TFLOP/s, bf16 sustained TFLOP/s, HBM GB/s, source)."""
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
             p = json.load(f)
-        return float(p["bf16_tflops"]), float(p["hbm_gbs"]), "measured"
+        return float(p["bf16_tflops"]), float(p["bf16_tflops_sustained"]), float(p["hbm_gbs"]), "measured"
     except Exception:
-        return 1900.0, 6800.0, "fallback"
+        return 1900.0, 1700.0, 6800.0, "fallback"
 
 
 # DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) per call of a
@@ -475,24 +476,50 @@ def run_gpu(args, rank, world, local_rank):
     out = step.loss if hasattr(step, "loss") else step.LSE[0, :1]
     d2h = out.numel() * out.element_size()
     pinned_out = torch.empty(out.shape, dtype=out.dtype).pin_memory()
+    # Every step uploads its own inputs and reads its loss back inside the
+    # timed region. As a training loop that prefetches its next batch does,
+    # step i + 1's inputs are copied on a copy stream while step i computes,
+    # into the other of two device input sets.
+    sets = [step.d, dict(step.d)]
+    for k in host:
+        sets[1][k] = torch.empty_like(step.d[k])
+    copy = torch.cuda.Stream(dev)
+    ready = [torch.cuda.Event(), torch.cuda.Event()]
+    used = [torch.cuda.Event(), torch.cuda.Event()]
+
+    def upload(i):
+        with torch.cuda.stream(copy):
+            for k, v in host.items():
+                sets[i % 2][k].copy_(v, non_blocking=True)
+            ready[i % 2].record(copy)
+
     barrier()
     torch.cuda.synchronize()
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
     e0.record(step.stream)
-    for _ in range(args.steps):
-        step.upload(host)
+    copy.wait_event(e0)
+    upload(0)
+    for i in range(args.steps):
+        if i + 1 < args.steps:
+            if i >= 1:
+                copy.wait_event(used[(i + 1) % 2])   # step i - 1 read that set
+            upload(i + 1)
+        step.stream.wait_event(ready[i % 2])
+        step.d = sets[i % 2]
         step.run()
+        used[i % 2].record(step.stream)
         pinned_out.copy_(out, non_blocking=True)
     e1.record(step.stream)
     torch.cuda.synchronize()
+    step.d = sets[0]
     e2e_ms = reduce_max(e0.elapsed_time(e1) / args.steps, world, dev)
 
     if rank != 0:
         return
     scored = step.scored()
     flops = step.flops()
-    peak_tf, hbm, peak_kind = _peaks()
+    peak_tf, peak_sus, hbm, peak_kind = _peaks()
     dom = max(per_call, key=per_call.get)
     dom_flops = {"mw_masked_attn_fwd": 4.0 / 14.0 * flops.get("attn", 0),
                  "mw_masked_attn_bwd": 10.0 / 14.0 * flops.get("attn", 0),
@@ -510,13 +537,17 @@ def run_gpu(args, rank, world, local_rank):
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": describe(w),
         "visible_tflops": total_tf, "visible_frac_of_peak": total_tf / peak_tf,
-        "roofline": {"bound": "tensor", "kernel": dom, "achieved": achieved, "peak": peak_tf,
-                     "unit": "TFLOP/s", "frac": achieved / peak_tf, "traffic": _traffic(w["cfg"], dom),
-                     "peak_kind": f"bf16 dense burst, {peak_kind}"},
+        "visible_frac_of_sustained_peak": total_tf / peak_sus,
+        # the dominant call is timed inside the step loop (seconds of back-to-back
+        # work under the power cap): the sustained peak is its denominator
+        "roofline": {"bound": "tensor", "kernel": dom, "achieved": achieved, "peak": peak_sus,
+                     "unit": "TFLOP/s", "frac": achieved / peak_sus, "traffic": _traffic(w["cfg"], dom),
+                     "peak_kind": f"bf16 dense sustained, {peak_kind} (burst {peak_tf})"},
         "per_call_ms": per_call,
         "cpu_baseline": cpu,
         "e2e": {"value": job_value(scored, world, e2e_ms), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
-                "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
+                "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms,
+                "upload": "pinned host -> device, step i + 1's inputs on a copy stream during step i"},
         "gpu_launches": launches,
         "clocks": clk,
     }
