@@ -238,8 +238,20 @@ __global__ void __launch_bounds__(NT_FWD, 1)
         const uint32_t lane_base = tmem + ((uint32_t)(qw * 32) << 16);
         float m = -INFINITY, l = 0.f;
         bool ok = true;
+        // list entries and view-mask words are loaded ahead (an entry two
+        // tiles, a mask word one tile), so no step waits on a global load once
+        // its S is ready
+        int e_cur = n > 0 ? v.fwd_idx[p0] : 0;
+        int e_nxt = n > 1 ? v.fwd_idx[p0 + 1] : 0;
+        uint4 w_cur = n > 0 ? km[e_cur >> 2] : make_uint4(0u, 0u, 0u, 0u);
         for (int j = 0; j < n; ++j) {
-            const int e = v.fwd_idx[p0 + j];
+            const int e = e_cur;
+            const uint4 wv = w_cur;
+            if (j + 1 < n) {
+                w_cur = km[e_nxt >> 2];
+                e_cur = e_nxt;
+                e_nxt = j + 2 < n ? v.fwd_idx[p0 + j + 2] : 0;
+            }
             const int kt = e >> 2, cls = e & 3;
             if (!mbar_wait(&s_full[j & 1], (j >> 1) & 1, status, 301)) { ok = false; break; }
             tc_fence_after();
@@ -255,8 +267,7 @@ __global__ void __launch_bounds__(NT_FWD, 1)
                     for (int x = 0; x < 32; ++x) s[c * 32 + x] = __uint_as_float(rr[c][x]);
             }
             if (cls != MW_TILE_FULL || kt == qt) {
-                uint4 w = km[kt];
-                uint32_t wd[4] = {w.x, w.y, w.z, w.w};
+                uint32_t wd[4] = {wv.x, wv.y, wv.z, wv.w};
                 if (kt == qt) {   // causal inside the diagonal tile: keys c <= ie - kt*128
                     const int lim = ie - kt * 128;
 #pragma unroll
@@ -540,8 +551,20 @@ __global__ void __launch_bounds__(NT_BWD, 1)
         const float2 ld = p.lsd[(int64_t)h * p.n_rows + g * 128 + rl];
         const uint64_t c2 = f2(p.scale_log2, p.scale_log2), n2 = f2(ld.x, ld.x), dl2 = f2(ld.y, ld.y);
         bool ok = true;
+        // list entries and view-mask words are loaded ahead (an entry two
+        // tiles, a mask word one tile), so no step waits on a global load once
+        // its S is ready
+        int e_cur = n > 0 ? v.fwd_idx[p0] : 0;
+        int e_nxt = n > 1 ? v.fwd_idx[p0 + 1] : 0;
+        uint4 w_cur = n > 0 ? km[e_cur >> 2] : make_uint4(0u, 0u, 0u, 0u);
         for (int j = 0; j < n; ++j) {
-            const int e = v.fwd_idx[p0 + j];
+            const int e = e_cur;
+            const uint4 wv = w_cur;
+            if (j + 1 < n) {
+                w_cur = km[e_nxt >> 2];
+                e_cur = e_nxt;
+                e_nxt = j + 2 < n ? v.fwd_idx[p0 + j + 2] : 0;
+            }
             const int kt = e >> 2, cls = e & 3;
             if (!mbar_wait(&s_full[j & 1], (j >> 1) & 1, status, 311)) { ok = false; break; }
             tc_fence_after();
@@ -558,8 +581,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             }
             uint32_t wd[4] = {0xffffffffu, 0xffffffffu, 0xffffffffu, 0xffffffffu};
             if (cls != MW_TILE_FULL || kt == qt) {
-                uint4 w = km[kt];
-                wd[0] = w.x; wd[1] = w.y; wd[2] = w.z; wd[3] = w.w;
+                wd[0] = wv.x; wd[1] = wv.y; wd[2] = wv.z; wd[3] = wv.w;
                 if (kt == qt) {
                     const int lim = ie - kt * 128;
 #pragma unroll
