@@ -205,6 +205,7 @@ mw_status mw_logprob_ws(int N, int M, int d, int Vocab, int dtype, size_t* ws_by
  *   rows[M] distinct physical rows (int32, device); lp_old, adv [M] float32.
  *   Outputs lp, ratio, lse [M] float32, loss: one float32 (device).
  * `ws` (mw_logprob_ws bytes) keeps dL/dlp per row for the backward.
+ * M = 0 is allowed: the loss is 0 (and the backward writes zero gradients).
  * dtype MW_BF16 requires d % 64 == 0; MW_F32 requires d <= 256.
  */
 mw_status mw_logprob_loss_fwd(const void* H, const void* W, const int32_t* targets,

@@ -91,6 +91,48 @@ def test_medium_bf16_gqa():
     assert_grad_bf16(np64(dV), dVr, "dV")
 
 
+# trajectories of 1, 127, 0, 128, 129 and 300 tokens in one record: a lone row,
+# one row short of a tile, an empty trajectory, an exact tile, a one-row second
+# tile and a ragged third tile
+_TILE_EDGE = (
+    [1, 127, 0, 128, 129, 300],
+    [[], [(100, [(10, 40)])], [], [(64, [(0, 32)]), (120, [(70, 100)])], [(128, [(5, 127)])],
+     [(150, [(20, 140)]), (280, [(150, 260)])]],
+)
+
+
+@pytest.mark.parametrize("Hq,Hkv", [(4, 4), (6, 2)])
+def test_bf16_tile_edges_and_group_sizes(Hq, Hkv):
+    """Tensor-core path on the tile-edge record, with one query head per KV
+    head and with groups of three."""
+    seqlens, edits = _TILE_EDGE
+    Q, K, V, dO = _tensors(sum(seqlens), Hq, Hkv, 128, 51 + Hq, torch.bfloat16)
+    scale = 128 ** -0.5
+    O, LSE, dQ, dK, dV = _run(seqlens, edits, Q, K, V, dO, scale)
+    Or, Lr = OA.attn_fwd(seqlens, edits, np64(Q), np64(K), np64(V), scale)
+    assert_maxabs(np64(O), Or, 2e-2, "O")
+    assert_maxabs(np64(LSE), Lr, 2e-2, "LSE")
+    dQr, dKr, dVr = OA.attn_bwd(seqlens, edits, np64(Q), np64(K), np64(V), np64(dO), scale)
+    assert_grad_bf16(np64(dQ), dQr, "dQ")
+    assert_grad_bf16(np64(dK), dKr, "dK")
+    assert_grad_bf16(np64(dV), dVr, "dV")
+
+
+def test_fp32_tile_edges():
+    """The exact-fp32 path (Dh 64, groups of two) on the tile-edge record."""
+    seqlens, edits = _TILE_EDGE
+    Q, K, V, dO = _tensors(sum(seqlens), 4, 2, 64, 61, torch.float32)
+    scale = 64 ** -0.5
+    O, LSE, dQ, dK, dV = _run(seqlens, edits, Q, K, V, dO, scale)
+    Or, Lr = OA.attn_fwd(seqlens, edits, np64(Q), np64(K), np64(V), scale)
+    assert_rel(np64(O), Or, 1e-4, "O")
+    assert_rel(np64(LSE), Lr, 1e-4, "LSE")
+    dQr, dKr, dVr = OA.attn_bwd(seqlens, edits, np64(Q), np64(K), np64(V), np64(dO), scale)
+    assert_rel(np64(dQ), dQr, 1e-4, "dQ")
+    assert_rel(np64(dK), dKr, 1e-4, "dK")
+    assert_rel(np64(dV), dVr, 1e-4, "dV")
+
+
 def test_no_edits_is_causal_attention():
     """K = 0 reduces to ordinary causal attention (library SDPA on the GPU
     output's inputs, float64 on the CPU)."""

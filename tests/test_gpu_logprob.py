@@ -92,12 +92,32 @@ def test_zero_weights_uniform():
     (500, 260, 960, 5003),      # C = 5, d-slice 192
     (600, 300, 1536, 2999),     # the config-3 hidden size (C = 6)
     (1200, 700, 3584, 152064),  # the config-4 hidden size and vocabulary (C = 14)
+    (200, 130, 64, 100),        # the smallest hidden size, a vocabulary below one 256-wide tile
 ])
 def test_tensor_core_shapes(N, M, d, V):
     rows = np.sort(np.random.default_rng(N).permutation(N)[:M])
     args = _case(N, d, V, rows, 70 + d, torch.bfloat16)
     out, dH, dW = _run(*args[:6], 0.2, 0.28, dloss=0.7)
     _check(*args, out, dH, dW, 0.2, 0.28, fp32=False, dloss=0.7)
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+def test_no_loss_rows(dtype):
+    """M = 0: the loss is 0 and dH, dW are written as zeros (the outputs start
+    uninitialised)."""
+    import paper_2609_00865_gb300 as mw
+    N, d, V = 300, 128, 1000
+    H = synth.normal((N, d), 81).to(dtype).cuda()
+    W = synth.normal((V, d), 82, std=0.02).to(dtype).cuda()
+    t = synth.uniform_int(N, V, 83).cuda()
+    rows = torch.zeros(0, dtype=torch.int32, device="cuda")
+    empty = torch.zeros(0, dtype=torch.float32, device="cuda")
+    out = mw.logprob_loss_fwd(H, W, t, rows, empty, empty, 0.2, 0.28)
+    dH, dW = mw.logprob_loss_bwd(H, W, t, rows, out["lse"], out["ws"], 1.0)
+    torch.cuda.synchronize()
+    assert out["lp"].numel() == 0
+    assert float(out["loss"].item()) == 0.0
+    assert (dH == 0).all() and (dW == 0).all()
 
 
 def test_config3_full_size_sampled():
