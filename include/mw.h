@@ -25,7 +25,8 @@
  *    junction, so causality alone hides them from earlier rows.
  *  - Tiles are 128 x 128, trajectory-local, the last one ragged. Class EMPTY
  *    (no visible in-range pair), FULL (all in-range pairs visible) or PARTIAL.
- *    Tile-list entries are int32 (tile << 2) | class.
+ *    Tile-list entries are int32 (tile << 4) | code, code = class plus the
+ *    MW_TILE_DEAD_* bits (see below).
  *  - Every device pointer is caller-owned device memory (the library never
  *    allocates device memory, never frees, never synchronises a stream except
  *    where stated). Host pointers are read during the call only.
@@ -60,12 +61,17 @@ typedef enum mw_status {
 enum { MW_F32 = 0, MW_BF16 = 1 };
 enum { MW_TILE = 128 };
 enum { MW_TILE_EMPTY = 0, MW_TILE_PARTIAL = 1, MW_TILE_FULL = 2 };
+/* Beside its class (bits 0-1), a PARTIAL off-diagonal tile carries DEAD_LO
+ * (bit 2) when no row of its q-tile sees any of the k-tile's keys 0..63, and
+ * DEAD_HI (bit 3) for keys 64..127 (every key of that half evicted before the
+ * q-tile starts, or past the trajectory's end). At most one is set. */
+enum { MW_TILE_DEAD_LO = 4, MW_TILE_DEAD_HI = 8 };
 
 /* Human-readable name of a status code (static string). */
 const char* mw_status_str(int status);
 /* Last CUDA error code seen by the library on this host thread (0 if none). */
 int mw_last_cuda_error(void);
-/* ABI version of this header (bumped on any signature change). */
+/* ABI version of this header (bumped on any signature or layout change). */
 int mw_abi_version(void);
 /* Number of CUDA kernels this library has launched in this process so far
  * (all threads, all devices); lets callers count launches in a timed region. */

@@ -21,13 +21,17 @@ Table "running-prefixes" in App. B.4):
 Tile conventions used by the GPU structures (not from the paper, which gives
 no kernel): 128x128 tiles, trajectory-local, the last tile ragged. A tile is
 EMPTY (0) when no in-range pair is visible, FULL (2) when every in-range pair
-is visible, else PARTIAL (1). Tile-list entries are ``(tile << 2) | class``.
+is visible, else PARTIAL (1). A PARTIAL off-diagonal tile also carries DEAD_LO
+(4) / DEAD_HI (8) when none of its pairs with the k-tile's first / second half
+of keys is visible. Tile-list entries are ``(tile << 4) | code``, code = class
+plus those bits.
 """
 
 import numpy as np
 
 TILE = 128
 EMPTY, PARTIAL, FULL = 0, 1, 2
+DEAD_LO, DEAD_HI = 4, 8
 NEVER = np.iinfo(np.int32).max  # lifetime end of a key that is never evicted
 
 
@@ -180,6 +184,30 @@ def tile_classes(T, edits, tile=TILE):
     return cls.astype(np.int32), counts
 
 
+def dead_halves(T, edits, cls, tile=TILE):
+    """DEAD_LO / DEAD_HI bits of every PARTIAL off-diagonal tile.
+
+    Key half h of tile (qt, kt) holds keys ``[kt*tile + h*tile/2, ... +
+    tile/2)``; it is dead when none of its pairs with the q-tile's rows is
+    visible. The counts come from the same per-segment view prefix sums as
+    the tile classes, at half-tile granularity: the q-tile's two half-row
+    tiles against the half-key tile. Halves past the trajectory's end are dead.
+    """
+    h = tile // 2
+    c, _ = tile_counts(T, edits, h)
+    nt = cls.shape[0]
+    c_pad = np.zeros((2 * nt + 2, 2 * nt + 2), dtype=np.int64)
+    c_pad[:c.shape[0], :c.shape[1]] = c
+    q = np.arange(nt)
+    partial_off = (cls == PARTIAL) & (q[:, None] > q[None, :])
+    out = np.zeros_like(cls)
+    for hh, bit in ((0, DEAD_LO), (1, DEAD_HI)):
+        kh = 2 * q + hh
+        cnt = c_pad[2 * q][:, kh] + c_pad[2 * q + 1][:, kh]
+        out |= np.where(partial_off & (cnt == 0), bit, 0).astype(cls.dtype)
+    return out
+
+
 def segment_keymask(T, edits, tile=TILE):
     """Per (segment, k-tile) 128-bit membership of the segment's live view.
 
@@ -207,7 +235,7 @@ def build(seqlens, edits_per_traj, tile=TILE):
     ``omega`` int32 [T_total]  lifetime end (trajectory-local, NEVER = int32 max)
     ``seg``   int32 [T_total]  segment id of each row
     ``qtile_traj`` int32 [n_tiles]
-    ``cls``   list of per-trajectory [nt, nt] class matrices
+    ``cls``   list of per-trajectory [nt, nt] tile codes (class | DEAD bits)
     ``fwd_ptr``/``fwd_idx``  per global q-tile, ascending non-empty k-tiles
     ``bwd_ptr``/``bwd_idx``  per global k-tile, ascending non-empty q-tiles
     ``pairs`` int64 [n_traj], ``pairs_total`` int
@@ -218,6 +246,7 @@ def build(seqlens, edits_per_traj, tile=TILE):
     pairs, keymask = [], []
     for b, (T, edits) in enumerate(zip(seqlens, edits_per_traj)):
         cls, counts = tile_classes(T, edits, tile)
+        cls = cls | dead_halves(T, edits, cls, tile)
         nt = cls.shape[0]
         om = lifetimes(T, edits)
         # The dense-mask path is the definition; lifetimes are stored as the
@@ -230,10 +259,10 @@ def build(seqlens, edits_per_traj, tile=TILE):
         # (row-major scan of the class matrix); bwd list of k-tile kt: its
         # non-EMPTY q-tiles in ascending order (scan of the transpose).
         q_nz, k_nz = np.nonzero(cls != EMPTY)
-        fwd_idx.extend(((k_nz << 2) | cls[q_nz, k_nz]).tolist())
+        fwd_idx.extend(((k_nz << 4) | cls[q_nz, k_nz]).tolist())
         fwd_ptr.extend((fwd_ptr[-1] + np.cumsum(np.bincount(q_nz, minlength=nt))).tolist())
         k_nz2, q_nz2 = np.nonzero(cls.T != EMPTY)
-        bwd_idx.extend(((q_nz2 << 2) | cls[q_nz2, k_nz2]).tolist())
+        bwd_idx.extend(((q_nz2 << 4) | cls[q_nz2, k_nz2]).tolist())
         bwd_ptr.extend((bwd_ptr[-1] + np.cumsum(np.bincount(k_nz2, minlength=nt))).tolist())
         pairs.append(int(counts.sum()))
         keymask.append(segment_keymask(T, edits, tile).reshape(-1, tile // 32))

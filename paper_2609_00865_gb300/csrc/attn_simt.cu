@@ -55,7 +55,7 @@ __global__ void __launch_bounds__(128) k_attn_fwd_simt(VisView v, int64_t total,
         for (int c = 0; c < NC; ++c) o[c] = 0.f;
         for (int p = p0; p < p1; ++p) {
             const int e = v.fwd_idx[p];
-            const int kt = e >> 2, cls = e & 3;
+            const int kt = e >> 4, cls = e & 3;
             const int jend = min(kt * MW_TILE + MW_TILE, i + 1);
             for (int j0 = kt * MW_TILE; j0 < jend; j0 += 32) {
                 const int j = j0 + lane;
@@ -141,7 +141,7 @@ __global__ void __launch_bounds__(128) k_attn_dq_simt(VisView v, int64_t total, 
         for (int c = 0; c < NC; ++c) dq[c] = 0.f;
         for (int p = p0; p < p1; ++p) {
             const int e = v.fwd_idx[p];
-            const int kt = e >> 2, cls = e & 3;
+            const int kt = e >> 4, cls = e & 3;
             const int jend = min(kt * MW_TILE + MW_TILE, i + 1);
             for (int j0 = kt * MW_TILE; j0 < jend; j0 += 32) {
                 const int j = j0 + lane;

@@ -23,6 +23,8 @@
 
 #include <math.h>
 
+#include <type_traits>
+
 #include "common.cuh"
 #include "tc.cuh"
 #include "tmap.cuh"
@@ -174,7 +176,7 @@ __global__ void __launch_bounds__(NT_FWD, 1)
             mbar_expect_tx(&q_full, TILE_B);
             load_tile(sm + SM_Q, &tmQ, &q_full, h, (int)(tok0 + qt * 128));
             for (int j = 0; j < n; ++j) {
-                const int kt = v.fwd_idx[p0 + j] >> 2;
+                const int kt = v.fwd_idx[p0 + j] >> 4;
                 const int s = j & 1;
                 const int row = (int)(tok0 + kt * 128);
                 if (j >= 2 && !mbar_wait(&k_empty[s], ((j - 2) >> 1) & 1, status, 101)) { abort_flag = 1; break; }
@@ -197,28 +199,48 @@ __global__ void __launch_bounds__(NT_FWD, 1)
             // O += P_t V_t with P_t (bf16, two keys per 32-bit column) read from
             // the first 64 columns of S buffer t & 1
             auto pv = [&](int t) -> bool {
+                const int e = v.fwd_idx[p0 + t];
                 if (!mbar_wait(&p_full[t & 1], (t >> 1) & 1, status, 202)) return false;
                 if (!mbar_wait(&v_full[t & 1], (t >> 1) & 1, status, 203)) return false;
                 tc_fence_after();
                 const uint32_t vb = sv + (t & 1) * TILE_B;
                 const uint32_t pa = tmem + TM_S0 + (t & 1) * 128;
+                if (e & (MW_TILE_DEAD_LO | MW_TILE_DEAD_HI)) {
+                    // K = 64: the live half's keys (16-row k-steps 4 lh .. 4 lh + 3 of V)
+                    const int kh = (e & MW_TILE_DEAD_LO) ? 4 : 0;
 #pragma unroll
-                for (int ks = 0; ks < 8; ++ks) mma_ts(tmem + TM_O, pa + 8 * ks, mnmaj(vb, ks), iO, (t > 0 || ks > 0));
+                    for (int ks = 0; ks < 4; ++ks)
+                        mma_ts(tmem + TM_O, pa + 8 * ks, mnmaj(vb, ks + kh), iO, (t > 0 || ks > 0));
+                } else {
+#pragma unroll
+                    for (int ks = 0; ks < 8; ++ks)
+                        mma_ts(tmem + TM_O, pa + 8 * ks, mnmaj(vb, ks), iO, (t > 0 || ks > 0));
+                }
                 mma_commit(&v_empty[t & 1]);
                 mma_commit(&s_free[t & 1]);
                 mma_commit(&o_done);
                 return true;
             };
             if (warp == 1) {
+                const uint32_t iS64 = idesc_bf16(128, 64, 0, 0);   // S over one live key half
                 for (int j = 0; ok && j < n; ++j) {
                     const int s = j & 1;
+                    const int e = v.fwd_idx[p0 + j];
                     if (!mbar_wait(&k_full[s], (j >> 1) & 1, status, 204)) { ok = false; break; }
                     if (j >= 2 && !mbar_wait(&s_free[s], ((j - 2) >> 1) & 1, status, 205)) { ok = false; break; }
                     tc_fence_after();
                     const uint32_t kb = sk + s * TILE_B;
+                    if (e & (MW_TILE_DEAD_LO | MW_TILE_DEAD_HI)) {
+                        // keys 64 lh .. 64 lh + 63: rows 64 lh.. of each 64-column panel
+                        const uint32_t kh = kb + ((e & MW_TILE_DEAD_LO) ? 64u * 128u : 0u);
 #pragma unroll
-                    for (int ks = 0; ks < 8; ++ks)
-                        mma_ss(tmem + TM_S0 + s * 128, kmaj(sq, ks), kmaj(kb, ks), iS, ks > 0);
+                        for (int ks = 0; ks < 8; ++ks)
+                            mma_ss(tmem + TM_S0 + s * 128, kmaj(sq, ks), kmaj(kh, ks), iS64, ks > 0);
+                    } else {
+#pragma unroll
+                        for (int ks = 0; ks < 8; ++ks)
+                            mma_ss(tmem + TM_S0 + s * 128, kmaj(sq, ks), kmaj(kb, ks), iS, ks > 0);
+                    }
                     mma_commit(&k_empty[s]);
                     mma_commit(&s_full[s]);
                 }
@@ -243,54 +265,50 @@ __global__ void __launch_bounds__(NT_FWD, 1)
         // its S is ready
         int e_cur = n > 0 ? v.fwd_idx[p0] : 0;
         int e_nxt = n > 1 ? v.fwd_idx[p0 + 1] : 0;
-        uint4 w_cur = n > 0 ? km[e_cur >> 2] : make_uint4(0u, 0u, 0u, 0u);
-        for (int j = 0; j < n; ++j) {
-            const int e = e_cur;
-            const uint4 wv = w_cur;
-            if (j + 1 < n) {
-                w_cur = km[e_nxt >> 2];
-                e_cur = e_nxt;
-                e_nxt = j + 2 < n ? v.fwd_idx[p0 + j + 2] : 0;
-            }
-            const int kt = e >> 2, cls = e & 3;
-            if (!mbar_wait(&s_full[j & 1], (j >> 1) & 1, status, 301)) { ok = false; break; }
-            tc_fence_after();
-            float s[128];
-            {   // all four loads in flight before one wait
-                uint32_t rr[4][32];
+        uint4 w_cur = n > 0 ? km[e_cur >> 4] : make_uint4(0u, 0u, 0u, 0u);
+        // One tile of the online softmax over NC 32-column chunks of S (4: the
+        // whole tile; 2: a live key half): mask, row max, P = 2^(S c - m) into
+        // the first NC * 16 columns of the buffer as bf16 pairs, row sum.
+        // `lim`: keys c <= lim are causal (diagonal tile); returns the factor
+        // by which O must be rescaled.
+        auto soft_tile = [&](auto ncc, uint32_t sbuf, bool masked, int lim, uint32_t w0, uint32_t w1, uint32_t w2,
+                             uint32_t w3) -> float {
+            constexpr int NC = decltype(ncc)::value;
+            constexpr int NS = NC * 32;
+            float s[NS];
+            {   // all loads in flight before one wait
+                uint32_t rr[NC][32];
 #pragma unroll
-                for (int c = 0; c < 4; ++c) tmem_ld32(lane_base + TM_S0 + (j & 1) * 128 + c * 32, rr[c]);
+                for (int c = 0; c < NC; ++c) tmem_ld32(sbuf + c * 32, rr[c]);
                 tmem_wait_ld();
 #pragma unroll
-                for (int c = 0; c < 4; ++c)
+                for (int c = 0; c < NC; ++c)
 #pragma unroll
                     for (int x = 0; x < 32; ++x) s[c * 32 + x] = __uint_as_float(rr[c][x]);
             }
-            if (cls != MW_TILE_FULL || kt == qt) {
-                uint32_t wd[4] = {wv.x, wv.y, wv.z, wv.w};
-                if (kt == qt) {   // causal inside the diagonal tile: keys c <= ie - kt*128
-                    const int lim = ie - kt * 128;
+            if (masked) {
+                uint32_t wd[4] = {w0, w1, w2, w3};
 #pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        const int hi = lim - 32 * q;   // keep bits 0..hi
-                        const uint32_t keep = hi >= 31 ? 0xffffffffu : (hi < 0 ? 0u : ((2u << hi) - 1u));
-                        wd[q] &= keep;
-                    }
+                for (int q = 0; q < NC; ++q) {   // causal inside the diagonal tile: keys c <= lim
+                    const int hi = lim - 32 * q;   // keep bits 0..hi
+                    wd[q] &= hi >= 31 ? 0xffffffffu : (hi < 0 ? 0u : ((2u << hi) - 1u));
                 }
 #pragma unroll
-                for (int c = 0; c < 128; ++c)
+                for (int c = 0; c < NS; ++c)
                     if (!((wd[c >> 5] >> (c & 31)) & 1u)) s[c] = -INFINITY;
             }
-            // row max and row sum as 8 independent partial chains (a single
-            // 128-long dependency chain per reduction bounds the warp's latency);
-            // the max folds two new elements per instruction
+            // row max as 8 independent partial chains (a single dependency chain
+            // bounds the warp's latency), two new elements per instruction
             float pm[8];
 #pragma unroll
             for (int k = 0; k < 8; ++k) pm[k] = s[k];
+            constexpr int NPAIR = (NS - 8) / 16;
 #pragma unroll
-            for (int c = 8; c < 128; c += 16)
+            for (int c = 8; c < 8 + 16 * NPAIR; c += 16)
 #pragma unroll
                 for (int k = 0; k < 8; ++k) pm[k] = max3(pm[k], s[c + k], s[c + 8 + k]);
+#pragma unroll
+            for (int k = 0; k < 8; ++k) pm[k] = fmaxf(pm[k], s[8 + 16 * NPAIR + k]);   // the last 8
             const float mx = max3(max3(pm[0], pm[1], pm[2]), max3(pm[3], pm[4], pm[5]), fmaxf(pm[6], pm[7]));
             const float mx2 = mx * p.scale_log2;
             float alpha = 1.f;
@@ -303,27 +321,48 @@ __global__ void __launch_bounds__(NT_FWD, 1)
             const uint64_t c2 = f2(p.scale_log2, p.scale_log2), n2 = f2(-mu, -mu);
             uint64_t ps[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
-            for (int c = 0; c < 128; c += 2) {
+            for (int c = 0; c < NS; c += 2) {
                 const uint64_t a = fma2(f2(s[c], s[c + 1]), c2, n2);
                 s[c] = ex2(f2_lo(a));
                 s[c + 1] = ex2(f2_hi(a));
                 ps[(c >> 1) & 3] = add2(ps[(c >> 1) & 3], f2(s[c], s[c + 1]));
             }
             const uint64_t ps2 = add2(add2(ps[0], ps[1]), add2(ps[2], ps[3]));
-            const float rs = f2_lo(ps2) + f2_hi(ps2);
-            l = l * alpha + rs;
-            // P_j (bf16 pairs) over the first 64 columns of its own S buffer; the
-            // PV MMA reads it from there, so P never touches shared memory
-            {
-                const uint32_t pt = lane_base + TM_S0 + (j & 1) * 128;
+            l = l * alpha + (f2_lo(ps2) + f2_hi(ps2));
+            // P (bf16 pairs) over the first NC * 16 columns of its own S buffer;
+            // the PV MMA reads it from there, so P never touches shared memory
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    uint32_t pk[16];
+            for (int q = 0; q < NC; ++q) {
+                uint32_t pk[16];
 #pragma unroll
-                    for (int x = 0; x < 16; ++x) pk[x] = pack_bf16(s[32 * q + 2 * x], s[32 * q + 2 * x + 1]);
-                    tmem_st16(pt + 16 * q, pk);
-                }
-                tmem_wait_st();
+                for (int x = 0; x < 16; ++x) pk[x] = pack_bf16(s[32 * q + 2 * x], s[32 * q + 2 * x + 1]);
+                tmem_st16(sbuf + 16 * q, pk);
+            }
+            tmem_wait_st();
+            return alpha;
+        };
+        for (int j = 0; j < n; ++j) {
+            const int e = e_cur;
+            const uint4 wv = w_cur;
+            if (j + 1 < n) {
+                w_cur = km[e_nxt >> 4];
+                e_cur = e_nxt;
+                e_nxt = j + 2 < n ? v.fwd_idx[p0 + j + 2] : 0;
+            }
+            const int kt = e >> 4, cls = e & 3;
+            if (!mbar_wait(&s_full[j & 1], (j >> 1) & 1, status, 301)) { ok = false; break; }
+            tc_fence_after();
+            // a tile whose first or second key half no row sees was computed as
+            // S = Q K_half^T (N = 64) over the first 64 columns of its buffer
+            const int lh = (e & MW_TILE_DEAD_LO) ? 1 : 0;
+            const uint32_t sbuf = lane_base + TM_S0 + (j & 1) * 128;
+            float alpha;
+            if (e & (MW_TILE_DEAD_LO | MW_TILE_DEAD_HI)) {
+                const uint32_t w0 = lh ? wv.z : wv.x, w1 = lh ? wv.w : wv.y;
+                alpha = soft_tile(std::integral_constant<int, 2>(), sbuf, true, 127, w0, w1, 0u, 0u);
+            } else {
+                alpha = soft_tile(std::integral_constant<int, 4>(), sbuf, cls != MW_TILE_FULL || kt == qt,
+                                  kt == qt ? ie - kt * 128 : 127, wv.x, wv.y, wv.z, wv.w);
             }
             // O was last written by PV_{j-1}; rescale it when the max moved
             if (j >= 1 && __any_sync(0xffffffffu, alpha != 1.f)) {
@@ -473,7 +512,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             load_tile(sm + DQ_Q, &tmQ, &q_full, h, row0);
             load_tile(sm + DQ_DO, &tmDO, &q_full, h, row0);
             for (int j = 0; j < n; ++j) {
-                const int kt = v.fwd_idx[p0 + j] >> 2;
+                const int kt = v.fwd_idx[p0 + j] >> 4;
                 const int s = j & 1;
                 const int row = (int)(tok0 + kt * 128);
                 if (j >= 2 && !mbar_wait(&v_empty[s], ((j - 2) >> 1) & 1, status, 111)) break;
@@ -556,16 +595,16 @@ __global__ void __launch_bounds__(NT_BWD, 1)
         // its S is ready
         int e_cur = n > 0 ? v.fwd_idx[p0] : 0;
         int e_nxt = n > 1 ? v.fwd_idx[p0 + 1] : 0;
-        uint4 w_cur = n > 0 ? km[e_cur >> 2] : make_uint4(0u, 0u, 0u, 0u);
+        uint4 w_cur = n > 0 ? km[e_cur >> 4] : make_uint4(0u, 0u, 0u, 0u);
         for (int j = 0; j < n; ++j) {
             const int e = e_cur;
             const uint4 wv = w_cur;
             if (j + 1 < n) {
-                w_cur = km[e_nxt >> 2];
+                w_cur = km[e_nxt >> 4];
                 e_cur = e_nxt;
                 e_nxt = j + 2 < n ? v.fwd_idx[p0 + j + 2] : 0;
             }
-            const int kt = e >> 2, cls = e & 3;
+            const int kt = e >> 4, cls = e & 3;
             if (!mbar_wait(&s_full[j & 1], (j >> 1) & 1, status, 311)) { ok = false; break; }
             tc_fence_after();
             float s[64];
@@ -757,7 +796,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
     struct Cursor {
         int e, rem, qt, qt_next;
     };
-    auto list_qt = [&](int e) -> int { return e >= 0 ? v.bwd_idx[p0 + e] >> 2 : 0; };
+    auto list_qt = [&](int e) -> int { return e >= 0 ? v.bwd_idx[p0 + e] >> 4 : 0; };
     const Cursor first{nlist - 1, 0, list_qt(nlist - 1), list_qt(nlist - 2)};
     auto advance = [&](Cursor& c) {
         if (++c.rem == 2 * grp) {

@@ -51,7 +51,7 @@ extern "C" const char* mw_status_str(int s) {
 }
 
 extern "C" int mw_last_cuda_error(void) { return g_last_cuda_error; }
-extern "C" int mw_abi_version(void) { return 2; }
+extern "C" int mw_abi_version(void) { return 3; }
 extern "C" uint64_t mw_kernel_launches(void) { return (uint64_t)g_launches.load(std::memory_order_relaxed); }
 
 static mw_status check_shape(int n_traj, const int32_t* cu, int n_junc, const int32_t* jt,
@@ -119,7 +119,7 @@ extern "C" mw_status mw_visibility_layout(int n_traj, const int32_t* cu, int n_j
     L->vis_bytes = o;
     o = 0;
     L->ws_off_spans = take(12 * (int64_t)n_spans);
-    L->ws_off_tstat = take(8 * tiles);
+    L->ws_off_tstat = take(16 * tiles);
     L->ws_off_cnt = take(8 * tiles);
     L->ws_bytes = o;
     return MW_OK;
@@ -152,7 +152,7 @@ struct BuildArgs {
     unsigned long long* pairs;
     uint32_t* keymask;
     const int32_t* spans;   // [n_spans][3]
-    int32_t* tstat;         // [n_tiles][2]
+    int32_t* tstat;         // [n_tiles][4] min, max lifetime; max over keys 0..63, 64..127
     int32_t* fwd_cnt;       // [n_tiles]
     int32_t* bwd_cnt;       // [n_tiles]
 };
@@ -227,20 +227,26 @@ __global__ void k_tile_stats(BuildArgs a) {
     if (threadIdx.x == 0) {
         int mn = min(min(smin[0], smin[1]), min(smin[2], smin[3]));
         int mx = max(max(smax[0], smax[1]), max(smax[2], smax[3]));
-        a.tstat[2 * g] = mn;
-        a.tstat[2 * g + 1] = mx;
+        a.tstat[4 * g] = mn;
+        a.tstat[4 * g + 1] = mx;
+        a.tstat[4 * g + 2] = max(smax[0], smax[1]);   // keys 0..63 (INT32_MIN when none in range)
+        a.tstat[4 * g + 3] = max(smax[2], smax[3]);   // keys 64..127
         unsigned long long p = spair[0] + spair[1] + spair[2] + spair[3];
         atomicAdd(&a.pairs[b], p);
         atomicAdd(&a.pairs[a.n_traj], p);
     }
 }
 
-__device__ __forceinline__ int tile_class(int qt, int kt, int T, int kmin, int kmax) {
+// Class of tile (qt, kt) from its k-tile's lifetime statistics st = (min, max,
+// max over keys 0..63, max over keys 64..127). Off the diagonal every key
+// precedes every row, so row i sees key j iff i < omega(j): a key half is seen
+// by some row iff its largest lifetime exceeds the q-tile's first row.
+__device__ __forceinline__ int tile_class(int qt, int kt, int T, const int32_t* st) {
     int q0 = qt * MW_TILE, q1 = min(q0 + MW_TILE, T);
     if (kt == qt) return (q1 - q0 == 1) ? MW_TILE_FULL : MW_TILE_PARTIAL;
-    if (kmin >= q1) return MW_TILE_FULL;
-    if (kmax <= q0) return MW_TILE_EMPTY;
-    return MW_TILE_PARTIAL;
+    if (st[0] >= q1) return MW_TILE_FULL;
+    if (st[1] <= q0) return MW_TILE_EMPTY;
+    return MW_TILE_PARTIAL | (st[2] <= q0 ? MW_TILE_DEAD_LO : 0) | (st[3] <= q0 ? MW_TILE_DEAD_HI : 0);
 }
 
 // One warp per global q-tile: classes of (qt, 0..qt) and the fwd list length.
@@ -255,7 +261,7 @@ __global__ void k_classify(BuildArgs a) {
     uint8_t* row = a.cls + a.traj_tri[b] + (int64_t)qt * (qt + 1) / 2;
     int cnt = 0;
     for (int kt = lane; kt <= qt; kt += 32) {
-        int c = tile_class(qt, kt, T, a.tstat[2 * (tb + kt)], a.tstat[2 * (tb + kt) + 1]);
+        int c = tile_class(qt, kt, T, a.tstat + 4 * (tb + kt));
         row[kt] = (uint8_t)c;
         cnt += c != MW_TILE_EMPTY;
     }
@@ -347,7 +353,7 @@ __global__ void k_fill(BuildArgs a) {
         int kt = k0 + lane;
         int c = kt <= t ? tri[(int64_t)t * (t + 1) / 2 + kt] : MW_TILE_EMPTY;
         uint32_t m = __ballot_sync(0xffffffffu, c != MW_TILE_EMPTY);
-        if (c != MW_TILE_EMPTY) a.fwd_idx[base + __popc(m & lt)] = (kt << 2) | c;
+        if (c != MW_TILE_EMPTY) a.fwd_idx[base + __popc(m & lt)] = (kt << 4) | c;
         base += __popc(m);
     }
     base = a.bwd_ptr[g];
@@ -355,7 +361,7 @@ __global__ void k_fill(BuildArgs a) {
         int qt = q0 + lane;
         int c = qt < nt ? tri[(int64_t)qt * (qt + 1) / 2 + t] : MW_TILE_EMPTY;
         uint32_t m = __ballot_sync(0xffffffffu, c != MW_TILE_EMPTY);
-        if (c != MW_TILE_EMPTY) a.bwd_idx[base + __popc(m & lt)] = (qt << 2) | c;
+        if (c != MW_TILE_EMPTY) a.bwd_idx[base + __popc(m & lt)] = (qt << 4) | c;
         base += __popc(m);
     }
 }

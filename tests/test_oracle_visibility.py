@@ -138,6 +138,39 @@ def test_tile_classes_brute_force(seed):
             assert cls[q, k] == want
 
 
+@pytest.mark.parametrize("seed", range(8))
+def test_dead_halves_brute_force(seed):
+    """A key half of a PARTIAL off-diagonal tile is flagged dead exactly when
+    the dense mask has no visible pair between the q-tile's rows and that
+    half's keys (keys past the end count as dead); never both halves, never
+    on FULL or diagonal tiles."""
+    rng = np.random.default_rng(300 + seed)
+    tile = 16
+    T = int(rng.integers(40, 260))
+    edits = _random_edits(T, rng, int(rng.integers(1, 7)))
+    mask = V.dense_mask(T, edits)
+    cls, _ = V.tile_classes(T, edits, tile=tile)
+    dead = V.dead_halves(T, edits, cls, tile=tile)
+    nt = (T + tile - 1) // tile
+    h = tile // 2
+    seen = 0
+    for q in range(nt):
+        for k in range(q + 1):
+            if cls[q, k] != V.PARTIAL or k == q:
+                assert dead[q, k] == 0
+                continue
+            rows = mask[q * tile:(q + 1) * tile]
+            want = 0
+            for hh, bit in ((0, V.DEAD_LO), (1, V.DEAD_HI)):
+                blk = rows[:, k * tile + hh * h:k * tile + (hh + 1) * h]
+                if not blk.any():
+                    want |= bit
+            assert dead[q, k] == want, (q, k)
+            assert want != V.DEAD_LO | V.DEAD_HI
+            seen += want != 0
+    assert seen > 0 or seed > 3   # the generator's evictions leave dead halves in most records
+
+
 def test_build_lists_and_pairs():
     r = synth.config_record(1)
     out = V.build(r.seqlens, r.edits, tile=V.TILE)
@@ -145,14 +178,14 @@ def test_build_lists_and_pairs():
     mask = V.dense_mask(T, r.edits[0])
     assert out["pairs_total"] == int(mask.sum())
     # fwd and bwd lists name the same tiles with the same classes
-    fwd = {(q, e >> 2, e & 3) for q in range(len(out["fwd_ptr"]) - 1)
+    fwd = {(q, e >> 4, e & 15) for q in range(len(out["fwd_ptr"]) - 1)
            for e in out["fwd_idx"][out["fwd_ptr"][q]:out["fwd_ptr"][q + 1]]}
-    bwd = {(e >> 2, k, e & 3) for k in range(len(out["bwd_ptr"]) - 1)
+    bwd = {(e >> 4, k, e & 15) for k in range(len(out["bwd_ptr"]) - 1)
            for e in out["bwd_idx"][out["bwd_ptr"][k]:out["bwd_ptr"][k + 1]]}
     assert fwd == bwd
     # every visible pair lies in a listed tile
     for (q, k, c) in fwd:
-        assert c in (V.PARTIAL, V.FULL)
+        assert c & 3 in (V.PARTIAL, V.FULL)
     nt = (T + 127) // 128
     listed = np.zeros((nt, nt), dtype=bool)
     for (q, k, _) in fwd:
