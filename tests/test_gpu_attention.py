@@ -133,6 +133,31 @@ def test_fp32_tile_edges():
     assert_rel(np64(dV), dVr, 1e-4, "dV")
 
 
+def test_later_edit_leaves_earlier_rows_unchanged():
+    """The conditioning invariant on the GPU path (§3.3): adding a junction at
+    row 600 that evicts tokens 100..399 changes nothing for rows before 600 --
+    their attention outputs, log-sum-exps and the log-probs scored from them
+    are bitwise equal (same visible keys, same tiles, same arithmetic order)."""
+    import paper_2609_00865_gb300 as mw
+    T, Hq, Hkv, Dh = 700, 8, 2, 128
+    base = [(200, [(20, 150)]), (450, [(160, 300)])]
+    later = base + [(600, [(100, 400)])]
+    Q, K, V, dO = _tensors(T, Hq, Hkv, Dh, 71, torch.bfloat16)
+    out = []
+    W = synth.normal((5000, Hq * Dh), 72, std=0.02).to(torch.bfloat16).cuda()
+    tg = synth.uniform_int(T, 5000, 73).cuda()
+    rows = torch.arange(0, 600, 3, dtype=torch.int32, device="cuda")
+    zeros = torch.zeros(rows.numel(), dtype=torch.float32, device="cuda")
+    for edits in (base, later):
+        O, LSE, *_ = _run([T], [edits], Q, K, V, dO, Dh ** -0.5)
+        lp = mw.logprob_loss_fwd(O.reshape(T, Hq * Dh), W, tg, rows, zeros, zeros)["lp"]
+        torch.cuda.synchronize()
+        out.append((O[:600].clone(), LSE[:, :600].clone(), lp.clone()))
+    assert torch.equal(out[0][0], out[1][0])
+    assert torch.equal(out[0][1], out[1][1])
+    assert torch.equal(out[0][2], out[1][2])
+
+
 def test_no_edits_is_causal_attention():
     """K = 0 reduces to ordinary causal attention (library SDPA on the GPU
     output's inputs, float64 on the CPU)."""
