@@ -147,8 +147,9 @@ def job_value(scored_per_rank, world, ms):
     return scored_per_rank * world / (ms * 1e-3)
 
 
-def make_workload(cfg, K=None, f=None, seed_offset=0, n_traj=None):
-    """Host-side inputs of one workload (pinned CPU tensors + record).
+def make_workload(cfg, K=None, f=None, seed_offset=0, n_traj=None, pin=True):
+    """Host-side inputs of one workload (CPU tensors, pinned unless ``pin`` is
+    False, + record).
 
     ``n_traj`` keeps only the first trajectories of the record (a smaller
     case of the same kernels, for profiler captures)."""
@@ -165,7 +166,8 @@ def make_workload(cfg, K=None, f=None, seed_offset=0, n_traj=None):
         t = torch.randn(*shape, generator=g, dtype=torch.float32)
         if std != 1.0:
             t.mul_(std)
-        return t.to(bf).pin_memory()
+        t = t.to(bf)
+        return t.pin_memory() if pin else t
 
     if cfg in (2, 4, 5):
         rec = synth.config_record(cfg, K=K, f=f)
@@ -189,11 +191,14 @@ def make_workload(cfg, K=None, f=None, seed_offset=0, n_traj=None):
             rows = w["record"].loss_rows()
         w["N"], w["d"], w["Vocab"] = N, d, c["V"]
         w["W"] = randn(c["V"], d, std=0.02)
-        w["targets"] = torch.randint(0, c["V"], (N,), generator=g, dtype=torch.int32).pin_memory()
-        w["rows"] = torch.tensor(rows, dtype=torch.int32).pin_memory()
+        w["targets"] = torch.randint(0, c["V"], (N,), generator=g, dtype=torch.int32)
+        w["rows"] = torch.tensor(rows, dtype=torch.int32)
         M = len(rows)
-        w["adv"] = torch.randn(M, generator=g).pin_memory()
-        w["noise"] = (0.05 * torch.randn(M, generator=g)).pin_memory()
+        w["adv"] = torch.randn(M, generator=g)
+        w["noise"] = 0.05 * torch.randn(M, generator=g)
+        if pin:
+            for k in ("targets", "rows", "adv", "noise"):
+                w[k] = w[k].pin_memory()
     return w
 
 
@@ -413,7 +418,7 @@ def cpu_sample(w, budget_s=15.0):
 def run_reference(args, rank, world):
     if rank != 0:
         return
-    w = make_workload(args.config, args.K, args.f, n_traj=args.n_traj)
+    w = make_workload(args.config, args.K, args.f, n_traj=args.n_traj, pin=False)   # the oracle runs on the host
     vals = []
     for i in range(args.warmup + args.steps):
         v, cores, desc = cpu_sample(w, budget_s=args.cpu_seconds / max(1, args.steps))
