@@ -221,6 +221,26 @@ mw_status mw_logprob_loss_fwd(const void* H, const void* W, const int32_t* targe
                               void* ws, void* stream);
 
 /*
+ * mw_logprob_loss_fwd plus the KL-to-reference term of GRPO training (App. F.1:
+ * coefficient beta, "low-variance estimator"), read as the k3 estimate per loss
+ * row with d_m = lp_ref_m - lp_m:
+ *   loss += beta * (1/M) sum_m (exp(d_m) - d_m - 1),
+ *   dL/dlp_m gains beta * (1 - exp(d_m)) / M (kept in `ws` for the backward,
+ *   which is unchanged).
+ *   lp_ref [M] float32 (device): the reference policy's log-prob of each loss
+ *   row's target. beta >= 0 and finite, else MW_EINVAL; beta > 0 with M > 0
+ *   requires lp_ref (MW_EINVAL); beta = 0 ignores lp_ref and equals
+ *   mw_logprob_loss_fwd. The paper has no closed form for the estimator; k3 is
+ *   the standard low-variance one.
+ */
+mw_status mw_logprob_loss_fwd_kl(const void* H, const void* W, const int32_t* targets,
+                                 const int32_t* rows, int M, const float* lp_old, const float* adv,
+                                 float eps_lo, float eps_hi, const float* lp_ref, float beta,
+                                 int N, int d, int Vocab, int dtype,
+                                 float* lp, float* ratio, float* lse, float* loss,
+                                 void* ws, void* stream);
+
+/*
  * Backward of mw_logprob_loss_fwd, scaled by the upstream gradient dloss:
  *   dz_{m,v} = dloss * g_m * (1[v = target] - softmax_v(z_m)),
  *   dH_t = sum_v dz_{m,v} W_v (rows outside `rows` get 0),

@@ -47,7 +47,17 @@ def logprob(H, W, targets, rows):
     return lp, lse
 
 
-def policy_loss(lp, lp_old, adv, eps_lo, eps_hi, dloss=1.0):
+def kl_k3(lp, lp_ref):
+    """Low-variance estimate of KL(pi_theta || pi_ref) per token (App. F.1 trains
+    with a KL coefficient and "the low-variance estimator"; the paper gives no
+    formula, and this is the standard one, k3): with ``d = lp_ref - lp``,
+    ``k3 = exp(d) - d - 1`` (>= 0, zero iff d = 0) and ``dk3/dlp = 1 - exp(d)``.
+    Returns ``(k3, dk3/dlp)``."""
+    d = np.asarray(lp_ref, dtype=np.float64) - np.asarray(lp, dtype=np.float64)
+    return np.expm1(d) - d, -np.expm1(d)
+
+
+def policy_loss(lp, lp_old, adv, eps_lo, eps_hi, dloss=1.0, lp_ref=None, beta=0.0):
     """Ratio, clipped surrogate, mean loss and ``g_t = dL/dlp_t``.
 
     ``rho = exp(lp - lp_old)``; ``l_t = -min(rho A, clip(rho) A)``;
@@ -56,7 +66,9 @@ def policy_loss(lp, lp_old, adv, eps_lo, eps_hi, dloss=1.0):
     strictly smaller, which happens exactly when ``A > 0, rho > 1 + eps_hi``
     or ``A < 0, rho < 1 - eps_lo``; there the surrogate is flat in lp and the
     gradient is 0. At equality both terms coincide and the unclipped branch
-    is used. ``dloss`` scales the gradient (upstream dL).
+    is used. ``dloss`` scales the gradient (upstream dL). With ``lp_ref`` and
+    ``beta`` each token adds ``beta * k3`` (``kl_k3``) to its loss term and
+    ``beta * dk3/dlp / M`` to ``g``.
     """
     lp = np.asarray(lp, dtype=np.float64)
     lp_old = np.asarray(lp_old, dtype=np.float64)
@@ -69,6 +81,11 @@ def policy_loss(lp, lp_old, adv, eps_lo, eps_hi, dloss=1.0):
     loss = per_tok.mean() if M else 0.0
     flat = clipped < unclipped
     g = np.where(flat, 0.0, -adv * ratio) / max(M, 1) * dloss
+    if lp_ref is not None and beta:
+        k3, dk3 = kl_k3(lp, lp_ref)
+        per_tok = per_tok + beta * k3
+        loss = per_tok.mean() if M else 0.0
+        g = g + beta * dk3 / max(M, 1) * dloss
     return ratio, per_tok, loss, g
 
 

@@ -25,6 +25,7 @@ from ._lib import (  # noqa: F401
     mw_logprob_check_status,
     mw_logprob_loss_bwd,
     mw_logprob_loss_fwd,
+    mw_logprob_loss_fwd_kl,
     mw_logprob_ws,
     mw_masked_attn_bwd,
     mw_masked_attn_bwd_ws,

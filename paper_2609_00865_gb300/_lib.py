@@ -57,6 +57,8 @@ _SIGS = {
     "mw_masked_attn_bwd": (_I, [_LP, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _F, _P, _P]),
     "mw_logprob_ws": (_I, [_I, _I, _I, _I, _I, ctypes.POINTER(ctypes.c_size_t)]),
     "mw_logprob_loss_fwd": (_I, [_P, _P, _P, _P, _I, _P, _P, _F, _F, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P]),
+    "mw_logprob_loss_fwd_kl": (_I, [_P, _P, _P, _P, _I, _P, _P, _F, _F, _P, _F, _I, _I, _I, _I, _P, _P, _P, _P, _P,
+                                    _P]),
     "mw_logprob_loss_bwd": (_I, [_P, _P, _P, _P, _I, _I, _I, _I, _I, _P, _P, _F, _P, _P, _P]),
     "mw_check_status": (_I, [_LP, _P, _P]),
     "mw_logprob_check_status": (_I, [_I, _I, _I, _I, _I, _P, _P]),
@@ -314,8 +316,19 @@ def mw_logprob_loss_fwd(H, W, targets, rows, lp_old, adv, eps_lo, eps_hi, lp, ra
                                       _stream(stream)), "mw_logprob_loss_fwd")
 
 
-def logprob_loss_fwd(H, W, targets, rows, lp_old, adv, eps_lo=0.2, eps_hi=0.2, stream=None):
-    """Allocate outputs + workspace; returns dict(lp, ratio, lse, loss, ws)."""
+def mw_logprob_loss_fwd_kl(H, W, targets, rows, lp_old, adv, eps_lo, eps_hi, lp_ref, beta, lp, ratio, lse, loss,
+                           ws, stream=None):
+    N, d = H.shape
+    _check(_lib().mw_logprob_loss_fwd_kl(_ptr(H), _ptr(W), _ptr(targets), _ptr(rows), int(rows.numel()),
+                                         _ptr(lp_old), _ptr(adv), float(eps_lo), float(eps_hi), _ptr(lp_ref),
+                                         float(beta), N, d, W.shape[0], _dtype_code(H), _ptr(lp), _ptr(ratio),
+                                         _ptr(lse), _ptr(loss), _ptr(ws), _stream(stream)), "mw_logprob_loss_fwd_kl")
+
+
+def logprob_loss_fwd(H, W, targets, rows, lp_old, adv, eps_lo=0.2, eps_hi=0.2, stream=None, lp_ref=None, beta=0.0):
+    """Allocate outputs + workspace; returns dict(lp, ratio, lse, loss, ws).
+    With ``lp_ref`` (float32 [M]) and ``beta`` > 0 the loss includes the KL
+    term of ``mw_logprob_loss_fwd_kl``."""
     import torch
     _need(H, "H")
     _need(W, "W", dtype=H.dtype)
@@ -329,8 +342,14 @@ def logprob_loss_fwd(H, W, targets, rows, lp_old, adv, eps_lo=0.2, eps_hi=0.2, s
                      dtype=torch.uint8, device=dev)
     out = {k: torch.empty(M, dtype=torch.float32, device=dev) for k in ("lp", "ratio", "lse")}
     out["loss"] = torch.empty(1, dtype=torch.float32, device=dev)
-    mw_logprob_loss_fwd(H, W, targets, rows, lp_old, adv, eps_lo, eps_hi, out["lp"], out["ratio"], out["lse"],
-                        out["loss"], ws, stream)
+    if lp_ref is not None or beta != 0.0:
+        if lp_ref is not None:
+            _need(lp_ref, "lp_ref", dtype=torch.float32)
+        mw_logprob_loss_fwd_kl(H, W, targets, rows, lp_old, adv, eps_lo, eps_hi, lp_ref, beta, out["lp"],
+                               out["ratio"], out["lse"], out["loss"], ws, stream)
+    else:
+        mw_logprob_loss_fwd(H, W, targets, rows, lp_old, adv, eps_lo, eps_hi, out["lp"], out["ratio"], out["lse"],
+                            out["loss"], ws, stream)
     out["ws"] = ws
     return out
 

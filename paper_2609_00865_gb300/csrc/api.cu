@@ -21,7 +21,8 @@ mw_status attn_fwd_tc(const mw_vis_layout*, const void*, const void*, const void
 mw_status attn_bwd_tc(const mw_vis_layout*, const void*, const void*, const void*, const void*, const void*,
                       const void*, const float*, void*, void*, void*, int, int, float, float*, cudaStream_t);
 int64_t attn_bwd_tc_ws(const mw_vis_layout*, int);
-__global__ void k_loss_epilogue(int, const float*, const float*, const float*, float, float, float*, float*, float*);
+__global__ void k_loss_epilogue(int, const float*, const float*, const float*, float, float, const float*, float, float*,
+                                float*, float*);
 
 struct LmPlan {
     int M_pad, R, NV, C, NVC, grid;
@@ -127,13 +128,17 @@ extern "C" mw_status mw_logprob_ws(int N, int M, int d, int V, int dtype, size_t
     return MW_OK;
 }
 
-extern "C" mw_status mw_logprob_loss_fwd(const void* H, const void* W, const int32_t* targets, const int32_t* rows,
-                                         int M, const float* lp_old, const float* adv, float eps_lo, float eps_hi,
-                                         int N, int d, int V, int dtype, float* lp, float* ratio, float* lse,
-                                         float* loss, void* ws, void* stream) {
+extern "C" mw_status mw_logprob_loss_fwd_kl(const void* H, const void* W, const int32_t* targets,
+                                            const int32_t* rows, int M, const float* lp_old, const float* adv,
+                                            float eps_lo, float eps_hi, const float* lp_ref, float beta, int N, int d,
+                                            int V, int dtype, float* lp, float* ratio, float* lse, float* loss,
+                                            void* ws, void* stream) {
     mw_status st = lm_args(N, M, d, V, dtype);
     if (st != MW_OK) return st;
     if (!(eps_lo >= 0.f && eps_lo < 1.f && eps_hi >= 0.f && isfinite(eps_hi))) return MW_EINVAL;
+    if (!(beta >= 0.f && isfinite(beta))) return MW_EINVAL;
+    if (beta > 0.f && M > 0 && !lp_ref) return MW_EINVAL;
+    if (beta == 0.f) lp_ref = nullptr;
     if (!loss || !ws) return MW_EINVAL;
     if (M > 0 && (!H || !W || !targets || !rows || !lp_old || !adv || !lp || !ratio || !lse)) return MW_EINVAL;
     cudaStream_t s = (cudaStream_t)stream;
@@ -149,8 +154,16 @@ extern "C" mw_status mw_logprob_loss_fwd(const void* H, const void* W, const int
     }
     if (st != MW_OK) return st;
     count_launches(1);
-    k_loss_epilogue<<<1, 1024, 0, s>>>(M, lp, lp_old, adv, eps_lo, eps_hi, ratio, g, loss);
+    k_loss_epilogue<<<1, 1024, 0, s>>>(M, lp, lp_old, adv, eps_lo, eps_hi, lp_ref, beta, ratio, g, loss);
     return launch_status();
+}
+
+extern "C" mw_status mw_logprob_loss_fwd(const void* H, const void* W, const int32_t* targets, const int32_t* rows,
+                                         int M, const float* lp_old, const float* adv, float eps_lo, float eps_hi,
+                                         int N, int d, int V, int dtype, float* lp, float* ratio, float* lse,
+                                         float* loss, void* ws, void* stream) {
+    return mw_logprob_loss_fwd_kl(H, W, targets, rows, M, lp_old, adv, eps_lo, eps_hi, nullptr, 0.f, N, d, V, dtype,
+                                  lp, ratio, lse, loss, ws, stream);
 }
 
 extern "C" mw_status mw_logprob_loss_bwd(const void* H, const void* W, const int32_t* targets, const int32_t* rows,

@@ -15,10 +15,14 @@
 namespace mw {
 
 // Shared by both LM-head paths: ratio, clipped surrogate, g, mean loss.
+// With lp_ref (may be null) each loss row also adds beta times the
+// low-variance KL estimate to the reference policy (App. F.1),
+//   k3 = exp(d) - d - 1 = expm1(d) - d,  d = lp_ref - lp,  dk3/dlp = -expm1(d).
 // One block of 1024 threads; the mean is reduced in a fixed order.
 __global__ void k_loss_epilogue(int M, const float* __restrict__ lp, const float* __restrict__ lp_old,
                                 const float* __restrict__ adv, float eps_lo, float eps_hi,
-                                float* __restrict__ ratio, float* __restrict__ gsave, float* __restrict__ loss) {
+                                const float* __restrict__ lp_ref, float beta, float* __restrict__ ratio,
+                                float* __restrict__ gsave, float* __restrict__ loss) {
     __shared__ float red[32];
     float part = 0.f;
     const float invM = M > 0 ? 1.f / (float)M : 0.f;
@@ -27,9 +31,16 @@ __global__ void k_loss_epilogue(int M, const float* __restrict__ lp, const float
         const float A = adv[m];
         const float unclipped = r * A;
         const float clipped = fminf(fmaxf(r, 1.f - eps_lo), 1.f + eps_hi) * A;
+        float g = (clipped < unclipped) ? 0.f : -A * r * invM;
         part += -fminf(unclipped, clipped);
+        if (lp_ref) {
+            const float d = lp_ref[m] - lp[m];
+            const float em1 = expm1f(d);
+            part += beta * (em1 - d);
+            g -= beta * em1 * invM;
+        }
         ratio[m] = r;
-        gsave[m] = (clipped < unclipped) ? 0.f : -A * r * invM;
+        gsave[m] = g;
     }
     part = warp_sum(part);
     if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = part;

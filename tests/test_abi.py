@@ -111,3 +111,9 @@ def test_attention_and_lmhead_reject_bad_args_on_host():
     assert h.mw_logprob_ws(10, 11, 128, 100, 0, ctypes.byref(n)) == 3
     assert h.mw_logprob_loss_fwd(P, P, P, P, 4, P, P, 1.5, 0.2, 10, 128, 100, 0, P, P, P, P, P, None) == 1
     assert h.mw_logprob_loss_fwd(P, P, P, P, 4, P, P, 0.2, 0.2, 10, 128, 100, 0, P, P, P, None, P, None) == 1
+    # KL term: negative or non-finite beta; beta > 0 without lp_ref
+    assert h.mw_logprob_loss_fwd_kl(P, P, P, P, 4, P, P, 0.2, 0.2, P, -1.0, 10, 128, 100, 0, P, P, P, P, P, None) == 1
+    assert h.mw_logprob_loss_fwd_kl(P, P, P, P, 4, P, P, 0.2, 0.2, P, float("nan"), 10, 128, 100, 0, P, P, P, P, P,
+                                    None) == 1
+    assert h.mw_logprob_loss_fwd_kl(P, P, P, P, 4, P, P, 0.2, 0.28, None, 1e-3, 10, 128, 100, 0, P, P, P, P, P,
+                                    None) == 1

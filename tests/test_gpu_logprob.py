@@ -120,6 +120,40 @@ def test_no_loss_rows(dtype):
     assert (dH == 0).all() and (dW == 0).all()
 
 
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+def test_kl_to_reference(dtype):
+    """The KL-to-reference term (App. F.1, low-variance k3 estimate) in the loss
+    and, through g, in dH and dW; asymmetric clip 0.2 / 0.28."""
+    import paper_2609_00865_gb300 as mw
+    N, d, V = 400, 128, 3000
+    rows = np.sort(np.random.default_rng(91).permutation(N)[:250])
+    H, W, targets, rows_t, lp_old, adv, lp_o, lse_o = _case(N, d, V, rows, 91, dtype)
+    M = len(rows)
+    lp_refpol = torch.tensor(lp_o + 0.2 * np.random.default_rng(92).standard_normal(M), dtype=torch.float32)
+    beta = 0.3
+    dev = [t.cuda() for t in (H, W, targets, rows_t, lp_old, adv)]
+    out = mw.logprob_loss_fwd(*dev, eps_lo=0.2, eps_hi=0.28, lp_ref=lp_refpol.cuda(), beta=beta)
+    dH, dW = mw.logprob_loss_bwd(dev[0], dev[1], dev[2], dev[3], out["lse"], out["ws"], 1.0)
+    torch.cuda.synchronize()
+    ratio_r, _, loss_r, g_r = OL.policy_loss(lp_o, np64(lp_old), np64(adv), 0.2, 0.28, lp_ref=np64(lp_refpol),
+                                             beta=beta)
+    edge = np.minimum(np.abs(ratio_r - 0.8), np.abs(ratio_r - 1.28)) < 1e-3
+    assert edge.sum() == 0
+    loss = float(out["loss"].item())
+    _, _, loss_plain, _ = OL.policy_loss(lp_o, np64(lp_old), np64(adv), 0.2, 0.28)
+    assert abs(loss_r - loss_plain) > 1e-3   # the term is not negligible here
+    assert abs(loss - loss_r) <= 1e-3 * max(abs(loss_r), np.mean(np.abs(ratio_r * np64(adv)))), (loss, loss_r)
+    dHr, dWr = OL.logprob_loss_bwd(np64(H), np64(W), targets.numpy(), rows, lse_o, g_r)
+    if dtype == torch.float32:
+        assert_rel(np64(out["lp"]), lp_o, 1e-4, "lp")
+        assert_rel(np64(dH), dHr, 1e-4, "dH")
+        assert_rel(np64(dW), dWr, 1e-4, "dW")
+    else:
+        assert_maxabs(np64(out["lp"]), lp_o, 1e-2, "lp")
+        assert_grad_bf16(np64(dH), dHr, "dH")
+        assert_grad_bf16(np64(dW), dWr, "dW")
+
+
 def test_config3_full_size_sampled():
     """N = 32,768, d = 1,536, V = 151,936, 70% loss rows, in the bench's launch
     configuration. lp / dH are checked on sampled rows, dW on sampled vocab

@@ -67,6 +67,48 @@ def test_policy_loss_gradient_equals_autograd():
     np.testing.assert_allclose(grad, x.grad.numpy(), rtol=1e-12, atol=1e-15)
 
 
+def test_kl_k3_is_unbiased_for_the_exact_kl():
+    """Averaged under pi_theta, the per-token estimate equals KL(pi_theta ||
+    pi_ref) computed directly from the two distributions; it is zero when
+    the policies agree and ~d^2 / 2 for a small log-ratio d."""
+    rng = np.random.default_rng(11)
+    for _ in range(5):
+        V = int(rng.integers(2, 40))
+        lp = np.log(rng.dirichlet(np.ones(V)))
+        lp_ref = np.log(rng.dirichlet(np.ones(V)))
+        k3, _ = LP.kl_k3(lp, lp_ref)
+        p = np.exp(lp)
+        exact_kl = float(np.sum(p * (lp - lp_ref)))
+        assert float(np.sum(p * k3)) == pytest.approx(exact_kl, rel=1e-12, abs=1e-14)
+    k3, dk3 = LP.kl_k3(np.array([-1.5, -0.2]), np.array([-1.5, -0.2]))
+    assert (k3 == 0).all() and (dk3 == 0).all()
+    d = 1e-4
+    k3, _ = LP.kl_k3(np.array([0.0]), np.array([d]))
+    assert k3[0] == pytest.approx(d * d / 2, rel=1e-3)
+
+
+def test_policy_loss_with_kl_gradient_equals_autograd():
+    g = np.random.default_rng(5)
+    lp = g.standard_normal(150) * 0.3 - 2.0
+    lp_old = lp + g.standard_normal(150) * 0.3
+    lp_ref = lp + g.standard_normal(150) * 0.5
+    adv = g.standard_normal(150)
+    _, _, loss, grad = LP.policy_loss(lp, lp_old, adv, 0.2, 0.28, dloss=0.9, lp_ref=lp_ref, beta=0.3)
+    x = torch.tensor(lp, requires_grad=True)
+    r = torch.exp(x - torch.tensor(lp_old))
+    a = torch.tensor(adv)
+    ratio_ref = torch.exp(torch.tensor(lp_ref) - x)          # pi_ref / pi_theta
+    kl = ratio_ref - torch.log(ratio_ref) - 1.0
+    L = (-torch.minimum(r * a, torch.clamp(r, 0.8, 1.28) * a) + 0.3 * kl).mean()
+    (0.9 * L).backward()
+    assert loss == pytest.approx(L.item(), rel=1e-13)
+    np.testing.assert_allclose(grad, x.grad.numpy(), rtol=1e-12, atol=1e-15)
+    # beta = 0 or no reference: the plain clipped loss
+    _, _, l0, g0 = LP.policy_loss(lp, lp_old, adv, 0.2, 0.28, lp_ref=lp_ref, beta=0.0)
+    _, _, l1, g1 = LP.policy_loss(lp, lp_old, adv, 0.2, 0.28)
+    assert l0 == l1 and (g0 == g1).all()
+
+
 def test_backward_equals_autograd():
     N, d, V, M = 30, 12, 200, 17
     H, W, t, rows = _case(N, d, V, M, 4)
