@@ -531,47 +531,77 @@ __global__ void __launch_bounds__(NT_BWD, 1)
                            sv = smem_u32(sm + DQ_V);
             bool ok = mbar_wait(&q_full, 0, status, 211);
             // S_j (needs K_j and a free S buffer)
-            auto issue_s = [&](int j) -> bool {
+            // A tile whose first or second key half no row sees is computed over
+            // the live half only: S and dP with N = 64, dQ += dS K with K = 64
+            const uint32_t iKK64 = idesc_bf16(128, 64, 0, 0);
+            auto issue_s = [&](int j, int e) -> bool {
                 const int s = j & 1;
                 if (!mbar_wait(&k_full[s], (j >> 1) & 1, status, 212)) return false;
                 if (j >= 2 && !mbar_wait(&s_free[s], ((j - 2) >> 1) & 1, status, 213)) return false;
                 tc_fence_after();
+                if (e & (MW_TILE_DEAD_LO | MW_TILE_DEAD_HI)) {
+                    // the live half's 64 keys: rows 64 lh.. of each 64-column panel
+                    const uint32_t kh = sk + s * TILE_B + ((e & MW_TILE_DEAD_LO) ? 64u * 128u : 0u);
 #pragma unroll
-                for (int ks = 0; ks < 8; ++ks)
-                    mma_ss(tmem + TM_S0 + s * 128, kmaj(sq, ks), kmaj(sk + s * TILE_B, ks), iKK, ks > 0);
+                    for (int ks = 0; ks < 8; ++ks) mma_ss(tmem + TM_S0 + s * 128, kmaj(sq, ks), kmaj(kh, ks), iKK64, ks > 0);
+                } else {
+#pragma unroll
+                    for (int ks = 0; ks < 8; ++ks)
+                        mma_ss(tmem + TM_S0 + s * 128, kmaj(sq, ks), kmaj(sk + s * TILE_B, ks), iKK, ks > 0);
+                }
                 mma_commit(&s_full[s]);
                 return true;
             };
             // dP_j (needs V_j and the softmax to have read dP_{j-1})
-            auto issue_dp = [&](int j) -> bool {
+            auto issue_dp = [&](int j, int e) -> bool {
                 const int s = j & 1;
                 if (!mbar_wait(&v_full[s], (j >> 1) & 1, status, 214)) return false;
                 if (j >= 1 && !mbar_wait(&dp_free, (j - 1) & 1, status, 215)) return false;
                 tc_fence_after();
+                if (e & (MW_TILE_DEAD_LO | MW_TILE_DEAD_HI)) {
+                    const uint32_t vh = sv + s * TILE_B + ((e & MW_TILE_DEAD_LO) ? 64u * 128u : 0u);
 #pragma unroll
-                for (int ks = 0; ks < 8; ++ks)
-                    mma_ss(tmem + TM_DP, kmaj(sdo, ks), kmaj(sv + s * TILE_B, ks), iKK, ks > 0);
+                    for (int ks = 0; ks < 8; ++ks) mma_ss(tmem + TM_DP, kmaj(sdo, ks), kmaj(vh, ks), iKK64, ks > 0);
+                } else {
+#pragma unroll
+                    for (int ks = 0; ks < 8; ++ks)
+                        mma_ss(tmem + TM_DP, kmaj(sdo, ks), kmaj(sv + s * TILE_B, ks), iKK, ks > 0);
+                }
                 mma_commit(&v_empty[s]);
                 mma_commit(&dp_full);
                 return true;
             };
             // dQ += dS_t K_t, dS_t (bf16 pairs) read from TMEM: keys 0..63 in
             // columns 0..31 and keys 64..127 in columns 64..95 of S buffer t & 1
+            // (half tile: the live half's keys 0..31 in columns 0..15, keys
+            // 32..63 in columns 32..47; K rows from 16-row k-step 4 lh on)
             auto issue_dq = [&](int t) -> bool {
+                const int e = v.fwd_idx[p0 + t];
                 if (!mbar_wait(&ds_full[t & 1], (t >> 1) & 1, status, 216)) return false;
                 tc_fence_after();
                 const uint32_t da = tmem + TM_S0 + (t & 1) * 128;
+                if (e & (MW_TILE_DEAD_LO | MW_TILE_DEAD_HI)) {
+                    const int kh = (e & MW_TILE_DEAD_LO) ? 4 : 0;
 #pragma unroll
-                for (int ks = 0; ks < 8; ++ks)
-                    mma_ts(tmem + TM_DQ, da + (ks < 4 ? 8 * ks : 64 + 8 * (ks - 4)), mnmaj(sk + (t & 1) * TILE_B, ks),
-                           iMN, (t > 0 || ks > 0));
+                    for (int ks = 0; ks < 4; ++ks)
+                        mma_ts(tmem + TM_DQ, da + (ks < 2 ? 8 * ks : 32 + 8 * (ks - 2)),
+                               mnmaj(sk + (t & 1) * TILE_B, ks + kh), iMN, (t > 0 || ks > 0));
+                } else {
+#pragma unroll
+                    for (int ks = 0; ks < 8; ++ks)
+                        mma_ts(tmem + TM_DQ, da + (ks < 4 ? 8 * ks : 64 + 8 * (ks - 4)),
+                               mnmaj(sk + (t & 1) * TILE_B, ks), iMN, (t > 0 || ks > 0));
+                }
                 mma_commit(&k_empty[t & 1]);
                 mma_commit(&s_free[t & 1]);
                 mma_commit(&dq_done);
                 return true;
             };
             if (warp == 1) {
-                for (int j = 0; ok && j < n; ++j) ok = issue_s(j) && issue_dp(j);
+                for (int j = 0; ok && j < n; ++j) {
+                    const int e = v.fwd_idx[p0 + j];
+                    ok = issue_s(j, e) && issue_dp(j, e);
+                }
             } else {
                 // dQ's K-stage release also covers S_j: dS_j exists only once S_j is done
                 for (int j = 0; ok && j < n; ++j) ok = issue_dq(j);
@@ -596,6 +626,66 @@ __global__ void __launch_bounds__(NT_BWD, 1)
         int e_cur = n > 0 ? v.fwd_idx[p0] : 0;
         int e_nxt = n > 1 ? v.fwd_idx[p0 + 1] : 0;
         uint4 w_cur = n > 0 ? km[e_cur >> 4] : make_uint4(0u, 0u, 0u, 0u);
+        // One k-tile for this thread's NC 32-key chunks (2: its 64 keys of a
+        // full tile; 1: its 32 of a live half), S and dP read at columns scol /
+        // dcol: P = 2^(S c - LSE2), two elements per instruction, masked pairs
+        // entering the exp2 as -inf (P = +0) instead of branching around it;
+        // dS = P (dP - Delta) as bf16 pairs over the first NC * 16 of its own S
+        // columns, which only this thread has read.
+        auto dq_step = [&](auto ncc, int j, uint32_t scol, uint32_t dcol, uint32_t w0, uint32_t w1) -> bool {
+            constexpr int NC = decltype(ncc)::value;
+            float s[NC * 32];
+            {   // all loads in flight before one wait
+                uint32_t rr[NC][32];
+#pragma unroll
+                for (int c = 0; c < NC; ++c) tmem_ld32(scol + c * 32, rr[c]);
+                tmem_wait_ld();
+#pragma unroll
+                for (int c = 0; c < NC; ++c)
+#pragma unroll
+                    for (int x = 0; x < 32; ++x) s[c * 32 + x] = __uint_as_float(rr[c][x]);
+            }
+            if (__all_sync(0xffffffffu, (NC == 2 ? (w0 & w1) : w0) == 0xffffffffu)) {
+#pragma unroll
+                for (int x = 0; x < NC * 16; ++x) {
+                    const uint64_t a = fma2(f2(s[2 * x], s[2 * x + 1]), c2, n2);
+                    s[2 * x] = ex2(f2_lo(a));
+                    s[2 * x + 1] = ex2(f2_hi(a));
+                }
+            } else {
+#pragma unroll
+                for (int x = 0; x < NC * 16; ++x) {
+                    const uint32_t wm = x < 16 ? w0 : w1;
+                    const int bit = (2 * x) & 31;
+                    const uint64_t a = fma2(f2(s[2 * x], s[2 * x + 1]), c2, n2);
+                    s[2 * x] = ex2(((wm >> bit) & 1u) ? f2_lo(a) : -INFINITY);
+                    s[2 * x + 1] = ex2(((wm >> (bit + 1)) & 1u) ? f2_hi(a) : -INFINITY);
+                }
+            }
+            if (!mbar_wait(&dp_full, j & 1, status, 312)) return false;
+            tc_fence_after();
+            uint32_t dpr[NC][32];   // all dP loads in flight before one wait
+#pragma unroll
+            for (int cc = 0; cc < NC; ++cc) tmem_ld32(dcol + cc * 32, dpr[cc]);
+            tmem_wait_ld();
+            tc_fence_before();
+            mbar_arrive(&dp_free);
+#pragma unroll
+            for (int cc = 0; cc < NC; ++cc) {
+                const uint32_t* dp = dpr[cc];
+                uint32_t pk[16];
+#pragma unroll
+                for (int x = 0; x < 16; ++x) {
+                    const int c0 = cc * 32 + 2 * x;
+                    const uint64_t d = mul2(f2(s[c0], s[c0 + 1]),
+                                            sub2(f2(__uint_as_float(dp[2 * x]), __uint_as_float(dp[2 * x + 1])), dl2));
+                    pk[x] = pack_bf16(f2_lo(d), f2_hi(d));
+                }
+                tmem_st16(scol + 16 * cc, pk);
+            }
+            tmem_wait_st();
+            return true;
+        };
         for (int j = 0; j < n; ++j) {
             const int e = e_cur;
             const uint4 wv = w_cur;
@@ -607,74 +697,30 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             const int kt = e >> 4, cls = e & 3;
             if (!mbar_wait(&s_full[j & 1], (j >> 1) & 1, status, 311)) { ok = false; break; }
             tc_fence_after();
-            float s[64];
-            {   // both loads in flight before one wait
-                uint32_t rr[2][32];
+            const uint32_t sbuf = lane_base + TM_S0 + (j & 1) * 128;
+            bool stepok;
+            if (e & (MW_TILE_DEAD_LO | MW_TILE_DEAD_HI)) {
+                // the live half's 64 keys, 32 per warp of the lane quarter
+                const bool hi_half = (e & MW_TILE_DEAD_LO) != 0;
+                const uint32_t wm = hi_half ? (ch ? wv.w : wv.z) : (ch ? wv.y : wv.x);
+                stepok = dq_step(std::integral_constant<int, 1>(), j, sbuf + 32 * ch, lane_base + TM_DP + 32 * ch, wm, 0u);
+            } else {
+                uint32_t wd[4] = {0xffffffffu, 0xffffffffu, 0xffffffffu, 0xffffffffu};
+                if (cls != MW_TILE_FULL || kt == qt) {
+                    wd[0] = wv.x; wd[1] = wv.y; wd[2] = wv.z; wd[3] = wv.w;
+                    if (kt == qt) {
+                        const int lim = ie - kt * 128;
 #pragma unroll
-                for (int c = 0; c < 2; ++c) tmem_ld32(lane_base + TM_S0 + (j & 1) * 128 + (2 * ch + c) * 32, rr[c]);
-                tmem_wait_ld();
-#pragma unroll
-                for (int c = 0; c < 2; ++c)
-#pragma unroll
-                    for (int x = 0; x < 32; ++x) s[c * 32 + x] = __uint_as_float(rr[c][x]);
-            }
-            uint32_t wd[4] = {0xffffffffu, 0xffffffffu, 0xffffffffu, 0xffffffffu};
-            if (cls != MW_TILE_FULL || kt == qt) {
-                wd[0] = wv.x; wd[1] = wv.y; wd[2] = wv.z; wd[3] = wv.w;
-                if (kt == qt) {
-                    const int lim = ie - kt * 128;
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        const int hi = lim - 32 * q;
-                        wd[q] &= hi >= 31 ? 0xffffffffu : (hi < 0 ? 0u : ((2u << hi) - 1u));
+                        for (int q = 0; q < 4; ++q) {
+                            const int hi = lim - 32 * q;
+                            wd[q] &= hi >= 31 ? 0xffffffffu : (hi < 0 ? 0u : ((2u << hi) - 1u));
+                        }
                     }
                 }
+                stepok = dq_step(std::integral_constant<int, 2>(), j, sbuf + 64 * ch, lane_base + TM_DP + 64 * ch,
+                                 ch ? wd[2] : wd[0], ch ? wd[3] : wd[1]);
             }
-            const uint32_t w0 = ch ? wd[2] : wd[0], w1 = ch ? wd[3] : wd[1];
-            // P = 2^(S c - LSE2), two elements per instruction; masked pairs
-            // enter the exp2 as -inf (P = +0) instead of branching around it
-            if (__all_sync(0xffffffffu, (w0 & w1) == 0xffffffffu)) {
-#pragma unroll
-                for (int x = 0; x < 32; ++x) {
-                    const uint64_t a = fma2(f2(s[2 * x], s[2 * x + 1]), c2, n2);
-                    s[2 * x] = ex2(f2_lo(a));
-                    s[2 * x + 1] = ex2(f2_hi(a));
-                }
-            } else {
-#pragma unroll
-                for (int x = 0; x < 32; ++x) {
-                    const uint32_t wm = x < 16 ? w0 : w1;
-                    const int bit = (2 * x) & 31;
-                    const uint64_t a = fma2(f2(s[2 * x], s[2 * x + 1]), c2, n2);
-                    s[2 * x] = ex2(((wm >> bit) & 1u) ? f2_lo(a) : -INFINITY);
-                    s[2 * x + 1] = ex2(((wm >> (bit + 1)) & 1u) ? f2_hi(a) : -INFINITY);
-                }
-            }
-            if (!mbar_wait(&dp_full, j & 1, status, 312)) { ok = false; break; }
-            tc_fence_after();
-            uint32_t dpr[2][32];   // both dP loads in flight before one wait
-#pragma unroll
-            for (int cc = 0; cc < 2; ++cc) tmem_ld32(lane_base + TM_DP + (2 * ch + cc) * 32, dpr[cc]);
-            tmem_wait_ld();
-            tc_fence_before();
-            mbar_arrive(&dp_free);
-            // dS = P (dP - Delta) as bf16 pairs over the first 32 of this warp's
-            // own 64 S columns, which only this thread has read
-            const uint32_t dst = lane_base + TM_S0 + (j & 1) * 128 + 64 * ch;
-#pragma unroll
-            for (int cc = 0; cc < 2; ++cc) {
-                const uint32_t* dp = dpr[cc];
-                uint32_t pk[16];
-#pragma unroll
-                for (int x = 0; x < 16; ++x) {
-                    const int c0 = cc * 32 + 2 * x;
-                    const uint64_t d = mul2(f2(s[c0], s[c0 + 1]),
-                                            sub2(f2(__uint_as_float(dp[2 * x]), __uint_as_float(dp[2 * x + 1])), dl2));
-                    pk[x] = pack_bf16(f2_lo(d), f2_hi(d));
-                }
-                tmem_st16(dst + 16 * cc, pk);
-            }
-            tmem_wait_st();
+            if (!stepok) { ok = false; break; }
             tc_fence_before();
             mbar_arrive(&ds_full[j & 1]);
         }
