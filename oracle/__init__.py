@@ -15,7 +15,10 @@ and slowly, in float64:
   M = M^causal (+) M^logical equation) as a second, independent formulation.
 * ``attention`` -- per-segment compact causal softmax attention (§4.1
   LogitTree: one forward per branch on that branch's own sequence), forward
-  and textbook backward, scattered back to physical rows.
+  and textbook backward, scattered back to physical rows; optionally with
+  rotary positions taken from each row's gap-free logical positions (§4.2).
+* ``visibility.logical_positions`` -- the rank of every key in every segment's
+  live view (§4.2 row-wise position reassignment).
 * ``logprob`` -- LM-head log-softmax, target gather, importance ratio and the
   clipped PPO/GRPO surrogate with its gradient (App. B.4 "Pitfall A, RL view";
   App. F.1 clip range), forward and backward.

@@ -15,6 +15,12 @@ Layouts (token-major, trajectories packed back to back):
 ``Q, O``: ``[T_total, Hq, Dh]``; ``K, V``: ``[T_total, Hkv, Dh]``;
 ``LSE``: ``[Hq, T_total]`` (natural log). Query head ``h`` reads KV head
 ``h // (Hq // Hkv)`` (contiguous GQA groups).
+
+Rotary positions (optional, ``rope_theta``): §4.2 gives every row position
+ids under which its visible keys form a gap-free sequence. On the compact
+sequence of a segment that is simply the compact index, so queries and keys
+are rotated by their index in ``view_s`` before the scores are taken, and the
+gradients are rotated back.
 """
 
 import numpy as np
@@ -34,6 +40,25 @@ def _segments(seqlens, edits_per_traj):
         base += T
 
 
+def rope(x, pos, theta, inverse=False):
+    """Rotary position embedding (RoFormer, Su et al. 2021) in the
+    rotate-half pairing: feature f (f < Dh/2) is paired with f + Dh/2 and the
+    pair is turned by the angle ``pos * theta ** (-2 f / Dh)``. ``x`` is
+    ``[n, ..., Dh]`` with one position per leading index; ``inverse`` turns by
+    the opposite angle (the transpose of the rotation).
+    """
+    x = np.asarray(x, dtype=np.float64)
+    half = x.shape[-1] // 2
+    w = float(theta) ** (-2.0 * np.arange(half, dtype=np.float64) / x.shape[-1])
+    ang = np.asarray(pos, dtype=np.float64)[:, None] * w[None, :]
+    if inverse:
+        ang = -ang
+    ang = ang.reshape((ang.shape[0],) + (1,) * (x.ndim - 2) + (half,))
+    c, s = np.cos(ang), np.sin(ang)
+    a, b = x[..., :half], x[..., half:]
+    return np.concatenate([a * c - b * s, b * c + a * s], axis=-1)
+
+
 def _scores(q, k, scale, compact_rows):
     """Scaled scores of compact rows against the compact keys, causal.
 
@@ -46,12 +71,13 @@ def _scores(q, k, scale, compact_rows):
     return s
 
 
-def attn_fwd(seqlens, edits_per_traj, Q, K, V, scale, rows=None, heads=None):
+def attn_fwd(seqlens, edits_per_traj, Q, K, V, scale, rows=None, heads=None, rope_theta=None):
     """Masked GQA attention forward via per-segment compact sequences.
 
     Returns ``(O_sel, LSE_sel)`` for the selected global rows (default: all)
     and query heads (default: all): ``O_sel[r, h_i, :]``, ``LSE_sel[h_i, r]``.
     Softmax over each row's visible keys exactly (no large-negative fill).
+    With ``rope_theta`` queries and keys are rotated by their compact index.
     """
     Q = np.asarray(Q, dtype=np.float64)
     K = np.asarray(K, dtype=np.float64)
@@ -80,6 +106,9 @@ def attn_fwd(seqlens, edits_per_traj, Q, K, V, scale, rows=None, heads=None):
                 k = K[idx, g]
                 v = V[idx, g]
                 q = Q[grows, h]
+                if rope_theta is not None:
+                    k = rope(k, np.arange(idx.size), rope_theta)
+                    q = rope(q, n_before + part, rope_theta)
                 s = _scores(q, k, scale, n_before + part)
                 m = s.max(axis=1, keepdims=True)
                 p = np.exp(s - m)
@@ -89,7 +118,7 @@ def attn_fwd(seqlens, edits_per_traj, Q, K, V, scale, rows=None, heads=None):
     return O, L
 
 
-def attn_bwd(seqlens, edits_per_traj, Q, K, V, dO, scale, groups=None):
+def attn_bwd(seqlens, edits_per_traj, Q, K, V, dO, scale, groups=None, rope_theta=None):
     """Textbook softmax-attention backward on every segment's compact sequence.
 
     For one segment and head (compact rows r, compact keys c):
@@ -100,6 +129,8 @@ def attn_bwd(seqlens, edits_per_traj, Q, K, V, dO, scale, groups=None):
 
     ``groups`` restricts the computation to some KV groups (all their query
     heads); returns full-size ``(dQ, dK, dV)`` with NaN outside the selection.
+    With ``rope_theta`` the scores use rotated q and k (compact index) and
+    dQ, dK are the rotated-space gradients turned back by the same angles.
     """
     Q = np.asarray(Q, dtype=np.float64)
     K = np.asarray(K, dtype=np.float64)
@@ -119,23 +150,33 @@ def attn_bwd(seqlens, edits_per_traj, Q, K, V, dO, scale, groups=None):
     for seg_rows, idx, n_before in _segments(seqlens, edits_per_traj):
         for c0 in range(0, seg_rows.size, _ROW_CHUNK):
             grows = seg_rows[c0 : c0 + _ROW_CHUNK]
+            crow = n_before + c0 + np.arange(grows.size)
             for g in groups:
                 k = K[idx, g]
                 v = V[idx, g]
+                if rope_theta is not None:
+                    k = rope(k, np.arange(idx.size), rope_theta)
                 dk = np.zeros_like(k)
                 dv = np.zeros_like(v)
                 for h in range(g * grp, (g + 1) * grp):
                     q = Q[grows, h]
+                    if rope_theta is not None:
+                        q = rope(q, crow, rope_theta)
                     do = dO[grows, h]
-                    s = _scores(q, k, scale, n_before + c0 + np.arange(grows.size))
+                    s = _scores(q, k, scale, crow)
                     m = s.max(axis=1, keepdims=True)
                     p = np.exp(s - m)
                     p /= p.sum(axis=1, keepdims=True)
                     dp = do @ v.T
                     ds = p * (dp - (p * dp).sum(axis=1, keepdims=True))
-                    dQ[grows, h] = scale * (ds @ k)
+                    dq = scale * (ds @ k)
+                    if rope_theta is not None:
+                        dq = rope(dq, crow, rope_theta, inverse=True)
+                    dQ[grows, h] = dq
                     dk += scale * (ds.T @ q)
                     dv += p.T @ do
+                if rope_theta is not None:
+                    dk = rope(dk, np.arange(idx.size), rope_theta, inverse=True)
                 np.add.at(dK[:, g], idx, dk)
                 np.add.at(dV[:, g], idx, dv)
     return dQ, dK, dV

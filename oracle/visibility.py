@@ -208,6 +208,24 @@ def dead_halves(T, edits, cls, tile=TILE):
     return out
 
 
+def logical_positions(T, edits):
+    """Row-wise logical position of every key in every segment's live view.
+
+    §4.2 reassigns position ids so that the keys a row sees form a gap-free
+    sequence (condition (ii) of the 4D-mask equivalence proposition, App. C):
+    in segment s the key at physical position j takes the position it has in
+    the compact list ``view_s``, i.e. its index there. Returns int64
+    ``[S, T]``, -1 where j is not a member of ``view_s``. A row i of segment s
+    is a member of its own view, so ``out[s, i]`` is the row's own position.
+    """
+    views = live_views(T, edits)
+    out = np.full((len(views), T), -1, dtype=np.int64)
+    for s, (_, _, view) in enumerate(views):
+        for n, j in enumerate(view):
+            out[s, j] = n
+    return out
+
+
 def segment_keymask(T, edits, tile=TILE):
     """Per (segment, k-tile) 128-bit membership of the segment's live view.
 
