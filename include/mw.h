@@ -197,6 +197,76 @@ mw_status mw_masked_attn_bwd(const mw_vis_layout* layout, const void* vis,
                              int Hq, int Hkv, int Dh, int dtype, float scale,
                              void* ws, void* stream);
 
+/*
+ * Row-wise logical positions (§4.2: position ids reassigned so that the keys a
+ * row sees form a gap-free sequence; condition (ii) of the 4D-mask equivalence
+ * proposition, App. C).
+ *   pos  int32 [layout->n_keymask * 128] (device, overwritten). Entry
+ *        (traj_km[b] + s * nt_b) * 128 + j, for trajectory b with nt_b tiles,
+ *        its segment s and key j < 128 nt_b, is the rank of key j in segment
+ *        s's live view (the number of view members before j), or -1 when j is
+ *        not a member (evicted by an edit <= s, after the segment, or past
+ *        T_b). traj_km is the vis array at layout->off_traj_km. A row i of
+ *        segment s is a member of its own view; its entry is its position.
+ * Computed from the view bits of `vis` (one prefix popcount per segment).
+ */
+mw_status mw_logical_positions(const mw_vis_layout* layout, const void* vis, int32_t* pos, void* stream);
+
+/*
+ * Rotary-embedding table (RoFormer rotate-half pairing; the paper fixes no
+ * positional encoding, only that it depend on the logical offset):
+ *   table float32 [n_pos][Dh/2][2] (device, overwritten) =
+ *   (cos, sin)(p * theta^(-2f/Dh)) for position p < n_pos and pair f < Dh/2,
+ *   evaluated in double precision and rounded once.
+ * Dh even and > 0; theta > 0 and finite (MW_ESHAPE / MW_EINVAL).
+ */
+mw_status mw_rope_table(int n_pos, int Dh, double theta, float* table, void* stream);
+
+/*
+ * Rotate every row by its own logical position: for row i of segment s with
+ * p = pos[(traj_km[b] + s nt_b) 128 + i], pair f of every head turns by the
+ * table angle of p (inverse != 0: by minus that angle, the transpose):
+ *   y_f = x_f cos - x_(f+Dh/2) sin,  y_(f+Dh/2) = x_(f+Dh/2) cos + x_f sin.
+ *   X, Y [total_tokens, H, Dh] (dtype); Y may equal X (in place).
+ * pos from mw_logical_positions, table from mw_rope_table with
+ * n_pos >= 128 * layout->max_tiles (else MW_ESHAPE).
+ */
+mw_status mw_rope_rows(const mw_vis_layout* layout, const void* vis, const int32_t* pos, const float* table,
+                       int n_pos, const void* X, void* Y, int H, int Dh, int dtype, int inverse, void* stream);
+
+/* Workspace bytes of mw_masked_attn_rope_fwd and of mw_masked_attn_rope_bwd. */
+mw_status mw_masked_attn_rope_ws(const mw_vis_layout* layout, int Hq, int Hkv, int Dh, int dtype,
+                                 size_t* fwd_bytes, size_t* bwd_bytes);
+
+/*
+ * mw_masked_attn_fwd with rotary positions reassigned per row (§4.2): the
+ * score of row i (segment s) and visible key j is
+ *   scale * (R(p_s(i)) q_i) . (R(p_s(j)) k_j),
+ * so it depends only on the logical offset p_s(i) - p_s(j), the number of
+ * keys of view_s in [j, i). Q, K are NOT rotated by the caller. The rotated
+ * queries and, for every segment, the keys of its view rotated to their
+ * positions in it (layout->n_keymask * 128 rows of [Hkv, Dh]) are written to
+ * `ws` (mw_masked_attn_rope_ws fwd_bytes). Other arguments as
+ * mw_masked_attn_fwd; pos and table as mw_rope_rows. Runs on the CUDA-core
+ * path for every dtype and Dh in {64, 128}.
+ */
+mw_status mw_masked_attn_rope_fwd(const mw_vis_layout* layout, const void* vis, const int32_t* pos,
+                                  const float* table, int n_pos, const void* Q, const void* K, const void* V,
+                                  void* O, float* LSE, int Hq, int Hkv, int Dh, int dtype, float scale,
+                                  void* ws, void* stream);
+
+/*
+ * Backward of mw_masked_attn_rope_fwd: dQ, dK, dV of the un-rotated inputs
+ * (dQ = R^T dQ_rot per row; dK_j = sum over the segments whose view holds j
+ * of R(p_s(j))^T times that segment's key-row gradient, accumulated in
+ * float32), all in dtype, overwritten. `ws`: mw_masked_attn_rope_ws
+ * bwd_bytes (recomputes the rotations; need not hold the forward's).
+ */
+mw_status mw_masked_attn_rope_bwd(const mw_vis_layout* layout, const void* vis, const int32_t* pos,
+                                  const float* table, int n_pos, const void* Q, const void* K, const void* V,
+                                  const void* O, const void* dO, const float* LSE, void* dQ, void* dK, void* dV,
+                                  int Hq, int Hkv, int Dh, int dtype, float scale, void* ws, void* stream);
+
 /* Bytes of device workspace the log-prob loss forward/backward pair needs. */
 mw_status mw_logprob_ws(int N, int M, int d, int Vocab, int dtype, size_t* ws_bytes);
 

@@ -16,10 +16,13 @@ from ._lib import (  # noqa: F401
     exported_names,
     flatten_record,
     kernel_launches,
+    logical_positions,
     logprob_loss_bwd,
     logprob_loss_fwd,
     masked_attn_bwd,
     masked_attn_fwd,
+    masked_attn_rope_bwd,
+    masked_attn_rope_fwd,
     mw_build_visibility,
     mw_build_visibility_noalloc,
     mw_logprob_check_status,
@@ -30,6 +33,10 @@ from ._lib import (  # noqa: F401
     mw_masked_attn_bwd,
     mw_masked_attn_bwd_ws,
     mw_masked_attn_fwd,
+    mw_masked_attn_rope_ws,
     mw_selftest_wait_timeout,
     mw_visibility_layout,
+    rope_n_pos,
+    rope_rows,
+    rope_table,
 )

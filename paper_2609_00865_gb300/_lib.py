@@ -60,6 +60,14 @@ _SIGS = {
     "mw_logprob_loss_fwd_kl": (_I, [_P, _P, _P, _P, _I, _P, _P, _F, _F, _P, _F, _I, _I, _I, _I, _P, _P, _P, _P, _P,
                                     _P]),
     "mw_logprob_loss_bwd": (_I, [_P, _P, _P, _P, _I, _I, _I, _I, _I, _P, _P, _F, _P, _P, _P]),
+    "mw_logical_positions": (_I, [_LP, _P, _P, _P]),
+    "mw_rope_table": (_I, [_I, _I, ctypes.c_double, _P, _P]),
+    "mw_rope_rows": (_I, [_LP, _P, _P, _P, _I, _P, _P, _I, _I, _I, _I, _P]),
+    "mw_masked_attn_rope_ws": (_I, [_LP, _I, _I, _I, _I, ctypes.POINTER(ctypes.c_size_t),
+                                    ctypes.POINTER(ctypes.c_size_t)]),
+    "mw_masked_attn_rope_fwd": (_I, [_LP, _P, _P, _P, _I, _P, _P, _P, _P, _P, _I, _I, _I, _I, _F, _P, _P]),
+    "mw_masked_attn_rope_bwd": (_I, [_LP, _P, _P, _P, _I, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _F,
+                                     _P, _P]),
     "mw_check_status": (_I, [_LP, _P, _P]),
     "mw_logprob_check_status": (_I, [_I, _I, _I, _I, _I, _P, _P]),
     "mw_selftest_wait_timeout": (_I, [ctypes.c_int64, _P, _P]),
@@ -297,6 +305,88 @@ def masked_attn_bwd(vis, Q, K, V, O, dO, LSE, scale=None, ws=None, stream=None):
         ws = torch.empty(max(nbytes, 1), dtype=torch.uint8, device=Q.device)
     dQ, dK, dV = torch.empty_like(Q), torch.empty_like(K), torch.empty_like(V)
     mw_masked_attn_bwd(vis, Q, K, V, O, dO, LSE, dQ, dK, dV, scale, ws, stream)
+    return dQ, dK, dV
+
+
+# --- row-wise logical positions and rotary attention ---------------------------
+
+def logical_positions(vis, stream=None):
+    """int32 [n_keymask * 128]: rank of key j in segment s's live view at
+    (traj_km[b] + s nt_b) 128 + j, -1 for non-members (mw_logical_positions)."""
+    import torch
+    L = vis.layout
+    pos = torch.empty(max(int(L.n_keymask) * TILE, 1), dtype=torch.int32, device=vis.vis.device)
+    _check(_lib().mw_logical_positions(ctypes.byref(L), _ptr(vis.vis), _ptr(pos), _stream(stream)),
+           "mw_logical_positions")
+    return pos
+
+
+def rope_table(n_pos, Dh, theta, device="cuda", stream=None):
+    """float32 [n_pos, Dh/2, 2] (cos, sin) table (mw_rope_table)."""
+    import torch
+    t = torch.empty(max(int(n_pos), 1), Dh // 2, 2, dtype=torch.float32, device=device)
+    _check(_lib().mw_rope_table(int(n_pos), int(Dh), float(theta), _ptr(t), _stream(stream)), "mw_rope_table")
+    return t
+
+
+def rope_n_pos(vis):
+    """Smallest table length the rotary entry points accept for this record."""
+    return TILE * int(vis.layout.max_tiles)
+
+
+def rope_rows(vis, pos, table, X, inverse=False, out=None, stream=None):
+    """Rotate every row of X [T, H, Dh] by its own logical position."""
+    import torch
+    _need(X, "X")
+    Y = torch.empty_like(X) if out is None else out
+    _check(_lib().mw_rope_rows(ctypes.byref(vis.layout), _ptr(vis.vis), _ptr(pos), _ptr(table), table.shape[0],
+                               _ptr(X), _ptr(Y), X.shape[1], X.shape[2], _dtype_code(X), int(bool(inverse)),
+                               _stream(stream)), "mw_rope_rows")
+    return Y
+
+
+def mw_masked_attn_rope_ws(vis, Hq, Hkv, Dh, dtype):
+    f, b = ctypes.c_size_t(), ctypes.c_size_t()
+    _check(_lib().mw_masked_attn_rope_ws(ctypes.byref(vis.layout), Hq, Hkv, Dh, dtype, ctypes.byref(f),
+                                         ctypes.byref(b)), "mw_masked_attn_rope_ws")
+    return int(f.value), int(b.value)
+
+
+def masked_attn_rope_fwd(vis, pos, table, Q, K, V, scale=None, ws=None, stream=None):
+    """Masked attention with per-row logical rotary positions; returns O, LSE."""
+    import torch
+    for t, n in ((Q, "Q"), (K, "K"), (V, "V")):
+        _need(t, n, dtype=Q.dtype)
+    Hq, Dh, Hkv = Q.shape[1], Q.shape[2], K.shape[1]
+    scale = float(Dh) ** -0.5 if scale is None else scale
+    if ws is None:
+        nbytes = mw_masked_attn_rope_ws(vis, Hq, Hkv, Dh, _dtype_code(Q))[0]
+        ws = torch.empty(max(nbytes, 1), dtype=torch.uint8, device=Q.device)
+    O = torch.empty_like(Q)
+    LSE = torch.empty(Hq, Q.shape[0], dtype=torch.float32, device=Q.device)
+    _check(_lib().mw_masked_attn_rope_fwd(ctypes.byref(vis.layout), _ptr(vis.vis), _ptr(pos), _ptr(table),
+                                          table.shape[0], _ptr(Q), _ptr(K), _ptr(V), _ptr(O), _ptr(LSE), Hq, Hkv,
+                                          Dh, _dtype_code(Q), float(scale), _ptr(ws), _stream(stream)),
+           "mw_masked_attn_rope_fwd")
+    return O, LSE
+
+
+def masked_attn_rope_bwd(vis, pos, table, Q, K, V, O, dO, LSE, scale=None, ws=None, stream=None):
+    """Backward of masked_attn_rope_fwd; returns dQ, dK, dV."""
+    import torch
+    for t, n in ((Q, "Q"), (K, "K"), (V, "V"), (O, "O"), (dO, "dO")):
+        _need(t, n, dtype=Q.dtype)
+    _need(LSE, "LSE", dtype=torch.float32)
+    Hq, Dh, Hkv = Q.shape[1], Q.shape[2], K.shape[1]
+    scale = float(Dh) ** -0.5 if scale is None else scale
+    if ws is None:
+        nbytes = mw_masked_attn_rope_ws(vis, Hq, Hkv, Dh, _dtype_code(Q))[1]
+        ws = torch.empty(max(nbytes, 1), dtype=torch.uint8, device=Q.device)
+    dQ, dK, dV = torch.empty_like(Q), torch.empty_like(K), torch.empty_like(V)
+    _check(_lib().mw_masked_attn_rope_bwd(ctypes.byref(vis.layout), _ptr(vis.vis), _ptr(pos), _ptr(table),
+                                          table.shape[0], _ptr(Q), _ptr(K), _ptr(V), _ptr(O), _ptr(dO), _ptr(LSE),
+                                          _ptr(dQ), _ptr(dK), _ptr(dV), Hq, Hkv, Dh, _dtype_code(Q), float(scale),
+                                          _ptr(ws), _stream(stream)), "mw_masked_attn_rope_bwd")
     return dQ, dK, dV
 
 

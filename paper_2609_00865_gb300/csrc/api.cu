@@ -21,6 +21,20 @@ mw_status attn_fwd_tc(const mw_vis_layout*, const void*, const void*, const void
 mw_status attn_bwd_tc(const mw_vis_layout*, const void*, const void*, const void*, const void*, const void*,
                       const void*, const float*, void*, void*, void*, int, int, float, float*, cudaStream_t);
 int64_t attn_bwd_tc_ws(const mw_vis_layout*, int);
+mw_status attn_delta(const mw_vis_layout*, const void*, const void*, int, int, int, float*, cudaStream_t);
+mw_status attn_fwd_simt_segk(const mw_vis_layout*, const void*, const void*, const void*, const void*, void*, float*,
+                             int, int, int, int, float, cudaStream_t);
+mw_status attn_bwd_simt_segk(const mw_vis_layout*, const void*, const void*, const void*, const void*, const void*,
+                             const float*, const float*, void*, float*, void*, int, int, int, int, float,
+                             cudaStream_t);
+mw_status logical_positions(const mw_vis_layout*, const void*, int32_t*, cudaStream_t);
+mw_status rope_table(int, int, double, float*, cudaStream_t);
+mw_status rope_rows(const mw_vis_layout*, const void*, const int32_t*, const float*, int, const void*, void*, int,
+                    int, int, bool, cudaStream_t);
+mw_status rope_segments(const mw_vis_layout*, const void*, const int32_t*, const float*, int, const void*, void*,
+                        int, int, int, cudaStream_t);
+mw_status rope_segments_bwd(const mw_vis_layout*, const void*, const int32_t*, const float*, int, const float*,
+                            void*, int, int, int, cudaStream_t);
 __global__ void k_loss_epilogue(int, const float*, const float*, const float*, float, float, const float*, float, float*,
                                 float*, float*);
 
@@ -200,4 +214,116 @@ extern "C" mw_status mw_logprob_check_status(int N, int M, int d, int V, int dty
         return st;
     if ((st = cuda_status(cudaStreamSynchronize((cudaStream_t)stream))) != MW_OK) return st;
     return h[1] ? MW_ETIMEOUT : MW_OK;
+}
+
+// --- row-wise logical positions and rotary attention (§4.2) -----------------
+
+// Byte offsets inside the rotary-attention workspace: rotated queries, the
+// segment key rows, then (backward only) Delta and the float32 gradient of
+// the segment key rows.
+struct RopeWs {
+    int64_t q, kseg, delta, dkseg, fwd_bytes, bwd_bytes;
+};
+static RopeWs rope_ws_layout(const mw_vis_layout* L, int Hq, int Hkv, int Dh, int dtype) {
+    RopeWs w;
+    const int64_t esz = dtype == MW_F32 ? 4 : 2;
+    const int64_t krows = L->n_keymask * MW_TILE;
+    int64_t o = 0;
+    w.q = o; o = align256(o + esz * L->total_tokens * Hq * Dh);
+    w.kseg = o; o = align256(o + esz * krows * Hkv * Dh);
+    w.fwd_bytes = o;
+    w.delta = o; o = align256(o + 4 * L->total_tokens * Hq);
+    w.dkseg = o; o = align256(o + 4 * krows * Hkv * Dh);
+    w.bwd_bytes = o;
+    return w;
+}
+
+static mw_status rope_args(const mw_vis_layout* L, const void* vis, const int32_t* pos, const float* table,
+                           int n_pos) {
+    if (!L) return MW_EINVAL;
+    if (L->total_tokens == 0) return MW_OK;
+    if (!vis || !pos || !table) return MW_EINVAL;
+    if (n_pos < MW_TILE * (int64_t)L->max_tiles) return MW_ESHAPE;   // every position < T_b <= 128 nt_b
+    return MW_OK;
+}
+
+extern "C" mw_status mw_logical_positions(const mw_vis_layout* L, const void* vis, int32_t* pos, void* stream) {
+    if (!L) return MW_EINVAL;
+    if (L->n_keymask == 0) return MW_OK;
+    if (!vis || !pos) return MW_EINVAL;
+    return logical_positions(L, vis, pos, (cudaStream_t)stream);
+}
+
+extern "C" mw_status mw_rope_table(int n_pos, int Dh, double theta, float* table, void* stream) {
+    if (n_pos < 0 || Dh <= 0 || Dh % 2 != 0) return MW_ESHAPE;
+    if (!(theta > 0.0) || !isfinite(theta)) return MW_EINVAL;
+    if (n_pos > 0 && !table) return MW_EINVAL;
+    return rope_table(n_pos, Dh, theta, table, (cudaStream_t)stream);
+}
+
+extern "C" mw_status mw_rope_rows(const mw_vis_layout* L, const void* vis, const int32_t* pos, const float* table,
+                                  int n_pos, const void* X, void* Y, int H, int Dh, int dtype, int inverse,
+                                  void* stream) {
+    if (dtype != MW_F32 && dtype != MW_BF16) return MW_EDTYPE;
+    if (H <= 0 || Dh <= 0 || Dh % 2 != 0) return MW_ESHAPE;
+    mw_status st = rope_args(L, vis, pos, table, n_pos);
+    if (st != MW_OK || L->total_tokens == 0) return st;
+    if (!X || !Y) return MW_EINVAL;
+    return rope_rows(L, vis, pos, table, n_pos, X, Y, H, Dh, dtype, inverse != 0, (cudaStream_t)stream);
+}
+
+extern "C" mw_status mw_masked_attn_rope_ws(const mw_vis_layout* L, int Hq, int Hkv, int Dh, int dtype,
+                                            size_t* fwd_bytes, size_t* bwd_bytes) {
+    if (!L || !fwd_bytes || !bwd_bytes) return MW_EINVAL;
+    if (dtype != MW_F32 && dtype != MW_BF16) return MW_EDTYPE;
+    if (Hq <= 0 || Hkv <= 0 || Hq % Hkv != 0 || !(Dh == 64 || Dh == 128)) return MW_ESHAPE;
+    RopeWs w = rope_ws_layout(L, Hq, Hkv, Dh, dtype);
+    *fwd_bytes = (size_t)w.fwd_bytes;
+    *bwd_bytes = (size_t)w.bwd_bytes;
+    return MW_OK;
+}
+
+extern "C" mw_status mw_masked_attn_rope_fwd(const mw_vis_layout* L, const void* vis, const int32_t* pos,
+                                             const float* table, int n_pos, const void* Q, const void* K,
+                                             const void* V, void* O, float* LSE, int Hq, int Hkv, int Dh, int dtype,
+                                             float scale, void* ws, void* stream) {
+    mw_status st = attn_args(L, vis, Hq, Hkv, Dh, dtype, scale);
+    if (st != MW_OK) return st;
+    if ((st = rope_args(L, vis, pos, table, n_pos)) != MW_OK) return st;
+    if (L->total_tokens == 0) return MW_OK;
+    if (!Q || !K || !V || !O || !LSE || !ws) return MW_EINVAL;
+    cudaStream_t s = (cudaStream_t)stream;
+    RopeWs w = rope_ws_layout(L, Hq, Hkv, Dh, dtype);
+    void* q = at<char>(ws, w.q);
+    void* kseg = at<char>(ws, w.kseg);
+    if ((st = rope_rows(L, vis, pos, table, n_pos, Q, q, Hq, Dh, dtype, false, s)) != MW_OK) return st;
+    if ((st = rope_segments(L, vis, pos, table, n_pos, K, kseg, Hkv, Dh, dtype, s)) != MW_OK) return st;
+    return attn_fwd_simt_segk(L, vis, q, kseg, V, O, LSE, Hq, Hkv, Dh, dtype, scale, s);
+}
+
+extern "C" mw_status mw_masked_attn_rope_bwd(const mw_vis_layout* L, const void* vis, const int32_t* pos,
+                                             const float* table, int n_pos, const void* Q, const void* K,
+                                             const void* V, const void* O, const void* dO, const float* LSE,
+                                             void* dQ, void* dK, void* dV, int Hq, int Hkv, int Dh, int dtype,
+                                             float scale, void* ws, void* stream) {
+    mw_status st = attn_args(L, vis, Hq, Hkv, Dh, dtype, scale);
+    if (st != MW_OK) return st;
+    if ((st = rope_args(L, vis, pos, table, n_pos)) != MW_OK) return st;
+    if (L->total_tokens == 0) return MW_OK;
+    if (!Q || !K || !V || !O || !dO || !LSE || !dQ || !dK || !dV || !ws) return MW_EINVAL;
+    cudaStream_t s = (cudaStream_t)stream;
+    RopeWs w = rope_ws_layout(L, Hq, Hkv, Dh, dtype);
+    void* q = at<char>(ws, w.q);
+    void* kseg = at<char>(ws, w.kseg);
+    float* delta = at<float>(ws, w.delta);
+    float* dkseg = at<float>(ws, w.dkseg);
+    if ((st = rope_rows(L, vis, pos, table, n_pos, Q, q, Hq, Dh, dtype, false, s)) != MW_OK) return st;
+    if ((st = rope_segments(L, vis, pos, table, n_pos, K, kseg, Hkv, Dh, dtype, s)) != MW_OK) return st;
+    if ((st = attn_delta(L, O, dO, Hq, Dh, dtype, delta, s)) != MW_OK) return st;
+    // dQ first holds the gradient of the rotated queries, then is turned back in place
+    if ((st = attn_bwd_simt_segk(L, vis, q, kseg, V, dO, LSE, delta, dQ, dkseg, dV, Hq, Hkv, Dh, dtype, scale, s)) !=
+        MW_OK)
+        return st;
+    if ((st = rope_rows(L, vis, pos, table, n_pos, dQ, dQ, Hq, Dh, dtype, true, s)) != MW_OK) return st;
+    return rope_segments_bwd(L, vis, pos, table, n_pos, dkseg, dK, Hkv, Dh, dtype, s);
 }

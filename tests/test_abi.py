@@ -117,3 +117,43 @@ def test_attention_and_lmhead_reject_bad_args_on_host():
                                     None) == 1
     assert h.mw_logprob_loss_fwd_kl(P, P, P, P, 4, P, P, 0.2, 0.28, None, 1e-3, 10, 128, 100, 0, P, P, P, P, P,
                                     None) == 1
+
+
+def test_rope_entry_points_reject_bad_args_on_host():
+    L, h = _lib()
+    lay = L.mw_visibility_layout(np.array([0, 10], np.int32), np.zeros(0, np.int32), 0)
+    P = ctypes.c_void_p(16)
+    # table: negative length, odd head dim, bad theta
+    assert h.mw_rope_table(-1, 128, 1e4, P, None) == 3
+    assert h.mw_rope_table(10, 127, 1e4, P, None) == 3
+    assert h.mw_rope_table(10, 128, 0.0, P, None) == 1
+    assert h.mw_rope_table(10, 128, float("inf"), P, None) == 1
+    assert h.mw_rope_table(10, 128, 1e4, None, None) == 1
+    # rows: table shorter than 128 * max_tiles, bad dtype, no heads, null pos
+    assert h.mw_rope_rows(ctypes.byref(lay), P, P, P, 64, P, P, 2, 128, 1, 0, None) == 3
+    assert h.mw_rope_rows(ctypes.byref(lay), P, P, P, 128, P, P, 2, 128, 7, 0, None) == 4
+    assert h.mw_rope_rows(ctypes.byref(lay), P, P, P, 128, P, P, 0, 128, 1, 0, None) == 3
+    assert h.mw_rope_rows(ctypes.byref(lay), P, None, P, 128, P, P, 2, 128, 1, 0, None) == 1
+    assert h.mw_logical_positions(ctypes.byref(lay), P, None, None) == 1
+    # attention: short table, missing workspace, GQA shape
+    args = (P, P, P, P, P, 4, 2, 128, 1, 0.1)   # Q K V O LSE Hq Hkv Dh dtype scale
+    assert h.mw_masked_attn_rope_fwd(ctypes.byref(lay), P, P, P, 64, *args, P, None) == 3
+    assert h.mw_masked_attn_rope_fwd(ctypes.byref(lay), P, P, P, 128, *args, None, None) == 1
+    assert h.mw_masked_attn_rope_fwd(ctypes.byref(lay), P, P, P, 128, P, P, P, P, P, 6, 4, 128, 1, 0.1, P,
+                                     None) == 3
+    assert h.mw_masked_attn_rope_bwd(ctypes.byref(lay), P, P, P, 64, P, P, P, P, P, P, P, P, P, 4, 2, 128, 1, 0.1,
+                                     P, None) == 3
+
+
+def test_rope_workspace_holds_rotated_queries_and_segment_keys():
+    L, h = _lib()
+    cu = np.array([0, 300, 1000], np.int32)
+    lay = L.mw_visibility_layout(cu, np.array([0, 1, 1], np.int32), 4)
+    Hq, Hkv, Dh = 4, 2, 128
+    for dtype, esz in ((0, 4), (1, 2)):
+        f, b = L.mw_masked_attn_rope_ws(L.Visibility(lay, None, None), Hq, Hkv, Dh, dtype)
+        need = esz * (lay.total_tokens * Hq * Dh + lay.n_keymask * 128 * Hkv * Dh)
+        assert need <= f < need + 1024
+        # backward adds Delta and the float32 segment-key gradient
+        need_b = f + 4 * lay.total_tokens * Hq + 4 * lay.n_keymask * 128 * Hkv * Dh
+        assert need_b <= b < need_b + 1024
