@@ -247,8 +247,11 @@ mw_status mw_masked_attn_rope_ws(const mw_vis_layout* layout, int Hq, int Hkv, i
  * queries and, for every segment, the keys of its view rotated to their
  * positions in it (layout->n_keymask * 128 rows of [Hkv, Dh]) are written to
  * `ws` (mw_masked_attn_rope_ws fwd_bytes). Other arguments as
- * mw_masked_attn_fwd; pos and table as mw_rope_rows. Runs on the CUDA-core
- * path for every dtype and Dh in {64, 128}.
+ * mw_masked_attn_fwd; pos and table as mw_rope_rows. bf16 with Dh 128 runs
+ * on the tensor-core kernels (one CTA per q-tile and segment it serves:
+ * tiles that a junction splits get one CTA per segment); float32, and bf16
+ * with Dh 64, on the CUDA-core kernels. MW_ESHAPE when n_keymask * 128 or
+ * the segment count exceeds the tensor-core kernels' int32 coordinates.
  */
 mw_status mw_masked_attn_rope_fwd(const mw_vis_layout* layout, const void* vis, const int32_t* pos,
                                   const float* table, int n_pos, const void* Q, const void* K, const void* V,
@@ -259,8 +262,9 @@ mw_status mw_masked_attn_rope_fwd(const mw_vis_layout* layout, const void* vis, 
  * Backward of mw_masked_attn_rope_fwd: dQ, dK, dV of the un-rotated inputs
  * (dQ = R^T dQ_rot per row; dK_j = sum over the segments whose view holds j
  * of R(p_s(j))^T times that segment's key-row gradient, accumulated in
- * float32), all in dtype, overwritten. `ws`: mw_masked_attn_rope_ws
- * bwd_bytes (recomputes the rotations; need not hold the forward's).
+ * float32), all in dtype, overwritten. dV_j likewise sums the per-segment
+ * parts on the tensor-core path. `ws`: mw_masked_attn_rope_ws bwd_bytes
+ * (recomputes the rotations; need not hold the forward's).
  */
 mw_status mw_masked_attn_rope_bwd(const mw_vis_layout* layout, const void* vis, const int32_t* pos,
                                   const float* table, int n_pos, const void* Q, const void* K, const void* V,

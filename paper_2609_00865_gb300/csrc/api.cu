@@ -34,7 +34,11 @@ mw_status rope_rows(const mw_vis_layout*, const void*, const int32_t*, const flo
 mw_status rope_segments(const mw_vis_layout*, const void*, const int32_t*, const float*, int, const void*, void*,
                         int, int, int, cudaStream_t);
 mw_status rope_segments_bwd(const mw_vis_layout*, const void*, const int32_t*, const float*, int, const float*,
-                            void*, int, int, int, cudaStream_t);
+                            void*, int, int, int, bool, cudaStream_t);
+mw_status attn_fwd_tc_segk(const mw_vis_layout*, const void*, const void*, const void*, const void*, void*, float*,
+                           int, int, float, cudaStream_t);
+mw_status attn_bwd_tc_segk(const mw_vis_layout*, const void*, const void*, const void*, const void*, const void*,
+                           const void*, const float*, void*, float*, float*, int, int, float, float*, cudaStream_t);
 __global__ void k_loss_epilogue(int, const float*, const float*, const float*, float, float, const float*, float, float*,
                                 float*, float*);
 
@@ -218,22 +222,29 @@ extern "C" mw_status mw_logprob_check_status(int N, int M, int d, int V, int dty
 
 // --- row-wise logical positions and rotary attention (§4.2) -----------------
 
+// The rotary attention's tensor-core path: bf16 with head dim 128, as the
+// plain attention's.
+static bool rope_tc(int Dh, int dtype) { return dtype == MW_BF16 && Dh == 128; }
+
 // Byte offsets inside the rotary-attention workspace: rotated queries, the
-// segment key rows, then (backward only) Delta and the float32 gradient of
-// the segment key rows.
+// segment key rows, then (backward only) Delta (tensor-core path: the
+// (-LSE log2 e, Delta) pair array), the float32 gradient of the segment key
+// rows and (tensor-core path) the float32 per-segment dV partials.
 struct RopeWs {
-    int64_t q, kseg, delta, dkseg, fwd_bytes, bwd_bytes;
+    int64_t q, kseg, delta, dkseg, dvseg, fwd_bytes, bwd_bytes;
 };
 static RopeWs rope_ws_layout(const mw_vis_layout* L, int Hq, int Hkv, int Dh, int dtype) {
     RopeWs w;
     const int64_t esz = dtype == MW_F32 ? 4 : 2;
     const int64_t krows = L->n_keymask * MW_TILE;
+    const bool tc = rope_tc(Dh, dtype);
     int64_t o = 0;
     w.q = o; o = align256(o + esz * L->total_tokens * Hq * Dh);
     w.kseg = o; o = align256(o + esz * krows * Hkv * Dh);
     w.fwd_bytes = o;
-    w.delta = o; o = align256(o + 4 * L->total_tokens * Hq);
+    w.delta = o; o = align256(o + (tc ? attn_bwd_tc_ws(L, Hq) : 4 * L->total_tokens * Hq));
     w.dkseg = o; o = align256(o + 4 * krows * Hkv * Dh);
+    w.dvseg = o; o = align256(o + (tc ? 4 * krows * Hkv * Dh : 0));
     w.bwd_bytes = o;
     return w;
 }
@@ -298,6 +309,7 @@ extern "C" mw_status mw_masked_attn_rope_fwd(const mw_vis_layout* L, const void*
     void* kseg = at<char>(ws, w.kseg);
     if ((st = rope_rows(L, vis, pos, table, n_pos, Q, q, Hq, Dh, dtype, false, s)) != MW_OK) return st;
     if ((st = rope_segments(L, vis, pos, table, n_pos, K, kseg, Hkv, Dh, dtype, s)) != MW_OK) return st;
+    if (rope_tc(Dh, dtype)) return attn_fwd_tc_segk(L, vis, q, kseg, V, O, LSE, Hq, Hkv, scale, s);
     return attn_fwd_simt_segk(L, vis, q, kseg, V, O, LSE, Hq, Hkv, Dh, dtype, scale, s);
 }
 
@@ -319,11 +331,20 @@ extern "C" mw_status mw_masked_attn_rope_bwd(const mw_vis_layout* L, const void*
     float* dkseg = at<float>(ws, w.dkseg);
     if ((st = rope_rows(L, vis, pos, table, n_pos, Q, q, Hq, Dh, dtype, false, s)) != MW_OK) return st;
     if ((st = rope_segments(L, vis, pos, table, n_pos, K, kseg, Hkv, Dh, dtype, s)) != MW_OK) return st;
-    if ((st = attn_delta(L, O, dO, Hq, Dh, dtype, delta, s)) != MW_OK) return st;
     // dQ first holds the gradient of the rotated queries, then is turned back in place
-    if ((st = attn_bwd_simt_segk(L, vis, q, kseg, V, dO, LSE, delta, dQ, dkseg, dV, Hq, Hkv, Dh, dtype, scale, s)) !=
-        MW_OK)
-        return st;
+    if (rope_tc(Dh, dtype)) {
+        float* dvseg = at<float>(ws, w.dvseg);
+        if ((st = attn_bwd_tc_segk(L, vis, q, kseg, V, O, dO, LSE, dQ, dkseg, dvseg, Hq, Hkv, scale, delta, s)) !=
+            MW_OK)
+            return st;
+        if ((st = rope_segments_bwd(L, vis, pos, table, n_pos, dvseg, dV, Hkv, Dh, dtype, false, s)) != MW_OK)
+            return st;
+    } else {
+        if ((st = attn_delta(L, O, dO, Hq, Dh, dtype, delta, s)) != MW_OK) return st;
+        if ((st = attn_bwd_simt_segk(L, vis, q, kseg, V, dO, LSE, delta, dQ, dkseg, dV, Hq, Hkv, Dh, dtype, scale,
+                                     s)) != MW_OK)
+            return st;
+    }
     if ((st = rope_rows(L, vis, pos, table, n_pos, dQ, dQ, Hq, Dh, dtype, true, s)) != MW_OK) return st;
-    return rope_segments_bwd(L, vis, pos, table, n_pos, dkseg, dK, Hkv, Dh, dtype, s);
+    return rope_segments_bwd(L, vis, pos, table, n_pos, dkseg, dK, Hkv, Dh, dtype, true, s);
 }

@@ -20,6 +20,15 @@
 //               shared memory, O / l and the log-sum-exp written at the end.
 // All waits are bounded (tc::mbar_wait); a timeout ends the CTA and is
 // reported through the visibility status word.
+//
+// SEGK instantiations read keys from "segment key rows" (row (traj_km[b] +
+// s nt_b) 128 + j holds key j as seen by segment s, e.g. rotated to its
+// logical position in view_s). A q-tile CTA then serves one segment: the main
+// launch the segment of the tile's first row, a second launch ("junction
+// items") one CTA per (junction inside a tile, head) for the segment that the
+// junction starts; each stores only its own segment's rows. The dK/dV kernel
+// takes one CTA per (k-tile, segment) over that segment's q-tiles and writes
+// float32 partial gradients per segment key row.
 
 #include <math.h>
 
@@ -73,7 +82,43 @@ struct FwdParams {
     float scale_log2;
     __nv_bfloat16* O;
     float* LSE;
+    int junction_items;   // SEGK: 0 = main launch, 1 = one CTA per (junction, head)
 };
+
+// Work item of a q-tile kernel: trajectory b, local q-tile qt, query head h
+// and (SEGK) the segment s whose rows the CTA stores. Main launch: heaviest
+// (largest qt) first, query heads of one KV group adjacent; s = segment of the
+// tile's first row. Junction items: blockIdx.x / Hq is a global segment index;
+// a segment that starts inside a tile (not at its first row) gets a CTA there.
+struct QItem {
+    int b, qt, h, s;
+    bool ok;
+};
+template <bool SEGK>
+__device__ __forceinline__ QItem q_item(const VisView& v, int Hq, int max_tiles, int n_traj, int junction_items) {
+    QItem it;
+    it.h = blockIdx.x % Hq;
+    const int r = blockIdx.x / Hq;
+    it.s = 0;
+    if (!SEGK || !junction_items) {
+        it.qt = max_tiles - 1 - r / n_traj;
+        it.b = r % n_traj;
+        it.ok = it.qt < v.traj_tile[it.b + 1] - v.traj_tile[it.b];
+        if (SEGK && it.ok) it.s = v.seg[v.traj_tok[it.b] + it.qt * 128];
+    } else {
+        int lo = 0, hi = n_traj;   // largest b with traj_seg[b] <= r
+        while (hi - lo > 1) {
+            const int mid = (lo + hi) >> 1;
+            if (v.traj_seg[mid] <= r) lo = mid; else hi = mid;
+        }
+        it.b = lo;
+        it.s = r - v.traj_seg[lo];
+        const int J = v.seg_start[r];
+        it.qt = J >> 7;
+        it.ok = it.s > 0 && (J & 127) != 0;
+    }
+    return it;
+}
 
 __device__ __forceinline__ float ex2(float x) {
     float y;
@@ -115,6 +160,7 @@ __device__ __forceinline__ uint64_t mnmaj(uint32_t base, int ks) {
     return sdesc_sw128(base + ks * 2048, HALF_B, 1024);
 }
 
+template <bool SEGK>
 __global__ void __launch_bounds__(NT_FWD, 1)
     k_attn_fwd_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                   const __grid_constant__ CUtensorMap tmV, FwdParams p) {
@@ -126,15 +172,11 @@ __global__ void __launch_bounds__(NT_FWD, 1)
     __shared__ int abort_flag;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    // item -> (local q-tile, trajectory, head); heaviest (largest qt) first,
-    // query heads of one KV group adjacent.
-    const int h = blockIdx.x % p.Hq;
-    const int r = blockIdx.x / p.Hq;
-    const int qt = p.max_tiles - 1 - r / p.n_traj;
-    const int b = r % p.n_traj;
     const VisView& v = p.v;
+    const QItem it = q_item<SEGK>(v, p.Hq, p.max_tiles, p.n_traj, p.junction_items);
+    if (!it.ok) return;
+    const int h = it.h, qt = it.qt, b = it.b;
     const int nt = v.traj_tile[b + 1] - v.traj_tile[b];
-    if (qt >= nt) return;
     const int64_t g = v.traj_tile[b] + qt;
     const int64_t tok0 = v.traj_tok[b];
     const int T = v.traj_tok[b + 1] - (int)tok0;
@@ -175,13 +217,15 @@ __global__ void __launch_bounds__(NT_FWD, 1)
             prefetch_tmap(&tmV);
             mbar_expect_tx(&q_full, TILE_B);
             load_tile(sm + SM_Q, &tmQ, &q_full, h, (int)(tok0 + qt * 128));
+            // first K row of the trajectory (SEGK: of the item's segment key rows)
+            const int64_t krow0 = SEGK ? (v.traj_km[b] + (int64_t)it.s * nt) * 128 : tok0;
             for (int j = 0; j < n; ++j) {
                 const int kt = v.fwd_idx[p0 + j] >> 4;
                 const int s = j & 1;
                 const int row = (int)(tok0 + kt * 128);
                 if (j >= 2 && !mbar_wait(&k_empty[s], ((j - 2) >> 1) & 1, status, 101)) { abort_flag = 1; break; }
                 mbar_expect_tx(&k_full[s], TILE_B);
-                load_tile(sm + SM_K + s * TILE_B, &tmK, &k_full[s], kvh, row);
+                load_tile(sm + SM_K + s * TILE_B, &tmK, &k_full[s], kvh, (int)(krow0 + kt * 128));
                 if (j >= 2 && !mbar_wait(&v_empty[s], ((j - 2) >> 1) & 1, status, 102)) { abort_flag = 1; break; }
                 mbar_expect_tx(&v_full[s], TILE_B);
                 load_tile(sm + SM_V + s * TILE_B, &tmV, &v_full[s], kvh, row);
@@ -392,11 +436,12 @@ __global__ void __launch_bounds__(NT_FWD, 1)
             const float inv = 1.f / l;
             __nv_bfloat16* orow = p.O + ((tok0 + ie) * p.Hq + h) * DH;
             uint32_t o[32];
+            const bool store = i < T && (!SEGK || seg == it.s);
 #pragma unroll
             for (int c = 0; c < 4; ++c) {
                 tmem_ld32(lane_base + TM_O + c * 32, o);
                 tmem_wait_ld();
-                if (i < T) {
+                if (store) {
 #pragma unroll
                     for (int x = 0; x < 4; ++x) {
                         uint4 pk;
@@ -408,7 +453,7 @@ __global__ void __launch_bounds__(NT_FWD, 1)
                     }
                 }
             }
-            if (i < T) p.LSE[(int64_t)h * p.total + tok0 + i] = (m + __log2f(l)) * 0.6931471805599453f;
+            if (store) p.LSE[(int64_t)h * p.total + tok0 + i] = (m + __log2f(l)) * 0.6931471805599453f;
         } else {
             abort_flag = 1;
         }
@@ -448,8 +493,12 @@ struct BwdParams {
     __nv_bfloat16* dQ;
     __nv_bfloat16* dK;
     __nv_bfloat16* dV;
+    int junction_items;    // SEGK dQ: as FwdParams
+    float* dKseg;          // SEGK dK/dV: float32 partials per segment key row [rows][Hkv][DH]
+    float* dVseg;
 };
 
+template <bool SEGK>
 __global__ void __launch_bounds__(NT_BWD, 1)
     k_attn_dq_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmDO,
                  const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, BwdParams p) {
@@ -460,13 +509,11 @@ __global__ void __launch_bounds__(NT_BWD, 1)
     __shared__ uint32_t tmem_base;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int h = blockIdx.x % p.Hq;
-    const int r = blockIdx.x / p.Hq;
-    const int qt = p.max_tiles - 1 - r / p.n_traj;
-    const int b = r % p.n_traj;
     const VisView& v = p.v;
+    const QItem it = q_item<SEGK>(v, p.Hq, p.max_tiles, p.n_traj, p.junction_items);
+    if (!it.ok) return;
+    const int h = it.h, qt = it.qt, b = it.b;
     const int nt = v.traj_tile[b + 1] - v.traj_tile[b];
-    if (qt >= nt) return;
     const int64_t g = v.traj_tile[b] + qt;
     const int64_t tok0 = v.traj_tok[b];
     const int T = v.traj_tok[b + 1] - (int)tok0;
@@ -511,6 +558,8 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             mbar_expect_tx(&q_full, 2 * TILE_B);
             load_tile(sm + DQ_Q, &tmQ, &q_full, h, row0);
             load_tile(sm + DQ_DO, &tmDO, &q_full, h, row0);
+            // first K row of the trajectory (SEGK: of the item's segment key rows)
+            const int64_t krow0 = SEGK ? (v.traj_km[b] + (int64_t)it.s * nt) * 128 : tok0;
             for (int j = 0; j < n; ++j) {
                 const int kt = v.fwd_idx[p0 + j] >> 4;
                 const int s = j & 1;
@@ -520,7 +569,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
                 load_tile(sm + DQ_V + s * TILE_B, &tmV, &v_full[s], kvh, row);
                 if (j >= 2 && !mbar_wait(&k_empty[s], ((j - 2) >> 1) & 1, status, 112)) break;
                 mbar_expect_tx(&k_full[s], TILE_B);
-                load_tile(sm + DQ_K + s * TILE_B, &tmK, &k_full[s], kvh, row);
+                load_tile(sm + DQ_K + s * TILE_B, &tmK, &k_full[s], kvh, (int)(krow0 + kt * 128));
             }
         }
     } else if (warp == 1 || warp == BWD_ACC_WARP) {
@@ -728,12 +777,13 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             tc_fence_after();
             __nv_bfloat16* qrow = p.dQ + ((tok0 + ie) * p.Hq + h) * DH;
             uint32_t o[32];
+            const bool store = i < T && (!SEGK || seg == it.s);
 #pragma unroll
             for (int cc = 0; cc < 2; ++cc) {
                 const int c = 2 * ch + cc;
                 tmem_ld32(lane_base + TM_DQ + c * 32, o);
                 tmem_wait_ld();
-                if (i < T) {
+                if (store) {
 #pragma unroll
                     for (int x = 0; x < 4; ++x) {
                         uint4 pk;
@@ -783,6 +833,7 @@ __device__ __forceinline__ uint64_t mnmaj_ht(uint32_t base, int ks) {
     return sdesc_sw128(base + ks * 2048, HT_HALF, 1024);
 }
 
+template <bool SEGK>
 __global__ void __launch_bounds__(NT_BWD, 1)
     k_attn_dkdv_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmDO,
                    const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, BwdParams p) {
@@ -805,8 +856,36 @@ __global__ void __launch_bounds__(NT_BWD, 1)
     const int64_t gk = v.traj_tile[b] + kt;
     const int64_t tok0 = v.traj_tok[b];
     const int T = v.traj_tok[b + 1] - (int)tok0;
-    const int p0 = v.bwd_ptr[gk];
-    const int nlist = v.bwd_ptr[gk + 1] - p0;
+    int p0 = v.bwd_ptr[gk];
+    int nlist = v.bwd_ptr[gk + 1] - p0;
+    int seg_lo = 0, seg_hi = T;        // SEGK: rows [seg_lo, seg_hi) of the item's segment
+    int64_t krow0 = tok0 + kt * 128;   // first K row of the tile
+    if (SEGK) {
+        // item (k-tile, segment blockIdx.y): only that segment's rows, which
+        // read the segment's key rows; its q-tiles are a contiguous run of the
+        // ascending list
+        const int sgb = v.traj_seg[b];
+        const int sk = blockIdx.y;
+        if (sk >= v.traj_seg[b + 1] - sgb) return;
+        seg_lo = v.seg_start[sgb + sk];
+        seg_hi = sgb + sk + 1 < v.traj_seg[b + 1] ? v.seg_start[sgb + sk + 1] : T;
+        if (kt * 128 >= seg_hi) return;   // every key of the tile comes after the segment
+        const int qlo = seg_lo >> 7, qhi = (seg_hi - 1) >> 7;
+        int a = 0, z = nlist;             // first entry with q-tile >= qlo
+        while (a < z) {
+            const int m = (a + z) >> 1;
+            if ((v.bwd_idx[p0 + m] >> 4) < qlo) a = m + 1; else z = m;
+        }
+        int c = a, y = nlist;             // first entry with q-tile > qhi
+        while (c < y) {
+            const int m = (c + y) >> 1;
+            if ((v.bwd_idx[p0 + m] >> 4) <= qhi) c = m + 1; else y = m;
+        }
+        p0 += a;
+        nlist = c - a;
+        if (nlist == 0) return;           // no row of the segment sees a key of the tile
+        krow0 = (v.traj_km[b] + (int64_t)sk * nt + kt) * 128;
+    }
     const int nsteps = nlist * grp * 2;
     int32_t* status = v.status;
     if (*(volatile int32_t*)&status[1]) return;
@@ -864,7 +943,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             prefetch_tmap(&tmK);
             prefetch_tmap(&tmV);
             mbar_expect_tx(&kv_full, 2 * TILE_B);
-            load_tile(sm + KV_K, &tmK, &kv_full, kvh, (int)(tok0 + kt * 128));
+            load_tile(sm + KV_K, &tmK, &kv_full, kvh, (int)krow0);
             load_tile(sm + KV_V, &tmV, &kv_full, kvh, (int)(tok0 + kt * 128));
             Cursor c = first;
             int s = 0;
@@ -940,7 +1019,9 @@ __global__ void __launch_bounds__(NT_BWD, 1)
         const int rl = qw * 32 + lane;               // key row inside the k-tile = TMEM lane
         const int jk = kt * 128 + rl;
         const int je = min(jk, T - 1);
-        const int iend = jk < T ? min(v.omega[tok0 + je], T) : 0;   // rows [jk, iend) see this key
+        const int iend0 = jk < T ? min(v.omega[tok0 + je], T) : 0;   // rows [jk, iend0) see this key
+        const int jlo = SEGK ? max(jk, seg_lo) : jk;                  // ... of which the item's rows:
+        const int iend = SEGK ? min(iend0, seg_hi) : iend0;            // [jlo, iend)
         const uint32_t lane_base = tmem + ((uint32_t)(qw * 32) << 16);
         bool ok = true;
         // (-LSE2, Delta) of this warp's 32 query rows of a step: 256 contiguous
@@ -981,7 +1062,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
                 }
             }
             // visible columns [lo, hi) of this warp's 32, as a bit mask
-            const int lo = min(max(jk, q0 + 32 * ch) - q0 - 32 * ch, 32);
+            const int lo = min(max(jlo, q0 + 32 * ch) - q0 - 32 * ch, 32);
             const int hi = max(min(min(iend, q0 + 64) - q0 - 32 * ch, 32), lo);
             const uint32_t vm = (hi >= 32 ? 0xffffffffu : ((1u << hi) - 1u)) & ~(lo >= 32 ? 0xffffffffu : ((1u << lo) - 1u));
             {   // P^T, dS^T (bf16 pairs) over the first 16 of this warp's own 32
@@ -1008,7 +1089,32 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             cur = nxt;
             advance(nxt);
         }
-        if (ok && nsteps > 0 && mbar_wait(&sd_free[(nsteps - 1) & 1], ((nsteps - 1) >> 1) & 1, status, 323)) {
+        if (SEGK && ok && mbar_wait(&sd_free[(nsteps - 1) & 1], ((nsteps - 1) >> 1) & 1, status, 323)) {
+            // float32 partials of this segment, unscaled dV and scaled dK
+            tc_fence_after();
+            const int64_t row = ((krow0 + rl) * p.Hkv + kvh) * DH;
+            uint32_t o[32];
+#pragma unroll
+            for (int pass = 0; pass < 2; ++pass) {
+                float* dst = (pass == 0 ? p.dVseg : p.dKseg) + row;
+                const float mul = pass == 0 ? 1.f : p.scale;
+                const uint32_t col = pass == 0 ? TM_DV : TM_DK;
+#pragma unroll
+                for (int cc = 0; cc < 2; ++cc) {
+                    const int c = 2 * ch + cc;
+                    tmem_ld32(lane_base + col + c * 32, o);
+                    tmem_wait_ld();
+                    if (jk < T) {
+#pragma unroll
+                        for (int x = 0; x < 8; ++x)
+                            *reinterpret_cast<float4*>(dst + c * 32 + 4 * x) =
+                                make_float4(__uint_as_float(o[4 * x + 0]) * mul, __uint_as_float(o[4 * x + 1]) * mul,
+                                            __uint_as_float(o[4 * x + 2]) * mul, __uint_as_float(o[4 * x + 3]) * mul);
+                    }
+                }
+            }
+        } else if (!SEGK && ok && nsteps > 0 &&
+                   mbar_wait(&sd_free[(nsteps - 1) & 1], ((nsteps - 1) >> 1) & 1, status, 323)) {
             tc_fence_after();
             const int64_t row = ((tok0 + je) * p.Hkv + kvh) * DH;
             uint32_t o[32];
@@ -1035,7 +1141,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
                     }
                 }
             }
-        } else if (jk < T) {
+        } else if (!SEGK && jk < T) {
             // no listed q-tile (cannot happen: the diagonal tile is always listed)
             const int64_t row = ((tok0 + je) * p.Hkv + kvh) * DH;
             for (int c = 0; c < DH; ++c) {
@@ -1072,12 +1178,53 @@ mw_status attn_fwd_tc(const mw_vis_layout* L, const void* vis, const void* Q, co
     p.scale_log2 = scale * LOG2E;
     p.O = (__nv_bfloat16*)O;
     p.LSE = LSE;
-    mw_status st = cuda_status(cudaFuncSetAttribute(k_attn_fwd_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    p.junction_items = 0;
+    mw_status st = cuda_status(cudaFuncSetAttribute(k_attn_fwd_tc<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                     (int)SMEM_FWD));
     if (st != MW_OK) return st;
     const unsigned grid = (unsigned)((int64_t)L->max_tiles * L->n_traj * Hq);
     count_launches(1);
-    k_attn_fwd_tc<<<grid, NT_FWD, SMEM_FWD, s>>>(tq, tk, tv, p);
+    k_attn_fwd_tc<false><<<grid, NT_FWD, SMEM_FWD, s>>>(tq, tk, tv, p);
+    return launch_status();
+}
+
+// Rows of segment key rows (keys per segment) and whether TMA's int32 row
+// coordinates and the junction-item grid reach them.
+static bool segk_fits(const mw_vis_layout* L, int Hq) {
+    return L->n_keymask * 128 <= INT32_MAX && L->n_segs * (int64_t)Hq <= INT32_MAX &&
+           L->n_segs - L->n_traj + 1 <= 65535;
+}
+
+mw_status attn_fwd_tc_segk(const mw_vis_layout* L, const void* vis, const void* Q, const void* Kseg, const void* V,
+                           void* O, float* LSE, int Hq, int Hkv, float scale, cudaStream_t s) {
+    if (L->n_tiles == 0) return MW_OK;
+    if (!segk_fits(L, Hq)) return MW_ESHAPE;
+    CUtensorMap tq, tk, tv;
+    const uint64_t T = (uint64_t)L->total_tokens;
+    if (!tmap_bf16_3d(&tq, Q, T, Hq, DH, 128, 64) ||
+        !tmap_bf16_3d(&tk, Kseg, (uint64_t)L->n_keymask * 128, Hkv, DH, 128, 64) ||
+        !tmap_bf16_3d(&tv, V, T, Hkv, DH, 128, 64))
+        return MW_ECUDA;
+    FwdParams p;
+    p.v = make_view(L, vis);
+    p.total = L->total_tokens;
+    p.n_traj = L->n_traj;
+    p.max_tiles = L->max_tiles;
+    p.Hq = Hq;
+    p.Hkv = Hkv;
+    p.scale_log2 = scale * LOG2E;
+    p.O = (__nv_bfloat16*)O;
+    p.LSE = LSE;
+    p.junction_items = 0;
+    mw_status st = cuda_status(cudaFuncSetAttribute(k_attn_fwd_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                    (int)SMEM_FWD));
+    if (st != MW_OK) return st;
+    count_launches(1);
+    k_attn_fwd_tc<true><<<(unsigned)((int64_t)L->max_tiles * L->n_traj * Hq), NT_FWD, SMEM_FWD, s>>>(tq, tk, tv, p);
+    if ((st = launch_status()) != MW_OK || L->n_junc == 0) return st;
+    p.junction_items = 1;
+    count_launches(1);
+    k_attn_fwd_tc<true><<<(unsigned)(L->n_segs * Hq), NT_FWD, SMEM_FWD, s>>>(tq, tk, tv, p);
     return launch_status();
 }
 
@@ -1150,16 +1297,82 @@ mw_status attn_bwd_tc(const mw_vis_layout* L, const void* vis, const void* Q, co
     p.dQ = (__nv_bfloat16*)dQ;
     p.dK = (__nv_bfloat16*)dK;
     p.dV = (__nv_bfloat16*)dV;
-    if ((st = cuda_status(cudaFuncSetAttribute(k_attn_dq_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    p.junction_items = 0;
+    p.dKseg = p.dVseg = nullptr;
+    if ((st = cuda_status(cudaFuncSetAttribute(k_attn_dq_tc<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                (int)SMEM_DQ))) != MW_OK)
         return st;
-    if ((st = cuda_status(cudaFuncSetAttribute(k_attn_dkdv_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    if ((st = cuda_status(cudaFuncSetAttribute(k_attn_dkdv_tc<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                (int)SMEM_KV))) != MW_OK)
         return st;
     count_launches(2);
-    k_attn_dq_tc<<<(unsigned)((int64_t)L->max_tiles * L->n_traj * Hq), NT_BWD, SMEM_DQ, s>>>(tq, tdo, tk, tv, p);
-    k_attn_dkdv_tc<<<(unsigned)((int64_t)L->max_tiles * L->n_traj * Hkv), NT_BWD, SMEM_KV, s>>>(tq64, tdo64, tk,
-                                                                                                   tv, p);
+    k_attn_dq_tc<false><<<(unsigned)((int64_t)L->max_tiles * L->n_traj * Hq), NT_BWD, SMEM_DQ, s>>>(tq, tdo, tk, tv,
+                                                                                                   p);
+    k_attn_dkdv_tc<false><<<(unsigned)((int64_t)L->max_tiles * L->n_traj * Hkv), NT_BWD, SMEM_KV, s>>>(
+        tq64, tdo64, tk, tv, p);
+    return launch_status();
+}
+
+// Backward with segment key rows: (-LSE2, Delta) pairs into `ws`, dQ of the
+// rotated queries (bf16, main + junction launches), and per segment key row
+// the float32 partials dKseg (scaled) and dVseg.
+mw_status attn_bwd_tc_segk(const mw_vis_layout* L, const void* vis, const void* Q, const void* Kseg, const void* V,
+                           const void* O, const void* dO, const float* LSE, void* dQ, float* dKseg, float* dVseg,
+                           int Hq, int Hkv, float scale, float* ws, cudaStream_t s) {
+    if (L->n_tiles == 0) return MW_OK;
+    if (!segk_fits(L, Hq)) return MW_ESHAPE;
+    const int64_t n_rows = L->n_tiles * 128;
+    float2* lsd = reinterpret_cast<float2*>(ws);
+    const VisView view = make_view(L, vis);
+    count_launches(1);
+    k_attn_lsd<<<(unsigned)std::min<int64_t>(ceil_div(n_rows * Hq, 8), 152 * 64), 256, 0, s>>>(
+        view, L->total_tokens, n_rows, Hq, (const __nv_bfloat16*)O, (const __nv_bfloat16*)dO, LSE, lsd);
+    mw_status st = launch_status();
+    if (st != MW_OK) return st;
+    const uint64_t T = (uint64_t)L->total_tokens;
+    const uint64_t KR = (uint64_t)L->n_keymask * 128;
+    CUtensorMap tq, tdo, tk, tv, tq64, tdo64;
+    if (!tmap_bf16_3d(&tq, Q, T, Hq, DH, 128, 64) || !tmap_bf16_3d(&tdo, dO, T, Hq, DH, 128, 64) ||
+        !tmap_bf16_3d(&tk, Kseg, KR, Hkv, DH, 128, 64) || !tmap_bf16_3d(&tv, V, T, Hkv, DH, 128, 64) ||
+        !tmap_bf16_3d(&tq64, Q, T, Hq, DH, 64, 64) || !tmap_bf16_3d(&tdo64, dO, T, Hq, DH, 64, 64))
+        return MW_ECUDA;
+    BwdParams p;
+    p.v = view;
+    p.total = L->total_tokens;
+    p.n_traj = L->n_traj;
+    p.max_tiles = L->max_tiles;
+    p.Hq = Hq;
+    p.Hkv = Hkv;
+    p.scale = scale;
+    p.scale_log2 = scale * LOG2E;
+    p.lsd = lsd;
+    p.n_rows = n_rows;
+    p.dQ = (__nv_bfloat16*)dQ;
+    p.dK = p.dV = nullptr;
+    p.dKseg = dKseg;
+    p.dVseg = dVseg;
+    p.junction_items = 0;
+    if ((st = cuda_status(cudaFuncSetAttribute(k_attn_dq_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               (int)SMEM_DQ))) != MW_OK)
+        return st;
+    if ((st = cuda_status(cudaFuncSetAttribute(k_attn_dkdv_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               (int)SMEM_KV))) != MW_OK)
+        return st;
+    count_launches(1);
+    k_attn_dq_tc<true><<<(unsigned)((int64_t)L->max_tiles * L->n_traj * Hq), NT_BWD, SMEM_DQ, s>>>(tq, tdo, tk, tv,
+                                                                                                  p);
+    if ((st = launch_status()) != MW_OK) return st;
+    if (L->n_junc > 0) {
+        p.junction_items = 1;
+        count_launches(1);
+        k_attn_dq_tc<true><<<(unsigned)(L->n_segs * Hq), NT_BWD, SMEM_DQ, s>>>(tq, tdo, tk, tv, p);
+        if ((st = launch_status()) != MW_OK) return st;
+        p.junction_items = 0;
+    }
+    // grid.y: the most segments one trajectory can have
+    const dim3 gk((unsigned)((int64_t)L->max_tiles * L->n_traj * Hkv), (unsigned)(L->n_segs - L->n_traj + 1));
+    count_launches(1);
+    k_attn_dkdv_tc<true><<<gk, NT_BWD, SMEM_KV, s>>>(tq64, tdo64, tk, tv, p);
     return launch_status();
 }
 

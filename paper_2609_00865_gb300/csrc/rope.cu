@@ -175,8 +175,9 @@ __global__ void __launch_bounds__(256) k_rope_segments(VisView v, const int32_t*
     }
 }
 
-// Transpose of k_rope_segments: dX[j] = sum_{s: j in view_s} R(p_s(j))^T dY_s[j].
-template <typename T>
+// Transpose of k_rope_segments: dX[j] = sum_{s: j in view_s} R(p_s(j))^T dY_s[j]
+// (ROT = false: the plain sum over those segments, for values read unrotated).
+template <typename T, bool ROT>
 __global__ void __launch_bounds__(256) k_rope_segments_bwd(VisView v, const int32_t* __restrict__ pos,
                                                            const float2* __restrict__ table, int n_pos,
                                                            const float* __restrict__ dY, T* __restrict__ dX,
@@ -192,12 +193,18 @@ __global__ void __launch_bounds__(256) k_rope_segments_bwd(VisView v, const int3
         for (int s = 0; s < r.nseg; ++s) {
             const int64_t row = (r.kmb + (int64_t)s * r.nt + r.kt) * MW_TILE + jj;
             const int p = pos[row];
-            if (p < 0 || !pos_ok(v, p, n_pos)) continue;
+            if (p < 0) continue;
             const int64_t yo = (row * H + h) * Dh + f;
-            float y0, y1;
-            rotate(dY[yo], dY[yo + half], table[(int64_t)p * half + f], -1.f, y0, y1);
-            a0 += y0;
-            a1 += y1;
+            if (ROT) {
+                if (!pos_ok(v, p, n_pos)) continue;
+                float y0, y1;
+                rotate(dY[yo], dY[yo + half], table[(int64_t)p * half + f], -1.f, y0, y1);
+                a0 += y0;
+                a1 += y1;
+            } else {
+                a0 += dY[yo];
+                a1 += dY[yo + half];
+            }
         }
         const int64_t xo = ((r.tok0 + r.kt * MW_TILE + jj) * H + h) * Dh + f;
         st_f(dX + xo, a0);
@@ -255,16 +262,26 @@ mw_status rope_segments(const mw_vis_layout* L, const void* vis, const int32_t* 
 }
 
 mw_status rope_segments_bwd(const mw_vis_layout* L, const void* vis, const int32_t* pos, const float* table,
-                            int n_pos, const float* dY, void* dX, int H, int Dh, int dtype, cudaStream_t s) {
+                            int n_pos, const float* dY, void* dX, int H, int Dh, int dtype, bool rotate_back,
+                            cudaStream_t s) {
     if (L->n_tiles == 0 || H == 0) return MW_OK;
     VisView v = make_view(L, vis);
     const float2* tb = reinterpret_cast<const float2*>(table);
+    const unsigned grid = (unsigned)L->n_tiles;
     count_launches(1);
-    if (dtype == MW_F32)
-        k_rope_segments_bwd<float><<<(unsigned)L->n_tiles, 256, 0, s>>>(v, pos, tb, n_pos, dY, (float*)dX, H, Dh);
-    else
-        k_rope_segments_bwd<__nv_bfloat16><<<(unsigned)L->n_tiles, 256, 0, s>>>(v, pos, tb, n_pos, dY,
-                                                                                (__nv_bfloat16*)dX, H, Dh);
+    if (dtype == MW_F32) {
+        if (rotate_back)
+            k_rope_segments_bwd<float, true><<<grid, 256, 0, s>>>(v, pos, tb, n_pos, dY, (float*)dX, H, Dh);
+        else
+            k_rope_segments_bwd<float, false><<<grid, 256, 0, s>>>(v, pos, tb, n_pos, dY, (float*)dX, H, Dh);
+    } else {
+        if (rotate_back)
+            k_rope_segments_bwd<__nv_bfloat16, true><<<grid, 256, 0, s>>>(v, pos, tb, n_pos, dY, (__nv_bfloat16*)dX,
+                                                                           H, Dh);
+        else
+            k_rope_segments_bwd<__nv_bfloat16, false><<<grid, 256, 0, s>>>(v, pos, tb, n_pos, dY, (__nv_bfloat16*)dX,
+                                                                            H, Dh);
+    }
     return launch_status();
 }
 

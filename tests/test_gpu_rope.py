@@ -155,6 +155,55 @@ def test_rope_attention_bf16_tile_edges():
     assert_grad_bf16(np64(dV), dVr, "dV")
 
 
+@pytest.mark.parametrize("Hq,Hkv", [(8, 2), (4, 4)])
+def test_rope_attention_bf16_tensor_cores(Hq, Hkv):
+    """bf16 with Dh 128 runs on the tensor-core kernels with segment key rows:
+    junctions inside q-tiles (one CTA per segment of such a tile) and keys
+    whose position differs between segments."""
+    seqlens, edits = _medium_record(8)
+    Q, K, V, dO = _tensors(sum(seqlens), Hq, Hkv, 128, 151 + Hq, torch.bfloat16)
+    scale, theta = 128 ** -0.5, 1e6
+    O, LSE, dQ, dK, dV = _run(seqlens, edits, Q, K, V, dO, scale, theta)
+    Or, Lr = OA.attn_fwd(seqlens, edits, np64(Q), np64(K), np64(V), scale, rope_theta=theta)
+    assert_maxabs(np64(O), Or, 2e-2, "O")
+    assert_maxabs(np64(LSE), Lr, 2e-2, "LSE")
+    dQr, dKr, dVr = OA.attn_bwd(seqlens, edits, np64(Q), np64(K), np64(V), np64(dO), scale, rope_theta=theta)
+    assert_grad_bf16(np64(dQ), dQr, "dQ")
+    assert_grad_bf16(np64(dK), dKr, "dK")
+    assert_grad_bf16(np64(dV), dVr, "dV")
+
+
+def test_rope_attention_bf16_junctions_on_tile_edges():
+    """Junctions at a tile's first row (128) and two and four rows into that
+    tile (130, 132): three segments inside one q-tile."""
+    seqlens = [700]
+    edits = [[(128, [(0, 100)]), (130, [(101, 120)]), (132, [(5, 7)]), (300, [(129, 250)])]]
+    Q, K, V, dO = _tensors(700, 4, 2, 128, 161, torch.bfloat16)
+    scale, theta = 128 ** -0.5, 1e4
+    O, LSE, dQ, dK, dV = _run(seqlens, edits, Q, K, V, dO, scale, theta)
+    Or, Lr = OA.attn_fwd(seqlens, edits, np64(Q), np64(K), np64(V), scale, rope_theta=theta)
+    assert_maxabs(np64(O), Or, 2e-2, "O")
+    assert_maxabs(np64(LSE), Lr, 2e-2, "LSE")
+    dQr, dKr, dVr = OA.attn_bwd(seqlens, edits, np64(Q), np64(K), np64(V), np64(dO), scale, rope_theta=theta)
+    assert_grad_bf16(np64(dQ), dQr, "dQ")
+    assert_grad_bf16(np64(dK), dKr, "dK")
+    assert_grad_bf16(np64(dV), dVr, "dV")
+
+
+def test_rope_attention_bf16_head_dim_64():
+    """bf16 with Dh 64 takes the CUDA-core kernels."""
+    seqlens, edits = _medium_record(9)
+    Q, K, V, dO = _tensors(sum(seqlens), 4, 2, 64, 171, torch.bfloat16)
+    scale, theta = 64 ** -0.5, 1e4
+    O, LSE, dQ, dK, dV = _run(seqlens, edits, Q, K, V, dO, scale, theta)
+    Or, Lr = OA.attn_fwd(seqlens, edits, np64(Q), np64(K), np64(V), scale, rope_theta=theta)
+    assert_maxabs(np64(O), Or, 2e-2, "O")
+    dQr, dKr, dVr = OA.attn_bwd(seqlens, edits, np64(Q), np64(K), np64(V), np64(dO), scale, rope_theta=theta)
+    assert_grad_bf16(np64(dQ), dQr, "dQ")
+    assert_grad_bf16(np64(dK), dKr, "dK")
+    assert_grad_bf16(np64(dV), dVr, "dV")
+
+
 def test_rope_later_edit_leaves_earlier_rows_unchanged():
     """Conditioning invariant (§3.3) with rotary positions: a junction added at
     row 600 changes neither the positions nor the outputs of rows before it."""
