@@ -147,12 +147,13 @@ def job_value(scored_per_rank, world, ms):
     return scored_per_rank * world / (ms * 1e-3)
 
 
-def make_workload(cfg, K=None, f=None, seed_offset=0, n_traj=None, pin=True):
+def make_workload(cfg, K=None, f=None, seed_offset=0, n_traj=None, pin=True, rope=None):
     """Host-side inputs of one workload (CPU tensors, pinned unless ``pin`` is
     False, + record).
 
     ``n_traj`` keeps only the first trajectories of the record (a smaller
-    case of the same kernels, for profiler captures)."""
+    case of the same kernels, for profiler captures). ``rope`` (a rotary
+    theta) runs the attention with row-wise logical rotary positions."""
     import numpy as np
     import torch
 
@@ -160,6 +161,8 @@ def make_workload(cfg, K=None, f=None, seed_offset=0, n_traj=None, pin=True):
     c = synth.CONFIGS[cfg]
     g = torch.Generator().manual_seed(replica_seed(cfg, seed_offset))
     w = {"cfg": cfg}
+    if rope is not None and cfg in (2, 4, 5):
+        w["rope"] = float(rope)
     bf = torch.bfloat16
 
     def randn(*shape, std=1.0):
@@ -213,6 +216,8 @@ def describe(w):
                  head_dim=w["heads"][2])
     if "rows" in w:
         d.update(loss_rows=int(w["rows"].numel()), hidden=w["d"], vocab=w["Vocab"])
+    if "rope" in w:
+        d["rope_theta"] = w["rope"]
     d["l2"] = "inputs larger than L2 (129 MB); no flush"
     return d
 
@@ -246,7 +251,14 @@ class Step:
             self.dQ = torch.empty_like(self.O)
             self.dK = torch.empty(T, Hkv, Dh, dtype=torch.bfloat16, device=device)
             self.dV = torch.empty_like(self.dK)
-            nb = mw.mw_masked_attn_bwd_ws(self.vis, Hq, Dh, mw.MW_BF16)
+            if "rope" in w:
+                # positions per (segment, key) and the cos/sin table (built once,
+                # like weights); one workspace serves both calls (shared prefix)
+                self.pos = torch.empty(max(self.L.n_keymask * mw.TILE, 1), dtype=torch.int32, device=device)
+                self.table = mw.rope_table(mw.TILE * self.L.max_tiles, Dh, w["rope"], device=device)
+                nb = mw.mw_masked_attn_rope_ws(self.vis, Hq, Hkv, Dh, mw.MW_BF16)[1]
+            else:
+                nb = mw.mw_masked_attn_bwd_ws(self.vis, Hq, Dh, mw.MW_BF16)
             self.attn_ws = torch.empty(max(nb, 1), dtype=torch.uint8, device=device)
         if "rows" in w:
             M = int(w["rows"].numel())
@@ -292,12 +304,24 @@ class Step:
         cu, J, jt, off, spans = self.flat
         self._ev("mw_build_visibility", lambda: self.mw.mw_build_visibility(
             self.L, cu, J, jt, off, spans, self.vis.ws, self.vis.vis, self.stream))
+        if "rope" in self.w:
+            self._ev("mw_logical_positions", lambda: self.mw.mw_logical_positions(self.vis, self.pos, self.stream))
 
     def attn_fwd(self):
+        if "rope" in self.w:
+            self._ev("mw_masked_attn_rope_fwd", lambda: self.mw.mw_masked_attn_rope_fwd(
+                self.vis, self.pos, self.table, self.d["Q"], self.d["K"], self.d["V"], self.O, self.LSE,
+                self.scale, self.attn_ws, self.stream))
+            return
         self._ev("mw_masked_attn_fwd", lambda: self.mw.mw_masked_attn_fwd(
             self.vis, self.d["Q"], self.d["K"], self.d["V"], self.O, self.LSE, self.scale, self.stream))
 
     def attn_bwd(self, dO):
+        if "rope" in self.w:
+            self._ev("mw_masked_attn_rope_bwd", lambda: self.mw.mw_masked_attn_rope_bwd(
+                self.vis, self.pos, self.table, self.d["Q"], self.d["K"], self.d["V"], self.O, dO, self.LSE,
+                self.dQ, self.dK, self.dV, self.scale, self.attn_ws, self.stream))
+            return
         self._ev("mw_masked_attn_bwd", lambda: self.mw.mw_masked_attn_bwd(
             self.vis, self.d["Q"], self.d["K"], self.d["V"], self.O, dO, self.LSE, self.dQ, self.dK, self.dV,
             self.scale, self.attn_ws, self.stream))
@@ -397,9 +421,10 @@ def cpu_sample(w, budget_s=15.0):
             r = w["record"]
             Hq, Hkv, Dh = w["heads"]
             parts.append("attention fwd+dQ, all heads")
-            O, _ = OA.attn_fwd(r.seqlens, r.edits, x["Q"], x["K"], x["V"], Dh ** -0.5, rows=rows)
+            th = w.get("rope")
+            O, _ = OA.attn_fwd(r.seqlens, r.edits, x["Q"], x["K"], x["V"], Dh ** -0.5, rows=rows, rope_theta=th)
             OA.attn_bwd_rows(r.seqlens, r.edits, x["Q"], x["K"], x["V"], x.get("dO", x["Q"]), Dh ** -0.5,
-                             rows, list(range(Hq)))
+                             rows, list(range(Hq)), rope_theta=th)
         if "rows" in w:
             parts.append("LM-head fwd over the full vocabulary + dH/dW")
             if "H" in x:
@@ -418,7 +443,8 @@ def cpu_sample(w, budget_s=15.0):
 def run_reference(args, rank, world):
     if rank != 0:
         return
-    w = make_workload(args.config, args.K, args.f, n_traj=args.n_traj, pin=False)   # the oracle runs on the host
+    w = make_workload(args.config, args.K, args.f, n_traj=args.n_traj, pin=False,   # the oracle runs on the host
+                      rope=args.rope)
     vals = []
     for i in range(args.warmup + args.steps):
         v, cores, desc = cpu_sample(w, budget_s=args.cpu_seconds / max(1, args.steps))
@@ -443,7 +469,7 @@ def run_gpu(args, rank, world, local_rank):
     import paper_2609_00865_gb300 as mw
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
-    w = make_workload(args.config, args.K, args.f, seed_offset=rank, n_traj=args.n_traj)
+    w = make_workload(args.config, args.K, args.f, seed_offset=rank, n_traj=args.n_traj, rope=args.rope)
     step = Step(w, dev)
     step.prime()
     for _ in range(args.warmup):
@@ -528,6 +554,8 @@ def run_gpu(args, rank, world, local_rank):
     dom = max(per_call, key=per_call.get)
     dom_flops = {"mw_masked_attn_fwd": 4.0 / 14.0 * flops.get("attn", 0),
                  "mw_masked_attn_bwd": 10.0 / 14.0 * flops.get("attn", 0),
+                 "mw_masked_attn_rope_fwd": 4.0 / 14.0 * flops.get("attn", 0),
+                 "mw_masked_attn_rope_bwd": 10.0 / 14.0 * flops.get("attn", 0),
                  "mw_logprob_loss_fwd": 2.0 / 8.0 * flops.get("lm", 0),
                  "mw_logprob_loss_bwd": 6.0 / 8.0 * flops.get("lm", 0)}.get(dom, 0.0)
     achieved = dom_flops / (per_call[dom] * 1e-3) / 1e12
@@ -575,6 +603,8 @@ def main():
                     help="keep only the first trajectories (smaller case for profiler captures)")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--rope", type=float, default=None, metavar="THETA",
+                    help="attention with row-wise logical rotary positions (theta of the rotary table)")
     args = ap.parse_args()
     rank = int(os.environ.get("RANK", 0))
     world = int(os.environ.get("WORLD_SIZE", args.gpus if args.gpus == 1 else 1))

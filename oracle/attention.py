@@ -182,10 +182,10 @@ def attn_bwd(seqlens, edits_per_traj, Q, K, V, dO, scale, groups=None, rope_thet
     return dQ, dK, dV
 
 
-def attn_bwd_rows(seqlens, edits_per_traj, Q, K, V, dO, scale, rows, heads):
+def attn_bwd_rows(seqlens, edits_per_traj, Q, K, V, dO, scale, rows, heads, rope_theta=None):
     """dQ of a few physical rows and query heads (same formulas as
-    ``attn_bwd``; a row's dQ needs only its own segment's compact view).
-    Returns ``dQ_sel[r, h_i, :]``."""
+    ``attn_bwd``, rotary positions included; a row's dQ needs only its own
+    segment's compact view). Returns ``dQ_sel[r, h_i, :]``."""
     Q = np.asarray(Q, dtype=np.float64)
     K = np.asarray(K, dtype=np.float64)
     V = np.asarray(V, dtype=np.float64)
@@ -206,13 +206,20 @@ def attn_bwd_rows(seqlens, edits_per_traj, Q, K, V, dO, scale, rows, heads):
         for hi, h in enumerate(heads):
             k = K[idx, h // grp]
             v = V[idx, h // grp]
-            s = _scores(Q[grows, h], k, scale, n_before + part)
+            q = Q[grows, h]
+            if rope_theta is not None:
+                k = rope(k, np.arange(idx.size), rope_theta)
+                q = rope(q, n_before + part, rope_theta)
+            s = _scores(q, k, scale, n_before + part)
             m = s.max(axis=1, keepdims=True)
             p = np.exp(s - m)
             p /= p.sum(axis=1, keepdims=True)
             dp = dO[grows, h] @ v.T
             ds = p * (dp - (p * dp).sum(axis=1, keepdims=True))
-            out[outp, hi] = scale * (ds @ k)
+            dq = scale * (ds @ k)
+            if rope_theta is not None:
+                dq = rope(dq, n_before + part, rope_theta, inverse=True)
+            out[outp, hi] = dq
     return out
 
 

@@ -32,7 +32,10 @@ from ._lib import (  # noqa: F401
     mw_logprob_ws,
     mw_masked_attn_bwd,
     mw_masked_attn_bwd_ws,
+    mw_logical_positions,
     mw_masked_attn_fwd,
+    mw_masked_attn_rope_bwd,
+    mw_masked_attn_rope_fwd,
     mw_masked_attn_rope_ws,
     mw_selftest_wait_timeout,
     mw_visibility_layout,

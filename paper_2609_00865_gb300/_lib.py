@@ -310,14 +310,18 @@ def masked_attn_bwd(vis, Q, K, V, O, dO, LSE, scale=None, ws=None, stream=None):
 
 # --- row-wise logical positions and rotary attention ---------------------------
 
+def mw_logical_positions(vis, pos, stream=None):
+    _check(_lib().mw_logical_positions(ctypes.byref(vis.layout), _ptr(vis.vis), _ptr(pos), _stream(stream)),
+           "mw_logical_positions")
+
+
 def logical_positions(vis, stream=None):
     """int32 [n_keymask * 128]: rank of key j in segment s's live view at
     (traj_km[b] + s nt_b) 128 + j, -1 for non-members (mw_logical_positions)."""
     import torch
     L = vis.layout
     pos = torch.empty(max(int(L.n_keymask) * TILE, 1), dtype=torch.int32, device=vis.vis.device)
-    _check(_lib().mw_logical_positions(ctypes.byref(L), _ptr(vis.vis), _ptr(pos), _stream(stream)),
-           "mw_logical_positions")
+    mw_logical_positions(vis, pos, stream)
     return pos
 
 
@@ -352,6 +356,22 @@ def mw_masked_attn_rope_ws(vis, Hq, Hkv, Dh, dtype):
     return int(f.value), int(b.value)
 
 
+def mw_masked_attn_rope_fwd(vis, pos, table, Q, K, V, O, LSE, scale, ws, stream=None):
+    Hq, Dh, Hkv = Q.shape[1], Q.shape[2], K.shape[1]
+    _check(_lib().mw_masked_attn_rope_fwd(ctypes.byref(vis.layout), _ptr(vis.vis), _ptr(pos), _ptr(table),
+                                          table.shape[0], _ptr(Q), _ptr(K), _ptr(V), _ptr(O), _ptr(LSE), Hq, Hkv,
+                                          Dh, _dtype_code(Q), float(scale), _ptr(ws), _stream(stream)),
+           "mw_masked_attn_rope_fwd")
+
+
+def mw_masked_attn_rope_bwd(vis, pos, table, Q, K, V, O, dO, LSE, dQ, dK, dV, scale, ws, stream=None):
+    Hq, Dh, Hkv = Q.shape[1], Q.shape[2], K.shape[1]
+    _check(_lib().mw_masked_attn_rope_bwd(ctypes.byref(vis.layout), _ptr(vis.vis), _ptr(pos), _ptr(table),
+                                          table.shape[0], _ptr(Q), _ptr(K), _ptr(V), _ptr(O), _ptr(dO), _ptr(LSE),
+                                          _ptr(dQ), _ptr(dK), _ptr(dV), Hq, Hkv, Dh, _dtype_code(Q), float(scale),
+                                          _ptr(ws), _stream(stream)), "mw_masked_attn_rope_bwd")
+
+
 def masked_attn_rope_fwd(vis, pos, table, Q, K, V, scale=None, ws=None, stream=None):
     """Masked attention with per-row logical rotary positions; returns O, LSE."""
     import torch
@@ -364,10 +384,7 @@ def masked_attn_rope_fwd(vis, pos, table, Q, K, V, scale=None, ws=None, stream=N
         ws = torch.empty(max(nbytes, 1), dtype=torch.uint8, device=Q.device)
     O = torch.empty_like(Q)
     LSE = torch.empty(Hq, Q.shape[0], dtype=torch.float32, device=Q.device)
-    _check(_lib().mw_masked_attn_rope_fwd(ctypes.byref(vis.layout), _ptr(vis.vis), _ptr(pos), _ptr(table),
-                                          table.shape[0], _ptr(Q), _ptr(K), _ptr(V), _ptr(O), _ptr(LSE), Hq, Hkv,
-                                          Dh, _dtype_code(Q), float(scale), _ptr(ws), _stream(stream)),
-           "mw_masked_attn_rope_fwd")
+    mw_masked_attn_rope_fwd(vis, pos, table, Q, K, V, O, LSE, scale, ws, stream)
     return O, LSE
 
 
@@ -383,10 +400,7 @@ def masked_attn_rope_bwd(vis, pos, table, Q, K, V, O, dO, LSE, scale=None, ws=No
         nbytes = mw_masked_attn_rope_ws(vis, Hq, Hkv, Dh, _dtype_code(Q))[1]
         ws = torch.empty(max(nbytes, 1), dtype=torch.uint8, device=Q.device)
     dQ, dK, dV = torch.empty_like(Q), torch.empty_like(K), torch.empty_like(V)
-    _check(_lib().mw_masked_attn_rope_bwd(ctypes.byref(vis.layout), _ptr(vis.vis), _ptr(pos), _ptr(table),
-                                          table.shape[0], _ptr(Q), _ptr(K), _ptr(V), _ptr(O), _ptr(dO), _ptr(LSE),
-                                          _ptr(dQ), _ptr(dK), _ptr(dV), Hq, Hkv, Dh, _dtype_code(Q), float(scale),
-                                          _ptr(ws), _stream(stream)), "mw_masked_attn_rope_bwd")
+    mw_masked_attn_rope_bwd(vis, pos, table, Q, K, V, O, dO, LSE, dQ, dK, dV, scale, ws, stream)
     return dQ, dK, dV
 
 

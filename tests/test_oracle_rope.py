@@ -242,3 +242,20 @@ def test_rope_without_edits_is_plain_causal_rope():
     ref = torch.nn.functional.scaled_dot_product_attention(q[None], k[None], torch.from_numpy(Vv[:, 0])[None],
                                                            is_causal=True, scale=0.5)[0]
     np.testing.assert_allclose(O[:, 0], ref.numpy(), rtol=1e-10, atol=1e-12)
+
+
+def test_rope_row_sampled_dq_matches_full():
+    """The sampled-row dQ (used to time the oracle on large workloads) equals
+    the full backward's rows with rotary positions too."""
+    rng = _rng(11)
+    seqlens = [70, 90]
+    edits = [_random_edits(rng, 70), _random_edits(rng, 90)]
+    T = sum(seqlens)
+    Q = rng.standard_normal((T, 4, 8))
+    K = rng.standard_normal((T, 2, 8))
+    Vv = rng.standard_normal((T, 2, 8))
+    dO = rng.standard_normal((T, 4, 8))
+    dQ, _, _ = A.attn_bwd(seqlens, edits, Q, K, Vv, dO, 0.3, rope_theta=300.0)
+    rows = np.array([0, 5, 69, 70, 111, 159])
+    got = A.attn_bwd_rows(seqlens, edits, Q, K, Vv, dO, 0.3, rows, [1, 3], rope_theta=300.0)
+    np.testing.assert_allclose(got, dQ[rows][:, [1, 3]], rtol=1e-12, atol=1e-12)
