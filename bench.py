@@ -29,6 +29,10 @@ sys.path.insert(0, ROOT)
 METRIC = "view-consistent scored tokens/sec (fwd+bwd)"
 
 
+# PPO / GRPO clip range of the loss: App. F.1 trains with the asymmetric 0.2 / 0.28
+EPS_LO, EPS_HI = 0.2, 0.28
+
+
 def _peaks():
     """(bf16 burst TFLOP/s, bf16 sustained TFLOP/s, HBM GB/s, source)."""
     try:
@@ -328,7 +332,7 @@ class Step:
 
     def lm_fwd(self):
         self._ev("mw_logprob_loss_fwd", lambda: self.mw.mw_logprob_loss_fwd(
-            self.H(), self.d["W"], self.d["targets"], self.d["rows"], self.lp_old, self.d["adv"], 0.2, 0.2,
+            self.H(), self.d["W"], self.d["targets"], self.d["rows"], self.lp_old, self.d["adv"], EPS_LO, EPS_HI,
             self.lp, self.ratio, self.lse, self.loss, self.lm_ws, self.stream))
 
     def lm_bwd(self):
@@ -433,7 +437,7 @@ def cpu_sample(w, budget_s=15.0):
                 H = np.zeros((w["N"], w["d"]))
                 H[rows] = O.reshape(len(rows), -1)
             lp, lse = OL.logprob(H, x["W"], w["targets"].numpy(), rows)
-            g = OL.policy_loss(lp, lp + 0.01, np.ones_like(lp), 0.2, 0.2)[3]
+            g = OL.policy_loss(lp, lp + 0.01, np.ones_like(lp), EPS_LO, EPS_HI)[3]
             OL.logprob_loss_bwd(H, x["W"], w["targets"].numpy(), rows, lse, g)
         done += batch
     dt = time.perf_counter() - t0

@@ -429,7 +429,7 @@ def mw_logprob_loss_fwd_kl(H, W, targets, rows, lp_old, adv, eps_lo, eps_hi, lp_
                                          _ptr(lse), _ptr(loss), _ptr(ws), _stream(stream)), "mw_logprob_loss_fwd_kl")
 
 
-def logprob_loss_fwd(H, W, targets, rows, lp_old, adv, eps_lo=0.2, eps_hi=0.2, stream=None, lp_ref=None, beta=0.0):
+def logprob_loss_fwd(H, W, targets, rows, lp_old, adv, eps_lo=0.2, eps_hi=0.28, stream=None, lp_ref=None, beta=0.0):
     """Allocate outputs + workspace; returns dict(lp, ratio, lse, loss, ws).
     With ``lp_ref`` (float32 [M]) and ``beta`` > 0 the loss includes the KL
     term of ``mw_logprob_loss_fwd_kl``."""
