@@ -22,8 +22,11 @@ and slowly, in float64:
 * ``logprob`` -- LM-head log-softmax, target gather, importance ratio and the
   clipped PPO/GRPO surrogate with its gradient (App. B.4 "Pitfall A, RL view";
   App. F.1 clip range), forward and backward.
+* ``sdcc`` -- SDCC (§5): the final compressed walk, diverging rows, the
+  teacher-prefix reconstruction, the forward KL(teacher || student) over the
+  vocabulary with the student's gradients, and the lambda ramp (App. F.1).
 
 Every function names the passage it follows in its docstring.
 """
 
-from . import visibility, attention, logprob  # noqa: F401
+from . import visibility, attention, logprob, sdcc  # noqa: F401

@@ -1,0 +1,169 @@
+"""Pins of the SDCC oracle (§5; App. B Def. "trajectory tree"; App. F.1).
+
+Diverging rows and final-walk prefixes against the paper's running example
+(App. B.4 Table "running-prefixes"), two independent formulations of
+divergence, the teacher-prefix reconstruction against the live views, the
+forward KL against a closed form and autograd, and the schedule of lambda.
+"""
+
+import json
+import os
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import sdcc as S
+from oracle import visibility as V
+
+HERE = os.path.dirname(__file__)
+
+
+def _golden():
+    with open(os.path.join(HERE, "golden", "running_example.json")) as f:
+        g = json.load(f)
+    edits = [(J, [tuple(s) for s in spans]) for J, spans in g["edits"]]
+    return g, g["tokens"], edits
+
+
+def _random_edits(rng, T, overlap=False):
+    n_j = int(rng.integers(1, 5))
+    Js = np.sort(rng.choice(np.arange(2, T - 1), size=n_j, replace=False))
+    edits = []
+    for J in Js:
+        spans = []
+        a = int(rng.integers(0, J))
+        while a < J and len(spans) < 3:
+            b = int(min(J, a + rng.integers(1, 12)))
+            spans.append((a, b))
+            a = b + int(rng.integers(1, 15))
+        if overlap and edits:
+            spans.append(edits[-1][1][0])   # evict an earlier edit's span again
+        edits.append((int(J), spans))
+    return edits
+
+
+def test_running_example_final_walk_prefixes():
+    g, tok, edits = _golden()
+    T = len(tok)
+    for leaf, names in g["final_walk_prefix"].items():
+        row = tok.index(leaf) - 1
+        assert S.walk_prefix(T, edits, row) == [0] + [tok.index(n) for n in names], leaf
+
+
+def test_running_example_diverging_rows():
+    """The table's divergence column: y6, y7 by y5; y9, y10 by y8; y12 by y11;
+    y_ans re-converges after the last junction."""
+    g, tok, edits = _golden()
+    T = len(tok)
+    div = S.diverging_rows(T, edits)
+    for leaf, by in g["diverges_by"].items():
+        row = tok.index(leaf) - 1
+        assert div[row] == bool(by), leaf
+        extra = set(S.live_prefix(T, edits, row)) - set(S.walk_prefix(T, edits, row))
+        assert extra == {tok.index(n) for n in by}, leaf
+    # rows whose prefixes precede every evicted span, and rows at or after the
+    # last junction, never diverge (App. B)
+    first_evicted = min(a for _, spans in edits for a, _ in spans)
+    assert not div[:first_evicted].any()
+    assert not div[edits[-1][0]:].any()
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_diverging_rows_two_formulations(seed):
+    rng = np.random.default_rng(400 + seed)
+    T = int(rng.integers(30, 150))
+    edits = _random_edits(rng, T, overlap=seed % 2 == 1)
+    np.testing.assert_array_equal(S.diverging_rows(T, edits), S.diverging_rows_from_lifetimes(T, edits))
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_teacher_reconstruction_equals_live_prefix(seed):
+    """Eq. "teacher-reconstruction" rebuilds exactly the prefix the token was
+    decoded from (overlapping spans included for odd seeds)."""
+    rng = np.random.default_rng(500 + seed)
+    T = int(rng.integers(30, 150))
+    edits = _random_edits(rng, T, overlap=seed % 2 == 1)
+    for r in range(T):
+        assert S.teacher_prefix(T, edits, r) == S.live_prefix(T, edits, r), r
+
+
+def test_running_example_teacher_prefix_single_span():
+    """The common case of Eq. "teacher-reconstruction" for y6: trunk
+    [s, y1..y4] + re-inserted span [y5] + empty suffix."""
+    _, tok, edits = _golden()
+    row = tok.index("y6") - 1
+    assert S.teacher_prefix(len(tok), edits, row) == [tok.index(n) for n in ("s", "y1", "y2", "y3", "y4", "y5")]
+
+
+def test_forward_kl_two_classes_closed_form():
+    """V = 2 with logits (0, x): the distributions are Bernoulli(sigmoid(x)),
+    whose KL is p log(p/q) + (1-p) log((1-p)/(1-q))."""
+    W = np.array([[0.0], [1.0]])
+    xt = np.array([[0.7], [-2.0], [3.0]])
+    xs = np.array([[-0.4], [-2.0], [0.5]])
+    kl, _, _ = S.forward_kl(xt, xs, W)
+    p = 1.0 / (1.0 + np.exp(-xt[:, 0]))
+    q = 1.0 / (1.0 + np.exp(-xs[:, 0]))
+    want = p * np.log(p / q) + (1 - p) * np.log((1 - p) / (1 - q))
+    np.testing.assert_allclose(kl, want, rtol=1e-12, atol=1e-15)
+
+
+def test_forward_kl_nonnegative_and_zero_on_equal_rows():
+    rng = np.random.default_rng(6)
+    W = rng.standard_normal((50, 8))
+    H = rng.standard_normal((5, 8))
+    kl, dh, dW = S.forward_kl(H, H, W)
+    np.testing.assert_allclose(kl, 0.0, atol=1e-12)
+    np.testing.assert_allclose(dh, 0.0, atol=1e-12)
+    np.testing.assert_allclose(dW, 0.0, atol=1e-12)
+    kl2, _, _ = S.forward_kl(H, rng.standard_normal((5, 8)), W)
+    assert (kl2 > 0).all()
+    # forward, not reverse: swapping teacher and student changes the value
+    kl3, _, _ = S.forward_kl(rng.standard_normal((5, 8)), H, W)
+    kl4, _, _ = S.forward_kl(H, rng.standard_normal((5, 8)), W)
+    assert not np.allclose(kl3, kl4)
+
+
+def test_forward_kl_gradients_equal_autograd_with_stopped_teacher():
+    rng = np.random.default_rng(7)
+    M, d, Vv = 6, 5, 40
+    HT = rng.standard_normal((M, d))
+    HS = rng.standard_normal((M, d))
+    W = rng.standard_normal((Vv, d)) * 0.5
+    kl, dHS, dW = S.forward_kl(HT, HS, W)
+    hs = torch.from_numpy(HS).requires_grad_()
+    w = torch.from_numpy(W).requires_grad_()
+    lt = torch.log_softmax(torch.from_numpy(HT) @ w.detach().T, dim=1)   # teacher: stop-gradient
+    ls = torch.log_softmax(hs @ w.T, dim=1)
+    loss = (lt.exp() * (lt - ls)).sum()
+    loss.backward()
+    np.testing.assert_allclose(kl.sum(), loss.item(), rtol=1e-12)
+    np.testing.assert_allclose(dHS, hs.grad.numpy(), rtol=1e-10, atol=1e-12)
+    np.testing.assert_allclose(dW, w.grad.numpy(), rtol=1e-10, atol=1e-12)
+
+
+def test_sdcc_penalty_is_leaf_gated():
+    rng = np.random.default_rng(8)
+    T, d, Vv = 20, 4, 30
+    HT, HS, W = rng.standard_normal((T, d)), rng.standard_normal((T, d)), rng.standard_normal((Vv, d))
+    none = np.zeros(T, dtype=bool)
+    pen, dHS, dW = S.sdcc_penalty(HT, HS, W, none, 0.1)
+    assert pen == 0.0 and not dHS.any() and not dW.any()
+    some = np.zeros(T, dtype=bool)
+    some[[3, 7, 8]] = True
+    pen0, _, _ = S.sdcc_penalty(HT, HS, W, some, 0.0)
+    assert pen0 == 0.0
+    pen, dHS, dW = S.sdcc_penalty(HT, HS, W, some, 0.1)
+    kl, _, _ = S.forward_kl(HT[[3, 7, 8]], HS[[3, 7, 8]], W)
+    assert abs(pen - 0.1 * kl.sum()) < 1e-12
+    assert not dHS[~some].any() and dHS[some].any()
+
+
+def test_lambda_ramp_schedule():
+    """App. F.1: linear from 0 to 0.1 over the first 20% of steps, then flat."""
+    assert S.lambda_ramp(0, 1000) == 0.0
+    assert abs(S.lambda_ramp(100, 1000) - 0.05) < 1e-15
+    assert abs(S.lambda_ramp(200, 1000) - 0.1) < 1e-15
+    assert S.lambda_ramp(900, 1000) == 0.1
+    assert S.lambda_ramp(10, 0) == 0.1
