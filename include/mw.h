@@ -271,6 +271,16 @@ mw_status mw_masked_attn_rope_bwd(const mw_vis_layout* layout, const void* vis, 
                                   const void* O, const void* dO, const float* LSE, void* dQ, void* dK, void* dV,
                                   int Hq, int Hkv, int Dh, int dtype, float scale, void* ws, void* stream);
 
+/*
+ * Diverging rows of SDCC (§5; App. B Def. "trajectory tree": a node whose
+ * live prefix differs from its prefix on the final compressed walk):
+ *   out uint8 [total_tokens] (device, overwritten) = 1 where row i saw a key
+ *   that a later edit evicts (some j <= i with i < omega(j) < INT32_MAX),
+ *   else 0. Row i scores token i + 1, so these are the leaves where SDCC adds
+ *   its KL term. One prefix-max scan of the lifetimes per trajectory.
+ */
+mw_status mw_diverging_rows(const mw_vis_layout* layout, const void* vis, uint8_t* out, void* stream);
+
 /* Bytes of device workspace the log-prob loss forward/backward pair needs. */
 mw_status mw_logprob_ws(int N, int M, int d, int Vocab, int dtype, size_t* ws_bytes);
 

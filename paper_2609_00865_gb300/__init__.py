@@ -13,6 +13,7 @@ from ._lib import (  # noqa: F401
     Visibility,
     VisLayout,
     build_visibility,
+    diverging_rows,
     exported_names,
     flatten_record,
     kernel_launches,

@@ -61,6 +61,7 @@ _SIGS = {
                                     _P]),
     "mw_logprob_loss_bwd": (_I, [_P, _P, _P, _P, _I, _I, _I, _I, _I, _P, _P, _F, _P, _P, _P]),
     "mw_logical_positions": (_I, [_LP, _P, _P, _P]),
+    "mw_diverging_rows": (_I, [_LP, _P, _P, _P]),
     "mw_rope_table": (_I, [_I, _I, ctypes.c_double, _P, _P]),
     "mw_rope_rows": (_I, [_LP, _P, _P, _P, _I, _P, _P, _I, _I, _I, _I, _P]),
     "mw_masked_attn_rope_ws": (_I, [_LP, _I, _I, _I, _I, ctypes.POINTER(ctypes.c_size_t),
@@ -309,6 +310,16 @@ def masked_attn_bwd(vis, Q, K, V, O, dO, LSE, scale=None, ws=None, stream=None):
 
 
 # --- row-wise logical positions and rotary attention ---------------------------
+
+def diverging_rows(vis, stream=None):
+    """uint8 [total_tokens]: 1 on the rows SDCC's KL term applies to
+    (mw_diverging_rows)."""
+    import torch
+    out = torch.empty(max(int(vis.layout.total_tokens), 1), dtype=torch.uint8, device=vis.vis.device)
+    _check(_lib().mw_diverging_rows(ctypes.byref(vis.layout), _ptr(vis.vis), _ptr(out), _stream(stream)),
+           "mw_diverging_rows")
+    return out
+
 
 def mw_logical_positions(vis, pos, stream=None):
     _check(_lib().mw_logical_positions(ctypes.byref(vis.layout), _ptr(vis.vis), _ptr(pos), _stream(stream)),

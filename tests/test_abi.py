@@ -163,3 +163,10 @@ def test_rope_workspace_holds_rotated_queries_and_segment_keys():
             # tiles, and float32 per-segment dK and dV partials
             need_b = f + 8 * lay.n_tiles * 128 * Hq + 2 * 4 * krows * Hkv * Dh
         assert need_b <= b < need_b + 1536
+
+
+def test_diverging_rows_rejects_null_output():
+    L, h = _lib()
+    lay = L.mw_visibility_layout(np.array([0, 10], np.int32), np.zeros(0, np.int32), 0)
+    assert h.mw_diverging_rows(ctypes.byref(lay), ctypes.c_void_p(16), None, None) == 1
+    assert h.mw_diverging_rows(None, ctypes.c_void_p(16), ctypes.c_void_p(16), None) == 1
