@@ -116,6 +116,7 @@ typedef struct mw_vis_layout {
     int64_t ws_off_tstat;   /* int32 [n_tiles][2] per k-tile min / max lifetime */
     int64_t ws_off_cnt;     /* int32 [2][n_tiles] fwd / bwd list lengths */
     int64_t ws_bytes;
+    int64_t max_segs;       /* max over trajectories of 1 + K_b (segments per trajectory) */
 } mw_vis_layout;
 
 /*

@@ -223,13 +223,15 @@ def attn_bwd_rows(seqlens, edits_per_traj, Q, K, V, dO, scale, rows, heads, rope
     return out
 
 
-def attn_bwd_keys(seqlens, edits_per_traj, Q, K, V, dO, scale, g, keys):
+def attn_bwd_keys(seqlens, edits_per_traj, Q, K, V, dO, scale, g, keys, rope_theta=None):
     """dK, dV of KV group ``g`` for a few physical key rows only.
 
-    Same textbook formulas as ``attn_bwd``; only the columns of the selected
-    keys of each segment's ``dS`` and ``P`` are accumulated, but every row's
-    softmax is still normalised over its full live view. Used for sampled
-    checks on workloads too large for the full backward.
+    Same textbook formulas as ``attn_bwd`` (rotary positions included: a key's
+    contribution from a segment is turned back by its angle in that segment);
+    only the columns of the selected keys of each segment's ``dS`` and ``P``
+    are accumulated, but every row's softmax is still normalised over its full
+    live view. Used for sampled checks on workloads too large for the full
+    backward.
     """
     Q = np.asarray(Q, dtype=np.float64)
     K = np.asarray(K, dtype=np.float64)
@@ -249,17 +251,25 @@ def attn_bwd_keys(seqlens, edits_per_traj, Q, K, V, dO, scale, g, keys):
         kc = np.asarray([b for _, b in cols])
         k = K[idx, g]
         v = V[idx, g]
+        if rope_theta is not None:
+            k = rope(k, np.arange(idx.size), rope_theta)
         for c0 in range(0, seg_rows.size, _ROW_CHUNK):
             grows = seg_rows[c0 : c0 + _ROW_CHUNK]
+            crow = n_before + c0 + np.arange(grows.size)
             for h in range(g * grp, (g + 1) * grp):
                 q = Q[grows, h]
+                if rope_theta is not None:
+                    q = rope(q, crow, rope_theta)
                 do = dO[grows, h]
-                s = _scores(q, k, scale, n_before + c0 + np.arange(grows.size))
+                s = _scores(q, k, scale, crow)
                 m = s.max(axis=1, keepdims=True)
                 p = np.exp(s - m)
                 p /= p.sum(axis=1, keepdims=True)
                 dp = do @ v.T
                 ds = p * (dp - (p * dp).sum(axis=1, keepdims=True))
-                np.add.at(dk_out, kn, scale * (ds[:, kc].T @ q))
+                dk = scale * (ds[:, kc].T @ q)
+                if rope_theta is not None:
+                    dk = rope(dk, kc, rope_theta, inverse=True)
+                np.add.at(dk_out, kn, dk)
                 np.add.at(dv_out, kn, p[:, kc].T @ do)
     return dk_out, dv_out

@@ -35,7 +35,7 @@ class VisLayout(ctypes.Structure):
                    "off_traj_tri", "off_traj_km", "off_seg_start", "off_tile_traj", "off_cls",
                    "off_fwd_ptr", "off_fwd_idx", "off_bwd_ptr", "off_bwd_idx", "off_pairs",
                    "off_keymask", "off_status", "vis_bytes",
-                   "ws_off_spans", "ws_off_tstat", "ws_off_cnt", "ws_bytes")]
+                   "ws_off_spans", "ws_off_tstat", "ws_off_cnt", "ws_bytes", "max_segs")]
 
 
 _P = ctypes.c_void_p

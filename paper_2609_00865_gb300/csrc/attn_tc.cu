@@ -1191,8 +1191,7 @@ mw_status attn_fwd_tc(const mw_vis_layout* L, const void* vis, const void* Q, co
 // Rows of segment key rows (keys per segment) and whether TMA's int32 row
 // coordinates and the junction-item grid reach them.
 static bool segk_fits(const mw_vis_layout* L, int Hq) {
-    return L->n_keymask * 128 <= INT32_MAX && L->n_segs * (int64_t)Hq <= INT32_MAX &&
-           L->n_segs - L->n_traj + 1 <= 65535;
+    return L->n_keymask * 128 <= INT32_MAX && L->n_segs * (int64_t)Hq <= INT32_MAX && L->max_segs <= 65535;
 }
 
 mw_status attn_fwd_tc_segk(const mw_vis_layout* L, const void* vis, const void* Q, const void* Kseg, const void* V,
@@ -1369,8 +1368,8 @@ mw_status attn_bwd_tc_segk(const mw_vis_layout* L, const void* vis, const void* 
         if ((st = launch_status()) != MW_OK) return st;
         p.junction_items = 0;
     }
-    // grid.y: the most segments one trajectory can have
-    const dim3 gk((unsigned)((int64_t)L->max_tiles * L->n_traj * Hkv), (unsigned)(L->n_segs - L->n_traj + 1));
+    // grid.y: the most segments of any trajectory
+    const dim3 gk((unsigned)((int64_t)L->max_tiles * L->n_traj * Hkv), (unsigned)L->max_segs);
     count_launches(1);
     k_attn_dkdv_tc<true><<<gk, NT_BWD, SMEM_KV, s>>>(tq64, tdo64, tk, tv, p);
     return launch_status();

@@ -78,7 +78,7 @@ extern "C" mw_status mw_visibility_layout(int n_traj, const int32_t* cu, int n_j
     L->n_traj = n_traj;
     L->n_junc = n_junc;
     L->n_spans = n_spans;
-    int64_t tiles = 0, tri = 0, km = 0;
+    int64_t tiles = 0, tri = 0, km = 0, max_segs = 0;
     int max_tiles = 0;
     int k = 0;
     for (int b = 0; b < n_traj; ++b) {
@@ -90,6 +90,7 @@ extern "C" mw_status mw_visibility_layout(int n_traj, const int32_t* cu, int n_j
         tri += nt * (nt + 1) / 2;
         km += (1 + Kb) * nt;
         if (nt > max_tiles) max_tiles = (int)nt;
+        if (1 + Kb > max_segs) max_segs = 1 + Kb;
     }
     L->max_tiles = max_tiles;
     L->total_tokens = n_traj > 0 ? cu[n_traj] : 0;
@@ -122,6 +123,7 @@ extern "C" mw_status mw_visibility_layout(int n_traj, const int32_t* cu, int n_j
     L->ws_off_tstat = take(16 * tiles);
     L->ws_off_cnt = take(8 * tiles);
     L->ws_bytes = o;
+    L->max_segs = max_segs;
     return MW_OK;
 }
 

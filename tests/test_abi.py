@@ -54,6 +54,7 @@ def test_layout_is_host_only_and_consistent():
     assert lay.n_tiles == 3 + 0 + 6
     assert lay.n_tri == 6 + 0 + 21
     assert lay.n_keymask == 2 * 3 + 1 * 0 + 3 * 6
+    assert lay.max_segs == 3
     offs = sorted(getattr(lay, f) for f, _ in L.VisLayout._fields_ if f.startswith("off_"))
     assert all(o % 256 == 0 for o in offs) and offs == sorted(set(offs))
     assert lay.vis_bytes >= offs[-1]

@@ -259,3 +259,20 @@ def test_rope_row_sampled_dq_matches_full():
     rows = np.array([0, 5, 69, 70, 111, 159])
     got = A.attn_bwd_rows(seqlens, edits, Q, K, Vv, dO, 0.3, rows, [1, 3], rope_theta=300.0)
     np.testing.assert_allclose(got, dQ[rows][:, [1, 3]], rtol=1e-12, atol=1e-12)
+
+
+def test_rope_key_sampled_dk_dv_match_full():
+    """The sampled-key dK / dV (keys whose positions differ between segments)
+    equal the full backward's rows with rotary positions."""
+    rng = _rng(12)
+    T = 120
+    edits = _random_edits(rng, T)
+    Q = rng.standard_normal((T, 4, 8))
+    K = rng.standard_normal((T, 2, 8))
+    Vv = rng.standard_normal((T, 2, 8))
+    dO = rng.standard_normal((T, 4, 8))
+    _, dK, dV = A.attn_bwd([T], [edits], Q, K, Vv, dO, 0.3, rope_theta=300.0)
+    keys = np.array([0, 3, 17, 40, 77, 119])
+    dk, dv = A.attn_bwd_keys([T], [edits], Q, K, Vv, dO, 0.3, 1, keys, rope_theta=300.0)
+    np.testing.assert_allclose(dk, dK[keys, 1], rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(dv, dV[keys, 1], rtol=1e-12, atol=1e-12)
