@@ -282,6 +282,36 @@ mw_status mw_masked_attn_rope_bwd(const mw_vis_layout* layout, const void* vis, 
  */
 mw_status mw_diverging_rows(const mw_vis_layout* layout, const void* vis, uint8_t* out, void* stream);
 
+/* Workspace bytes of the forward-KL pair (two float32 values per pair). */
+mw_status mw_forward_kl_ws(int M, int d, int Vocab, int dtype, size_t* ws_bytes);
+
+/*
+ * SDCC's consistency term (§5, Eq. "soft_loss"), forward: for pair m the
+ * teacher row HT[rows_T[m]] and the student row HS[rows_S[m]],
+ *   zT = hT W^T, zS = hS W^T (never stored),
+ *   kl[m] = KL(softmax(zT) || softmax(zS)) = sum_v pT (log pT - log pS),
+ *   loss  = lam * sum_m kl[m]  (one float32, device),
+ * the forward KL with the teacher first. HT [N_T, d], HS [N_S, d], W [Vocab, d]
+ * (dtype, W in torch Linear layout), rows_T / rows_S int32 [M] (device),
+ * rows_S distinct (M <= N_S), rows_T may repeat. Both lse per pair are kept in `ws` for the backward.
+ * Float32 arithmetic on CUDA cores; d <= 256 (MW_ESHAPE above). lam >= 0 and
+ * finite (MW_EINVAL). M = 0 gives loss = 0.
+ */
+mw_status mw_forward_kl_fwd(const void* HT, const int32_t* rows_T, const void* HS, const int32_t* rows_S, int M,
+                            const void* W, int N_T, int N_S, int d, int Vocab, int dtype, float lam,
+                            float* kl, float* loss, void* ws, void* stream);
+
+/*
+ * Backward of mw_forward_kl_fwd scaled by dloss, the teacher held fixed
+ * (stop-gradient): dzS = lam * dloss * (softmax(zS) - softmax(zT)),
+ *   dHS[rows_S[m]] = dzS_m W (other rows of dHS = 0),  dW = sum_m dzS_m^T hS_m.
+ * dHS [N_S, d] in dtype and dW [Vocab, d] float32 are overwritten. Needs the
+ * forward's `ws`.
+ */
+mw_status mw_forward_kl_bwd(const void* HT, const int32_t* rows_T, const void* HS, const int32_t* rows_S, int M,
+                            const void* W, int N_T, int N_S, int d, int Vocab, int dtype, float lam, float dloss,
+                            const void* ws, void* dHS, float* dW, void* stream);
+
 /* Bytes of device workspace the log-prob loss forward/backward pair needs. */
 mw_status mw_logprob_ws(int N, int M, int d, int Vocab, int dtype, size_t* ws_bytes);
 

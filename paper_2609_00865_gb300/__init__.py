@@ -16,6 +16,8 @@ from ._lib import (  # noqa: F401
     diverging_rows,
     exported_names,
     flatten_record,
+    forward_kl_bwd,
+    forward_kl_fwd,
     kernel_launches,
     logical_positions,
     logprob_loss_bwd,

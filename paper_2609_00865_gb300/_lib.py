@@ -62,6 +62,9 @@ _SIGS = {
     "mw_logprob_loss_bwd": (_I, [_P, _P, _P, _P, _I, _I, _I, _I, _I, _P, _P, _F, _P, _P, _P]),
     "mw_logical_positions": (_I, [_LP, _P, _P, _P]),
     "mw_diverging_rows": (_I, [_LP, _P, _P, _P]),
+    "mw_forward_kl_ws": (_I, [_I, _I, _I, _I, ctypes.POINTER(ctypes.c_size_t)]),
+    "mw_forward_kl_fwd": (_I, [_P, _P, _P, _P, _I, _P, _I, _I, _I, _I, _I, _F, _P, _P, _P, _P]),
+    "mw_forward_kl_bwd": (_I, [_P, _P, _P, _P, _I, _P, _I, _I, _I, _I, _I, _F, _F, _P, _P, _P, _P]),
     "mw_rope_table": (_I, [_I, _I, ctypes.c_double, _P, _P]),
     "mw_rope_rows": (_I, [_LP, _P, _P, _P, _I, _P, _P, _I, _I, _I, _I, _P]),
     "mw_masked_attn_rope_ws": (_I, [_LP, _I, _I, _I, _I, ctypes.POINTER(ctypes.c_size_t),
@@ -319,6 +322,37 @@ def diverging_rows(vis, stream=None):
     _check(_lib().mw_diverging_rows(ctypes.byref(vis.layout), _ptr(vis.vis), _ptr(out), _stream(stream)),
            "mw_diverging_rows")
     return out
+
+
+def forward_kl_fwd(HT, rows_T, HS, rows_S, W, lam=1.0, stream=None):
+    """SDCC consistency term: kl [M], loss (lam * sum kl) and the workspace
+    the backward needs (mw_forward_kl_fwd)."""
+    import torch
+    _need(HT, "HT")
+    _need(HS, "HS", dtype=HT.dtype)
+    _need(W, "W", dtype=HT.dtype)
+    M, d, V = int(rows_T.numel()), HT.shape[1], W.shape[0]
+    n = ctypes.c_size_t()
+    _check(_lib().mw_forward_kl_ws(M, d, V, _dtype_code(HT), ctypes.byref(n)), "mw_forward_kl_ws")
+    ws = torch.empty(max(int(n.value), 1), dtype=torch.uint8, device=HT.device)
+    kl = torch.empty(max(M, 1), dtype=torch.float32, device=HT.device)
+    loss = torch.empty(1, dtype=torch.float32, device=HT.device)
+    _check(_lib().mw_forward_kl_fwd(_ptr(HT), _ptr(rows_T), _ptr(HS), _ptr(rows_S), M, _ptr(W), HT.shape[0],
+                                    HS.shape[0], d, V, _dtype_code(HT), float(lam), _ptr(kl), _ptr(loss), _ptr(ws),
+                                    _stream(stream)), "mw_forward_kl_fwd")
+    return kl[:M], loss, ws
+
+
+def forward_kl_bwd(HT, rows_T, HS, rows_S, W, ws, lam=1.0, dloss=1.0, stream=None):
+    """Student gradients of the SDCC term: dHS (like HS), dW (float32)."""
+    import torch
+    M, d, V = int(rows_T.numel()), HT.shape[1], W.shape[0]
+    dHS = torch.empty_like(HS)
+    dW = torch.empty(V, d, dtype=torch.float32, device=HT.device)
+    _check(_lib().mw_forward_kl_bwd(_ptr(HT), _ptr(rows_T), _ptr(HS), _ptr(rows_S), M, _ptr(W), HT.shape[0],
+                                    HS.shape[0], d, V, _dtype_code(HT), float(lam), float(dloss), _ptr(ws),
+                                    _ptr(dHS), _ptr(dW), _stream(stream)), "mw_forward_kl_bwd")
+    return dHS, dW
 
 
 def mw_logical_positions(vis, pos, stream=None):

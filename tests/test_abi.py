@@ -171,3 +171,19 @@ def test_diverging_rows_rejects_null_output():
     lay = L.mw_visibility_layout(np.array([0, 10], np.int32), np.zeros(0, np.int32), 0)
     assert h.mw_diverging_rows(ctypes.byref(lay), ctypes.c_void_p(16), None, None) == 1
     assert h.mw_diverging_rows(None, ctypes.c_void_p(16), ctypes.c_void_p(16), None) == 1
+
+
+def test_forward_kl_rejects_bad_args_on_host():
+    L, h = _lib()
+    P = ctypes.c_void_p(16)
+    n = ctypes.c_size_t()
+    assert h.mw_forward_kl_ws(4, 512, 100, 0, ctypes.byref(n)) == 3          # d above the CUDA-core limit
+    assert h.mw_forward_kl_ws(4, 64, 100, 9, ctypes.byref(n)) == 4           # dtype
+    assert h.mw_forward_kl_ws(4, 64, 100, 0, ctypes.byref(n)) == 0 and n.value >= 2 * 4 * 4
+    # more pairs than (distinct) student rows, no teacher rows, negative lambda, null loss
+    assert h.mw_forward_kl_fwd(P, P, P, P, 5, P, 8, 4, 64, 100, 0, 0.1, P, P, P, None) == 3
+    assert h.mw_forward_kl_fwd(P, P, P, P, 4, P, 0, 8, 64, 100, 0, 0.1, P, P, P, None) == 3
+    assert h.mw_forward_kl_fwd(P, P, P, P, 4, P, 4, 8, 64, 100, 0, -0.1, P, P, P, None) == 1
+    assert h.mw_forward_kl_fwd(P, P, P, P, 4, P, 4, 8, 64, 100, 0, 0.1, P, None, P, None) == 1
+    assert h.mw_forward_kl_bwd(P, P, P, P, 4, P, 4, 8, 64, 100, 0, 0.1, float("nan"), P, P, P, None) == 1
+    assert h.mw_forward_kl_bwd(P, P, P, P, 4, P, 4, 8, 64, 100, 0, 0.1, 1.0, P, P, None, None) == 1

@@ -8,6 +8,7 @@ import numpy as np
 import pytest
 import torch
 
+from helpers import assert_grad_bf16, assert_maxabs, assert_rel, np64
 from oracle import sdcc as OS
 
 pytestmark = pytest.mark.gpu
@@ -41,3 +42,69 @@ def test_packed_ragged_record_with_overlaps():
              [(1100, [(10, 900)]), (2000, [(1000, 1900), (5, 8)]), (2400, [(2001, 2300)])],
              [(128, [(5, 127)])]]
     _check(seqlens, edits)
+
+
+def _kl_case(M, N_T, N_S, d, V, seed, dtype):
+    rng = np.random.default_rng(seed)
+    HT = torch.from_numpy(rng.standard_normal((N_T, d))).to(dtype)
+    HS = torch.from_numpy(rng.standard_normal((N_S, d))).to(dtype)
+    W = torch.from_numpy(0.3 * rng.standard_normal((V, d))).to(dtype)
+    rows_T = torch.from_numpy(rng.integers(0, N_T, M).astype(np.int32))
+    rows_S = torch.from_numpy(rng.permutation(N_S)[:M].astype(np.int32))   # distinct
+    return HT, HS, W, rows_T, rows_S
+
+
+def _kl_run(HT, HS, W, rows_T, rows_S, lam, dloss):
+    import paper_2609_00865_gb300 as mw
+    dev = [t.cuda() for t in (HT, rows_T, HS, rows_S, W)]
+    kl, loss, ws = mw.forward_kl_fwd(*dev, lam=lam)
+    dHS, dW = mw.forward_kl_bwd(*dev, ws, lam=lam, dloss=dloss)
+    torch.cuda.synchronize()
+    return kl, loss, dHS, dW
+
+
+def _kl_ref(HT, HS, W, rows_T, rows_S, lam, dloss):
+    from oracle import sdcc as OSd
+    rt, rs = rows_T.numpy().astype(np.int64), rows_S.numpy().astype(np.int64)
+    kl, dh, dW = OSd.forward_kl(np64(HT)[rt], np64(HS)[rs], np64(W))
+    dHS = np.zeros(tuple(HS.shape))
+    dHS[rs] = lam * dloss * dh
+    return kl, lam * kl.sum(), dHS, lam * dloss * dW
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+def test_forward_kl_matches_oracle(dtype):
+    """Forward KL(teacher || student) over a 3,001-column vocabulary (a ragged
+    last tile of 256 columns), 37 pairs (ragged blocks of 8, 16 and 32),
+    teacher rows drawn with repeats, student rows distinct; both gradients
+    of the student."""
+    d = 64 if dtype == torch.float32 else 128
+    case = _kl_case(37, 50, 45, d, 3001, 7, dtype)
+    kl, loss, dHS, dW = _kl_run(*case, lam=0.1, dloss=1.3)
+    klr, lossr, dHSr, dWr = _kl_ref(*case, lam=0.1, dloss=1.3)
+    assert_rel(np64(kl), klr, 1e-4, "kl")
+    assert_rel(np64(loss), [lossr], 1e-4, "loss")
+    if dtype == torch.float32:
+        assert_rel(np64(dHS), dHSr, 1e-4, "dHS")
+    else:
+        assert_grad_bf16(np64(dHS), dHSr, "dHS")
+    assert_rel(np64(dW), dWr, 1e-4, "dW")
+    untouched = np.setdiff1d(np.arange(case[1].shape[0]), case[4].numpy())
+    assert not np64(dHS)[untouched].any()
+
+
+def test_forward_kl_of_equal_rows_is_zero():
+    HT, _, W, _, _ = _kl_case(10, 10, 10, 32, 500, 9, torch.float32)
+    rows = torch.arange(10, dtype=torch.int32)
+    kl, loss, dHS, dW = _kl_run(HT, HT, W, rows, rows, 1.0, 1.0)
+    assert_maxabs(np64(kl), np.zeros(10), 1e-5, "kl")
+    assert_maxabs(np64(dHS), np.zeros(tuple(HT.shape)), 1e-6, "dHS")
+    assert_maxabs(np64(dW), np.zeros(tuple(W.shape)), 1e-6, "dW")
+
+
+def test_forward_kl_without_pairs():
+    HT, HS, W, _, _ = _kl_case(0, 5, 6, 32, 300, 10, torch.float32)
+    empty = torch.zeros(0, dtype=torch.int32)
+    kl, loss, dHS, dW = _kl_run(HT, HS, W, empty, empty, 0.1, 1.0)
+    assert float(loss.item()) == 0.0
+    assert not dHS.any() and not dW.any()
