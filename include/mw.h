@@ -371,6 +371,15 @@ mw_status mw_logprob_loss_bwd(const void* H, const void* W, const int32_t* targe
                               void* dH, float* dW, void* stream);
 
 /*
+ * Train-inference logits drift (Eq. "logdiff", §3): out = (1/M) sum_m
+ * |lp_train[m] - lp_rollout[m]| over the loss-carrying tokens, one float32
+ * (device). lp_train, lp_rollout float32 [M] (device), e.g. this library's
+ * log-probs and the rollout's (the lp_old of the loss). M = 0 gives 0.
+ * Fixed reduction order (deterministic).
+ */
+mw_status mw_logdiff(const float* lp_train, const float* lp_rollout, int M, float* out, void* stream);
+
+/*
  * Copy the device status words of a visibility buffer to the host after
  * synchronising `stream`; returns MW_OK, MW_ETIMEOUT or MW_EDEVICE.
  */

@@ -130,3 +130,15 @@ def logprob_loss_bwd_vocab(H, W, targets, rows, lse, g, vocab):
     onehot = (tgt[:, None] == vocab[None, :]).astype(np.float64)
     dz = np.asarray(g, dtype=np.float64)[:, None] * (onehot - p)
     return dz.T @ H[rows]
+
+
+def logdiff(lp_train, lp_rollout):
+    """Eq. "logdiff" (§3): the train-inference logits drift, the mean over
+    the loss-carrying tokens of |log p(y_t | c_train) - log p(y_t | c_rollout)|
+    under one set of weights. Returns 0 for no tokens."""
+    a = np.asarray(lp_train, dtype=np.float64)
+    b = np.asarray(lp_rollout, dtype=np.float64)
+    if a.size == 0:
+        return 0.0
+    return float(np.abs(a - b).mean())
+

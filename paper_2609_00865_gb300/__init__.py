@@ -19,6 +19,7 @@ from ._lib import (  # noqa: F401
     forward_kl_bwd,
     forward_kl_fwd,
     kernel_launches,
+    logdiff,
     logical_positions,
     logprob_loss_bwd,
     logprob_loss_fwd,

@@ -62,6 +62,7 @@ _SIGS = {
     "mw_logprob_loss_bwd": (_I, [_P, _P, _P, _P, _I, _I, _I, _I, _I, _P, _P, _F, _P, _P, _P]),
     "mw_logical_positions": (_I, [_LP, _P, _P, _P]),
     "mw_diverging_rows": (_I, [_LP, _P, _P, _P]),
+    "mw_logdiff": (_I, [_P, _P, _I, _P, _P]),
     "mw_forward_kl_ws": (_I, [_I, _I, _I, _I, ctypes.POINTER(ctypes.c_size_t)]),
     "mw_forward_kl_fwd": (_I, [_P, _P, _P, _P, _I, _P, _I, _I, _I, _I, _I, _F, _P, _P, _P, _P]),
     "mw_forward_kl_bwd": (_I, [_P, _P, _P, _P, _I, _P, _I, _I, _I, _I, _I, _F, _F, _P, _P, _P, _P]),
@@ -321,6 +322,18 @@ def diverging_rows(vis, stream=None):
     out = torch.empty(max(int(vis.layout.total_tokens), 1), dtype=torch.uint8, device=vis.vis.device)
     _check(_lib().mw_diverging_rows(ctypes.byref(vis.layout), _ptr(vis.vis), _ptr(out), _stream(stream)),
            "mw_diverging_rows")
+    return out
+
+
+def logdiff(lp_train, lp_rollout, stream=None):
+    """Eq. "logdiff": mean |lp_train - lp_rollout| as a one-element float32
+    device tensor (mw_logdiff)."""
+    import torch
+    _need(lp_train, "lp_train", dtype=torch.float32)
+    _need(lp_rollout, "lp_rollout", dtype=torch.float32)
+    out = torch.empty(1, dtype=torch.float32, device=lp_train.device)
+    _check(_lib().mw_logdiff(_ptr(lp_train), _ptr(lp_rollout), int(lp_train.numel()), _ptr(out), _stream(stream)),
+           "mw_logdiff")
     return out
 
 

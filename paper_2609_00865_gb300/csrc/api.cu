@@ -41,6 +41,7 @@ mw_status attn_bwd_tc_segk(const mw_vis_layout*, const void*, const void*, const
                            const void*, const float*, void*, float*, float*, int, int, float, float*, cudaStream_t);
 __global__ void k_loss_epilogue(int, const float*, const float*, const float*, float, float, const float*, float, float*,
                                 float*, float*);
+__global__ void k_logdiff(int, const float*, const float*, float*);
 
 struct LmPlan {
     int M_pad, R, NV, C, NVC, grid;
@@ -203,6 +204,14 @@ extern "C" mw_status mw_logprob_loss_bwd(const void* H, const void* W, const int
     }
     return lm_bwd_simt(H, W, targets, rows, M, N, d, V, dtype, lse, at<float>(ws, w.g), dloss, dH, dW,
                        (cudaStream_t)stream);
+}
+
+extern "C" mw_status mw_logdiff(const float* lp_train, const float* lp_rollout, int M, float* out, void* stream) {
+    if (M < 0) return MW_ESHAPE;
+    if (!out || (M > 0 && (!lp_train || !lp_rollout))) return MW_EINVAL;
+    count_launches(1);
+    k_logdiff<<<1, 1024, 0, (cudaStream_t)stream>>>(M, lp_train, lp_rollout, out);
+    return launch_status();
 }
 
 extern "C" mw_status mw_logprob_check_status(int N, int M, int d, int V, int dtype, const void* ws, void* stream) {

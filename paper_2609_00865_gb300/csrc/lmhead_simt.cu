@@ -52,6 +52,22 @@ __global__ void k_loss_epilogue(int M, const float* __restrict__ lp, const float
     }
 }
 
+// Eq. "logdiff": mean_m |lp_train[m] - lp_rollout[m]|, one block of 1024
+// threads in a fixed order (0 for M = 0).
+__global__ void k_logdiff(int M, const float* __restrict__ a, const float* __restrict__ b, float* __restrict__ out) {
+    __shared__ float red[32];
+    float part = 0.f;
+    for (int m = threadIdx.x; m < M; m += blockDim.x) part += fabsf(a[m] - b[m]);
+    part = warp_sum(part);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = part;
+    __syncthreads();
+    if (threadIdx.x < 32) {
+        float x = threadIdx.x < (blockDim.x >> 5) ? red[threadIdx.x] : 0.f;
+        x = warp_sum(x);
+        if (threadIdx.x == 0) *out = M > 0 ? x / (float)M : 0.f;
+    }
+}
+
 namespace {
 
 constexpr int FR = 16;  // loss rows per block (forward / dH)

@@ -108,3 +108,18 @@ def test_forward_kl_without_pairs():
     kl, loss, dHS, dW = _kl_run(HT, HS, W, empty, empty, 0.1, 1.0)
     assert float(loss.item()) == 0.0
     assert not dHS.any() and not dW.any()
+
+
+@pytest.mark.parametrize("M", [0, 1, 1000, 70001])
+def test_logdiff_matches_oracle(M):
+    """Eq. "logdiff" over M tokens (one block of 1,024 threads: 69 strides
+    each at M = 70,001)."""
+    import paper_2609_00865_gb300 as mw
+    from oracle import logprob as OL
+    rng = np.random.default_rng(M)
+    a = torch.from_numpy(rng.standard_normal(M).astype(np.float32))
+    b = torch.from_numpy((rng.standard_normal(M) * 0.1).astype(np.float32)) + a
+    got = mw.logdiff(a.cuda(), b.cuda())
+    torch.cuda.synchronize()
+    want = OL.logdiff(np64(a), np64(b))
+    assert abs(float(got.item()) - want) <= 1e-5 * want   # exact 0 without tokens

@@ -167,3 +167,37 @@ def test_lambda_ramp_schedule():
     assert abs(S.lambda_ramp(200, 1000) - 0.1) < 1e-15
     assert S.lambda_ramp(900, 1000) == 0.1
     assert S.lambda_ramp(10, 0) == 0.1
+
+
+@pytest.mark.parametrize("seed", range(3))
+def test_walk_scoring_drifts_exactly_on_diverging_rows(seed):
+    """Eq. "logdiff" between scoring on the final compressed walk
+    (Naive-Compressed) and scoring under the live views (the exact methods),
+    one attention layer + LM head: a row's log-prob moves iff the row
+    diverges, since a non-diverging row attends to the same set of keys in
+    both (no positional encoding)."""
+    from oracle import attention as A
+    from oracle import logprob as LP
+    rng = np.random.default_rng(600 + seed)
+    T, Dh, Vv = 90, 8, 50
+    edits = _random_edits(rng, T)
+    Q = rng.standard_normal((T, 1, Dh))
+    K = rng.standard_normal((T, 1, Dh))
+    Vx = rng.standard_normal((T, 1, Dh))
+    W = rng.standard_normal((Vv, Dh))
+    targets = rng.integers(0, Vv, T)
+    live, _ = A.attn_fwd([T], [edits], Q, K, Vx, 0.4)
+    walk = S.final_walk(T, edits)
+    wo, _ = A.attn_fwd([len(walk)], [[]], Q[walk], K[walk], Vx[walk], 0.4)
+    where = {j: n for n, j in enumerate(walk)}
+    # the student predicts y_(r+1) from the walk row of the last survivor <= r
+    rows = [r for r in range(T) if S.walk_prefix(T, edits, r)]
+    stud = np.stack([wo[where[S.walk_prefix(T, edits, r)[-1]], 0] for r in rows])
+    lp_live, _ = LP.logprob(live[:, 0], W, targets, np.array(rows))
+    lp_walk, _ = LP.logprob(stud, W, np.asarray(targets)[rows], np.arange(len(rows)))
+    div = S.diverging_rows(T, edits)[rows]
+    drift = np.abs(lp_live - lp_walk)
+    assert (drift[~div] < 1e-12).all()
+    assert (drift[div] > 1e-9).all()
+    assert abs(LP.logdiff(lp_live, lp_walk) - drift.mean()) < 1e-15
+    assert LP.logdiff([], []) == 0.0
