@@ -211,6 +211,15 @@ def make_workload(cfg, K=None, f=None, seed_offset=0, n_traj=None, pin=True, rop
     return w
 
 
+def e2e_inputs(w, device_keys):
+    """The host tensors the end-to-end leg uploads every step: the workload's
+    per-step inputs that the step holds on the device, not the resident model
+    state (RESIDENT)."""
+    import torch
+    return {k: v for k, v in w.items()
+            if isinstance(v, torch.Tensor) and k in device_keys and k not in RESIDENT}
+
+
 def describe(w):
     import synth
     c = synth.CONFIGS[w["cfg"]]
@@ -510,7 +519,7 @@ def run_gpu(args, rank, world, local_rank):
     # e2e: pinned host inputs -> device, step, loss/metric read back. The
     # per-step inputs are uploaded; the LM-head weight W is model state, resident
     # on the device across steps as in a training loop.
-    host = {k: v for k, v in w.items() if isinstance(v, torch.Tensor) and k in step.d and k not in RESIDENT}
+    host = e2e_inputs(w, step.d)
     h2d = sum(v.numel() * v.element_size() for v in host.values())
     out = step.loss if hasattr(step, "loss") else step.LSE[0, :1]
     d2h = out.numel() * out.element_size()
