@@ -126,3 +126,57 @@ def sdcc_penalty(HT, HS, W, diverging, lam):
     kl, dh, dW = forward_kl(HT[idx], HS[idx], W)
     dHS[idx] = lam * dh
     return lam * float(kl.sum()), dHS, lam * dW
+
+
+def student_rows(T, edits):
+    """For every row r with a non-empty final-walk prefix, the index on the
+    final walk of the row that makes the student's prediction of y_(r+1): the
+    last surviving position <= r (§5: the student is f(H_comp) at the leaf's
+    place in the compressed walk). Returns {r: walk index}."""
+    walk = final_walk(T, edits)
+    where = {j: n for n, j in enumerate(walk)}
+    out = {}
+    for r in range(T):
+        pre = walk_prefix(T, edits, r)
+        if pre:
+            out[r] = where[pre[-1]]
+    return out
+
+
+def sdcc_objective(T, edits, Q, K, V, W, targets, loss_rows, lp_old, adv, lam, scale, eps_lo=0.2, eps_hi=0.28):
+    """Eq. "soft_loss" for one trajectory and one attention layer feeding the
+    LM head (hidden row = attention output, heads concatenated):
+
+      student  attention over the final compressed walk (causal, no edits),
+               task loss = the clipped surrogate on the loss rows that survive
+               on the walk, scored at their walk position (Naive-Compressed);
+      teacher  attention under each row's live view (the exact 4D mask),
+               gradients stopped;
+      penalty  lam * sum over diverging rows of KL(teacher || student).
+
+    Returns (objective, task, penalty). Plain composition of the oracle's own
+    attention, log-prob and KL functions, in their definitions' order.
+    """
+    from .attention import attn_fwd
+    from .logprob import logprob, policy_loss
+    Q = np.asarray(Q, dtype=np.float64)
+    K = np.asarray(K, dtype=np.float64)
+    V = np.asarray(V, dtype=np.float64)
+    walk = final_walk(T, edits)
+    where = {j: n for n, j in enumerate(walk)}
+    Os, _ = attn_fwd([len(walk)], [[]], Q[walk], K[walk], V[walk], scale)
+    Hs = Os.reshape(len(walk), -1)
+    Ot, _ = attn_fwd([T], [edits], Q, K, V, scale)
+    Ht = Ot.reshape(T, -1)
+    rows = [r for r in loss_rows if r in where]
+    lp, _ = logprob(Hs, W, np.asarray(targets)[walk], np.array([where[r] for r in rows], dtype=np.int64))
+    sel = [list(loss_rows).index(r) for r in rows]
+    _, _, task, _ = policy_loss(lp, np.asarray(lp_old)[sel], np.asarray(adv)[sel], eps_lo, eps_hi)
+    div = diverging_rows(T, edits)
+    srow = student_rows(T, edits)
+    pairs = [(r, srow[r]) for r in range(T) if div[r] and r in srow]
+    penalty = 0.0
+    if pairs and lam != 0.0:
+        kl, _, _ = forward_kl(Ht[[a for a, _ in pairs]], Hs[[b for _, b in pairs]], W)
+        penalty = lam * float(kl.sum())
+    return task + penalty, task, penalty

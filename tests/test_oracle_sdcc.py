@@ -201,3 +201,65 @@ def test_walk_scoring_drifts_exactly_on_diverging_rows(seed):
     assert (drift[div] > 1e-9).all()
     assert abs(LP.logdiff(lp_live, lp_walk) - drift.mean()) < 1e-15
     assert LP.logdiff([], []) == 0.0
+
+
+def _torch_objective(T, edits, Q, K, Vx, W, targets, loss_rows, lp_old, adv, lam, scale):
+    """The same objective through torch: the teacher from dense attention
+    under the lifetime mask, the student from causal SDPA over the surviving
+    positions, torch log-softmax and KL."""
+    q, k, v, w = (torch.from_numpy(np.asarray(x, dtype=np.float64)) for x in (Q, K, Vx, W))
+    walk = S.final_walk(T, edits)
+    mask = torch.from_numpy(V.lifetime_mask(T, edits))
+    st = torch.nn.functional.scaled_dot_product_attention(
+        q[walk].transpose(0, 1), k[walk].transpose(0, 1), v[walk].transpose(0, 1), is_causal=True,
+        scale=scale).transpose(0, 1).reshape(len(walk), -1)
+    te = torch.nn.functional.scaled_dot_product_attention(
+        q.transpose(0, 1), k.transpose(0, 1), v.transpose(0, 1), attn_mask=mask, scale=scale
+    ).transpose(0, 1).reshape(T, -1)
+    where = {j: n for n, j in enumerate(walk)}
+    rows = [r for r in loss_rows if r in where]
+    sel = [list(loss_rows).index(r) for r in rows]
+    ls = torch.log_softmax(st @ w.T, dim=1)
+    lp = ls[[where[r] for r in rows], torch.from_numpy(np.asarray(targets)[rows])]
+    ratio = torch.exp(lp - torch.from_numpy(np.asarray(lp_old)[sel]))
+    a = torch.from_numpy(np.asarray(adv)[sel])
+    task = -torch.minimum(ratio * a, ratio.clamp(0.8, 1.28) * a).mean()
+    pen = torch.zeros((), dtype=torch.float64)
+    div = S.diverging_rows(T, edits)
+    srow = S.student_rows(T, edits)
+    for r in range(T):
+        if div[r] and r in srow:
+            lt = torch.log_softmax(te[r] @ w.T, dim=0)
+            pen = pen + (lt.exp() * (lt - ls[srow[r]])).sum()
+    return float(task + lam * pen), float(task), float(lam * pen)
+
+
+@pytest.mark.parametrize("seed", range(3))
+def test_sdcc_objective_matches_an_independent_composition(seed):
+    rng = np.random.default_rng(700 + seed)
+    T, H, Dh, Vv = 70, 2, 4, 40
+    edits = _random_edits(rng, T)
+    Q, K, Vx = (rng.standard_normal((T, H, Dh)) for _ in range(3))
+    W = rng.standard_normal((Vv, H * Dh)) * 0.5
+    targets = rng.integers(0, Vv, T)
+    loss_rows = np.sort(rng.choice(T, 40, replace=False))
+    lp_old = rng.standard_normal(40) * 0.1 - 3.5
+    adv = rng.standard_normal(40)
+    got = S.sdcc_objective(T, edits, Q, K, Vx, W, targets, loss_rows, lp_old, adv, 0.1, 0.5)
+    want = _torch_objective(T, edits, Q, K, Vx, W, targets, loss_rows, lp_old, adv, 0.1, 0.5)
+    np.testing.assert_allclose(got, want, rtol=1e-10, atol=1e-12)
+    assert got[2] > 0
+    # lambda = 0 is Naive-Compressed exactly
+    z = S.sdcc_objective(T, edits, Q, K, Vx, W, targets, loss_rows, lp_old, adv, 0.0, 0.5)
+    assert z[0] == z[1] == got[1] and z[2] == 0.0
+
+
+def test_sdcc_objective_without_edits_is_the_task_loss():
+    rng = np.random.default_rng(710)
+    T = 30
+    Q, K, Vx = (rng.standard_normal((T, 1, 4)) for _ in range(3))
+    W = rng.standard_normal((20, 4))
+    rows = np.arange(T)
+    obj, task, pen = S.sdcc_objective(T, [], Q, K, Vx, W, rng.integers(0, 20, T), rows,
+                                      np.full(T, -3.0), rng.standard_normal(T), 0.1, 0.5)
+    assert pen == 0.0 and obj == task
