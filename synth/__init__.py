@@ -123,7 +123,7 @@ CONFIGS = {
                  "512-token summaries",
             n_traj=8, T=16384, K=4, evict=0.6, summary=512, prompt=256, Lp=200, Lo=400,
             Hq=32, Hkv=8, Dh=128, dtype="bf16"),
-    3: dict(name="bf16 fused log-prob loss: N=32768, d=1536, V=151936, 70% loss rows, eps 0.2",
+    3: dict(name="bf16 fused log-prob loss: N=32768, d=1536, V=151936, 70% loss rows, clip 0.2/0.28",
             N=32768, d=1536, V=151936, loss_frac=0.7, dtype="bf16"),
     4: dict(name="7B-shaped layer step: 2x65536 tokens, 28/4 heads Dh 128, 8 junctions at 70%, "
                  "1024-token summaries, LM head d=3584 V=152064",
