@@ -282,6 +282,20 @@ mw_status mw_masked_attn_rope_bwd(const mw_vis_layout* layout, const void* vis, 
  */
 mw_status mw_diverging_rows(const mw_vis_layout* layout, const void* vis, uint8_t* out, void* stream);
 
+/*
+ * The final compressed walk of every trajectory (§5: the replay sequence left
+ * after every edit, the student's input): its never-evicted positions in order.
+ *   walk_index  int32 [total_tokens]: position of token j on its trajectory's
+ *               walk (0-based), -1 if some edit evicts j;
+ *   student_row int32 [total_tokens]: for row r, the walk index of the last
+ *               surviving position <= r (the walk row whose prediction is the
+ *               student's for y_(r+1)), -1 if none;
+ *   walk_len    int32 [n_traj]: the walk's length per trajectory.
+ * All device, overwritten. One prefix count of survivors per trajectory.
+ */
+mw_status mw_final_walk(const mw_vis_layout* layout, const void* vis, int32_t* walk_index, int32_t* student_row,
+                        int32_t* walk_len, void* stream);
+
 /* Workspace bytes of the forward-KL pair (two float32 values per pair). */
 mw_status mw_forward_kl_ws(int M, int d, int Vocab, int dtype, size_t* ws_bytes);
 

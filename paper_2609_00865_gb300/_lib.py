@@ -62,6 +62,7 @@ _SIGS = {
     "mw_logprob_loss_bwd": (_I, [_P, _P, _P, _P, _I, _I, _I, _I, _I, _P, _P, _F, _P, _P, _P]),
     "mw_logical_positions": (_I, [_LP, _P, _P, _P]),
     "mw_diverging_rows": (_I, [_LP, _P, _P, _P]),
+    "mw_final_walk": (_I, [_LP, _P, _P, _P, _P, _P]),
     "mw_logdiff": (_I, [_P, _P, _I, _P, _P]),
     "mw_forward_kl_ws": (_I, [_I, _I, _I, _I, ctypes.POINTER(ctypes.c_size_t)]),
     "mw_forward_kl_fwd": (_I, [_P, _P, _P, _P, _I, _P, _I, _I, _I, _I, _I, _F, _P, _P, _P, _P]),
@@ -323,6 +324,20 @@ def diverging_rows(vis, stream=None):
     _check(_lib().mw_diverging_rows(ctypes.byref(vis.layout), _ptr(vis.vis), _ptr(out), _stream(stream)),
            "mw_diverging_rows")
     return out
+
+
+def final_walk(vis, stream=None):
+    """(walk_index [T], student_row [T], walk_len [n_traj]) int32 device
+    tensors of the final compressed walk (mw_final_walk)."""
+    import torch
+    L = vis.layout
+    dev = vis.vis.device
+    wi = torch.empty(max(int(L.total_tokens), 1), dtype=torch.int32, device=dev)
+    sr = torch.empty_like(wi)
+    wl = torch.empty(max(int(L.n_traj), 1), dtype=torch.int32, device=dev)
+    _check(_lib().mw_final_walk(ctypes.byref(L), _ptr(vis.vis), _ptr(wi), _ptr(sr), _ptr(wl), _stream(stream)),
+           "mw_final_walk")
+    return wi, sr, wl
 
 
 def logdiff(lp_train, lp_rollout, stream=None):

@@ -60,6 +60,46 @@ __global__ void __launch_bounds__(DIV_NT) k_diverging_rows(VisView v, uint8_t* _
     }
 }
 
+// Final compressed walk of every trajectory: the never-evicted positions in
+// order (omega = never). One inclusive prefix count of survivors per
+// trajectory gives each token's walk index (or -1), each row's student row
+// (the walk index of the last survivor <= r, i.e. count - 1, -1 when none)
+// and the walk length.
+__global__ void __launch_bounds__(DIV_NT) k_final_walk(VisView v, int32_t* __restrict__ walk_index,
+                                                       int32_t* __restrict__ student_row,
+                                                       int32_t* __restrict__ walk_len) {
+    __shared__ int wsum[DIV_NT / 32];
+    __shared__ int carry_s;
+    const int b = blockIdx.x;
+    const int64_t tok0 = v.traj_tok[b];
+    const int T = v.traj_tok[b + 1] - (int)tok0;
+    const int t = threadIdx.x, lane = t & 31, w = t >> 5;
+    if (t == 0) carry_s = 0;
+    __syncthreads();
+    for (int c0 = 0; c0 < T; c0 += DIV_NT) {
+        const int r = c0 + t;
+        const int alive = (r < T && v.omega[tok0 + r] == INT32_MAX) ? 1 : 0;
+        int x = alive;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, x, o);
+            if (lane >= o) x += y;
+        }
+        if (lane == 31) wsum[w] = x;
+        __syncthreads();
+        int incl = carry_s + x;
+        for (int q = 0; q < w; ++q) incl += wsum[q];
+        if (r < T) {
+            walk_index[tok0 + r] = alive ? incl - 1 : -1;
+            student_row[tok0 + r] = incl - 1;
+        }
+        __syncthreads();
+        if (t == DIV_NT - 1) carry_s = incl;
+        __syncthreads();
+    }
+    if (t == 0) walk_len[b] = carry_s;
+}
+
 // ---------------------------------------------------------------- forward KL
 
 constexpr int KR = 8;    // pairs per forward block
@@ -362,6 +402,17 @@ mw_status kl_bwd_t(const void* HT, const int32_t* rowsT, const void* HS, const i
 }  // namespace mw
 
 using namespace mw;
+
+extern "C" mw_status mw_final_walk(const mw_vis_layout* L, const void* vis, int32_t* walk_index,
+                                   int32_t* student_row, int32_t* walk_len, void* stream) {
+    if (!L) return MW_EINVAL;
+    if (L->n_traj == 0) return MW_OK;
+    if (!vis || !walk_len || (L->total_tokens > 0 && (!walk_index || !student_row))) return MW_EINVAL;
+    count_launches(1);
+    k_final_walk<<<(unsigned)L->n_traj, DIV_NT, 0, (cudaStream_t)stream>>>(make_view(L, vis), walk_index,
+                                                                          student_row, walk_len);
+    return launch_status();
+}
 
 static mw_status kl_args(int M, int N_T, int N_S, int d, int Vocab, int dtype) {
     if (M < 0 || N_T < 0 || N_S < 0 || d <= 0 || Vocab <= 0) return MW_ESHAPE;

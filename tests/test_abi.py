@@ -195,3 +195,12 @@ def test_logdiff_rejects_bad_args_on_host():
     assert h.mw_logdiff(P, P, -1, P, None) == 3
     assert h.mw_logdiff(P, P, 4, None, None) == 1
     assert h.mw_logdiff(None, P, 4, P, None) == 1
+
+
+def test_final_walk_rejects_null_outputs():
+    L, h = _lib()
+    lay = L.mw_visibility_layout(np.array([0, 10], np.int32), np.zeros(0, np.int32), 0)
+    P = ctypes.c_void_p(16)
+    assert h.mw_final_walk(ctypes.byref(lay), P, P, P, None, None) == 1
+    assert h.mw_final_walk(ctypes.byref(lay), P, None, P, P, None) == 1
+    assert h.mw_final_walk(None, P, P, P, P, None) == 1

@@ -44,6 +44,39 @@ def test_packed_ragged_record_with_overlaps():
     _check(seqlens, edits)
 
 
+def _check_walk(seqlens, edits):
+    import paper_2609_00865_gb300 as mw
+    vis = mw.build_visibility(seqlens, edits)
+    wi, sr, wl = mw.final_walk(vis)
+    torch.cuda.synchronize()
+    want_wi, want_sr, want_wl = [], [], []
+    for T, e in zip(seqlens, edits):
+        walk = OS.final_walk(T, e) if T else []
+        w = np.full(T, -1)
+        w[walk] = np.arange(len(walk))
+        srow = OS.student_rows(T, e) if T else {}
+        want_wi.append(w)
+        want_sr.append([srow.get(r, -1) for r in range(T)])
+        want_wl.append(len(walk))
+    n = sum(seqlens)
+    np.testing.assert_array_equal(wi.cpu().numpy()[:n], np.concatenate(want_wi))
+    np.testing.assert_array_equal(sr.cpu().numpy()[:n], np.concatenate([np.asarray(x, dtype=np.int64)
+                                                                         for x in want_sr]))
+    np.testing.assert_array_equal(wl.cpu().numpy()[: len(seqlens)], want_wl)
+
+
+def test_final_walk_running_example_and_ragged_record():
+    """Walk indices, student rows and walk lengths, bit for bit (§5)."""
+    with open(os.path.join(HERE, "golden", "running_example.json")) as f:
+        g = json.load(f)
+    edits = [(J, [tuple(s) for s in spans]) for J, spans in g["edits"]]
+    _check_walk([len(g["tokens"])], [edits])
+    _check_walk([1, 0, 300, 2500, 129],
+                [[], [], [(150, [(20, 140)]), (280, [(150, 260), (20, 40)])],
+                 [(1100, [(10, 900)]), (2000, [(1000, 1900), (5, 8)]), (2400, [(2001, 2300)])],
+                 [(128, [(5, 127)])]])
+
+
 def _kl_case(M, N_T, N_S, d, V, seed, dtype):
     rng = np.random.default_rng(seed)
     HT = torch.from_numpy(rng.standard_normal((N_T, d))).to(dtype)
