@@ -22,6 +22,9 @@ and slowly, in float64:
 * ``logprob`` -- LM-head log-softmax, target gather, importance ratio and the
   clipped PPO/GRPO surrogate with its gradient (App. B.4 "Pitfall A, RL view";
   App. F.1 clip range), forward and backward.
+* ``nonmonotone`` -- live views when edits also bring spans back (MemexRL's
+  offload / retrieve, App. F): ordered view lists, a per-key replay as second
+  formulation, rotary positions in view order, compact attention.
 * ``sdcc`` -- SDCC (§5): the final compressed walk, diverging rows, the
   teacher-prefix reconstruction, the forward KL(teacher || student) over the
   vocabulary with the student's gradients, and the lambda ramp (App. F.1).
@@ -29,4 +32,4 @@ and slowly, in float64:
 Every function names the passage it follows in its docstring.
 """
 
-from . import visibility, attention, logprob, sdcc  # noqa: F401
+from . import visibility, attention, logprob, nonmonotone, sdcc  # noqa: F401
