@@ -204,3 +204,47 @@ def test_final_walk_rejects_null_outputs():
     assert h.mw_final_walk(ctypes.byref(lay), P, P, P, None, None) == 1
     assert h.mw_final_walk(ctypes.byref(lay), P, None, P, P, None) == 1
     assert h.mw_final_walk(None, P, P, P, P, None) == 1
+
+
+_C_PROGRAM = r"""
+#include <stdio.h>
+#include <string.h>
+#include "mw.h"
+int main(void) {
+    int32_t cu[3] = {0, 300, 1000};
+    int32_t jt[2] = {1, 1};
+    mw_vis_layout L;
+    if (mw_visibility_layout(2, cu, 2, jt, 3, &L) != MW_OK) return 2;
+    if (L.n_tiles != 3 + 6 || L.max_segs != 3 || L.vis_bytes <= 0) return 3;
+    if (mw_visibility_layout(2, cu, 2, jt, -1, &L) == MW_OK) return 4;   /* negative span count */
+    if (strcmp(mw_status_str(MW_OK), "ok") != 0) return 5;
+    printf("%d %lld\n", mw_abi_version(), (long long)L.n_keymask);
+    return 0;
+}
+"""
+
+
+def test_c_program_links_and_calls_the_abi(tmp_path):
+    """The boundary is a C ABI: a C99 program includes the header, links
+    libmw.so and calls its host-only entry points (no GPU needed)."""
+    import shutil
+    import subprocess
+    gcc = shutil.which("gcc")
+    if gcc is None:
+        pytest.skip("no C compiler")
+    L, _ = _lib()
+    src = tmp_path / "abi.c"
+    src.write_text(_C_PROGRAM)
+    exe = tmp_path / "abi"
+    libdir = os.path.dirname(L.LIB_PATH)
+    r = subprocess.run([gcc, "-std=c99", "-Wall", "-Werror", "-pedantic", "-I", os.path.join(ROOT, "include"),
+                        str(src), "-L", libdir, "-lmw", "-Wl,-rpath," + libdir, "-o", str(exe)],
+                       capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
+    env = dict(os.environ)
+    env["LD_LIBRARY_PATH"] = ":".join(p for p in (libdir, "/usr/local/cuda/lib64", env.get("LD_LIBRARY_PATH", ""))
+                                      if p)
+    run = subprocess.run([str(exe)], capture_output=True, text=True, env=env)
+    assert run.returncode == 0, (run.returncode, run.stderr)
+    ver, n_keymask = map(int, run.stdout.split())
+    assert ver >= 4 and n_keymask == (1 + 0) * 3 + (1 + 2) * 6
