@@ -288,8 +288,8 @@ mw_status mw_diverging_rows(const mw_vis_layout* layout, const void* vis, uint8_
  *   walk_index  int32 [total_tokens]: position of token j on its trajectory's
  *               walk (0-based), -1 if some edit evicts j;
  *   student_row int32 [total_tokens]: for row r, the walk index of the last
- *               surviving position <= r (the walk row whose prediction is the
- *               student's for y_(r+1)), -1 if none;
+ *               surviving position <= r, -1 if none (when token r+1 survives,
+ *               the walk row whose prediction is the student's for it);
  *   walk_len    int32 [n_traj]: the walk's length per trajectory.
  * All device, overwritten. One prefix count of survivors per trajectory.
  */

@@ -129,10 +129,11 @@ def sdcc_penalty(HT, HS, W, diverging, lam):
 
 
 def student_rows(T, edits):
-    """For every row r with a non-empty final-walk prefix, the index on the
-    final walk of the row that makes the student's prediction of y_(r+1): the
-    last surviving position <= r (§5: the student is f(H_comp) at the leaf's
-    place in the compressed walk). Returns {r: walk index}."""
+    """For every row r with a non-empty final-walk prefix, the walk index of
+    the last surviving position <= r. When the leaf y_(r+1) survives on the
+    walk this is the walk row just before it, whose output is the student's
+    prediction of it (§5: f(H_comp) at the leaf's place). Returns
+    {r: walk index}."""
     walk = final_walk(T, edits)
     where = {j: n for n, j in enumerate(walk)}
     out = {}
@@ -147,12 +148,15 @@ def sdcc_objective(T, edits, Q, K, V, W, targets, loss_rows, lp_old, adv, lam, s
     """Eq. "soft_loss" for one trajectory and one attention layer feeding the
     LM head (hidden row = attention output, heads concatenated):
 
-      student  attention over the final compressed walk (causal, no edits),
-               task loss = the clipped surrogate on the loss rows that survive
-               on the walk, scored at their walk position (Naive-Compressed);
+      student  attention over the final compressed walk (causal, no edits);
+               a leaf y_(r+1) (loss row r) is a token of the walk only if it
+               survives every edit, and the walk row before it predicts it
+               (``student_rows``); task loss = the clipped surrogate over those
+               leaves (Naive-Compressed);
       teacher  attention under each row's live view (the exact 4D mask),
                gradients stopped;
-      penalty  lam * sum over diverging rows of KL(teacher || student).
+      penalty  lam * sum over the diverging ones of those leaves of
+               KL(teacher || student) (§5: the set C of diverging leaves).
 
     Returns (objective, task, penalty). Plain composition of the oracle's own
     attention, log-prob and KL functions, in their definitions' order.
@@ -168,13 +172,17 @@ def sdcc_objective(T, edits, Q, K, V, W, targets, loss_rows, lp_old, adv, lam, s
     Hs = Os.reshape(len(walk), -1)
     Ot, _ = attn_fwd([T], [edits], Q, K, V, scale)
     Ht = Ot.reshape(T, -1)
-    rows = [r for r in loss_rows if r in where]
-    lp, _ = logprob(Hs, W, np.asarray(targets)[walk], np.array([where[r] for r in rows], dtype=np.int64))
-    sel = [list(loss_rows).index(r) for r in rows]
+    srow = student_rows(T, edits)
+    leaves = [r for r in loss_rows if r + 1 < T and (r + 1) in where]
+    # the walk row before leaf y_(r+1) predicts it; its target is y_(r+1)'s id
+    tg = np.zeros(len(walk), dtype=np.int64)
+    for r in leaves:
+        tg[srow[r]] = np.asarray(targets)[r]
+    lp, _ = logprob(Hs, W, tg, np.array([srow[r] for r in leaves], dtype=np.int64))
+    sel = [list(loss_rows).index(r) for r in leaves]
     _, _, task, _ = policy_loss(lp, np.asarray(lp_old)[sel], np.asarray(adv)[sel], eps_lo, eps_hi)
     div = diverging_rows(T, edits)
-    srow = student_rows(T, edits)
-    pairs = [(r, srow[r]) for r in range(T) if div[r] and r in srow]
+    pairs = [(r, srow[r]) for r in leaves if div[r]]
     penalty = 0.0
     if pairs and lam != 0.0:
         kl, _, _ = forward_kl(Ht[[a for a, _ in pairs]], Hs[[b for _, b in pairs]], W)

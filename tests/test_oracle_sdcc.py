@@ -217,20 +217,20 @@ def _torch_objective(T, edits, Q, K, Vx, W, targets, loss_rows, lp_old, adv, lam
         q.transpose(0, 1), k.transpose(0, 1), v.transpose(0, 1), attn_mask=mask, scale=scale
     ).transpose(0, 1).reshape(T, -1)
     where = {j: n for n, j in enumerate(walk)}
-    rows = [r for r in loss_rows if r in where]
+    rows = [r for r in loss_rows if r + 1 < T and (r + 1) in where]      # surviving leaves
+    pred = [where[r + 1] - 1 for r in rows]                              # the walk row before each
     sel = [list(loss_rows).index(r) for r in rows]
     ls = torch.log_softmax(st @ w.T, dim=1)
-    lp = ls[[where[r] for r in rows], torch.from_numpy(np.asarray(targets)[rows])]
+    lp = ls[pred, torch.from_numpy(np.asarray(targets)[rows])]
     ratio = torch.exp(lp - torch.from_numpy(np.asarray(lp_old)[sel]))
     a = torch.from_numpy(np.asarray(adv)[sel])
     task = -torch.minimum(ratio * a, ratio.clamp(0.8, 1.28) * a).mean()
     pen = torch.zeros((), dtype=torch.float64)
     div = S.diverging_rows(T, edits)
-    srow = S.student_rows(T, edits)
-    for r in range(T):
-        if div[r] and r in srow:
+    for r, pr in zip(rows, pred):
+        if div[r]:
             lt = torch.log_softmax(te[r] @ w.T, dim=0)
-            pen = pen + (lt.exp() * (lt - ls[srow[r]])).sum()
+            pen = pen + (lt.exp() * (lt - ls[pr])).sum()
     return float(task + lam * pen), float(task), float(lam * pen)
 
 

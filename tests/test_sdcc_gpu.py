@@ -156,3 +156,50 @@ def test_logdiff_matches_oracle(M):
     torch.cuda.synchronize()
     want = OL.logdiff(np64(a), np64(b))
     assert abs(float(got.item()) - want) <= 1e-5 * want   # exact 0 without tokens
+
+
+def test_sdcc_objective_end_to_end():
+    """SDCC's objective for one layer (Eq. "soft_loss") assembled from the GPU
+    entry points: masked attention under the live views (teacher), the final
+    walk and causal attention over it (student), the clipped task loss on the
+    leaves that survive on the walk, the diverging rows and the forward KL;
+    equal to oracle.sdcc.sdcc_objective in float32."""
+    import paper_2609_00865_gb300 as mw
+    rng = np.random.default_rng(77)
+    T, H, Dh, Vv = 300, 2, 64, 500
+    edits = [(90, [(10, 40)]), (150, [(50, 80), (100, 120)]), (230, [(5, 9), (160, 200)])]
+    Q, K, Vx = (torch.from_numpy(rng.standard_normal((T, H, Dh)).astype(np.float32)) for _ in range(3))
+    W = torch.from_numpy((0.05 * rng.standard_normal((Vv, H * Dh))).astype(np.float32))
+    targets = rng.integers(0, Vv, T).astype(np.int32)
+    loss_rows = np.sort(rng.choice(T - 1, 150, replace=False))
+    lp_old = rng.standard_normal(150) * 0.1 - 6.0
+    adv = rng.standard_normal(150)
+    lam, scale = 0.1, Dh ** -0.5
+    vis = mw.build_visibility([T], [edits])
+    Ot, _ = mw.masked_attn_fwd(vis, Q.cuda(), K.cuda(), Vx.cuda(), scale)            # teacher
+    wi, sr, wl = mw.final_walk(vis)
+    div = mw.diverging_rows(vis)
+    torch.cuda.synchronize()
+    wi, sr, div, n = wi.cpu().numpy()[:T], sr.cpu().numpy()[:T], div.cpu().numpy()[:T] > 0, int(wl.cpu()[0])
+    walk = np.argsort(np.where(wi >= 0, wi, T + np.arange(T)))[:n]                    # walk order
+    vis_w = mw.build_visibility([n], [[]])
+    Os, _ = mw.masked_attn_fwd(vis_w, Q[walk].cuda(), K[walk].cuda(), Vx[walk].cuda(), scale)   # student
+    leaves = [i for i, r in enumerate(loss_rows) if wi[r + 1] >= 0]
+    srows = np.array([sr[loss_rows[i]] for i in leaves], dtype=np.int32)
+    tg = np.zeros(n, dtype=np.int32)
+    tg[srows] = targets[loss_rows[leaves]]
+    out = mw.logprob_loss_fwd(Os.reshape(n, -1).contiguous(), W.cuda(), torch.from_numpy(tg).cuda(),
+                              torch.from_numpy(srows).cuda(),
+                              torch.from_numpy(lp_old[leaves].astype(np.float32)).cuda(),
+                              torch.from_numpy(adv[leaves].astype(np.float32)).cuda(), 0.2, 0.28)
+    pairs = [(loss_rows[i], sr[loss_rows[i]]) for i in leaves if div[loss_rows[i]]]
+    assert pairs
+    rt = torch.tensor([a for a, _ in pairs], dtype=torch.int32).cuda()
+    rs = torch.tensor([b for _, b in pairs], dtype=torch.int32).cuda()
+    _, pen, _ = mw.forward_kl_fwd(Ot.reshape(T, -1).contiguous(), rt, Os.reshape(n, -1).contiguous(), rs,
+                                  W.cuda(), lam=lam)
+    torch.cuda.synchronize()
+    _, task, penalty = OS.sdcc_objective(T, edits, np64(Q), np64(K), np64(Vx), np64(W), targets, loss_rows,
+                                         lp_old, adv, lam, scale)
+    assert abs(float(out["loss"].item()) - task) <= 1e-4 * abs(task) + 1e-6
+    assert abs(float(pen.item()) - penalty) <= 1e-4 * abs(penalty)
