@@ -21,13 +21,27 @@ ids under which its visible keys form a gap-free sequence. On the compact
 sequence of a segment that is simply the compact index, so queries and keys
 are rotated by their index in ``view_s`` before the scores are taken, and the
 gradients are rotated back.
+
+Arithmetic: float64 CPU tensors (torch), so that the library's matrix
+products and element-wise passes use every host core; inputs and outputs are
+numpy arrays. Each formula below is the textbook one, evaluated as written.
 """
 
 import numpy as np
+import torch
 
 from .visibility import live_views
 
 _ROW_CHUNK = 512
+
+
+def _t(x):
+    """float64 CPU tensor view of an array (copies only when it must)."""
+    return torch.from_numpy(np.ascontiguousarray(np.asarray(x, dtype=np.float64)))
+
+
+def _ix(x):
+    return torch.from_numpy(np.asarray(x, dtype=np.int64))
 
 
 def _segments(seqlens, edits_per_traj):
@@ -40,35 +54,42 @@ def _segments(seqlens, edits_per_traj):
         base += T
 
 
-def rope(x, pos, theta, inverse=False):
+def _rope_t(x, pos, theta, inverse=False):
     """Rotary position embedding (RoFormer, Su et al. 2021) in the
-    rotate-half pairing: feature f (f < Dh/2) is paired with f + Dh/2 and the
-    pair is turned by the angle ``pos * theta ** (-2 f / Dh)``. ``x`` is
-    ``[n, ..., Dh]`` with one position per leading index; ``inverse`` turns by
-    the opposite angle (the transpose of the rotation).
-    """
-    x = np.asarray(x, dtype=np.float64)
+    rotate-half pairing on a float64 tensor: feature f (f < Dh/2) is paired
+    with f + Dh/2 and the pair is turned by the angle
+    ``pos * theta ** (-2 f / Dh)``. ``x`` is ``[n, ..., Dh]`` with one
+    position per leading index; ``inverse`` turns by the opposite angle (the
+    transpose of the rotation)."""
     half = x.shape[-1] // 2
-    w = float(theta) ** (-2.0 * np.arange(half, dtype=np.float64) / x.shape[-1])
-    ang = np.asarray(pos, dtype=np.float64)[:, None] * w[None, :]
+    w = float(theta) ** (-2.0 * torch.arange(half, dtype=torch.float64) / x.shape[-1])
+    ang = torch.as_tensor(np.asarray(pos, dtype=np.float64))[:, None] * w[None, :]
     if inverse:
         ang = -ang
     ang = ang.reshape((ang.shape[0],) + (1,) * (x.ndim - 2) + (half,))
-    c, s = np.cos(ang), np.sin(ang)
+    c, s = torch.cos(ang), torch.sin(ang)
     a, b = x[..., :half], x[..., half:]
-    return np.concatenate([a * c - b * s, b * c + a * s], axis=-1)
+    return torch.cat([a * c - b * s, b * c + a * s], dim=-1)
 
 
-def _scores(q, k, scale, compact_rows):
-    """Scaled scores of compact rows against the compact keys, causal.
+def rope(x, pos, theta, inverse=False):
+    """``_rope_t`` on numpy arrays (float64 in, float64 out)."""
+    return _rope_t(_t(x), pos, theta, inverse).numpy()
 
-    ``compact_rows[r]`` is the compact index of row r of ``q``; that row may
-    see compact keys ``0 .. compact_rows[r]`` and nothing after.
-    """
+
+def _probs(q, k, scale, compact_rows):
+    """Row softmax of the scaled scores of compact rows against the compact
+    keys, causal: ``compact_rows[r]`` is the compact index of row r of ``q``,
+    which sees compact keys ``0 .. compact_rows[r]`` and nothing after.
+    Masked entries are excluded exactly (their exponential is 0). Returns
+    ``(P, row max, row sum)``."""
     s = (q @ k.T) * scale
-    c = np.arange(k.shape[0])[None, :]
-    s[c > np.asarray(compact_rows)[:, None]] = -np.inf
-    return s
+    c = torch.arange(k.shape[0])[None, :]
+    s.masked_fill_(c > _ix(compact_rows)[:, None], float("-inf"))
+    m = s.amax(dim=1, keepdim=True)
+    p = torch.exp(s - m)
+    l = p.sum(dim=1, keepdim=True)
+    return p, m, l
 
 
 def attn_fwd(seqlens, edits_per_traj, Q, K, V, scale, rows=None, heads=None, rope_theta=None):
@@ -79,43 +100,44 @@ def attn_fwd(seqlens, edits_per_traj, Q, K, V, scale, rows=None, heads=None, rop
     Softmax over each row's visible keys exactly (no large-negative fill).
     With ``rope_theta`` queries and keys are rotated by their compact index.
     """
-    Q = np.asarray(Q, dtype=np.float64)
-    K = np.asarray(K, dtype=np.float64)
-    V = np.asarray(V, dtype=np.float64)
+    Q, K, V = _t(Q), _t(K), _t(V)
     Ttot, Hq, Dh = Q.shape
     Hkv = K.shape[1]
     grp = Hq // Hkv
     heads = list(range(Hq)) if heads is None else list(heads)
     rows = np.arange(Ttot) if rows is None else np.asarray(rows, dtype=np.int64)
-    pos_of = {int(r): n for n, r in enumerate(rows)}
-    O = np.full((len(rows), len(heads), Dh), np.nan)
-    L = np.full((len(heads), len(rows)), np.nan)
+    pos_of = np.full(Ttot, -1, dtype=np.int64)
+    pos_of[rows] = np.arange(rows.size)
+    O = torch.full((len(rows), len(heads), Dh), float("nan"), dtype=torch.float64)
+    L = torch.full((len(heads), len(rows)), float("nan"), dtype=torch.float64)
     want = np.zeros(Ttot, dtype=bool)
     want[rows] = True
     for seg_rows, idx, n_before in _segments(seqlens, edits_per_traj):
         sel = np.nonzero(want[seg_rows])[0]
         if sel.size == 0:
             continue
-        for c0 in range(0, sel.size, _ROW_CHUNK):
-            part = sel[c0 : c0 + _ROW_CHUNK]
-            # compact index of each selected row = n_before + local offset
-            grows = seg_rows[part]
-            out_pos = [pos_of[int(r)] for r in grows]
-            for hi, h in enumerate(heads):
-                g = h // grp
-                k = K[idx, g]
-                v = V[idx, g]
-                q = Q[grows, h]
-                if rope_theta is not None:
-                    k = rope(k, np.arange(idx.size), rope_theta)
-                    q = rope(q, n_before + part, rope_theta)
-                s = _scores(q, k, scale, n_before + part)
-                m = s.max(axis=1, keepdims=True)
-                p = np.exp(s - m)
-                l = p.sum(axis=1, keepdims=True)
-                O[out_pos, hi] = (p @ v) / l
-                L[hi, out_pos] = (m + np.log(l))[:, 0]
-    return O, L
+        ti = _ix(idx)
+        for g in sorted({h // grp for h in heads}):
+            # the segment's compact key / value sequence of KV head g
+            k = K[ti, g]
+            v = V[ti, g]
+            if rope_theta is not None:
+                k = _rope_t(k, np.arange(idx.size), rope_theta)
+            for c0 in range(0, sel.size, _ROW_CHUNK):
+                part = sel[c0 : c0 + _ROW_CHUNK]
+                # compact index of each selected row = n_before + local offset
+                grows = _ix(seg_rows[part])
+                out_pos = _ix(pos_of[seg_rows[part]])
+                for hi, h in enumerate(heads):
+                    if h // grp != g:
+                        continue
+                    q = Q[grows, h]
+                    if rope_theta is not None:
+                        q = _rope_t(q, n_before + part, rope_theta)
+                    p, m, l = _probs(q, k, scale, n_before + part)
+                    O[out_pos, hi] = (p @ v) / l
+                    L[hi, out_pos] = (m + torch.log(l))[:, 0]
+    return O.numpy(), L.numpy()
 
 
 def attn_bwd(seqlens, edits_per_traj, Q, K, V, dO, scale, groups=None, rope_theta=None):
@@ -132,95 +154,92 @@ def attn_bwd(seqlens, edits_per_traj, Q, K, V, dO, scale, groups=None, rope_thet
     With ``rope_theta`` the scores use rotated q and k (compact index) and
     dQ, dK are the rotated-space gradients turned back by the same angles.
     """
-    Q = np.asarray(Q, dtype=np.float64)
-    K = np.asarray(K, dtype=np.float64)
-    V = np.asarray(V, dtype=np.float64)
-    dO = np.asarray(dO, dtype=np.float64)
+    Q, K, V, dO = _t(Q), _t(K), _t(V), _t(dO)
     Ttot, Hq, Dh = Q.shape
     Hkv = K.shape[1]
     grp = Hq // Hkv
     groups = list(range(Hkv)) if groups is None else list(groups)
-    dQ = np.full_like(Q, np.nan)
-    dK = np.full_like(K, np.nan)
-    dV = np.full_like(V, np.nan)
+    dQ = torch.full_like(Q, float("nan"))
+    dK = torch.full_like(K, float("nan"))
+    dV = torch.full_like(V, float("nan"))
     for g in groups:
         dQ[:, g * grp : (g + 1) * grp] = 0.0
         dK[:, g] = 0.0
         dV[:, g] = 0.0
     for seg_rows, idx, n_before in _segments(seqlens, edits_per_traj):
-        for c0 in range(0, seg_rows.size, _ROW_CHUNK):
-            grows = seg_rows[c0 : c0 + _ROW_CHUNK]
-            crow = n_before + c0 + np.arange(grows.size)
-            for g in groups:
-                k = K[idx, g]
-                v = V[idx, g]
-                if rope_theta is not None:
-                    k = rope(k, np.arange(idx.size), rope_theta)
-                dk = np.zeros_like(k)
-                dv = np.zeros_like(v)
+        ti = _ix(idx)
+        for g in groups:
+            k = K[ti, g]
+            v = V[ti, g]
+            if rope_theta is not None:
+                k = _rope_t(k, np.arange(idx.size), rope_theta)
+            dk = torch.zeros_like(k)
+            dv = torch.zeros_like(v)
+            for c0 in range(0, seg_rows.size, _ROW_CHUNK):
+                grows = _ix(seg_rows[c0 : c0 + _ROW_CHUNK])
+                crow = n_before + c0 + np.arange(grows.numel())
                 for h in range(g * grp, (g + 1) * grp):
                     q = Q[grows, h]
                     if rope_theta is not None:
-                        q = rope(q, crow, rope_theta)
+                        q = _rope_t(q, crow, rope_theta)
                     do = dO[grows, h]
-                    s = _scores(q, k, scale, crow)
-                    m = s.max(axis=1, keepdims=True)
-                    p = np.exp(s - m)
-                    p /= p.sum(axis=1, keepdims=True)
+                    p, _, l = _probs(q, k, scale, crow)
+                    p = p / l
                     dp = do @ v.T
-                    ds = p * (dp - (p * dp).sum(axis=1, keepdims=True))
+                    ds = p * (dp - (p * dp).sum(dim=1, keepdim=True))
                     dq = scale * (ds @ k)
                     if rope_theta is not None:
-                        dq = rope(dq, crow, rope_theta, inverse=True)
+                        dq = _rope_t(dq, crow, rope_theta, inverse=True)
                     dQ[grows, h] = dq
                     dk += scale * (ds.T @ q)
                     dv += p.T @ do
-                if rope_theta is not None:
-                    dk = rope(dk, np.arange(idx.size), rope_theta, inverse=True)
-                np.add.at(dK[:, g], idx, dk)
-                np.add.at(dV[:, g], idx, dv)
-    return dQ, dK, dV
+            if rope_theta is not None:
+                dk = _rope_t(dk, np.arange(idx.size), rope_theta, inverse=True)
+            dK[:, g].index_add_(0, ti, dk)
+            dV[:, g].index_add_(0, ti, dv)
+    return dQ.numpy(), dK.numpy(), dV.numpy()
 
 
 def attn_bwd_rows(seqlens, edits_per_traj, Q, K, V, dO, scale, rows, heads, rope_theta=None):
     """dQ of a few physical rows and query heads (same formulas as
     ``attn_bwd``, rotary positions included; a row's dQ needs only its own
-    segment's compact view). Returns ``dQ_sel[r, h_i, :]``."""
-    Q = np.asarray(Q, dtype=np.float64)
-    K = np.asarray(K, dtype=np.float64)
-    V = np.asarray(V, dtype=np.float64)
-    dO = np.asarray(dO, dtype=np.float64)
+    segment's compact view and its own dO row). Returns ``dQ_sel[r, h_i, :]``."""
+    Q, K, V, dO = _t(Q), _t(K), _t(V), _t(dO)
     Hq = Q.shape[1]
     grp = Hq // K.shape[1]
     rows = np.asarray(rows, dtype=np.int64)
-    pos_of = {int(r): n for n, r in enumerate(rows)}
-    out = np.full((rows.size, len(heads), Q.shape[2]), np.nan)
+    pos_of = np.full(Q.shape[0], -1, dtype=np.int64)
+    pos_of[rows] = np.arange(rows.size)
+    out = torch.full((rows.size, len(heads), Q.shape[2]), float("nan"), dtype=torch.float64)
     want = np.zeros(Q.shape[0], dtype=bool)
     want[rows] = True
     for seg_rows, idx, n_before in _segments(seqlens, edits_per_traj):
         part = np.nonzero(want[seg_rows])[0]
         if part.size == 0:
             continue
-        grows = seg_rows[part]
-        outp = [pos_of[int(r)] for r in grows]
+        ti = _ix(idx)
+        grows = _ix(seg_rows[part])
+        outp = _ix(pos_of[seg_rows[part]])
+        kv = {}
         for hi, h in enumerate(heads):
-            k = K[idx, h // grp]
-            v = V[idx, h // grp]
+            if h // grp not in kv:
+                k = K[ti, h // grp]
+                if rope_theta is not None:
+                    k = _rope_t(k, np.arange(idx.size), rope_theta)
+                kv = {h // grp: (k, V[ti, h // grp])}
+            k, v = kv[h // grp]
             q = Q[grows, h]
             if rope_theta is not None:
-                k = rope(k, np.arange(idx.size), rope_theta)
-                q = rope(q, n_before + part, rope_theta)
-            s = _scores(q, k, scale, n_before + part)
-            m = s.max(axis=1, keepdims=True)
-            p = np.exp(s - m)
-            p /= p.sum(axis=1, keepdims=True)
+                q = _rope_t(q, n_before + part, rope_theta)
+            p, _, l = _probs(q, k, scale, n_before + part)
+            p = p / l
             dp = dO[grows, h] @ v.T
-            ds = p * (dp - (p * dp).sum(axis=1, keepdims=True))
+            ds = p * (dp - (p * dp).sum(dim=1, keepdim=True))
             dq = scale * (ds @ k)
             if rope_theta is not None:
-                dq = rope(dq, n_before + part, rope_theta, inverse=True)
+                dq = _rope_t(dq, n_before + part, rope_theta, inverse=True)
             out[outp, hi] = dq
-    return out
+    return out.numpy()
 
 
 def attn_bwd_keys(seqlens, edits_per_traj, Q, K, V, dO, scale, g, keys, rope_theta=None):
@@ -230,46 +249,47 @@ def attn_bwd_keys(seqlens, edits_per_traj, Q, K, V, dO, scale, g, keys, rope_the
     contribution from a segment is turned back by its angle in that segment);
     only the columns of the selected keys of each segment's ``dS`` and ``P``
     are accumulated, but every row's softmax is still normalised over its full
-    live view. Used for sampled checks on workloads too large for the full
-    backward.
+    live view. A row before a key never sees it (the compact sequence is
+    causal), so each segment's rows are taken from the first one at or after
+    its earliest selected key. Used for sampled checks on workloads too large
+    for the full backward.
     """
-    Q = np.asarray(Q, dtype=np.float64)
-    K = np.asarray(K, dtype=np.float64)
-    V = np.asarray(V, dtype=np.float64)
-    dO = np.asarray(dO, dtype=np.float64)
+    Q, K, V, dO = _t(Q), _t(K), _t(V), _t(dO)
     Hq = Q.shape[1]
     grp = Hq // K.shape[1]
     keys = np.asarray(keys, dtype=np.int64)
-    dk_out = np.zeros((keys.size, K.shape[2]))
-    dv_out = np.zeros((keys.size, K.shape[2]))
+    dk_out = torch.zeros((keys.size, K.shape[2]), dtype=torch.float64)
+    dv_out = torch.zeros((keys.size, K.shape[2]), dtype=torch.float64)
     for seg_rows, idx, n_before in _segments(seqlens, edits_per_traj):
         where = {int(p): c for c, p in enumerate(idx)}
         cols = [(n, where[int(kk)]) for n, kk in enumerate(keys) if int(kk) in where]
         if not cols:
             continue
-        kn = np.asarray([a for a, _ in cols])
-        kc = np.asarray([b for _, b in cols])
-        k = K[idx, g]
-        v = V[idx, g]
+        kn = _ix([a for a, _ in cols])
+        kc_np = np.asarray([b for _, b in cols])
+        kc = _ix(kc_np)
+        ti = _ix(idx)
+        k = K[ti, g]
+        v = V[ti, g]
         if rope_theta is not None:
-            k = rope(k, np.arange(idx.size), rope_theta)
-        for c0 in range(0, seg_rows.size, _ROW_CHUNK):
-            grows = seg_rows[c0 : c0 + _ROW_CHUNK]
-            crow = n_before + c0 + np.arange(grows.size)
+            k = _rope_t(k, np.arange(idx.size), rope_theta)
+        # compact row c sees compact key c' only if c' <= c
+        first = max(0, int(kc_np.min()) - n_before)
+        for c0 in range(first, seg_rows.size, _ROW_CHUNK):
+            grows = _ix(seg_rows[c0 : c0 + _ROW_CHUNK])
+            crow = n_before + c0 + np.arange(grows.numel())
             for h in range(g * grp, (g + 1) * grp):
                 q = Q[grows, h]
                 if rope_theta is not None:
-                    q = rope(q, crow, rope_theta)
+                    q = _rope_t(q, crow, rope_theta)
                 do = dO[grows, h]
-                s = _scores(q, k, scale, crow)
-                m = s.max(axis=1, keepdims=True)
-                p = np.exp(s - m)
-                p /= p.sum(axis=1, keepdims=True)
+                p, _, l = _probs(q, k, scale, crow)
+                p = p / l
                 dp = do @ v.T
-                ds = p * (dp - (p * dp).sum(axis=1, keepdims=True))
+                ds = p * (dp - (p * dp).sum(dim=1, keepdim=True))
                 dk = scale * (ds[:, kc].T @ q)
                 if rope_theta is not None:
-                    dk = rope(dk, kc, rope_theta, inverse=True)
-                np.add.at(dk_out, kn, dk)
-                np.add.at(dv_out, kn, p[:, kc].T @ do)
-    return dk_out, dv_out
+                    dk = _rope_t(dk, kc_np, rope_theta, inverse=True)
+                dk_out.index_add_(0, kn, dk)
+                dv_out.index_add_(0, kn, p[:, kc].T @ do)
+    return dk_out.numpy(), dv_out.numpy()

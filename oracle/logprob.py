@@ -12,18 +12,29 @@ loss-carrying tokens (the logdiff average of Eq. 1 runs over the same set).
 Layouts: ``H [N, d]`` hidden rows, ``W [V, d]`` LM-head weight (torch Linear
 layout), ``targets [N]`` next-token ids by physical row, ``rows [M]`` the
 physical rows that carry loss (distinct), ``lp_old, adv [M]``.
+
+Arithmetic: the logit products and the softmax passes run on float64 CPU
+tensors (torch, every host core); inputs and outputs are numpy arrays.
 """
 
 import numpy as np
+import torch
 
 _ROW_CHUNK = 256
 
 
+def _t(x):
+    """float64 CPU tensor view of an array (copies only when it must)."""
+    return torch.from_numpy(np.ascontiguousarray(np.asarray(x, dtype=np.float64)))
+
+
+def _ix(x):
+    return torch.from_numpy(np.asarray(x, dtype=np.int64))
+
+
 def logits(H, W, rows):
     """``z[m, v] = sum_d H[rows[m], d] W[v, d]`` (small problems only)."""
-    H = np.asarray(H, dtype=np.float64)
-    W = np.asarray(W, dtype=np.float64)
-    return H[np.asarray(rows)] @ W.T
+    return (_t(H)[_ix(rows)] @ _t(W).T).numpy()
 
 
 def logprob(H, W, targets, rows):
@@ -31,20 +42,19 @@ def logprob(H, W, targets, rows):
 
     Rows are processed in chunks; each row is independent.
     """
-    H = np.asarray(H, dtype=np.float64)
-    W = np.asarray(W, dtype=np.float64)
+    H, W = _t(H), _t(W)
     rows = np.asarray(rows, dtype=np.int64)
-    tgt = np.asarray(targets, dtype=np.int64)[rows]
-    lse = np.empty(rows.size)
-    lp = np.empty(rows.size)
+    tgt = _ix(np.asarray(targets, dtype=np.int64)[rows])
+    lse = torch.empty(rows.size, dtype=torch.float64)
+    lp = torch.empty(rows.size, dtype=torch.float64)
     for c0 in range(0, rows.size, _ROW_CHUNK):
-        r = rows[c0 : c0 + _ROW_CHUNK]
+        r = _ix(rows[c0 : c0 + _ROW_CHUNK])
         z = H[r] @ W.T
-        m = z.max(axis=1, keepdims=True)
-        l = m[:, 0] + np.log(np.exp(z - m).sum(axis=1))
-        lse[c0 : c0 + r.size] = l
-        lp[c0 : c0 + r.size] = z[np.arange(r.size), tgt[c0 : c0 + r.size]] - l
-    return lp, lse
+        m = z.amax(dim=1, keepdim=True)
+        l = m[:, 0] + torch.log(torch.exp(z - m).sum(dim=1))
+        lse[c0 : c0 + r.numel()] = l
+        lp[c0 : c0 + r.numel()] = z[torch.arange(r.numel()), tgt[c0 : c0 + r.numel()]] - l
+    return lp.numpy(), lse.numpy()
 
 
 def kl_k3(lp, lp_ref):
@@ -89,47 +99,54 @@ def policy_loss(lp, lp_old, adv, eps_lo, eps_hi, dloss=1.0, lp_ref=None, beta=0.
     return ratio, per_tok, loss, g
 
 
-def logprob_loss_bwd(H, W, targets, rows, lse, g):
+def logprob_loss_bwd(H, W, targets, rows, lse, g, dh_rows=None):
     """Gradients of ``L`` with respect to ``H`` and ``W``.
 
     With ``lp_t = z_{t,tgt} - lse_t``, ``dlp_t/dz_{t,v} = 1[v = tgt] - p_{t,v}``
     where ``p = softmax(z_t)``, so ``dz_{t,v} = g_t (1[v = tgt] - p_{t,v})``;
     ``dH_t = sum_v dz_{t,v} W_v`` (zero on rows outside the loss) and
     ``dW_v = sum_t dz_{t,v} H_t``.
+
+    ``dh_rows`` (optional, a subset of ``rows``) computes only those rows' dH
+    and skips dW (returned as None): sampled checks on big heads.
     """
-    H = np.asarray(H, dtype=np.float64)
-    W = np.asarray(W, dtype=np.float64)
+    H, W = _t(H), _t(W)
     rows = np.asarray(rows, dtype=np.int64)
-    tgt = np.asarray(targets, dtype=np.int64)[rows]
-    lse = np.asarray(lse, dtype=np.float64)
-    g = np.asarray(g, dtype=np.float64)
-    dH = np.zeros_like(H)
-    dW = np.zeros_like(W)
-    for c0 in range(0, rows.size, _ROW_CHUNK):
-        r = rows[c0 : c0 + _ROW_CHUNK]
-        sl = slice(c0, c0 + r.size)
+    tgt_all = np.asarray(targets, dtype=np.int64)[rows]
+    lse_all = np.asarray(lse, dtype=np.float64)
+    g_all = np.asarray(g, dtype=np.float64)
+    sel = np.arange(rows.size)
+    if dh_rows is not None:
+        sel = np.nonzero(np.isin(rows, np.asarray(dh_rows, dtype=np.int64)))[0]
+    dH = torch.zeros_like(H)
+    dW = None if dh_rows is not None else torch.zeros_like(W)
+    for c0 in range(0, sel.size, _ROW_CHUNK):
+        s = sel[c0 : c0 + _ROW_CHUNK]
+        r = _ix(rows[s])
         z = H[r] @ W.T
-        p = np.exp(z - lse[sl, None])
-        onehot = np.zeros_like(p)
-        onehot[np.arange(r.size), tgt[sl]] = 1.0
-        dz = g[sl, None] * (onehot - p)
+        p = torch.exp(z - _t(lse_all[s])[:, None])
+        onehot = torch.zeros_like(p)
+        onehot[torch.arange(s.size), _ix(tgt_all[s])] = 1.0
+        dz = _t(g_all[s])[:, None] * (onehot - p)
         dH[r] = dz @ W
-        dW += dz.T @ H[r]
-    return dH, dW
+        if dW is not None:
+            dW += dz.T @ H[r]
+    return dH.numpy(), (None if dW is None else dW.numpy())
 
 
 def logprob_loss_bwd_vocab(H, W, targets, rows, lse, g, vocab):
     """``dW`` for a few vocabulary rows only (sampled checks on big heads)."""
-    H = np.asarray(H, dtype=np.float64)
-    Wv = np.asarray(W, dtype=np.float64)[np.asarray(vocab)]
+    H = _t(H)
+    Wv = _t(W)[_ix(vocab)]
     rows = np.asarray(rows, dtype=np.int64)
     tgt = np.asarray(targets, dtype=np.int64)[rows]
     vocab = np.asarray(vocab, dtype=np.int64)
-    z = H[rows] @ Wv.T
-    p = np.exp(z - np.asarray(lse, dtype=np.float64)[:, None])
-    onehot = (tgt[:, None] == vocab[None, :]).astype(np.float64)
-    dz = np.asarray(g, dtype=np.float64)[:, None] * (onehot - p)
-    return dz.T @ H[rows]
+    Hr = H[_ix(rows)]
+    z = Hr @ Wv.T
+    p = torch.exp(z - _t(lse)[:, None])
+    onehot = _t((tgt[:, None] == vocab[None, :]).astype(np.float64))
+    dz = _t(g)[:, None] * (onehot - p)
+    return (dz.T @ Hr).numpy()
 
 
 def logdiff(lp_train, lp_rollout):

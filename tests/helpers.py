@@ -1,4 +1,5 @@
-"""Shared test helpers: tolerances and tensor plumbing (no method arithmetic)."""
+"""Shared test helpers: tolerances, tensor plumbing and sample choice (no
+method arithmetic)."""
 
 import numpy as np
 import torch
@@ -50,3 +51,29 @@ def assert_grad_bf16(got, ref, what=""):
     assert rf <= 1e-2, f"{what}: relative Frobenius {rf:.3g} > 1e-2"
     scale = float(np.abs(ref).max()) if ref.size else 0.0
     assert_maxabs(got, ref, 5e-2 * scale, what)
+
+
+def lifetime_keys(T, edits, early=(1, 4), n_late=3, seed=0):
+    """Keys of one trajectory chosen by where their lifetimes end: for every
+    junction the last key it evicts (its visible rows end at that junction,
+    inside a PARTIAL q-tile), for the junctions numbered in ``early`` (0-based)
+    also a key it evicts from before the previous junction (visible rows
+    spanning a whole segment), and never-evicted keys late in the last segment
+    plus the last token. The oracle's cost for a key grows with the rows that
+    see it, so the choice keeps every key's visible row range to about one
+    segment."""
+    from oracle.visibility import lifetimes   # the record's lifetimes pick the sample
+    om = lifetimes(T, edits)
+    Js = [J for J, _ in edits]
+    keys = {T - 1}
+    for k, J in enumerate(Js):
+        ev = np.nonzero(om == J)[0]
+        if ev.size:
+            keys.add(int(ev.max()))
+            if k >= 1 and k in early:
+                early = ev[ev < Js[k - 1]]
+                if early.size:
+                    keys.add(int(early.max()))
+    lo = max(Js[-1] if Js else 0, T - 2048)
+    keys.update(np.random.default_rng(seed).integers(lo, T, n_late).tolist())
+    return np.array(sorted(keys), dtype=np.int64)

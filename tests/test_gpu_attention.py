@@ -5,7 +5,7 @@ import pytest
 import torch
 
 import synth
-from helpers import assert_grad_bf16, assert_maxabs, assert_rel, np64
+from helpers import assert_grad_bf16, assert_maxabs, assert_rel, lifetime_keys, np64
 from oracle import attention as OA
 
 pytestmark = pytest.mark.gpu
@@ -214,7 +214,7 @@ def test_sweep_forward_sampled(K, f):
     _full_size_fwd(synth.config_record(5, K=K, f=f), synth.CONFIGS[5], 200 + K)
 
 
-def _full_size_bwd(rec, c, seed, keys_mode):
+def _full_size_bwd(rec, c, seed, keys_mode, early=(1, 4)):
     import paper_2609_00865_gb300 as mw
     T = rec.total
     g = torch.Generator(device="cuda").manual_seed(seed)
@@ -240,9 +240,8 @@ def _full_size_bwd(rec, c, seed, keys_mode):
         keys = np.unique(np.concatenate([[0, 1, 127, 128, t0.T - 1],
                                          [a for J, sp in t0.edits for a, _ in sp[:2]],
                                          rng.integers(0, t0.T, 10)]))
-    else:                          # keys of the last segment only (cheap oracle)
-        J_last = t0.edits[-1][0] if t0.edits else 0
-        keys = np.unique(np.concatenate([[J_last, t0.T - 1], rng.integers(J_last, t0.T, 10)]))
+    else:                          # keys whose lifetimes end at every junction, and never
+        keys = lifetime_keys(t0.T, t0.edits, early=early, seed=seed)
     dkr, dvr = OA.attn_bwd_keys(rec.seqlens[:1], rec.edits[:1], Q64[: t0.T], K64[: t0.T], V64[: t0.T],
                                 dO64[: t0.T], scale, grp, keys)
     assert_grad_bf16(np64(dK[keys, grp]), dkr, "dK (sampled keys)")
@@ -254,8 +253,13 @@ def test_full_size_backward_config2():
 
 
 def test_full_size_backward_config4():
-    _full_size_bwd(synth.config_record(4), synth.CONFIGS[4], 304, "last")
+    """Keys whose lifetimes end at each of the 8 junctions (the PARTIAL-tile
+    interval [j, omega(j)) of the dK/dV kernel), keys visible across a whole
+    segment, and never-evicted keys."""
+    _full_size_bwd(synth.config_record(4), synth.CONFIGS[4], 304, "lifetimes")
 
 
-def test_sweep_backward_sampled():
-    _full_size_bwd(synth.config_record(5, K=8, f=0.6), synth.CONFIGS[5], 305, "last")
+@pytest.mark.parametrize("K,f,early", [(1, 0.3, ()), (8, 0.6, (4,)), (32, 0.9, (1, 16))])
+def test_sweep_backward_sampled(K, f, early):
+    """The sweep's sparsest, middle and densest-eviction points."""
+    _full_size_bwd(synth.config_record(5, K=K, f=f), synth.CONFIGS[5], 305 + K, "lifetimes", early)

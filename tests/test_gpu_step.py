@@ -7,21 +7,22 @@ import pytest
 import torch
 
 import synth
-from helpers import assert_grad_bf16, assert_maxabs, assert_rel, np64
+from helpers import assert_grad_bf16, assert_maxabs, assert_rel, lifetime_keys, np64
 from oracle import attention as OA
 from oracle import logprob as OL
+from oracle.visibility import lifetimes
 
 pytestmark = pytest.mark.gpu
 
 
-def _gpu_chain(rec, Q, K, V, W, tg, rows, lp_old, adv, eps):
+def _gpu_chain(rec, Q, K, V, W, tg, rows, lp_old, adv, eps, eps_hi=None):
     import paper_2609_00865_gb300 as mw
     T, Hq, Dh = Q.shape
     scale = Dh ** -0.5
     vis = mw.build_visibility(rec.seqlens, rec.edits)
     O, LSE = mw.masked_attn_fwd(vis, Q, K, V, scale)
     H = O.view(T, Hq * Dh)
-    out = mw.logprob_loss_fwd(H, W, tg, rows, lp_old, adv, eps, eps)
+    out = mw.logprob_loss_fwd(H, W, tg, rows, lp_old, adv, eps, eps if eps_hi is None else eps_hi)
     dH, dW = mw.logprob_loss_bwd(H, W, tg, rows, out["lse"], out["ws"])
     dQ, dK, dV = mw.masked_attn_bwd(vis, Q, K, V, O, dH.view(T, Hq, Dh), LSE, scale)
     torch.cuda.synchronize()
@@ -63,6 +64,92 @@ def test_config1_chained_fp32():
     assert_rel(np64(dQ), dQr, 1e-4, "dQ")
     assert_rel(np64(dK), dKr, 1e-4, "dK")
     assert_rel(np64(dV), dVr, 1e-4, "dV")
+
+
+EPS_LO, EPS_HI = 0.2, 0.28       # App. F.1's clip range, as the bench runs the step
+
+
+@pytest.mark.slow
+def test_config4_chained_full():
+    """The full-size 7B-shaped layer step exactly as bench.py runs it (bf16,
+    clip 0.2 / 0.28), against the oracle's own chain (§4.3 Theorem
+    "materialization equivalence"): attention at every loss row, the LM head
+    over the whole vocabulary at every loss row, ratio, clipped loss and g
+    (lp_old = the oracle's lp + N(0, 0.05^2)). Compared: O and lp at every
+    loss row, the mean loss (1e-3 relative), and the chained backward at
+    sampled places -- dH rows, dW vocabulary rows, dQ rows, and dK / dV of
+    keys whose lifetimes end at the first two junctions or never end (their
+    rows' dO is the oracle's own dH; keys ending at every junction are checked
+    with a random dO in ``test_gpu_attention``)."""
+    c = synth.CONFIGS[4]
+    rec = synth.config_record(4)
+    T, Hq, Hkv, Dh, V = rec.total, c["Hq"], c["Hkv"], c["Dh"], c["V"]
+    d = Hq * Dh
+    scale = Dh ** -0.5
+    g = torch.Generator(device="cuda").manual_seed(404)
+    Q = torch.randn(T, Hq, Dh, device="cuda", generator=g).to(torch.bfloat16)
+    K = torch.randn(T, Hkv, Dh, device="cuda", generator=g).to(torch.bfloat16)
+    Vv = torch.randn(T, Hkv, Dh, device="cuda", generator=g).to(torch.bfloat16)
+    W = (0.02 * torch.randn(V, d, device="cuda", generator=g)).to(torch.bfloat16)
+    tg = torch.randint(0, V, (T,), device="cuda", generator=g, dtype=torch.int32)
+    rows = rec.loss_rows()
+    M = len(rows)
+    adv = torch.randn(M, device="cuda", generator=g)
+    Q64, K64, V64, W64, t_np, adv64 = np64(Q), np64(K), np64(Vv), np64(W), tg.cpu().numpy(), np64(adv)
+
+    # oracle forward chain over every loss row
+    Or, _ = OA.attn_fwd(rec.seqlens, rec.edits, Q64, K64, V64, scale, rows=rows)
+    Hr = np.zeros((T, d))
+    Hr[rows] = Or.reshape(M, d)
+    lp_r, lse_r = OL.logprob(Hr, W64, t_np, rows)
+    rng = np.random.default_rng(44)
+    lp_old = lp_r + 0.05 * rng.standard_normal(M)
+    ratio_r, _, loss_r, g_r = OL.policy_loss(lp_r, lp_old, adv64, EPS_LO, EPS_HI)
+    # no ratio may sit where fp32 and fp64 could pick different clip branches
+    assert np.min(np.abs(ratio_r - (1 - EPS_LO))) > 1e-3 and np.min(np.abs(ratio_r - (1 + EPS_HI))) > 1e-3
+
+    lp_old_t = torch.tensor(lp_old, dtype=torch.float32, device="cuda")
+    O, out, dH, dW, dQ, dK, dV = _gpu_chain(rec, Q, K, Vv, W, tg, torch.tensor(rows, dtype=torch.int32).cuda(),
+                                            lp_old_t, adv, EPS_LO, EPS_HI)
+    assert_maxabs(np64(O[rows]), Or, 2e-2, "O (every loss row)")
+    assert_maxabs(np64(out["lp"]), lp_r, 1e-2, "lp (every loss row)")
+    loss = float(out["loss"].item())
+    assert abs(loss - loss_r) <= 1e-3 * max(abs(loss_r), np.mean(np.abs(ratio_r * adv64))), (loss, loss_r)
+
+    # chained backward at sampled places
+    t0 = rec.trajs[0]
+    om = lifetimes(t0.T, t0.edits)
+    J2, J_last = t0.edits[1][0], t0.edits[-1][0]
+    # keys whose lifetimes end at the first two junctions (one of them visible
+    # across a whole segment) and never-evicted keys of the last segment: the
+    # oracle's dH is needed at every loss row that sees them
+    keys = np.array([j for j in lifetime_keys(t0.T, t0.edits, seed=4) if om[j] <= J2 or j >= J_last])
+    in_loss = np.zeros(T, dtype=bool)
+    in_loss[rows] = True
+    need = np.zeros(T, dtype=bool)          # rows whose dO the sampled keys read
+    for j in keys:
+        need[j : min(int(om[j]), t0.T)] = True
+    pick = np.sort(rng.choice(M, 24, replace=False))
+    qrows = rows[pick]
+    need[qrows] = True
+    dh_rows = np.nonzero(need & in_loss)[0]
+    dHr, _ = OL.logprob_loss_bwd(Hr, W64, t_np, rows, lse_r, g_r, dh_rows=dh_rows)
+    assert_grad_bf16(np64(dH[dh_rows]), dHr[dh_rows], "dH (sampled rows)")
+    assert float(dH[~torch.from_numpy(in_loss).cuda()].abs().max()) == 0.0, "dH off the loss rows"
+
+    vocab = np.unique(np.concatenate([[0, V - 1], t_np[qrows[:8]], rng.integers(0, V, 48)]))
+    dWr = OL.logprob_loss_bwd_vocab(Hr, W64, t_np, rows, lse_r, g_r, vocab)
+    assert_grad_bf16(np64(dW[torch.from_numpy(vocab).cuda()]), dWr, "dW (sampled vocabulary rows)")
+
+    dO64 = dHr.reshape(T, Hq, Dh)
+    heads = [0, 13, Hq - 1]
+    dQr = OA.attn_bwd_rows(rec.seqlens, rec.edits, Q64, K64, V64, dO64, scale, qrows, heads)
+    assert_grad_bf16(np64(dQ[qrows][:, heads]), dQr, "dQ (sampled rows)")
+    grp = 1
+    dkr, dvr = OA.attn_bwd_keys(rec.seqlens[:1], rec.edits[:1], Q64[: t0.T], K64[: t0.T], V64[: t0.T],
+                                dO64[: t0.T], scale, grp, keys)
+    assert_grad_bf16(np64(dK[keys, grp]), dkr, "dK (keys by lifetime)")
+    assert_grad_bf16(np64(dV[keys, grp]), dvr, "dV (keys by lifetime)")
 
 
 def test_config4_chained_sampled():
