@@ -407,8 +407,9 @@ class Step:
 def cpu_sample(w, budget_s=15.0):
     """Time the oracle on a bounded sample of loss rows of this workload.
 
-    Per sampled row: attention fwd + dQ over all query heads (its segment's
-    compact view), LM-head log-prob over the full vocabulary and the dH/dW
+    Per sampled row: attention fwd and the row's whole attention backward over
+    all query heads (its segment's compact view: dQ and its contributions to
+    dK and dV), LM-head log-prob over the full vocabulary and the dH/dW
     contributions of that row. Returns (tokens/s, cores, description).
     """
     import numpy as np
@@ -435,11 +436,11 @@ def cpu_sample(w, budget_s=15.0):
         if "record" in w:
             r = w["record"]
             Hq, Hkv, Dh = w["heads"]
-            parts.append("attention fwd+dQ, all heads")
+            parts.append("attention fwd + bwd (dQ, dK, dV contributions), all heads")
             th = w.get("rope")
             O, _ = OA.attn_fwd(r.seqlens, r.edits, x["Q"], x["K"], x["V"], Dh ** -0.5, rows=rows, rope_theta=th)
             OA.attn_bwd_rows(r.seqlens, r.edits, x["Q"], x["K"], x["V"], x.get("dO", x["Q"]), Dh ** -0.5,
-                             rows, list(range(Hq)), rope_theta=th)
+                             rows, list(range(Hq)), rope_theta=th, with_kv=True)
         if "rows" in w:
             parts.append("LM-head fwd over the full vocabulary + dH/dW")
             if "H" in x:
@@ -466,8 +467,12 @@ def run_reference(args, rank, world):
         if i >= args.warmup:
             vals.append(v)
     v = sorted(vals)[len(vals) // 2]
+    scored = int(w["rows"].numel()) if "rows" in w else w["record"].total
+    # one whole step at the sampled rate (extrapolated: each timed step is a sample)
     line = {"impl": "reference", "metric": METRIC, "value": v, "unit": "tokens/s", "n_gpus": world,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 / v, "higher_is_better": True,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * scored / v,
+            "ms_per_step_kind": f"extrapolated: {scored} scored tokens per step at the sampled rate",
+            "ms_per_scored_token": 1e3 / v, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": describe(w),
             "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": cores, "kind": "oracle", "sample": desc},

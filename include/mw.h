@@ -157,7 +157,12 @@ mw_status mw_build_visibility(const mw_vis_layout* layout, const int32_t* cu_seq
  *   on every GPU that loads the library until process exit. Records whose
  *   layout->ws_bytes exceeds 1 MiB are rejected with MW_ENOSPACE (nothing is
  *   launched). The first call on a device looks up the array's address with
- *   that device current; make that first call before any stream capture.
+ *   that device current. With CUDA's lazy module loading (the default) that
+ *   first lookup also loads libmw's device code on the device, which places
+ *   the fixed array and may synchronise the device: make one warm-up call at
+ *   set-up time, before any stream capture. The address is kept for the life
+ *   of the process; after cudaDeviceReset on a device it is stale, so a
+ *   process that resets a device must not call this entry point on it again.
  *   All calls on a device share the array: calls whose GPU work overlaps
  *   (other streams or threads) race and must be serialised by the caller.
  *   The caller still provides `vis` (layout->vis_bytes, device). No device
@@ -292,6 +297,10 @@ mw_status mw_diverging_rows(const mw_vis_layout* layout, const void* vis, uint8_
  *               the walk row whose prediction is the student's for it);
  *   walk_len    int32 [n_traj]: the walk's length per trajectory.
  * All device, overwritten. One prefix count of survivors per trajectory.
+ * student_row is defined for every row, including rows whose leaf y_(r+1) is
+ * evicted; SDCC scores a leaf on the student side only when its token survives
+ * on the walk, so a caller keeps loss row r only where walk_index[r + 1] >= 0
+ * (and r + 1 lies inside the trajectory).
  */
 mw_status mw_final_walk(const mw_vis_layout* layout, const void* vis, int32_t* walk_index, int32_t* student_row,
                         int32_t* walk_len, void* stream);

@@ -200,10 +200,15 @@ def attn_bwd(seqlens, edits_per_traj, Q, K, V, dO, scale, groups=None, rope_thet
     return dQ.numpy(), dK.numpy(), dV.numpy()
 
 
-def attn_bwd_rows(seqlens, edits_per_traj, Q, K, V, dO, scale, rows, heads, rope_theta=None):
+def attn_bwd_rows(seqlens, edits_per_traj, Q, K, V, dO, scale, rows, heads, rope_theta=None, with_kv=False):
     """dQ of a few physical rows and query heads (same formulas as
     ``attn_bwd``, rotary positions included; a row's dQ needs only its own
-    segment's compact view and its own dO row). Returns ``dQ_sel[r, h_i, :]``."""
+    segment's compact view and its own dO row). Returns ``dQ_sel[r, h_i, :]``.
+
+    With ``with_kv`` also returns those rows' contributions to dK and dV
+    (``scale dS^T q`` and ``P^T dO`` of the selected rows and heads,
+    scatter-added to the physical key rows, float64 ``[T_total, Hkv, Dh]``):
+    summed over every row and head they are ``attn_bwd``'s dK and dV."""
     Q, K, V, dO = _t(Q), _t(K), _t(V), _t(dO)
     Hq = Q.shape[1]
     grp = Hq // K.shape[1]
@@ -211,6 +216,8 @@ def attn_bwd_rows(seqlens, edits_per_traj, Q, K, V, dO, scale, rows, heads, rope
     pos_of = np.full(Q.shape[0], -1, dtype=np.int64)
     pos_of[rows] = np.arange(rows.size)
     out = torch.full((rows.size, len(heads), Q.shape[2]), float("nan"), dtype=torch.float64)
+    dK = torch.zeros_like(K) if with_kv else None
+    dV = torch.zeros_like(V) if with_kv else None
     want = np.zeros(Q.shape[0], dtype=bool)
     want[rows] = True
     for seg_rows, idx, n_before in _segments(seqlens, edits_per_traj):
@@ -239,6 +246,15 @@ def attn_bwd_rows(seqlens, edits_per_traj, Q, K, V, dO, scale, rows, heads, rope
             if rope_theta is not None:
                 dq = _rope_t(dq, n_before + part, rope_theta, inverse=True)
             out[outp, hi] = dq
+            if with_kv:
+                q = Q[grows, h] if rope_theta is None else _rope_t(Q[grows, h], n_before + part, rope_theta)
+                dk = scale * (ds.T @ q)
+                if rope_theta is not None:
+                    dk = _rope_t(dk, np.arange(idx.size), rope_theta, inverse=True)
+                dK[:, h // grp].index_add_(0, ti, dk)
+                dV[:, h // grp].index_add_(0, ti, p.T @ dO[grows, h])
+    if with_kv:
+        return out.numpy(), dK.numpy(), dV.numpy()
     return out.numpy()
 
 

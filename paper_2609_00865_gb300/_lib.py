@@ -328,7 +328,11 @@ def diverging_rows(vis, stream=None):
 
 def final_walk(vis, stream=None):
     """(walk_index [T], student_row [T], walk_len [n_traj]) int32 device
-    tensors of the final compressed walk (mw_final_walk)."""
+    tensors of the final compressed walk (mw_final_walk).
+
+    ``student_row`` is given for every row; an SDCC caller keeps loss row r
+    only where ``walk_index[r + 1] >= 0`` (leaf y_(r+1) survives on the walk,
+    inside the same trajectory), since an evicted token has no student score."""
     import torch
     L = vis.layout
     dev = vis.vis.device

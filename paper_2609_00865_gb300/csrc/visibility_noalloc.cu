@@ -14,6 +14,12 @@
 // before they are read). Calls whose GPU work overlaps (different streams or
 // threads on one device) race on the array and must be serialised by the
 // caller.
+//
+// With lazy module loading (CUDA's default) the first cudaGetSymbolAddress on
+// a device loads this library's device code there, which places the array
+// and may synchronise the device; callers make a warm-up call at set-up time.
+// The looked-up address is cached per device ordinal for the life of the
+// process and is stale after a cudaDeviceReset of that device.
 
 #include <mutex>
 

@@ -156,3 +156,22 @@ def test_row_sampled_dq_matches_full():
     rows = [0, 63, 20, 41]
     got = A.attn_bwd_rows([T], [edits], Q, K, V_, dO, 0.4, rows, [0, 3])
     np.testing.assert_allclose(got, dQ[rows][:, [0, 3]], rtol=1e-11, atol=1e-13)
+
+
+def test_row_sampled_kv_contributions_sum_to_full():
+    """The per-row dK / dV contributions (``with_kv``, which the CPU baseline
+    times per sampled row) add up over a partition of the rows and all heads
+    to the full backward's dK / dV, and their dQ is unchanged."""
+    T, Hq, Hkv, Dh = 64, 4, 2, 8
+    edits = _edits(T, 31, 3)
+    Q, K, V_, dO = _inputs(T, Hq, Hkv, Dh, 31)
+    dQ, dK, dV = A.attn_bwd([T], [edits], Q, K, V_, dO, 0.4)
+    parts = [np.arange(0, T, 3), np.arange(1, T, 3), np.arange(2, T, 3)]
+    sk, sv = np.zeros_like(dK), np.zeros_like(dV)
+    for rows in parts:
+        dq, dk, dv = A.attn_bwd_rows([T], [edits], Q, K, V_, dO, 0.4, rows, list(range(Hq)), with_kv=True)
+        np.testing.assert_allclose(dq, dQ[rows], rtol=1e-11, atol=1e-13)
+        sk += dk
+        sv += dv
+    np.testing.assert_allclose(sk, dK, rtol=1e-10, atol=1e-12)
+    np.testing.assert_allclose(sv, dV, rtol=1e-10, atol=1e-12)

@@ -276,3 +276,25 @@ def test_rope_key_sampled_dk_dv_match_full():
     dk, dv = A.attn_bwd_keys([T], [edits], Q, K, Vv, dO, 0.3, 1, keys, rope_theta=300.0)
     np.testing.assert_allclose(dk, dK[keys, 1], rtol=1e-12, atol=1e-12)
     np.testing.assert_allclose(dv, dV[keys, 1], rtol=1e-12, atol=1e-12)
+
+
+def test_rope_row_sampled_kv_contributions_sum_to_full():
+    """Per-row dK / dV contributions with rotary positions (each turned back by
+    the key's angle in the row's segment) add up to the full backward."""
+    rng = _rng(13)
+    seqlens = [70, 90]
+    edits = [_random_edits(rng, 70), _random_edits(rng, 90)]
+    T = sum(seqlens)
+    Q = rng.standard_normal((T, 4, 8))
+    K = rng.standard_normal((T, 2, 8))
+    Vv = rng.standard_normal((T, 2, 8))
+    dO = rng.standard_normal((T, 4, 8))
+    _, dK, dV = A.attn_bwd(seqlens, edits, Q, K, Vv, dO, 0.3, rope_theta=300.0)
+    sk, sv = np.zeros_like(dK), np.zeros_like(dV)
+    for rows in (np.arange(0, T, 2), np.arange(1, T, 2)):
+        _, dk, dv = A.attn_bwd_rows(seqlens, edits, Q, K, Vv, dO, 0.3, rows, [0, 1, 2, 3],
+                                    rope_theta=300.0, with_kv=True)
+        sk += dk
+        sv += dv
+    np.testing.assert_allclose(sk, dK, rtol=1e-10, atol=1e-12)
+    np.testing.assert_allclose(sv, dV, rtol=1e-10, atol=1e-12)
