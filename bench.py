@@ -578,8 +578,10 @@ def run_gpu(args, rank, world, local_rank):
                  "mw_masked_attn_bwd": 10.0 / 14.0 * flops.get("attn", 0),
                  "mw_masked_attn_rope_fwd": 4.0 / 14.0 * flops.get("attn", 0),
                  "mw_masked_attn_rope_bwd": 10.0 / 14.0 * flops.get("attn", 0),
-                 "mw_logprob_loss_fwd": 2.0 / 8.0 * flops.get("lm", 0),
-                 "mw_logprob_loss_bwd": 6.0 / 8.0 * flops.get("lm", 0)}.get(dom, 0.0)
+                 # the forward forms the logits and E = sum_v p_v W_v (the dH
+                 # product); the backward recomputes the logits for dW
+                 "mw_logprob_loss_fwd": 4.0 / 8.0 * flops.get("lm", 0),
+                 "mw_logprob_loss_bwd": 4.0 / 8.0 * flops.get("lm", 0)}.get(dom, 0.0)
     achieved = dom_flops / (per_call[dom] * 1e-3) / 1e12
     total_tf = sum(flops.values()) / (ms * 1e-3) / 1e12
     cpu = None

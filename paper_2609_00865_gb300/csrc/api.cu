@@ -43,25 +43,27 @@ __global__ void k_loss_epilogue(int, const float*, const float*, const float*, f
                                 float*, float*);
 __global__ void k_logdiff(int, const float*, const float*, float*);
 
-struct LmPlan {
-    int M_pad, R, NV, C, NVC, grid;
-};
-LmPlan lm_plan(int M, int V);
-mw_status lm_fwd_tc(const void*, const void*, const int32_t*, const int32_t*, int, int, int, void*, int32_t*,
-                    float2*, float*, float*, float*, int32_t*, cudaStream_t);
+mw_status lm_ref_tc(const void*, const void*, const int32_t*, const int32_t*, int, int, int, void*, int32_t*,
+                    float2*, float*, float4*, int32_t*, cudaStream_t);
 
 bool lm_bwd_tc_supported(int d);
 int64_t lm_bwd_tc_scratch(int M, int d);
+int64_t lm_fwd_grp_bytes(int M, int d);
+mw_status lm_fwd_grp_tc(const void*, int, int, int, const void*, const int32_t*, float*, float*, float*, int32_t*,
+                        void*, void*, cudaStream_t);
 mw_status lm_bwd_tc(const void*, int, int, int, int, const int32_t*, const void*, const int32_t*, const float*,
-                    const float*, float, void*, float*, int32_t*, void*, cudaStream_t);
+                    const float*, float, void*, float*, int32_t*, void*, void*, cudaStream_t);
 
 // Tensor-core LM-head path: bf16 with d a multiple of 64 that the clustered
 // backward can split (d / C <= 448 for a cluster of C <= 8 CTAs).
 static bool lm_tc(int d, int dtype) { return dtype == MW_BF16 && d % 64 == 0 && lm_bwd_tc_supported(d); }
 
-// Byte offsets inside the log-prob workspace.
+// Byte offsets inside the log-prob workspace. The bf16 path keeps, between
+// forward and backward: g, the gathered rows (hg, tg) and the fused
+// forward's E and 1 / l (fwd); `part` holds the reference prepass's partials,
+// `bwd` the group passes' parameters, exchange ring and counters.
 struct LmWs {
-    int64_t g, zt, hg, tg, part, bwd, status, bytes;
+    int64_t g, zt, hg, tg, part, bwd, fwd, status, bytes;
 };
 static LmWs lm_ws_layout(int N, int M, int d, int V, int dtype) {
     (void)N; (void)V;
@@ -71,12 +73,13 @@ static LmWs lm_ws_layout(int N, int M, int d, int V, int dtype) {
     w.g = o; o = align256(o + 4 * (int64_t)M);
     w.zt = o; o = align256(o + 4 * (int64_t)M);
     w.status = o; o = align256(o + 32);
-    w.hg = w.tg = w.part = w.bwd = o;
+    w.hg = w.tg = w.part = w.bwd = w.fwd = o;
     if (lm_tc(d, dtype)) {
         w.hg = o; o = align256(o + 2 * M_pad * d);
         w.tg = o; o = align256(o + 4 * M_pad);
         w.part = o; o = align256(o + 8 * 64 * M_pad);
         w.bwd = o; o = align256(o + lm_bwd_tc_scratch(M, d));
+        w.fwd = o; o = align256(o + lm_fwd_grp_bytes(M, d));
     }
     w.bytes = o;
     return w;
@@ -166,8 +169,13 @@ extern "C" mw_status mw_logprob_loss_fwd_kl(const void* H, const void* W, const 
     float* zt = at<float>(ws, w.zt);
     if (lm_tc(d, dtype)) {
         if ((st = cuda_status(cudaMemsetAsync(at<char>(ws, w.status), 0, 32, s))) != MW_OK) return st;
-        st = lm_fwd_tc(H, W, targets, rows, M, d, V, at<char>(ws, w.hg), at<int32_t>(ws, w.tg),
-                       at<float2>(ws, w.part), zt, lse, lp, at<int32_t>(ws, w.status), s);
+        // references from the first vocabulary entries, then the fused pass
+        // over the whole vocabulary (lse, lp, and E for the backward)
+        st = lm_ref_tc(H, W, targets, rows, M, d, V, at<char>(ws, w.hg), at<int32_t>(ws, w.tg),
+                       at<float2>(ws, w.part), zt, at<float4>(ws, w.bwd), at<int32_t>(ws, w.status), s);
+        if (st == MW_OK)
+            st = lm_fwd_grp_tc(W, M, d, V, at<char>(ws, w.hg), at<int32_t>(ws, w.tg), zt, lse, lp,
+                               at<int32_t>(ws, w.status), at<char>(ws, w.bwd), at<char>(ws, w.fwd), s);
     } else {
         st = lm_fwd_simt(H, W, targets, rows, M, d, V, dtype, lse, zt, lp, s);
     }
@@ -195,12 +203,13 @@ extern "C" mw_status mw_logprob_loss_bwd(const void* H, const void* W, const int
     if (M > 0 && (!H || !W || !targets || !rows || !lse)) return MW_EINVAL;
     LmWs w = lm_ws_layout(N, M, d, V, dtype);
     if (lm_tc(d, dtype)) {
-        // the backward reads the forward's gathered rows and g; it writes the
-        // status words and its own scratch region of the workspace
+        // the backward reads the forward's gathered rows, g, E and 1 / l; it
+        // writes the status words and the group passes' scratch
         if ((st = cuda_status(cudaMemsetAsync(at<char>(ws, w.status), 0, 32, (cudaStream_t)stream))) != MW_OK)
             return st;
         return lm_bwd_tc(W, M, N, d, V, rows, at<char>(ws, w.hg), at<int32_t>(ws, w.tg), lse, at<float>(ws, w.g),
-                         dloss, dH, dW, at<int32_t>(ws, w.status), at<char>(ws, w.bwd), (cudaStream_t)stream);
+                         dloss, dH, dW, at<int32_t>(ws, w.status), at<char>(ws, w.bwd), at<char>(ws, w.fwd),
+                         (cudaStream_t)stream);
     }
     return lm_bwd_simt(H, W, targets, rows, M, N, d, V, dtype, lse, at<float>(ws, w.g), dloss, dH, dW,
                        (cudaStream_t)stream);

@@ -1,8 +1,21 @@
-// Tensor-core LM-head backward without materialising logits.
+// Tensor-core LM-head passes over the whole vocabulary without materialising
+// logits, z = Hg W^T (Hg: the gathered loss rows):
 //
-//   dz_{m,v} = dloss g_m (1[v = tgt_m] - exp(z_{m,v} - lse_m)),  z = Hg W^T
-//   dH_{rows[m]} = sum_v dz_{m,v} W_v        (pass 0: loss rows stationary)
-//   dW_v         = sum_m dz_{m,v} Hg_m       (pass 1: vocab rows stationary)
+//   fused forward (mode 2, loss rows stationary): with a fixed per-row
+//     reference r_m (log2 units, the row's largest logit over the first
+//     vocabulary entries), p~_{m,v} = 2^(z_{m,v} log2 e - r_m) and
+//       l_m = sum_v p~_{m,v},  E_m = sum_v p~_{m,v} W_v,  z_{m,tgt_m},
+//     so that lse_m = ln 2 (r_m + log2 l_m) and the softmax-weighted mean
+//     of the W rows, E_m / l_m, is ready for the backward;
+//   dW pass (mode 1, vocab rows stationary):
+//     dz_{m,v} = dloss g_m (1[v = tgt_m] - exp(z_{m,v} - lse_m)),
+//     dW_v = sum_m dz_{m,v} Hg_m;
+//   dH (elementwise, k_lm_dh_from_e): dH_{rows[m]} = sum_v dz_{m,v} W_v
+//     = dloss g_m (W_{tgt_m} - E_m / l_m).
+// A logit more than kGuard (log2 units) above its row's reference is
+// clamped and flags the row; k_lm_repair then recomputes that row's r, l, E
+// and target logit exactly on CUDA cores, so the result never depends on
+// how well the reference was chosen, only the speed does.
 //
 // A pass holds a 128-row tile X of the stationary operand and streams the
 // other operand Y. The tile's accumulator over the whole hidden size (128 x d
@@ -59,19 +72,26 @@ constexpr uint32_t SMEM = S * SLOT + 1024;
 constexpr int MAX_R = 4;             // ring depth
 constexpr int RING_CTAS = 160;       // ring capacity, in CTAs
 constexpr float LOG2E_B = 1.4426950408889634f;
+// Largest exponent (log2 units above the row's reference) the fused forward
+// accepts: p~ <= 2^96 keeps bf16 p~, the fp32 row sums (<= 2^96 V) and E
+// finite with room to spare; a larger one flags the row for k_lm_repair.
+constexpr float kGuard = 96.f;
 
 struct LmBwdParams {
-    int mode;            // 0: dH pass, 1: dW pass
+    int mode;            // 1: dW pass, 2: fused forward (E, row sums, target logit)
     int C, ds;           // cluster size, d-slice (<= 256)
     int L, R;            // accumulation lag in steps, ring depth R = L + 2
     int KD;              // 64-wide k-slices of d
     int NS;              // steps per tile
     int tiles, nclus;    // stationary tiles, clusters in the grid
     int M, M_pad, V;
-    const int32_t* rows;   // [M]
-    const float4* par;     // [M_pad] per loss row: (dloss g, lse log2 e, target bits, -)
-    __nv_bfloat16* dH;     // [N, d]
+    const float4* par;     // [M_pad] per loss row: mode 1 (dloss g, lse log2 e, target bits, -);
+                           // mode 2 (-, r, target bits, -)
     float* dW;             // [V, d]
+    float* E;              // mode 2: [M_pad, d] sum_v p~ W_v
+    float* lpart;          // mode 2: [C][M_pad] row sums of p~ over each group rank's columns
+    float* zt;             // mode 2: [M] target logits
+    int32_t* flag;         // mode 2: [M_pad] set where a logit exceeded the reference by kGuard
     __nv_bfloat16* ring;   // [nclus][R][C][128][NY] dz exchange ring
     uint32_t* ready;       // [nclus][R] dz tiles published into the slot, all uses
     uint32_t* freed;       // [nclus][R] CTAs done reading the slot, all uses
@@ -343,51 +363,46 @@ __global__ void __launch_bounds__(NT, 1)
         const int rl = qw * 32 + lane;
         const uint32_t lane_base = tmem + ((uint32_t)(qw * 32) << 16);
         bool ok = true;
-        // drain the accumulator of tile `tile` (its `n`-th) into dH / dW
+        // drain the accumulator of tile `tile` (its `n`-th) into dW (mode 1) or E (mode 2)
         auto output = [&](int tile, int n) -> bool {
             if (!mbar_wait(&acc_full, (uint32_t)n & 1u, status, 621)) return false;
             tc_fence_after();
             const int srow = tile * 128 + rl;
-            const bool valid = p.mode == 0 ? srow < p.M : srow < p.V;
-            const int64_t orow = valid ? (p.mode == 0 ? (int64_t)p.rows[srow] : (int64_t)srow) : 0;
+            const bool valid = p.mode == 1 ? srow < p.V : srow < p.M;
+            const int64_t orow = valid ? (int64_t)srow : 0;
             const int64_t d = (int64_t)C * ds;
             for (int c0 = 0; c0 < ds; c0 += 32) {
                 uint32_t o[32];
                 tmem_ld32(lane_base + TM_ACC + c0, o);
                 tmem_wait_ld();
                 if (!valid) continue;
-                if (p.mode == 0) {
-                    __nv_bfloat16* dst = p.dH + orow * d + col0 + c0;
+                float* dst = (p.mode == 1 ? p.dW : p.E) + orow * d + col0 + c0;
 #pragma unroll
-                    for (int x = 0; x < 4; ++x) {
-                        uint4 pk;
-                        pk.x = pack_bf16(__uint_as_float(o[8 * x + 0]), __uint_as_float(o[8 * x + 1]));
-                        pk.y = pack_bf16(__uint_as_float(o[8 * x + 2]), __uint_as_float(o[8 * x + 3]));
-                        pk.z = pack_bf16(__uint_as_float(o[8 * x + 4]), __uint_as_float(o[8 * x + 5]));
-                        pk.w = pack_bf16(__uint_as_float(o[8 * x + 6]), __uint_as_float(o[8 * x + 7]));
-                        reinterpret_cast<uint4*>(dst)[x] = pk;
-                    }
-                } else {
-                    float* dst = p.dW + orow * d + col0 + c0;
-#pragma unroll
-                    for (int x = 0; x < 8; ++x)
-                        reinterpret_cast<uint4*>(dst)[x] = make_uint4(o[4 * x], o[4 * x + 1], o[4 * x + 2], o[4 * x + 3]);
-                }
+                for (int x = 0; x < 8; ++x)
+                    reinterpret_cast<uint4*>(dst)[x] = make_uint4(o[4 * x], o[4 * x + 1], o[4 * x + 2], o[4 * x + 3]);
             }
             tc_fence_before();
             mbar_arrive(&acc_free);
             return true;
         };
-        // dz = x ((c == tgt) - 2^(z log2 e - y)) with (x, y, tgt) = (dloss g, lse
-        // log2 e, target) of the loss row: per thread in pass 0, per column in
-        // pass 1. Padded loss rows carry x = 0; streamed rows past the end are
+        // mode 1: dz = x ((c == tgt) - 2^(z log2 e - y)) with (x, y, tgt) =
+        // (dloss g, lse log2 e, target) of the loss row of each column; padded
+        // loss rows carry x = 0. Mode 2: dz = p~ = 2^(z log2 e - r) of this
+        // thread's row, 0 past the vocabulary. Streamed rows past the end are
         // zero-filled by TMA, so their dz contributes nothing.
         float4 rp = make_float4(0.f, 0.f, __int_as_float(-1), 0.f);
+        float lsum = 0.f, zt_v = 0.f, xmax = -INFINITY;   // mode 2: this row over this CTA's columns
+        bool zt_found = false;
         int t = 0, tile = cid, slot = 0, drained = 0;
         uint32_t uses = 0;                      // earlier uses of ring slot `slot`
         int next_drain = NS + L - 1;            // step after which tile `drained` is complete
         for (int gt = 0; ok && gt < G; ++gt) {
-            if (p.mode == 0 && t == 0) rp = p.par[tile * 128 + rl];
+            if (p.mode != 1 && t == 0) {
+                rp = p.par[tile * 128 + rl];
+                lsum = 0.f;
+                xmax = -INFINITY;
+                zt_found = false;
+            }
             const int cb = t * C * NY + rank * NY;   // first streamed row of this CTA's tile
             float4 cpar[NY / 32];                    // pass 1: parameters of columns cb + 32 j + lane
             if (p.mode == 1) {
@@ -415,7 +430,8 @@ __global__ void __launch_bounds__(NT, 1)
             }
             __nv_bfloat16* dst = p.ring + (int64_t)(ring_row(slot, rank) + rl) * NY;
             const int vrow = tile * 128 + rl;        // pass 1: this row's vocabulary entry
-            const int tj = __float_as_int(rp.z) - cb;   // pass 0: target column inside the tile
+            const int tj = __float_as_int(rp.z) - cb;   // passes 0, 2: target column inside the tile
+            const int nvalid = p.V - cb;                // mode 2: columns inside the vocabulary
 #pragma unroll
             for (int j = 0; j < NY / 32; ++j) {
                 uint32_t z[32];
@@ -433,9 +449,20 @@ __global__ void __launch_bounds__(NT, 1)
                     for (int y = 0; y < 2; ++y) {
                         const int c = 32 * j + x + y;
                         const float zv = __uint_as_float(z[x + y]);
-                        if (p.mode == 0) {
-                            const float pr = ex2f_approx(fmaf(zv, LOG2E_B, -rp.y));
-                            dz[y] = rp.x * ((c == tj ? 1.f : 0.f) - pr);
+                        if (p.mode == 2) {
+                            // columns past the vocabulary (zero-filled W rows) get p~ = 0
+                            float pr = 0.f;
+                            if (c < nvalid) {
+                                const float xe = fmaf(zv, LOG2E_B, -rp.y);
+                                xmax = fmaxf(xmax, xe);
+                                pr = ex2f_approx(fminf(xe, kGuard));
+                                lsum += pr;
+                            }
+                            if (c == tj) {
+                                zt_v = zv;
+                                zt_found = true;
+                            }
+                            dz[y] = pr;
                         } else {
                             const float cx = __shfl_sync(0xffffffffu, cpar[j].x, x + y);
                             const float cy = __shfl_sync(0xffffffffu, cpar[j].y, x + y);
@@ -456,6 +483,13 @@ __global__ void __launch_bounds__(NT, 1)
             if (++slot == R) {
                 slot = 0;
                 ++uses;
+            }
+            if (p.mode == 2 && t == NS - 1) {
+                // the row has met all of this CTA's columns
+                const int m = tile * 128 + rl;
+                p.lpart[(int64_t)rank * p.M_pad + m] = lsum;
+                if (zt_found && m < p.M) p.zt[m] = zt_v;
+                if (xmax > kGuard && m < p.M) p.flag[m] = 1;
             }
             if (++t == NS) {
                 t = 0;
@@ -490,45 +524,168 @@ __global__ void k_lm_bwd_par(int M, int M_pad, const float* __restrict__ g, cons
                    : make_float4(0.f, 0.f, __int_as_float(-1), 0.f);
 }
 
+// Exact recomputation of a flagged row of the fused forward (some logit more
+// than kGuard above the row's reference), on CUDA cores: r = the row's largest
+// logit over the whole vocabulary (log2 units), l = sum_v 2^(z_v log2 e - r),
+// E = sum_v 2^(z_v log2 e - r) W_v, the target logit. One block per flagged
+// row (grid-stride over the rows; unflagged rows return at once); warp w takes
+// vocabulary entries w, w + 8, ...; a logit is a warp dot product over d in
+// float32. Both passes form z_v the same way, so the weights of pass 2 are
+// consistent with r and l of pass 1.
+constexpr int RP_WARPS = 8;
+__global__ void __launch_bounds__(RP_WARPS * 32)
+    k_lm_repair(int M, int M_pad, int d, int V, int C, const __nv_bfloat16* __restrict__ Hg,
+                const __nv_bfloat16* __restrict__ W, const int32_t* __restrict__ tg, const int32_t* __restrict__ flag,
+                float4* __restrict__ par, float* __restrict__ lpart, float* __restrict__ zt, float* __restrict__ E) {
+    extern __shared__ float rp_smem[];
+    float* h = rp_smem;               // [d]
+    float* acc = rp_smem + d;         // [RP_WARPS][d]
+    __shared__ float wm[RP_WARPS], wl[RP_WARPS];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int nvec = d / 8;           // 16-byte vectors of a row
+    for (int m = blockIdx.x; m < M; m += gridDim.x) {
+        if (!flag[m]) continue;       // uniform over the block
+        for (int k = threadIdx.x; k < d; k += blockDim.x) h[k] = __bfloat162float(Hg[(int64_t)m * d + k]);
+        for (int k = threadIdx.x; k < RP_WARPS * d; k += blockDim.x) acc[k] = 0.f;
+        __syncthreads();
+        auto logit = [&](int v) -> float {
+            const uint4* wr = reinterpret_cast<const uint4*>(W + (int64_t)v * d);
+            float a = 0.f;
+            for (int k = lane; k < nvec; k += 32) {
+                const uint4 u = __ldg(&wr[k]);
+                const uint32_t w4[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    a = fmaf(__uint_as_float(w4[e] << 16), h[8 * k + 2 * e], a);
+                    a = fmaf(__uint_as_float(w4[e] & 0xffff0000u), h[8 * k + 2 * e + 1], a);
+                }
+            }
+            return warp_sum(a);
+        };
+        const int t = tg[m];
+        // pass 1: online (max, sum) per warp, log2 units
+        float mx = -INFINITY, l = 0.f;
+        for (int v = warp; v < V; v += RP_WARPS) {
+            const float z = logit(v);
+            if (v == t && lane == 0) zt[m] = z;
+            const float x = z * LOG2E_B;
+            if (x > mx) {
+                l = l * exp2f(mx - x) + 1.f;
+                mx = x;
+            } else {
+                l += exp2f(x - mx);
+            }
+        }
+        if (lane == 0) {
+            wm[warp] = mx;
+            wl[warp] = l;
+        }
+        __syncthreads();
+        float r = -INFINITY;
+        for (int w = 0; w < RP_WARPS; ++w) r = fmaxf(r, wm[w]);
+        float lt = 0.f;
+        for (int w = 0; w < RP_WARPS; ++w) lt += wl[w] > 0.f ? wl[w] * exp2f(wm[w] - r) : 0.f;
+        // pass 2: E = sum_v 2^(z_v log2 e - r) W_v, per warp into its own row of acc
+        float* aw = acc + warp * d;
+        for (int v = warp; v < V; v += RP_WARPS) {
+            const float pv = exp2f(logit(v) * LOG2E_B - r);
+            const uint4* wr = reinterpret_cast<const uint4*>(W + (int64_t)v * d);
+            for (int k = lane; k < nvec; k += 32) {
+                const uint4 u = __ldg(&wr[k]);
+                const uint32_t w4[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    aw[8 * k + 2 * e] = fmaf(pv, __uint_as_float(w4[e] << 16), aw[8 * k + 2 * e]);
+                    aw[8 * k + 2 * e + 1] = fmaf(pv, __uint_as_float(w4[e] & 0xffff0000u), aw[8 * k + 2 * e + 1]);
+                }
+            }
+        }
+        __syncthreads();
+        for (int k = threadIdx.x; k < d; k += blockDim.x) {
+            float e = 0.f;
+            for (int w = 0; w < RP_WARPS; ++w) e += acc[w * d + k];
+            E[(int64_t)m * d + k] = e;
+        }
+        if (threadIdx.x == 0) {
+            float4 q = par[m];
+            q.y = r;
+            par[m] = q;
+            lpart[m] = lt;
+            for (int c = 1; c < C; ++c) lpart[(int64_t)c * M_pad + m] = 0.f;
+        }
+        __syncthreads();
+    }
+}
+
+// lse = ln 2 (r + log2 sum_c lpart_c), lp = z_target - lse, 1 / l for the dH.
+__global__ void k_lm_grp_combine(int M, int M_pad, int C, const float4* __restrict__ par,
+                                 const float* __restrict__ lpart, const float* __restrict__ zt,
+                                 float* __restrict__ lse, float* __restrict__ lp, float* __restrict__ linv) {
+    const int m = blockIdx.x * blockDim.x + threadIdx.x;
+    if (m >= M) return;
+    float l = 0.f;
+    for (int c = 0; c < C; ++c) l += lpart[(int64_t)c * M_pad + m];
+    const float v = (par[m].y + log2f(l)) * 0.6931471805599453f;
+    lse[m] = v;
+    lp[m] = zt[m] - v;
+    linv[m] = 1.f / l;
+}
+
+// dH_{rows[m]} = dloss g_m (W_{tgt_m} - E_m / l_m), bf16; one block per loss
+// row (grid-stride), 16-byte vectors along d. Rows outside the loss stay 0.
+__global__ void k_lm_dh_from_e(int M, int d, const __nv_bfloat16* __restrict__ W, const int32_t* __restrict__ tg,
+                               const float* __restrict__ E, const float* __restrict__ linv,
+                               const float* __restrict__ g, float dloss, const int32_t* __restrict__ rows,
+                               __nv_bfloat16* __restrict__ dH) {
+    const int nvec = d / 8;
+    for (int m = blockIdx.x; m < M; m += gridDim.x) {
+        const float a = dloss * g[m], il = linv[m];
+        const uint4* wr = reinterpret_cast<const uint4*>(W + (int64_t)tg[m] * d);
+        const float4* er = reinterpret_cast<const float4*>(E + (int64_t)m * d);
+        uint4* out = reinterpret_cast<uint4*>(dH + (int64_t)rows[m] * d);
+        for (int k = threadIdx.x; k < nvec; k += blockDim.x) {
+            const uint4 u = __ldg(&wr[k]);
+            const float4 e0 = er[2 * k], e1 = er[2 * k + 1];
+            const float ev[8] = {e0.x, e0.y, e0.z, e0.w, e1.x, e1.y, e1.z, e1.w};
+            const uint32_t w4[4] = {u.x, u.y, u.z, u.w};
+            uint32_t o[4];
+#pragma unroll
+            for (int x = 0; x < 4; ++x) {
+                const float lo = a * (__uint_as_float(w4[x] << 16) - ev[2 * x] * il);
+                const float hi = a * (__uint_as_float(w4[x] & 0xffff0000u) - ev[2 * x + 1] * il);
+                o[x] = pack_bf16(lo, hi);
+            }
+            out[k] = make_uint4(o[0], o[1], o[2], o[3]);
+        }
+    }
+}
+
 // Group sizes whose d-slice fits beside a 256-column logit tile in TMEM
 // (ds <= 256) and keeps 32-column output chunks (ds % 32 == 0).
 bool slice_ok(int d, int C) { return d % C == 0 && d / C <= 256 && (d / C) % 32 == 0; }
 constexpr int kGroupSizes[] = {1, 2, 3, 4, 5, 6, 7, 8, 10, 12, 14, 16};
-constexpr int64_t kCounterBytes = 2 * 2 * RING_CTAS * MAX_R * 4;   // per pass: ready, freed
+constexpr int kMaxGroup = 16;
+constexpr int64_t kCounterBytes = 2 * RING_CTAS * MAX_R * 4;   // ready, freed
 
-}  // namespace
-
-bool lm_bwd_tc_supported(int d) {
-    if (d % 64) return false;
-    for (int C : kGroupSizes)
-        if (slice_ok(d, C)) return true;
-    return false;
+// The fewest CTAs per group (the widest slice): a CTA's tensor work per
+// step is 2 * 128 * NY * d FLOP for any C, but its dz chunk loads, stages
+// and waits per step grow with C (d = 3584 measured: C = 14, 140 CTAs,
+// 114 ms; C = 16, 144 CTAs, 127 ms; d = 1536: C = 6 beats C = 8 and 12).
+int group_size(int d) {
+    for (int c : kGroupSizes)
+        if (slice_ok(d, c)) return c;
+    return 0;
 }
 
-// Scratch of the backward inside the log-prob workspace: the per-row
-// parameters, the dz exchange ring and the ring slots' counters.
-int64_t lm_bwd_tc_scratch(int M, int d) {
-    if (!lm_bwd_tc_supported(d)) return 0;
-    const int64_t M_pad = ceil_div(M, 128) * 128;
-    return align256(16 * M_pad) + (int64_t)RING_CTAS * MAX_R * 128 * NY * 2 + kCounterBytes;
-}
-
-mw_status lm_bwd_tc(const void* W, int M, int N, int d, int V, const int32_t* rows, const void* Hg, const int32_t* tg,
-                    const float* lse, const float* g, float dloss, void* dH, float* dW, int32_t* status, void* scratch,
-                    cudaStream_t s) {
-    if (!lm_bwd_tc_supported(d)) return MW_ESHAPE;
-    mw_status st = cuda_status(cudaMemsetAsync(dH, 0, (size_t)N * d * 2, s));
-    if (st != MW_OK) return st;
-    if (M == 0) return cuda_status(cudaMemsetAsync(dW, 0, (size_t)V * d * 4, s));
+// One launch of k_lm_bwd_tc in `mode` over M loss rows; the scratch holds the
+// per-row parameters (filled by the caller), the ring and its counters.
+mw_status launch_group(LmBwdParams p, const void* W, int d, const void* Hg, void* scratch, cudaStream_t s) {
+    const int M = p.M, V = p.V;
     const int M_pad = (int)ceil_div(M, 128) * 128;
-    float4* par = (float4*)scratch;
     __nv_bfloat16* ring = at<__nv_bfloat16>(scratch, align256(16 * (int64_t)M_pad));
     uint32_t* counters = at<uint32_t>(ring, (int64_t)RING_CTAS * MAX_R * 128 * NY * 2);
-    if ((st = cuda_status(cudaMemsetAsync(counters, 0, kCounterBytes, s))) != MW_OK) return st;
-    count_launches(1);
-    k_lm_bwd_par<<<(unsigned)ceil_div(M_pad, 256), 256, 0, s>>>(M, M_pad, g, lse, tg, dloss, par);
-    if ((st = launch_status()) != MW_OK) return st;
-
+    mw_status st = cuda_status(cudaMemsetAsync(counters, 0, kCounterBytes, s));
+    if (st != MW_OK) return st;
     if ((st = cuda_status(cudaFuncSetAttribute(k_lm_bwd_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                (int)SMEM))) != MW_OK)
         return st;
@@ -541,16 +698,7 @@ mw_status lm_bwd_tc(const void* W, int M, int N, int d, int V, const int32_t* ro
         (st = cuda_status(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_lm_bwd_tc, NT, SMEM))) != MW_OK)
         return st;
     const int resident = std::min(per_sm * sms, RING_CTAS);
-    // The fewest CTAs per group (the widest slice): a CTA's tensor work per
-    // step is 2 * 128 * NY * d FLOP for any C, but its dz chunk loads, stages
-    // and waits per step grow with C (d = 3584 measured: C = 14, 140 CTAs,
-    // 114 ms; C = 16, 144 CTAs, 127 ms; d = 1536: C = 6 beats C = 8 and 12).
-    int C = 0;
-    for (int c : kGroupSizes)
-        if (slice_ok(d, c)) {
-            C = c;
-            break;
-        }
+    const int C = group_size(d);
     const int max_groups = C > 0 ? resident / C : 0;
     if (max_groups == 0) return MW_EDEVICE;
     cudaLaunchConfig_t cfg = {};
@@ -564,41 +712,128 @@ mw_status lm_bwd_tc(const void* W, int M, int N, int d, int V, const int32_t* ro
     cfg.numAttrs = 1;
 
     const int ring_rows = RING_CTAS * MAX_R * 128;
-    CUtensorMap hx, hyz, hya, wx, wyz, wya, dm;
-    if (!tmap_bf16_2d(&hx, Hg, M_pad, d, d, 128, 64) || !tmap_bf16_2d(&hyz, Hg, M_pad, d, d, NY, 64) ||
-        !tmap_bf16_2d(&hya, Hg, M_pad, d, d, 64, 64) || !tmap_bf16_2d(&wx, W, V, d, d, 128, 64) ||
-        !tmap_bf16_2d(&wyz, W, V, d, d, NY, 64) || !tmap_bf16_2d(&wya, W, V, d, d, 64, 64) ||
-        !tmap_bf16_2d(&dm, ring, ring_rows, NY, NY, 128, 64))
-        return MW_ECUDA;
+    const bool rows_x = p.mode != 1;   // loss rows stationary
+    CUtensorMap tx, tyz, tya, dm;
+    const bool ok = rows_x ? (tmap_bf16_2d(&tx, Hg, M_pad, d, d, 128, 64) && tmap_bf16_2d(&tyz, W, V, d, d, NY, 64) &&
+                              tmap_bf16_2d(&tya, W, V, d, d, 64, 64))
+                           : (tmap_bf16_2d(&tx, W, V, d, d, 128, 64) && tmap_bf16_2d(&tyz, Hg, M_pad, d, d, NY, 64) &&
+                              tmap_bf16_2d(&tya, Hg, M_pad, d, d, 64, 64));
+    if (!ok || !tmap_bf16_2d(&dm, ring, ring_rows, NY, NY, 128, 64)) return MW_ECUDA;
 
-    LmBwdParams p;
     p.C = C;
     p.ds = d / C;
     p.L = 2;
     p.R = p.L + 2;
     p.KD = d / 64;
-    p.M = M;
     p.M_pad = M_pad;
-    p.V = V;
-    p.rows = rows;
-    p.par = par;
-    p.dH = (__nv_bfloat16*)dH;
-    p.dW = dW;
+    p.par = (const float4*)scratch;
     p.ring = ring;
+    p.ready = counters;
+    p.freed = counters + RING_CTAS * MAX_R;
+    p.tiles = rows_x ? M_pad / 128 : (int)ceil_div(V, 128);
+    p.NS = (int)ceil_div(rows_x ? V : M_pad, (int64_t)C * NY);
+    p.nclus = std::min(p.tiles, max_groups);
+    cfg.gridDim = dim3((unsigned)(p.nclus * C));
+    count_launches(1);
+    if ((st = cuda_status(cudaLaunchKernelEx(&cfg, k_lm_bwd_tc, tx, tyz, tya, dm, p))) != MW_OK) return st;
+    return launch_status();
+}
+
+}  // namespace
+
+bool lm_bwd_tc_supported(int d) {
+    if (d % 64) return false;
+    return group_size(d) > 0;
+}
+
+// Scratch of the group passes inside the log-prob workspace: the per-row
+// parameters, the dz exchange ring and the ring slots' counters.
+int64_t lm_bwd_tc_scratch(int M, int d) {
+    if (!lm_bwd_tc_supported(d)) return 0;
+    const int64_t M_pad = ceil_div(M, 128) * 128;
+    return align256(16 * M_pad) + (int64_t)RING_CTAS * MAX_R * 128 * NY * 2 + kCounterBytes;
+}
+
+// Fused-forward arrays inside the log-prob workspace, after the scratch:
+// E [M_pad, d] fp32, lpart [kMaxGroup][M_pad], linv [M_pad], flag [M_pad].
+int64_t lm_fwd_grp_bytes(int M, int d) {
+    if (!lm_bwd_tc_supported(d)) return 0;
+    const int64_t M_pad = ceil_div(M, 128) * 128;
+    return align256(4 * M_pad * d) + align256(4 * kMaxGroup * M_pad) + 2 * align256(4 * M_pad);
+}
+
+struct GrpArrays {
+    float *E, *lpart, *linv;
+    int32_t* flag;
+};
+static GrpArrays grp_arrays(void* fwd, int M, int d) {
+    const int64_t M_pad = ceil_div(M, 128) * 128;
+    GrpArrays a;
+    a.E = (float*)fwd;
+    a.lpart = at<float>(a.E, align256(4 * M_pad * d));
+    a.linv = at<float>(a.lpart, align256(4 * kMaxGroup * M_pad));
+    a.flag = at<int32_t>(a.linv, align256(4 * M_pad));
+    return a;
+}
+
+// Fused forward over the whole vocabulary: the gathered rows Hg / tg and the
+// references in the scratch's parameter array (k_lm_ref) are in place. Writes
+// lse, lp (per loss row), zt, and keeps E and 1 / l for the backward.
+mw_status lm_fwd_grp_tc(const void* W, int M, int d, int V, const void* Hg, const int32_t* tg, float* zt, float* lse,
+                        float* lp, int32_t* status, void* scratch, void* fwd, cudaStream_t s) {
+    if (!lm_bwd_tc_supported(d)) return MW_ESHAPE;
+    if (M == 0) return MW_OK;
+    const int M_pad = (int)ceil_div(M, 128) * 128;
+    GrpArrays a = grp_arrays(fwd, M, d);
+    mw_status st = cuda_status(cudaMemsetAsync(a.flag, 0, 4 * (size_t)M_pad, s));
+    if (st != MW_OK) return st;
+    LmBwdParams p = {};
+    p.mode = 2;
+    p.M = M;
+    p.V = V;
+    p.E = a.E;
+    p.lpart = a.lpart;
+    p.zt = zt;
+    p.flag = a.flag;
     p.status = status;
-    for (int mode = 0; mode < 2; ++mode) {
-        p.mode = mode;
-        p.ready = counters + mode * 2 * RING_CTAS * MAX_R;
-        p.freed = p.ready + RING_CTAS * MAX_R;
-        p.tiles = mode == 0 ? M_pad / 128 : (int)ceil_div(V, 128);
-        p.NS = (int)ceil_div(mode == 0 ? V : M_pad, (int64_t)C * NY);
-        p.nclus = std::min(p.tiles, max_groups);
-        cfg.gridDim = dim3((unsigned)(p.nclus * C));
-        count_launches(1);
-        if ((st = cuda_status(cudaLaunchKernelEx(&cfg, k_lm_bwd_tc, mode == 0 ? hx : wx, mode == 0 ? wyz : hyz,
-                                                 mode == 0 ? wya : hya, dm, p))) != MW_OK)
-            return st;
-    }
+    if ((st = launch_group(p, W, d, Hg, scratch, s)) != MW_OK) return st;
+    const size_t rp_smem = (size_t)(RP_WARPS + 1) * d * 4;
+    if ((st = cuda_status(cudaFuncSetAttribute(k_lm_repair, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               (int)rp_smem))) != MW_OK)
+        return st;
+    const int C = group_size(d);
+    count_launches(2);
+    k_lm_repair<<<(unsigned)std::min(M, 4 * 152), RP_WARPS * 32, rp_smem, s>>>(
+        M, M_pad, d, V, C, (const __nv_bfloat16*)Hg, (const __nv_bfloat16*)W, tg, a.flag, (float4*)scratch, a.lpart,
+        zt, a.E);
+    k_lm_grp_combine<<<(unsigned)ceil_div(M, 256), 256, 0, s>>>(M, M_pad, C, (const float4*)scratch, a.lpart, zt,
+                                                                lse, lp, a.linv);
+    return launch_status();
+}
+
+// Backward: dW by the vocabulary-stationary pass, dH from the forward's E.
+mw_status lm_bwd_tc(const void* W, int M, int N, int d, int V, const int32_t* rows, const void* Hg, const int32_t* tg,
+                    const float* lse, const float* g, float dloss, void* dH, float* dW, int32_t* status, void* scratch,
+                    void* fwd, cudaStream_t s) {
+    if (!lm_bwd_tc_supported(d)) return MW_ESHAPE;
+    mw_status st = cuda_status(cudaMemsetAsync(dH, 0, (size_t)N * d * 2, s));
+    if (st != MW_OK) return st;
+    if (M == 0) return cuda_status(cudaMemsetAsync(dW, 0, (size_t)V * d * 4, s));
+    const int M_pad = (int)ceil_div(M, 128) * 128;
+    count_launches(1);
+    k_lm_bwd_par<<<(unsigned)ceil_div(M_pad, 256), 256, 0, s>>>(M, M_pad, g, lse, tg, dloss, (float4*)scratch);
+    if ((st = launch_status()) != MW_OK) return st;
+    LmBwdParams p = {};
+    p.mode = 1;
+    p.M = M;
+    p.V = V;
+    p.dW = dW;
+    p.status = status;
+    if ((st = launch_group(p, W, d, Hg, scratch, s)) != MW_OK) return st;
+    GrpArrays a = grp_arrays(fwd, M, d);
+    count_launches(1);
+    k_lm_dh_from_e<<<(unsigned)std::min(M, 8 * 152), 128, 0, s>>>(
+        M, d, (const __nv_bfloat16*)W, tg, a.E, a.linv, g, dloss, rows, (__nv_bfloat16*)dH);
     return launch_status();
 }
 

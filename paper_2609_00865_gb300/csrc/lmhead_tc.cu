@@ -1,18 +1,24 @@
-// Tensor-core fused LM-head log-prob (bf16 in, fp32 accumulate): no logits
-// tensor is stored.
+// Tensor-core LM-head row maxima over a vocabulary range (bf16 in, fp32
+// accumulate): the reference prepass of the fused forward. No logits tensor
+// is stored.
 //
 //   gather   Hg[m] = H[rows[m]] (bf16, zero-padded to a multiple of 128 rows),
 //            tg[m] = targets[rows[m]]
-//   forward  persistent CTAs over (vocab chunk, 128-row tile) items; per item
+//   partials persistent CTAs over (vocab chunk, 128-row tile) items; per item
 //            the chunk's 256-wide vocab tiles are computed as
 //            Z = Hg_tile W_tile^T with tcgen05.mma into one of two TMEM
 //            accumulators (128 x 256 fp32 each) fed by a 4-stage TMA ring, while
 //            four epilogue warps fold the previous tile into a running
 //            (max, sum 2^(z log2 e - max)) per row and pick out the target
 //            logit. Each item writes one (max, sum) partial per row.
-//   combine  lse = ln 2 (M + log2 sum_c l_c 2^(m_c - M)), lp = z_target - lse.
+//   k_lm_ref the row's reference: the largest of its partial maxima.
 // Concurrent CTAs work on the same vocab chunk, so each W tile is read from
 // HBM about once per wave and shared through L2.
+//
+// The training path runs this only over the first kRefVocab vocabulary
+// entries (lm_ref_tc): the row maxima there are the fixed per-row references
+// of the fused forward in lmhead_bwd_tc.cu, which computes the log-softmax
+// over the whole vocabulary.
 
 #include <math.h>
 
@@ -34,6 +40,8 @@ constexpr uint32_t ST_B = A_B + B_B;
 constexpr int NSTAGE = 4;
 constexpr uint32_t SMEM_LMF = NSTAGE * ST_B + 1024;
 constexpr float LOG2E_F = 1.4426950408889634f;
+// vocabulary entries whose row maxima serve as the fused forward's references
+constexpr int kRefVocab = 2048;
 
 struct LmFwdParams {
     int M, M_pad, d, V;
@@ -213,20 +221,19 @@ __global__ void k_lm_gather(int M, int M_pad, int d, const __nv_bfloat16* __rest
     }
 }
 
-__global__ void k_lm_combine(int M, int M_pad, int C, const float2* __restrict__ part, const float* __restrict__ zt,
-                             float* __restrict__ lse, float* __restrict__ lp) {
+// par[m] = (0, ref, target bits, 0): ref = the row's largest logit over the
+// vocabulary subset, in log2 units (max over the chunk partials); padded rows
+// (m >= M) get ref 0 and target -1.
+__global__ void k_lm_ref(int M, int M_pad, int C, const float2* __restrict__ part, const int32_t* __restrict__ tg,
+                         float4* __restrict__ par) {
     const int m = blockIdx.x * blockDim.x + threadIdx.x;
-    if (m >= M) return;
-    float mx = -INFINITY;
-    for (int c = 0; c < C; ++c) mx = fmaxf(mx, part[(int64_t)c * M_pad + m].x);
-    float l = 0.f;
-    for (int c = 0; c < C; ++c) {
-        const float2 q = part[(int64_t)c * M_pad + m];
-        if (q.y > 0.f) l += q.y * exp2f(q.x - mx);
+    if (m >= M_pad) return;
+    float mx = 0.f;
+    if (m < M) {
+        mx = -INFINITY;
+        for (int c = 0; c < C; ++c) mx = fmaxf(mx, part[(int64_t)c * M_pad + m].x);
     }
-    const float v = (mx + log2f(l)) * 0.6931471805599453f;
-    lse[m] = v;
-    lp[m] = zt[m] - v;
+    par[m] = make_float4(0.f, mx, __int_as_float(m < M ? tg[m] : -1), 0.f);
 }
 
 }  // namespace
@@ -263,15 +270,11 @@ LmPlan lm_plan(int M, int V) {
     return q;
 }
 
-mw_status lm_fwd_tc(const void* H, const void* W, const int32_t* targets, const int32_t* rows, int M, int d, int V,
-                    void* Hg, int32_t* tg, float2* part, float* zt, float* lse, float* lp, int32_t* status,
-                    cudaStream_t s) {
-    if (M == 0) return MW_OK;
-    const LmPlan q = lm_plan(M, V);
-    count_launches(3);
-    const int64_t vec = (int64_t)q.M_pad * (d / 8);
-    k_lm_gather<<<(unsigned)std::min<int64_t>(ceil_div(vec, 256), 152 * 32), 256, 0, s>>>(
-        M, q.M_pad, d, (const __nv_bfloat16*)H, targets, rows, (__nv_bfloat16*)Hg, tg);
+// Forward partials of the loss rows against vocabulary entries [0, V): the
+// gathered rows (Hg, tg) must already be in place.
+static mw_status lm_partials(const void* W, int M, int d, int V, const void* Hg, const int32_t* tg, float2* part,
+                             float* zt, int32_t* status, cudaStream_t s, LmPlan& q) {
+    q = lm_plan(M, V);
     CUtensorMap ta, tb;
     if (!tmap_bf16_2d(&ta, Hg, q.M_pad, d, d, BM, BK) || !tmap_bf16_2d(&tb, W, V, d, d, BN, BK)) return MW_ECUDA;
     LmFwdParams p;
@@ -292,8 +295,32 @@ mw_status lm_fwd_tc(const void* H, const void* W, const int32_t* targets, const 
     mw_status st = cuda_status(cudaFuncSetAttribute(k_lm_fwd_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                     (int)SMEM_LMF));
     if (st != MW_OK) return st;
+    count_launches(1);
     k_lm_fwd_tc<<<q.grid, NT, SMEM_LMF, s>>>(ta, tb, p);
-    k_lm_combine<<<(unsigned)ceil_div(M, 256), 256, 0, s>>>(M, q.M_pad, q.C, part, zt, lse, lp);
+    return launch_status();
+}
+
+static mw_status lm_gather(const void* H, const int32_t* targets, const int32_t* rows, int M, int d, void* Hg,
+                           int32_t* tg, cudaStream_t s) {
+    const int64_t M_pad = ceil_div(M, BM) * BM;
+    const int64_t vec = M_pad * (d / 8);
+    count_launches(1);
+    k_lm_gather<<<(unsigned)std::min<int64_t>(ceil_div(vec, 256), 152 * 32), 256, 0, s>>>(
+        M, (int)M_pad, d, (const __nv_bfloat16*)H, targets, rows, (__nv_bfloat16*)Hg, tg);
+    return launch_status();
+}
+
+int lm_ref_vocab(int V) { return std::min(V, kRefVocab); }
+
+mw_status lm_ref_tc(const void* H, const void* W, const int32_t* targets, const int32_t* rows, int M, int d, int V,
+                    void* Hg, int32_t* tg, float2* part, float* zt, float4* par, int32_t* status, cudaStream_t s) {
+    if (M == 0) return MW_OK;
+    mw_status st = lm_gather(H, targets, rows, M, d, Hg, tg, s);
+    LmPlan q;
+    if (st == MW_OK) st = lm_partials(W, M, d, lm_ref_vocab(V), Hg, tg, part, zt, status, s, q);
+    if (st != MW_OK) return st;
+    count_launches(1);
+    k_lm_ref<<<(unsigned)ceil_div(q.M_pad, 256), 256, 0, s>>>(M, q.M_pad, q.C, part, tg, par);
     return launch_status();
 }
 

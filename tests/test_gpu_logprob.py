@@ -189,3 +189,33 @@ def test_config3_full_size_sampled():
     vocab = np.unique(np.concatenate([rng.integers(0, V, 40), t_np[rows[:8]], [0, V - 1]]))
     dWr = OL.logprob_loss_bwd_vocab(H64, W64, t_np, rows, lse_ref, g_r, vocab)
     assert_grad_bf16(np64(dW)[vocab], dWr, "dW (sampled vocab rows)")
+
+
+@pytest.mark.parametrize("d", [256, 1536])
+def test_logits_far_above_the_reference_are_repaired(d):
+    """The bf16 forward measures each row's logits against a fixed reference,
+    its largest logit over the first vocabulary entries; a logit more than
+    2^96 (66 nats) above it flags the row, which is recomputed exactly. Here
+    a third of the rows have one late vocabulary entry (id 4000, past the
+    reference range) about 128 nats above all others, some of them as their
+    target: lp, the loss, dH and dW must still match the oracle."""
+    N, V = 300, 5003
+    H = synth.normal((N, d), 91).to(torch.bfloat16)
+    W = synth.normal((V, d), 92, std=0.02)
+    sign = torch.sign(synth.normal((d,), 93))
+    sign[sign == 0] = 1.0
+    peaked = torch.arange(0, N, 3)
+    H[peaked] = sign.to(torch.bfloat16)                 # rows aligned with W[4000]
+    W[4000] = 0.5 * sign * (256.0 / d)                   # logit 128 for those rows
+    W = W.to(torch.bfloat16)
+    targets = synth.uniform_int(N, V, 94)
+    targets[peaked[::2]] = 4000
+    rows = np.arange(0, N, 1)
+    M = len(rows)
+    lp_ref, lse_ref = OL.logprob(np64(H), np64(W), targets.numpy(), rows)
+    assert lse_ref[peaked.numpy()].min() > 127.0
+    adv = synth.normal((M,), 95)
+    lp_old = torch.tensor(lp_ref + 0.05 * np.random.default_rng(96).standard_normal(M), dtype=torch.float32)
+    r = torch.tensor(rows, dtype=torch.int32)
+    out, dH, dW = _run(H, W, targets, r, lp_old, adv, 0.2, 0.28)
+    _check(H, W, targets, r, lp_old, adv, lp_ref, lse_ref, out, dH, dW, 0.2, 0.28, fp32=False)
