@@ -273,7 +273,9 @@ class Step:
                 self.table = mw.rope_table(mw.TILE * self.L.max_tiles, Dh, w["rope"], device=device)
                 nb = mw.mw_masked_attn_rope_ws(self.vis, Hq, Hkv, Dh, mw.MW_BF16)[1]
             else:
-                nb = mw.mw_masked_attn_bwd_ws(self.vis, Hq, Dh, mw.MW_BF16)
+                nb = mw.mw_masked_attn_bwd_ws(self.vis, Hq, Hkv, Dh, mw.MW_BF16)
+                nf = mw.mw_masked_attn_fwd_ws(self.vis, Hkv, Dh, mw.MW_BF16)
+                self.attn_fwd_ws = torch.empty(max(nf, 1), dtype=torch.uint8, device=device)
             self.attn_ws = torch.empty(max(nb, 1), dtype=torch.uint8, device=device)
         if "rows" in w:
             M = int(w["rows"].numel())
@@ -329,7 +331,8 @@ class Step:
                 self.scale, self.attn_ws, self.stream))
             return
         self._ev("mw_masked_attn_fwd", lambda: self.mw.mw_masked_attn_fwd(
-            self.vis, self.d["Q"], self.d["K"], self.d["V"], self.O, self.LSE, self.scale, self.stream))
+            self.vis, self.d["Q"], self.d["K"], self.d["V"], self.O, self.LSE, self.scale, self.attn_fwd_ws,
+            self.stream))
 
     def attn_bwd(self, dO):
         if "rope" in self.w:

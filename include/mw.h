@@ -117,6 +117,13 @@ typedef struct mw_vis_layout {
     int64_t ws_off_cnt;     /* int32 [2][n_tiles] fwd / bwd list lengths */
     int64_t ws_bytes;
     int64_t max_segs;       /* max over trajectories of 1 + K_b (segments per trajectory) */
+    /* --- compact views (in `vis`; byte offsets). Segment s of trajectory b
+     * owns the 128 nt_b entries starting at (traj_km[b] + s nt_b) 128, the
+     * same indexing as the keymask entries times 128. --- */
+    int64_t off_seg_len;    /* int32 [n_segs] |view_s|, the length of each segment's compact sequence */
+    int64_t off_cpos;       /* int32 [n_keymask][128] rank of key j in view_s (the compact index), -1 if absent */
+    int64_t off_csrc;       /* int32 [n_keymask][128] key (traj-local) at compact index c of view_s;
+                               -1 from |view_s| to the end of its last 128-entry tile, unset after */
 } mw_vis_layout;
 
 /*
@@ -173,29 +180,42 @@ mw_status mw_build_visibility_noalloc(const mw_vis_layout* layout, const int32_t
                                       const int32_t* junc_span_off, const int32_t* spans,
                                       void* vis, void* stream);
 
+/* Bytes of device workspace mw_masked_attn_fwd needs for these sizes (0 for
+ * the fp32 path). bf16 with Dh 128: the compact K and V, 2 x 2 bytes per
+ * element of [128 n_keymask, Hkv, Dh]. */
+mw_status mw_masked_attn_fwd_ws(const mw_vis_layout* layout, int Hkv, int Dh, int dtype, size_t* ws_bytes);
+
 /*
  * Eviction-aware masked GQA attention forward (§4.2 mask; §4.3 equivalence).
  *   Q, O  [total_tokens, Hq, Dh]   K, V [total_tokens, Hkv, Dh]   (dtype)
  *   LSE   [Hq, total_tokens] float32, natural-log row log-sum-exp (saved for bwd)
  *   O_i = sum_{j visible} softmax_j(scale q_i . k_j) v_j;  q-head h reads
- *   kv-head h / (Hq / Hkv). Only non-EMPTY tiles are visited.
+ *   kv-head h / (Hq / Hkv).
  * dtype MW_BF16 requires Dh == 128 (tensor-core path); MW_F32 accepts Dh 64
- * or 128 (exact-fp32 SIMT path). Hq % Hkv == 0.
+ * or 128 (exact-fp32 SIMT path, which visits the non-EMPTY tiles of the
+ * lists). Hq % Hkv == 0.
+ * The bf16 path gathers each segment's live view into its compact sequence
+ * (the segment's view_s in order, as §4.1 materialises a branch; the compact
+ * maps of `vis`) in `ws` (mw_masked_attn_fwd_ws bytes, device, overwritten)
+ * and runs causal attention of the segment's rows over it; a q-tile holding
+ * rows of several segments is computed once per segment.
  */
 mw_status mw_masked_attn_fwd(const mw_vis_layout* layout, const void* vis,
                              const void* Q, const void* K, const void* V, void* O, float* LSE,
-                             int Hq, int Hkv, int Dh, int dtype, float scale, void* stream);
+                             int Hq, int Hkv, int Dh, int dtype, float scale, void* ws, void* stream);
 
 /* Bytes of device workspace mw_masked_attn_bwd needs for these sizes. */
-mw_status mw_masked_attn_bwd_ws(const mw_vis_layout* layout, int Hq, int Dh, int dtype,
+mw_status mw_masked_attn_bwd_ws(const mw_vis_layout* layout, int Hq, int Hkv, int Dh, int dtype,
                                 size_t* ws_bytes);
 
 /*
  * Backward of mw_masked_attn_fwd for upstream dO (same layout as O).
  * Writes dQ (like Q), dK, dV (like K, V), all in `dtype`, overwriting them.
- * Delta_i = rowsum(dO_i * O_i) (for bf16 with Dh 128: the pair (LSE_i log2 e,
- * Delta_i) per row, rows padded to whole 128-row tiles) lives in `ws`
- * (mw_masked_attn_bwd_ws bytes).
+ * `ws` (mw_masked_attn_bwd_ws bytes, device, overwritten) holds Delta_i =
+ * rowsum(dO_i * O_i); for bf16 with Dh 128 the pair (-LSE_i log2 e, Delta_i)
+ * per row (rows padded to whole 128-row tiles), the compact K and V, and
+ * float32 dK / dV partials per compact row, which are summed per key in
+ * segment order (deterministic; no atomics).
  */
 mw_status mw_masked_attn_bwd(const mw_vis_layout* layout, const void* vis,
                              const void* Q, const void* K, const void* V, const void* O,

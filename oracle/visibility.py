@@ -258,10 +258,18 @@ def build(seqlens, edits_per_traj, tile=TILE):
     ``bwd_ptr``/``bwd_idx``  per global k-tile, ascending non-empty q-tiles
     ``pairs`` int64 [n_traj], ``pairs_total`` int
     ``keymask`` uint32 [sum_b S_b * nt_b, 4] (per trajectory: segment-major)
+    ``seg_len`` int32 [n_segs]  length of each segment's live view (its compact sequence)
+    ``cpos``  int32 [sum_b S_b * nt_b * 128] rank of key j in view_s (``logical_positions``,
+              -1 if absent), entry ``(km_b + s nt_b) 128 + j`` with km_b the trajectory's
+              first keymask entry
+    ``csrc``  int32, same indexing by rank c: the key at index c of the list view_s,
+              -1 from ``len(view_s)`` to the end of its last 128-entry tile, -2 after
+              (left unspecified)
     """
     omega, seg, qtraj, classes = [], [], [], []
     fwd_ptr, fwd_idx, bwd_ptr, bwd_idx = [0], [], [0], []
     pairs, keymask = [], []
+    seg_len, cpos, csrc = [], [], []
     for b, (T, edits) in enumerate(zip(seqlens, edits_per_traj)):
         cls, counts = tile_classes(T, edits, tile)
         cls = cls | dead_halves(T, edits, cls, tile)
@@ -284,6 +292,17 @@ def build(seqlens, edits_per_traj, tile=TILE):
         bwd_ptr.extend((bwd_ptr[-1] + np.cumsum(np.bincount(k_nz2, minlength=nt))).tolist())
         pairs.append(int(counts.sum()))
         keymask.append(segment_keymask(T, edits, tile).reshape(-1, tile // 32))
+        lp = logical_positions(T, edits)
+        for s, (_, _, view) in enumerate(live_views(T, edits)):
+            seg_len.append(len(view))
+            pos = np.full(nt * tile, -1, dtype=np.int64)
+            pos[:T] = lp[s]
+            cpos.append(pos)
+            src = np.full(nt * tile, -2, dtype=np.int64)
+            src[: -(-len(view) // tile) * tile] = -1
+            src[: len(view)] = view
+            csrc.append(src)
+    cat = (lambda xs: np.concatenate(xs).astype(np.int32)) if cpos else (lambda xs: np.zeros(0, np.int32))
     return {
         "omega": np.concatenate(omega),
         "seg": np.concatenate(seg),
@@ -296,4 +315,7 @@ def build(seqlens, edits_per_traj, tile=TILE):
         "pairs": np.asarray(pairs, dtype=np.int64),
         "pairs_total": int(sum(pairs)),
         "keymask": np.concatenate(keymask) if keymask else np.zeros((0, tile // 32), np.uint32),
+        "seg_len": np.asarray(seg_len, dtype=np.int32),
+        "cpos": cat(cpos),
+        "csrc": cat(csrc),
     }

@@ -35,7 +35,8 @@ class VisLayout(ctypes.Structure):
                    "off_traj_tri", "off_traj_km", "off_seg_start", "off_tile_traj", "off_cls",
                    "off_fwd_ptr", "off_fwd_idx", "off_bwd_ptr", "off_bwd_idx", "off_pairs",
                    "off_keymask", "off_status", "vis_bytes",
-                   "ws_off_spans", "ws_off_tstat", "ws_off_cnt", "ws_bytes", "max_segs")]
+                   "ws_off_spans", "ws_off_tstat", "ws_off_cnt", "ws_bytes", "max_segs",
+                   "off_seg_len", "off_cpos", "off_csrc")]
 
 
 _P = ctypes.c_void_p
@@ -52,8 +53,9 @@ _SIGS = {
     "mw_visibility_layout": (_I, [_I, _IP, _I, _IP, _I, _LP]),
     "mw_build_visibility": (_I, [_LP, _IP, _I, _IP, _IP, _IP, _IP, _P, _P, _P]),
     "mw_build_visibility_noalloc": (_I, [_LP, _IP, _I, _IP, _IP, _IP, _IP, _P, _P]),
-    "mw_masked_attn_fwd": (_I, [_LP, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _F, _P]),
-    "mw_masked_attn_bwd_ws": (_I, [_LP, _I, _I, _I, ctypes.POINTER(ctypes.c_size_t)]),
+    "mw_masked_attn_fwd_ws": (_I, [_LP, _I, _I, _I, ctypes.POINTER(ctypes.c_size_t)]),
+    "mw_masked_attn_fwd": (_I, [_LP, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _F, _P, _P]),
+    "mw_masked_attn_bwd_ws": (_I, [_LP, _I, _I, _I, _I, ctypes.POINTER(ctypes.c_size_t)]),
     "mw_masked_attn_bwd": (_I, [_LP, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _F, _P, _P]),
     "mw_logprob_ws": (_I, [_I, _I, _I, _I, _I, ctypes.POINTER(ctypes.c_size_t)]),
     "mw_logprob_loss_fwd": (_I, [_P, _P, _P, _P, _I, _P, _P, _F, _F, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P]),
@@ -238,6 +240,9 @@ class Visibility:
             "pairs_total": int(pairs[-1]),
             "keymask": self._arr(L.off_keymask, L.n_keymask * 4, np.uint32).reshape(-1, 4),
             "traj_tok": tok,
+            "seg_len": self._arr(L.off_seg_len, L.n_segs, np.int32),
+            "cpos": self._arr(L.off_cpos, L.n_keymask * TILE, np.int32),
+            "csrc": self._arr(L.off_csrc, L.n_keymask * TILE, np.int32),
         }
 
     @property
@@ -263,29 +268,40 @@ def build_visibility(seqlens, edits_per_traj, device="cuda", stream=None):
 
 # --- attention ----------------------------------------------------------------
 
-def mw_masked_attn_fwd(vis, Q, K, V, O, LSE, scale, stream=None):
+def mw_masked_attn_fwd_ws(vis, Hkv, Dh, dtype):
+    n = ctypes.c_size_t()
+    _check(_lib().mw_masked_attn_fwd_ws(ctypes.byref(vis.layout), Hkv, Dh, dtype, ctypes.byref(n)),
+           "mw_masked_attn_fwd_ws")
+    return int(n.value)
+
+
+def mw_masked_attn_fwd(vis, Q, K, V, O, LSE, scale, ws, stream=None):
     Hq, Dh = Q.shape[1], Q.shape[2]
     Hkv = K.shape[1]
     _check(_lib().mw_masked_attn_fwd(ctypes.byref(vis.layout), _ptr(vis.vis), _ptr(Q), _ptr(K), _ptr(V),
                                      _ptr(O), _ptr(LSE), Hq, Hkv, Dh, _dtype_code(Q), float(scale),
-                                     _stream(stream)), "mw_masked_attn_fwd")
+                                     _ptr(ws), _stream(stream)), "mw_masked_attn_fwd")
 
 
-def masked_attn_fwd(vis, Q, K, V, scale=None, stream=None):
-    """Allocate O [T, Hq, Dh] and LSE [Hq, T] and run the forward."""
+def masked_attn_fwd(vis, Q, K, V, scale=None, ws=None, stream=None):
+    """Allocate O [T, Hq, Dh] and LSE [Hq, T] (and the workspace) and run the
+    forward."""
     import torch
     for t, n in ((Q, "Q"), (K, "K"), (V, "V")):
         _need(t, n, dtype=Q.dtype)
     scale = float(Q.shape[2]) ** -0.5 if scale is None else scale
+    if ws is None:
+        nbytes = mw_masked_attn_fwd_ws(vis, K.shape[1], Q.shape[2], _dtype_code(Q))
+        ws = torch.empty(max(nbytes, 1), dtype=torch.uint8, device=Q.device)
     O = torch.empty_like(Q)
     LSE = torch.empty(Q.shape[1], Q.shape[0], dtype=torch.float32, device=Q.device)
-    mw_masked_attn_fwd(vis, Q, K, V, O, LSE, scale, stream)
+    mw_masked_attn_fwd(vis, Q, K, V, O, LSE, scale, ws, stream)
     return O, LSE
 
 
-def mw_masked_attn_bwd_ws(vis, Hq, Dh, dtype):
+def mw_masked_attn_bwd_ws(vis, Hq, Hkv, Dh, dtype):
     n = ctypes.c_size_t()
-    _check(_lib().mw_masked_attn_bwd_ws(ctypes.byref(vis.layout), Hq, Dh, dtype, ctypes.byref(n)),
+    _check(_lib().mw_masked_attn_bwd_ws(ctypes.byref(vis.layout), Hq, Hkv, Dh, dtype, ctypes.byref(n)),
            "mw_masked_attn_bwd_ws")
     return int(n.value)
 
@@ -307,7 +323,7 @@ def masked_attn_bwd(vis, Q, K, V, O, dO, LSE, scale=None, ws=None, stream=None):
     _need(LSE, "LSE", dtype=torch.float32)
     scale = float(Q.shape[2]) ** -0.5 if scale is None else scale
     if ws is None:
-        nbytes = mw_masked_attn_bwd_ws(vis, Q.shape[1], Q.shape[2], _dtype_code(Q))
+        nbytes = mw_masked_attn_bwd_ws(vis, Q.shape[1], K.shape[1], Q.shape[2], _dtype_code(Q))
         ws = torch.empty(max(nbytes, 1), dtype=torch.uint8, device=Q.device)
     dQ, dK, dV = torch.empty_like(Q), torch.empty_like(K), torch.empty_like(V)
     mw_masked_attn_bwd(vis, Q, K, V, O, dO, LSE, dQ, dK, dV, scale, ws, stream)

@@ -17,10 +17,12 @@ mw_status lm_fwd_simt(const void*, const void*, const int32_t*, const int32_t*, 
 mw_status lm_bwd_simt(const void*, const void*, const int32_t*, const int32_t*, int, int, int, int, int,
                       const float*, const float*, float, void*, float*, cudaStream_t);
 mw_status attn_fwd_tc(const mw_vis_layout*, const void*, const void*, const void*, const void*, void*, float*, int,
-                      int, float, cudaStream_t);
+                      int, float, void*, cudaStream_t);
 mw_status attn_bwd_tc(const mw_vis_layout*, const void*, const void*, const void*, const void*, const void*,
-                      const void*, const float*, void*, void*, void*, int, int, float, float*, cudaStream_t);
-int64_t attn_bwd_tc_ws(const mw_vis_layout*, int);
+                      const void*, const float*, void*, void*, void*, int, int, float, void*, cudaStream_t);
+int64_t attn_fwd_tc_ws(const mw_vis_layout*, int);
+int64_t attn_bwd_tc_ws(const mw_vis_layout*, int, int);
+int64_t attn_lsd_ws(const mw_vis_layout*, int);
 mw_status attn_delta(const mw_vis_layout*, const void*, const void*, int, int, int, float*, cudaStream_t);
 mw_status attn_fwd_simt_segk(const mw_vis_layout*, const void*, const void*, const void*, const void*, void*, float*,
                              int, int, int, int, float, cudaStream_t);
@@ -100,22 +102,33 @@ static mw_status attn_args(const mw_vis_layout* L, const void* vis, int Hq, int 
 
 using namespace mw;
 
+extern "C" mw_status mw_masked_attn_fwd_ws(const mw_vis_layout* L, int Hkv, int Dh, int dtype, size_t* bytes) {
+    if (!L || !bytes) return MW_EINVAL;
+    if (Hkv <= 0) return MW_ESHAPE;
+    *bytes = dtype == MW_BF16 && Dh == 128 ? (size_t)attn_fwd_tc_ws(L, Hkv) : 0;
+    return MW_OK;
+}
+
 extern "C" mw_status mw_masked_attn_fwd(const mw_vis_layout* L, const void* vis, const void* Q, const void* K,
                                         const void* V, void* O, float* LSE, int Hq, int Hkv, int Dh, int dtype,
-                                        float scale, void* stream) {
+                                        float scale, void* ws, void* stream) {
     mw_status st = attn_args(L, vis, Hq, Hkv, Dh, dtype, scale);
     if (st != MW_OK) return st;
     if (L->total_tokens == 0) return MW_OK;
     if (!Q || !K || !V || !O || !LSE) return MW_EINVAL;
-    if (dtype == MW_BF16 && Dh == 128)
-        return attn_fwd_tc(L, vis, Q, K, V, O, LSE, Hq, Hkv, scale, (cudaStream_t)stream);
+    if (dtype == MW_BF16 && Dh == 128) {
+        if (!ws) return MW_EINVAL;
+        return attn_fwd_tc(L, vis, Q, K, V, O, LSE, Hq, Hkv, scale, ws, (cudaStream_t)stream);
+    }
     return attn_fwd_simt(L, vis, Q, K, V, O, LSE, Hq, Hkv, Dh, dtype, scale, (cudaStream_t)stream);
 }
 
-extern "C" mw_status mw_masked_attn_bwd_ws(const mw_vis_layout* L, int Hq, int Dh, int dtype, size_t* bytes) {
+extern "C" mw_status mw_masked_attn_bwd_ws(const mw_vis_layout* L, int Hq, int Hkv, int Dh, int dtype,
+                                           size_t* bytes) {
     if (!L || !bytes) return MW_EINVAL;
+    if (Hq <= 0 || Hkv <= 0) return MW_ESHAPE;
     int64_t b = 4 * L->total_tokens * (int64_t)Hq;   // Delta per (head, row)
-    if (dtype == MW_BF16 && Dh == 128) b = std::max(b, attn_bwd_tc_ws(L, Hq));
+    if (dtype == MW_BF16 && Dh == 128) b = std::max(b, attn_bwd_tc_ws(L, Hq, Hkv));
     *bytes = (size_t)align256(b);
     return MW_OK;
 }
@@ -129,7 +142,7 @@ extern "C" mw_status mw_masked_attn_bwd(const mw_vis_layout* L, const void* vis,
     if (L->total_tokens == 0) return MW_OK;
     if (!Q || !K || !V || !O || !dO || !LSE || !dQ || !dK || !dV || !ws) return MW_EINVAL;
     if (dtype == MW_BF16 && Dh == 128)
-        return attn_bwd_tc(L, vis, Q, K, V, O, dO, LSE, dQ, dK, dV, Hq, Hkv, scale, (float*)ws, (cudaStream_t)stream);
+        return attn_bwd_tc(L, vis, Q, K, V, O, dO, LSE, dQ, dK, dV, Hq, Hkv, scale, ws, (cudaStream_t)stream);
     return attn_bwd_simt(L, vis, Q, K, V, O, dO, LSE, dQ, dK, dV, Hq, Hkv, Dh, dtype, scale, (float*)ws,
                          (cudaStream_t)stream);
 }
@@ -260,7 +273,7 @@ static RopeWs rope_ws_layout(const mw_vis_layout* L, int Hq, int Hkv, int Dh, in
     w.q = o; o = align256(o + esz * L->total_tokens * Hq * Dh);
     w.kseg = o; o = align256(o + esz * krows * Hkv * Dh);
     w.fwd_bytes = o;
-    w.delta = o; o = align256(o + (tc ? attn_bwd_tc_ws(L, Hq) : 4 * L->total_tokens * Hq));
+    w.delta = o; o = align256(o + (tc ? attn_lsd_ws(L, Hq) : 4 * L->total_tokens * Hq));
     w.dkseg = o; o = align256(o + 4 * krows * Hkv * Dh);
     w.dvseg = o; o = align256(o + (tc ? 4 * krows * Hkv * Dh : 0));
     w.bwd_bytes = o;

@@ -1,5 +1,17 @@
 // Tensor-core masked GQA attention, bf16 in / fp32 accumulate, head dim 128.
 //
+// The plain path (MODE 2, "compact") scores each segment's rows against that
+// segment's compact sequence -- its live view gathered in order (§4.1's
+// materialised branch; the builder's csrc / cpos maps), so that a row's keys
+// are a prefix of it: tiles are FULL or hold a per-row prefix, and the
+// evicted keys inside a physical tile cost nothing. Per q-tile item the keys
+// are compact tiles 0 .. (last row's index) / 128; dK / dV run per (compact
+// key tile, segment) into float32 partials per compact row, summed per key
+// in segment order (k_cmp_reduce). This is the same 4D-masked computation
+// (§4.3 Theorem "materialization equivalence"): every row still reads each
+// visible key once.
+//
+// The rotary path (MODE 1, below) keeps physical key tiles:
 // Mask (§4.2): key j is visible to row i iff j <= i < omega(j). A tile's
 // class comes from the visibility builder: EMPTY tiles are never listed,
 // FULL tiles run unmasked, PARTIAL and diagonal tiles apply the row's
@@ -120,6 +132,50 @@ __device__ __forceinline__ QItem q_item(const VisView& v, int Hq, int max_tiles,
     return it;
 }
 
+// Compact mode (MODE 2): keys come from each segment's compact sequence
+// (view_s gathered in order, §4.1 LogitTree), stored at rows
+// (traj_km[b] + s nt) 128 + c of a compact K / V buffer. A q-tile item serves
+// the rows of one segment, whose compact index is nb + (i - seg_lo) with nb
+// the keys of view_s before the segment's own rows; row i sees compact keys
+// 0 .. its own index, so a compact tile is FULL (every row of a whole tile
+// sees every key), or PARTIAL with a prefix of keys visible to each row
+// (DEAD_HI when no row reaches its second half).
+struct CPiece {
+    int r0, r1;          // the item's rows (trajectory-local) [r0, r1)
+    int seg_lo, nb;      // first row of the segment; keys of view_s before it
+    int cfirst, clast;   // compact indices of rows r0 and r1 - 1
+    bool whole;          // the item covers all 128 rows of its q-tile
+};
+__device__ __forceinline__ CPiece cmp_piece(const VisView& v, int b, int s, int qt, int T) {
+    CPiece c;
+    const int gs = v.traj_seg[b] + s;
+    const int nseg = v.traj_seg[b + 1] - v.traj_seg[b];
+    c.seg_lo = v.seg_start[gs];
+    const int seg_hi = s + 1 < nseg ? v.seg_start[gs + 1] : T;
+    c.nb = v.seg_len[gs] - (seg_hi - c.seg_lo);
+    c.r0 = max(c.seg_lo, qt * 128);
+    c.r1 = min(seg_hi, qt * 128 + 128);
+    c.cfirst = c.nb + c.r0 - c.seg_lo;
+    c.clast = c.nb + c.r1 - 1 - c.seg_lo;
+    c.whole = c.r0 == qt * 128 && c.r1 == qt * 128 + 128;
+    return c;
+}
+// list entry (tile << 4) | code of compact key tile j for a piece
+__device__ __forceinline__ int cmp_entry(const CPiece& c, int j) {
+    if (c.whole && j * 128 + 127 <= c.cfirst) return (j << 4) | MW_TILE_FULL;
+    return (j << 4) | MW_TILE_PARTIAL | (c.clast - j * 128 < 64 ? MW_TILE_DEAD_HI : 0);
+}
+// 128-bit mask with keys 0 .. lim set (none for lim < 0)
+__device__ __forceinline__ uint4 prefix_words(int lim) {
+    uint32_t w[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const int hi = lim - 32 * q;
+        w[q] = hi >= 31 ? 0xffffffffu : (hi < 0 ? 0u : ((2u << hi) - 1u));
+    }
+    return make_uint4(w[0], w[1], w[2], w[3]);
+}
+
 __device__ __forceinline__ float ex2(float x) {
     float y;
     asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
@@ -160,20 +216,21 @@ __device__ __forceinline__ uint64_t mnmaj(uint32_t base, int ks) {
     return sdesc_sw128(base + ks * 2048, HALF_B, 1024);
 }
 
-template <bool SEGK>
+template <int MODE>
 __global__ void __launch_bounds__(NT_FWD, 1)
     k_attn_fwd_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                   const __grid_constant__ CUtensorMap tmV, FwdParams p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~uintptr_t(1023));
     __shared__ __align__(8) uint64_t q_full, k_full[2], k_empty[2], v_full[2], v_empty[2], s_full[2], s_free[2],
-        p_full[2], o_done;
+        p_full[2], o_done, o_fin;
     __shared__ uint32_t tmem_base;
     __shared__ int abort_flag;
 
+    constexpr bool SEGK = MODE == 1, CMP = MODE == 2;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const VisView& v = p.v;
-    const QItem it = q_item<SEGK>(v, p.Hq, p.max_tiles, p.n_traj, p.junction_items);
+    const QItem it = q_item<MODE != 0>(v, p.Hq, p.max_tiles, p.n_traj, p.junction_items);
     if (!it.ok) return;
     const int h = it.h, qt = it.qt, b = it.b;
     const int nt = v.traj_tile[b + 1] - v.traj_tile[b];
@@ -181,8 +238,11 @@ __global__ void __launch_bounds__(NT_FWD, 1)
     const int64_t tok0 = v.traj_tok[b];
     const int T = v.traj_tok[b + 1] - (int)tok0;
     const int kvh = h / (p.Hq / p.Hkv);
-    const int p0 = v.fwd_ptr[g];
-    const int n = v.fwd_ptr[g + 1] - p0;
+    CPiece cp{};
+    if (CMP) cp = cmp_piece(v, b, it.s, qt, T);
+    const int p0 = CMP ? 0 : v.fwd_ptr[g];
+    const int n = CMP ? cp.clast / 128 + 1 : v.fwd_ptr[g + 1] - p0;
+    auto entry = [&](int j) -> int { return CMP ? cmp_entry(cp, j) : v.fwd_idx[p0 + j]; };
     int32_t* status = v.status;
 
     if (threadIdx.x == 0) {
@@ -197,6 +257,7 @@ __global__ void __launch_bounds__(NT_FWD, 1)
             mbar_init(&p_full[s], 128);   // per S buffer
         }
         mbar_init(&o_done, 1);
+        mbar_init(&o_fin, 1);   // one phase: the last PV's completion
         abort_flag = 0;
         fence_mbar_init();
     }
@@ -217,12 +278,13 @@ __global__ void __launch_bounds__(NT_FWD, 1)
             prefetch_tmap(&tmV);
             mbar_expect_tx(&q_full, TILE_B);
             load_tile(sm + SM_Q, &tmQ, &q_full, h, (int)(tok0 + qt * 128));
-            // first K row of the trajectory (SEGK: of the item's segment key rows)
-            const int64_t krow0 = SEGK ? (v.traj_km[b] + (int64_t)it.s * nt) * 128 : tok0;
+            // first K row of the trajectory (SEGK: of the item's segment key
+            // rows; CMP: of the segment's compact sequence, for V as well)
+            const int64_t krow0 = MODE != 0 ? (v.traj_km[b] + (int64_t)it.s * nt) * 128 : tok0;
             for (int j = 0; j < n; ++j) {
-                const int kt = v.fwd_idx[p0 + j] >> 4;
+                const int kt = entry(j) >> 4;
                 const int s = j & 1;
-                const int row = (int)(tok0 + kt * 128);
+                const int row = (int)((CMP ? krow0 : tok0) + kt * 128);
                 if (j >= 2 && !mbar_wait(&k_empty[s], ((j - 2) >> 1) & 1, status, 101)) { abort_flag = 1; break; }
                 mbar_expect_tx(&k_full[s], TILE_B);
                 load_tile(sm + SM_K + s * TILE_B, &tmK, &k_full[s], kvh, (int)(krow0 + kt * 128));
@@ -243,7 +305,7 @@ __global__ void __launch_bounds__(NT_FWD, 1)
             // O += P_t V_t with P_t (bf16, two keys per 32-bit column) read from
             // the first 64 columns of S buffer t & 1
             auto pv = [&](int t) -> bool {
-                const int e = v.fwd_idx[p0 + t];
+                const int e = entry(t);
                 if (!mbar_wait(&p_full[t & 1], (t >> 1) & 1, status, 202)) return false;
                 if (!mbar_wait(&v_full[t & 1], (t >> 1) & 1, status, 203)) return false;
                 tc_fence_after();
@@ -263,13 +325,14 @@ __global__ void __launch_bounds__(NT_FWD, 1)
                 mma_commit(&v_empty[t & 1]);
                 mma_commit(&s_free[t & 1]);
                 mma_commit(&o_done);
+                if (t == n - 1) mma_commit(&o_fin);
                 return true;
             };
             if (warp == 1) {
                 const uint32_t iS64 = idesc_bf16(128, 64, 0, 0);   // S over one live key half
                 for (int j = 0; ok && j < n; ++j) {
                     const int s = j & 1;
-                    const int e = v.fwd_idx[p0 + j];
+                    const int e = entry(j);
                     if (!mbar_wait(&k_full[s], (j >> 1) & 1, status, 204)) { ok = false; break; }
                     if (j >= 2 && !mbar_wait(&s_free[s], ((j - 2) >> 1) & 1, status, 205)) { ok = false; break; }
                     tc_fence_after();
@@ -301,15 +364,19 @@ __global__ void __launch_bounds__(NT_FWD, 1)
         const int ie = min(i, T - 1);
         const int seg = v.seg[tok0 + ie];
         const uint4* km = reinterpret_cast<const uint4*>(v.keymask) + v.traj_km[b] + (int64_t)seg * nt;
+        // CMP: this row's compact index (rows outside the item see no key)
+        const bool in_piece = !CMP || (i >= cp.r0 && i < cp.r1);
+        const int crow = CMP ? (in_piece ? cp.cfirst + i - cp.r0 : -(1 << 30)) : 0;
+        auto mask_words = [&](int e) -> uint4 { return CMP ? prefix_words(crow - (e >> 4) * 128) : km[e >> 4]; };
         const uint32_t lane_base = tmem + ((uint32_t)(qw * 32) << 16);
         float m = -INFINITY, l = 0.f;
         bool ok = true;
         // list entries and view-mask words are loaded ahead (an entry two
         // tiles, a mask word one tile), so no step waits on a global load once
         // its S is ready
-        int e_cur = n > 0 ? v.fwd_idx[p0] : 0;
-        int e_nxt = n > 1 ? v.fwd_idx[p0 + 1] : 0;
-        uint4 w_cur = n > 0 ? km[e_cur >> 4] : make_uint4(0u, 0u, 0u, 0u);
+        int e_cur = n > 0 ? entry(0) : 0;
+        int e_nxt = n > 1 ? entry(1) : 0;
+        uint4 w_cur = n > 0 ? mask_words(e_cur) : make_uint4(0u, 0u, 0u, 0u);
         // One tile of the online softmax over NC 32-column chunks of S (4: the
         // whole tile; 2: a live key half): mask, row max, P = 2^(S c - m) into
         // the first NC * 16 columns of the buffer as bf16 pairs, row sum.
@@ -389,11 +456,12 @@ __global__ void __launch_bounds__(NT_FWD, 1)
             const int e = e_cur;
             const uint4 wv = w_cur;
             if (j + 1 < n) {
-                w_cur = km[e_nxt >> 4];
+                w_cur = mask_words(e_nxt);
                 e_cur = e_nxt;
-                e_nxt = j + 2 < n ? v.fwd_idx[p0 + j + 2] : 0;
+                e_nxt = j + 2 < n ? entry(j + 2) : 0;
             }
             const int kt = e >> 4, cls = e & 3;
+            const bool diag = !CMP && kt == qt;   // compact tiles carry causality in their mask words
             if (!mbar_wait(&s_full[j & 1], (j >> 1) & 1, status, 301)) { ok = false; break; }
             tc_fence_after();
             // a tile whose first or second key half no row sees was computed as
@@ -405,8 +473,8 @@ __global__ void __launch_bounds__(NT_FWD, 1)
                 const uint32_t w0 = lh ? wv.z : wv.x, w1 = lh ? wv.w : wv.y;
                 alpha = soft_tile(std::integral_constant<int, 2>(), sbuf, true, 127, w0, w1, 0u, 0u);
             } else {
-                alpha = soft_tile(std::integral_constant<int, 4>(), sbuf, cls != MW_TILE_FULL || kt == qt,
-                                  kt == qt ? ie - kt * 128 : 127, wv.x, wv.y, wv.z, wv.w);
+                alpha = soft_tile(std::integral_constant<int, 4>(), sbuf, cls != MW_TILE_FULL || diag,
+                                  diag ? ie - kt * 128 : 127, wv.x, wv.y, wv.z, wv.w);
             }
             // O was last written by PV_{j-1}; rescale it when the max moved
             if (j >= 1 && __any_sync(0xffffffffu, alpha != 1.f)) {
@@ -430,13 +498,16 @@ __global__ void __launch_bounds__(NT_FWD, 1)
             tc_fence_before();
             mbar_arrive(&p_full[j & 1]);
         }
-        // epilogue: O / l, LSE (natural log)
-        if (ok && n > 0 && mbar_wait(&o_done, (n - 1) & 1, status, 303)) {
+        // epilogue: O / l, LSE (natural log). The final PV is awaited on its
+        // own one-phase barrier: a parity wait on o_done for phase n - 1 would
+        // also pass while o_done is still in phase n - 2 (same parity as n),
+        // i.e. before the last two PVs have completed.
+        if (ok && n > 0 && mbar_wait(&o_fin, 0, status, 303)) {
             tc_fence_after();
             const float inv = 1.f / l;
             __nv_bfloat16* orow = p.O + ((tok0 + ie) * p.Hq + h) * DH;
             uint32_t o[32];
-            const bool store = i < T && (!SEGK || seg == it.s);
+            const bool store = CMP ? in_piece : i < T && (!SEGK || seg == it.s);
 #pragma unroll
             for (int c = 0; c < 4; ++c) {
                 tmem_ld32(lane_base + TM_O + c * 32, o);
@@ -498,19 +569,20 @@ struct BwdParams {
     float* dVseg;
 };
 
-template <bool SEGK>
+template <int MODE>
 __global__ void __launch_bounds__(NT_BWD, 1)
     k_attn_dq_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmDO,
                  const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, BwdParams p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sm = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~uintptr_t(1023));
     __shared__ __align__(8) uint64_t q_full, k_full[2], k_empty[2], v_full[2], v_empty[2], s_full[2], s_free[2],
-        dp_full, dp_free, ds_full[2], dq_done;
+        dp_full, dp_free, ds_full[2], dq_fin;
     __shared__ uint32_t tmem_base;
 
+    constexpr bool SEGK = MODE == 1, CMP = MODE == 2;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const VisView& v = p.v;
-    const QItem it = q_item<SEGK>(v, p.Hq, p.max_tiles, p.n_traj, p.junction_items);
+    const QItem it = q_item<MODE != 0>(v, p.Hq, p.max_tiles, p.n_traj, p.junction_items);
     if (!it.ok) return;
     const int h = it.h, qt = it.qt, b = it.b;
     const int nt = v.traj_tile[b + 1] - v.traj_tile[b];
@@ -518,8 +590,11 @@ __global__ void __launch_bounds__(NT_BWD, 1)
     const int64_t tok0 = v.traj_tok[b];
     const int T = v.traj_tok[b + 1] - (int)tok0;
     const int kvh = h / (p.Hq / p.Hkv);
-    const int p0 = v.fwd_ptr[g];
-    const int n = v.fwd_ptr[g + 1] - p0;
+    CPiece cp{};
+    if (CMP) cp = cmp_piece(v, b, it.s, qt, T);
+    const int p0 = CMP ? 0 : v.fwd_ptr[g];
+    const int n = CMP ? cp.clast / 128 + 1 : v.fwd_ptr[g + 1] - p0;
+    auto entry = [&](int j) -> int { return CMP ? cmp_entry(cp, j) : v.fwd_idx[p0 + j]; };
     int32_t* status = v.status;
     if (*(volatile int32_t*)&status[1]) return;
 
@@ -536,7 +611,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
         }
         mbar_init(&dp_full, 1);
         mbar_init(&dp_free, NEW);
-        mbar_init(&dq_done, 1);
+        mbar_init(&dq_fin, 1);   // one phase: the last dQ MMA's completion
         fence_mbar_init();
     }
     if (warp == 1) {
@@ -558,12 +633,13 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             mbar_expect_tx(&q_full, 2 * TILE_B);
             load_tile(sm + DQ_Q, &tmQ, &q_full, h, row0);
             load_tile(sm + DQ_DO, &tmDO, &q_full, h, row0);
-            // first K row of the trajectory (SEGK: of the item's segment key rows)
-            const int64_t krow0 = SEGK ? (v.traj_km[b] + (int64_t)it.s * nt) * 128 : tok0;
+            // first K row of the trajectory (SEGK: of the item's segment key
+            // rows; CMP: of the segment's compact sequence, for V as well)
+            const int64_t krow0 = MODE != 0 ? (v.traj_km[b] + (int64_t)it.s * nt) * 128 : tok0;
             for (int j = 0; j < n; ++j) {
-                const int kt = v.fwd_idx[p0 + j] >> 4;
+                const int kt = entry(j) >> 4;
                 const int s = j & 1;
-                const int row = (int)(tok0 + kt * 128);
+                const int row = (int)((CMP ? krow0 : tok0) + kt * 128);
                 if (j >= 2 && !mbar_wait(&v_empty[s], ((j - 2) >> 1) & 1, status, 111)) break;
                 mbar_expect_tx(&v_full[s], TILE_B);
                 load_tile(sm + DQ_V + s * TILE_B, &tmV, &v_full[s], kvh, row);
@@ -625,7 +701,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             // (half tile: the live half's keys 0..31 in columns 0..15, keys
             // 32..63 in columns 32..47; K rows from 16-row k-step 4 lh on)
             auto issue_dq = [&](int t) -> bool {
-                const int e = v.fwd_idx[p0 + t];
+                const int e = entry(t);
                 if (!mbar_wait(&ds_full[t & 1], (t >> 1) & 1, status, 216)) return false;
                 tc_fence_after();
                 const uint32_t da = tmem + TM_S0 + (t & 1) * 128;
@@ -643,12 +719,12 @@ __global__ void __launch_bounds__(NT_BWD, 1)
                 }
                 mma_commit(&k_empty[t & 1]);
                 mma_commit(&s_free[t & 1]);
-                mma_commit(&dq_done);
+                if (t == n - 1) mma_commit(&dq_fin);
                 return true;
             };
             if (warp == 1) {
                 for (int j = 0; ok && j < n; ++j) {
-                    const int e = v.fwd_idx[p0 + j];
+                    const int e = entry(j);
                     ok = issue_s(j, e) && issue_dp(j, e);
                 }
             } else {
@@ -665,6 +741,10 @@ __global__ void __launch_bounds__(NT_BWD, 1)
         const int ie = min(i, T - 1);
         const int seg = v.seg[tok0 + ie];
         const uint4* km = reinterpret_cast<const uint4*>(v.keymask) + v.traj_km[b] + (int64_t)seg * nt;
+        // CMP: this row's compact index (rows outside the item see no key)
+        const bool in_piece = !CMP || (i >= cp.r0 && i < cp.r1);
+        const int crow = CMP ? (in_piece ? cp.cfirst + i - cp.r0 : -(1 << 30)) : 0;
+        auto mask_words = [&](int e) -> uint4 { return CMP ? prefix_words(crow - (e >> 4) * 128) : km[e >> 4]; };
         const uint32_t lane_base = tmem + ((uint32_t)(qw * 32) << 16);
         const float2 ld = p.lsd[(int64_t)h * p.n_rows + g * 128 + rl];
         const uint64_t c2 = f2(p.scale_log2, p.scale_log2), n2 = f2(ld.x, ld.x), dl2 = f2(ld.y, ld.y);
@@ -672,9 +752,9 @@ __global__ void __launch_bounds__(NT_BWD, 1)
         // list entries and view-mask words are loaded ahead (an entry two
         // tiles, a mask word one tile), so no step waits on a global load once
         // its S is ready
-        int e_cur = n > 0 ? v.fwd_idx[p0] : 0;
-        int e_nxt = n > 1 ? v.fwd_idx[p0 + 1] : 0;
-        uint4 w_cur = n > 0 ? km[e_cur >> 4] : make_uint4(0u, 0u, 0u, 0u);
+        int e_cur = n > 0 ? entry(0) : 0;
+        int e_nxt = n > 1 ? entry(1) : 0;
+        uint4 w_cur = n > 0 ? mask_words(e_cur) : make_uint4(0u, 0u, 0u, 0u);
         // One k-tile for this thread's NC 32-key chunks (2: its 64 keys of a
         // full tile; 1: its 32 of a live half), S and dP read at columns scol /
         // dcol: P = 2^(S c - LSE2), two elements per instruction, masked pairs
@@ -739,11 +819,12 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             const int e = e_cur;
             const uint4 wv = w_cur;
             if (j + 1 < n) {
-                w_cur = km[e_nxt >> 4];
+                w_cur = mask_words(e_nxt);
                 e_cur = e_nxt;
-                e_nxt = j + 2 < n ? v.fwd_idx[p0 + j + 2] : 0;
+                e_nxt = j + 2 < n ? entry(j + 2) : 0;
             }
             const int kt = e >> 4, cls = e & 3;
+            const bool diag = !CMP && kt == qt;   // compact tiles carry causality in their mask words
             if (!mbar_wait(&s_full[j & 1], (j >> 1) & 1, status, 311)) { ok = false; break; }
             tc_fence_after();
             const uint32_t sbuf = lane_base + TM_S0 + (j & 1) * 128;
@@ -755,9 +836,9 @@ __global__ void __launch_bounds__(NT_BWD, 1)
                 stepok = dq_step(std::integral_constant<int, 1>(), j, sbuf + 32 * ch, lane_base + TM_DP + 32 * ch, wm, 0u);
             } else {
                 uint32_t wd[4] = {0xffffffffu, 0xffffffffu, 0xffffffffu, 0xffffffffu};
-                if (cls != MW_TILE_FULL || kt == qt) {
+                if (cls != MW_TILE_FULL || diag) {
                     wd[0] = wv.x; wd[1] = wv.y; wd[2] = wv.z; wd[3] = wv.w;
-                    if (kt == qt) {
+                    if (diag) {
                         const int lim = ie - kt * 128;
 #pragma unroll
                         for (int q = 0; q < 4; ++q) {
@@ -773,11 +854,13 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             tc_fence_before();
             mbar_arrive(&ds_full[j & 1]);
         }
-        if (ok && n > 0 && mbar_wait(&dq_done, (n - 1) & 1, status, 314)) {
+        // awaited on a one-phase barrier (a parity wait on a per-tile barrier
+        // could pass one phase early, before the last dQ MMAs complete)
+        if (ok && n > 0 && mbar_wait(&dq_fin, 0, status, 314)) {
             tc_fence_after();
             __nv_bfloat16* qrow = p.dQ + ((tok0 + ie) * p.Hq + h) * DH;
             uint32_t o[32];
-            const bool store = i < T && (!SEGK || seg == it.s);
+            const bool store = CMP ? in_piece : i < T && (!SEGK || seg == it.s);
 #pragma unroll
             for (int cc = 0; cc < 2; ++cc) {
                 const int c = 2 * ch + cc;
@@ -833,7 +916,7 @@ __device__ __forceinline__ uint64_t mnmaj_ht(uint32_t base, int ks) {
     return sdesc_sw128(base + ks * 2048, HT_HALF, 1024);
 }
 
-template <bool SEGK>
+template <int MODE>
 __global__ void __launch_bounds__(NT_BWD, 1)
     k_attn_dkdv_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmDO,
                    const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, BwdParams p) {
@@ -842,6 +925,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
     __shared__ __align__(8) uint64_t kv_full, qd_full[QD_ST], qd_empty[QD_ST], sd_full[2], sd_free[2], pd_full[2];
     __shared__ uint32_t tmem_base;
 
+    constexpr bool SEGK = MODE == 1, CMP = MODE == 2;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int grp = p.Hq / p.Hkv;
     // KV head outermost: the CTAs resident at one time share one head's Q / dO
@@ -856,10 +940,28 @@ __global__ void __launch_bounds__(NT_BWD, 1)
     const int64_t gk = v.traj_tile[b] + kt;
     const int64_t tok0 = v.traj_tok[b];
     const int T = v.traj_tok[b + 1] - (int)tok0;
-    int p0 = v.bwd_ptr[gk];
-    int nlist = v.bwd_ptr[gk + 1] - p0;
-    int seg_lo = 0, seg_hi = T;        // SEGK: rows [seg_lo, seg_hi) of the item's segment
+    int p0 = CMP ? 0 : v.bwd_ptr[gk];
+    int nlist = CMP ? 0 : v.bwd_ptr[gk + 1] - p0;
+    int seg_lo = 0, seg_hi = T;        // SEGK, CMP: rows [seg_lo, seg_hi) of the item's segment
     int64_t krow0 = tok0 + kt * 128;   // first K row of the tile
+    int nb = 0, qlo = 0, clen = 0;     // CMP: keys of view_s before the segment, first q-tile, |view_s|
+    if (CMP) {
+        // item (compact key tile kt, segment blockIdx.y): keys kt*128.. of
+        // view_s; the rows that see one of them are the segment's rows whose
+        // compact index reaches kt*128, a contiguous run of q-tiles
+        const int sgb = v.traj_seg[b];
+        const int sk = blockIdx.y;
+        if (sk >= v.traj_seg[b + 1] - sgb) return;
+        clen = v.seg_len[sgb + sk];
+        if (kt * 128 >= clen) return;
+        seg_lo = v.seg_start[sgb + sk];
+        seg_hi = sgb + sk + 1 < v.traj_seg[b + 1] ? v.seg_start[sgb + sk + 1] : T;
+        nb = clen - (seg_hi - seg_lo);
+        const int rs = seg_lo + max(0, kt * 128 - nb);
+        qlo = rs >> 7;
+        nlist = ((seg_hi - 1) >> 7) - qlo + 1;
+        krow0 = (v.traj_km[b] + (int64_t)sk * nt + kt) * 128;
+    }
     if (SEGK) {
         // item (k-tile, segment blockIdx.y): only that segment's rows, which
         // read the segment's key rows; its q-tiles are a contiguous run of the
@@ -921,7 +1023,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
     struct Cursor {
         int e, rem, qt, qt_next;
     };
-    auto list_qt = [&](int e) -> int { return e >= 0 ? v.bwd_idx[p0 + e] >> 4 : 0; };
+    auto list_qt = [&](int e) -> int { return e >= 0 ? (CMP ? qlo + e : v.bwd_idx[p0 + e] >> 4) : 0; };
     const Cursor first{nlist - 1, 0, list_qt(nlist - 1), list_qt(nlist - 2)};
     auto advance = [&](Cursor& c) {
         if (++c.rem == 2 * grp) {
@@ -944,7 +1046,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             prefetch_tmap(&tmV);
             mbar_expect_tx(&kv_full, 2 * TILE_B);
             load_tile(sm + KV_K, &tmK, &kv_full, kvh, (int)krow0);
-            load_tile(sm + KV_V, &tmV, &kv_full, kvh, (int)(tok0 + kt * 128));
+            load_tile(sm + KV_V, &tmV, &kv_full, kvh, (int)(CMP ? krow0 : tok0 + kt * 128));
             Cursor c = first;
             int s = 0;
             uint32_t ph = 0;
@@ -1020,8 +1122,11 @@ __global__ void __launch_bounds__(NT_BWD, 1)
         const int jk = kt * 128 + rl;
         const int je = min(jk, T - 1);
         const int iend0 = jk < T ? min(v.omega[tok0 + je], T) : 0;   // rows [jk, iend0) see this key
-        const int jlo = SEGK ? max(jk, seg_lo) : jk;                  // ... of which the item's rows:
-        const int iend = SEGK ? min(iend0, seg_hi) : iend0;            // [jlo, iend)
+        // ... of which the item's rows: [jlo, iend). CMP: compact key jk of
+        // view_s is seen by the segment's rows whose compact index reaches it
+        const bool kin = !CMP || jk < clen;
+        const int jlo = CMP ? (kin ? seg_lo + max(0, jk - nb) : 0) : SEGK ? max(jk, seg_lo) : jk;
+        const int iend = CMP ? (kin ? seg_hi : 0) : SEGK ? min(iend0, seg_hi) : iend0;
         const uint32_t lane_base = tmem + ((uint32_t)(qw * 32) << 16);
         bool ok = true;
         // (-LSE2, Delta) of this warp's 32 query rows of a step: 256 contiguous
@@ -1089,8 +1194,9 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             cur = nxt;
             advance(nxt);
         }
-        if (SEGK && ok && mbar_wait(&sd_free[(nsteps - 1) & 1], ((nsteps - 1) >> 1) & 1, status, 323)) {
+        if (MODE != 0 && ok && mbar_wait(&sd_free[(nsteps - 1) & 1], ((nsteps - 1) >> 1) & 1, status, 323)) {
             // float32 partials of this segment, unscaled dV and scaled dK
+            // (SEGK: per segment key row; CMP: per compact row)
             tc_fence_after();
             const int64_t row = ((krow0 + rl) * p.Hkv + kvh) * DH;
             uint32_t o[32];
@@ -1104,7 +1210,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
                     const int c = 2 * ch + cc;
                     tmem_ld32(lane_base + col + c * 32, o);
                     tmem_wait_ld();
-                    if (jk < T) {
+                    if (CMP ? kin : jk < T) {
 #pragma unroll
                         for (int x = 0; x < 8; ++x)
                             *reinterpret_cast<float4*>(dst + c * 32 + 4 * x) =
@@ -1113,7 +1219,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
                     }
                 }
             }
-        } else if (!SEGK && ok && nsteps > 0 &&
+        } else if (MODE == 0 && ok && nsteps > 0 &&
                    mbar_wait(&sd_free[(nsteps - 1) & 1], ((nsteps - 1) >> 1) & 1, status, 323)) {
             tc_fence_after();
             const int64_t row = ((tok0 + je) * p.Hkv + kvh) * DH;
@@ -1141,7 +1247,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
                     }
                 }
             }
-        } else if (!SEGK && jk < T) {
+        } else if (MODE == 0 && jk < T) {
             // no listed q-tile (cannot happen: the diagonal tile is always listed)
             const int64_t row = ((tok0 + je) * p.Hkv + kvh) * DH;
             for (int c = 0; c < DH; ++c) {
@@ -1159,34 +1265,6 @@ __global__ void __launch_bounds__(NT_BWD, 1)
 }
 
 }  // namespace
-
-mw_status attn_fwd_tc(const mw_vis_layout* L, const void* vis, const void* Q, const void* K, const void* V,
-                      void* O, float* LSE, int Hq, int Hkv, float scale, cudaStream_t s) {
-    if (L->n_tiles == 0) return MW_OK;
-    CUtensorMap tq, tk, tv;
-    const uint64_t T = (uint64_t)L->total_tokens;
-    if (!tmap_bf16_3d(&tq, Q, T, Hq, DH, 128, 64) || !tmap_bf16_3d(&tk, K, T, Hkv, DH, 128, 64) ||
-        !tmap_bf16_3d(&tv, V, T, Hkv, DH, 128, 64))
-        return MW_ECUDA;
-    FwdParams p;
-    p.v = make_view(L, vis);
-    p.total = L->total_tokens;
-    p.n_traj = L->n_traj;
-    p.max_tiles = L->max_tiles;
-    p.Hq = Hq;
-    p.Hkv = Hkv;
-    p.scale_log2 = scale * LOG2E;
-    p.O = (__nv_bfloat16*)O;
-    p.LSE = LSE;
-    p.junction_items = 0;
-    mw_status st = cuda_status(cudaFuncSetAttribute(k_attn_fwd_tc<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                    (int)SMEM_FWD));
-    if (st != MW_OK) return st;
-    const unsigned grid = (unsigned)((int64_t)L->max_tiles * L->n_traj * Hq);
-    count_launches(1);
-    k_attn_fwd_tc<false><<<grid, NT_FWD, SMEM_FWD, s>>>(tq, tk, tv, p);
-    return launch_status();
-}
 
 // Rows of segment key rows (keys per segment) and whether TMA's int32 row
 // coordinates and the junction-item grid reach them.
@@ -1215,15 +1293,15 @@ mw_status attn_fwd_tc_segk(const mw_vis_layout* L, const void* vis, const void* 
     p.O = (__nv_bfloat16*)O;
     p.LSE = LSE;
     p.junction_items = 0;
-    mw_status st = cuda_status(cudaFuncSetAttribute(k_attn_fwd_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    mw_status st = cuda_status(cudaFuncSetAttribute(k_attn_fwd_tc<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                     (int)SMEM_FWD));
     if (st != MW_OK) return st;
     count_launches(1);
-    k_attn_fwd_tc<true><<<(unsigned)((int64_t)L->max_tiles * L->n_traj * Hq), NT_FWD, SMEM_FWD, s>>>(tq, tk, tv, p);
+    k_attn_fwd_tc<1><<<(unsigned)((int64_t)L->max_tiles * L->n_traj * Hq), NT_FWD, SMEM_FWD, s>>>(tq, tk, tv, p);
     if ((st = launch_status()) != MW_OK || L->n_junc == 0) return st;
     p.junction_items = 1;
     count_launches(1);
-    k_attn_fwd_tc<true><<<(unsigned)(L->n_segs * Hq), NT_FWD, SMEM_FWD, s>>>(tq, tk, tv, p);
+    k_attn_fwd_tc<1><<<(unsigned)(L->n_segs * Hq), NT_FWD, SMEM_FWD, s>>>(tq, tk, tv, p);
     return launch_status();
 }
 
@@ -1260,55 +1338,103 @@ __global__ void k_attn_lsd(VisView v, int64_t total, int64_t n_rows, int Hq, con
     }
 }
 
+// Compact K / V: row (traj_km[b] + s nt) 128 + c of Kc, Vc holds the key at
+// rank c of view_s (csrc) for c < |view_s|, zeros up to the end of that
+// tile. One block per (segment, tile) entry with keys in it; 16-byte vectors.
+__global__ void __launch_bounds__(256) k_cmp_gather(VisView v, int n_traj, int Hkv,
+                                                    const __nv_bfloat16* __restrict__ K,
+                                                    const __nv_bfloat16* __restrict__ V, __nv_bfloat16* __restrict__ Kc,
+                                                    __nv_bfloat16* __restrict__ Vc) {
+    const int64_t e = blockIdx.x;
+    int lo = 0, hi = n_traj;   // the trajectory holding entry e: largest b with traj_km[b] <= e
+    while (hi - lo > 1) {
+        const int mid = (lo + hi) >> 1;
+        if (v.traj_km[mid] <= e) lo = mid; else hi = mid;
+    }
+    const int b = lo;
+    const int nt = v.traj_tile[b + 1] - v.traj_tile[b];
+    const int64_t rel = e - v.traj_km[b];
+    const int s = (int)(rel / nt), kt = (int)(rel - (int64_t)s * nt);
+    if (kt * 128 >= v.seg_len[v.traj_seg[b] + s]) return;
+    const int64_t tok0 = v.traj_tok[b];
+    const int vec = Hkv * (DH / 8);   // 16-byte vectors per key row
+    for (int x = threadIdx.x; x < 128 * vec; x += blockDim.x) {
+        const int r = x / vec, k = x - r * vec;
+        const int j = v.csrc[e * 128 + r];
+        uint4 kv = make_uint4(0u, 0u, 0u, 0u), vv = kv;
+        if (j >= 0) {
+            kv = reinterpret_cast<const uint4*>(K + (tok0 + j) * Hkv * DH)[k];
+            vv = reinterpret_cast<const uint4*>(V + (tok0 + j) * Hkv * DH)[k];
+        }
+        reinterpret_cast<uint4*>(Kc + (e * 128 + r) * Hkv * DH)[k] = kv;
+        reinterpret_cast<uint4*>(Vc + (e * 128 + r) * Hkv * DH)[k] = vv;
+    }
+}
+
+// dK, dV of every key from the compact float32 partials: the sum, in segment
+// order, over the segments whose views hold the key, each taken at the key's
+// rank there (cpos); dKc carries the softmax scale already. A key enters the
+// views at its own segment, so the scan starts there. One block per key tile;
+// the order of the additions is fixed, so the result is deterministic.
+__global__ void __launch_bounds__(256) k_cmp_reduce(VisView v, int Hkv, const float* __restrict__ dKc,
+                                                    const float* __restrict__ dVc, __nv_bfloat16* __restrict__ dK,
+                                                    __nv_bfloat16* __restrict__ dV) {
+    const int64_t g = blockIdx.x;
+    const int b = v.tile_traj[g];
+    const int nt = v.traj_tile[b + 1] - v.traj_tile[b];
+    const int kt = (int)(g - v.traj_tile[b]);
+    const int64_t tok0 = v.traj_tok[b];
+    const int T = v.traj_tok[b + 1] - (int)tok0;
+    const int nseg = v.traj_seg[b + 1] - v.traj_seg[b];
+    const int vec = Hkv * (DH / 8);   // 8-element chunks per key row
+    for (int x = threadIdx.x; x < 128 * vec; x += blockDim.x) {
+        const int r = x / vec, k = x - r * vec;
+        const int j = kt * 128 + r;
+        if (j >= T) continue;
+        float ak[8], av[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) ak[q] = av[q] = 0.f;
+        for (int s = v.seg[tok0 + j]; s < nseg; ++s) {
+            const int64_t base = (v.traj_km[b] + (int64_t)s * nt) * 128;
+            const int c = v.cpos[base + j];
+            if (c < 0) continue;
+            const float4* pk = reinterpret_cast<const float4*>(dKc + (base + c) * Hkv * DH) + 2 * k;
+            const float4* pv = reinterpret_cast<const float4*>(dVc + (base + c) * Hkv * DH) + 2 * k;
+            const float4 k0 = pk[0], k1 = pk[1], v0 = pv[0], v1 = pv[1];
+            ak[0] += k0.x; ak[1] += k0.y; ak[2] += k0.z; ak[3] += k0.w;
+            ak[4] += k1.x; ak[5] += k1.y; ak[6] += k1.z; ak[7] += k1.w;
+            av[0] += v0.x; av[1] += v0.y; av[2] += v0.z; av[3] += v0.w;
+            av[4] += v1.x; av[5] += v1.y; av[6] += v1.z; av[7] += v1.w;
+        }
+        reinterpret_cast<uint4*>(dK + (tok0 + j) * Hkv * DH)[k] =
+            make_uint4(pack_bf16(ak[0], ak[1]), pack_bf16(ak[2], ak[3]), pack_bf16(ak[4], ak[5]), pack_bf16(ak[6], ak[7]));
+        reinterpret_cast<uint4*>(dV + (tok0 + j) * Hkv * DH)[k] =
+            make_uint4(pack_bf16(av[0], av[1]), pack_bf16(av[2], av[3]), pack_bf16(av[4], av[5]), pack_bf16(av[6], av[7]));
+    }
+}
+
 }  // namespace
 
-int64_t attn_bwd_tc_ws(const mw_vis_layout* L, int Hq) { return 8 * L->n_tiles * 128 * (int64_t)Hq; }
+// Compact key rows: one 128-row region per (segment, k-tile) entry, of which
+// each segment uses its first ceil(|view_s| / 128) tiles.
+static int64_t cmp_rows(const mw_vis_layout* L) { return L->n_keymask * 128; }
 
-mw_status attn_bwd_tc(const mw_vis_layout* L, const void* vis, const void* Q, const void* K, const void* V,
-                      const void* O, const void* dO, const float* LSE, void* dQ, void* dK, void* dV, int Hq, int Hkv,
-                      float scale, float* ws, cudaStream_t s) {
-    if (L->n_tiles == 0) return MW_OK;
-    const int64_t n_rows = L->n_tiles * 128;
-    float2* lsd = reinterpret_cast<float2*>(ws);
-    const VisView view = make_view(L, vis);
+// The (-LSE2, Delta) pair array alone (the rotary path's backward).
+int64_t attn_lsd_ws(const mw_vis_layout* L, int Hq) { return 8 * L->n_tiles * 128 * (int64_t)Hq; }
+
+int64_t attn_fwd_tc_ws(const mw_vis_layout* L, int Hkv) { return align256(4 * cmp_rows(L) * Hkv * DH); }
+
+int64_t attn_bwd_tc_ws(const mw_vis_layout* L, int Hq, int Hkv) {
+    return align256(8 * L->n_tiles * 128 * (int64_t)Hq) + attn_fwd_tc_ws(L, Hkv) +
+           align256(8 * cmp_rows(L) * Hkv * DH);
+}
+
+static mw_status cmp_gather(const mw_vis_layout* L, const VisView& v, int Hkv, const void* K, const void* V, void* Kc,
+                            void* Vc, cudaStream_t s) {
     count_launches(1);
-    k_attn_lsd<<<(unsigned)std::min<int64_t>(ceil_div(n_rows * Hq, 8), 152 * 64), 256, 0, s>>>(
-        view, L->total_tokens, n_rows, Hq, (const __nv_bfloat16*)O, (const __nv_bfloat16*)dO, LSE, lsd);
-    mw_status st = launch_status();
-    if (st != MW_OK) return st;
-    const uint64_t T = (uint64_t)L->total_tokens;
-    CUtensorMap tq, tdo, tk, tv, tq64, tdo64;
-    if (!tmap_bf16_3d(&tq, Q, T, Hq, DH, 128, 64) || !tmap_bf16_3d(&tdo, dO, T, Hq, DH, 128, 64) ||
-        !tmap_bf16_3d(&tk, K, T, Hkv, DH, 128, 64) || !tmap_bf16_3d(&tv, V, T, Hkv, DH, 128, 64) ||
-        !tmap_bf16_3d(&tq64, Q, T, Hq, DH, 64, 64) || !tmap_bf16_3d(&tdo64, dO, T, Hq, DH, 64, 64))
-        return MW_ECUDA;
-    BwdParams p;
-    p.v = make_view(L, vis);
-    p.total = L->total_tokens;
-    p.n_traj = L->n_traj;
-    p.max_tiles = L->max_tiles;
-    p.Hq = Hq;
-    p.Hkv = Hkv;
-    p.scale = scale;
-    p.scale_log2 = scale * LOG2E;
-    p.lsd = lsd;
-    p.n_rows = n_rows;
-    p.dQ = (__nv_bfloat16*)dQ;
-    p.dK = (__nv_bfloat16*)dK;
-    p.dV = (__nv_bfloat16*)dV;
-    p.junction_items = 0;
-    p.dKseg = p.dVseg = nullptr;
-    if ((st = cuda_status(cudaFuncSetAttribute(k_attn_dq_tc<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                               (int)SMEM_DQ))) != MW_OK)
-        return st;
-    if ((st = cuda_status(cudaFuncSetAttribute(k_attn_dkdv_tc<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                               (int)SMEM_KV))) != MW_OK)
-        return st;
-    count_launches(2);
-    k_attn_dq_tc<false><<<(unsigned)((int64_t)L->max_tiles * L->n_traj * Hq), NT_BWD, SMEM_DQ, s>>>(tq, tdo, tk, tv,
-                                                                                                   p);
-    k_attn_dkdv_tc<false><<<(unsigned)((int64_t)L->max_tiles * L->n_traj * Hkv), NT_BWD, SMEM_KV, s>>>(
-        tq64, tdo64, tk, tv, p);
+    k_cmp_gather<<<(unsigned)L->n_keymask, 256, 0, s>>>(v, L->n_traj, Hkv, (const __nv_bfloat16*)K,
+                                                        (const __nv_bfloat16*)V, (__nv_bfloat16*)Kc,
+                                                        (__nv_bfloat16*)Vc);
     return launch_status();
 }
 
@@ -1351,27 +1477,135 @@ mw_status attn_bwd_tc_segk(const mw_vis_layout* L, const void* vis, const void* 
     p.dKseg = dKseg;
     p.dVseg = dVseg;
     p.junction_items = 0;
-    if ((st = cuda_status(cudaFuncSetAttribute(k_attn_dq_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    if ((st = cuda_status(cudaFuncSetAttribute(k_attn_dq_tc<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                (int)SMEM_DQ))) != MW_OK)
         return st;
-    if ((st = cuda_status(cudaFuncSetAttribute(k_attn_dkdv_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    if ((st = cuda_status(cudaFuncSetAttribute(k_attn_dkdv_tc<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                (int)SMEM_KV))) != MW_OK)
         return st;
     count_launches(1);
-    k_attn_dq_tc<true><<<(unsigned)((int64_t)L->max_tiles * L->n_traj * Hq), NT_BWD, SMEM_DQ, s>>>(tq, tdo, tk, tv,
+    k_attn_dq_tc<1><<<(unsigned)((int64_t)L->max_tiles * L->n_traj * Hq), NT_BWD, SMEM_DQ, s>>>(tq, tdo, tk, tv,
                                                                                                   p);
     if ((st = launch_status()) != MW_OK) return st;
     if (L->n_junc > 0) {
         p.junction_items = 1;
         count_launches(1);
-        k_attn_dq_tc<true><<<(unsigned)(L->n_segs * Hq), NT_BWD, SMEM_DQ, s>>>(tq, tdo, tk, tv, p);
+        k_attn_dq_tc<1><<<(unsigned)(L->n_segs * Hq), NT_BWD, SMEM_DQ, s>>>(tq, tdo, tk, tv, p);
         if ((st = launch_status()) != MW_OK) return st;
         p.junction_items = 0;
     }
     // grid.y: the most segments of any trajectory
     const dim3 gk((unsigned)((int64_t)L->max_tiles * L->n_traj * Hkv), (unsigned)L->max_segs);
     count_launches(1);
-    k_attn_dkdv_tc<true><<<gk, NT_BWD, SMEM_KV, s>>>(tq64, tdo64, tk, tv, p);
+    k_attn_dkdv_tc<1><<<gk, NT_BWD, SMEM_KV, s>>>(tq64, tdo64, tk, tv, p);
+    return launch_status();
+}
+
+// Compact forward: gather every segment's view into Kc / Vc (in `ws`), then
+// one CTA per (q-tile, segment of its first row, head) plus one per (segment
+// starting inside a q-tile, head), each over its segment's compact keys.
+mw_status attn_fwd_tc(const mw_vis_layout* L, const void* vis, const void* Q, const void* K, const void* V, void* O,
+                      float* LSE, int Hq, int Hkv, float scale, void* ws, cudaStream_t s) {
+    if (L->n_tiles == 0) return MW_OK;
+    if (!segk_fits(L, Hq)) return MW_ESHAPE;
+    const VisView view = make_view(L, vis);
+    const int64_t KR = cmp_rows(L);
+    void* Kc = ws;
+    void* Vc = at<char>(ws, 2 * KR * Hkv * DH);
+    mw_status st = cmp_gather(L, view, Hkv, K, V, Kc, Vc, s);
+    if (st != MW_OK) return st;
+    CUtensorMap tq, tk, tv;
+    const uint64_t T = (uint64_t)L->total_tokens;
+    if (!tmap_bf16_3d(&tq, Q, T, Hq, DH, 128, 64) || !tmap_bf16_3d(&tk, Kc, (uint64_t)KR, Hkv, DH, 128, 64) ||
+        !tmap_bf16_3d(&tv, Vc, (uint64_t)KR, Hkv, DH, 128, 64))
+        return MW_ECUDA;
+    FwdParams p;
+    p.v = view;
+    p.total = L->total_tokens;
+    p.n_traj = L->n_traj;
+    p.max_tiles = L->max_tiles;
+    p.Hq = Hq;
+    p.Hkv = Hkv;
+    p.scale_log2 = scale * LOG2E;
+    p.O = (__nv_bfloat16*)O;
+    p.LSE = LSE;
+    p.junction_items = 0;
+    if ((st = cuda_status(cudaFuncSetAttribute(k_attn_fwd_tc<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               (int)SMEM_FWD))) != MW_OK)
+        return st;
+    count_launches(1);
+    k_attn_fwd_tc<2><<<(unsigned)((int64_t)L->max_tiles * L->n_traj * Hq), NT_FWD, SMEM_FWD, s>>>(tq, tk, tv, p);
+    if ((st = launch_status()) != MW_OK || L->n_junc == 0) return st;
+    p.junction_items = 1;
+    count_launches(1);
+    k_attn_fwd_tc<2><<<(unsigned)(L->n_segs * Hq), NT_FWD, SMEM_FWD, s>>>(tq, tk, tv, p);
+    return launch_status();
+}
+
+// Compact backward: (-LSE2, Delta) pairs, the compact gather, dQ (main +
+// junction launches), dK / dV per (compact key tile, segment) into float32
+// partials per compact row, and their deterministic sum per key.
+mw_status attn_bwd_tc(const mw_vis_layout* L, const void* vis, const void* Q, const void* K, const void* V,
+                      const void* O, const void* dO, const float* LSE, void* dQ, void* dK, void* dV, int Hq, int Hkv,
+                      float scale, void* ws, cudaStream_t s) {
+    if (L->n_tiles == 0) return MW_OK;
+    if (!segk_fits(L, Hq)) return MW_ESHAPE;
+    const int64_t n_rows = L->n_tiles * 128;
+    const int64_t KR = cmp_rows(L);
+    float2* lsd = reinterpret_cast<float2*>(ws);
+    void* Kc = at<char>(ws, align256(8 * n_rows * (int64_t)Hq));
+    void* Vc = at<char>(Kc, 2 * KR * Hkv * DH);
+    float* dKc = at<float>(Kc, attn_fwd_tc_ws(L, Hkv));
+    float* dVc = dKc + KR * Hkv * DH;
+    const VisView view = make_view(L, vis);
+    count_launches(1);
+    k_attn_lsd<<<(unsigned)std::min<int64_t>(ceil_div(n_rows * Hq, 8), 152 * 64), 256, 0, s>>>(
+        view, L->total_tokens, n_rows, Hq, (const __nv_bfloat16*)O, (const __nv_bfloat16*)dO, LSE, lsd);
+    mw_status st = launch_status();
+    if (st == MW_OK) st = cmp_gather(L, view, Hkv, K, V, Kc, Vc, s);
+    if (st != MW_OK) return st;
+    const uint64_t T = (uint64_t)L->total_tokens;
+    CUtensorMap tq, tdo, tk, tv, tq64, tdo64;
+    if (!tmap_bf16_3d(&tq, Q, T, Hq, DH, 128, 64) || !tmap_bf16_3d(&tdo, dO, T, Hq, DH, 128, 64) ||
+        !tmap_bf16_3d(&tk, Kc, (uint64_t)KR, Hkv, DH, 128, 64) || !tmap_bf16_3d(&tv, Vc, (uint64_t)KR, Hkv, DH, 128, 64) ||
+        !tmap_bf16_3d(&tq64, Q, T, Hq, DH, 64, 64) || !tmap_bf16_3d(&tdo64, dO, T, Hq, DH, 64, 64))
+        return MW_ECUDA;
+    BwdParams p;
+    p.v = view;
+    p.total = L->total_tokens;
+    p.n_traj = L->n_traj;
+    p.max_tiles = L->max_tiles;
+    p.Hq = Hq;
+    p.Hkv = Hkv;
+    p.scale = scale;
+    p.scale_log2 = scale * LOG2E;
+    p.lsd = lsd;
+    p.n_rows = n_rows;
+    p.dQ = (__nv_bfloat16*)dQ;
+    p.dK = p.dV = nullptr;
+    p.dKseg = dKc;
+    p.dVseg = dVc;
+    p.junction_items = 0;
+    if ((st = cuda_status(cudaFuncSetAttribute(k_attn_dq_tc<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               (int)SMEM_DQ))) != MW_OK)
+        return st;
+    if ((st = cuda_status(cudaFuncSetAttribute(k_attn_dkdv_tc<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               (int)SMEM_KV))) != MW_OK)
+        return st;
+    count_launches(1);
+    k_attn_dq_tc<2><<<(unsigned)((int64_t)L->max_tiles * L->n_traj * Hq), NT_BWD, SMEM_DQ, s>>>(tq, tdo, tk, tv, p);
+    if ((st = launch_status()) != MW_OK) return st;
+    if (L->n_junc > 0) {
+        p.junction_items = 1;
+        count_launches(1);
+        k_attn_dq_tc<2><<<(unsigned)(L->n_segs * Hq), NT_BWD, SMEM_DQ, s>>>(tq, tdo, tk, tv, p);
+        if ((st = launch_status()) != MW_OK) return st;
+        p.junction_items = 0;
+    }
+    const dim3 gk((unsigned)((int64_t)L->max_tiles * L->n_traj * Hkv), (unsigned)L->max_segs);
+    count_launches(2);
+    k_attn_dkdv_tc<2><<<gk, NT_BWD, SMEM_KV, s>>>(tq64, tdo64, tk, tv, p);
+    k_cmp_reduce<<<(unsigned)L->n_tiles, 256, 0, s>>>(view, Hkv, dKc, dVc, (__nv_bfloat16*)dK, (__nv_bfloat16*)dV);
     return launch_status();
 }
 

@@ -66,6 +66,9 @@ struct VisView {
     const int32_t* bwd_ptr;
     const int32_t* bwd_idx;
     const uint32_t* keymask;
+    const int32_t* seg_len;   // [n_segs] |view_s|
+    const int32_t* cpos;      // [n_keymask][128] rank of key j in view_s, -1 if absent
+    const int32_t* csrc;      // [n_keymask][128] key (traj-local) at each rank of view_s
     int32_t* status;
 };
 
@@ -86,6 +89,9 @@ inline VisView make_view(const mw_vis_layout* L, const void* vis) {
     v.bwd_ptr = at<int32_t>(vis, L->off_bwd_ptr);
     v.bwd_idx = at<int32_t>(vis, L->off_bwd_idx);
     v.keymask = at<uint32_t>(vis, L->off_keymask);
+    v.seg_len = at<int32_t>(vis, L->off_seg_len);
+    v.cpos = at<int32_t>(vis, L->off_cpos);
+    v.csrc = at<int32_t>(vis, L->off_csrc);
     v.status = const_cast<int32_t*>(at<int32_t>(vis, L->off_status));
     return v;
 }

@@ -51,7 +51,7 @@ extern "C" const char* mw_status_str(int s) {
 }
 
 extern "C" int mw_last_cuda_error(void) { return g_last_cuda_error; }
-extern "C" int mw_abi_version(void) { return 4; }
+extern "C" int mw_abi_version(void) { return 5; }
 extern "C" uint64_t mw_kernel_launches(void) { return (uint64_t)g_launches.load(std::memory_order_relaxed); }
 
 static mw_status check_shape(int n_traj, const int32_t* cu, int n_junc, const int32_t* jt,
@@ -117,6 +117,9 @@ extern "C" mw_status mw_visibility_layout(int n_traj, const int32_t* cu, int n_j
     L->off_pairs = take(8 * (n_traj + 1));
     L->off_keymask = take(16 * km);
     L->off_status = take(4 * 8);
+    L->off_seg_len = take(4 * L->n_segs);
+    L->off_cpos = take(4 * MW_TILE * km);
+    L->off_csrc = take(4 * MW_TILE * km);
     L->vis_bytes = o;
     o = 0;
     L->ws_off_spans = take(12 * (int64_t)n_spans);
@@ -153,6 +156,9 @@ struct BuildArgs {
     int32_t* bwd_idx;
     unsigned long long* pairs;
     uint32_t* keymask;
+    int32_t* seg_len;       // [n_segs]
+    int32_t* cpos;          // [n_keymask][128]
+    int32_t* csrc;          // [n_keymask][128]
     const int32_t* spans;   // [n_spans][3]
     int32_t* tstat;         // [n_tiles][4] min, max lifetime; max over keys 0..63, 64..127
     int32_t* fwd_cnt;       // [n_tiles]
@@ -368,6 +374,72 @@ __global__ void k_fill(BuildArgs a) {
     }
 }
 
+// Compact views: one block per global segment. An exclusive prefix popcount
+// of the segment's view bits, tile by tile, gives every member key its rank in
+// view_s (cpos; -1 for non-members) and the inverse map (csrc: the key at each
+// rank); the total is |view_s|, and csrc is -1 from there to the end of the
+// last 128-entry tile. For a monotone record view_s is in physical order, so
+// the rank is the key's index in the segment's compact sequence (§4.1).
+__global__ void __launch_bounds__(256) k_compact_map(BuildArgs a) {
+    __shared__ int tp[256];
+    __shared__ int wsum[8];
+    __shared__ int carry_s;
+    const int sg = blockIdx.x;
+    int lo = 0, hi = a.n_traj;   // largest b with traj_seg[b] <= sg
+    while (hi - lo > 1) {
+        const int mid = (lo + hi) >> 1;
+        if (a.traj_seg[mid] <= sg) lo = mid; else hi = mid;
+    }
+    const int b = lo;
+    const int s = sg - a.traj_seg[b];
+    const int nt = a.traj_tile[b + 1] - a.traj_tile[b];
+    const int64_t ent0 = a.traj_km[b] + (int64_t)s * nt;   // keymask entry of (s, kt = 0)
+    const uint32_t* km = a.keymask + ent0 * 4;
+    int32_t* pos = a.cpos + ent0 * MW_TILE;
+    int32_t* src = a.csrc + ent0 * MW_TILE;
+    const int t = threadIdx.x, lane = t & 31, w = t >> 5;
+    if (t == 0) carry_s = 0;
+    __syncthreads();
+    for (int c0 = 0; c0 < nt; c0 += 256) {
+        const int kt = c0 + t;
+        int cnt = 0;
+        if (kt < nt)
+            cnt = __popc(km[4 * kt]) + __popc(km[4 * kt + 1]) + __popc(km[4 * kt + 2]) + __popc(km[4 * kt + 3]);
+        int incl = cnt;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += y;
+        }
+        if (lane == 31) wsum[w] = incl;
+        __syncthreads();
+        int before = carry_s;
+        for (int q = 0; q < w; ++q) before += wsum[q];
+        tp[t] = before + incl - cnt;
+        __syncthreads();
+        const int ntc = min(256, nt - c0);
+        for (int k = t; k < ntc * MW_TILE; k += 256) {
+            const int tl = k >> 7, jj = k & 127, wd = jj >> 5, bit = jj & 31;
+            const uint32_t* tw = km + 4 * (c0 + tl);
+            const uint32_t word = tw[wd];
+            int32_t r = -1;
+            if ((word >> bit) & 1u) {
+                r = tp[tl] + __popc(word & ((1u << bit) - 1u));
+                for (int q = 0; q < wd; ++q) r += __popc(tw[q]);
+                src[r] = (c0 + tl) * MW_TILE + jj;
+            }
+            pos[(int64_t)(c0 + tl) * MW_TILE + jj] = r;
+        }
+        __syncthreads();
+        if (t == 255) carry_s = tp[255] + cnt;
+        __syncthreads();
+    }
+    const int len = carry_s;
+    if (t == 0) a.seg_len[sg] = len;
+    const int end = (len + MW_TILE - 1) / MW_TILE * MW_TILE;
+    for (int r = len + t; r < end; r += 256) src[r] = -1;
+}
+
 }  // namespace
 
 // ---------------------------------------------------------------------------
@@ -485,12 +557,15 @@ extern "C" mw_status mw_build_visibility(const mw_vis_layout* L, const int32_t* 
     a.bwd_idx = at<int32_t>(vis, L->off_bwd_idx);
     a.pairs = at<unsigned long long>(vis, L->off_pairs);
     a.keymask = at<uint32_t>(vis, L->off_keymask);
+    a.seg_len = at<int32_t>(vis, L->off_seg_len);
+    a.cpos = at<int32_t>(vis, L->off_cpos);
+    a.csrc = at<int32_t>(vis, L->off_csrc);
     a.spans = at<int32_t>(ws, L->ws_off_spans);
     a.tstat = at<int32_t>(ws, L->ws_off_tstat);
     a.fwd_cnt = at<int32_t>(ws, L->ws_off_cnt);
     a.bwd_cnt = at<int32_t>(ws, L->ws_off_cnt) + n_tiles;
 
-    count_launches((a.total > 0 ? 1 + (L->n_spans > 0) : 0) + (n_tiles > 0 ? 3 : 0) + 1 + (n_tiles > 0));
+    count_launches((a.total > 0 ? 1 + (L->n_spans > 0) : 0) + (n_tiles > 0 ? 3 : 0) + 1 + 2 * (n_tiles > 0));
     if (a.total > 0) {
         int grid = (int)std::min<int64_t>(ceil_div(a.total, 256), 152 * 16);
         k_init_tokens<<<grid, 256, 0, stream>>>(a);
@@ -503,7 +578,10 @@ extern "C" mw_status mw_build_visibility(const mw_vis_layout* L, const int32_t* 
         k_bwd_count<<<wgrid, 256, 0, stream>>>(a);
     }
     k_scan<<<1, 1024, 0, stream>>>(a);
-    if (n_tiles > 0) k_fill<<<(unsigned)ceil_div(n_tiles * 32, 256), 256, 0, stream>>>(a);
+    if (n_tiles > 0) {
+        k_fill<<<(unsigned)ceil_div(n_tiles * 32, 256), 256, 0, stream>>>(a);
+        k_compact_map<<<(unsigned)L->n_segs, 256, 0, stream>>>(a);
+    }
     return launch_status();
 }
 

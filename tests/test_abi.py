@@ -102,11 +102,11 @@ def test_attention_and_lmhead_reject_bad_args_on_host():
     lay = L.mw_visibility_layout(np.array([0, 10], np.int32), np.zeros(0, np.int32), 0)
     P = ctypes.c_void_p(16)
     # Hq not a multiple of Hkv
-    assert h.mw_masked_attn_fwd(ctypes.byref(lay), P, P, P, P, P, P, 6, 4, 128, 1, 0.1, None) == 3
+    assert h.mw_masked_attn_fwd(ctypes.byref(lay), P, P, P, P, P, P, 6, 4, 128, 1, 0.1, P, None) == 3
     # bad dtype, bad head dim, bad scale
-    assert h.mw_masked_attn_fwd(ctypes.byref(lay), P, P, P, P, P, P, 4, 4, 128, 7, 0.1, None) == 4
-    assert h.mw_masked_attn_fwd(ctypes.byref(lay), P, P, P, P, P, P, 4, 4, 96, 1, 0.1, None) == 3
-    assert h.mw_masked_attn_fwd(ctypes.byref(lay), P, P, P, P, P, P, 4, 4, 128, 1, -1.0, None) == 1
+    assert h.mw_masked_attn_fwd(ctypes.byref(lay), P, P, P, P, P, P, 4, 4, 128, 7, 0.1, P, None) == 4
+    assert h.mw_masked_attn_fwd(ctypes.byref(lay), P, P, P, P, P, P, 4, 4, 96, 1, 0.1, P, None) == 3
+    assert h.mw_masked_attn_fwd(ctypes.byref(lay), P, P, P, P, P, P, 4, 4, 128, 1, -1.0, P, None) == 1
     # log-prob: M > N, bad eps, null loss
     n = ctypes.c_size_t()
     assert h.mw_logprob_ws(10, 11, 128, 100, 0, ctypes.byref(n)) == 3

@@ -24,8 +24,11 @@ def _gpu(seqlens, edits):
 def _compare(seqlens, edits):
     got = _gpu(seqlens, edits)
     want = OV.build(seqlens, edits)
-    for key in ("omega", "seg", "qtile_traj", "fwd_ptr", "fwd_idx", "bwd_ptr", "bwd_idx", "pairs", "keymask"):
+    for key in ("omega", "seg", "qtile_traj", "fwd_ptr", "fwd_idx", "bwd_ptr", "bwd_idx", "pairs", "keymask",
+                "seg_len", "cpos"):
         np.testing.assert_array_equal(got[key], want[key], err_msg=key)
+    defined = want["csrc"] != -2          # the compact maps past a segment's last tile are unspecified
+    np.testing.assert_array_equal(got["csrc"][defined], want["csrc"][defined], err_msg="csrc")
     assert got["pairs_total"] == want["pairs_total"]
     assert len(got["cls"]) == len(want["cls"])
     for a, b in zip(got["cls"], want["cls"]):

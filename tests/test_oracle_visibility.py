@@ -228,3 +228,47 @@ def test_conditioning_invariant_on_views():
 def test_invalid_records_rejected(bad):
     with pytest.raises(V.RecordError):
         V.live_views(100, bad)
+
+
+def test_compact_maps_running_example():
+    """Each segment's compact sequence (``csrc``) read up to a row's own index
+    is exactly the prefix Table "running-prefixes" prints for the leaf that
+    row predicts; ``cpos`` is its inverse and ``seg_len`` its length."""
+    g = _load("running_example.json")
+    tok = g["tokens"]
+    pos = {t: n for n, t in enumerate(tok)}
+    edits = _edits(g["edits"])
+    T = len(tok)
+    out = V.build([T], [edits])
+    nt = -(-T // V.TILE)
+    seg = V.segment_ids(T, edits)
+    for leaf, prefix in g["live_view_prefix"].items():
+        row = pos[leaf] - 1
+        s = int(seg[row])
+        base = s * nt * V.TILE
+        c_row = int(out["cpos"][base + row])
+        assert c_row >= 0
+        got = out["csrc"][base: base + c_row + 1].tolist()
+        assert got == sorted({0} | {pos[t] for t in prefix}), leaf
+    assert out["seg_len"].tolist() == [7, 9, 10, 11]
+
+
+@pytest.mark.parametrize("seed", range(5))
+def test_compact_maps_inverse(seed):
+    rng = np.random.default_rng(seed)
+    T = int(rng.integers(130, 600))
+    Js = sorted(rng.choice(np.arange(2, T), size=4, replace=False).tolist())
+    edits = [(J, [(int(a), int(min(J, a + rng.integers(1, 40))))
+                  for a in rng.integers(0, J - 1, 3)]) for J in Js]
+    out = V.build([T], [edits])
+    nt = -(-T // V.TILE)
+    for s, (lo, hi, view) in enumerate(V.live_views(T, edits)):
+        base = s * nt * V.TILE
+        src = out["csrc"][base: base + nt * V.TILE]
+        pos = out["cpos"][base: base + nt * V.TILE]
+        L = int(out["seg_len"][s])
+        assert L == len(view)
+        assert all(pos[src[c]] == c for c in range(L))
+        assert int((pos[:T] >= 0).sum()) == L
+        assert (src[L: -(-L // V.TILE) * V.TILE] == -1).all()
+        assert src[L - (hi - lo): L].tolist() == list(range(lo, hi))   # the segment's rows are the tail
