@@ -124,7 +124,16 @@ typedef struct mw_vis_layout {
     int64_t off_cpos;       /* int32 [n_keymask][128] rank of key j in view_s (the compact index), -1 if absent */
     int64_t off_csrc;       /* int32 [n_keymask][128] key (traj-local) at compact index c of view_s;
                                -1 from |view_s| to the end of its last 128-entry tile, unset after */
+    int64_t kind;           /* MW_VIEWS_EDITS (mw_visibility_layout) or MW_VIEWS_EVENTS (mw_events_layout) */
 } mw_vis_layout;
+
+/* Record kinds. EDITS: each edit only evicts (one lifetime interval per key),
+ * every array of `vis` is built. EVENTS: an edit may also bring earlier
+ * evicted spans back (offload / retrieve), so a view is an ordered list that
+ * need not follow physical order; `vis` then holds the segments, the compact
+ * views (seg_len, cpos, csrc), the view bits and the pair counts, and no
+ * lifetimes (omega reads INT32_MAX), tile classes or tile lists (empty). */
+enum { MW_VIEWS_EDITS = 0, MW_VIEWS_EVENTS = 1 };
 
 /*
  * Fill `out` for a record shape. Host-only; launches nothing.
@@ -134,6 +143,37 @@ typedef struct mw_vis_layout {
  */
 mw_status mw_visibility_layout(int n_traj, const int32_t* cu_seqlens, int n_junc,
                                const int32_t* junc_traj, int n_spans, mw_vis_layout* out);
+
+/*
+ * Layout of an EVENTS record (offload / retrieve): the same shape arguments as
+ * mw_visibility_layout, n_spans counting out- and in-spans together. Sets
+ * kind = MW_VIEWS_EVENTS and sizes the build workspace for the event replay.
+ */
+mw_status mw_events_layout(int n_traj, const int32_t* cu_seqlens, int n_junc, const int32_t* junc_traj,
+                           int n_spans, mw_vis_layout* out);
+
+/*
+ * Views of an EVENTS record (the paper's MemexRL harness, App. F: offload
+ * evicts a span, retrieve brings it back). Event k fires at junction J_k like
+ * an edit (rows i >= J_k see the post-event view): first the out-spans
+ * spans[out_off[k] .. out_off[k+1]) leave the view, then the in-spans
+ * spans[in_off[k] .. in_off[k+1]) -- positions out of the view at J_k --
+ * re-enter at its end in the given order, before the segment's own rows
+ * (the harness figure's MemexRL panel draws retrieved tokens after the ones
+ * decoded meanwhile). A row sees the members of its segment's list up to and
+ * including itself.
+ *   junctions, junc_traj as for mw_build_visibility; out_off, in_off host
+ *   int32 [n_junc + 1] (CSR into spans, non-decreasing, within [0, n_spans]);
+ *   spans host int32 [n_spans][2] half-open [a, b) with 0 <= a < b <= J_k.
+ * MW_EEDITS if a retrieved position is not out of the view when its event
+ * fires, or on any convention of mw_build_visibility. `layout` must come from
+ * mw_events_layout; `ws` and `vis` as for mw_build_visibility. The masked
+ * attention (bf16, Dh 128) accepts such views; entry points that need
+ * single-interval lifetimes return MW_ESHAPE for them.
+ */
+mw_status mw_build_views_events(const mw_vis_layout* layout, const int32_t* cu_seqlens, int n_junc,
+                                const int32_t* junctions, const int32_t* junc_traj, const int32_t* out_off,
+                                const int32_t* in_off, const int32_t* spans, void* ws, void* vis, void* stream);
 
 /*
  * Build every visibility artefact of a record (§4.2 lifetimes; App. B.1

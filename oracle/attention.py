@@ -44,11 +44,17 @@ def _ix(x):
     return torch.from_numpy(np.asarray(x, dtype=np.int64))
 
 
-def _segments(seqlens, edits_per_traj):
-    """Yield ``(global_rows, global_view_positions, n_before)`` per segment."""
+def _segments(seqlens, edits_per_traj, views=None):
+    """Yield ``(global_rows, global_view_positions, n_before)`` per segment.
+
+    ``views`` maps ``(T, edits)`` to the ``[(row_lo, row_hi, view)]`` lists of
+    each segment (default: ``visibility.live_views``; ``nonmonotone.live_views``
+    for records whose events also bring spans back). The compact sequence is
+    the view list in its own order."""
+    views = live_views if views is None else views
     base = 0
     for T, edits in zip(seqlens, edits_per_traj):
-        for lo, hi, view in live_views(T, edits):
+        for lo, hi, view in views(T, edits):
             idx = np.asarray(view, dtype=np.int64) + base
             yield np.arange(lo, hi, dtype=np.int64) + base, idx, len(view) - (hi - lo)
         base += T
@@ -92,7 +98,7 @@ def _probs(q, k, scale, compact_rows):
     return p, m, l
 
 
-def attn_fwd(seqlens, edits_per_traj, Q, K, V, scale, rows=None, heads=None, rope_theta=None):
+def attn_fwd(seqlens, edits_per_traj, Q, K, V, scale, rows=None, heads=None, rope_theta=None, views=None):
     """Masked GQA attention forward via per-segment compact sequences.
 
     Returns ``(O_sel, LSE_sel)`` for the selected global rows (default: all)
@@ -112,7 +118,7 @@ def attn_fwd(seqlens, edits_per_traj, Q, K, V, scale, rows=None, heads=None, rop
     L = torch.full((len(heads), len(rows)), float("nan"), dtype=torch.float64)
     want = np.zeros(Ttot, dtype=bool)
     want[rows] = True
-    for seg_rows, idx, n_before in _segments(seqlens, edits_per_traj):
+    for seg_rows, idx, n_before in _segments(seqlens, edits_per_traj, views):
         sel = np.nonzero(want[seg_rows])[0]
         if sel.size == 0:
             continue
@@ -140,7 +146,7 @@ def attn_fwd(seqlens, edits_per_traj, Q, K, V, scale, rows=None, heads=None, rop
     return O.numpy(), L.numpy()
 
 
-def attn_bwd(seqlens, edits_per_traj, Q, K, V, dO, scale, groups=None, rope_theta=None):
+def attn_bwd(seqlens, edits_per_traj, Q, K, V, dO, scale, groups=None, rope_theta=None, views=None):
     """Textbook softmax-attention backward on every segment's compact sequence.
 
     For one segment and head (compact rows r, compact keys c):
@@ -166,7 +172,7 @@ def attn_bwd(seqlens, edits_per_traj, Q, K, V, dO, scale, groups=None, rope_thet
         dQ[:, g * grp : (g + 1) * grp] = 0.0
         dK[:, g] = 0.0
         dV[:, g] = 0.0
-    for seg_rows, idx, n_before in _segments(seqlens, edits_per_traj):
+    for seg_rows, idx, n_before in _segments(seqlens, edits_per_traj, views):
         ti = _ix(idx)
         for g in groups:
             k = K[ti, g]
@@ -200,7 +206,7 @@ def attn_bwd(seqlens, edits_per_traj, Q, K, V, dO, scale, groups=None, rope_thet
     return dQ.numpy(), dK.numpy(), dV.numpy()
 
 
-def attn_bwd_rows(seqlens, edits_per_traj, Q, K, V, dO, scale, rows, heads, rope_theta=None, with_kv=False):
+def attn_bwd_rows(seqlens, edits_per_traj, Q, K, V, dO, scale, rows, heads, rope_theta=None, with_kv=False, views=None):
     """dQ of a few physical rows and query heads (same formulas as
     ``attn_bwd``, rotary positions included; a row's dQ needs only its own
     segment's compact view and its own dO row). Returns ``dQ_sel[r, h_i, :]``.
@@ -220,7 +226,7 @@ def attn_bwd_rows(seqlens, edits_per_traj, Q, K, V, dO, scale, rows, heads, rope
     dV = torch.zeros_like(V) if with_kv else None
     want = np.zeros(Q.shape[0], dtype=bool)
     want[rows] = True
-    for seg_rows, idx, n_before in _segments(seqlens, edits_per_traj):
+    for seg_rows, idx, n_before in _segments(seqlens, edits_per_traj, views):
         part = np.nonzero(want[seg_rows])[0]
         if part.size == 0:
             continue
@@ -258,7 +264,7 @@ def attn_bwd_rows(seqlens, edits_per_traj, Q, K, V, dO, scale, rows, heads, rope
     return out.numpy()
 
 
-def attn_bwd_keys(seqlens, edits_per_traj, Q, K, V, dO, scale, g, keys, rope_theta=None):
+def attn_bwd_keys(seqlens, edits_per_traj, Q, K, V, dO, scale, g, keys, rope_theta=None, views=None):
     """dK, dV of KV group ``g`` for a few physical key rows only.
 
     Same textbook formulas as ``attn_bwd`` (rotary positions included: a key's
@@ -276,7 +282,7 @@ def attn_bwd_keys(seqlens, edits_per_traj, Q, K, V, dO, scale, g, keys, rope_the
     keys = np.asarray(keys, dtype=np.int64)
     dk_out = torch.zeros((keys.size, K.shape[2]), dtype=torch.float64)
     dv_out = torch.zeros((keys.size, K.shape[2]), dtype=torch.float64)
-    for seg_rows, idx, n_before in _segments(seqlens, edits_per_traj):
+    for seg_rows, idx, n_before in _segments(seqlens, edits_per_traj, views):
         where = {int(p): c for c, p in enumerate(idx)}
         cols = [(n, where[int(kk)]) for n, kk in enumerate(keys) if int(kk) in where]
         if not cols:

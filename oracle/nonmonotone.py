@@ -15,7 +15,10 @@ A view is therefore an ordered list that need not follow physical order; a
 row's keys are the members of its segment's list up to and including itself,
 and its rotary positions are list indices.
 
-Nothing here is used by the GPU path (which has no non-monotone support).
+``build`` gives the artefacts the GPU builder of such records produces (the
+segments, each segment's compact sequence and its ranks, the view bits and
+the visible pairs), straight from the lists; the attention oracle runs on the
+same lists (``oracle.attention`` with ``views=live_views``).
 """
 
 import numpy as np
@@ -134,3 +137,45 @@ def attn_fwd(T, events, Q, K, V, scale, rope_theta=None):
             p = np.exp(s - s.max(axis=1, keepdims=True))
             O[lo:hi, h] = (p / p.sum(axis=1, keepdims=True)) @ V[idx, h // grp]
     return O
+
+
+def build(seqlens, events_per_traj, tile=128):
+    """Per packed record (trajectories back to back), in the GPU layout:
+    ``seg`` int32 [T_total] segment of each row; ``seg_len`` int32 [n_segs]
+    length of each view list; ``cpos`` / ``csrc`` int32 (entry
+    ``(km_b + s nt_b) tile + j``, km_b the trajectory's first (segment, tile)
+    entry): the index of key j in view_s (-1 if absent) and the key at index
+    c (-1 from the list's end to the end of its last tile, -2 after, left
+    unspecified); ``keymask`` uint32 [entries][tile / 32] view membership
+    bits; ``pairs`` int64 [n_traj] visible pairs (a row at list index c sees
+    c + 1 keys) and ``pairs_total``."""
+    seg, seg_len, cpos, csrc, keymask, pairs = [], [], [], [], [], []
+    for T, events in zip(seqlens, events_per_traj):
+        nt = -(-T // tile)
+        sg = np.zeros(T, dtype=np.int32)
+        npairs = 0
+        for s, (lo, hi, view) in enumerate(live_views(T, events)):
+            sg[lo:hi] = s
+            seg_len.append(len(view))
+            pos = np.full(nt * tile, -1, dtype=np.int64)
+            pos[np.asarray(view, dtype=np.int64)] = np.arange(len(view))
+            cpos.append(pos)
+            src = np.full(nt * tile, -2, dtype=np.int64)
+            src[: -(-len(view) // tile) * tile] = -1
+            src[: len(view)] = view
+            csrc.append(src)
+            bits = (pos >= 0).reshape(nt, tile // 32, 32).astype(np.uint64)
+            keymask.append((bits << np.arange(32, dtype=np.uint64)).sum(-1).astype(np.uint32))
+            npairs += sum(view.index(i) + 1 for i in range(lo, hi))
+        seg.append(sg)
+        pairs.append(npairs)
+    cat = lambda xs, dt: np.concatenate(xs).astype(dt) if xs else np.zeros(0, dt)   # noqa: E731
+    return {
+        "seg": cat(seg, np.int32),
+        "seg_len": np.asarray(seg_len, dtype=np.int32),
+        "cpos": cat(cpos, np.int32),
+        "csrc": cat(csrc, np.int32),
+        "keymask": np.concatenate(keymask) if keymask else np.zeros((0, tile // 32), np.uint32),
+        "pairs": np.asarray(pairs, dtype=np.int64),
+        "pairs_total": int(sum(pairs)),
+    }

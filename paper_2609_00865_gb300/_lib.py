@@ -36,7 +36,7 @@ class VisLayout(ctypes.Structure):
                    "off_fwd_ptr", "off_fwd_idx", "off_bwd_ptr", "off_bwd_idx", "off_pairs",
                    "off_keymask", "off_status", "vis_bytes",
                    "ws_off_spans", "ws_off_tstat", "ws_off_cnt", "ws_bytes", "max_segs",
-                   "off_seg_len", "off_cpos", "off_csrc")]
+                   "off_seg_len", "off_cpos", "off_csrc", "kind")]
 
 
 _P = ctypes.c_void_p
@@ -53,6 +53,8 @@ _SIGS = {
     "mw_visibility_layout": (_I, [_I, _IP, _I, _IP, _I, _LP]),
     "mw_build_visibility": (_I, [_LP, _IP, _I, _IP, _IP, _IP, _IP, _P, _P, _P]),
     "mw_build_visibility_noalloc": (_I, [_LP, _IP, _I, _IP, _IP, _IP, _IP, _P, _P]),
+    "mw_events_layout": (_I, [_I, _IP, _I, _IP, _I, _LP]),
+    "mw_build_views_events": (_I, [_LP, _IP, _I, _IP, _IP, _IP, _IP, _IP, _P, _P, _P]),
     "mw_masked_attn_fwd_ws": (_I, [_LP, _I, _I, _I, ctypes.POINTER(ctypes.c_size_t)]),
     "mw_masked_attn_fwd": (_I, [_LP, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _F, _P, _P]),
     "mw_masked_attn_bwd_ws": (_I, [_LP, _I, _I, _I, _I, ctypes.POINTER(ctypes.c_size_t)]),
@@ -194,6 +196,60 @@ def mw_build_visibility_noalloc(layout, cu_seqlens, junctions, junc_traj, junc_s
                                               _ptr(vis), _stream(stream)), "mw_build_visibility_noalloc")
 
 
+def flatten_events(seqlens, events_per_traj):
+    """Events record -> (cu_seqlens, junctions, junc_traj, out_off, in_off,
+    spans): the out-spans of every event in event order, then the in-spans,
+    in one span table; out_off / in_off are the CSR offsets of each event's
+    ranges in it."""
+    cu = np.zeros(len(seqlens) + 1, dtype=np.int32)
+    cu[1:] = np.cumsum(seqlens)
+    J, jt, outs, ins, out_off, in_off = [], [], [], [], [0], [0]
+    for b, events in enumerate(events_per_traj):
+        for j, sp_out, sp_in in events:
+            J.append(j)
+            jt.append(b)
+            outs.extend((a, e) for a, e in sp_out)
+            ins.extend((a, e) for a, e in sp_in)
+            out_off.append(len(outs))
+            in_off.append(len(ins))
+    spans = np.asarray(outs + ins, np.int32).reshape(-1, 2)
+    return (cu, np.asarray(J, np.int32), np.asarray(jt, np.int32), np.asarray(out_off, np.int32),
+            np.asarray(in_off, np.int32) + len(outs), spans)
+
+
+def mw_events_layout(cu_seqlens, junc_traj, n_spans):
+    L = VisLayout()
+    cu, cup = _i32(cu_seqlens)
+    jt, jtp = _i32(junc_traj)
+    _check(_lib().mw_events_layout(len(cu) - 1, cup, len(jt), jtp, int(n_spans), ctypes.byref(L)),
+           "mw_events_layout")
+    return L
+
+
+def mw_build_views_events(layout, cu_seqlens, junctions, junc_traj, out_off, in_off, spans, ws, vis, stream=None):
+    cu, cup = _i32(cu_seqlens)
+    J, Jp = _i32(junctions)
+    jt, jtp = _i32(junc_traj)
+    oo, oop = _i32(out_off)
+    io, iop = _i32(in_off)
+    sp, spp = _i32(np.asarray(spans).reshape(-1))
+    _check(_lib().mw_build_views_events(ctypes.byref(layout), cup, len(J), Jp, jtp, oop, iop, spp, _ptr(ws),
+                                        _ptr(vis), _stream(stream)), "mw_build_views_events")
+
+
+def build_views_events(seqlens, events_per_traj, device="cuda", stream=None):
+    """Views of an events (offload / retrieve) record: flatten, allocate with
+    torch, run the builder. ``events_per_traj[b]`` lists (J, out_spans,
+    in_spans) per event."""
+    import torch
+    cu, J, jt, oo, io, spans = flatten_events(seqlens, events_per_traj)
+    L = mw_events_layout(cu, jt, len(spans))
+    vis = torch.empty(max(int(L.vis_bytes), 1), dtype=torch.uint8, device=device)
+    ws = torch.empty(max(int(L.ws_bytes), 1), dtype=torch.uint8, device=device)
+    mw_build_views_events(L, cu, J, jt, oo, io, spans, ws, vis, stream)
+    return Visibility(L, vis, ws)
+
+
 class Visibility:
     """Device visibility buffer of one packed record plus its layout."""
 
@@ -212,7 +268,7 @@ class Visibility:
         """Copy every artefact to the host in the oracle's ``build`` format."""
         L = self.layout
         n = L.n_tiles
-        fwd_ptr = self._arr(L.off_fwd_ptr, n + 1, np.int32)
+        fwd_ptr = self._arr(L.off_fwd_ptr, n + 1, np.int32)   # all zero for an events record
         bwd_ptr = self._arr(L.off_bwd_ptr, n + 1, np.int32)
         tok = self._arr(L.off_traj_tok, L.n_traj + 1, np.int32)
         tile = self._arr(L.off_traj_tile, L.n_traj + 1, np.int32)

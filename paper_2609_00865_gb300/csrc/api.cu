@@ -114,6 +114,8 @@ extern "C" mw_status mw_masked_attn_fwd(const mw_vis_layout* L, const void* vis,
                                         float scale, void* ws, void* stream) {
     mw_status st = attn_args(L, vis, Hq, Hkv, Dh, dtype, scale);
     if (st != MW_OK) return st;
+    // views of an EVENTS record have no tile lists: only the compact path reads them
+    if (L->kind != MW_VIEWS_EDITS && !(dtype == MW_BF16 && Dh == 128)) return MW_ESHAPE;
     if (L->total_tokens == 0) return MW_OK;
     if (!Q || !K || !V || !O || !LSE) return MW_EINVAL;
     if (dtype == MW_BF16 && Dh == 128) {
@@ -139,6 +141,8 @@ extern "C" mw_status mw_masked_attn_bwd(const mw_vis_layout* L, const void* vis,
                                         void* ws, void* stream) {
     mw_status st = attn_args(L, vis, Hq, Hkv, Dh, dtype, scale);
     if (st != MW_OK) return st;
+    // views of an EVENTS record have no tile lists: only the compact path reads them
+    if (L->kind != MW_VIEWS_EDITS && !(dtype == MW_BF16 && Dh == 128)) return MW_ESHAPE;
     if (L->total_tokens == 0) return MW_OK;
     if (!Q || !K || !V || !O || !dO || !LSE || !dQ || !dK || !dV || !ws) return MW_EINVAL;
     if (dtype == MW_BF16 && Dh == 128)
@@ -290,6 +294,7 @@ static mw_status rope_args(const mw_vis_layout* L, const void* vis, const int32_
 }
 
 extern "C" mw_status mw_logical_positions(const mw_vis_layout* L, const void* vis, int32_t* pos, void* stream) {
+    if (L && L->kind != MW_VIEWS_EDITS) return MW_ESHAPE;   // rotary kernels read the tile lists
     if (!L) return MW_EINVAL;
     if (L->n_keymask == 0) return MW_OK;
     if (!vis || !pos) return MW_EINVAL;
@@ -306,6 +311,7 @@ extern "C" mw_status mw_rope_table(int n_pos, int Dh, double theta, float* table
 extern "C" mw_status mw_rope_rows(const mw_vis_layout* L, const void* vis, const int32_t* pos, const float* table,
                                   int n_pos, const void* X, void* Y, int H, int Dh, int dtype, int inverse,
                                   void* stream) {
+    if (L && L->kind != MW_VIEWS_EDITS) return MW_ESHAPE;   // rotary kernels read the tile lists
     if (dtype != MW_F32 && dtype != MW_BF16) return MW_EDTYPE;
     if (H <= 0 || Dh <= 0 || Dh % 2 != 0) return MW_ESHAPE;
     mw_status st = rope_args(L, vis, pos, table, n_pos);
@@ -316,6 +322,7 @@ extern "C" mw_status mw_rope_rows(const mw_vis_layout* L, const void* vis, const
 
 extern "C" mw_status mw_masked_attn_rope_ws(const mw_vis_layout* L, int Hq, int Hkv, int Dh, int dtype,
                                             size_t* fwd_bytes, size_t* bwd_bytes) {
+    if (L && L->kind != MW_VIEWS_EDITS) return MW_ESHAPE;   // rotary kernels read the tile lists
     if (!L || !fwd_bytes || !bwd_bytes) return MW_EINVAL;
     if (dtype != MW_F32 && dtype != MW_BF16) return MW_EDTYPE;
     if (Hq <= 0 || Hkv <= 0 || Hq % Hkv != 0 || !(Dh == 64 || Dh == 128)) return MW_ESHAPE;
@@ -329,6 +336,7 @@ extern "C" mw_status mw_masked_attn_rope_fwd(const mw_vis_layout* L, const void*
                                              const float* table, int n_pos, const void* Q, const void* K,
                                              const void* V, void* O, float* LSE, int Hq, int Hkv, int Dh, int dtype,
                                              float scale, void* ws, void* stream) {
+    if (L && L->kind != MW_VIEWS_EDITS) return MW_ESHAPE;   // rotary kernels read the tile lists
     mw_status st = attn_args(L, vis, Hq, Hkv, Dh, dtype, scale);
     if (st != MW_OK) return st;
     if ((st = rope_args(L, vis, pos, table, n_pos)) != MW_OK) return st;
@@ -349,6 +357,7 @@ extern "C" mw_status mw_masked_attn_rope_bwd(const mw_vis_layout* L, const void*
                                              const void* V, const void* O, const void* dO, const float* LSE,
                                              void* dQ, void* dK, void* dV, int Hq, int Hkv, int Dh, int dtype,
                                              float scale, void* ws, void* stream) {
+    if (L && L->kind != MW_VIEWS_EDITS) return MW_ESHAPE;   // rotary kernels read the tile lists
     mw_status st = attn_args(L, vis, Hq, Hkv, Dh, dtype, scale);
     if (st != MW_OK) return st;
     if ((st = rope_args(L, vis, pos, table, n_pos)) != MW_OK) return st;

@@ -405,6 +405,7 @@ using namespace mw;
 
 extern "C" mw_status mw_final_walk(const mw_vis_layout* L, const void* vis, int32_t* walk_index,
                                    int32_t* student_row, int32_t* walk_len, void* stream) {
+    if (L && L->kind != MW_VIEWS_EDITS) return MW_ESHAPE;   // needs single-interval lifetimes
     if (!L) return MW_EINVAL;
     if (L->n_traj == 0) return MW_OK;
     if (!vis || !walk_len || (L->total_tokens > 0 && (!walk_index || !student_row))) return MW_EINVAL;
@@ -471,6 +472,7 @@ extern "C" mw_status mw_forward_kl_bwd(const void* HT, const int32_t* rows_T, co
 }
 
 extern "C" mw_status mw_diverging_rows(const mw_vis_layout* L, const void* vis, uint8_t* out, void* stream) {
+    if (L && L->kind != MW_VIEWS_EDITS) return MW_ESHAPE;   // needs single-interval lifetimes
     if (!L) return MW_EINVAL;
     if (L->total_tokens == 0) return MW_OK;
     if (!vis || !out) return MW_EINVAL;

@@ -130,6 +130,21 @@ extern "C" mw_status mw_visibility_layout(int n_traj, const int32_t* cu, int n_j
     return MW_OK;
 }
 
+extern "C" mw_status mw_events_layout(int n_traj, const int32_t* cu, int n_junc, const int32_t* jt, int n_spans,
+                                      mw_vis_layout* L) {
+    mw_status st = mw_visibility_layout(n_traj, cu, n_junc, jt, n_spans, L);
+    if (st != MW_OK) return st;
+    L->kind = MW_VIEWS_EVENTS;
+    // build workspace: spans (a, b), the per-event span ranges, one flag per token
+    int64_t o = 0;
+    auto take = [&](int64_t bytes) { int64_t r = o; o = align256(o + bytes); return r; };
+    L->ws_off_spans = take(8 * (int64_t)n_spans);
+    L->ws_off_tstat = take(16 * (int64_t)n_junc);
+    L->ws_off_cnt = take(4 * L->total_tokens);
+    L->ws_bytes = o;
+    return MW_OK;
+}
+
 // ---------------------------------------------------------------------------
 // kernels
 
@@ -440,40 +455,121 @@ __global__ void __launch_bounds__(256) k_compact_map(BuildArgs a) {
     for (int r = len + t; r < end; r += 256) src[r] = -1;
 }
 
+// EVENTS records: one block per trajectory replays its events segment by
+// segment into the compact views. view_s = (view_{s-1} without the event's
+// out-spans, order kept) + the in-spans in the given order + the segment's
+// rows. A key is dropped when its flag holds the current segment (set from
+// the out-spans just before); flags never need clearing. Also the per-row
+// compact index sum gives the visible pairs: a row at index c sees c + 1 keys.
+struct EventArgs {
+    int n_traj;
+    const int32_t* traj_tok;
+    const int32_t* traj_tile;
+    const int32_t* traj_seg;
+    const int64_t* traj_km;
+    const int32_t* seg_start;
+    const int32_t* spans;    // [n_spans][2] global positions
+    const int32_t* jtab;     // [n_junc][4] out begin, out end, in begin, in end (into spans)
+    int32_t* flag;           // [total] segment that last evicted the key, -1 never
+    int32_t* seg_len;
+    int32_t* cpos;
+    int32_t* csrc;
+    unsigned long long* pairs;
+};
+
+__global__ void __launch_bounds__(1024) k_event_views(EventArgs a) {
+    __shared__ int wsum[32];
+    __shared__ int n_s;
+    const int b = blockIdx.x;
+    const int t = threadIdx.x, lane = t & 31, w = t >> 5;
+    const int64_t tok0 = a.traj_tok[b];
+    const int T = a.traj_tok[b + 1] - (int)tok0;
+    const int nt = a.traj_tile[b + 1] - a.traj_tile[b];
+    const int g0 = a.traj_seg[b], S = a.traj_seg[b + 1] - g0;
+    if (T == 0) {   // an empty trajectory has one empty segment
+        if (t == 0) {
+            for (int s = 0; s < S; ++s) a.seg_len[g0 + s] = 0;
+            a.pairs[b] = 0;
+        }
+        return;
+    }
+    int32_t* flag = a.flag + tok0;
+    unsigned long long pairs = 0;
+    for (int s = 0; s < S; ++s) {
+        const int64_t base = (a.traj_km[b] + (int64_t)s * nt) * MW_TILE;
+        const int64_t prev = base - (int64_t)nt * MW_TILE;
+        const int lo = a.seg_start[g0 + s], hi = s + 1 < S ? a.seg_start[g0 + s + 1] : T;
+        for (int x = t; x < nt * MW_TILE; x += blockDim.x) a.cpos[base + x] = -1;
+        int n = 0;
+        if (s >= 1) {
+            const int32_t* jt = a.jtab + 4 * (int64_t)(g0 - b + s - 1);   // this trajectory's event s - 1
+            for (int q = jt[0]; q < jt[1]; ++q)
+                for (int j = a.spans[2 * q] + t; j < a.spans[2 * q + 1]; j += blockDim.x) flag[j - tok0] = s;
+            __syncthreads();
+            // ordered compaction of view_{s-1} without the keys flagged s
+            const int Lp = a.seg_len[g0 + s - 1];
+            for (int c0 = 0; c0 < Lp; c0 += blockDim.x) {
+                const int c = c0 + t;
+                const int key = c < Lp ? a.csrc[prev + c] : -1;
+                const int keep = c < Lp && flag[key] != s;
+                const unsigned bal = __ballot_sync(0xffffffffu, keep);
+                if (lane == 0) wsum[w] = __popc(bal);
+                __syncthreads();
+                int before = 0, total = 0;
+                for (int q = 0; q < 32; ++q) {
+                    before += q < w ? wsum[q] : 0;
+                    total += wsum[q];
+                }
+                if (keep) a.csrc[base + n + before + __popc(bal & ((1u << lane) - 1u))] = key;
+                n += total;
+                __syncthreads();
+            }
+            for (int q = jt[2]; q < jt[3]; ++q) {
+                const int ga = a.spans[2 * q], gb = a.spans[2 * q + 1];
+                for (int j = ga + t; j < gb; j += blockDim.x) a.csrc[base + n + (j - ga)] = (int)(j - tok0);
+                n += gb - ga;
+            }
+        }
+        for (int r = lo + t; r < hi; r += blockDim.x) a.csrc[base + n + (r - lo)] = r;
+        const int R = hi - lo;
+        pairs += (unsigned long long)R * (unsigned long long)n + (unsigned long long)R * (R + 1) / 2;
+        n += R;
+        const int end = (n + MW_TILE - 1) / MW_TILE * MW_TILE;
+        for (int c = n + t; c < end; c += blockDim.x) a.csrc[base + c] = -1;
+        if (t == 0) a.seg_len[g0 + s] = n;
+        __syncthreads();
+        for (int c = t; c < n; c += blockDim.x) a.cpos[base + a.csrc[base + c]] = c;
+        __syncthreads();
+    }
+    if (t == 0) {
+        a.pairs[b] = pairs;
+        atomicAdd(&a.pairs[a.n_traj], pairs);
+    }
+}
+
+// View bits from the compact ranks: one warp per (segment, k-tile) entry.
+__global__ void k_event_keymask(int64_t n_keymask, const int32_t* __restrict__ cpos, uint32_t* __restrict__ km) {
+    const int64_t e = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    if (e >= n_keymask) return;
+#pragma unroll
+    for (int w = 0; w < 4; ++w) {
+        const unsigned bal = __ballot_sync(0xffffffffu, cpos[e * MW_TILE + 32 * w + lane] >= 0);
+        if (lane == 0) km[e * 4 + w] = bal;
+    }
+}
+
 }  // namespace
 
 // ---------------------------------------------------------------------------
 
-extern "C" mw_status mw_build_visibility(const mw_vis_layout* L, const int32_t* cu, int n_junc,
-                                         const int32_t* J, const int32_t* jt,
-                                         const int32_t* span_off, const int32_t* spans,
-                                         void* ws, void* vis, void* stream_) {
-    if (!L) return MW_EINVAL;
-    if (n_junc != L->n_junc) return MW_EINVAL;
-    mw_status st = check_shape(L->n_traj, cu, n_junc, jt, L->n_spans);
-    if (st != MW_OK) return st;
+// Host image of the per-trajectory tables (token, tile, segment, triangle and
+// keymask offsets, segment starts, tile owners), copied into the metadata
+// region [off_traj_tok, off_cls) of `vis` with one copy.
+static mw_status copy_meta(const mw_vis_layout* L, const int32_t* cu, int n_junc, const int32_t* J,
+                           const int32_t* jt, void* vis, cudaStream_t stream) {
     const int n_traj = L->n_traj;
-    if (n_traj > 0 && cu[n_traj] != L->total_tokens) return MW_EINVAL;
-    if (n_junc > 0 && (!J || !span_off)) return MW_EINVAL;
-    if (L->n_spans > 0 && !spans) return MW_EINVAL;
-    if (L->vis_bytes > 0 && !vis) return MW_EINVAL;
-    if (L->ws_bytes > 0 && !ws) return MW_EINVAL;
-    if (n_junc > 0 && (span_off[0] != 0 || span_off[n_junc] != L->n_spans)) return MW_EEDITS;
-    // validate junctions and spans (App. B Def. "trajectory tree")
-    for (int k = 0; k < n_junc; ++k) {
-        int b = jt[k];
-        int T = cu[b + 1] - cu[b];
-        if (J[k] < 1 || J[k] > T - 1) return MW_EEDITS;
-        if (k > 0 && jt[k - 1] == b && J[k] <= J[k - 1]) return MW_EEDITS;
-        if (span_off[k + 1] < span_off[k]) return MW_EEDITS;
-        for (int s = span_off[k]; s < span_off[k + 1]; ++s) {
-            int a0 = spans[2 * s], b0 = spans[2 * s + 1];
-            if (!(0 <= a0 && a0 < b0 && b0 <= J[k])) return MW_EEDITS;
-        }
-    }
-    cudaStream_t stream = (cudaStream_t)stream_;
-    if (L->vis_bytes == 0) return MW_OK;
-
+    mw_status st = MW_OK;
     // host-side packing of the small per-trajectory tables
     const int64_t n_tiles = L->n_tiles;
     std::vector<int32_t> traj_tile(n_traj + 1), traj_seg(n_traj + 1), seg_start(L->n_segs),
@@ -502,16 +598,9 @@ extern "C" mw_status mw_build_visibility(const mw_vis_layout* L, const int32_t* 
         traj_km[n_traj] = km;
         traj_seg[n_traj] = segs;
     }
-    std::vector<int32_t> span3(3 * (size_t)L->n_spans);
-    for (int k = 0; k < n_junc; ++k)
-        for (int s = span_off[k]; s < span_off[k + 1]; ++s) {
-            span3[3 * s] = cu[jt[k]] + spans[2 * s];
-            span3[3 * s + 1] = cu[jt[k]] + spans[2 * s + 1];
-            span3[3 * s + 2] = J[k];
-        }
-
     // one contiguous host image of the metadata region [off_traj_tok, off_cls)
-    // plus the span table; two copies.
+    // (a copy from pageable memory: the runtime stages the image before the
+    // call returns)
     const int64_t meta0 = L->off_traj_tok, meta1 = L->off_cls;
     std::vector<char> img(meta1 - meta0, 0);
     auto put = [&](int64_t off, const void* src, size_t bytes) {
@@ -527,6 +616,49 @@ extern "C" mw_status mw_build_visibility(const mw_vis_layout* L, const int32_t* 
     if ((st = cuda_status(cudaMemcpyAsync(at<char>(vis, meta0), img.data(), img.size(),
                                           cudaMemcpyHostToDevice, stream))) != MW_OK)
         return st;
+    return MW_OK;
+}
+
+extern "C" mw_status mw_build_visibility(const mw_vis_layout* L, const int32_t* cu, int n_junc,
+                                         const int32_t* J, const int32_t* jt,
+                                         const int32_t* span_off, const int32_t* spans,
+                                         void* ws, void* vis, void* stream_) {
+    if (!L) return MW_EINVAL;
+    if (L->kind != MW_VIEWS_EDITS || n_junc != L->n_junc) return MW_EINVAL;
+    mw_status st = check_shape(L->n_traj, cu, n_junc, jt, L->n_spans);
+    if (st != MW_OK) return st;
+    const int n_traj = L->n_traj;
+    if (n_traj > 0 && cu[n_traj] != L->total_tokens) return MW_EINVAL;
+    if (n_junc > 0 && (!J || !span_off)) return MW_EINVAL;
+    if (L->n_spans > 0 && !spans) return MW_EINVAL;
+    if (L->vis_bytes > 0 && !vis) return MW_EINVAL;
+    if (L->ws_bytes > 0 && !ws) return MW_EINVAL;
+    if (n_junc > 0 && (span_off[0] != 0 || span_off[n_junc] != L->n_spans)) return MW_EEDITS;
+    // validate junctions and spans (App. B Def. "trajectory tree")
+    for (int k = 0; k < n_junc; ++k) {
+        int b = jt[k];
+        int T = cu[b + 1] - cu[b];
+        if (J[k] < 1 || J[k] > T - 1) return MW_EEDITS;
+        if (k > 0 && jt[k - 1] == b && J[k] <= J[k - 1]) return MW_EEDITS;
+        if (span_off[k + 1] < span_off[k]) return MW_EEDITS;
+        for (int s = span_off[k]; s < span_off[k + 1]; ++s) {
+            int a0 = spans[2 * s], b0 = spans[2 * s + 1];
+            if (!(0 <= a0 && a0 < b0 && b0 <= J[k])) return MW_EEDITS;
+        }
+    }
+    cudaStream_t stream = (cudaStream_t)stream_;
+    if (L->vis_bytes == 0) return MW_OK;
+
+    const int64_t n_tiles = L->n_tiles;
+    if ((st = copy_meta(L, cu, n_junc, J, jt, vis, stream)) != MW_OK) return st;
+    std::vector<int32_t> span3(3 * (size_t)L->n_spans);
+    for (int k = 0; k < n_junc; ++k)
+        for (int s = span_off[k]; s < span_off[k + 1]; ++s) {
+            span3[3 * s] = cu[jt[k]] + spans[2 * s];
+            span3[3 * s + 1] = cu[jt[k]] + spans[2 * s + 1];
+            span3[3 * s + 2] = J[k];
+        }
+
     if (L->n_spans > 0 &&
         (st = cuda_status(cudaMemcpyAsync(at<char>(ws, L->ws_off_spans), span3.data(),
                                           span3.size() * 4, cudaMemcpyHostToDevice, stream))) != MW_OK)
@@ -581,6 +713,121 @@ extern "C" mw_status mw_build_visibility(const mw_vis_layout* L, const int32_t* 
     if (n_tiles > 0) {
         k_fill<<<(unsigned)ceil_div(n_tiles * 32, 256), 256, 0, stream>>>(a);
         k_compact_map<<<(unsigned)L->n_segs, 256, 0, stream>>>(a);
+    }
+    return launch_status();
+}
+
+extern "C" mw_status mw_build_views_events(const mw_vis_layout* L, const int32_t* cu, int n_junc, const int32_t* J,
+                                           const int32_t* jt, const int32_t* out_off, const int32_t* in_off,
+                                           const int32_t* spans, void* ws, void* vis, void* stream_) {
+    if (!L) return MW_EINVAL;
+    if (L->kind != MW_VIEWS_EVENTS || n_junc != L->n_junc) return MW_EINVAL;
+    mw_status st = check_shape(L->n_traj, cu, n_junc, jt, L->n_spans);
+    if (st != MW_OK) return st;
+    const int n_traj = L->n_traj;
+    const int n_spans = L->n_spans;
+    if (n_traj > 0 && cu[n_traj] != L->total_tokens) return MW_EINVAL;
+    if (n_junc > 0 && (!J || !out_off || !in_off)) return MW_EINVAL;
+    if (n_spans > 0 && !spans) return MW_EINVAL;
+    if (L->vis_bytes > 0 && !vis) return MW_EINVAL;
+    if (L->ws_bytes > 0 && !ws) return MW_EINVAL;
+    // validate: junctions ascending inside [1, T-1], spans inside [0, J), and
+    // every retrieved position out of the view when its event fires (replayed
+    // per trajectory on the host, one state byte per position)
+    std::vector<int32_t> jtab(4 * (size_t)n_junc), sp2(2 * (size_t)n_spans);
+    {
+        std::vector<uint8_t> out;
+        int cur = -1;
+        for (int k = 0; k < n_junc; ++k) {
+            const int b = jt[k];
+            const int T = cu[b + 1] - cu[b];
+            if (b != cur) {
+                out.assign((size_t)T, 0);
+                cur = b;
+            } else if (J[k] <= J[k - 1]) {
+                return MW_EEDITS;
+            }
+            if (J[k] < 1 || J[k] > T - 1) return MW_EEDITS;
+            const int r[4] = {out_off[k], out_off[k + 1], in_off[k], in_off[k + 1]};
+            if (r[0] < 0 || r[0] > r[1] || r[1] > n_spans || r[2] < 0 || r[2] > r[3] || r[3] > n_spans)
+                return MW_EEDITS;
+            for (int part = 0; part < 2; ++part)
+                for (int q = r[2 * part]; q < r[2 * part + 1]; ++q) {
+                    const int a0 = spans[2 * q], b0 = spans[2 * q + 1];
+                    if (!(0 <= a0 && a0 < b0 && b0 <= J[k])) return MW_EEDITS;
+                }
+            for (int q = r[0]; q < r[1]; ++q)
+                for (int j = spans[2 * q]; j < spans[2 * q + 1]; ++j) out[j] = 1;
+            for (int q = r[2]; q < r[3]; ++q)
+                for (int j = spans[2 * q]; j < spans[2 * q + 1]; ++j) {
+                    if (!out[j]) return MW_EEDITS;
+                    out[j] = 0;
+                }
+            for (int x = 0; x < 4; ++x) jtab[4 * k + x] = r[x];
+        }
+        for (int k = 0; k < n_junc; ++k)
+            for (int part = 0; part < 2; ++part)
+                for (int q = jtab[4 * k + 2 * part]; q < jtab[4 * k + 2 * part + 1]; ++q) {
+                    sp2[2 * q] = cu[jt[k]] + spans[2 * q];
+                    sp2[2 * q + 1] = cu[jt[k]] + spans[2 * q + 1];
+                }
+    }
+    cudaStream_t stream = (cudaStream_t)stream_;
+    if (L->vis_bytes == 0) return MW_OK;
+    const int64_t n_tiles = L->n_tiles;
+    if ((st = copy_meta(L, cu, n_junc, J, jt, vis, stream)) != MW_OK) return st;
+    if (n_spans > 0 && (st = cuda_status(cudaMemcpyAsync(at<char>(ws, L->ws_off_spans), sp2.data(), sp2.size() * 4,
+                                                         cudaMemcpyHostToDevice, stream))) != MW_OK)
+        return st;
+    if (n_junc > 0 && (st = cuda_status(cudaMemcpyAsync(at<char>(ws, L->ws_off_tstat), jtab.data(), jtab.size() * 4,
+                                                        cudaMemcpyHostToDevice, stream))) != MW_OK)
+        return st;
+    // no tile classes or lists for these views: empty lists, zero classes
+    if ((st = cuda_status(cudaMemsetAsync(at<char>(vis, L->off_cls), 0, (size_t)L->n_tri, stream))) != MW_OK ||
+        (st = cuda_status(cudaMemsetAsync(at<char>(vis, L->off_fwd_ptr), 0, 4 * (size_t)(n_tiles + 1), stream))) !=
+            MW_OK ||
+        (st = cuda_status(cudaMemsetAsync(at<char>(vis, L->off_bwd_ptr), 0, 4 * (size_t)(n_tiles + 1), stream))) !=
+            MW_OK ||
+        (st = cuda_status(cudaMemsetAsync(at<char>(vis, L->off_pairs), 0, 8 * (size_t)(n_traj + 1), stream))) !=
+            MW_OK ||
+        (st = cuda_status(cudaMemsetAsync(at<char>(vis, L->off_status), 0, 32, stream))) != MW_OK ||
+        (st = cuda_status(cudaMemsetAsync(at<char>(ws, L->ws_off_cnt), 0xff, 4 * (size_t)L->total_tokens, stream))) !=
+            MW_OK)
+        return st;
+    BuildArgs a = {};
+    a.n_traj = n_traj;
+    a.total = L->total_tokens;
+    a.omega = at<int32_t>(vis, L->off_omega);
+    a.seg = at<int32_t>(vis, L->off_seg);
+    a.traj_tok = at<int32_t>(vis, L->off_traj_tok);
+    a.traj_seg = at<int32_t>(vis, L->off_traj_seg);
+    a.seg_start = at<int32_t>(vis, L->off_seg_start);
+    EventArgs e;
+    e.n_traj = n_traj;
+    e.traj_tok = at<int32_t>(vis, L->off_traj_tok);
+    e.traj_tile = at<int32_t>(vis, L->off_traj_tile);
+    e.traj_seg = at<int32_t>(vis, L->off_traj_seg);
+    e.traj_km = at<int64_t>(vis, L->off_traj_km);
+    e.seg_start = at<int32_t>(vis, L->off_seg_start);
+    e.spans = at<int32_t>(ws, L->ws_off_spans);
+    e.jtab = at<int32_t>(ws, L->ws_off_tstat);
+    e.flag = at<int32_t>(ws, L->ws_off_cnt);
+    e.seg_len = at<int32_t>(vis, L->off_seg_len);
+    e.cpos = at<int32_t>(vis, L->off_cpos);
+    e.csrc = at<int32_t>(vis, L->off_csrc);
+    e.pairs = at<unsigned long long>(vis, L->off_pairs);
+    if (a.total > 0) {
+        count_launches(1);
+        k_init_tokens<<<(int)std::min<int64_t>(ceil_div(a.total, 256), 152 * 16), 256, 0, stream>>>(a);
+    }
+    if (n_traj > 0) {
+        count_launches(1);
+        k_event_views<<<(unsigned)n_traj, 1024, 0, stream>>>(e);
+    }
+    if (L->n_keymask > 0) {
+        count_launches(1);
+        k_event_keymask<<<(unsigned)ceil_div(L->n_keymask * 32, 256), 256, 0, stream>>>(
+            L->n_keymask, e.cpos, at<uint32_t>(vis, L->off_keymask));
     }
     return launch_status();
 }

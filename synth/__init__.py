@@ -64,12 +64,19 @@ def _rng(seed):
     return np.random.Generator(np.random.Philox(int(seed)))
 
 
-def trajectory(T, K, evict, summary, prompt, Lp, Lo, seed):
+def trajectory(T, K, evict, summary, prompt, Lp, Lo, seed, on_policy_summary=False):
     """One synthetic trajectory (see module docstring).
 
     ``evict`` is ``"half_spans"`` (evict round(0.5 x count) whole spans) or a
     float f (evict spans in shuffled order until at least f x the visible
     observation tokens are gone).
+
+    ``on_policy_summary`` (AgentFold, App. F harness notes: the policy
+    summarises the foldable prefix and the summary is trained): the
+    ``summary`` tokens are policy tokens decoded before the fold, right after
+    the policy span that reaches the target, and the junction is their last
+    token, so they are scored under the pre-fold view and carry loss; later
+    rows see the summary but not the folded spans.
     """
     rng = _rng(seed)
     kinds = np.full(T, PROMPT, dtype=np.int8)
@@ -82,6 +89,12 @@ def trajectory(T, K, evict, summary, prompt, Lp, Lo, seed):
         end = min(pos + int(rng.geometric(1.0 / Lp)), T)
         kinds[pos:end] = POLICY
         J = end - 1
+        if on_policy_summary and k < K and J >= targets[k]:
+            # the summary is decoded by the policy under the pre-fold view;
+            # the fold fires at its last token
+            s_end = min(end + summary, T)
+            kinds[end:s_end] = POLICY
+            J = s_end - 1
         if k < K and J >= targets[k] and J <= T - 1:
             order = rng.permutation(len(visible_obs))
             if evict == "half_spans":
@@ -97,9 +110,12 @@ def trajectory(T, K, evict, summary, prompt, Lp, Lo, seed):
             chosen = sorted(visible_obs[o] for o in take)
             visible_obs = [s for n, s in enumerate(visible_obs) if n not in set(int(t) for t in take)]
             edits.append((int(J), [(int(a), int(b)) for a, b in chosen]))
-            s_end = min(J + 1 + summary, T)
-            kinds[J + 1 : s_end] = SUMMARY
-            pos = s_end
+            if on_policy_summary:
+                pos = J + 1
+            else:
+                s_end = min(J + 1 + summary, T)
+                kinds[J + 1 : s_end] = SUMMARY
+                pos = s_end
             k += 1
             continue
         pos = end
@@ -136,10 +152,10 @@ CONFIGS = {
 }
 
 
-def record(n_traj, T, K, evict, summary, prompt, Lp, Lo, seed_base):
+def record(n_traj, T, K, evict, summary, prompt, Lp, Lo, seed_base, on_policy_summary=False):
     """``n_traj`` trajectories; trajectory b uses seed ``seed_base + b``."""
     lens = T if isinstance(T, (list, tuple)) else [T] * n_traj
-    return Record([trajectory(lens[b], K, evict, summary, prompt, Lp, Lo, seed_base + b)
+    return Record([trajectory(lens[b], K, evict, summary, prompt, Lp, Lo, seed_base + b, on_policy_summary)
                    for b in range(n_traj)])
 
 

@@ -66,6 +66,42 @@ def test_config1_chained_fp32():
     assert_rel(np64(dV), dVr, 1e-4, "dV")
 
 
+def test_on_policy_summaries_chained_fp32():
+    """AgentFold-style record (the policy writes each fold's summary under the
+    pre-fold view; the summary rows carry loss): the whole chain in fp32
+    against the oracle at 1e-4, on every loss row, summary rows included."""
+    rec = synth.record(2, 700, 3, 0.6, 40, 32, 40, 30, 123, on_policy_summary=True)
+    T, Hq, Hkv, Dh, V = rec.total, 2, 2, 64, 1024
+    Q = synth.normal((T, Hq, Dh), 131)
+    K = synth.normal((T, Hkv, Dh), 132)
+    Vv = synth.normal((T, Hkv, Dh), 133)
+    W = synth.normal((V, Hq * Dh), 134, std=0.02)
+    tg = synth.uniform_int(T, V, 135)
+    rows = rec.loss_rows()
+    M = len(rows)
+    adv = synth.normal((M,), 136)
+    scale = Dh ** -0.5
+    Or, _ = OA.attn_fwd(rec.seqlens, rec.edits, np64(Q), np64(K), np64(Vv), scale)
+    Hr = Or.reshape(T, Hq * Dh)
+    lp_r, lse_r = OL.logprob(Hr, np64(W), tg.numpy(), rows)
+    lp_old = torch.tensor(lp_r + np64(synth.normal((M,), 137, std=0.05)), dtype=torch.float32)
+    ratio_r, _, loss_r, g_r = OL.policy_loss(lp_r, np64(lp_old), np64(adv), 0.2, 0.28)
+    dHr, dWr = OL.logprob_loss_bwd(Hr, np64(W), tg.numpy(), rows, lse_r, g_r)
+    dQr, dKr, dVr = OA.attn_bwd(rec.seqlens, rec.edits, np64(Q), np64(K), np64(Vv), dHr.reshape(T, Hq, Dh), scale)
+    dev = lambda t: t.cuda()
+    O, out, dH, dW, dQ, dK, dV = _gpu_chain(rec, dev(Q), dev(K), dev(Vv), dev(W), dev(tg),
+                                            torch.tensor(rows, dtype=torch.int32).cuda(), dev(lp_old),
+                                            dev(adv), 0.2, 0.28)
+    summary_rows = [i for b, t in enumerate(rec.trajs) for J, _ in t.edits
+                    for i in range(sum(rec.seqlens[:b]) + J - 40, sum(rec.seqlens[:b]) + J)]
+    assert set(summary_rows) <= set(rows.tolist())
+    assert_rel(np64(O), Or, 1e-4, "O")
+    assert_rel(np64(out["lp"]), lp_r, 1e-4, "lp")
+    assert abs(out["loss"].item() - loss_r) <= 1e-4 * max(abs(loss_r), 1e-6)
+    for got, ref, what in ((dH, dHr, "dH"), (dW, dWr, "dW"), (dQ, dQr, "dQ"), (dK, dKr, "dK"), (dV, dVr, "dV")):
+        assert_rel(np64(got), ref, 1e-4, what)
+
+
 EPS_LO, EPS_HI = 0.2, 0.28       # App. F.1's clip range, as the bench runs the step
 
 

@@ -143,3 +143,75 @@ def test_rotary_attention_uses_view_order():
     edits = [(4, [(1, 4)])]
     np.testing.assert_allclose(N.attn_fwd(T, [(4, [(1, 4)], [])], Q, K, Vx, 0.35, rope_theta=100.0),
                                A.attn_fwd([T], [edits], Q, K, Vx, 0.35, rope_theta=100.0)[0], rtol=1e-12)
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_build_matches_replay_and_lists(seed):
+    """``build``'s artefacts against the replay formulation and the lists:
+    the visible pairs are the replay mask's, a row's compact index is the
+    number of keys it sees minus one, each segment's membership bits are its
+    view's keys, and csrc / cpos invert each other."""
+    rng = np.random.default_rng(970 + seed)
+    seqlens = [int(rng.integers(130, 300)), int(rng.integers(60, 140))]
+    events = [_random_events(rng, T) for T in seqlens]
+    out = N.build(seqlens, events)
+    assert out["pairs_total"] == sum(int(N.replay_mask(T, e).sum()) for T, e in zip(seqlens, events))
+    base_t, km = 0, 0
+    for T, e in zip(seqlens, events):
+        nt = -(-T // 128)
+        rep = N.replay_mask(T, e)
+        for s, (lo, hi, view) in enumerate(N.live_views(T, e)):
+            base = (km + s * nt) * 128
+            pos = out["cpos"][base: base + nt * 128]
+            src = out["csrc"][base: base + nt * 128]
+            for i in range(lo, hi):
+                assert pos[i] == rep[i].sum() - 1              # row i's index = keys it sees - 1
+            members = np.nonzero(pos >= 0)[0]
+            assert sorted(members.tolist()) == sorted(view)
+            assert all(pos[src[c]] == c for c in range(len(view)))
+            bits = out["keymask"][km + s * nt: km + (s + 1) * nt]
+            got = [128 * t + 32 * w + c for t in range(nt) for w in range(4) for c in range(32)
+                   if (int(bits[t, w]) >> c) & 1]
+            assert got == sorted(view)
+            assert (out["seg"][base_t + lo: base_t + hi] == s).all()
+        base_t += T
+        km += (1 + len(e)) * nt
+
+
+def test_build_memexrl_panel():
+    """The panel's last row sees its prefix list in view order (retrieved
+    y1..y3 after y4) as csrc's first entries."""
+    g, tok, events = _panel()
+    T = len(tok)
+    out = N.build([T], [events])
+    nt = 1
+    S = 1 + len(events)
+    base = (S - 1) * nt * 128
+    view = N.live_views(T, events)[-1][2]
+    assert out["csrc"][base: base + len(view)].tolist() == view
+    assert out["seg_len"][-1] == len(view)
+
+
+@pytest.mark.parametrize("seed", range(3))
+def test_attention_oracle_on_event_views(seed):
+    """``oracle.attention`` run on event views equals SDPA with the replay
+    mask (forward) and autograd through it (backward): its compact-sequence
+    formulas need no single-interval lifetimes."""
+    rng = np.random.default_rng(990 + seed)
+    T = 90
+    events = _random_events(rng, T)
+    Q, K, Vx, dO = (rng.standard_normal((T, h, 8)) for h in (4, 2, 2, 4))
+    O, _ = A.attn_fwd([T], [events], Q, K, Vx, 0.35, views=N.live_views)
+    np.testing.assert_allclose(O[:, :, :], N.attn_fwd(T, events, Q, K, Vx, 0.35), rtol=1e-10, atol=1e-12)
+    mask = torch.from_numpy(N.replay_mask(T, events))
+    q, k, v = (torch.tensor(x, requires_grad=True) for x in (Q, K, Vx))
+    kk = k.repeat_interleave(2, dim=1)
+    vv = v.repeat_interleave(2, dim=1)
+    ref = torch.nn.functional.scaled_dot_product_attention(
+        q.transpose(0, 1), kk.transpose(0, 1), vv.transpose(0, 1), attn_mask=mask, scale=0.35).transpose(0, 1)
+    np.testing.assert_allclose(O, ref.detach().numpy(), rtol=1e-10, atol=1e-12)
+    ref.backward(torch.from_numpy(dO))
+    dQ, dK, dV = A.attn_bwd([T], [events], Q, K, Vx, dO, 0.35, views=N.live_views)
+    np.testing.assert_allclose(dQ, q.grad.numpy(), rtol=1e-9, atol=1e-11)
+    np.testing.assert_allclose(dK, k.grad.numpy(), rtol=1e-9, atol=1e-11)
+    np.testing.assert_allclose(dV, v.grad.numpy(), rtol=1e-9, atol=1e-11)

@@ -272,3 +272,23 @@ def test_compact_maps_inverse(seed):
         assert int((pos[:T] >= 0).sum()) == L
         assert (src[L: -(-L // V.TILE) * V.TILE] == -1).all()
         assert src[L - (hi - lo): L].tolist() == list(range(lo, hi))   # the segment's rows are the tail
+
+
+def test_on_policy_summary_rows_see_the_folded_prefix():
+    """On-policy summaries (AgentFold: the policy summarises the foldable
+    prefix, the summary is trained, then the prefix is replaced by it): the
+    fold's junction is the summary's last token, so the rows that decode the
+    summary see the folded spans, and every later row sees the summary but
+    not the folded spans."""
+    r = synth.record(1, 700, 2, 0.6, 40, 32, 40, 30, 5, on_policy_summary=True)
+    t = r.trajs[0]
+    mask = V.dense_mask(t.T, t.edits)
+    for J, spans in t.edits:
+        gone = [j for a, b in spans for j in range(a, b)]
+        assert gone
+        summary = range(J - 39, J + 1)
+        for i in range(J - 40, J):                  # rows predicting summary tokens
+            assert mask[i, gone].all()
+        for i in range(J, min(t.T, J + 30)):
+            assert not mask[i, gone].any()
+            assert mask[i, list(summary)].all()

@@ -88,3 +88,15 @@ def test_generation_is_deterministic():
     r1 = synth.loss_rows_fraction(1000, 0.7, 5)
     assert (r1 == synth.loss_rows_fraction(1000, 0.7, 5)).all() and len(r1) == 700
     assert (np.diff(r1) > 0).all()
+
+
+def test_on_policy_summaries():
+    """AgentFold-style records: every junction is the last token of an m-token
+    policy span (the summary), whose rows carry loss; no inserted summaries."""
+    r = synth.record(2, 900, 3, 0.6, 48, 32, 40, 30, 77, on_policy_summary=True)
+    for t in r.trajs:
+        assert (t.kinds != synth.SUMMARY).all()
+        rows = set(t.loss_rows.tolist())
+        for J, _ in t.edits:
+            assert (t.kinds[J - 47: J + 1] == synth.POLICY).all()
+            assert all(i in rows for i in range(J - 48, J))     # rows predicting the summary tokens
