@@ -365,7 +365,7 @@ mw_status mw_diverging_rows(const mw_vis_layout* layout, const void* vis, uint8_
 mw_status mw_final_walk(const mw_vis_layout* layout, const void* vis, int32_t* walk_index, int32_t* student_row,
                         int32_t* walk_len, void* stream);
 
-/* Workspace bytes of the forward-KL pair (two float32 values per pair). */
+/* Workspace bytes of the forward-KL pair (kept from forward to backward). */
 mw_status mw_forward_kl_ws(int M, int d, int Vocab, int dtype, size_t* ws_bytes);
 
 /*
@@ -376,9 +376,15 @@ mw_status mw_forward_kl_ws(int M, int d, int Vocab, int dtype, size_t* ws_bytes)
  *   loss  = lam * sum_m kl[m]  (one float32, device),
  * the forward KL with the teacher first. HT [N_T, d], HS [N_S, d], W [Vocab, d]
  * (dtype, W in torch Linear layout), rows_T / rows_S int32 [M] (device),
- * rows_S distinct (M <= N_S), rows_T may repeat. Both lse per pair are kept in `ws` for the backward.
- * Float32 arithmetic on CUDA cores; d <= 256 (MW_ESHAPE above). lam >= 0 and
- * finite (MW_EINVAL). M = 0 gives loss = 0.
+ * rows_S distinct (M <= N_S), rows_T may repeat. lam >= 0 and finite
+ * (MW_EINVAL). M = 0 gives loss = 0.
+ * bf16 with d a multiple of 64 that the LM head's CTA groups split (as for
+ * mw_logprob_loss_fwd): tensor cores. For the teacher rows and then the
+ * student rows, one fused pass over the vocabulary gives lse and
+ * E = sum_v p_v W_v; since z = h W^T, E_pT[zT - zS] = (hT - hS) . E_T, so
+ * kl = (hT - hS) . E_T - lse_T + lse_S. Otherwise (fp32; bf16 with d <= 256
+ * not split that way): float32 on CUDA cores. `ws` keeps lse (and E) for the
+ * backward.
  */
 mw_status mw_forward_kl_fwd(const void* HT, const int32_t* rows_T, const void* HS, const int32_t* rows_S, int M,
                             const void* W, int N_T, int N_S, int d, int Vocab, int dtype, float lam,
@@ -389,11 +395,17 @@ mw_status mw_forward_kl_fwd(const void* HT, const int32_t* rows_T, const void* H
  * (stop-gradient): dzS = lam * dloss * (softmax(zS) - softmax(zT)),
  *   dHS[rows_S[m]] = dzS_m W (other rows of dHS = 0),  dW = sum_m dzS_m^T hS_m.
  * dHS [N_S, d] in dtype and dW [Vocab, d] float32 are overwritten. Needs the
- * forward's `ws`.
+ * forward's `ws` (the tensor-core path also uses it as scratch). Tensor cores:
+ * dHS = lam dloss (E_S - E_T) from the forward, dW by two vocabulary-
+ * stationary passes (the student's softmax, then the teacher's added in).
  */
 mw_status mw_forward_kl_bwd(const void* HT, const int32_t* rows_T, const void* HS, const int32_t* rows_S, int M,
                             const void* W, int N_T, int N_S, int d, int Vocab, int dtype, float lam, float dloss,
-                            const void* ws, void* dHS, float* dW, void* stream);
+                            void* ws, void* dHS, float* dW, void* stream);
+
+/* Synchronise `stream` and report a bounded device wait of the tensor-core
+ * KL passes that gave up (MW_ETIMEOUT), from `ws`. */
+mw_status mw_forward_kl_check_status(int M, int d, int Vocab, int dtype, void* ws, void* stream);
 
 /* Bytes of device workspace the log-prob loss forward/backward pair needs. */
 mw_status mw_logprob_ws(int N, int M, int d, int Vocab, int dtype, size_t* ws_bytes);

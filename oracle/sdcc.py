@@ -111,6 +111,19 @@ def forward_kl(HT, HS, W):
     return kl, dz @ W, dz.T @ HS
 
 
+def forward_kl_dw_vocab(HT, HS, W, vocab):
+    """``forward_kl``'s dW for a few vocabulary rows only (sampled checks on
+    big heads): each row's full softmax of both sides, then
+    ``dW[v] = sum_m (pS - pT)_{m,v} HS_m`` for the selected v."""
+    HT = np.asarray(HT, dtype=np.float64)
+    HS = np.asarray(HS, dtype=np.float64)
+    W = np.asarray(W, dtype=np.float64)
+    vocab = np.asarray(vocab, dtype=np.int64)
+    lt = _log_softmax(HT @ W.T)[:, vocab]
+    ls = _log_softmax(HS @ W.T)[:, vocab]
+    return (np.exp(ls) - np.exp(lt)).T @ HS
+
+
 def sdcc_penalty(HT, HS, W, diverging, lam):
     """The SDCC term of Eq. "soft_loss" for one trajectory: ``lam`` times the
     sum of the forward KLs over the diverging rows (leaf-gated: rows that do

@@ -71,6 +71,7 @@ _SIGS = {
     "mw_forward_kl_ws": (_I, [_I, _I, _I, _I, ctypes.POINTER(ctypes.c_size_t)]),
     "mw_forward_kl_fwd": (_I, [_P, _P, _P, _P, _I, _P, _I, _I, _I, _I, _I, _F, _P, _P, _P, _P]),
     "mw_forward_kl_bwd": (_I, [_P, _P, _P, _P, _I, _P, _I, _I, _I, _I, _I, _F, _F, _P, _P, _P, _P]),
+    "mw_forward_kl_check_status": (_I, [_I, _I, _I, _I, _P, _P]),
     "mw_rope_table": (_I, [_I, _I, ctypes.c_double, _P, _P]),
     "mw_rope_rows": (_I, [_LP, _P, _P, _P, _I, _P, _P, _I, _I, _I, _I, _P]),
     "mw_masked_attn_rope_ws": (_I, [_LP, _I, _I, _I, _I, ctypes.POINTER(ctypes.c_size_t),
@@ -445,6 +446,13 @@ def forward_kl_fwd(HT, rows_T, HS, rows_S, W, lam=1.0, stream=None):
                                     HS.shape[0], d, V, _dtype_code(HT), float(lam), _ptr(kl), _ptr(loss), _ptr(ws),
                                     _stream(stream)), "mw_forward_kl_fwd")
     return kl[:M], loss, ws
+
+
+def forward_kl_check_status(rows_T, HT, W, ws, stream=None):
+    """Synchronise and raise if a bounded device wait of the tensor-core KL
+    passes gave up (mw_forward_kl_check_status)."""
+    _check(_lib().mw_forward_kl_check_status(int(rows_T.numel()), HT.shape[1], W.shape[0], _dtype_code(HT),
+                                             _ptr(ws), _stream(stream)), "mw_forward_kl_check_status")
 
 
 def forward_kl_bwd(HT, rows_T, HS, rows_S, W, ws, lam=1.0, dloss=1.0, stream=None):

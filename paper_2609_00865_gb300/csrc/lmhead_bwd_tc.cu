@@ -79,6 +79,7 @@ constexpr float kGuard = 96.f;
 
 struct LmBwdParams {
     int mode;            // 1: dW pass, 2: fused forward (E, row sums, target logit)
+    int add;             // mode 1: add the pass's dW to the array instead of overwriting it
     int C, ds;           // cluster size, d-slice (<= 256)
     int L, R;            // accumulation lag in steps, ring depth R = L + 2
     int KD;              // 64-wide k-slices of d
@@ -377,9 +378,22 @@ __global__ void __launch_bounds__(NT, 1)
                 tmem_wait_ld();
                 if (!valid) continue;
                 float* dst = (p.mode == 1 ? p.dW : p.E) + orow * d + col0 + c0;
+                if (p.add) {
 #pragma unroll
-                for (int x = 0; x < 8; ++x)
-                    reinterpret_cast<uint4*>(dst)[x] = make_uint4(o[4 * x], o[4 * x + 1], o[4 * x + 2], o[4 * x + 3]);
+                    for (int x = 0; x < 8; ++x) {
+                        float4 q = reinterpret_cast<float4*>(dst)[x];
+                        q.x += __uint_as_float(o[4 * x]);
+                        q.y += __uint_as_float(o[4 * x + 1]);
+                        q.z += __uint_as_float(o[4 * x + 2]);
+                        q.w += __uint_as_float(o[4 * x + 3]);
+                        reinterpret_cast<float4*>(dst)[x] = q;
+                    }
+                } else {
+#pragma unroll
+                    for (int x = 0; x < 8; ++x)
+                        reinterpret_cast<uint4*>(dst)[x] =
+                            make_uint4(o[4 * x], o[4 * x + 1], o[4 * x + 2], o[4 * x + 3]);
+                }
             }
             tc_fence_before();
             mbar_arrive(&acc_free);
@@ -660,6 +674,65 @@ __global__ void k_lm_dh_from_e(int M, int d, const __nv_bfloat16* __restrict__ W
     }
 }
 
+// SDCC's forward KL from the fused passes of the teacher and the student
+// rows of each pair (E_T, E_S: sum_v p~ W_v; linv: 1 / l). With z = h W^T,
+// E_{p_T}[z_T - z_S] = (h_T - h_S) . Ebar_T, Ebar_T = E_T / l_T, so
+//   KL(p_T || p_S) = (h_T - h_S) . Ebar_T - lse_T + lse_S.
+// One warp per pair, float32 over d.
+__global__ void k_kl_from_e(int M, int d, const __nv_bfloat16* __restrict__ hgT, const __nv_bfloat16* __restrict__ hgS,
+                            const float* __restrict__ ET, const float* __restrict__ linvT,
+                            const float* __restrict__ lseT, const float* __restrict__ lseS, float* __restrict__ kl) {
+    const int m = (int)((blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5);
+    const int lane = threadIdx.x & 31;
+    if (m >= M) return;
+    const uint4* t8 = reinterpret_cast<const uint4*>(hgT + (int64_t)m * d);
+    const uint4* s8 = reinterpret_cast<const uint4*>(hgS + (int64_t)m * d);
+    const float4* e4 = reinterpret_cast<const float4*>(ET + (int64_t)m * d);
+    float a = 0.f;
+    for (int k = lane; k < d / 8; k += 32) {
+        const uint4 ut = t8[k], us = s8[k];
+        const float4 e0 = e4[2 * k], e1 = e4[2 * k + 1];
+        const uint32_t tw[4] = {ut.x, ut.y, ut.z, ut.w}, sw[4] = {us.x, us.y, us.z, us.w};
+        const float ev[8] = {e0.x, e0.y, e0.z, e0.w, e1.x, e1.y, e1.z, e1.w};
+#pragma unroll
+        for (int x = 0; x < 4; ++x) {
+            a = fmaf(__uint_as_float(tw[x] << 16) - __uint_as_float(sw[x] << 16), ev[2 * x], a);
+            a = fmaf(__uint_as_float(tw[x] & 0xffff0000u) - __uint_as_float(sw[x] & 0xffff0000u), ev[2 * x + 1], a);
+        }
+    }
+    a = warp_sum(a);
+    if (lane == 0) kl[m] = a * linvT[m] - lseT[m] + lseS[m];
+}
+
+// dH_S of the KL: c (Ebar_S - Ebar_T) at the student row of each pair (bf16).
+// Both products are rounded before the difference (no fused multiply-add), so
+// a student equal to its teacher gets exactly 0.
+__global__ void k_kl_dh_from_e(int M, int d, const float* __restrict__ ES, const float* __restrict__ linvS,
+                               const float* __restrict__ ET, const float* __restrict__ linvT, float c,
+                               const int32_t* __restrict__ rowsS, __nv_bfloat16* __restrict__ dHS) {
+    for (int m = blockIdx.x; m < M; m += gridDim.x) {
+        const float as = c * linvS[m], at_ = c * linvT[m];
+        const float4* s4 = reinterpret_cast<const float4*>(ES + (int64_t)m * d);
+        const float4* t4 = reinterpret_cast<const float4*>(ET + (int64_t)m * d);
+        uint2* out = reinterpret_cast<uint2*>(dHS + (int64_t)rowsS[m] * d);
+        for (int k = threadIdx.x; k < d / 4; k += blockDim.x) {
+            const float4 x = s4[k], y = t4[k];
+            out[k] = make_uint2(pack_bf16(__fmul_rn(as, x.x) - __fmul_rn(at_, y.x),
+                                          __fmul_rn(as, x.y) - __fmul_rn(at_, y.y)),
+                                pack_bf16(__fmul_rn(as, x.z) - __fmul_rn(at_, y.z),
+                                          __fmul_rn(as, x.w) - __fmul_rn(at_, y.w)));
+        }
+    }
+}
+
+// Per-pair parameters of a softmax-only dW pass: dz_v = -x p_v (no target).
+__global__ void k_kl_par(int M, int M_pad, float x, const float* __restrict__ lse, float4* __restrict__ par) {
+    const int m = blockIdx.x * blockDim.x + threadIdx.x;
+    if (m >= M_pad) return;
+    par[m] = m < M ? make_float4(x, lse[m] * LOG2E_B, __int_as_float(-1), 1.f)
+                   : make_float4(0.f, 0.f, __int_as_float(-1), 0.f);
+}
+
 // Group sizes whose d-slice fits beside a 256-column logit tile in TMEM
 // (ds <= 256) and keeps 32-column output chunks (ds % 32 == 0).
 bool slice_ok(int d, int C) { return d % C == 0 && d / C <= 256 && (d / C) % 32 == 0; }
@@ -678,8 +751,12 @@ int group_size(int d) {
 }
 
 // One launch of k_lm_bwd_tc in `mode` over M loss rows; the scratch holds the
-// per-row parameters (filled by the caller), the ring and its counters.
-mw_status launch_group(LmBwdParams p, const void* W, int d, const void* Hg, void* scratch, cudaStream_t s) {
+// per-row parameters (filled by the caller), the ring and its counters. Mode
+// 1 forms the logits from the rows Hg and takes the dW product with the rows
+// HgA (the same rows unless the caller passes others).
+mw_status launch_group(LmBwdParams p, const void* W, int d, const void* Hg, void* scratch, cudaStream_t s,
+                       const void* HgA = nullptr) {
+    if (!HgA) HgA = Hg;
     const int M = p.M, V = p.V;
     const int M_pad = (int)ceil_div(M, 128) * 128;
     __nv_bfloat16* ring = at<__nv_bfloat16>(scratch, align256(16 * (int64_t)M_pad));
@@ -717,7 +794,7 @@ mw_status launch_group(LmBwdParams p, const void* W, int d, const void* Hg, void
     const bool ok = rows_x ? (tmap_bf16_2d(&tx, Hg, M_pad, d, d, 128, 64) && tmap_bf16_2d(&tyz, W, V, d, d, NY, 64) &&
                               tmap_bf16_2d(&tya, W, V, d, d, 64, 64))
                            : (tmap_bf16_2d(&tx, W, V, d, d, 128, 64) && tmap_bf16_2d(&tyz, Hg, M_pad, d, d, NY, 64) &&
-                              tmap_bf16_2d(&tya, Hg, M_pad, d, d, 64, 64));
+                              tmap_bf16_2d(&tya, HgA, M_pad, d, d, 64, 64));
     if (!ok || !tmap_bf16_2d(&dm, ring, ring_rows, NY, NY, 128, 64)) return MW_ECUDA;
 
     p.C = C;
@@ -836,5 +913,107 @@ mw_status lm_bwd_tc(const void* W, int M, int N, int d, int V, const int32_t* ro
         M, d, (const __nv_bfloat16*)W, tg, a.E, a.linv, g, dloss, rows, (__nv_bfloat16*)dH);
     return launch_status();
 }
+
+// SDCC's forward KL on the tensor cores (§5, Eq. "soft_loss"). Workspace:
+// gathered teacher and student rows, the reference prepass's partials,
+// dummy targets / target logits / log-probs, lse of both, status words, the
+// group passes' scratch and the two fused forwards' arrays (E, 1 / l).
+struct KlWs {
+    int64_t hgT, hgS, tg, part, zt, lp, lseT, lseS, status, scratch, fwdT, fwdS, bytes;
+};
+static KlWs kl_ws_layout(int M, int d) {
+    KlWs w;
+    const int64_t M_pad = ceil_div(M, 128) * 128;
+    int64_t o = 0;
+    auto take = [&](int64_t b) { int64_t r = o; o = align256(o + b); return r; };
+    w.hgT = take(2 * M_pad * d);
+    w.hgS = take(2 * M_pad * d);
+    w.tg = take(4 * M_pad);
+    w.part = take(8 * 64 * M_pad);
+    w.zt = take(4 * M_pad);
+    w.lp = take(4 * M_pad);
+    w.lseT = take(4 * M_pad);
+    w.lseS = take(4 * M_pad);
+    w.status = take(32);
+    w.scratch = take(lm_bwd_tc_scratch(M, d));
+    w.fwdT = take(lm_fwd_grp_bytes(M, d));
+    w.fwdS = take(lm_fwd_grp_bytes(M, d));
+    w.bytes = o;
+    return w;
+}
+
+int64_t kl_tc_ws(int M, int d) { return lm_bwd_tc_supported(d) ? kl_ws_layout(M, d).bytes : 0; }
+
+mw_status lm_ref_tc(const void*, const void*, const int32_t*, const int32_t*, int, int, int, void*, int32_t*, float2*,
+                    float*, float4*, int32_t*, cudaStream_t);
+
+// Forward: for the teacher rows and then the student rows, the reference
+// prepass and the fused pass (lse, E, 1 / l); then KL per pair.
+mw_status kl_fwd_tc(const void* HT, const int32_t* rowsT, const void* HS, const int32_t* rowsS, int M, const void* W,
+                    int d, int V, float* kl, void* ws, cudaStream_t s) {
+    if (!lm_bwd_tc_supported(d)) return MW_ESHAPE;
+    const KlWs w = kl_ws_layout(M, d);
+    mw_status st = cuda_status(cudaMemsetAsync(at<char>(ws, w.status), 0, 32, s));
+    if (st == MW_OK) st = cuda_status(cudaMemsetAsync(at<char>(ws, w.zt), 0, 4 * (size_t)M, s));
+    for (int side = 0; st == MW_OK && side < 2; ++side) {
+        const void* H = side == 0 ? HT : HS;
+        const int32_t* rows = side == 0 ? rowsT : rowsS;
+        void* hg = at<char>(ws, side == 0 ? w.hgT : w.hgS);
+        st = lm_ref_tc(H, W, nullptr, rows, M, d, V, hg, at<int32_t>(ws, w.tg), at<float2>(ws, w.part),
+                       at<float>(ws, w.zt), at<float4>(ws, w.scratch), at<int32_t>(ws, w.status), s);
+        if (st == MW_OK)
+            st = lm_fwd_grp_tc(W, M, d, V, hg, at<int32_t>(ws, w.tg), at<float>(ws, w.zt),
+                               at<float>(ws, side == 0 ? w.lseT : w.lseS), at<float>(ws, w.lp),
+                               at<int32_t>(ws, w.status), at<char>(ws, w.scratch),
+                               at<char>(ws, side == 0 ? w.fwdT : w.fwdS), s);
+    }
+    if (st != MW_OK) return st;
+    const GrpArrays aT = grp_arrays(at<char>(ws, w.fwdT), M, d);
+    count_launches(1);
+    k_kl_from_e<<<(unsigned)ceil_div((int64_t)M * 32, 256), 256, 0, s>>>(
+        M, d, at<__nv_bfloat16>(ws, w.hgT), at<__nv_bfloat16>(ws, w.hgS), aT.E, aT.linv, at<float>(ws, w.lseT),
+        at<float>(ws, w.lseS), kl);
+    return launch_status();
+}
+
+// Backward (teacher stopped), c = lam dloss: dH_S = c (Ebar_S - Ebar_T) at
+// the student rows; dW = c sum_m (p_S - p_T) h_S as two dW passes over the
+// same rows' product: softmax-only with the student's logits, then with the
+// teacher's logits added in.
+mw_status kl_bwd_tc(const int32_t* rowsS, int M, const void* W, int N_S, int d, int V, float c, void* ws,
+                    void* dHS, float* dW, cudaStream_t s) {
+    if (!lm_bwd_tc_supported(d)) return MW_ESHAPE;
+    mw_status st = cuda_status(cudaMemsetAsync(dHS, 0, (size_t)N_S * d * 2, s));
+    if (st != MW_OK) return st;
+    if (M == 0) return cuda_status(cudaMemsetAsync(dW, 0, (size_t)V * d * 4, s));
+    const KlWs w = kl_ws_layout(M, d);
+    const int M_pad = (int)ceil_div(M, 128) * 128;
+    if ((st = cuda_status(cudaMemsetAsync(at<char>(ws, w.status), 0, 32, s))) != MW_OK) return st;
+    const GrpArrays aT = grp_arrays(at<char>(ws, w.fwdT), M, d), aS = grp_arrays(at<char>(ws, w.fwdS), M, d);
+    count_launches(1);
+    k_kl_dh_from_e<<<(unsigned)std::min(M, 8 * 152), 128, 0, s>>>(M, d, aS.E, aS.linv, aT.E, aT.linv, c, rowsS,
+                                                                  (__nv_bfloat16*)dHS);
+    if ((st = launch_status()) != MW_OK) return st;
+    for (int side = 0; side < 2; ++side) {   // student: dz = c p_S; teacher: dz = -c p_T
+        count_launches(1);
+        k_kl_par<<<(unsigned)ceil_div(M_pad, 256), 256, 0, s>>>(M, M_pad, side == 0 ? -c : c,
+                                                                at<float>(ws, side == 0 ? w.lseS : w.lseT),
+                                                                at<float4>(ws, w.scratch));
+        if ((st = launch_status()) != MW_OK) return st;
+        LmBwdParams p = {};
+        p.mode = 1;
+        p.add = side;
+        p.M = M;
+        p.V = V;
+        p.dW = dW;
+        p.status = at<int32_t>(ws, w.status);
+        if ((st = launch_group(p, W, d, at<char>(ws, side == 0 ? w.hgS : w.hgT), at<char>(ws, w.scratch), s,
+                               at<char>(ws, w.hgS))) != MW_OK)
+            return st;
+    }
+    return MW_OK;
+}
+
+int32_t* kl_tc_status(int M, int d, void* ws) { return at<int32_t>(ws, kl_ws_layout(M, d).status); }
 
 }  // namespace mw

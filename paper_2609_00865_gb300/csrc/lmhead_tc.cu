@@ -217,7 +217,7 @@ __global__ void k_lm_gather(int M, int M_pad, int d, const __nv_bfloat16* __rest
         uint4 val = make_uint4(0, 0, 0, 0);
         if (m < M) val = reinterpret_cast<const uint4*>(H + (int64_t)rows[m] * d)[k];
         reinterpret_cast<uint4*>(Hg + (int64_t)m * d)[k] = val;
-        if (k == 0) tg[m] = m < M ? targets[rows[m]] : -1;
+        if (k == 0) tg[m] = m < M && targets ? targets[rows[m]] : -1;   // no targets: -1
     }
 }
 

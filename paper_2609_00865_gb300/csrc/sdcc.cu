@@ -415,22 +415,49 @@ extern "C" mw_status mw_final_walk(const mw_vis_layout* L, const void* vis, int3
     return launch_status();
 }
 
+namespace mw {
+bool lm_bwd_tc_supported(int d);
+int64_t kl_tc_ws(int M, int d);
+mw_status kl_fwd_tc(const void*, const int32_t*, const void*, const int32_t*, int, const void*, int, int, float*,
+                    void*, cudaStream_t);
+mw_status kl_bwd_tc(const int32_t*, int, const void*, int, int, int, float, void*, void*, float*, cudaStream_t);
+int32_t* kl_tc_status(int M, int d, void* ws);
+}  // namespace mw
+
+// bf16 with a hidden size the LM head's CTA groups can split runs on the
+// tensor cores; fp32 (and bf16 with other d <= 256) on CUDA cores.
+static bool kl_tc(int d, int dtype) { return dtype == MW_BF16 && lm_bwd_tc_supported(d); }
+
 static mw_status kl_args(int M, int N_T, int N_S, int d, int Vocab, int dtype) {
     if (M < 0 || N_T < 0 || N_S < 0 || d <= 0 || Vocab <= 0) return MW_ESHAPE;
     if (M > N_S) return MW_ESHAPE;        // student rows are distinct; teacher rows may repeat
     if (M > 0 && N_T == 0) return MW_ESHAPE;
     if (dtype != MW_F32 && dtype != MW_BF16) return MW_EDTYPE;
-    if (d > 256) return MW_ESHAPE;
+    if (!kl_tc(d, dtype) && d > 256) return MW_ESHAPE;
     return MW_OK;
 }
 
-// Workspace: lse of the teacher and of the student per pair.
+// Workspace: CUDA cores, lse of the teacher and of the student per pair;
+// tensor cores, the fused passes' arrays (see kl_tc_ws).
 extern "C" mw_status mw_forward_kl_ws(int M, int d, int Vocab, int dtype, size_t* bytes) {
     if (!bytes) return MW_EINVAL;
     mw_status st = kl_args(M, M, M, d, Vocab, dtype);
     if (st != MW_OK) return st;
-    *bytes = (size_t)(2 * align256(4 * (int64_t)M) + 256);
+    *bytes = kl_tc(d, dtype) ? (size_t)kl_tc_ws(M, d) : (size_t)(2 * align256(4 * (int64_t)M) + 256);
     return MW_OK;
+}
+
+extern "C" mw_status mw_forward_kl_check_status(int M, int d, int Vocab, int dtype, void* ws, void* stream) {
+    mw_status st = kl_args(M, M, M, d, Vocab, dtype);
+    if (st != MW_OK) return st;
+    if (!ws) return MW_EINVAL;
+    if (!kl_tc(d, dtype)) return cuda_status(cudaStreamSynchronize((cudaStream_t)stream));
+    int32_t h[8];
+    if ((st = cuda_status(cudaMemcpyAsync(h, kl_tc_status(M, d, ws), sizeof(h), cudaMemcpyDeviceToHost,
+                                          (cudaStream_t)stream))) != MW_OK)
+        return st;
+    if ((st = cuda_status(cudaStreamSynchronize((cudaStream_t)stream))) != MW_OK) return st;
+    return h[1] ? MW_ETIMEOUT : MW_OK;
 }
 
 extern "C" mw_status mw_forward_kl_fwd(const void* HT, const int32_t* rows_T, const void* HS, const int32_t* rows_S,
@@ -449,6 +476,12 @@ extern "C" mw_status mw_forward_kl_fwd(const void* HT, const int32_t* rows_T, co
         k_kl_loss<<<1, 1024, 0, s>>>(0, kl, lam, loss);
         return launch_status();
     }
+    if (kl_tc(d, dtype)) {
+        if ((st = kl_fwd_tc(HT, rows_T, HS, rows_S, M, W, d, Vocab, kl, ws, s)) != MW_OK) return st;
+        count_launches(1);
+        k_kl_loss<<<1, 1024, 0, s>>>(M, kl, lam, loss);
+        return launch_status();
+    }
     return dtype == MW_F32 ? kl_fwd_t<float>(HT, rows_T, HS, rows_S, M, W, d, Vocab, lam, kl, loss, lseT, lseS, s)
                            : kl_fwd_t<__nv_bfloat16>(HT, rows_T, HS, rows_S, M, W, d, Vocab, lam, kl, loss, lseT,
                                                      lseS, s);
@@ -456,7 +489,7 @@ extern "C" mw_status mw_forward_kl_fwd(const void* HT, const int32_t* rows_T, co
 
 extern "C" mw_status mw_forward_kl_bwd(const void* HT, const int32_t* rows_T, const void* HS, const int32_t* rows_S,
                                        int M, const void* W, int N_T, int N_S, int d, int Vocab, int dtype,
-                                       float lam, float dloss, const void* ws, void* dHS, float* dW, void* stream) {
+                                       float lam, float dloss, void* ws, void* dHS, float* dW, void* stream) {
     mw_status st = kl_args(M, N_T, N_S, d, Vocab, dtype);
     if (st != MW_OK) return st;
     if (!(lam >= 0.f) || !isfinite(lam) || !isfinite(dloss)) return MW_EINVAL;
@@ -466,6 +499,7 @@ extern "C" mw_status mw_forward_kl_bwd(const void* HT, const int32_t* rows_T, co
     const float* lseT = at<float>(ws, 0);
     const float* lseS = at<float>(ws, align256(4 * (int64_t)M));
     const float c = lam * dloss;
+    if (kl_tc(d, dtype)) return kl_bwd_tc(rows_S, M, W, N_S, d, Vocab, c, ws, dHS, dW, s);
     return dtype == MW_F32
                ? kl_bwd_t<float>(HT, rows_T, HS, rows_S, M, W, N_S, d, Vocab, c, lseT, lseS, dHS, dW, s)
                : kl_bwd_t<__nv_bfloat16>(HT, rows_T, HS, rows_S, M, W, N_S, d, Vocab, c, lseT, lseS, dHS, dW, s);

@@ -263,3 +263,12 @@ def test_sdcc_objective_without_edits_is_the_task_loss():
     obj, task, pen = S.sdcc_objective(T, [], Q, K, Vx, W, rng.integers(0, 20, T), rows,
                                       np.full(T, -3.0), rng.standard_normal(T), 0.1, 0.5)
     assert pen == 0.0 and obj == task
+
+
+def test_forward_kl_dw_vocab_matches_full():
+    """The sampled-vocabulary dW equals the full dW's rows."""
+    rng = np.random.default_rng(31)
+    HT, HS, W = rng.standard_normal((7, 16)), rng.standard_normal((7, 16)), 0.4 * rng.standard_normal((50, 16))
+    _, _, dW = S.forward_kl(HT, HS, W)
+    vocab = np.array([0, 3, 17, 49])
+    np.testing.assert_allclose(S.forward_kl_dw_vocab(HT, HS, W, vocab), dW[vocab], rtol=1e-12, atol=1e-14)

@@ -96,6 +96,22 @@ def _kl_run(HT, HS, W, rows_T, rows_S, lam, dloss):
     return kl, loss, dHS, dW
 
 
+def _assert_kl_bf16(kl, HT, HS, W, rows_T, rows_S):
+    """The tensor-core KL takes E_pT[z_S] = h_S . sum_v pT_v W_v with the
+    weights pT rounded to bf16 (relative error <= 2^-9 each), so per pair
+    |dKL| <= 2^-9 sum_v pT_v |zT_v - zS_v| plus float32 rounding; the bar is
+    twice that bound plus 1e-3, with the logits from a plain float64 product."""
+    from oracle import sdcc as OSd
+    rt, rs = rows_T.numpy().astype(np.int64), rows_S.numpy().astype(np.int64)
+    klr, _, _ = OSd.forward_kl(np64(HT)[rt], np64(HS)[rs], np64(W))
+    zt, zs = np64(HT)[rt] @ np64(W).T, np64(HS)[rs] @ np64(W).T
+    pt = np.exp(zt - zt.max(axis=1, keepdims=True))
+    pt /= pt.sum(axis=1, keepdims=True)
+    bound = 2.0 ** -8 * (pt * np.abs(zt - zs)).sum(axis=1) + 1e-3
+    err = np.abs(np64(kl) - klr)
+    assert (err <= bound).all(), f"kl: worst err / bound {float((err / bound).max()):.3g}"
+
+
 def _kl_ref(HT, HS, W, rows_T, rows_S, lam, dloss):
     from oracle import sdcc as OSd
     rt, rs = rows_T.numpy().astype(np.int64), rows_S.numpy().astype(np.int64)
@@ -115,13 +131,16 @@ def test_forward_kl_matches_oracle(dtype):
     case = _kl_case(37, 50, 45, d, 3001, 7, dtype)
     kl, loss, dHS, dW = _kl_run(*case, lam=0.1, dloss=1.3)
     klr, lossr, dHSr, dWr = _kl_ref(*case, lam=0.1, dloss=1.3)
-    assert_rel(np64(kl), klr, 1e-4, "kl")
-    assert_rel(np64(loss), [lossr], 1e-4, "loss")
-    if dtype == torch.float32:
+    if dtype == torch.float32:      # CUDA cores, float32 throughout
+        assert_rel(np64(kl), klr, 1e-4, "kl")
+        assert_rel(np64(loss), [lossr], 1e-4, "loss")
         assert_rel(np64(dHS), dHSr, 1e-4, "dHS")
-    else:
+        assert_rel(np64(dW), dWr, 1e-4, "dW")
+    else:                           # tensor cores: bf16 softmax weights in E
+        _assert_kl_bf16(kl, *case)
+        assert abs(float(loss.item()) - lossr) <= 1e-3 * abs(lossr)
         assert_grad_bf16(np64(dHS), dHSr, "dHS")
-    assert_rel(np64(dW), dWr, 1e-4, "dW")
+        assert_grad_bf16(np64(dW), dWr, "dW")
     untouched = np.setdiff1d(np.arange(case[1].shape[0]), case[4].numpy())
     assert not np64(dHS)[untouched].any()
 
@@ -133,6 +152,43 @@ def test_forward_kl_of_equal_rows_is_zero():
     assert_maxabs(np64(kl), np.zeros(10), 1e-5, "kl")
     assert_maxabs(np64(dHS), np.zeros(tuple(HT.shape)), 1e-6, "dHS")
     assert_maxabs(np64(dW), np.zeros(tuple(W.shape)), 1e-6, "dW")
+
+
+def test_forward_kl_tc_equal_rows_is_exactly_zero():
+    """Tensor-core path: a student equal to its teacher gives KL 0, dHS 0 and
+    dW 0 bit for bit (both passes form the same numbers; the two dW passes
+    cancel exactly)."""
+    HT, _, W, _, _ = _kl_case(40, 40, 40, 128, 1000, 19, torch.bfloat16)
+    rows = torch.arange(40, dtype=torch.int32)
+    kl, loss, dHS, dW = _kl_run(HT, HT, W, rows, rows, 0.5, 1.0)
+    assert not np64(kl).any() and not np64(dHS).any() and not np64(dW).any()
+
+
+@pytest.mark.parametrize("d,V", [(1536, 151936), (3584, 152064)])
+def test_forward_kl_tc_workload_sizes(d, V):
+    """The hidden sizes and vocabularies of the log-prob and 7B-shaped
+    workloads (W ~ N(0, 0.02^2), rows ~ N(0, 1)), 512 pairs with repeated
+    teacher rows: kl per pair and the loss, dHS on every student row, dW on
+    sampled vocabulary rows."""
+    from oracle import sdcc as OSd
+    M = 512
+    g = torch.Generator().manual_seed(d)
+    HT = torch.randn(600, d, generator=g).to(torch.bfloat16)
+    HS = torch.randn(700, d, generator=g).to(torch.bfloat16)
+    W = (0.02 * torch.randn(V, d, generator=g)).to(torch.bfloat16)
+    rng = np.random.default_rng(d)
+    rows_T = torch.from_numpy(rng.integers(0, 600, M).astype(np.int32))
+    rows_S = torch.from_numpy(rng.permutation(700)[:M].astype(np.int32))
+    kl, loss, dHS, dW = _kl_run(HT, HS, W, rows_T, rows_S, 0.1, 1.0)
+    rt, rs = rows_T.numpy().astype(np.int64), rows_S.numpy().astype(np.int64)
+    klr, dhr, _ = OSd.forward_kl(np64(HT)[rt], np64(HS)[rs], np64(W))
+    _assert_kl_bf16(kl, HT, HS, W, rows_T, rows_S)
+    lossr = 0.1 * klr.sum()
+    assert abs(float(loss.item()) - lossr) <= 1e-3 * abs(lossr)
+    assert_grad_bf16(np64(dHS)[rs], 0.1 * dhr, "dHS")
+    vocab = np.unique(np.concatenate([[0, V - 1], rng.integers(0, V, 62)]))
+    dWr = OSd.forward_kl_dw_vocab(np64(HT)[rt], np64(HS)[rs], np64(W), vocab)
+    assert_grad_bf16(np64(dW)[vocab], 0.1 * dWr, "dW (sampled vocabulary rows)")
 
 
 def test_forward_kl_without_pairs():
