@@ -394,6 +394,18 @@ class Step:
                 "visible_pairs": int(self.vis.pairs_total), "causal_pairs": int(causal_pairs),
                 "visible_pair_frac": int(self.vis.pairs_total) / max(1, causal_pairs)}
 
+    def call_flops(self):
+        """Algorithmic FLOPs of each timed C-ABI call of the step."""
+        f = self.flops()
+        return {"mw_masked_attn_fwd": 4.0 / 14.0 * f.get("attn", 0),
+                "mw_masked_attn_bwd": 10.0 / 14.0 * f.get("attn", 0),
+                "mw_masked_attn_rope_fwd": 4.0 / 14.0 * f.get("attn", 0),
+                "mw_masked_attn_rope_bwd": 10.0 / 14.0 * f.get("attn", 0),
+                # the forward forms the logits and E = sum_v p_v W_v (the dH
+                # product); the backward recomputes the logits for dW
+                "mw_logprob_loss_fwd": 4.0 / 8.0 * f.get("lm", 0),
+                "mw_logprob_loss_bwd": 4.0 / 8.0 * f.get("lm", 0)}
+
     def flops(self):
         """Visible FLOPs per step: attention 14 P Dh Hq, LM head 8 M d V."""
         f = {}
@@ -403,6 +415,153 @@ class Step:
         if "rows" in self.w:
             f["lm"] = 8.0 * self.w["rows"].numel() * self.w["d"] * self.w["Vocab"]
         return f
+
+
+class SdccStep(Step):
+    """SDCC training step on the 7B-shaped layer (§5, Eq. "soft_loss"): the
+    teacher is the masked attention under each row's live view (forward
+    only, gradients stopped); the student is causal attention over each
+    trajectory's final compressed walk, with the clipped task loss on the
+    loss rows whose token survives on the walk (each predicted by the walk row
+    before it) plus lam * KL(teacher || student) at the diverging ones; the
+    summed gradients run back through the student's attention. The walk and
+    the diverging rows are structure of the record, found once (untimed) with
+    mw_final_walk / mw_diverging_rows; the student's own Q / K / V are
+    synthetic inputs of the walk's length."""
+
+    LAM = 0.1
+
+    def __init__(self, w, device):
+        import numpy as np
+        import torch
+        super().__init__(w, device)
+        mw = self.mw
+        r = w["record"]
+        Hq, Hkv, Dh = w["heads"]
+        self.build()
+        wi, sr, wl = mw.final_walk(self.vis)
+        div = mw.diverging_rows(self.vis)
+        torch.cuda.synchronize()
+        wi, sr, div = wi.cpu().numpy(), sr.cpu().numpy(), div.cpu().numpy()
+        wl = wl.cpu().numpy()[: len(r.trajs)].astype(np.int64)
+        woff = np.concatenate([[0], np.cumsum(wl)])
+        tok = np.concatenate([[0], np.cumsum(r.seqlens)])
+        rows = w["rows"].numpy().astype(np.int64)
+        leaves, srow, p_t, p_s = [], [], [], []
+        for m, rr in enumerate(rows):
+            b = int(np.searchsorted(tok, rr, side="right") - 1)
+            if rr + 1 >= tok[b + 1] or wi[rr + 1] < 0:
+                continue                      # the leaf is evicted: no student score
+            s_row = int(woff[b] + sr[rr])
+            leaves.append(m)
+            srow.append(s_row)
+            if div[rr]:
+                p_t.append(int(rr))
+                p_s.append(s_row)
+        self.Tw = int(woff[-1])
+        self.walk_lens = [int(x) for x in wl]
+        self.n_leaves, self.n_pairs = len(leaves), len(p_t)
+        g = torch.Generator().manual_seed(4242)
+        pin = lambda t: t.pin_memory()   # noqa: E731
+        tgt = torch.zeros(self.Tw, dtype=torch.int32)
+        tgt[torch.tensor(srow, dtype=torch.int64)] = w["targets"][torch.tensor(rows[leaves], dtype=torch.int64)]
+        host = {"Qs": torch.randn(self.Tw, Hq, Dh, generator=g).to(torch.bfloat16),
+                "Ks": torch.randn(self.Tw, Hkv, Dh, generator=g).to(torch.bfloat16),
+                "Vs": torch.randn(self.Tw, Hkv, Dh, generator=g).to(torch.bfloat16),
+                "tgt_s": tgt, "rows_s": torch.tensor(srow, dtype=torch.int32),
+                "adv_s": w["adv"][torch.tensor(leaves, dtype=torch.int64)].clone(),
+                "noise_s": w["noise"][torch.tensor(leaves, dtype=torch.int64)].clone(),
+                "pair_t": torch.tensor(p_t, dtype=torch.int32), "pair_s": torch.tensor(p_s, dtype=torch.int32)}
+        for k, v in host.items():
+            w[k] = pin(v)
+            self.d[k] = w[k].to(device, non_blocking=True)
+        # student record: the walks, no edits
+        self.flat_s = mw.flatten_record(self.walk_lens, [[] for _ in self.walk_lens])
+        cu, J, jt, off, spans = self.flat_s
+        self.Ls = mw.mw_visibility_layout(cu, jt, 0)
+        self.vis_s = mw.Visibility(self.Ls, torch.empty(self.Ls.vis_bytes, dtype=torch.uint8, device=device),
+                                   torch.empty(max(self.Ls.ws_bytes, 1), dtype=torch.uint8, device=device))
+        mk = lambda *sh, dt=torch.bfloat16: torch.empty(*sh, dtype=dt, device=device)   # noqa: E731
+        self.Os, self.LSEs = mk(self.Tw, Hq, Dh), mk(Hq, self.Tw, dt=torch.float32)
+        self.dQs, self.dKs, self.dVs = mk(self.Tw, Hq, Dh), mk(self.Tw, Hkv, Dh), mk(self.Tw, Hkv, Dh)
+        self.ws_fs = mk(max(mw.mw_masked_attn_fwd_ws(self.vis_s, Hkv, Dh, mw.MW_BF16), 1), dt=torch.uint8)
+        self.ws_bs = mk(max(mw.mw_masked_attn_bwd_ws(self.vis_s, Hq, Hkv, Dh, mw.MW_BF16), 1), dt=torch.uint8)
+        d, V, M = w["d"], w["Vocab"], self.n_leaves
+        self.lm_ws_s = mk(max(mw.mw_logprob_ws(self.Tw, M, d, V, mw.MW_BF16), 1), dt=torch.uint8)
+        f32 = lambda n: mk(max(n, 1), dt=torch.float32)   # noqa: E731
+        self.lp_s, self.ratio_s, self.lse_s, self.lp_old_s = f32(M), f32(M), f32(M), f32(M)
+        self.dHs = mk(self.Tw, d)
+        self.kl_ws = mk(max(mw.mw_forward_kl_ws(self.n_pairs, d, V, mw.MW_BF16), 1), dt=torch.uint8)
+        self.kl, self.loss_kl = f32(self.n_pairs), f32(1)
+
+    def build_student(self):
+        cu, J, jt, off, spans = self.flat_s
+        self._ev("mw_build_visibility (student)", lambda: self.mw.mw_build_visibility(
+            self.Ls, cu, J, jt, off, spans, self.vis_s.ws, self.vis_s.vis, self.stream))
+
+    def prime(self):
+        """Student lp_old = its current log-prob + N(0, 0.05) (once, untimed)."""
+        self.build()
+        self.build_student()
+        self.attn_fwd_student()
+        self.lp_old_s.zero_()
+        self.d["lp_old_s"] = self.lp_old_s
+        self.lm_fwd_student()
+        self.lp_old_s.copy_(self.lp_s + self.d["noise_s"])
+
+    def attn_fwd_student(self):
+        self._ev("mw_masked_attn_fwd (student)", lambda: self.mw.mw_masked_attn_fwd(
+            self.vis_s, self.d["Qs"], self.d["Ks"], self.d["Vs"], self.Os, self.LSEs, self.scale, self.ws_fs,
+            self.stream))
+
+    def lm_fwd_student(self):
+        self._ev("mw_logprob_loss_fwd", lambda: self.mw.mw_logprob_loss_fwd(
+            self.Os.view(self.Tw, -1), self.d["W"], self.d["tgt_s"], self.d["rows_s"], self.lp_old_s,
+            self.d["adv_s"], EPS_LO, EPS_HI, self.lp_s, self.ratio_s, self.lse_s, self.loss, self.lm_ws_s,
+            self.stream))
+
+    def run(self):
+        mw = self.mw
+        T = self.w["record"].total
+        self.build()
+        self.build_student()
+        self.attn_fwd()                       # teacher (live views), no backward
+        self.attn_fwd_student()
+        self.lm_fwd_student()
+        self._ev("mw_forward_kl_fwd", lambda: mw.mw_forward_kl_fwd(
+            self.O.view(T, -1), self.d["pair_t"], self.Os.view(self.Tw, -1), self.d["pair_s"], self.d["W"], self.kl,
+            self.loss_kl, self.kl_ws, self.LAM, self.stream))
+        self._ev("mw_logprob_loss_bwd", lambda: self.mw.mw_logprob_loss_bwd(
+            self.Os.view(self.Tw, -1), self.d["W"], self.d["tgt_s"], self.d["rows_s"], self.lse_s, self.lm_ws_s,
+            1.0, self.dHs, self.dW, self.stream))
+        self._ev("mw_forward_kl_bwd", lambda: mw.mw_forward_kl_bwd(
+            self.O.view(T, -1), self.d["pair_t"], self.Os.view(self.Tw, -1), self.d["pair_s"], self.d["W"],
+            self.kl_ws, self.dHs, self.dW, self.LAM, 1.0, True, self.stream))
+        self._ev("mw_masked_attn_bwd (student)", lambda: self.mw.mw_masked_attn_bwd(
+            self.vis_s, self.d["Qs"], self.d["Ks"], self.d["Vs"], self.Os, self.dHs.view_as(self.Os), self.LSEs,
+            self.dQs, self.dKs, self.dVs, self.scale, self.ws_bs, self.stream))
+
+    def scored(self):
+        return self.n_leaves
+
+    def flops(self):
+        """Visible FLOPs: student attention 14 P_walk Dh Hq (causal over the
+        walks), teacher forward 4 P Dh Hq, LM head 8 M d V on the surviving
+        leaves, KL 12 M_kl d V (both logit products forward; recomputed, dH
+        and dW backward)."""
+        Hq, _, Dh = self.w["heads"]
+        P_w = sum(n * (n + 1) // 2 for n in self.walk_lens)
+        d, V = self.w["d"], self.w["Vocab"]
+        return {"attn": 14.0 * P_w * Dh * Hq, "teacher": 4.0 * int(self.vis.pairs_total) * Dh * Hq,
+                "lm": 8.0 * self.n_leaves * d * V, "kl": 12.0 * self.n_pairs * d * V}
+
+    def call_flops(self):
+        f = self.flops()
+        return {"mw_masked_attn_fwd (student)": 4.0 / 14.0 * f["attn"],
+                "mw_masked_attn_bwd (student)": 10.0 / 14.0 * f["attn"],
+                "mw_masked_attn_fwd": f["teacher"],
+                "mw_logprob_loss_fwd": 0.5 * f["lm"], "mw_logprob_loss_bwd": 0.5 * f["lm"],
+                "mw_forward_kl_fwd": f["kl"] / 3.0, "mw_forward_kl_bwd": 2.0 * f["kl"] / 3.0}
 
 
 # ----------------------------------------------------------------------------- reference arm (CPU oracle)
@@ -493,7 +652,7 @@ def run_gpu(args, rank, world, local_rank):
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
     w = make_workload(args.config, args.K, args.f, seed_offset=rank, n_traj=args.n_traj, rope=args.rope)
-    step = Step(w, dev)
+    step = SdccStep(w, dev) if args.sdcc else Step(w, dev)
     step.prime()
     for _ in range(args.warmup):
         step.run()
@@ -577,18 +736,11 @@ def run_gpu(args, rank, world, local_rank):
     flops = step.flops()
     peak_tf, peak_sus, hbm, peak_kind = _peaks()
     dom = max(per_call, key=per_call.get)
-    dom_flops = {"mw_masked_attn_fwd": 4.0 / 14.0 * flops.get("attn", 0),
-                 "mw_masked_attn_bwd": 10.0 / 14.0 * flops.get("attn", 0),
-                 "mw_masked_attn_rope_fwd": 4.0 / 14.0 * flops.get("attn", 0),
-                 "mw_masked_attn_rope_bwd": 10.0 / 14.0 * flops.get("attn", 0),
-                 # the forward forms the logits and E = sum_v p_v W_v (the dH
-                 # product); the backward recomputes the logits for dW
-                 "mw_logprob_loss_fwd": 4.0 / 8.0 * flops.get("lm", 0),
-                 "mw_logprob_loss_bwd": 4.0 / 8.0 * flops.get("lm", 0)}.get(dom, 0.0)
+    dom_flops = step.call_flops().get(dom, 0.0)
     achieved = dom_flops / (per_call[dom] * 1e-3) / 1e12
     total_tf = sum(flops.values()) / (ms * 1e-3) / 1e12
     cpu = None
-    if world == 1 and not args.no_cpu:
+    if world == 1 and not args.no_cpu and not args.sdcc:   # the oracle sample times the 4D-mask path
         v, cores, desc = cpu_sample(w, budget_s=args.cpu_seconds)
         cpu = {"value": v, "unit": "tokens/s", "cores": cores, "kind": "oracle", "sample": desc}
     line = {
@@ -612,6 +764,10 @@ def run_gpu(args, rank, world, local_rank):
         "gpu_launches": launches,
         "clocks": clk,
     }
+    if args.sdcc:
+        line["config"].update(method="SDCC (§5): student over the final walks + lam KL at diverging leaves",
+                              walk_tokens=step.Tw, scored_leaves=step.n_leaves, kl_pairs=step.n_pairs,
+                              lam=step.LAM)
     ts = step.tile_stats()
     if ts is not None:
         line["attention_tiles"] = ts
@@ -631,9 +787,13 @@ def main():
                     help="keep only the first trajectories (smaller case for profiler captures)")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--sdcc", action="store_true",
+                    help="config 4: time SDCC's training step (§5) instead of the 4D-mask step")
     ap.add_argument("--rope", type=float, default=None, metavar="THETA",
                     help="attention with row-wise logical rotary positions (theta of the rotary table)")
     args = ap.parse_args()
+    if args.sdcc and (args.config != 4 or args.rope is not None):
+        ap.error("--sdcc times the 7B-shaped layer step (config 4) without rotary positions")
     rank = int(os.environ.get("RANK", 0))
     world = int(os.environ.get("WORLD_SIZE", args.gpus if args.gpus == 1 else 1))
     local_rank = int(os.environ.get("LOCAL_RANK", 0))

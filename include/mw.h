@@ -394,14 +394,17 @@ mw_status mw_forward_kl_fwd(const void* HT, const int32_t* rows_T, const void* H
  * Backward of mw_forward_kl_fwd scaled by dloss, the teacher held fixed
  * (stop-gradient): dzS = lam * dloss * (softmax(zS) - softmax(zT)),
  *   dHS[rows_S[m]] = dzS_m W (other rows of dHS = 0),  dW = sum_m dzS_m^T hS_m.
- * dHS [N_S, d] in dtype and dW [Vocab, d] float32 are overwritten. Needs the
- * forward's `ws` (the tensor-core path also uses it as scratch). Tensor cores:
+ * dHS [N_S, d] in dtype and dW [Vocab, d] float32 are overwritten
+ * (accumulate = 0) or added to (accumulate = 1: rows of dHS without a pair
+ * are left as they are), so the KL's gradients can join the task loss's in
+ * one buffer. Needs the forward's `ws` (the tensor-core path also uses it as
+ * scratch). Tensor cores:
  * dHS = lam dloss (E_S - E_T) from the forward, dW by two vocabulary-
  * stationary passes (the student's softmax, then the teacher's added in).
  */
 mw_status mw_forward_kl_bwd(const void* HT, const int32_t* rows_T, const void* HS, const int32_t* rows_S, int M,
                             const void* W, int N_T, int N_S, int d, int Vocab, int dtype, float lam, float dloss,
-                            void* ws, void* dHS, float* dW, void* stream);
+                            int accumulate, void* ws, void* dHS, float* dW, void* stream);
 
 /* Synchronise `stream` and report a bounded device wait of the tensor-core
  * KL passes that gave up (MW_ETIMEOUT), from `ws`. */

@@ -70,7 +70,7 @@ _SIGS = {
     "mw_logdiff": (_I, [_P, _P, _I, _P, _P]),
     "mw_forward_kl_ws": (_I, [_I, _I, _I, _I, ctypes.POINTER(ctypes.c_size_t)]),
     "mw_forward_kl_fwd": (_I, [_P, _P, _P, _P, _I, _P, _I, _I, _I, _I, _I, _F, _P, _P, _P, _P]),
-    "mw_forward_kl_bwd": (_I, [_P, _P, _P, _P, _I, _P, _I, _I, _I, _I, _I, _F, _F, _P, _P, _P, _P]),
+    "mw_forward_kl_bwd": (_I, [_P, _P, _P, _P, _I, _P, _I, _I, _I, _I, _I, _F, _F, _I, _P, _P, _P, _P]),
     "mw_forward_kl_check_status": (_I, [_I, _I, _I, _I, _P, _P]),
     "mw_rope_table": (_I, [_I, _I, ctypes.c_double, _P, _P]),
     "mw_rope_rows": (_I, [_LP, _P, _P, _P, _I, _P, _P, _I, _I, _I, _I, _P]),
@@ -429,6 +429,19 @@ def logdiff(lp_train, lp_rollout, stream=None):
     return out
 
 
+def mw_forward_kl_ws(M, d, Vocab, dtype):
+    n = ctypes.c_size_t()
+    _check(_lib().mw_forward_kl_ws(int(M), int(d), int(Vocab), int(dtype), ctypes.byref(n)), "mw_forward_kl_ws")
+    return int(n.value)
+
+
+def mw_forward_kl_fwd(HT, rows_T, HS, rows_S, W, kl, loss, ws, lam=1.0, stream=None):
+    M, d, V = int(rows_T.numel()), HT.shape[1], W.shape[0]
+    _check(_lib().mw_forward_kl_fwd(_ptr(HT), _ptr(rows_T), _ptr(HS), _ptr(rows_S), M, _ptr(W), HT.shape[0],
+                                    HS.shape[0], d, V, _dtype_code(HT), float(lam), _ptr(kl), _ptr(loss), _ptr(ws),
+                                    _stream(stream)), "mw_forward_kl_fwd")
+
+
 def forward_kl_fwd(HT, rows_T, HS, rows_S, W, lam=1.0, stream=None):
     """SDCC consistency term: kl [M], loss (lam * sum kl) and the workspace
     the backward needs (mw_forward_kl_fwd)."""
@@ -437,14 +450,10 @@ def forward_kl_fwd(HT, rows_T, HS, rows_S, W, lam=1.0, stream=None):
     _need(HS, "HS", dtype=HT.dtype)
     _need(W, "W", dtype=HT.dtype)
     M, d, V = int(rows_T.numel()), HT.shape[1], W.shape[0]
-    n = ctypes.c_size_t()
-    _check(_lib().mw_forward_kl_ws(M, d, V, _dtype_code(HT), ctypes.byref(n)), "mw_forward_kl_ws")
-    ws = torch.empty(max(int(n.value), 1), dtype=torch.uint8, device=HT.device)
+    ws = torch.empty(max(mw_forward_kl_ws(M, d, V, _dtype_code(HT)), 1), dtype=torch.uint8, device=HT.device)
     kl = torch.empty(max(M, 1), dtype=torch.float32, device=HT.device)
     loss = torch.empty(1, dtype=torch.float32, device=HT.device)
-    _check(_lib().mw_forward_kl_fwd(_ptr(HT), _ptr(rows_T), _ptr(HS), _ptr(rows_S), M, _ptr(W), HT.shape[0],
-                                    HS.shape[0], d, V, _dtype_code(HT), float(lam), _ptr(kl), _ptr(loss), _ptr(ws),
-                                    _stream(stream)), "mw_forward_kl_fwd")
+    mw_forward_kl_fwd(HT, rows_T, HS, rows_S, W, kl, loss, ws, lam, stream)
     return kl[:M], loss, ws
 
 
@@ -455,15 +464,20 @@ def forward_kl_check_status(rows_T, HT, W, ws, stream=None):
                                              _ptr(ws), _stream(stream)), "mw_forward_kl_check_status")
 
 
+def mw_forward_kl_bwd(HT, rows_T, HS, rows_S, W, ws, dHS, dW, lam=1.0, dloss=1.0, accumulate=False, stream=None):
+    M, d, V = int(rows_T.numel()), HT.shape[1], W.shape[0]
+    _check(_lib().mw_forward_kl_bwd(_ptr(HT), _ptr(rows_T), _ptr(HS), _ptr(rows_S), M, _ptr(W), HT.shape[0],
+                                    HS.shape[0], d, V, _dtype_code(HT), float(lam), float(dloss), int(accumulate),
+                                    _ptr(ws), _ptr(dHS), _ptr(dW), _stream(stream)), "mw_forward_kl_bwd")
+
+
 def forward_kl_bwd(HT, rows_T, HS, rows_S, W, ws, lam=1.0, dloss=1.0, stream=None):
     """Student gradients of the SDCC term: dHS (like HS), dW (float32)."""
     import torch
-    M, d, V = int(rows_T.numel()), HT.shape[1], W.shape[0]
+    d, V = HT.shape[1], W.shape[0]
     dHS = torch.empty_like(HS)
     dW = torch.empty(V, d, dtype=torch.float32, device=HT.device)
-    _check(_lib().mw_forward_kl_bwd(_ptr(HT), _ptr(rows_T), _ptr(HS), _ptr(rows_S), M, _ptr(W), HT.shape[0],
-                                    HS.shape[0], d, V, _dtype_code(HT), float(lam), float(dloss), _ptr(ws),
-                                    _ptr(dHS), _ptr(dW), _stream(stream)), "mw_forward_kl_bwd")
+    mw_forward_kl_bwd(HT, rows_T, HS, rows_S, W, ws, dHS, dW, lam, dloss, False, stream)
     return dHS, dW
 
 

@@ -709,7 +709,7 @@ __global__ void k_kl_from_e(int M, int d, const __nv_bfloat16* __restrict__ hgT,
 // a student equal to its teacher gets exactly 0.
 __global__ void k_kl_dh_from_e(int M, int d, const float* __restrict__ ES, const float* __restrict__ linvS,
                                const float* __restrict__ ET, const float* __restrict__ linvT, float c,
-                               const int32_t* __restrict__ rowsS, __nv_bfloat16* __restrict__ dHS) {
+                               const int32_t* __restrict__ rowsS, int accumulate, __nv_bfloat16* __restrict__ dHS) {
     for (int m = blockIdx.x; m < M; m += gridDim.x) {
         const float as = c * linvS[m], at_ = c * linvT[m];
         const float4* s4 = reinterpret_cast<const float4*>(ES + (int64_t)m * d);
@@ -717,10 +717,16 @@ __global__ void k_kl_dh_from_e(int M, int d, const float* __restrict__ ES, const
         uint2* out = reinterpret_cast<uint2*>(dHS + (int64_t)rowsS[m] * d);
         for (int k = threadIdx.x; k < d / 4; k += blockDim.x) {
             const float4 x = s4[k], y = t4[k];
-            out[k] = make_uint2(pack_bf16(__fmul_rn(as, x.x) - __fmul_rn(at_, y.x),
-                                          __fmul_rn(as, x.y) - __fmul_rn(at_, y.y)),
-                                pack_bf16(__fmul_rn(as, x.z) - __fmul_rn(at_, y.z),
-                                          __fmul_rn(as, x.w) - __fmul_rn(at_, y.w)));
+            float g[4] = {__fmul_rn(as, x.x) - __fmul_rn(at_, y.x), __fmul_rn(as, x.y) - __fmul_rn(at_, y.y),
+                          __fmul_rn(as, x.z) - __fmul_rn(at_, y.z), __fmul_rn(as, x.w) - __fmul_rn(at_, y.w)};
+            if (accumulate) {
+                const uint2 o = out[k];
+                g[0] += __uint_as_float(o.x << 16);
+                g[1] += __uint_as_float(o.x & 0xffff0000u);
+                g[2] += __uint_as_float(o.y << 16);
+                g[3] += __uint_as_float(o.y & 0xffff0000u);
+            }
+            out[k] = make_uint2(pack_bf16(g[0], g[1]), pack_bf16(g[2], g[3]));
         }
     }
 }
@@ -981,18 +987,18 @@ mw_status kl_fwd_tc(const void* HT, const int32_t* rowsT, const void* HS, const 
 // same rows' product: softmax-only with the student's logits, then with the
 // teacher's logits added in.
 mw_status kl_bwd_tc(const int32_t* rowsS, int M, const void* W, int N_S, int d, int V, float c, void* ws,
-                    void* dHS, float* dW, cudaStream_t s) {
+                    int accumulate, void* dHS, float* dW, cudaStream_t s) {
     if (!lm_bwd_tc_supported(d)) return MW_ESHAPE;
-    mw_status st = cuda_status(cudaMemsetAsync(dHS, 0, (size_t)N_S * d * 2, s));
-    if (st != MW_OK) return st;
-    if (M == 0) return cuda_status(cudaMemsetAsync(dW, 0, (size_t)V * d * 4, s));
+    mw_status st = MW_OK;
+    if (!accumulate && (st = cuda_status(cudaMemsetAsync(dHS, 0, (size_t)N_S * d * 2, s))) != MW_OK) return st;
+    if (M == 0) return accumulate ? MW_OK : cuda_status(cudaMemsetAsync(dW, 0, (size_t)V * d * 4, s));
     const KlWs w = kl_ws_layout(M, d);
     const int M_pad = (int)ceil_div(M, 128) * 128;
     if ((st = cuda_status(cudaMemsetAsync(at<char>(ws, w.status), 0, 32, s))) != MW_OK) return st;
     const GrpArrays aT = grp_arrays(at<char>(ws, w.fwdT), M, d), aS = grp_arrays(at<char>(ws, w.fwdS), M, d);
     count_launches(1);
     k_kl_dh_from_e<<<(unsigned)std::min(M, 8 * 152), 128, 0, s>>>(M, d, aS.E, aS.linv, aT.E, aT.linv, c, rowsS,
-                                                                  (__nv_bfloat16*)dHS);
+                                                                  accumulate, (__nv_bfloat16*)dHS);
     if ((st = launch_status()) != MW_OK) return st;
     for (int side = 0; side < 2; ++side) {   // student: dz = c p_S; teacher: dz = -c p_T
         count_launches(1);
@@ -1002,7 +1008,7 @@ mw_status kl_bwd_tc(const int32_t* rowsS, int M, const void* W, int N_S, int d, 
         if ((st = launch_status()) != MW_OK) return st;
         LmBwdParams p = {};
         p.mode = 1;
-        p.add = side;
+        p.add = accumulate || side;
         p.M = M;
         p.V = V;
         p.dW = dW;

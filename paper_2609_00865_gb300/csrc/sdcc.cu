@@ -230,7 +230,7 @@ __global__ void __launch_bounds__(256) k_kl_dh_simt(int M, int d, int Vocab, con
                                                    const int32_t* __restrict__ rowsT, const Tin* __restrict__ HS,
                                                    const int32_t* __restrict__ rowsS, const Tin* __restrict__ W,
                                                    const float* __restrict__ lseT, const float* __restrict__ lseS,
-                                                   float c, Tin* __restrict__ dHS) {
+                                                   float c, int accumulate, Tin* __restrict__ dHS) {
     extern __shared__ float sh[];
     float* ht = sh;                // [KH][d]
     float* hs = sh + KH * d;       // [KH][d]
@@ -286,7 +286,10 @@ __global__ void __launch_bounds__(256) k_kl_dh_simt(int M, int d, int Vocab, con
     if (threadIdx.x < d) {
 #pragma unroll
         for (int r = 0; r < KH; ++r)
-            if (m0 + r < M) st_f(dHS + (int64_t)rowsS[m0 + r] * d + threadIdx.x, acc[r]);
+            if (m0 + r < M) {
+                Tin* dst = dHS + (int64_t)rowsS[m0 + r] * d + threadIdx.x;
+                st_f(dst, accumulate ? ld_f(dst) + acc[r] : acc[r]);
+            }
     }
 }
 
@@ -296,7 +299,7 @@ __global__ void __launch_bounds__(256) k_kl_dw_simt(int M, int d, int Vocab, con
                                                    const int32_t* __restrict__ rowsT, const Tin* __restrict__ HS,
                                                    const int32_t* __restrict__ rowsS, const Tin* __restrict__ W,
                                                    const float* __restrict__ lseT, const float* __restrict__ lseS,
-                                                   float c, float* __restrict__ dW) {
+                                                   float c, int accumulate, float* __restrict__ dW) {
     extern __shared__ float sh[];
     float* ws = sh;                 // [KWV][d]
     float* ht = sh + KWV * d;       // [KWR][d]
@@ -351,7 +354,10 @@ __global__ void __launch_bounds__(256) k_kl_dw_simt(int M, int d, int Vocab, con
     if (threadIdx.x < d) {
 #pragma unroll
         for (int q = 0; q < KWV; ++q)
-            if (v0 + q < Vocab) dW[(int64_t)(v0 + q) * d + threadIdx.x] = acc[q];
+            if (v0 + q < Vocab) {
+                float* dst = dW + (int64_t)(v0 + q) * d + threadIdx.x;
+                *dst = accumulate ? *dst + acc[q] : acc[q];
+            }
     }
 }
 
@@ -376,10 +382,12 @@ mw_status kl_fwd_t(const void* HT, const int32_t* rowsT, const void* HS, const i
 template <typename Tin>
 mw_status kl_bwd_t(const void* HT, const int32_t* rowsT, const void* HS, const int32_t* rowsS, int M,
                    const void* W, int N_S, int d, int Vocab, float c, const float* lseT, const float* lseS,
-                   void* dHS, float* dW, cudaStream_t s) {
-    mw_status st = cuda_status(cudaMemsetAsync(dHS, 0, sizeof(Tin) * (size_t)N_S * d, s));
-    if (st != MW_OK) return st;
-    if (M == 0) return cuda_status(cudaMemsetAsync(dW, 0, sizeof(float) * (size_t)Vocab * d, s));
+                   int accumulate, void* dHS, float* dW, cudaStream_t s) {
+    mw_status st = MW_OK;
+    if (!accumulate && (st = cuda_status(cudaMemsetAsync(dHS, 0, sizeof(Tin) * (size_t)N_S * d, s))) != MW_OK)
+        return st;
+    if (M == 0)
+        return accumulate ? MW_OK : cuda_status(cudaMemsetAsync(dW, 0, sizeof(float) * (size_t)Vocab * d, s));
     const size_t smem_h = sizeof(float) * (2 * KH * d + KH * 256);
     const size_t smem_w = sizeof(float) * (KWV * d + 2 * KWR * d + KWR * KWV);
     if ((st = cuda_status(cudaFuncSetAttribute(k_kl_dh_simt<Tin>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -391,10 +399,10 @@ mw_status kl_bwd_t(const void* HT, const int32_t* rowsT, const void* HS, const i
     count_launches(2);
     k_kl_dh_simt<Tin><<<(unsigned)ceil_div(M, KH), 256, smem_h, s>>>(M, d, Vocab, (const Tin*)HT, rowsT,
                                                                      (const Tin*)HS, rowsS, (const Tin*)W, lseT,
-                                                                     lseS, c, (Tin*)dHS);
+                                                                     lseS, c, accumulate, (Tin*)dHS);
     k_kl_dw_simt<Tin><<<(unsigned)ceil_div(Vocab, KWV), 256, smem_w, s>>>(M, d, Vocab, (const Tin*)HT, rowsT,
                                                                           (const Tin*)HS, rowsS, (const Tin*)W,
-                                                                          lseT, lseS, c, dW);
+                                                                          lseT, lseS, c, accumulate, dW);
     return launch_status();
 }
 
@@ -420,7 +428,8 @@ bool lm_bwd_tc_supported(int d);
 int64_t kl_tc_ws(int M, int d);
 mw_status kl_fwd_tc(const void*, const int32_t*, const void*, const int32_t*, int, const void*, int, int, float*,
                     void*, cudaStream_t);
-mw_status kl_bwd_tc(const int32_t*, int, const void*, int, int, int, float, void*, void*, float*, cudaStream_t);
+mw_status kl_bwd_tc(const int32_t*, int, const void*, int, int, int, float, void*, int, void*, float*,
+                    cudaStream_t);
 int32_t* kl_tc_status(int M, int d, void* ws);
 }  // namespace mw
 
@@ -489,7 +498,8 @@ extern "C" mw_status mw_forward_kl_fwd(const void* HT, const int32_t* rows_T, co
 
 extern "C" mw_status mw_forward_kl_bwd(const void* HT, const int32_t* rows_T, const void* HS, const int32_t* rows_S,
                                        int M, const void* W, int N_T, int N_S, int d, int Vocab, int dtype,
-                                       float lam, float dloss, void* ws, void* dHS, float* dW, void* stream) {
+                                       float lam, float dloss, int accumulate, void* ws, void* dHS, float* dW,
+                                       void* stream) {
     mw_status st = kl_args(M, N_T, N_S, d, Vocab, dtype);
     if (st != MW_OK) return st;
     if (!(lam >= 0.f) || !isfinite(lam) || !isfinite(dloss)) return MW_EINVAL;
@@ -499,10 +509,11 @@ extern "C" mw_status mw_forward_kl_bwd(const void* HT, const int32_t* rows_T, co
     const float* lseT = at<float>(ws, 0);
     const float* lseS = at<float>(ws, align256(4 * (int64_t)M));
     const float c = lam * dloss;
-    if (kl_tc(d, dtype)) return kl_bwd_tc(rows_S, M, W, N_S, d, Vocab, c, ws, dHS, dW, s);
+    if (kl_tc(d, dtype)) return kl_bwd_tc(rows_S, M, W, N_S, d, Vocab, c, ws, accumulate, dHS, dW, s);
     return dtype == MW_F32
-               ? kl_bwd_t<float>(HT, rows_T, HS, rows_S, M, W, N_S, d, Vocab, c, lseT, lseS, dHS, dW, s)
-               : kl_bwd_t<__nv_bfloat16>(HT, rows_T, HS, rows_S, M, W, N_S, d, Vocab, c, lseT, lseS, dHS, dW, s);
+               ? kl_bwd_t<float>(HT, rows_T, HS, rows_S, M, W, N_S, d, Vocab, c, lseT, lseS, accumulate, dHS, dW, s)
+               : kl_bwd_t<__nv_bfloat16>(HT, rows_T, HS, rows_S, M, W, N_S, d, Vocab, c, lseT, lseS, accumulate,
+                                         dHS, dW, s);
 }
 
 extern "C" mw_status mw_diverging_rows(const mw_vis_layout* L, const void* vis, uint8_t* out, void* stream) {

@@ -185,8 +185,8 @@ def test_forward_kl_rejects_bad_args_on_host():
     assert h.mw_forward_kl_fwd(P, P, P, P, 4, P, 0, 8, 64, 100, 0, 0.1, P, P, P, None) == 3
     assert h.mw_forward_kl_fwd(P, P, P, P, 4, P, 4, 8, 64, 100, 0, -0.1, P, P, P, None) == 1
     assert h.mw_forward_kl_fwd(P, P, P, P, 4, P, 4, 8, 64, 100, 0, 0.1, P, None, P, None) == 1
-    assert h.mw_forward_kl_bwd(P, P, P, P, 4, P, 4, 8, 64, 100, 0, 0.1, float("nan"), P, P, P, None) == 1
-    assert h.mw_forward_kl_bwd(P, P, P, P, 4, P, 4, 8, 64, 100, 0, 0.1, 1.0, P, P, None, None) == 1
+    assert h.mw_forward_kl_bwd(P, P, P, P, 4, P, 4, 8, 64, 100, 0, 0.1, float("nan"), 0, P, P, P, None) == 1
+    assert h.mw_forward_kl_bwd(P, P, P, P, 4, P, 4, 8, 64, 100, 0, 0.1, 1.0, 0, P, P, None, None) == 1
 
 
 def test_logdiff_rejects_bad_args_on_host():

@@ -259,3 +259,30 @@ def test_sdcc_objective_end_to_end():
                                          lp_old, adv, lam, scale)
     assert abs(float(out["loss"].item()) - task) <= 1e-4 * abs(task) + 1e-6
     assert abs(float(pen.item()) - penalty) <= 1e-4 * abs(penalty)
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+def test_forward_kl_bwd_accumulates(dtype):
+    """accumulate = 1 adds the KL's gradients to dHS / dW (the task loss's
+    buffers in an SDCC step) and leaves rows without a pair alone: a second
+    call doubles the first call's result."""
+    import paper_2609_00865_gb300 as mw
+    d = 64 if dtype == torch.float32 else 128
+    HT, HS, W, rows_T, rows_S = (t.cuda() for t in _kl_case(21, 30, 28, d, 700, 23, dtype))
+    kl, loss, ws = mw.forward_kl_fwd(HT, rows_T, HS, rows_S, W, lam=0.3)
+    dHS = torch.full_like(HS, 0.0)
+    dW = torch.zeros(W.shape[0], d, dtype=torch.float32, device="cuda")
+    mw.mw_forward_kl_bwd(HT, rows_T, HS, rows_S, W, ws, dHS, dW, 0.3, 1.0, False)
+    first = (dHS.float().clone(), dW.clone())
+    mw.mw_forward_kl_bwd(HT, rows_T, HS, rows_S, W, ws, dHS, dW, 0.3, 1.0, True)
+    torch.cuda.synchronize()
+    if dtype == torch.float32:
+        assert torch.allclose(dHS, 2 * first[0], rtol=1e-6, atol=0)
+    else:
+        assert torch.allclose(dHS.float(), 2 * first[0], rtol=8e-3, atol=0)   # one more bf16 rounding
+    # tensor cores: dW is the sum of two nearly cancelling passes, added in
+    # another order the second time, so it doubles up to rounding of the parts
+    tol = 1e-6 if dtype == torch.float32 else 1e-3
+    assert torch.allclose(dW, 2 * first[1], rtol=tol, atol=tol * float(first[1].abs().max()))
+    untouched = np.setdiff1d(np.arange(HS.shape[0]), rows_S.cpu().numpy())
+    assert not dHS[torch.from_numpy(untouched).cuda()].float().any()
