@@ -410,6 +410,27 @@ mw_status mw_forward_kl_bwd(const void* HT, const int32_t* rows_T, const void* H
  * KL passes that gave up (MW_ETIMEOUT), from `ws`. */
 mw_status mw_forward_kl_check_status(int M, int d, int Vocab, int dtype, void* ws, void* stream);
 
+/*
+ * Branch-replicated packing for stacked layers (App. G). From the second layer
+ * on a token's state differs between the segments' branches that hold it, so
+ * the exact multi-layer step runs every branch's compact sequence (its live
+ * view in order, §4.1) through all layers. Packed rows: the branches back to
+ * back in global segment order, branch g at rows off_g = sum of the earlier
+ * seg_len values, |view_g| rows (total: the sum of seg_len); a packed record
+ * of those lengths with no edits is what the layers attend over.
+ *   mw_branch_pack:       Xp[off_g + c] = X[csrc_g(c)]  (c < |view_g|)
+ *   mw_branch_unpack_add: dX[j] = sum over the segments g holding j, in
+ *                         segment order, of dXp[off_g + cpos_g(j)]
+ *                         (float32 accumulation, written in dtype)
+ * X, dX [total_tokens, row_elems], Xp, dXp [sum seg_len, row_elems] (dtype,
+ * device); row_elems * element size a multiple of 16 bytes (MW_ESHAPE).
+ * `vis` from either builder.
+ */
+mw_status mw_branch_pack(const mw_vis_layout* layout, const void* vis, const void* X, void* Xp, int row_elems,
+                         int dtype, void* stream);
+mw_status mw_branch_unpack_add(const mw_vis_layout* layout, const void* vis, const void* dXp, void* dX,
+                               int row_elems, int dtype, void* stream);
+
 /* Bytes of device workspace the log-prob loss forward/backward pair needs. */
 mw_status mw_logprob_ws(int N, int M, int d, int Vocab, int dtype, size_t* ws_bytes);
 

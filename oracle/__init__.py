@@ -32,4 +32,4 @@ and slowly, in float64:
 Every function names the passage it follows in its docstring.
 """
 
-from . import visibility, attention, logprob, nonmonotone, sdcc  # noqa: F401
+from . import visibility, attention, logprob, nonmonotone, sdcc, multilayer  # noqa: F401

@@ -54,6 +54,8 @@ _SIGS = {
     "mw_build_visibility": (_I, [_LP, _IP, _I, _IP, _IP, _IP, _IP, _P, _P, _P]),
     "mw_build_visibility_noalloc": (_I, [_LP, _IP, _I, _IP, _IP, _IP, _IP, _P, _P]),
     "mw_events_layout": (_I, [_I, _IP, _I, _IP, _I, _LP]),
+    "mw_branch_pack": (_I, [_LP, _P, _P, _P, _I, _I, _P]),
+    "mw_branch_unpack_add": (_I, [_LP, _P, _P, _P, _I, _I, _P]),
     "mw_build_views_events": (_I, [_LP, _IP, _I, _IP, _IP, _IP, _IP, _IP, _P, _P, _P]),
     "mw_masked_attn_fwd_ws": (_I, [_LP, _I, _I, _I, ctypes.POINTER(ctypes.c_size_t)]),
     "mw_masked_attn_fwd": (_I, [_LP, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _F, _P, _P]),
@@ -321,6 +323,36 @@ def build_visibility(seqlens, edits_per_traj, device="cuda", stream=None):
     ws = torch.empty(max(int(L.ws_bytes), 1), dtype=torch.uint8, device=device)
     mw_build_visibility(L, cu, J, jt, off, spans, ws, vis, stream)
     return Visibility(L, vis, ws)
+
+
+# --- branch-replicated packing (stacked layers) --------------------------------
+
+def branch_lengths(vis):
+    """Host list of every segment's compact-sequence length (|view_s|, read
+    back from the build; the packed branches' record)."""
+    return [int(x) for x in vis._arr(vis.layout.off_seg_len, vis.layout.n_segs, np.int32)]
+
+
+def branch_pack(vis, X, n_packed, stream=None):
+    """Packed branch copies [n_packed, ...] of the per-token rows of X
+    (mw_branch_pack)."""
+    import torch
+    Xp = torch.empty((n_packed,) + tuple(X.shape[1:]), dtype=X.dtype, device=X.device)
+    row = int(np.prod(X.shape[1:]))
+    _check(_lib().mw_branch_pack(ctypes.byref(vis.layout), _ptr(vis.vis), _ptr(X), _ptr(Xp), row, _dtype_code(X),
+                                 _stream(stream)), "mw_branch_pack")
+    return Xp
+
+
+def branch_unpack_add(vis, dXp, stream=None):
+    """Per-token sums [total_tokens, ...] of the packed copies' rows
+    (mw_branch_unpack_add)."""
+    import torch
+    dX = torch.empty((int(vis.layout.total_tokens),) + tuple(dXp.shape[1:]), dtype=dXp.dtype, device=dXp.device)
+    row = int(np.prod(dXp.shape[1:]))
+    _check(_lib().mw_branch_unpack_add(ctypes.byref(vis.layout), _ptr(vis.vis), _ptr(dXp), _ptr(dX), row,
+                                       _dtype_code(dXp), _stream(stream)), "mw_branch_unpack_add")
+    return dX
 
 
 # --- attention ----------------------------------------------------------------

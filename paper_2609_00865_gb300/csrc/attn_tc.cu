@@ -98,25 +98,24 @@ struct FwdParams {
 };
 
 // Work item of a q-tile kernel: trajectory b, local q-tile qt, query head h
-// and (SEGK) the segment s whose rows the CTA stores. Main launch: heaviest
-// (largest qt) first, query heads of one KV group adjacent; s = segment of the
-// tile's first row. Junction items: blockIdx.x / Hq is a global segment index;
-// a segment that starts inside a tile (not at its first row) gets a CTA there.
+// and the segment s whose rows the CTA stores. Main launch: heaviest (largest
+// qt) first, query heads of one KV group adjacent; s = segment of the tile's
+// first row. Junction items: blockIdx.x / Hq is a global segment index; a
+// segment that starts inside a tile (not at its first row) gets a CTA there.
 struct QItem {
     int b, qt, h, s;
     bool ok;
 };
-template <bool SEGK>
 __device__ __forceinline__ QItem q_item(const VisView& v, int Hq, int max_tiles, int n_traj, int junction_items) {
     QItem it;
     it.h = blockIdx.x % Hq;
     const int r = blockIdx.x / Hq;
     it.s = 0;
-    if (!SEGK || !junction_items) {
+    if (!junction_items) {
         it.qt = max_tiles - 1 - r / n_traj;
         it.b = r % n_traj;
         it.ok = it.qt < v.traj_tile[it.b + 1] - v.traj_tile[it.b];
-        if (SEGK && it.ok) it.s = v.seg[v.traj_tok[it.b] + it.qt * 128];
+        if (it.ok) it.s = v.seg[v.traj_tok[it.b] + it.qt * 128];
     } else {
         int lo = 0, hi = n_traj;   // largest b with traj_seg[b] <= r
         while (hi - lo > 1) {
@@ -227,10 +226,11 @@ __global__ void __launch_bounds__(NT_FWD, 1)
     __shared__ uint32_t tmem_base;
     __shared__ int abort_flag;
 
-    constexpr bool SEGK = MODE == 1, CMP = MODE == 2;
+    static_assert(MODE == 1 || MODE == 2, "segment key rows (1) or compact views (2)");
+    constexpr bool CMP = MODE == 2;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const VisView& v = p.v;
-    const QItem it = q_item<MODE != 0>(v, p.Hq, p.max_tiles, p.n_traj, p.junction_items);
+    const QItem it = q_item(v, p.Hq, p.max_tiles, p.n_traj, p.junction_items);
     if (!it.ok) return;
     const int h = it.h, qt = it.qt, b = it.b;
     const int nt = v.traj_tile[b + 1] - v.traj_tile[b];
@@ -280,7 +280,7 @@ __global__ void __launch_bounds__(NT_FWD, 1)
             load_tile(sm + SM_Q, &tmQ, &q_full, h, (int)(tok0 + qt * 128));
             // first K row of the trajectory (SEGK: of the item's segment key
             // rows; CMP: of the segment's compact sequence, for V as well)
-            const int64_t krow0 = MODE != 0 ? (v.traj_km[b] + (int64_t)it.s * nt) * 128 : tok0;
+            const int64_t krow0 = (v.traj_km[b] + (int64_t)it.s * nt) * 128;
             for (int j = 0; j < n; ++j) {
                 const int kt = entry(j) >> 4;
                 const int s = j & 1;
@@ -507,7 +507,7 @@ __global__ void __launch_bounds__(NT_FWD, 1)
             const float inv = 1.f / l;
             __nv_bfloat16* orow = p.O + ((tok0 + ie) * p.Hq + h) * DH;
             uint32_t o[32];
-            const bool store = CMP ? in_piece : i < T && (!SEGK || seg == it.s);
+            const bool store = CMP ? in_piece : i < T && seg == it.s;
 #pragma unroll
             for (int c = 0; c < 4; ++c) {
                 tmem_ld32(lane_base + TM_O + c * 32, o);
@@ -562,10 +562,8 @@ struct BwdParams {
     const float2* lsd;     // [Hq][n_tiles * 128] (-LSE_i log2 e, Delta_i), rows padded to whole tiles
     int64_t n_rows;        // n_tiles * 128
     __nv_bfloat16* dQ;
-    __nv_bfloat16* dK;
-    __nv_bfloat16* dV;
     int junction_items;    // SEGK dQ: as FwdParams
-    float* dKseg;          // SEGK dK/dV: float32 partials per segment key row [rows][Hkv][DH]
+    float* dKseg;          // dK/dV: float32 partials per segment key row (SEGK) or compact row [rows][Hkv][DH]
     float* dVseg;
 };
 
@@ -579,10 +577,11 @@ __global__ void __launch_bounds__(NT_BWD, 1)
         dp_full, dp_free, ds_full[2], dq_fin;
     __shared__ uint32_t tmem_base;
 
-    constexpr bool SEGK = MODE == 1, CMP = MODE == 2;
+    static_assert(MODE == 1 || MODE == 2, "segment key rows (1) or compact views (2)");
+    constexpr bool CMP = MODE == 2;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const VisView& v = p.v;
-    const QItem it = q_item<MODE != 0>(v, p.Hq, p.max_tiles, p.n_traj, p.junction_items);
+    const QItem it = q_item(v, p.Hq, p.max_tiles, p.n_traj, p.junction_items);
     if (!it.ok) return;
     const int h = it.h, qt = it.qt, b = it.b;
     const int nt = v.traj_tile[b + 1] - v.traj_tile[b];
@@ -635,7 +634,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             load_tile(sm + DQ_DO, &tmDO, &q_full, h, row0);
             // first K row of the trajectory (SEGK: of the item's segment key
             // rows; CMP: of the segment's compact sequence, for V as well)
-            const int64_t krow0 = MODE != 0 ? (v.traj_km[b] + (int64_t)it.s * nt) * 128 : tok0;
+            const int64_t krow0 = (v.traj_km[b] + (int64_t)it.s * nt) * 128;
             for (int j = 0; j < n; ++j) {
                 const int kt = entry(j) >> 4;
                 const int s = j & 1;
@@ -860,7 +859,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             tc_fence_after();
             __nv_bfloat16* qrow = p.dQ + ((tok0 + ie) * p.Hq + h) * DH;
             uint32_t o[32];
-            const bool store = CMP ? in_piece : i < T && (!SEGK || seg == it.s);
+            const bool store = CMP ? in_piece : i < T && seg == it.s;
 #pragma unroll
             for (int cc = 0; cc < 2; ++cc) {
                 const int c = 2 * ch + cc;
@@ -925,7 +924,8 @@ __global__ void __launch_bounds__(NT_BWD, 1)
     __shared__ __align__(8) uint64_t kv_full, qd_full[QD_ST], qd_empty[QD_ST], sd_full[2], sd_free[2], pd_full[2];
     __shared__ uint32_t tmem_base;
 
-    constexpr bool SEGK = MODE == 1, CMP = MODE == 2;
+    static_assert(MODE == 1 || MODE == 2, "segment key rows (1) or compact views (2)");
+    constexpr bool CMP = MODE == 2;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int grp = p.Hq / p.Hkv;
     // KV head outermost: the CTAs resident at one time share one head's Q / dO
@@ -962,7 +962,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
         nlist = ((seg_hi - 1) >> 7) - qlo + 1;
         krow0 = (v.traj_km[b] + (int64_t)sk * nt + kt) * 128;
     }
-    if (SEGK) {
+    if (!CMP) {
         // item (k-tile, segment blockIdx.y): only that segment's rows, which
         // read the segment's key rows; its q-tiles are a contiguous run of the
         // ascending list
@@ -1125,8 +1125,8 @@ __global__ void __launch_bounds__(NT_BWD, 1)
         // ... of which the item's rows: [jlo, iend). CMP: compact key jk of
         // view_s is seen by the segment's rows whose compact index reaches it
         const bool kin = !CMP || jk < clen;
-        const int jlo = CMP ? (kin ? seg_lo + max(0, jk - nb) : 0) : SEGK ? max(jk, seg_lo) : jk;
-        const int iend = CMP ? (kin ? seg_hi : 0) : SEGK ? min(iend0, seg_hi) : iend0;
+        const int jlo = CMP ? (kin ? seg_lo + max(0, jk - nb) : 0) : max(jk, seg_lo);
+        const int iend = CMP ? (kin ? seg_hi : 0) : min(iend0, seg_hi);
         const uint32_t lane_base = tmem + ((uint32_t)(qw * 32) << 16);
         bool ok = true;
         // (-LSE2, Delta) of this warp's 32 query rows of a step: 256 contiguous
@@ -1194,7 +1194,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             cur = nxt;
             advance(nxt);
         }
-        if (MODE != 0 && ok && mbar_wait(&sd_free[(nsteps - 1) & 1], ((nsteps - 1) >> 1) & 1, status, 323)) {
+        if (ok && mbar_wait(&sd_free[(nsteps - 1) & 1], ((nsteps - 1) >> 1) & 1, status, 323)) {
             // float32 partials of this segment, unscaled dV and scaled dK
             // (SEGK: per segment key row; CMP: per compact row)
             tc_fence_after();
@@ -1218,41 +1218,6 @@ __global__ void __launch_bounds__(NT_BWD, 1)
                                             __uint_as_float(o[4 * x + 2]) * mul, __uint_as_float(o[4 * x + 3]) * mul);
                     }
                 }
-            }
-        } else if (MODE == 0 && ok && nsteps > 0 &&
-                   mbar_wait(&sd_free[(nsteps - 1) & 1], ((nsteps - 1) >> 1) & 1, status, 323)) {
-            tc_fence_after();
-            const int64_t row = ((tok0 + je) * p.Hkv + kvh) * DH;
-            uint32_t o[32];
-#pragma unroll
-            for (int pass = 0; pass < 2; ++pass) {
-                __nv_bfloat16* dst = (pass == 0 ? p.dV : p.dK) + row;
-                const float mul = pass == 0 ? 1.f : p.scale;
-                const uint32_t col = pass == 0 ? TM_DV : TM_DK;
-#pragma unroll
-                for (int cc = 0; cc < 2; ++cc) {
-                    const int c = 2 * ch + cc;
-                    tmem_ld32(lane_base + col + c * 32, o);
-                    tmem_wait_ld();
-                    if (jk < T) {
-#pragma unroll
-                        for (int x = 0; x < 4; ++x) {
-                            uint4 pk;
-                            pk.x = pack_bf16(__uint_as_float(o[8 * x + 0]) * mul, __uint_as_float(o[8 * x + 1]) * mul);
-                            pk.y = pack_bf16(__uint_as_float(o[8 * x + 2]) * mul, __uint_as_float(o[8 * x + 3]) * mul);
-                            pk.z = pack_bf16(__uint_as_float(o[8 * x + 4]) * mul, __uint_as_float(o[8 * x + 5]) * mul);
-                            pk.w = pack_bf16(__uint_as_float(o[8 * x + 6]) * mul, __uint_as_float(o[8 * x + 7]) * mul);
-                            *reinterpret_cast<uint4*>(dst + c * 32 + 8 * x) = pk;
-                        }
-                    }
-                }
-            }
-        } else if (MODE == 0 && jk < T) {
-            // no listed q-tile (cannot happen: the diagonal tile is always listed)
-            const int64_t row = ((tok0 + je) * p.Hkv + kvh) * DH;
-            for (int c = 0; c < DH; ++c) {
-                p.dK[row + c] = __float2bfloat16(0.f);
-                p.dV[row + c] = __float2bfloat16(0.f);
             }
         }
     }
@@ -1473,7 +1438,6 @@ mw_status attn_bwd_tc_segk(const mw_vis_layout* L, const void* vis, const void* 
     p.lsd = lsd;
     p.n_rows = n_rows;
     p.dQ = (__nv_bfloat16*)dQ;
-    p.dK = p.dV = nullptr;
     p.dKseg = dKseg;
     p.dVseg = dVseg;
     p.junction_items = 0;
@@ -1582,7 +1546,6 @@ mw_status attn_bwd_tc(const mw_vis_layout* L, const void* vis, const void* Q, co
     p.lsd = lsd;
     p.n_rows = n_rows;
     p.dQ = (__nv_bfloat16*)dQ;
-    p.dK = p.dV = nullptr;
     p.dKseg = dKc;
     p.dVseg = dVc;
     p.junction_items = 0;
