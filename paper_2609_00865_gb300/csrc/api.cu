@@ -17,9 +17,10 @@ mw_status lm_fwd_simt(const void*, const void*, const int32_t*, const int32_t*, 
 mw_status lm_bwd_simt(const void*, const void*, const int32_t*, const int32_t*, int, int, int, int, int,
                       const float*, const float*, float, void*, float*, cudaStream_t);
 mw_status attn_fwd_tc(const mw_vis_layout*, const void*, const void*, const void*, const void*, void*, float*, int,
-                      int, float, void*, cudaStream_t);
+                      int, float, void*, cudaStream_t, const float* = nullptr);
 mw_status attn_bwd_tc(const mw_vis_layout*, const void*, const void*, const void*, const void*, const void*,
-                      const void*, const float*, void*, void*, void*, int, int, float, void*, cudaStream_t);
+                      const void*, const float*, void*, void*, void*, int, int, float, void*, cudaStream_t,
+                      const float* = nullptr);
 int64_t attn_fwd_tc_ws(const mw_vis_layout*, int);
 int64_t attn_bwd_tc_ws(const mw_vis_layout*, int, int);
 int64_t attn_lsd_ws(const mw_vis_layout*, int);
@@ -274,6 +275,13 @@ static RopeWs rope_ws_layout(const mw_vis_layout* L, int Hq, int Hkv, int Dh, in
     const int64_t krows = L->n_keymask * MW_TILE;
     const bool tc = rope_tc(Dh, dtype);
     int64_t o = 0;
+    if (tc) {   // rotated queries, then the compact attention's own workspace (keys rotated by rank)
+        w.q = o; o = align256(o + esz * L->total_tokens * Hq * Dh);
+        w.kseg = w.delta = w.dkseg = w.dvseg = o;
+        w.fwd_bytes = o + attn_fwd_tc_ws(L, Hkv);
+        w.bwd_bytes = o + attn_bwd_tc_ws(L, Hq, Hkv);
+        return w;
+    }
     w.q = o; o = align256(o + esz * L->total_tokens * Hq * Dh);
     w.kseg = o; o = align256(o + esz * krows * Hkv * Dh);
     w.fwd_bytes = o;
@@ -294,10 +302,12 @@ static mw_status rope_args(const mw_vis_layout* L, const void* vis, const int32_
 }
 
 extern "C" mw_status mw_logical_positions(const mw_vis_layout* L, const void* vis, int32_t* pos, void* stream) {
-    if (L && L->kind != MW_VIEWS_EDITS) return MW_ESHAPE;   // rotary kernels read the tile lists
     if (!L) return MW_EINVAL;
     if (L->n_keymask == 0) return MW_OK;
     if (!vis || !pos) return MW_EINVAL;
+    if (L->kind != MW_VIEWS_EDITS)   // views in list order: the positions are the build's ranks
+        return cuda_status(cudaMemcpyAsync(pos, at<char>(vis, L->off_cpos), 4 * MW_TILE * (size_t)L->n_keymask,
+                                           cudaMemcpyDeviceToDevice, (cudaStream_t)stream));
     return logical_positions(L, vis, pos, (cudaStream_t)stream);
 }
 
@@ -311,7 +321,6 @@ extern "C" mw_status mw_rope_table(int n_pos, int Dh, double theta, float* table
 extern "C" mw_status mw_rope_rows(const mw_vis_layout* L, const void* vis, const int32_t* pos, const float* table,
                                   int n_pos, const void* X, void* Y, int H, int Dh, int dtype, int inverse,
                                   void* stream) {
-    if (L && L->kind != MW_VIEWS_EDITS) return MW_ESHAPE;   // rotary kernels read the tile lists
     if (dtype != MW_F32 && dtype != MW_BF16) return MW_EDTYPE;
     if (H <= 0 || Dh <= 0 || Dh % 2 != 0) return MW_ESHAPE;
     mw_status st = rope_args(L, vis, pos, table, n_pos);
@@ -322,7 +331,6 @@ extern "C" mw_status mw_rope_rows(const mw_vis_layout* L, const void* vis, const
 
 extern "C" mw_status mw_masked_attn_rope_ws(const mw_vis_layout* L, int Hq, int Hkv, int Dh, int dtype,
                                             size_t* fwd_bytes, size_t* bwd_bytes) {
-    if (L && L->kind != MW_VIEWS_EDITS) return MW_ESHAPE;   // rotary kernels read the tile lists
     if (!L || !fwd_bytes || !bwd_bytes) return MW_EINVAL;
     if (dtype != MW_F32 && dtype != MW_BF16) return MW_EDTYPE;
     if (Hq <= 0 || Hkv <= 0 || Hq % Hkv != 0 || !(Dh == 64 || Dh == 128)) return MW_ESHAPE;
@@ -336,7 +344,8 @@ extern "C" mw_status mw_masked_attn_rope_fwd(const mw_vis_layout* L, const void*
                                              const float* table, int n_pos, const void* Q, const void* K,
                                              const void* V, void* O, float* LSE, int Hq, int Hkv, int Dh, int dtype,
                                              float scale, void* ws, void* stream) {
-    if (L && L->kind != MW_VIEWS_EDITS) return MW_ESHAPE;   // rotary kernels read the tile lists
+    // views of an EVENTS record have no tile lists: only the compact path reads them
+    if (L && L->kind != MW_VIEWS_EDITS && !rope_tc(Dh, dtype)) return MW_ESHAPE;
     mw_status st = attn_args(L, vis, Hq, Hkv, Dh, dtype, scale);
     if (st != MW_OK) return st;
     if ((st = rope_args(L, vis, pos, table, n_pos)) != MW_OK) return st;
@@ -347,8 +356,9 @@ extern "C" mw_status mw_masked_attn_rope_fwd(const mw_vis_layout* L, const void*
     void* q = at<char>(ws, w.q);
     void* kseg = at<char>(ws, w.kseg);
     if ((st = rope_rows(L, vis, pos, table, n_pos, Q, q, Hq, Dh, dtype, false, s)) != MW_OK) return st;
+    // compact path: each key turned by its rank in the segment's view (its logical position) as it is gathered
+    if (rope_tc(Dh, dtype)) return attn_fwd_tc(L, vis, q, K, V, O, LSE, Hq, Hkv, scale, kseg, s, table);
     if ((st = rope_segments(L, vis, pos, table, n_pos, K, kseg, Hkv, Dh, dtype, s)) != MW_OK) return st;
-    if (rope_tc(Dh, dtype)) return attn_fwd_tc_segk(L, vis, q, kseg, V, O, LSE, Hq, Hkv, scale, s);
     return attn_fwd_simt_segk(L, vis, q, kseg, V, O, LSE, Hq, Hkv, Dh, dtype, scale, s);
 }
 
@@ -357,7 +367,7 @@ extern "C" mw_status mw_masked_attn_rope_bwd(const mw_vis_layout* L, const void*
                                              const void* V, const void* O, const void* dO, const float* LSE,
                                              void* dQ, void* dK, void* dV, int Hq, int Hkv, int Dh, int dtype,
                                              float scale, void* ws, void* stream) {
-    if (L && L->kind != MW_VIEWS_EDITS) return MW_ESHAPE;   // rotary kernels read the tile lists
+    if (L && L->kind != MW_VIEWS_EDITS && !rope_tc(Dh, dtype)) return MW_ESHAPE;
     mw_status st = attn_args(L, vis, Hq, Hkv, Dh, dtype, scale);
     if (st != MW_OK) return st;
     if ((st = rope_args(L, vis, pos, table, n_pos)) != MW_OK) return st;
@@ -370,21 +380,18 @@ extern "C" mw_status mw_masked_attn_rope_bwd(const mw_vis_layout* L, const void*
     float* delta = at<float>(ws, w.delta);
     float* dkseg = at<float>(ws, w.dkseg);
     if ((st = rope_rows(L, vis, pos, table, n_pos, Q, q, Hq, Dh, dtype, false, s)) != MW_OK) return st;
-    if ((st = rope_segments(L, vis, pos, table, n_pos, K, kseg, Hkv, Dh, dtype, s)) != MW_OK) return st;
     // dQ first holds the gradient of the rotated queries, then is turned back in place
     if (rope_tc(Dh, dtype)) {
-        float* dvseg = at<float>(ws, w.dvseg);
-        if ((st = attn_bwd_tc_segk(L, vis, q, kseg, V, O, dO, LSE, dQ, dkseg, dvseg, Hq, Hkv, scale, delta, s)) !=
-            MW_OK)
+        // compact path: keys turned by rank as they are gathered, dK partials turned back as they are summed
+        if ((st = attn_bwd_tc(L, vis, q, K, V, O, dO, LSE, dQ, dK, dV, Hq, Hkv, scale, kseg, s, table)) != MW_OK)
             return st;
-        if ((st = rope_segments_bwd(L, vis, pos, table, n_pos, dvseg, dV, Hkv, Dh, dtype, false, s)) != MW_OK)
-            return st;
-    } else {
-        if ((st = attn_delta(L, O, dO, Hq, Dh, dtype, delta, s)) != MW_OK) return st;
-        if ((st = attn_bwd_simt_segk(L, vis, q, kseg, V, dO, LSE, delta, dQ, dkseg, dV, Hq, Hkv, Dh, dtype, scale,
-                                     s)) != MW_OK)
-            return st;
+        return rope_rows(L, vis, pos, table, n_pos, dQ, dQ, Hq, Dh, dtype, true, s);
     }
+    if ((st = rope_segments(L, vis, pos, table, n_pos, K, kseg, Hkv, Dh, dtype, s)) != MW_OK) return st;
+    if ((st = attn_delta(L, O, dO, Hq, Dh, dtype, delta, s)) != MW_OK) return st;
+    if ((st = attn_bwd_simt_segk(L, vis, q, kseg, V, dO, LSE, delta, dQ, dkseg, dV, Hq, Hkv, Dh, dtype, scale, s)) !=
+        MW_OK)
+        return st;
     if ((st = rope_rows(L, vis, pos, table, n_pos, dQ, dQ, Hq, Dh, dtype, true, s)) != MW_OK) return st;
     return rope_segments_bwd(L, vis, pos, table, n_pos, dkseg, dK, Hkv, Dh, dtype, true, s);
 }

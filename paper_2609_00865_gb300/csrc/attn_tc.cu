@@ -1,46 +1,42 @@
 // Tensor-core masked GQA attention, bf16 in / fp32 accumulate, head dim 128.
 //
-// The plain path (MODE 2, "compact") scores each segment's rows against that
-// segment's compact sequence -- its live view gathered in order (§4.1's
-// materialised branch; the builder's csrc / cpos maps), so that a row's keys
-// are a prefix of it: tiles are FULL or hold a per-row prefix, and the
-// evicted keys inside a physical tile cost nothing. Per q-tile item the keys
-// are compact tiles 0 .. (last row's index) / 128; dK / dV run per (compact
-// key tile, segment) into float32 partials per compact row, summed per key
-// in segment order (k_cmp_reduce). This is the same 4D-masked computation
-// (§4.3 Theorem "materialization equivalence"): every row still reads each
-// visible key once.
+// Each segment's rows are scored against the segment's compact sequence: its
+// live view gathered in order (§4.1's materialised branch; the visibility
+// build's csrc / cpos / seg_len), so a row's visible keys are the prefix of
+// that sequence up to its own index -- the 4D-masked computation (§4.2 mask,
+// §4.3 Theorem "materialization equivalence") with every visible key read
+// once per row and the evicted keys inside a physical tile costing nothing.
+// Row i of segment s has compact index nb_s + (i - J_s), nb_s being the keys
+// of view_s before the segment's rows. For rotary positions the keys are
+// gathered already turned to their rank (their logical position in view_s)
+// and the dK partials turned back as they are summed.
 //
-// The rotary path (MODE 1, below) keeps physical key tiles:
-// Mask (§4.2): key j is visible to row i iff j <= i < omega(j). A tile's
-// class comes from the visibility builder: EMPTY tiles are never listed,
-// FULL tiles run unmasked, PARTIAL and diagonal tiles apply the row's
-// per-(segment, k-tile) view bits (and causality on the diagonal). For a row
-// of segment s, "omega(j) > i" is the same as "j is in view_s", because every
-// lifetime ends at a junction; so one 128-bit word per (segment, k-tile)
-// replaces 128 lifetime compares.
+// q-tile kernels (forward, dQ): one CTA per (q-tile, query head) serving the
+// segment of the tile's first row, heaviest q-tiles first, plus a second
+// launch ("junction items") with one CTA per (segment starting inside a
+// tile, head); a CTA stores only its own segment's rows. It walks compact key
+// tiles 0 .. (last row's index) / 128: FULL when it covers the whole q-tile
+// and every row reaches the tile's last key, otherwise PARTIAL with a
+// per-row prefix mask, DEAD_HI when no row reaches the tile's second half.
 //
-// Forward kernel (one CTA per (q-tile, q-head), heaviest q-tiles first):
-//   warp 0      TMA producer: Q once, then K_j / V_j of each listed k-tile
+// Forward kernel:
+//   warp 0      TMA producer: Q once, then K_j / V_j of each compact tile
 //               (2-stage rings, 128-byte swizzle)
 //   warp 1      TMEM allocator + single-thread tcgen05.mma issuer:
-//               S_j = Q K_j^T into one of two TMEM S buffers, then
-//               O += P_{j-1} V_{j-1} once the softmax has written P_{j-1}
+//               S_j = Q K_j^T into one of two TMEM S buffers
 //   warps 2..5  softmax / epilogue, one query row per thread: online softmax
 //               in the exp2 domain with lazy rescaling of O (only when the
-//               running max grows by more than 2^8), P written as bf16 into
-//               shared memory, O / l and the log-sum-exp written at the end.
+//               running max grows by more than 2^8), P written as bf16 over
+//               its own S buffer, O / l and the log-sum-exp written at the end
+//   warp 6      O += P_{j} V_{j} once the softmax has written P_{j}
+//
+// dK / dV kernel: one CTA per (compact key tile, segment, KV head) over the
+// run of q-tiles whose rows see its keys, writing float32 partials per
+// compact row; k_cmp_reduce sums each key's partials over the segments
+// holding it, in segment order (deterministic, no atomics).
+//
 // All waits are bounded (tc::mbar_wait); a timeout ends the CTA and is
 // reported through the visibility status word.
-//
-// SEGK instantiations read keys from "segment key rows" (row (traj_km[b] +
-// s nt_b) 128 + j holds key j as seen by segment s, e.g. rotated to its
-// logical position in view_s). A q-tile CTA then serves one segment: the main
-// launch the segment of the tile's first row, a second launch ("junction
-// items") one CTA per (junction inside a tile, head) for the segment that the
-// junction starts; each stores only its own segment's rows. The dK/dV kernel
-// takes one CTA per (k-tile, segment) over that segment's q-tiles and writes
-// float32 partial gradients per segment key row.
 
 #include <math.h>
 
@@ -94,7 +90,7 @@ struct FwdParams {
     float scale_log2;
     __nv_bfloat16* O;
     float* LSE;
-    int junction_items;   // SEGK: 0 = main launch, 1 = one CTA per (junction, head)
+    int junction_items;   // 0 = main launch, 1 = one CTA per (segment starting inside a tile, head)
 };
 
 // Work item of a q-tile kernel: trajectory b, local q-tile qt, query head h
@@ -131,7 +127,7 @@ __device__ __forceinline__ QItem q_item(const VisView& v, int Hq, int max_tiles,
     return it;
 }
 
-// Compact mode (MODE 2): keys come from each segment's compact sequence
+// Compact views: keys come from each segment's compact sequence
 // (view_s gathered in order, §4.1 LogitTree), stored at rows
 // (traj_km[b] + s nt) 128 + c of a compact K / V buffer. A q-tile item serves
 // the rows of one segment, whose compact index is nb + (i - seg_lo) with nb
@@ -215,7 +211,6 @@ __device__ __forceinline__ uint64_t mnmaj(uint32_t base, int ks) {
     return sdesc_sw128(base + ks * 2048, HALF_B, 1024);
 }
 
-template <int MODE>
 __global__ void __launch_bounds__(NT_FWD, 1)
     k_attn_fwd_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                   const __grid_constant__ CUtensorMap tmV, FwdParams p) {
@@ -226,8 +221,6 @@ __global__ void __launch_bounds__(NT_FWD, 1)
     __shared__ uint32_t tmem_base;
     __shared__ int abort_flag;
 
-    static_assert(MODE == 1 || MODE == 2, "segment key rows (1) or compact views (2)");
-    constexpr bool CMP = MODE == 2;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const VisView& v = p.v;
     const QItem it = q_item(v, p.Hq, p.max_tiles, p.n_traj, p.junction_items);
@@ -238,11 +231,9 @@ __global__ void __launch_bounds__(NT_FWD, 1)
     const int64_t tok0 = v.traj_tok[b];
     const int T = v.traj_tok[b + 1] - (int)tok0;
     const int kvh = h / (p.Hq / p.Hkv);
-    CPiece cp{};
-    if (CMP) cp = cmp_piece(v, b, it.s, qt, T);
-    const int p0 = CMP ? 0 : v.fwd_ptr[g];
-    const int n = CMP ? cp.clast / 128 + 1 : v.fwd_ptr[g + 1] - p0;
-    auto entry = [&](int j) -> int { return CMP ? cmp_entry(cp, j) : v.fwd_idx[p0 + j]; };
+    const CPiece cp = cmp_piece(v, b, it.s, qt, T);
+    const int n = cp.clast / 128 + 1;   // compact key tiles 0 .. (last row's index) / 128
+    auto entry = [&](int j) -> int { return cmp_entry(cp, j); };
     int32_t* status = v.status;
 
     if (threadIdx.x == 0) {
@@ -278,13 +269,12 @@ __global__ void __launch_bounds__(NT_FWD, 1)
             prefetch_tmap(&tmV);
             mbar_expect_tx(&q_full, TILE_B);
             load_tile(sm + SM_Q, &tmQ, &q_full, h, (int)(tok0 + qt * 128));
-            // first K row of the trajectory (SEGK: of the item's segment key
-            // rows; CMP: of the segment's compact sequence, for V as well)
+            // first K / V row of the item's segment's compact sequence
             const int64_t krow0 = (v.traj_km[b] + (int64_t)it.s * nt) * 128;
             for (int j = 0; j < n; ++j) {
                 const int kt = entry(j) >> 4;
                 const int s = j & 1;
-                const int row = (int)((CMP ? krow0 : tok0) + kt * 128);
+                const int row = (int)(krow0 + kt * 128);
                 if (j >= 2 && !mbar_wait(&k_empty[s], ((j - 2) >> 1) & 1, status, 101)) { abort_flag = 1; break; }
                 mbar_expect_tx(&k_full[s], TILE_B);
                 load_tile(sm + SM_K + s * TILE_B, &tmK, &k_full[s], kvh, (int)(krow0 + kt * 128));
@@ -362,12 +352,10 @@ __global__ void __launch_bounds__(NT_FWD, 1)
         const int rl = qw * 32 + lane;          // row inside the q-tile = TMEM lane
         const int i = qt * 128 + rl;
         const int ie = min(i, T - 1);
-        const int seg = v.seg[tok0 + ie];
-        const uint4* km = reinterpret_cast<const uint4*>(v.keymask) + v.traj_km[b] + (int64_t)seg * nt;
-        // CMP: this row's compact index (rows outside the item see no key)
-        const bool in_piece = !CMP || (i >= cp.r0 && i < cp.r1);
-        const int crow = CMP ? (in_piece ? cp.cfirst + i - cp.r0 : -(1 << 30)) : 0;
-        auto mask_words = [&](int e) -> uint4 { return CMP ? prefix_words(crow - (e >> 4) * 128) : km[e >> 4]; };
+        // this row's compact index (rows outside the item see no key)
+        const bool in_piece = i >= cp.r0 && i < cp.r1;
+        const int crow = in_piece ? cp.cfirst + i - cp.r0 : -(1 << 30);
+        auto mask_words = [&](int e) -> uint4 { return prefix_words(crow - (e >> 4) * 128); };
         const uint32_t lane_base = tmem + ((uint32_t)(qw * 32) << 16);
         float m = -INFINITY, l = 0.f;
         bool ok = true;
@@ -461,7 +449,6 @@ __global__ void __launch_bounds__(NT_FWD, 1)
                 e_nxt = j + 2 < n ? entry(j + 2) : 0;
             }
             const int kt = e >> 4, cls = e & 3;
-            const bool diag = !CMP && kt == qt;   // compact tiles carry causality in their mask words
             if (!mbar_wait(&s_full[j & 1], (j >> 1) & 1, status, 301)) { ok = false; break; }
             tc_fence_after();
             // a tile whose first or second key half no row sees was computed as
@@ -473,8 +460,8 @@ __global__ void __launch_bounds__(NT_FWD, 1)
                 const uint32_t w0 = lh ? wv.z : wv.x, w1 = lh ? wv.w : wv.y;
                 alpha = soft_tile(std::integral_constant<int, 2>(), sbuf, true, 127, w0, w1, 0u, 0u);
             } else {
-                alpha = soft_tile(std::integral_constant<int, 4>(), sbuf, cls != MW_TILE_FULL || diag,
-                                  diag ? ie - kt * 128 : 127, wv.x, wv.y, wv.z, wv.w);
+                alpha = soft_tile(std::integral_constant<int, 4>(), sbuf, cls != MW_TILE_FULL, 127, wv.x, wv.y,
+                                  wv.z, wv.w);
             }
             // O was last written by PV_{j-1}; rescale it when the max moved
             if (j >= 1 && __any_sync(0xffffffffu, alpha != 1.f)) {
@@ -507,7 +494,7 @@ __global__ void __launch_bounds__(NT_FWD, 1)
             const float inv = 1.f / l;
             __nv_bfloat16* orow = p.O + ((tok0 + ie) * p.Hq + h) * DH;
             uint32_t o[32];
-            const bool store = CMP ? in_piece : i < T && seg == it.s;
+            const bool store = in_piece;
 #pragma unroll
             for (int c = 0; c < 4; ++c) {
                 tmem_ld32(lane_base + TM_O + c * 32, o);
@@ -562,12 +549,11 @@ struct BwdParams {
     const float2* lsd;     // [Hq][n_tiles * 128] (-LSE_i log2 e, Delta_i), rows padded to whole tiles
     int64_t n_rows;        // n_tiles * 128
     __nv_bfloat16* dQ;
-    int junction_items;    // SEGK dQ: as FwdParams
-    float* dKseg;          // dK/dV: float32 partials per segment key row (SEGK) or compact row [rows][Hkv][DH]
+    int junction_items;    // dQ: as FwdParams
+    float* dKseg;          // dK/dV: float32 partials per compact row [rows][Hkv][DH]
     float* dVseg;
 };
 
-template <int MODE>
 __global__ void __launch_bounds__(NT_BWD, 1)
     k_attn_dq_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmDO,
                  const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, BwdParams p) {
@@ -577,8 +563,6 @@ __global__ void __launch_bounds__(NT_BWD, 1)
         dp_full, dp_free, ds_full[2], dq_fin;
     __shared__ uint32_t tmem_base;
 
-    static_assert(MODE == 1 || MODE == 2, "segment key rows (1) or compact views (2)");
-    constexpr bool CMP = MODE == 2;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const VisView& v = p.v;
     const QItem it = q_item(v, p.Hq, p.max_tiles, p.n_traj, p.junction_items);
@@ -589,11 +573,9 @@ __global__ void __launch_bounds__(NT_BWD, 1)
     const int64_t tok0 = v.traj_tok[b];
     const int T = v.traj_tok[b + 1] - (int)tok0;
     const int kvh = h / (p.Hq / p.Hkv);
-    CPiece cp{};
-    if (CMP) cp = cmp_piece(v, b, it.s, qt, T);
-    const int p0 = CMP ? 0 : v.fwd_ptr[g];
-    const int n = CMP ? cp.clast / 128 + 1 : v.fwd_ptr[g + 1] - p0;
-    auto entry = [&](int j) -> int { return CMP ? cmp_entry(cp, j) : v.fwd_idx[p0 + j]; };
+    const CPiece cp = cmp_piece(v, b, it.s, qt, T);
+    const int n = cp.clast / 128 + 1;   // compact key tiles 0 .. (last row's index) / 128
+    auto entry = [&](int j) -> int { return cmp_entry(cp, j); };
     int32_t* status = v.status;
     if (*(volatile int32_t*)&status[1]) return;
 
@@ -632,13 +614,12 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             mbar_expect_tx(&q_full, 2 * TILE_B);
             load_tile(sm + DQ_Q, &tmQ, &q_full, h, row0);
             load_tile(sm + DQ_DO, &tmDO, &q_full, h, row0);
-            // first K row of the trajectory (SEGK: of the item's segment key
-            // rows; CMP: of the segment's compact sequence, for V as well)
+            // first K / V row of the item's segment's compact sequence
             const int64_t krow0 = (v.traj_km[b] + (int64_t)it.s * nt) * 128;
             for (int j = 0; j < n; ++j) {
                 const int kt = entry(j) >> 4;
                 const int s = j & 1;
-                const int row = (int)((CMP ? krow0 : tok0) + kt * 128);
+                const int row = (int)(krow0 + kt * 128);
                 if (j >= 2 && !mbar_wait(&v_empty[s], ((j - 2) >> 1) & 1, status, 111)) break;
                 mbar_expect_tx(&v_full[s], TILE_B);
                 load_tile(sm + DQ_V + s * TILE_B, &tmV, &v_full[s], kvh, row);
@@ -738,12 +719,10 @@ __global__ void __launch_bounds__(NT_BWD, 1)
         const int rl = qw * 32 + lane;
         const int i = qt * 128 + rl;
         const int ie = min(i, T - 1);
-        const int seg = v.seg[tok0 + ie];
-        const uint4* km = reinterpret_cast<const uint4*>(v.keymask) + v.traj_km[b] + (int64_t)seg * nt;
-        // CMP: this row's compact index (rows outside the item see no key)
-        const bool in_piece = !CMP || (i >= cp.r0 && i < cp.r1);
-        const int crow = CMP ? (in_piece ? cp.cfirst + i - cp.r0 : -(1 << 30)) : 0;
-        auto mask_words = [&](int e) -> uint4 { return CMP ? prefix_words(crow - (e >> 4) * 128) : km[e >> 4]; };
+        // this row's compact index (rows outside the item see no key)
+        const bool in_piece = i >= cp.r0 && i < cp.r1;
+        const int crow = in_piece ? cp.cfirst + i - cp.r0 : -(1 << 30);
+        auto mask_words = [&](int e) -> uint4 { return prefix_words(crow - (e >> 4) * 128); };
         const uint32_t lane_base = tmem + ((uint32_t)(qw * 32) << 16);
         const float2 ld = p.lsd[(int64_t)h * p.n_rows + g * 128 + rl];
         const uint64_t c2 = f2(p.scale_log2, p.scale_log2), n2 = f2(ld.x, ld.x), dl2 = f2(ld.y, ld.y);
@@ -823,7 +802,6 @@ __global__ void __launch_bounds__(NT_BWD, 1)
                 e_nxt = j + 2 < n ? entry(j + 2) : 0;
             }
             const int kt = e >> 4, cls = e & 3;
-            const bool diag = !CMP && kt == qt;   // compact tiles carry causality in their mask words
             if (!mbar_wait(&s_full[j & 1], (j >> 1) & 1, status, 311)) { ok = false; break; }
             tc_fence_after();
             const uint32_t sbuf = lane_base + TM_S0 + (j & 1) * 128;
@@ -835,16 +813,8 @@ __global__ void __launch_bounds__(NT_BWD, 1)
                 stepok = dq_step(std::integral_constant<int, 1>(), j, sbuf + 32 * ch, lane_base + TM_DP + 32 * ch, wm, 0u);
             } else {
                 uint32_t wd[4] = {0xffffffffu, 0xffffffffu, 0xffffffffu, 0xffffffffu};
-                if (cls != MW_TILE_FULL || diag) {
+                if (cls != MW_TILE_FULL) {
                     wd[0] = wv.x; wd[1] = wv.y; wd[2] = wv.z; wd[3] = wv.w;
-                    if (diag) {
-                        const int lim = ie - kt * 128;
-#pragma unroll
-                        for (int q = 0; q < 4; ++q) {
-                            const int hi = lim - 32 * q;
-                            wd[q] &= hi >= 31 ? 0xffffffffu : (hi < 0 ? 0u : ((2u << hi) - 1u));
-                        }
-                    }
                 }
                 stepok = dq_step(std::integral_constant<int, 2>(), j, sbuf + 64 * ch, lane_base + TM_DP + 64 * ch,
                                  ch ? wd[2] : wd[0], ch ? wd[3] : wd[1]);
@@ -859,7 +829,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             tc_fence_after();
             __nv_bfloat16* qrow = p.dQ + ((tok0 + ie) * p.Hq + h) * DH;
             uint32_t o[32];
-            const bool store = CMP ? in_piece : i < T && seg == it.s;
+            const bool store = in_piece;
 #pragma unroll
             for (int cc = 0; cc < 2; ++cc) {
                 const int c = 2 * ch + cc;
@@ -888,15 +858,16 @@ __global__ void __launch_bounds__(NT_BWD, 1)
 }
 
 // ----------------------------------------------------------------------------
-// dK / dV kernel (KV-stationary, one CTA per (k-tile, kv-head), smallest
-// k-tiles -- the longest lists -- first). Steps run over the k-tile's bwd list
-// (last q-tile first) x the group's query heads x two 64-row halves:
+// dK / dV kernel (KV-stationary, one CTA per (compact key tile, kv-head,
+// segment), smallest key tiles -- the longest runs -- first). Steps run over
+// the run of q-tiles whose rows see the tile's keys (last q-tile first) x the
+// group's query heads x two 64-row halves:
 //   S^T = K Q^T, dP^T = V dO^T   (M=128 keys, N=64 rows; TMEM, double-buffered)
 //   P^T = exp2(S^T c - LSE2_i), dS^T = P^T (dP^T - Delta_i) on visible pairs,
 //   written as bf16 over their own S^T / dP^T TMEM buffers
 //   dV += P^T dO, dK += dS^T Q   (P^T, dS^T TMEM operands; dO, Q MN-major in smem)
-// The rows that see key j form the interval [j, min(omega(j), T)), so the mask
-// is two compares per element.
+// The segment's rows that see compact key c form the interval
+// [J_s + max(0, c - nb_s), J_{s+1}), so the mask is two compares per element.
 constexpr uint32_t HT_B = 64 * DH * 2;     // 64-row half tile: two [64][64] swizzled halves
 constexpr uint32_t HT_HALF = HT_B / 2;
 constexpr uint32_t KV_K = 0;
@@ -915,7 +886,6 @@ __device__ __forceinline__ uint64_t mnmaj_ht(uint32_t base, int ks) {
     return sdesc_sw128(base + ks * 2048, HT_HALF, 1024);
 }
 
-template <int MODE>
 __global__ void __launch_bounds__(NT_BWD, 1)
     k_attn_dkdv_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmDO,
                    const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, BwdParams p) {
@@ -924,8 +894,6 @@ __global__ void __launch_bounds__(NT_BWD, 1)
     __shared__ __align__(8) uint64_t kv_full, qd_full[QD_ST], qd_empty[QD_ST], sd_full[2], sd_free[2], pd_full[2];
     __shared__ uint32_t tmem_base;
 
-    static_assert(MODE == 1 || MODE == 2, "segment key rows (1) or compact views (2)");
-    constexpr bool CMP = MODE == 2;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int grp = p.Hq / p.Hkv;
     // KV head outermost: the CTAs resident at one time share one head's Q / dO
@@ -937,57 +905,22 @@ __global__ void __launch_bounds__(NT_BWD, 1)
     const VisView& v = p.v;
     const int nt = v.traj_tile[b + 1] - v.traj_tile[b];
     if (kt >= nt) return;
-    const int64_t gk = v.traj_tile[b] + kt;
     const int64_t tok0 = v.traj_tok[b];
     const int T = v.traj_tok[b + 1] - (int)tok0;
-    int p0 = CMP ? 0 : v.bwd_ptr[gk];
-    int nlist = CMP ? 0 : v.bwd_ptr[gk + 1] - p0;
-    int seg_lo = 0, seg_hi = T;        // SEGK, CMP: rows [seg_lo, seg_hi) of the item's segment
-    int64_t krow0 = tok0 + kt * 128;   // first K row of the tile
-    int nb = 0, qlo = 0, clen = 0;     // CMP: keys of view_s before the segment, first q-tile, |view_s|
-    if (CMP) {
-        // item (compact key tile kt, segment blockIdx.y): keys kt*128.. of
-        // view_s; the rows that see one of them are the segment's rows whose
-        // compact index reaches kt*128, a contiguous run of q-tiles
-        const int sgb = v.traj_seg[b];
-        const int sk = blockIdx.y;
-        if (sk >= v.traj_seg[b + 1] - sgb) return;
-        clen = v.seg_len[sgb + sk];
-        if (kt * 128 >= clen) return;
-        seg_lo = v.seg_start[sgb + sk];
-        seg_hi = sgb + sk + 1 < v.traj_seg[b + 1] ? v.seg_start[sgb + sk + 1] : T;
-        nb = clen - (seg_hi - seg_lo);
-        const int rs = seg_lo + max(0, kt * 128 - nb);
-        qlo = rs >> 7;
-        nlist = ((seg_hi - 1) >> 7) - qlo + 1;
-        krow0 = (v.traj_km[b] + (int64_t)sk * nt + kt) * 128;
-    }
-    if (!CMP) {
-        // item (k-tile, segment blockIdx.y): only that segment's rows, which
-        // read the segment's key rows; its q-tiles are a contiguous run of the
-        // ascending list
-        const int sgb = v.traj_seg[b];
-        const int sk = blockIdx.y;
-        if (sk >= v.traj_seg[b + 1] - sgb) return;
-        seg_lo = v.seg_start[sgb + sk];
-        seg_hi = sgb + sk + 1 < v.traj_seg[b + 1] ? v.seg_start[sgb + sk + 1] : T;
-        if (kt * 128 >= seg_hi) return;   // every key of the tile comes after the segment
-        const int qlo = seg_lo >> 7, qhi = (seg_hi - 1) >> 7;
-        int a = 0, z = nlist;             // first entry with q-tile >= qlo
-        while (a < z) {
-            const int m = (a + z) >> 1;
-            if ((v.bwd_idx[p0 + m] >> 4) < qlo) a = m + 1; else z = m;
-        }
-        int c = a, y = nlist;             // first entry with q-tile > qhi
-        while (c < y) {
-            const int m = (c + y) >> 1;
-            if ((v.bwd_idx[p0 + m] >> 4) <= qhi) c = m + 1; else y = m;
-        }
-        p0 += a;
-        nlist = c - a;
-        if (nlist == 0) return;           // no row of the segment sees a key of the tile
-        krow0 = (v.traj_km[b] + (int64_t)sk * nt + kt) * 128;
-    }
+    // item (compact key tile kt, segment blockIdx.y): keys kt*128.. of view_s;
+    // the rows that see one of them are the segment's rows whose compact index
+    // reaches kt*128, a contiguous run of q-tiles
+    const int sgb = v.traj_seg[b];
+    const int sk = blockIdx.y;
+    if (sk >= v.traj_seg[b + 1] - sgb) return;
+    const int clen = v.seg_len[sgb + sk];                  // |view_s|
+    if (kt * 128 >= clen) return;
+    const int seg_lo = v.seg_start[sgb + sk];
+    const int seg_hi = sgb + sk + 1 < v.traj_seg[b + 1] ? v.seg_start[sgb + sk + 1] : T;
+    const int nb = clen - (seg_hi - seg_lo);               // keys of view_s before the segment's rows
+    const int qlo = (seg_lo + max(0, kt * 128 - nb)) >> 7;
+    const int nlist = ((seg_hi - 1) >> 7) - qlo + 1;
+    const int64_t krow0 = (v.traj_km[b] + (int64_t)sk * nt + kt) * 128;   // first compact K / V row
     const int nsteps = nlist * grp * 2;
     int32_t* status = v.status;
     if (*(volatile int32_t*)&status[1]) return;
@@ -1023,7 +956,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
     struct Cursor {
         int e, rem, qt, qt_next;
     };
-    auto list_qt = [&](int e) -> int { return e >= 0 ? (CMP ? qlo + e : v.bwd_idx[p0 + e] >> 4) : 0; };
+    auto list_qt = [&](int e) -> int { return e >= 0 ? qlo + e : 0; };
     const Cursor first{nlist - 1, 0, list_qt(nlist - 1), list_qt(nlist - 2)};
     auto advance = [&](Cursor& c) {
         if (++c.rem == 2 * grp) {
@@ -1046,7 +979,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             prefetch_tmap(&tmV);
             mbar_expect_tx(&kv_full, 2 * TILE_B);
             load_tile(sm + KV_K, &tmK, &kv_full, kvh, (int)krow0);
-            load_tile(sm + KV_V, &tmV, &kv_full, kvh, (int)(CMP ? krow0 : tok0 + kt * 128));
+            load_tile(sm + KV_V, &tmV, &kv_full, kvh, (int)krow0);
             Cursor c = first;
             int s = 0;
             uint32_t ph = 0;
@@ -1119,14 +1052,12 @@ __global__ void __launch_bounds__(NT_BWD, 1)
         const int qw = warp & 3;
         const int ch = (warp - 2) >> 2;
         const int rl = qw * 32 + lane;               // key row inside the k-tile = TMEM lane
-        const int jk = kt * 128 + rl;
-        const int je = min(jk, T - 1);
-        const int iend0 = jk < T ? min(v.omega[tok0 + je], T) : 0;   // rows [jk, iend0) see this key
-        // ... of which the item's rows: [jlo, iend). CMP: compact key jk of
-        // view_s is seen by the segment's rows whose compact index reaches it
-        const bool kin = !CMP || jk < clen;
-        const int jlo = CMP ? (kin ? seg_lo + max(0, jk - nb) : 0) : max(jk, seg_lo);
-        const int iend = CMP ? (kin ? seg_hi : 0) : min(iend0, seg_hi);
+        const int jk = kt * 128 + rl;                // this thread's compact key
+        // compact key jk of view_s is seen by the segment's rows whose compact
+        // index reaches it: [jlo, iend)
+        const bool kin = jk < clen;
+        const int jlo = kin ? seg_lo + max(0, jk - nb) : 0;
+        const int iend = kin ? seg_hi : 0;
         const uint32_t lane_base = tmem + ((uint32_t)(qw * 32) << 16);
         bool ok = true;
         // (-LSE2, Delta) of this warp's 32 query rows of a step: 256 contiguous
@@ -1196,7 +1127,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
         }
         if (ok && mbar_wait(&sd_free[(nsteps - 1) & 1], ((nsteps - 1) >> 1) & 1, status, 323)) {
             // float32 partials of this segment, unscaled dV and scaled dK
-            // (SEGK: per segment key row; CMP: per compact row)
+            // per compact row
             tc_fence_after();
             const int64_t row = ((krow0 + rl) * p.Hkv + kvh) * DH;
             uint32_t o[32];
@@ -1210,7 +1141,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
                     const int c = 2 * ch + cc;
                     tmem_ld32(lane_base + col + c * 32, o);
                     tmem_wait_ld();
-                    if (CMP ? kin : jk < T) {
+                    if (kin) {
 #pragma unroll
                         for (int x = 0; x < 8; ++x)
                             *reinterpret_cast<float4*>(dst + c * 32 + 4 * x) =
@@ -1235,39 +1166,6 @@ __global__ void __launch_bounds__(NT_BWD, 1)
 // coordinates and the junction-item grid reach them.
 static bool segk_fits(const mw_vis_layout* L, int Hq) {
     return L->n_keymask * 128 <= INT32_MAX && L->n_segs * (int64_t)Hq <= INT32_MAX && L->max_segs <= 65535;
-}
-
-mw_status attn_fwd_tc_segk(const mw_vis_layout* L, const void* vis, const void* Q, const void* Kseg, const void* V,
-                           void* O, float* LSE, int Hq, int Hkv, float scale, cudaStream_t s) {
-    if (L->n_tiles == 0) return MW_OK;
-    if (!segk_fits(L, Hq)) return MW_ESHAPE;
-    CUtensorMap tq, tk, tv;
-    const uint64_t T = (uint64_t)L->total_tokens;
-    if (!tmap_bf16_3d(&tq, Q, T, Hq, DH, 128, 64) ||
-        !tmap_bf16_3d(&tk, Kseg, (uint64_t)L->n_keymask * 128, Hkv, DH, 128, 64) ||
-        !tmap_bf16_3d(&tv, V, T, Hkv, DH, 128, 64))
-        return MW_ECUDA;
-    FwdParams p;
-    p.v = make_view(L, vis);
-    p.total = L->total_tokens;
-    p.n_traj = L->n_traj;
-    p.max_tiles = L->max_tiles;
-    p.Hq = Hq;
-    p.Hkv = Hkv;
-    p.scale_log2 = scale * LOG2E;
-    p.O = (__nv_bfloat16*)O;
-    p.LSE = LSE;
-    p.junction_items = 0;
-    mw_status st = cuda_status(cudaFuncSetAttribute(k_attn_fwd_tc<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                    (int)SMEM_FWD));
-    if (st != MW_OK) return st;
-    count_launches(1);
-    k_attn_fwd_tc<1><<<(unsigned)((int64_t)L->max_tiles * L->n_traj * Hq), NT_FWD, SMEM_FWD, s>>>(tq, tk, tv, p);
-    if ((st = launch_status()) != MW_OK || L->n_junc == 0) return st;
-    p.junction_items = 1;
-    count_launches(1);
-    k_attn_fwd_tc<1><<<(unsigned)(L->n_segs * Hq), NT_FWD, SMEM_FWD, s>>>(tq, tk, tv, p);
-    return launch_status();
 }
 
 namespace {
@@ -1305,45 +1203,89 @@ __global__ void k_attn_lsd(VisView v, int64_t total, int64_t n_rows, int Hq, con
 
 // Compact K / V: row (traj_km[b] + s nt) 128 + c of Kc, Vc holds the key at
 // rank c of view_s (csrc) for c < |view_s|, zeros up to the end of that
-// tile. One block per (segment, tile) entry with keys in it; 16-byte vectors.
-__global__ void __launch_bounds__(256) k_cmp_gather(VisView v, int n_traj, int Hkv,
-                                                    const __nv_bfloat16* __restrict__ K,
-                                                    const __nv_bfloat16* __restrict__ V, __nv_bfloat16* __restrict__ Kc,
-                                                    __nv_bfloat16* __restrict__ Vc) {
-    const int64_t e = blockIdx.x;
+// tile. With a rotary table the K row is also turned to position c, its
+// logical position in view_s (§4.2): feature f pairs with f + 64 and turns by
+// table[c][f] = (cos, sin). One block per (segment, tile) entry with keys in
+// it; 16-byte vectors.
+__device__ __forceinline__ int cmp_entry_traj(const VisView& v, int n_traj, int64_t e, int& s, int& kt, int& nt) {
     int lo = 0, hi = n_traj;   // the trajectory holding entry e: largest b with traj_km[b] <= e
     while (hi - lo > 1) {
         const int mid = (lo + hi) >> 1;
         if (v.traj_km[mid] <= e) lo = mid; else hi = mid;
     }
-    const int b = lo;
-    const int nt = v.traj_tile[b + 1] - v.traj_tile[b];
-    const int64_t rel = e - v.traj_km[b];
-    const int s = (int)(rel / nt), kt = (int)(rel - (int64_t)s * nt);
+    nt = v.traj_tile[lo + 1] - v.traj_tile[lo];
+    const int64_t rel = e - v.traj_km[lo];
+    s = (int)(rel / nt);
+    kt = (int)(rel - (int64_t)s * nt);
+    return lo;
+}
+
+__global__ void __launch_bounds__(256) k_cmp_gather(VisView v, int n_traj, int Hkv,
+                                                    const __nv_bfloat16* __restrict__ K,
+                                                    const __nv_bfloat16* __restrict__ V, __nv_bfloat16* __restrict__ Kc,
+                                                    __nv_bfloat16* __restrict__ Vc, const float2* __restrict__ table) {
+    const int64_t e = blockIdx.x;
+    int s, kt, nt;
+    const int b = cmp_entry_traj(v, n_traj, e, s, kt, nt);
     if (kt * 128 >= v.seg_len[v.traj_seg[b] + s]) return;
     const int64_t tok0 = v.traj_tok[b];
     const int vec = Hkv * (DH / 8);   // 16-byte vectors per key row
     for (int x = threadIdx.x; x < 128 * vec; x += blockDim.x) {
         const int r = x / vec, k = x - r * vec;
         const int j = v.csrc[e * 128 + r];
-        uint4 kv = make_uint4(0u, 0u, 0u, 0u), vv = kv;
-        if (j >= 0) {
-            kv = reinterpret_cast<const uint4*>(K + (tok0 + j) * Hkv * DH)[k];
-            vv = reinterpret_cast<const uint4*>(V + (tok0 + j) * Hkv * DH)[k];
-        }
-        reinterpret_cast<uint4*>(Kc + (e * 128 + r) * Hkv * DH)[k] = kv;
+        uint4 vv = make_uint4(0u, 0u, 0u, 0u);
+        if (j >= 0) vv = reinterpret_cast<const uint4*>(V + (tok0 + j) * Hkv * DH)[k];
         reinterpret_cast<uint4*>(Vc + (e * 128 + r) * Hkv * DH)[k] = vv;
+        if (!table) {
+            uint4 kv = make_uint4(0u, 0u, 0u, 0u);
+            if (j >= 0) kv = reinterpret_cast<const uint4*>(K + (tok0 + j) * Hkv * DH)[k];
+            reinterpret_cast<uint4*>(Kc + (e * 128 + r) * Hkv * DH)[k] = kv;
+        } else if ((k & 15) < 8) {
+            // vector k of head k / 16 holds features 8 (k % 16) ..; with its
+            // partner 64 features on, it is one rotated 16-element unit
+            const int h = k >> 4, f0 = 8 * (k & 15);
+            const int64_t c = (int64_t)kt * 128 + r;   // the key's rank in view_s
+            uint4 lo = make_uint4(0u, 0u, 0u, 0u), hi = lo;
+            if (j >= 0) {
+                const __nv_bfloat16* src = K + ((tok0 + j) * Hkv + h) * DH;
+                const uint4 x0 = *reinterpret_cast<const uint4*>(src + f0);
+                const uint4 x1 = *reinterpret_cast<const uint4*>(src + 64 + f0);
+                const uint32_t a[4] = {x0.x, x0.y, x0.z, x0.w}, bq[4] = {x1.x, x1.y, x1.z, x1.w};
+                uint32_t ya[4], yb[4];
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    float y[4];
+#pragma unroll
+                    for (int u = 0; u < 2; ++u) {
+                        const float2 cs = table[c * 64 + f0 + 2 * q + u];
+                        const float p0 = u ? __uint_as_float(a[q] & 0xffff0000u) : __uint_as_float(a[q] << 16);
+                        const float p1 = u ? __uint_as_float(bq[q] & 0xffff0000u) : __uint_as_float(bq[q] << 16);
+                        y[u] = fmaf(p0, cs.x, -p1 * cs.y);
+                        y[2 + u] = fmaf(p1, cs.x, p0 * cs.y);
+                    }
+                    ya[q] = pack_bf16(y[0], y[1]);
+                    yb[q] = pack_bf16(y[2], y[3]);
+                }
+                lo = make_uint4(ya[0], ya[1], ya[2], ya[3]);
+                hi = make_uint4(yb[0], yb[1], yb[2], yb[3]);
+            }
+            __nv_bfloat16* dst = Kc + ((e * 128 + r) * Hkv + h) * DH;
+            *reinterpret_cast<uint4*>(dst + f0) = lo;
+            *reinterpret_cast<uint4*>(dst + 64 + f0) = hi;
+        }
     }
 }
 
 // dK, dV of every key from the compact float32 partials: the sum, in segment
 // order, over the segments whose views hold the key, each taken at the key's
-// rank there (cpos); dKc carries the softmax scale already. A key enters the
-// views at its own segment, so the scan starts there. One block per key tile;
-// the order of the additions is fixed, so the result is deterministic.
+// rank there (cpos); dKc carries the softmax scale already. With a rotary
+// table each dK partial is first turned back by the key's position in that
+// segment (its rank). A key enters the views at its own segment, so the scan
+// starts there. One block per key tile; the order of the additions is fixed,
+// so the result is deterministic.
 __global__ void __launch_bounds__(256) k_cmp_reduce(VisView v, int Hkv, const float* __restrict__ dKc,
                                                     const float* __restrict__ dVc, __nv_bfloat16* __restrict__ dK,
-                                                    __nv_bfloat16* __restrict__ dV) {
+                                                    __nv_bfloat16* __restrict__ dV, const float2* __restrict__ table) {
     const int64_t g = blockIdx.x;
     const int b = v.tile_traj[g];
     const int nt = v.traj_tile[b + 1] - v.traj_tile[b];
@@ -1356,25 +1298,52 @@ __global__ void __launch_bounds__(256) k_cmp_reduce(VisView v, int Hkv, const fl
         const int r = x / vec, k = x - r * vec;
         const int j = kt * 128 + r;
         if (j >= T) continue;
-        float ak[8], av[8];
+        // dV: chunk k; dK: chunk k, or (rotary) the pair of chunks k, k + 8
+        // of one head when k is in the first half of its head
+        const bool rot = table != nullptr;
+        const bool kdo = !rot || (k & 15) < 8;
+        const int kk = rot ? ((k >> 4) << 4) + (k & 15) + 8 : k;   // partner chunk (rotary)
+        float ak[8], ak2[8], av[8];
 #pragma unroll
-        for (int q = 0; q < 8; ++q) ak[q] = av[q] = 0.f;
+        for (int q = 0; q < 8; ++q) ak[q] = ak2[q] = av[q] = 0.f;
         for (int s = v.seg[tok0 + j]; s < nseg; ++s) {
             const int64_t base = (v.traj_km[b] + (int64_t)s * nt) * 128;
             const int c = v.cpos[base + j];
             if (c < 0) continue;
-            const float4* pk = reinterpret_cast<const float4*>(dKc + (base + c) * Hkv * DH) + 2 * k;
             const float4* pv = reinterpret_cast<const float4*>(dVc + (base + c) * Hkv * DH) + 2 * k;
-            const float4 k0 = pk[0], k1 = pk[1], v0 = pv[0], v1 = pv[1];
-            ak[0] += k0.x; ak[1] += k0.y; ak[2] += k0.z; ak[3] += k0.w;
-            ak[4] += k1.x; ak[5] += k1.y; ak[6] += k1.z; ak[7] += k1.w;
+            const float4 v0 = pv[0], v1 = pv[1];
             av[0] += v0.x; av[1] += v0.y; av[2] += v0.z; av[3] += v0.w;
             av[4] += v1.x; av[5] += v1.y; av[6] += v1.z; av[7] += v1.w;
+            if (!kdo) continue;
+            const float4* pk = reinterpret_cast<const float4*>(dKc + (base + c) * Hkv * DH);
+            const float4 k0 = pk[2 * k], k1 = pk[2 * k + 1];
+            const float x0[8] = {k0.x, k0.y, k0.z, k0.w, k1.x, k1.y, k1.z, k1.w};
+            if (!rot) {
+#pragma unroll
+                for (int q = 0; q < 8; ++q) ak[q] += x0[q];
+            } else {
+                const float4 m0 = pk[2 * kk], m1 = pk[2 * kk + 1];
+                const float x1[8] = {m0.x, m0.y, m0.z, m0.w, m1.x, m1.y, m1.z, m1.w};
+                const int f0 = 8 * (k & 15);
+#pragma unroll
+                for (int q = 0; q < 8; ++q) {   // turn back: the transpose of the rotation
+                    const float2 cs = table[(int64_t)c * 64 + f0 + q];
+                    ak[q] += fmaf(x0[q], cs.x, x1[q] * cs.y);
+                    ak2[q] += fmaf(x1[q], cs.x, -x0[q] * cs.y);
+                }
+            }
         }
-        reinterpret_cast<uint4*>(dK + (tok0 + j) * Hkv * DH)[k] =
-            make_uint4(pack_bf16(ak[0], ak[1]), pack_bf16(ak[2], ak[3]), pack_bf16(ak[4], ak[5]), pack_bf16(ak[6], ak[7]));
         reinterpret_cast<uint4*>(dV + (tok0 + j) * Hkv * DH)[k] =
             make_uint4(pack_bf16(av[0], av[1]), pack_bf16(av[2], av[3]), pack_bf16(av[4], av[5]), pack_bf16(av[6], av[7]));
+        if (kdo) {
+            reinterpret_cast<uint4*>(dK + (tok0 + j) * Hkv * DH)[k] =
+                make_uint4(pack_bf16(ak[0], ak[1]), pack_bf16(ak[2], ak[3]), pack_bf16(ak[4], ak[5]),
+                           pack_bf16(ak[6], ak[7]));
+            if (rot)
+                reinterpret_cast<uint4*>(dK + (tok0 + j) * Hkv * DH)[kk] =
+                    make_uint4(pack_bf16(ak2[0], ak2[1]), pack_bf16(ak2[2], ak2[3]), pack_bf16(ak2[4], ak2[5]),
+                               pack_bf16(ak2[6], ak2[7]));
+        }
     }
 }
 
@@ -1395,73 +1364,11 @@ int64_t attn_bwd_tc_ws(const mw_vis_layout* L, int Hq, int Hkv) {
 }
 
 static mw_status cmp_gather(const mw_vis_layout* L, const VisView& v, int Hkv, const void* K, const void* V, void* Kc,
-                            void* Vc, cudaStream_t s) {
+                            void* Vc, const float* table, cudaStream_t s) {
     count_launches(1);
     k_cmp_gather<<<(unsigned)L->n_keymask, 256, 0, s>>>(v, L->n_traj, Hkv, (const __nv_bfloat16*)K,
                                                         (const __nv_bfloat16*)V, (__nv_bfloat16*)Kc,
-                                                        (__nv_bfloat16*)Vc);
-    return launch_status();
-}
-
-// Backward with segment key rows: (-LSE2, Delta) pairs into `ws`, dQ of the
-// rotated queries (bf16, main + junction launches), and per segment key row
-// the float32 partials dKseg (scaled) and dVseg.
-mw_status attn_bwd_tc_segk(const mw_vis_layout* L, const void* vis, const void* Q, const void* Kseg, const void* V,
-                           const void* O, const void* dO, const float* LSE, void* dQ, float* dKseg, float* dVseg,
-                           int Hq, int Hkv, float scale, float* ws, cudaStream_t s) {
-    if (L->n_tiles == 0) return MW_OK;
-    if (!segk_fits(L, Hq)) return MW_ESHAPE;
-    const int64_t n_rows = L->n_tiles * 128;
-    float2* lsd = reinterpret_cast<float2*>(ws);
-    const VisView view = make_view(L, vis);
-    count_launches(1);
-    k_attn_lsd<<<(unsigned)std::min<int64_t>(ceil_div(n_rows * Hq, 8), 152 * 64), 256, 0, s>>>(
-        view, L->total_tokens, n_rows, Hq, (const __nv_bfloat16*)O, (const __nv_bfloat16*)dO, LSE, lsd);
-    mw_status st = launch_status();
-    if (st != MW_OK) return st;
-    const uint64_t T = (uint64_t)L->total_tokens;
-    const uint64_t KR = (uint64_t)L->n_keymask * 128;
-    CUtensorMap tq, tdo, tk, tv, tq64, tdo64;
-    if (!tmap_bf16_3d(&tq, Q, T, Hq, DH, 128, 64) || !tmap_bf16_3d(&tdo, dO, T, Hq, DH, 128, 64) ||
-        !tmap_bf16_3d(&tk, Kseg, KR, Hkv, DH, 128, 64) || !tmap_bf16_3d(&tv, V, T, Hkv, DH, 128, 64) ||
-        !tmap_bf16_3d(&tq64, Q, T, Hq, DH, 64, 64) || !tmap_bf16_3d(&tdo64, dO, T, Hq, DH, 64, 64))
-        return MW_ECUDA;
-    BwdParams p;
-    p.v = view;
-    p.total = L->total_tokens;
-    p.n_traj = L->n_traj;
-    p.max_tiles = L->max_tiles;
-    p.Hq = Hq;
-    p.Hkv = Hkv;
-    p.scale = scale;
-    p.scale_log2 = scale * LOG2E;
-    p.lsd = lsd;
-    p.n_rows = n_rows;
-    p.dQ = (__nv_bfloat16*)dQ;
-    p.dKseg = dKseg;
-    p.dVseg = dVseg;
-    p.junction_items = 0;
-    if ((st = cuda_status(cudaFuncSetAttribute(k_attn_dq_tc<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                               (int)SMEM_DQ))) != MW_OK)
-        return st;
-    if ((st = cuda_status(cudaFuncSetAttribute(k_attn_dkdv_tc<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                               (int)SMEM_KV))) != MW_OK)
-        return st;
-    count_launches(1);
-    k_attn_dq_tc<1><<<(unsigned)((int64_t)L->max_tiles * L->n_traj * Hq), NT_BWD, SMEM_DQ, s>>>(tq, tdo, tk, tv,
-                                                                                                  p);
-    if ((st = launch_status()) != MW_OK) return st;
-    if (L->n_junc > 0) {
-        p.junction_items = 1;
-        count_launches(1);
-        k_attn_dq_tc<1><<<(unsigned)(L->n_segs * Hq), NT_BWD, SMEM_DQ, s>>>(tq, tdo, tk, tv, p);
-        if ((st = launch_status()) != MW_OK) return st;
-        p.junction_items = 0;
-    }
-    // grid.y: the most segments of any trajectory
-    const dim3 gk((unsigned)((int64_t)L->max_tiles * L->n_traj * Hkv), (unsigned)L->max_segs);
-    count_launches(1);
-    k_attn_dkdv_tc<1><<<gk, NT_BWD, SMEM_KV, s>>>(tq64, tdo64, tk, tv, p);
+                                                        (__nv_bfloat16*)Vc, reinterpret_cast<const float2*>(table));
     return launch_status();
 }
 
@@ -1469,14 +1376,14 @@ mw_status attn_bwd_tc_segk(const mw_vis_layout* L, const void* vis, const void* 
 // one CTA per (q-tile, segment of its first row, head) plus one per (segment
 // starting inside a q-tile, head), each over its segment's compact keys.
 mw_status attn_fwd_tc(const mw_vis_layout* L, const void* vis, const void* Q, const void* K, const void* V, void* O,
-                      float* LSE, int Hq, int Hkv, float scale, void* ws, cudaStream_t s) {
+                      float* LSE, int Hq, int Hkv, float scale, void* ws, cudaStream_t s, const float* table) {
     if (L->n_tiles == 0) return MW_OK;
     if (!segk_fits(L, Hq)) return MW_ESHAPE;
     const VisView view = make_view(L, vis);
     const int64_t KR = cmp_rows(L);
     void* Kc = ws;
     void* Vc = at<char>(ws, 2 * KR * Hkv * DH);
-    mw_status st = cmp_gather(L, view, Hkv, K, V, Kc, Vc, s);
+    mw_status st = cmp_gather(L, view, Hkv, K, V, Kc, Vc, table, s);
     if (st != MW_OK) return st;
     CUtensorMap tq, tk, tv;
     const uint64_t T = (uint64_t)L->total_tokens;
@@ -1494,15 +1401,15 @@ mw_status attn_fwd_tc(const mw_vis_layout* L, const void* vis, const void* Q, co
     p.O = (__nv_bfloat16*)O;
     p.LSE = LSE;
     p.junction_items = 0;
-    if ((st = cuda_status(cudaFuncSetAttribute(k_attn_fwd_tc<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    if ((st = cuda_status(cudaFuncSetAttribute(k_attn_fwd_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                (int)SMEM_FWD))) != MW_OK)
         return st;
     count_launches(1);
-    k_attn_fwd_tc<2><<<(unsigned)((int64_t)L->max_tiles * L->n_traj * Hq), NT_FWD, SMEM_FWD, s>>>(tq, tk, tv, p);
+    k_attn_fwd_tc<<<(unsigned)((int64_t)L->max_tiles * L->n_traj * Hq), NT_FWD, SMEM_FWD, s>>>(tq, tk, tv, p);
     if ((st = launch_status()) != MW_OK || L->n_junc == 0) return st;
     p.junction_items = 1;
     count_launches(1);
-    k_attn_fwd_tc<2><<<(unsigned)(L->n_segs * Hq), NT_FWD, SMEM_FWD, s>>>(tq, tk, tv, p);
+    k_attn_fwd_tc<<<(unsigned)(L->n_segs * Hq), NT_FWD, SMEM_FWD, s>>>(tq, tk, tv, p);
     return launch_status();
 }
 
@@ -1511,7 +1418,7 @@ mw_status attn_fwd_tc(const mw_vis_layout* L, const void* vis, const void* Q, co
 // partials per compact row, and their deterministic sum per key.
 mw_status attn_bwd_tc(const mw_vis_layout* L, const void* vis, const void* Q, const void* K, const void* V,
                       const void* O, const void* dO, const float* LSE, void* dQ, void* dK, void* dV, int Hq, int Hkv,
-                      float scale, void* ws, cudaStream_t s) {
+                      float scale, void* ws, cudaStream_t s, const float* table) {
     if (L->n_tiles == 0) return MW_OK;
     if (!segk_fits(L, Hq)) return MW_ESHAPE;
     const int64_t n_rows = L->n_tiles * 128;
@@ -1526,7 +1433,7 @@ mw_status attn_bwd_tc(const mw_vis_layout* L, const void* vis, const void* Q, co
     k_attn_lsd<<<(unsigned)std::min<int64_t>(ceil_div(n_rows * Hq, 8), 152 * 64), 256, 0, s>>>(
         view, L->total_tokens, n_rows, Hq, (const __nv_bfloat16*)O, (const __nv_bfloat16*)dO, LSE, lsd);
     mw_status st = launch_status();
-    if (st == MW_OK) st = cmp_gather(L, view, Hkv, K, V, Kc, Vc, s);
+    if (st == MW_OK) st = cmp_gather(L, view, Hkv, K, V, Kc, Vc, table, s);
     if (st != MW_OK) return st;
     const uint64_t T = (uint64_t)L->total_tokens;
     CUtensorMap tq, tdo, tk, tv, tq64, tdo64;
@@ -1549,26 +1456,27 @@ mw_status attn_bwd_tc(const mw_vis_layout* L, const void* vis, const void* Q, co
     p.dKseg = dKc;
     p.dVseg = dVc;
     p.junction_items = 0;
-    if ((st = cuda_status(cudaFuncSetAttribute(k_attn_dq_tc<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    if ((st = cuda_status(cudaFuncSetAttribute(k_attn_dq_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                (int)SMEM_DQ))) != MW_OK)
         return st;
-    if ((st = cuda_status(cudaFuncSetAttribute(k_attn_dkdv_tc<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    if ((st = cuda_status(cudaFuncSetAttribute(k_attn_dkdv_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                (int)SMEM_KV))) != MW_OK)
         return st;
     count_launches(1);
-    k_attn_dq_tc<2><<<(unsigned)((int64_t)L->max_tiles * L->n_traj * Hq), NT_BWD, SMEM_DQ, s>>>(tq, tdo, tk, tv, p);
+    k_attn_dq_tc<<<(unsigned)((int64_t)L->max_tiles * L->n_traj * Hq), NT_BWD, SMEM_DQ, s>>>(tq, tdo, tk, tv, p);
     if ((st = launch_status()) != MW_OK) return st;
     if (L->n_junc > 0) {
         p.junction_items = 1;
         count_launches(1);
-        k_attn_dq_tc<2><<<(unsigned)(L->n_segs * Hq), NT_BWD, SMEM_DQ, s>>>(tq, tdo, tk, tv, p);
+        k_attn_dq_tc<<<(unsigned)(L->n_segs * Hq), NT_BWD, SMEM_DQ, s>>>(tq, tdo, tk, tv, p);
         if ((st = launch_status()) != MW_OK) return st;
         p.junction_items = 0;
     }
     const dim3 gk((unsigned)((int64_t)L->max_tiles * L->n_traj * Hkv), (unsigned)L->max_segs);
     count_launches(2);
-    k_attn_dkdv_tc<2><<<gk, NT_BWD, SMEM_KV, s>>>(tq64, tdo64, tk, tv, p);
-    k_cmp_reduce<<<(unsigned)L->n_tiles, 256, 0, s>>>(view, Hkv, dKc, dVc, (__nv_bfloat16*)dK, (__nv_bfloat16*)dV);
+    k_attn_dkdv_tc<<<gk, NT_BWD, SMEM_KV, s>>>(tq64, tdo64, tk, tv, p);
+    k_cmp_reduce<<<(unsigned)L->n_tiles, 256, 0, s>>>(view, Hkv, dKc, dVc, (__nv_bfloat16*)dK, (__nv_bfloat16*)dV,
+                                                      reinterpret_cast<const float2*>(table));
     return launch_status();
 }
 

@@ -146,7 +146,7 @@ def test_rope_entry_points_reject_bad_args_on_host():
                                      P, None) == 3
 
 
-def test_rope_workspace_holds_rotated_queries_and_segment_keys():
+def test_rope_workspace_holds_rotated_queries_and_keys():
     L, h = _lib()
     cu = np.array([0, 300, 1000], np.int32)
     lay = L.mw_visibility_layout(cu, np.array([0, 1, 1], np.int32), 4)
@@ -154,14 +154,16 @@ def test_rope_workspace_holds_rotated_queries_and_segment_keys():
     krows = lay.n_keymask * 128
     for dtype, esz in ((0, 4), (1, 2)):
         f, b = L.mw_masked_attn_rope_ws(L.Visibility(lay, None, None), Hq, Hkv, Dh, dtype)
-        need = esz * (lay.total_tokens * Hq * Dh + krows * Hkv * Dh)
+        # rotated queries, then (CUDA cores) the segment key rows or (tensor
+        # cores) the compact K and V, both krows rows
+        need = esz * lay.total_tokens * Hq * Dh + (esz if dtype == 0 else 2 * esz) * krows * Hkv * Dh
         assert need <= f < need + 1024
         if dtype == 0:
             # CUDA-core backward: Delta per (head, row) and the float32 segment-key gradient
             need_b = f + 4 * lay.total_tokens * Hq + 4 * krows * Hkv * Dh
         else:
             # tensor-core backward: the (-LSE log2 e, Delta) pair array over whole
-            # tiles, and float32 per-segment dK and dV partials
+            # tiles, and float32 dK and dV partials per compact row
             need_b = f + 8 * lay.n_tiles * 128 * Hq + 2 * 4 * krows * Hkv * Dh
         assert need_b <= b < need_b + 1536
 

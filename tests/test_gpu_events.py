@@ -122,3 +122,35 @@ def test_event_records_rejected_where_lifetimes_are_needed():
     with pytest.raises(mw.MWError) as e:               # retrieving a position that is in the view
         mw.build_views_events([50], [[(10, [], [(2, 4)])]])
     assert e.value.status == 2
+
+
+def test_rotary_attention_on_event_views():
+    """Rotary positions on event views are list indices (reading 3): a
+    re-entered span takes positions after the tokens decoded meanwhile. The
+    bf16 rotary attention (keys turned by their rank as they are gathered)
+    forward and backward against the oracle's compact computation with
+    rotary positions on the same views."""
+    import paper_2609_00865_gb300 as mw
+    rng = np.random.default_rng(4300)
+    seqlens = [900, 600]
+    events = [_memex_record(rng, T, 4) for T in seqlens]
+    assert any(ev[2] for e in events for ev in e)
+    vis = _compare(seqlens, events)
+    T = sum(seqlens)
+    Q, K, Vx, dO = (synth.normal((T, h, 128), 4400 + n).to(torch.bfloat16) for n, h in enumerate((8, 2, 2, 8)))
+    q, k, v, do = (t.cuda() for t in (Q, K, Vx, dO))
+    theta, scale = 1e4, 128 ** -0.5
+    pos = mw.logical_positions(vis)              # the build's ranks: list indices
+    table = mw.rope_table(mw.rope_n_pos(vis), 128, theta)
+    O, LSE = mw.masked_attn_rope_fwd(vis, pos, table, q, k, v, scale)
+    dQ, dK, dV = mw.masked_attn_rope_bwd(vis, pos, table, q, k, v, O, do, LSE, scale)
+    torch.cuda.synchronize()
+    vis.check_status()
+    Or, Lr = OA.attn_fwd(seqlens, events, np64(Q), np64(K), np64(Vx), scale, rope_theta=theta, views=N.live_views)
+    assert_maxabs(np64(O), Or, 2e-2, "O")
+    assert_maxabs(np64(LSE), Lr, 2e-2, "LSE")
+    dQr, dKr, dVr = OA.attn_bwd(seqlens, events, np64(Q), np64(K), np64(Vx), np64(dO), scale, rope_theta=theta,
+                                views=N.live_views)
+    assert_grad_bf16(np64(dQ), dQr, "dQ")
+    assert_grad_bf16(np64(dK), dKr, "dK")
+    assert_grad_bf16(np64(dV), dVr, "dV")
