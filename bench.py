@@ -178,6 +178,8 @@ def make_workload(cfg, K=None, f=None, seed_offset=0, n_traj=None, pin=True, rop
         t = t.to(bf)
         return t.pin_memory() if pin else t
 
+    if cfg == 5:
+        w["sweep"] = (K, f)
     if cfg in (2, 4, 5):
         rec = synth.config_record(cfg, K=K, f=f)
         if n_traj:
@@ -231,6 +233,8 @@ def describe(w):
                  head_dim=w["heads"][2])
     if "rows" in w:
         d.update(loss_rows=int(w["rows"].numel()), hidden=w["d"], vocab=w["Vocab"])
+    if "sweep" in w:
+        d.update(sweep_K=w["sweep"][0], evicted_fraction=w["sweep"][1])
     if "rope" in w:
         d["rope_theta"] = w["rope"]
     d["l2"] = "inputs larger than L2 (129 MB); no flush"
@@ -774,6 +778,92 @@ def run_gpu(args, rank, world, local_rank):
     print(json.dumps(line), flush=True)
 
 
+BUILDER_BATCH = 64
+
+
+def run_builder(args, rank, world, local_rank):
+    """The visibility builder alone, batched: 64 sweep-shaped trajectories of
+    131,072 tokens (K junctions at eviction fraction f) per build. One
+    trajectory is a few MB of structure and launch-bound, so the builder's
+    bandwidth is measured on the batch. HBM roofline over the builder's
+    algorithmic bytes: the packed record read once (12 B per evicted span,
+    the per-trajectory and per-junction tables) and the structure written
+    once (all of it but the compact source lists past each segment's last
+    compact tile, which stay unspecified). The record is host data by the builder's API (the
+    call packs it and uploads the span list), so the timed call includes that
+    upload: ``value`` and ``e2e`` are the same measurement."""
+    import torch
+
+    import paper_2609_00865_gb300 as mw
+    import synth
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    c = synth.CONFIGS[5]
+    seed = 1000 * 5 + 100 * args.K + int(round(10 * args.f)) + 10000 * (rank + 1)
+    rec = synth.record(BUILDER_BATCH, c["T"], args.K, args.f, c["summary"], c["prompt"], c["Lp"], c["Lo"], seed)
+    cu, J, jt, off, spans = mw.flatten_record(rec.seqlens, rec.edits)
+    L = mw.mw_visibility_layout(cu, jt, len(spans))
+    vis = mw.Visibility(L, torch.empty(L.vis_bytes, dtype=torch.uint8, device=dev),
+                        torch.empty(max(L.ws_bytes, 1), dtype=torch.uint8, device=dev))
+    stream = torch.cuda.current_stream(dev)
+
+    def build():
+        mw.mw_build_visibility(L, cu, J, jt, off, spans, vis.ws, vis.vis, stream)
+
+    for _ in range(args.warmup):
+        build()
+    torch.cuda.synchronize()
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+    clocks = Clocks(local_rank)
+    torch.cuda.synchronize()
+    clocks.start()
+    n0 = mw.kernel_launches()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        build()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    launches = mw.kernel_launches() - n0
+    clk = clocks.stop()
+    ms = reduce_max(e0.elapsed_time(e1) / args.steps, world, dev)
+    if rank != 0:
+        return
+    import numpy as np
+    n_spans = int(L.n_spans)
+    # written: the whole structure except csrc past each segment's last compact
+    # tile (left unspecified); read: the packed span list and the small tables
+    seg_len = vis.seg_len.astype(np.int64)
+    csrc_used = 4 * mw.TILE * int(((seg_len + mw.TILE - 1) // mw.TILE).sum())
+    nbytes = (int(L.vis_bytes) - 4 * mw.TILE * int(L.n_keymask) + csrc_used
+              + 12 * n_spans + 4 * (len(rec.seqlens) + 1) + 8 * int(L.n_junc))
+    peak_tf, peak_sus, hbm, peak_kind = _peaks()
+    gbs = nbytes / (ms * 1e-3) / 1e9
+    tokens = rec.total
+    value = job_value(tokens, world, ms)
+    line = {
+        "metric": "visibility-build tokens/sec", "value": value, "unit": "tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "int32", "data": "synthetic",
+        "config": {"workload": f"visibility builder batched: {BUILDER_BATCH}x{c['T']} tokens, "
+                               f"{args.K} junctions at {args.f}",
+                   "trajectories": len(rec.seqlens), "tokens": tokens, "junctions": int(L.n_junc),
+                   "evicted_spans": n_spans, "listed_tiles": int(L.n_tiles), "structure_bytes": int(L.vis_bytes),
+                   "l2": "structure larger than L2 (129 MB); no flush"},
+        "roofline": {"bound": "hbm", "kernel": "mw_build_visibility (all kernels + host packing)",
+                     "achieved": gbs, "peak": hbm, "unit": "GB/s", "frac": gbs / hbm, "traffic": None,
+                     "algorithmic_bytes": nbytes, "peak_kind": f"copy bandwidth, {peak_kind}"},
+        "e2e": {"value": value, "unit": "tokens/s", "ms_per_step": ms,
+                "note": "host record in, device structure out: the timed call packs and uploads the record"},
+        "gpu_launches": launches,
+        "clocks": clk,
+    }
+    print(json.dumps(line), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -791,6 +881,8 @@ def main():
                     help="config 4: time SDCC's training step (§5) instead of the 4D-mask step")
     ap.add_argument("--rope", type=float, default=None, metavar="THETA",
                     help="attention with row-wise logical rotary positions (theta of the rotary table)")
+    ap.add_argument("--builder", action="store_true",
+                    help="time the visibility builder alone on 64 sweep trajectories (131,072 tokens, --K, --f)")
     args = ap.parse_args()
     if args.sdcc and (args.config != 4 or args.rope is not None):
         ap.error("--sdcc times the 7B-shaped layer step (config 4) without rotary positions")
@@ -802,6 +894,8 @@ def main():
         dist.init_process_group("nccl" if args.impl == "mw" else "gloo")
     if args.impl == "reference":
         run_reference(args, rank, world)
+    elif args.builder:
+        run_builder(args, rank, world, local_rank)
     else:
         run_gpu(args, rank, world, local_rank)
     if world > 1:

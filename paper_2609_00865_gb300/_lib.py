@@ -305,6 +305,12 @@ class Visibility:
         }
 
     @property
+    def seg_len(self):
+        """Length of every segment's live view, in global segment order (host copy)."""
+        L = self.layout
+        return self._arr(L.off_seg_len, L.n_segs, np.int32)
+
+    @property
     def pairs_total(self):
         L = self.layout
         return int(self._arr(L.off_pairs + 8 * L.n_traj, 1, np.int64)[0])

@@ -94,10 +94,13 @@ struct FwdParams {
 };
 
 // Work item of a q-tile kernel: trajectory b, local q-tile qt, query head h
-// and the segment s whose rows the CTA stores. Main launch: heaviest (largest
-// qt) first, query heads of one KV group adjacent; s = segment of the tile's
-// first row. Junction items: blockIdx.x / Hq is a global segment index; a
-// segment that starts inside a tile (not at its first row) gets a CTA there.
+// and the segment s whose rows the CTA stores. Main launch: one trajectory
+// after another, its heaviest (largest) q-tiles first, query heads of one KV
+// group adjacent; s = segment of the tile's first row. Taking trajectories in
+// turn keeps the resident CTAs on one trajectory's compact K / V, whose
+// working set then stays in L2. Junction items: blockIdx.x / Hq is a global
+// segment index; a segment that starts inside a tile (not at its first row)
+// gets a CTA there.
 struct QItem {
     int b, qt, h, s;
     bool ok;
@@ -108,8 +111,8 @@ __device__ __forceinline__ QItem q_item(const VisView& v, int Hq, int max_tiles,
     const int r = blockIdx.x / Hq;
     it.s = 0;
     if (!junction_items) {
-        it.qt = max_tiles - 1 - r / n_traj;
-        it.b = r % n_traj;
+        it.b = r / max_tiles;
+        it.qt = max_tiles - 1 - (r - it.b * max_tiles);
         it.ok = it.qt < v.traj_tile[it.b + 1] - v.traj_tile[it.b];
         if (it.ok) it.s = v.seg[v.traj_tok[it.b] + it.qt * 128];
     } else {
@@ -196,6 +199,10 @@ __device__ __forceinline__ void soft_pair(float s0, float s1, float dp0, float d
     ds_pk = pack_bf16(f2_lo(d), f2_hi(d));
 }
 
+// float index of n for padded row r of the (n, Delta) row-pair array; Delta
+// sits 2 floats further
+__device__ __forceinline__ int64_t lsd_index(int64_t r) { return ((r >> 1) << 2) + (r & 1); }
+
 __device__ __forceinline__ void load_tile(uint8_t* dst, const CUtensorMap* map, uint64_t* bar, int head, int row) {
     tma_load_3d(dst, map, bar, 0, head, row);
     tma_load_3d(dst + HALF_B, map, bar, 64, head, row);
@@ -227,7 +234,6 @@ __global__ void __launch_bounds__(NT_FWD, 1)
     if (!it.ok) return;
     const int h = it.h, qt = it.qt, b = it.b;
     const int nt = v.traj_tile[b + 1] - v.traj_tile[b];
-    const int64_t g = v.traj_tile[b] + qt;
     const int64_t tok0 = v.traj_tok[b];
     const int T = v.traj_tok[b + 1] - (int)tok0;
     const int kvh = h / (p.Hq / p.Hkv);
@@ -448,7 +454,7 @@ __global__ void __launch_bounds__(NT_FWD, 1)
                 e_cur = e_nxt;
                 e_nxt = j + 2 < n ? entry(j + 2) : 0;
             }
-            const int kt = e >> 4, cls = e & 3;
+            const int cls = e & 3;
             if (!mbar_wait(&s_full[j & 1], (j >> 1) & 1, status, 301)) { ok = false; break; }
             tc_fence_after();
             // a tile whose first or second key half no row sees was computed as
@@ -546,7 +552,8 @@ struct BwdParams {
     int64_t total;
     int n_traj, max_tiles, Hq, Hkv;
     float scale, scale_log2;
-    const float2* lsd;     // [Hq][n_tiles * 128] (-LSE_i log2 e, Delta_i), rows padded to whole tiles
+    const float* lsd;      // [Hq][n_tiles * 64] float4 (n_i, n_i+1, Delta_i, Delta_i+1), n = -LSE log2 e;
+                           // rows padded to whole tiles
     int64_t n_rows;        // n_tiles * 128
     __nv_bfloat16* dQ;
     int junction_items;    // dQ: as FwdParams
@@ -724,8 +731,8 @@ __global__ void __launch_bounds__(NT_BWD, 1)
         const int crow = in_piece ? cp.cfirst + i - cp.r0 : -(1 << 30);
         auto mask_words = [&](int e) -> uint4 { return prefix_words(crow - (e >> 4) * 128); };
         const uint32_t lane_base = tmem + ((uint32_t)(qw * 32) << 16);
-        const float2 ld = p.lsd[(int64_t)h * p.n_rows + g * 128 + rl];
-        const uint64_t c2 = f2(p.scale_log2, p.scale_log2), n2 = f2(ld.x, ld.x), dl2 = f2(ld.y, ld.y);
+        const float* ld = p.lsd + lsd_index((int64_t)h * p.n_rows + g * 128 + rl);
+        const uint64_t c2 = f2(p.scale_log2, p.scale_log2), n2 = f2(ld[0], ld[0]), dl2 = f2(ld[2], ld[2]);
         bool ok = true;
         // list entries and view-mask words are loaded ahead (an entry two
         // tiles, a mask word one tile), so no step waits on a global load once
@@ -801,7 +808,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
                 e_cur = e_nxt;
                 e_nxt = j + 2 < n ? entry(j + 2) : 0;
             }
-            const int kt = e >> 4, cls = e & 3;
+            const int cls = e & 3;
             if (!mbar_wait(&s_full[j & 1], (j >> 1) & 1, status, 311)) { ok = false; break; }
             tc_fence_after();
             const uint32_t sbuf = lane_base + TM_S0 + (j & 1) * 128;
@@ -1061,13 +1068,15 @@ __global__ void __launch_bounds__(NT_BWD, 1)
         const uint32_t lane_base = tmem + ((uint32_t)(qw * 32) << 16);
         bool ok = true;
         // (-LSE2, Delta) of this warp's 32 query rows of a step: 256 contiguous
-        // bytes of the tile-padded pair array, read by every lane (broadcast)
-        // at the start of the step, after a prefetch into L1 one step earlier.
-        const float2* lsd_k = p.lsd + (int64_t)v.traj_tile[b] * 128 + 32 * ch;
+        // bytes of the tile-padded row-pair array, read by every lane
+        // (broadcast) at the start of the step, after a prefetch into L1 one
+        // step earlier. A float4 holds two rows' (n, n', Delta, Delta'), so its
+        // halves are the register pairs the paired arithmetic takes.
+        const int64_t lsd_k = (int64_t)v.traj_tile[b] * 128 + 32 * ch;
         auto lsd_row = [&](const Cursor& c) -> const float4* {
             int hq;
             const int q0 = cur_q0(c, hq);
-            return reinterpret_cast<const float4*>(lsd_k + (int64_t)hq * p.n_rows + q0);
+            return reinterpret_cast<const float4*>(p.lsd + lsd_index(lsd_k + (int64_t)hq * p.n_rows + q0));
         };
         Cursor cur = first, nxt = first;   // steps t and t + 1
         advance(nxt);
@@ -1108,13 +1117,13 @@ __global__ void __launch_bounds__(NT_BWD, 1)
                 if (__all_sync(0xffffffffu, vm == 0xffffffffu)) {
 #pragma unroll
                     for (int x = 0; x < 16; ++x)
-                        soft_pair<false>(sv[2 * x], sv[2 * x + 1], dp[2 * x], dp[2 * x + 1], c2, f2(lv[x].x, lv[x].z),
-                                         f2(lv[x].y, lv[x].w), vm, 2 * x, pa[x], pd[x]);
+                        soft_pair<false>(sv[2 * x], sv[2 * x + 1], dp[2 * x], dp[2 * x + 1], c2, f2(lv[x].x, lv[x].y),
+                                         f2(lv[x].z, lv[x].w), vm, 2 * x, pa[x], pd[x]);
                 } else {
 #pragma unroll
                     for (int x = 0; x < 16; ++x)
-                        soft_pair<true>(sv[2 * x], sv[2 * x + 1], dp[2 * x], dp[2 * x + 1], c2, f2(lv[x].x, lv[x].z),
-                                        f2(lv[x].y, lv[x].w), vm, 2 * x, pa[x], pd[x]);
+                        soft_pair<true>(sv[2 * x], sv[2 * x + 1], dp[2 * x], dp[2 * x + 1], c2, f2(lv[x].x, lv[x].y),
+                                        f2(lv[x].z, lv[x].w), vm, 2 * x, pa[x], pd[x]);
                 }
                 tmem_st16(lane_base + TM_ST + s * 64 + 32 * ch, pa);
                 tmem_st16(lane_base + TM_DPT + s * 64 + 32 * ch, pd);
@@ -1170,13 +1179,14 @@ static bool segk_fits(const mw_vis_layout* L, int Hq) {
 
 namespace {
 
-// (-LSE_i log2 e, Delta_i = rowsum(dO_i * O_i)) per (head, row) in the
-// tile-padded layout [Hq][n_tiles * 128]: row r of global tile g sits at
-// g * 128 + r, so any 32 rows of a tile are 256 contiguous, 16-byte aligned
+// (n_i = -LSE_i log2 e, Delta_i = rowsum(dO_i * O_i)) per (head, row) in the
+// tile-padded layout [Hq][n_tiles * 128 rows]: padded row r = h n_rows + g 128
+// + (row in tile g) sits in float4 r / 2 as (n_r, n_r+1, Delta_r, Delta_r+1)
+// (r even), so any 32 rows of a tile are 256 contiguous, 16-byte aligned
 // bytes. Rows past a trajectory's end hold zeros. One warp per (row, head).
 __global__ void k_attn_lsd(VisView v, int64_t total, int64_t n_rows, int Hq, const __nv_bfloat16* __restrict__ O,
                            const __nv_bfloat16* __restrict__ dO, const float* __restrict__ LSE,
-                           float2* __restrict__ lsd) {
+                           float* __restrict__ lsd) {
     const int lane = threadIdx.x & 31;
     const int64_t nw = (int64_t)gridDim.x * (blockDim.x >> 5);
     for (int64_t w = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5; w < n_rows * Hq; w += nw) {
@@ -1197,7 +1207,11 @@ __global__ void k_attn_lsd(VisView v, int64_t total, int64_t n_rows, int Hq, con
             const float acc = warp_sum(fmaf(o0.x, d0.x, fmaf(o0.y, d0.y, fmaf(o1.x, d1.x, o1.y * d1.y))));
             out = make_float2(-LSE[(int64_t)h * total + tok0 + i] * LOG2E, acc);
         }
-        if (lane == 0) lsd[(int64_t)h * n_rows + gr] = out;
+        if (lane == 0) {
+            const int64_t at = lsd_index((int64_t)h * n_rows + gr);
+            lsd[at] = out.x;
+            lsd[at + 2] = out.y;
+        }
     }
 }
 
@@ -1423,7 +1437,7 @@ mw_status attn_bwd_tc(const mw_vis_layout* L, const void* vis, const void* Q, co
     if (!segk_fits(L, Hq)) return MW_ESHAPE;
     const int64_t n_rows = L->n_tiles * 128;
     const int64_t KR = cmp_rows(L);
-    float2* lsd = reinterpret_cast<float2*>(ws);
+    float* lsd = reinterpret_cast<float*>(ws);
     void* Kc = at<char>(ws, align256(8 * n_rows * (int64_t)Hq));
     void* Vc = at<char>(Kc, 2 * KR * Hkv * DH);
     float* dKc = at<float>(Kc, attn_fwd_tc_ws(L, Hkv));

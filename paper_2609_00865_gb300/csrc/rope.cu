@@ -149,6 +149,53 @@ __global__ void __launch_bounds__(256) k_rope_rows(VisView v, const int32_t* __r
     }
 }
 
+// The same with 16-byte vectors: a thread turns VEC consecutive features of
+// both halves of one (row, head), with the VEC table entries as float4 loads.
+// Needs half a row (Dh / 2 elements) to be whole vectors and X, Y 16-byte
+// aligned (checked by the launcher).
+template <typename T>
+__global__ void __launch_bounds__(256) k_rope_rows_vec(VisView v, const int32_t* __restrict__ pos,
+                                                       const float2* __restrict__ table, int n_pos, const T* X, T* Y,
+                                                       int H, int Dh, float sgn) {
+    constexpr int VEC = 16 / sizeof(T);
+    const TrajRef r = traj_of_tile(v, blockIdx.x);
+    const int half = Dh >> 1;
+    const int hv = half / VEC;   // vectors per half row
+    const int rows = min(MW_TILE, r.T - r.kt * MW_TILE);
+    const int per_row = H * hv;
+    for (int e = threadIdx.x; e < rows * per_row; e += blockDim.x) {
+        const int jj = e / per_row, rem = e - jj * per_row;
+        const int h = rem / hv, f = (rem - h * hv) * VEC;
+        const int i = r.kt * MW_TILE + jj;
+        const int64_t gi = r.tok0 + i;
+        const int s = v.seg[gi];
+        const int p = pos[(r.kmb + (int64_t)s * r.nt) * MW_TILE + i];
+        const int64_t o = (gi * H + h) * Dh + f;
+        uint4 y0v = make_uint4(0u, 0u, 0u, 0u), y1v = y0v;
+        if (pos_ok(v, p, n_pos)) {
+            const uint4 x0v = *reinterpret_cast<const uint4*>(X + o), x1v = *reinterpret_cast<const uint4*>(X + o + half);
+            const T* x0 = reinterpret_cast<const T*>(&x0v);
+            const T* x1 = reinterpret_cast<const T*>(&x1v);
+            T* y0 = reinterpret_cast<T*>(&y0v);
+            T* y1 = reinterpret_cast<T*>(&y1v);
+            const float4* tb = reinterpret_cast<const float4*>(table + (int64_t)p * half + f);
+#pragma unroll
+            for (int q = 0; q < VEC / 2; ++q) {
+                const float4 cs = tb[q];
+                float a0, a1, b0, b1;
+                rotate(ld_f(x0 + 2 * q), ld_f(x1 + 2 * q), make_float2(cs.x, cs.y), sgn, a0, a1);
+                rotate(ld_f(x0 + 2 * q + 1), ld_f(x1 + 2 * q + 1), make_float2(cs.z, cs.w), sgn, b0, b1);
+                st_f(y0 + 2 * q, a0);
+                st_f(y1 + 2 * q, a1);
+                st_f(y0 + 2 * q + 1, b0);
+                st_f(y1 + 2 * q + 1, b1);
+            }
+        }
+        *reinterpret_cast<uint4*>(Y + o) = y0v;
+        *reinterpret_cast<uint4*>(Y + o + half) = y1v;
+    }
+}
+
 // Segment key rows: Y[(kmb + s nt) 128 + j] = R(p_s(j)) X[j], zero off-view.
 template <typename T>
 __global__ void __launch_bounds__(256) k_rope_segments(VisView v, const int32_t* __restrict__ pos,
@@ -237,12 +284,23 @@ mw_status rope_rows(const mw_vis_layout* L, const void* vis, const int32_t* pos,
     const float2* tb = reinterpret_cast<const float2*>(table);
     const float sgn = inverse ? -1.f : 1.f;
     count_launches(1);
-    if (dtype == MW_F32)
-        k_rope_rows<float><<<(unsigned)L->n_tiles, 256, 0, s>>>(v, pos, tb, n_pos, (const float*)X, (float*)Y, H, Dh,
-                                                                sgn);
-    else
-        k_rope_rows<__nv_bfloat16><<<(unsigned)L->n_tiles, 256, 0, s>>>(
-            v, pos, tb, n_pos, (const __nv_bfloat16*)X, (__nv_bfloat16*)Y, H, Dh, sgn);
+    const int esz = dtype == MW_F32 ? 4 : 2;
+    const bool vec = ((Dh / 2) * esz) % 16 == 0 && ((uintptr_t)X | (uintptr_t)Y) % 16 == 0;
+    if (dtype == MW_F32) {
+        if (vec)
+            k_rope_rows_vec<float><<<(unsigned)L->n_tiles, 256, 0, s>>>(v, pos, tb, n_pos, (const float*)X, (float*)Y,
+                                                                        H, Dh, sgn);
+        else
+            k_rope_rows<float><<<(unsigned)L->n_tiles, 256, 0, s>>>(v, pos, tb, n_pos, (const float*)X, (float*)Y, H,
+                                                                    Dh, sgn);
+    } else {
+        if (vec)
+            k_rope_rows_vec<__nv_bfloat16><<<(unsigned)L->n_tiles, 256, 0, s>>>(
+                v, pos, tb, n_pos, (const __nv_bfloat16*)X, (__nv_bfloat16*)Y, H, Dh, sgn);
+        else
+            k_rope_rows<__nv_bfloat16><<<(unsigned)L->n_tiles, 256, 0, s>>>(
+                v, pos, tb, n_pos, (const __nv_bfloat16*)X, (__nv_bfloat16*)Y, H, Dh, sgn);
+    }
     return launch_status();
 }
 

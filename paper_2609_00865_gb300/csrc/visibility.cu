@@ -255,8 +255,8 @@ __global__ void k_tile_stats(BuildArgs a) {
         a.tstat[4 * g + 2] = max(smax[0], smax[1]);   // keys 0..63 (INT32_MIN when none in range)
         a.tstat[4 * g + 3] = max(smax[2], smax[3]);   // keys 64..127
         unsigned long long p = spair[0] + spair[1] + spair[2] + spair[3];
-        atomicAdd(&a.pairs[b], p);
-        atomicAdd(&a.pairs[a.n_traj], p);
+        atomicAdd(&a.pairs[b], p);   // the job total is summed by k_scan (one address for
+                                     // every tile would serialise the tiles' atomics)
     }
 }
 
@@ -307,21 +307,29 @@ __global__ void k_bwd_count(BuildArgs a) {
     if (lane == 0) a.bwd_cnt[g] = cnt;
 }
 
-// Single block: exclusive scans of both count arrays into the list pointers.
+// Single block: exclusive scans of both count arrays into the list pointers,
+// four consecutive counts per thread (a pass covers 4 x blockDim tiles).
 __global__ void k_scan(BuildArgs a) {
+    constexpr int VPT = 4;
     __shared__ int carry[2];
     __shared__ int wsum[2][32];
     int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
     if (threadIdx.x < 2) carry[threadIdx.x] = 0;
     __syncthreads();
-    for (int64_t c0 = 0; c0 < a.n_tiles; c0 += blockDim.x) {
-        int64_t i = c0 + threadIdx.x;
-        int v[2];
-        v[0] = i < a.n_tiles ? a.fwd_cnt[i] : 0;
-        v[1] = i < a.n_tiles ? a.bwd_cnt[i] : 0;
+    for (int64_t c0 = 0; c0 < a.n_tiles; c0 += (int64_t)blockDim.x * VPT) {
+        const int64_t i0 = c0 + (int64_t)threadIdx.x * VPT;
+        int v[2][VPT], tot[2] = {0, 0};
+#pragma unroll
+        for (int k = 0; k < VPT; ++k) {
+            const bool in = i0 + k < a.n_tiles;
+            v[0][k] = in ? a.fwd_cnt[i0 + k] : 0;
+            v[1][k] = in ? a.bwd_cnt[i0 + k] : 0;
+            tot[0] += v[0][k];
+            tot[1] += v[1][k];
+        }
         int inc[2];
         for (int q = 0; q < 2; ++q) {
-            int x = v[q];
+            int x = tot[q];
 #pragma unroll
             for (int o = 1; o < 32; o <<= 1) {
                 int y = __shfl_up_sync(0xffffffffu, x, o);
@@ -344,9 +352,13 @@ __global__ void k_scan(BuildArgs a) {
         }
         __syncthreads();
         for (int q = 0; q < 2; ++q) {
-            int before = carry[q] + (w > 0 ? wsum[q][w - 1] : 0) + inc[q] - v[q];
+            int before = carry[q] + (w > 0 ? wsum[q][w - 1] : 0) + inc[q] - tot[q];
             int32_t* ptr = q == 0 ? a.fwd_ptr : a.bwd_ptr;
-            if (i < a.n_tiles) ptr[i] = before;
+#pragma unroll
+            for (int k = 0; k < VPT; ++k) {
+                if (i0 + k < a.n_tiles) ptr[i0 + k] = before;
+                before += v[q][k];
+            }
         }
         __syncthreads();
         if (threadIdx.x == 0) {
@@ -358,6 +370,19 @@ __global__ void k_scan(BuildArgs a) {
     if (threadIdx.x == 0) {
         a.fwd_ptr[a.n_tiles] = carry[0];
         a.bwd_ptr[a.n_tiles] = carry[1];
+    }
+    // job total of the visible pairs (the trajectories' sums are complete:
+    // k_tile_stats ran before this launch)
+    unsigned long long tp = 0;
+    for (int b = threadIdx.x; b < a.n_traj; b += blockDim.x) tp += a.pairs[b];
+    tp = warp_sum_u64(tp);
+    __shared__ unsigned long long psum[32];
+    if (lane == 0) psum[w] = tp;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        unsigned long long t = 0;
+        for (int q = 0; q < nw; ++q) t += psum[q];
+        a.pairs[a.n_traj] = t;
     }
 }
 
@@ -479,7 +504,6 @@ struct EventArgs {
 
 __global__ void __launch_bounds__(1024) k_event_views(EventArgs a) {
     __shared__ int wsum[32];
-    __shared__ int n_s;
     const int b = blockIdx.x;
     const int t = threadIdx.x, lane = t & 31, w = t >> 5;
     const int64_t tok0 = a.traj_tok[b];

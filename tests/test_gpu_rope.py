@@ -83,14 +83,17 @@ def test_rope_table_matches_float64():
     assert_maxabs(t[..., 1], np.sin(ang), 1e-7, "sin")
 
 
+# Dh 64: 16-byte vector kernel for both dtypes; 40: vectors for float32 only
+# (half a bf16 row is 40 bytes); 36: element kernel for both
+@pytest.mark.parametrize("Dh", [64, 40, 36])
 @pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
-def test_rope_rows_rotate_by_own_logical_position(dtype):
+def test_rope_rows_rotate_by_own_logical_position(dtype, Dh):
     import paper_2609_00865_gb300 as mw
     seqlens, edits = _medium_record(4)
     vis = mw.build_visibility(seqlens, edits)
     pos = mw.logical_positions(vis)
-    table = mw.rope_table(mw.rope_n_pos(vis), 64, 1e4)
-    X = synth.normal((sum(seqlens), 3, 64), 77).to(dtype)
+    table = mw.rope_table(mw.rope_n_pos(vis), Dh, 1e4)
+    X = synth.normal((sum(seqlens), 3, Dh), 77).to(dtype)
     x = X.cuda()
     Y = mw.rope_rows(vis, pos, table, x)
     # own position of every row, from the oracle's views
