@@ -66,7 +66,10 @@ constexpr int FWD_PV_WARP = 6;
 // Backward kernels: warp 0 TMA, warp 1 the recomputed products, warps 2..9
 // elementwise, warp 10 the gradient accumulation. Two elementwise warps per TMEM
 // lane quarter split each row's columns, which hides the latency of the exp /
-// scale / pack chains that bound the kernels with one warp per quarter.
+// scale / pack chains that bound the kernels with one warp per quarter. The two
+// MMA warps issue warp-converged (tc::mma_*_w: the whole warp runs the loop, one
+// elected lane issues), which cuts the issue cost of their many N = 64 / N = 128
+// products; the forward keeps single-lane issue, measured faster there.
 constexpr int NT_BWD = 352;
 constexpr int BWD_ACC_WARP = 10;
 constexpr int NEW = 256;   // elementwise threads
@@ -636,88 +639,86 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             }
         }
     } else if (warp == 1 || warp == BWD_ACC_WARP) {
-        if (lane == 0) {
-            const uint32_t iKK = idesc_bf16(128, 128, 0, 0);  // both operands K-major
-            const uint32_t iMN = idesc_bf16(128, 128, 0, 1);  // B MN-major
-            const uint32_t sq = smem_u32(sm + DQ_Q), sdo = smem_u32(sm + DQ_DO), sk = smem_u32(sm + DQ_K),
-                           sv = smem_u32(sm + DQ_V);
-            bool ok = mbar_wait(&q_full, 0, status, 211);
-            // S_j (needs K_j and a free S buffer)
-            // A tile whose first or second key half no row sees is computed over
-            // the live half only: S and dP with N = 64, dQ += dS K with K = 64
-            const uint32_t iKK64 = idesc_bf16(128, 64, 0, 0);
-            auto issue_s = [&](int j, int e) -> bool {
-                const int s = j & 1;
-                if (!mbar_wait(&k_full[s], (j >> 1) & 1, status, 212)) return false;
-                if (j >= 2 && !mbar_wait(&s_free[s], ((j - 2) >> 1) & 1, status, 213)) return false;
-                tc_fence_after();
-                if (e & (MW_TILE_DEAD_LO | MW_TILE_DEAD_HI)) {
-                    // the live half's 64 keys: rows 64 lh.. of each 64-column panel
-                    const uint32_t kh = sk + s * TILE_B + ((e & MW_TILE_DEAD_LO) ? 64u * 128u : 0u);
+        const uint32_t iKK = idesc_bf16(128, 128, 0, 0);  // both operands K-major
+        const uint32_t iMN = idesc_bf16(128, 128, 0, 1);  // B MN-major
+        const uint32_t sq = smem_u32(sm + DQ_Q), sdo = smem_u32(sm + DQ_DO), sk = smem_u32(sm + DQ_K),
+                       sv = smem_u32(sm + DQ_V);
+        bool ok = mbar_wait_warp(&q_full, 0, status, 211);
+        // S_j (needs K_j and a free S buffer)
+        // A tile whose first or second key half no row sees is computed over
+        // the live half only: S and dP with N = 64, dQ += dS K with K = 64
+        const uint32_t iKK64 = idesc_bf16(128, 64, 0, 0);
+        auto issue_s = [&](int j, int e) -> bool {
+            const int s = j & 1;
+            if (!mbar_wait_warp(&k_full[s], (j >> 1) & 1, status, 212)) return false;
+            if (j >= 2 && !mbar_wait_warp(&s_free[s], ((j - 2) >> 1) & 1, status, 213)) return false;
+            tc_fence_after();
+            if (e & (MW_TILE_DEAD_LO | MW_TILE_DEAD_HI)) {
+                // the live half's 64 keys: rows 64 lh.. of each 64-column panel
+                const uint32_t kh = sk + s * TILE_B + ((e & MW_TILE_DEAD_LO) ? 64u * 128u : 0u);
 #pragma unroll
-                    for (int ks = 0; ks < 8; ++ks) mma_ss(tmem + TM_S0 + s * 128, kmaj(sq, ks), kmaj(kh, ks), iKK64, ks > 0);
-                } else {
-#pragma unroll
-                    for (int ks = 0; ks < 8; ++ks)
-                        mma_ss(tmem + TM_S0 + s * 128, kmaj(sq, ks), kmaj(sk + s * TILE_B, ks), iKK, ks > 0);
-                }
-                mma_commit(&s_full[s]);
-                return true;
-            };
-            // dP_j (needs V_j and the softmax to have read dP_{j-1})
-            auto issue_dp = [&](int j, int e) -> bool {
-                const int s = j & 1;
-                if (!mbar_wait(&v_full[s], (j >> 1) & 1, status, 214)) return false;
-                if (j >= 1 && !mbar_wait(&dp_free, (j - 1) & 1, status, 215)) return false;
-                tc_fence_after();
-                if (e & (MW_TILE_DEAD_LO | MW_TILE_DEAD_HI)) {
-                    const uint32_t vh = sv + s * TILE_B + ((e & MW_TILE_DEAD_LO) ? 64u * 128u : 0u);
-#pragma unroll
-                    for (int ks = 0; ks < 8; ++ks) mma_ss(tmem + TM_DP, kmaj(sdo, ks), kmaj(vh, ks), iKK64, ks > 0);
-                } else {
-#pragma unroll
-                    for (int ks = 0; ks < 8; ++ks)
-                        mma_ss(tmem + TM_DP, kmaj(sdo, ks), kmaj(sv + s * TILE_B, ks), iKK, ks > 0);
-                }
-                mma_commit(&v_empty[s]);
-                mma_commit(&dp_full);
-                return true;
-            };
-            // dQ += dS_t K_t, dS_t (bf16 pairs) read from TMEM: keys 0..63 in
-            // columns 0..31 and keys 64..127 in columns 64..95 of S buffer t & 1
-            // (half tile: the live half's keys 0..31 in columns 0..15, keys
-            // 32..63 in columns 32..47; K rows from 16-row k-step 4 lh on)
-            auto issue_dq = [&](int t) -> bool {
-                const int e = entry(t);
-                if (!mbar_wait(&ds_full[t & 1], (t >> 1) & 1, status, 216)) return false;
-                tc_fence_after();
-                const uint32_t da = tmem + TM_S0 + (t & 1) * 128;
-                if (e & (MW_TILE_DEAD_LO | MW_TILE_DEAD_HI)) {
-                    const int kh = (e & MW_TILE_DEAD_LO) ? 4 : 0;
-#pragma unroll
-                    for (int ks = 0; ks < 4; ++ks)
-                        mma_ts(tmem + TM_DQ, da + (ks < 2 ? 8 * ks : 32 + 8 * (ks - 2)),
-                               mnmaj(sk + (t & 1) * TILE_B, ks + kh), iMN, (t > 0 || ks > 0));
-                } else {
-#pragma unroll
-                    for (int ks = 0; ks < 8; ++ks)
-                        mma_ts(tmem + TM_DQ, da + (ks < 4 ? 8 * ks : 64 + 8 * (ks - 4)),
-                               mnmaj(sk + (t & 1) * TILE_B, ks), iMN, (t > 0 || ks > 0));
-                }
-                mma_commit(&k_empty[t & 1]);
-                mma_commit(&s_free[t & 1]);
-                if (t == n - 1) mma_commit(&dq_fin);
-                return true;
-            };
-            if (warp == 1) {
-                for (int j = 0; ok && j < n; ++j) {
-                    const int e = entry(j);
-                    ok = issue_s(j, e) && issue_dp(j, e);
-                }
+                for (int ks = 0; ks < 8; ++ks) mma_ss_w(tmem + TM_S0 + s * 128, kmaj(sq, ks), kmaj(kh, ks), iKK64, ks > 0);
             } else {
-                // dQ's K-stage release also covers S_j: dS_j exists only once S_j is done
-                for (int j = 0; ok && j < n; ++j) ok = issue_dq(j);
+#pragma unroll
+                for (int ks = 0; ks < 8; ++ks)
+                    mma_ss_w(tmem + TM_S0 + s * 128, kmaj(sq, ks), kmaj(sk + s * TILE_B, ks), iKK, ks > 0);
             }
+            mma_commit_w(&s_full[s]);
+            return true;
+        };
+        // dP_j (needs V_j and the softmax to have read dP_{j-1})
+        auto issue_dp = [&](int j, int e) -> bool {
+            const int s = j & 1;
+            if (!mbar_wait_warp(&v_full[s], (j >> 1) & 1, status, 214)) return false;
+            if (j >= 1 && !mbar_wait_warp(&dp_free, (j - 1) & 1, status, 215)) return false;
+            tc_fence_after();
+            if (e & (MW_TILE_DEAD_LO | MW_TILE_DEAD_HI)) {
+                const uint32_t vh = sv + s * TILE_B + ((e & MW_TILE_DEAD_LO) ? 64u * 128u : 0u);
+#pragma unroll
+                for (int ks = 0; ks < 8; ++ks) mma_ss_w(tmem + TM_DP, kmaj(sdo, ks), kmaj(vh, ks), iKK64, ks > 0);
+            } else {
+#pragma unroll
+                for (int ks = 0; ks < 8; ++ks)
+                    mma_ss_w(tmem + TM_DP, kmaj(sdo, ks), kmaj(sv + s * TILE_B, ks), iKK, ks > 0);
+            }
+            mma_commit_w(&v_empty[s]);
+            mma_commit_w(&dp_full);
+            return true;
+        };
+        // dQ += dS_t K_t, dS_t (bf16 pairs) read from TMEM: keys 0..63 in
+        // columns 0..31 and keys 64..127 in columns 64..95 of S buffer t & 1
+        // (half tile: the live half's keys 0..31 in columns 0..15, keys
+        // 32..63 in columns 32..47; K rows from 16-row k-step 4 lh on)
+        auto issue_dq = [&](int t) -> bool {
+            const int e = entry(t);
+            if (!mbar_wait_warp(&ds_full[t & 1], (t >> 1) & 1, status, 216)) return false;
+            tc_fence_after();
+            const uint32_t da = tmem + TM_S0 + (t & 1) * 128;
+            if (e & (MW_TILE_DEAD_LO | MW_TILE_DEAD_HI)) {
+                const int kh = (e & MW_TILE_DEAD_LO) ? 4 : 0;
+#pragma unroll
+                for (int ks = 0; ks < 4; ++ks)
+                    mma_ts_w(tmem + TM_DQ, da + (ks < 2 ? 8 * ks : 32 + 8 * (ks - 2)),
+                           mnmaj(sk + (t & 1) * TILE_B, ks + kh), iMN, (t > 0 || ks > 0));
+            } else {
+#pragma unroll
+                for (int ks = 0; ks < 8; ++ks)
+                    mma_ts_w(tmem + TM_DQ, da + (ks < 4 ? 8 * ks : 64 + 8 * (ks - 4)),
+                           mnmaj(sk + (t & 1) * TILE_B, ks), iMN, (t > 0 || ks > 0));
+            }
+            mma_commit_w(&k_empty[t & 1]);
+            mma_commit_w(&s_free[t & 1]);
+            if (t == n - 1) mma_commit_w(&dq_fin);
+            return true;
+        };
+        if (warp == 1) {
+            for (int j = 0; ok && j < n; ++j) {
+                const int e = entry(j);
+                ok = issue_s(j, e) && issue_dp(j, e);
+            }
+        } else {
+            // dQ's K-stage release also covers S_j: dS_j exists only once S_j is done
+            for (int j = 0; ok && j < n; ++j) ok = issue_dq(j);
         }
     } else {
         // row rl = TMEM lane; this warp's 64 of the 128 key columns: [64 ch, 64 ch + 64)
@@ -1007,51 +1008,49 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             }
         }
     } else if (warp == 1 || warp == BWD_ACC_WARP) {
-        if (lane == 0) {
-            const uint32_t iSD = idesc_bf16(128, 64, 0, 0);
-            const uint32_t iAC = idesc_bf16(128, 128, 0, 1);
-            const uint32_t sk = smem_u32(sm + KV_K), sv = smem_u32(sm + KV_V), sq = smem_u32(sm + KV_Q);
-            bool ok = mbar_wait(&kv_full, 0, status, 221);
-            auto issue_sd = [&](int t) -> bool {
-                const int s = t & 1, qs = t % QD_ST;
-                if (!mbar_wait(&qd_full[qs], (t / QD_ST) & 1, status, 222)) return false;
-                if (t >= 2 && !mbar_wait(&sd_free[s], ((t - 2) >> 1) & 1, status, 223)) return false;
-                tc_fence_after();
-                const uint32_t qb = sq + qs * 2 * HT_B, db = qb + HT_B;
+        const uint32_t iSD = idesc_bf16(128, 64, 0, 0);
+        const uint32_t iAC = idesc_bf16(128, 128, 0, 1);
+        const uint32_t sk = smem_u32(sm + KV_K), sv = smem_u32(sm + KV_V), sq = smem_u32(sm + KV_Q);
+        bool ok = mbar_wait_warp(&kv_full, 0, status, 221);
+        auto issue_sd = [&](int t) -> bool {
+            const int s = t & 1, qs = t % QD_ST;
+            if (!mbar_wait_warp(&qd_full[qs], (t / QD_ST) & 1, status, 222)) return false;
+            if (t >= 2 && !mbar_wait_warp(&sd_free[s], ((t - 2) >> 1) & 1, status, 223)) return false;
+            tc_fence_after();
+            const uint32_t qb = sq + qs * 2 * HT_B, db = qb + HT_B;
 #pragma unroll
-                for (int ks = 0; ks < 8; ++ks) mma_ss(tmem + TM_ST + s * 64, kmaj(sk, ks), kmaj_ht(qb, ks), iSD, ks > 0);
+            for (int ks = 0; ks < 8; ++ks) mma_ss_w(tmem + TM_ST + s * 64, kmaj(sk, ks), kmaj_ht(qb, ks), iSD, ks > 0);
 #pragma unroll
-                for (int ks = 0; ks < 8; ++ks) mma_ss(tmem + TM_DPT + s * 64, kmaj(sv, ks), kmaj_ht(db, ks), iSD, ks > 0);
-                mma_commit(&sd_full[s]);
-                return true;
-            };
-            auto issue_acc = [&](int t) -> bool {
-                const int s = t & 1, qs = t % QD_ST;
-                if (!mbar_wait(&pd_full[s], (t >> 1) & 1, status, 224)) return false;
-                tc_fence_after();
-                const uint32_t qb = sq + qs * 2 * HT_B, db = qb + HT_B;
-                // P^T, dS^T (bf16 pairs of query rows) in TMEM: rows 0..31 of the
-                // half-step in columns 0..15, rows 32..63 in columns 32..47 of
-                // their S^T / dP^T buffer
+            for (int ks = 0; ks < 8; ++ks) mma_ss_w(tmem + TM_DPT + s * 64, kmaj(sv, ks), kmaj_ht(db, ks), iSD, ks > 0);
+            mma_commit_w(&sd_full[s]);
+            return true;
+        };
+        auto issue_acc = [&](int t) -> bool {
+            const int s = t & 1, qs = t % QD_ST;
+            if (!mbar_wait_warp(&pd_full[s], (t >> 1) & 1, status, 224)) return false;
+            tc_fence_after();
+            const uint32_t qb = sq + qs * 2 * HT_B, db = qb + HT_B;
+            // P^T, dS^T (bf16 pairs of query rows) in TMEM: rows 0..31 of the
+            // half-step in columns 0..15, rows 32..63 in columns 32..47 of
+            // their S^T / dP^T buffer
 #pragma unroll
-                for (int ks = 0; ks < 4; ++ks)
-                    mma_ts(tmem + TM_DV, tmem + TM_ST + s * 64 + 32 * (ks >> 1) + 8 * (ks & 1), mnmaj_ht(db, ks), iAC,
-                           (t > 0 || ks > 0));
+            for (int ks = 0; ks < 4; ++ks)
+                mma_ts_w(tmem + TM_DV, tmem + TM_ST + s * 64 + 32 * (ks >> 1) + 8 * (ks & 1), mnmaj_ht(db, ks), iAC,
+                       (t > 0 || ks > 0));
 #pragma unroll
-                for (int ks = 0; ks < 4; ++ks)
-                    mma_ts(tmem + TM_DK, tmem + TM_DPT + s * 64 + 32 * (ks >> 1) + 8 * (ks & 1), mnmaj_ht(qb, ks), iAC,
-                           (t > 0 || ks > 0));
-                mma_commit(&qd_empty[qs]);
-                mma_commit(&sd_free[s]);
-                return true;
-            };
-            if (warp == 1) {
-                for (int t = 0; ok && t < nsteps; ++t) ok = issue_sd(t);
-            } else {
-                // the Q/dO stage release also covers S^T_t, dP^T_t: P^T_t, dS^T_t
-                // exist only once those are done
-                for (int t = 0; ok && t < nsteps; ++t) ok = issue_acc(t);
-            }
+            for (int ks = 0; ks < 4; ++ks)
+                mma_ts_w(tmem + TM_DK, tmem + TM_DPT + s * 64 + 32 * (ks >> 1) + 8 * (ks & 1), mnmaj_ht(qb, ks), iAC,
+                       (t > 0 || ks > 0));
+            mma_commit_w(&qd_empty[qs]);
+            mma_commit_w(&sd_free[s]);
+            return true;
+        };
+        if (warp == 1) {
+            for (int t = 0; ok && t < nsteps; ++t) ok = issue_sd(t);
+        } else {
+            // the Q/dO stage release also covers S^T_t, dP^T_t: P^T_t, dS^T_t
+            // exist only once those are done
+            for (int t = 0; ok && t < nsteps; ++t) ok = issue_acc(t);
         }
     } else {
         // key row rl = TMEM lane; this warp's 32 of a half-step's 64 query
