@@ -51,14 +51,15 @@ def _peaks():
 # value it had when the counters were taken.
 TRAFFIC = {
     (4, "mw_logprob_loss_bwd"): {
-        "bytes": 79358121984 + 11882540288 + 86699048960 + 14107458304,   # dH pass + dW pass
+        "bytes": 456960 + (75984701184 + 14093292288) + (807883264 + 247791360),   # par, dW pass, dH from E
         "source": "paper_2609_00865_gb300/csrc/lmhead_bwd_tc.cu",
-        "sha256": "5657c62c221bfbecae71d0954adb5970de2d73155845e6fa0d1761f9c1df110e",
+        "sha256": "e37a7e91c915817da7a63c8ebadd255f857d5416446f4690c688316990724030",
     },
     (4, "mw_masked_attn_bwd"): {
-        "bytes": (1894422272 + 28065792) + (30600770560 + 908907264) + (63477532416 + 263952896),   # lsd, dQ, dK/dV
+        # lsd, compact gather, dQ (main + junction items), dK/dV, per-key reduce
+        "bytes": 1922954752 + 1162634496 + (5043770112 + 522220544) + 5442257408 + 1764790528,
         "source": "paper_2609_00865_gb300/csrc/attn_tc.cu",
-        "sha256": "e5b85e37e292919afdef3229f3f80edc0e1bcb77282b62adcab6eb45c08821d1",
+        "sha256": "ae00024ee8b3ca55fc8c484243bd1002812d7be78b2656cc923c2f786dcf1891",
     },
 }
 
@@ -592,11 +593,9 @@ def cpu_sample(w, budget_s=15.0):
         pool = w["rows"].numpy().astype(np.int64)
     else:
         pool = np.arange(w["record"].total)
-    done, t0 = 0, time.perf_counter()
     batch = 8
-    parts = []
-    while time.perf_counter() - t0 < budget_s and done < 4096:
-        rows = np.sort(rng.choice(pool, size=batch, replace=False))
+
+    def one_batch(rows):
         parts = []
         O = None
         if "record" in w:
@@ -617,6 +616,15 @@ def cpu_sample(w, budget_s=15.0):
             lp, lse = OL.logprob(H, x["W"], w["targets"].numpy(), rows)
             g = OL.policy_loss(lp, lp + 0.01, np.ones_like(lp), EPS_LO, EPS_HI)[3]
             OL.logprob_loss_bwd(H, x["W"], w["targets"].numpy(), rows, lse, g)
+        return parts
+
+    # one untimed batch first: the first call of the process pays one-time costs
+    # (thread pools, first touch of the float64 copies) that no later batch does
+    one_batch(np.sort(rng.choice(pool, size=batch, replace=False)))
+    done, t0 = 0, time.perf_counter()
+    parts = []
+    while time.perf_counter() - t0 < budget_s and done < 4096:
+        parts = one_batch(np.sort(rng.choice(pool, size=batch, replace=False)))
         done += batch
     dt = time.perf_counter() - t0
     return done / dt, cores, f"{done} sampled scored tokens ({' + '.join(parts)}), {dt:.1f} s"
