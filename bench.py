@@ -618,9 +618,12 @@ def cpu_sample(w, budget_s=15.0):
             OL.logprob_loss_bwd(H, x["W"], w["targets"].numpy(), rows, lse, g)
         return parts
 
-    # one untimed batch first: the first call of the process pays one-time costs
-    # (thread pools, first touch of the float64 copies) that no later batch does
-    one_batch(np.sort(rng.choice(pool, size=batch, replace=False)))
+    # one untimed batch on the first call: the first batch of a process pays
+    # one-time costs (thread pools, first touch of the float64 copies) that no
+    # later batch does
+    if not w.get("_warm"):
+        one_batch(np.sort(rng.choice(pool, size=batch, replace=False)))
+        w["_warm"] = True
     done, t0 = 0, time.perf_counter()
     parts = []
     while time.perf_counter() - t0 < budget_s and done < 4096:
