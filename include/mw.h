@@ -178,7 +178,9 @@ mw_status mw_build_views_events(const mw_vis_layout* layout, const int32_t* cu_s
 /*
  * Build every visibility artefact of a record (§4.2 lifetimes; App. B.1
  * segments) into `vis` (layout->vis_bytes, device) using `ws`
- * (layout->ws_bytes, device).
+ * (layout->ws_bytes, device). Both must be 256-byte aligned (every array of
+ * the layout sits at a 256-byte offset; cudaMalloc's alignment suffices), else
+ * MW_EINVAL.
  *   junctions[n_junc]      host int32, traj-local J_k, strictly ascending
  *                          within a trajectory, 1 <= J_k <= T_b - 1
  *   junc_traj[n_junc]      host int32, owning trajectory, non-decreasing

@@ -19,6 +19,9 @@
 
 namespace mw {
 
+// tiles per block of the list-pointer scan
+constexpr int SCAN_BLOCK = 1024;
+
 static thread_local int g_last_cuda_error = 0;
 
 mw_status cuda_status(cudaError_t e) {
@@ -124,7 +127,9 @@ extern "C" mw_status mw_visibility_layout(int n_traj, const int32_t* cu, int n_j
     o = 0;
     L->ws_off_spans = take(12 * (int64_t)n_spans);
     L->ws_off_tstat = take(16 * tiles);
-    L->ws_off_cnt = take(8 * tiles);
+    // fwd / bwd counts [2][tiles] int32, per-tile pairs [tiles] uint64, the
+    // scan's per-block sums and offsets [2][2][scan blocks] int32
+    L->ws_off_cnt = take(8 * tiles + 8 * tiles + 16 * ceil_div(tiles, (int64_t)SCAN_BLOCK));
     L->ws_bytes = o;
     L->max_segs = max_segs;
     return MW_OK;
@@ -178,6 +183,8 @@ struct BuildArgs {
     int32_t* tstat;         // [n_tiles][4] min, max lifetime; max over keys 0..63, 64..127
     int32_t* fwd_cnt;       // [n_tiles]
     int32_t* bwd_cnt;       // [n_tiles]
+    unsigned long long* tpairs;   // [n_tiles] visible pairs per k-tile
+    int32_t* bsum;          // [2][n_scan_blocks] per-block count sums, then exclusive offsets
 };
 
 __device__ __forceinline__ int find_traj(const int32_t* off, int n, int64_t t) {
@@ -189,20 +196,56 @@ __device__ __forceinline__ int find_traj(const int32_t* off, int n, int64_t t) {
     return lo;
 }
 
-// omega = never; seg = number of junctions <= local row.
+// omega = never; seg = number of junctions <= local row. A thread takes 16
+// consecutive tokens: one search for the first token's trajectory and
+// segment, then it steps across boundaries, and stores 64-byte runs.
+constexpr int INIT_TPT = 16;
 __global__ void k_init_tokens(BuildArgs a) {
-    for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < a.total;
-         t += (int64_t)gridDim.x * blockDim.x) {
-        int b = find_traj(a.traj_tok, a.n_traj, t);
-        int i = (int)(t - a.traj_tok[b]);
+    const int64_t n_chunks = (a.total + INIT_TPT - 1) / INIT_TPT;
+    for (int64_t c = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; c < n_chunks;
+         c += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t t0 = c * INIT_TPT;
+        int b = find_traj(a.traj_tok, a.n_traj, t0);
         int s0 = a.traj_seg[b], s1 = a.traj_seg[b + 1];
-        int lo = s0, hi = s1;  // seg_start[lo] <= i (seg_start[s0] = 0)
+        int i0 = (int)(t0 - a.traj_tok[b]);
+        int lo = s0, hi = s1;   // seg_start[lo] <= i0 (seg_start[s0] = 0)
         while (hi - lo > 1) {
-            int mid = (lo + hi) >> 1;
-            if (a.seg_start[mid] <= i) lo = mid; else hi = mid;
+            const int mid = (lo + hi) >> 1;
+            if (a.seg_start[mid] <= i0) lo = mid; else hi = mid;
         }
-        a.omega[t] = INT32_MAX;
-        a.seg[t] = lo - s0;
+        int32_t segv[INIT_TPT];
+#pragma unroll
+        for (int k = 0; k < INIT_TPT; ++k) {
+            const int64_t t = t0 + k;
+            if (t < a.total) {
+                while (t >= a.traj_tok[b + 1]) {   // next non-empty trajectory
+                    ++b;
+                    s0 = a.traj_seg[b];
+                    s1 = a.traj_seg[b + 1];
+                    lo = s0;
+                }
+                const int i = (int)(t - a.traj_tok[b]);
+                while (lo + 1 < s1 && a.seg_start[lo + 1] <= i) ++lo;
+                segv[k] = lo - s0;
+            }
+        }
+        if (t0 + INIT_TPT <= a.total) {
+            const int4 never = make_int4(INT32_MAX, INT32_MAX, INT32_MAX, INT32_MAX);
+#pragma unroll
+            for (int q = 0; q < INIT_TPT / 4; ++q) {
+                reinterpret_cast<int4*>(a.omega + t0)[q] = never;
+                reinterpret_cast<int4*>(a.seg + t0)[q] = make_int4(segv[4 * q], segv[4 * q + 1], segv[4 * q + 2],
+                                                                   segv[4 * q + 3]);
+            }
+        } else {
+#pragma unroll
+            for (int k = 0; k < INIT_TPT; ++k) {
+                if (t0 + k < a.total) {
+                    a.omega[t0 + k] = INT32_MAX;
+                    a.seg[t0 + k] = segv[k];
+                }
+            }
+        }
     }
 }
 
@@ -214,49 +257,65 @@ __global__ void k_scatter_spans(BuildArgs a) {
     }
 }
 
-// One block (128 threads) per global k-tile: min / max lifetime over its keys,
-// visible pairs sum_j (min(omega_j, T) - j), and the per-segment view bits.
-__global__ void k_tile_stats(BuildArgs a) {
-    int64_t g = blockIdx.x;
-    int b = a.tile_traj[g];
-    int kt = (int)(g - a.traj_tile[b]);
-    int T = a.traj_tok[b + 1] - a.traj_tok[b];
-    int j = kt * MW_TILE + threadIdx.x;
-    bool in = j < T;
-    int om = in ? a.omega[a.traj_tok[b] + j] : 0;
-    int omc = in ? min(om, T) : 0;
-    int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-    __shared__ int smin[4], smax[4];
-    __shared__ unsigned long long spair[4];
-    int vmin = in ? om : INT32_MAX, vmax = in ? om : INT32_MIN;
-    unsigned long long pr = in ? (unsigned long long)(omc - j) : 0ull;
+// One warp per global k-tile (a lane takes keys lane, lane + 32, lane + 64,
+// lane + 96): min / max lifetime over its keys, visible pairs sum_j
+// (min(omega_j, T) - j) (per tile; the scan sums them per trajectory), and the
+// per-segment view bits, one 16-byte store per segment. No block-level
+// synchronisation: the warps of a block are independent.
+__global__ void __launch_bounds__(256) k_tile_stats(BuildArgs a) {
+    const int64_t g = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    if (g >= a.n_tiles) return;   // uniform over the warp
+    const int b = a.tile_traj[g];
+    const int kt = (int)(g - a.traj_tile[b]);
+    const int T = a.traj_tok[b + 1] - a.traj_tok[b];
+    const int64_t tok0 = a.traj_tok[b];
+    int om[4];
+    int vmin[4], vmax[4];
+    unsigned long long pr = 0ull;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const int j = kt * MW_TILE + 32 * q + lane;
+        const bool in = j < T;
+        om[q] = in ? a.omega[tok0 + j] : 0;
+        vmin[q] = in ? om[q] : INT32_MAX;
+        vmax[q] = in ? om[q] : INT32_MIN;
+        if (in) pr += (unsigned long long)(min(om[q], T) - j);
+    }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
-        vmin = min(vmin, __shfl_xor_sync(0xffffffffu, vmin, o));
-        vmax = max(vmax, __shfl_xor_sync(0xffffffffu, vmax, o));
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            vmin[q] = min(vmin[q], __shfl_xor_sync(0xffffffffu, vmin[q], o));
+            vmax[q] = max(vmax[q], __shfl_xor_sync(0xffffffffu, vmax[q], o));
+        }
         pr += __shfl_xor_sync(0xffffffffu, pr, o);
     }
-    if (lane == 0) { smin[w] = vmin; smax[w] = vmax; spair[w] = pr; }
-    // view bits: key j is in segment s's view iff omega(j) > J_s and j < J_{s+1}
-    int s0 = a.traj_seg[b], nseg = a.traj_seg[b + 1] - s0;
+    // view bits: key j is in segment s's view iff omega(j) > J_s and j < J_{s+1};
+    // lane s holds J_s of the first 32 segments (later ones come from L2)
+    const int s0 = a.traj_seg[b], nseg = a.traj_seg[b + 1] - s0;
+    const int nt = a.traj_tile[b + 1] - a.traj_tile[b];
+    const int my_start = lane < nseg ? a.seg_start[s0 + lane] : T;
+    uint4* km = reinterpret_cast<uint4*>(a.keymask) + a.traj_km[b] + kt;
     for (int s = 0; s < nseg; ++s) {
-        int Js = a.seg_start[s0 + s];
-        int Jn = (s + 1 < nseg) ? a.seg_start[s0 + s + 1] : T;
-        bool bit = in && om > Js && j < Jn;
-        uint32_t word = __ballot_sync(0xffffffffu, bit);
-        if (lane == 0) a.keymask[(a.traj_km[b] + (int64_t)s * (a.traj_tile[b + 1] - a.traj_tile[b]) + kt) * 4 + w] = word;
+        const int Js = s < 32 ? __shfl_sync(0xffffffffu, my_start, s) : a.seg_start[s0 + s];
+        const int Jn = s + 1 < 32 ? __shfl_sync(0xffffffffu, my_start, s + 1)
+                                  : (s + 1 < nseg ? a.seg_start[s0 + s + 1] : T);
+        uint32_t wd[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const int j = kt * MW_TILE + 32 * q + lane;
+            wd[q] = __ballot_sync(0xffffffffu, j < T && om[q] > Js && j < Jn);
+        }
+        if (lane == 0) km[(int64_t)s * nt] = make_uint4(wd[0], wd[1], wd[2], wd[3]);
     }
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        int mn = min(min(smin[0], smin[1]), min(smin[2], smin[3]));
-        int mx = max(max(smax[0], smax[1]), max(smax[2], smax[3]));
-        a.tstat[4 * g] = mn;
-        a.tstat[4 * g + 1] = mx;
-        a.tstat[4 * g + 2] = max(smax[0], smax[1]);   // keys 0..63 (INT32_MIN when none in range)
-        a.tstat[4 * g + 3] = max(smax[2], smax[3]);   // keys 64..127
-        unsigned long long p = spair[0] + spair[1] + spair[2] + spair[3];
-        atomicAdd(&a.pairs[b], p);   // the job total is summed by k_scan (one address for
-                                     // every tile would serialise the tiles' atomics)
+    if (lane == 0) {
+        *reinterpret_cast<int4*>(a.tstat + 4 * g) =
+            make_int4(min(min(vmin[0], vmin[1]), min(vmin[2], vmin[3])),
+                      max(max(vmax[0], vmax[1]), max(vmax[2], vmax[3])),
+                      max(vmax[0], vmax[1]),    // keys 0..63 (INT32_MIN when none in range)
+                      max(vmax[2], vmax[3]));   // keys 64..127
+        a.tpairs[g] = pr;
     }
 }
 
@@ -264,12 +323,16 @@ __global__ void k_tile_stats(BuildArgs a) {
 // max over keys 0..63, max over keys 64..127). Off the diagonal every key
 // precedes every row, so row i sees key j iff i < omega(j): a key half is seen
 // by some row iff its largest lifetime exceeds the q-tile's first row.
-__device__ __forceinline__ int tile_class(int qt, int kt, int T, const int32_t* st) {
+__device__ __forceinline__ int tile_class(int qt, int kt, int T, int4 st) {
     int q0 = qt * MW_TILE, q1 = min(q0 + MW_TILE, T);
     if (kt == qt) return (q1 - q0 == 1) ? MW_TILE_FULL : MW_TILE_PARTIAL;
-    if (st[0] >= q1) return MW_TILE_FULL;
-    if (st[1] <= q0) return MW_TILE_EMPTY;
-    return MW_TILE_PARTIAL | (st[2] <= q0 ? MW_TILE_DEAD_LO : 0) | (st[3] <= q0 ? MW_TILE_DEAD_HI : 0);
+    if (st.x >= q1) return MW_TILE_FULL;
+    if (st.y <= q0) return MW_TILE_EMPTY;
+    return MW_TILE_PARTIAL | (st.z <= q0 ? MW_TILE_DEAD_LO : 0) | (st.w <= q0 ? MW_TILE_DEAD_HI : 0);
+}
+// statistics of global k-tile g (16-byte aligned: the workspace region is)
+__device__ __forceinline__ int4 tile_stat(const int32_t* tstat, int64_t g) {
+    return *reinterpret_cast<const int4*>(tstat + 4 * g);
 }
 
 // One warp per global q-tile: classes of (qt, 0..qt) and the fwd list length.
@@ -283,8 +346,9 @@ __global__ void k_classify(BuildArgs a) {
     int T = a.traj_tok[b + 1] - a.traj_tok[b];
     uint8_t* row = a.cls + a.traj_tri[b] + (int64_t)qt * (qt + 1) / 2;
     int cnt = 0;
+#pragma unroll 4
     for (int kt = lane; kt <= qt; kt += 32) {
-        int c = tile_class(qt, kt, T, a.tstat + 4 * (tb + kt));
+        int c = tile_class(qt, kt, T, tile_stat(a.tstat, tb + kt));
         row[kt] = (uint8_t)c;
         cnt += c != MW_TILE_EMPTY;
     }
@@ -292,47 +356,72 @@ __global__ void k_classify(BuildArgs a) {
     if (lane == 0) a.fwd_cnt[g] = cnt;
 }
 
-// One warp per global k-tile: bwd list length (column of the class triangle).
+// One thread per global k-tile: bwd list length, the non-EMPTY tiles of its
+// column of the class triangle. The diagonal tile is never EMPTY; below it
+// (qt > kt) a tile is EMPTY exactly when the k-tile's largest lifetime is at
+// most the q-tile's first row (tile_class), so the column's non-EMPTY tiles
+// are the q-tiles kt .. ceil(min(max lifetime, T) / 128) - 1.
 __global__ void k_bwd_count(BuildArgs a) {
-    int64_t g = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
-    int lane = threadIdx.x & 31;
+    const int64_t g = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
     if (g >= a.n_tiles) return;
-    int b = a.tile_traj[g];
-    int tb = a.traj_tile[b], nt = a.traj_tile[b + 1] - tb;
-    int kt = (int)(g - tb);
-    const uint8_t* tri = a.cls + a.traj_tri[b];
-    int cnt = 0;
-    for (int qt = kt + lane; qt < nt; qt += 32) cnt += tri[(int64_t)qt * (qt + 1) / 2 + kt] != MW_TILE_EMPTY;
-    cnt = warp_sum_i(cnt);
-    if (lane == 0) a.bwd_cnt[g] = cnt;
+    const int b = a.tile_traj[g];
+    const int tb = a.traj_tile[b], nt = a.traj_tile[b + 1] - tb;
+    const int kt = (int)(g - tb);
+    const int T = a.traj_tok[b + 1] - a.traj_tok[b];
+    const int lim = min(a.tstat[4 * g + 1], T);
+    a.bwd_cnt[g] = 1 + max(0, min(nt, (lim + MW_TILE - 1) / MW_TILE) - kt - 1);
 }
 
-// Single block: exclusive scans of both count arrays into the list pointers,
-// four consecutive counts per thread (a pass covers 4 x blockDim tiles).
-__global__ void k_scan(BuildArgs a) {
-    constexpr int VPT = 4;
-    __shared__ int carry[2];
+// List pointers: exclusive scans of both count arrays, in three launches of
+// SCAN_BLOCK-tile blocks (a single block's serial passes were the builder's
+// slowest step at batch sizes).
+// Phase 1, one block per SCAN_BLOCK tiles: the block's count sums, and the
+// visible pairs added into each tile's trajectory (one atomic per warp whose
+// 32 tiles share a trajectory, else one per tile).
+__global__ void __launch_bounds__(SCAN_BLOCK) k_scan_sums(BuildArgs a) {
+    __shared__ int ws[2][SCAN_BLOCK / 32];
+    const int64_t i = (int64_t)blockIdx.x * SCAN_BLOCK + threadIdx.x;
+    const bool in = i < a.n_tiles;
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+    const int f = warp_sum_i(in ? a.fwd_cnt[i] : 0);
+    const int k = warp_sum_i(in ? a.bwd_cnt[i] : 0);
+    if (lane == 0) { ws[0][w] = f; ws[1][w] = k; }
+    const int bt = in ? a.tile_traj[i] : -1;
+    const unsigned long long pr = in ? a.tpairs[i] : 0ull;
+    const int b0 = __shfl_sync(0xffffffffu, bt, 0);
+    if (__all_sync(0xffffffffu, bt == b0)) {
+        const unsigned long long sum = warp_sum_u64(pr);
+        if (lane == 0 && b0 >= 0) atomicAdd(&a.pairs[b0], sum);
+    } else if (in) {
+        atomicAdd(&a.pairs[bt], pr);
+    }
+    __syncthreads();
+    if (threadIdx.x < 2) {
+        int t = 0;
+        for (int q = 0; q < SCAN_BLOCK / 32; ++q) t += ws[threadIdx.x][q];
+        a.bsum[threadIdx.x * gridDim.x + blockIdx.x] = t;
+    }
+}
+
+// Phase 2, one block: exclusive offsets of the block sums (in place), both
+// lists' totals, and the job total of the visible pairs (phase 1 completed
+// every trajectory's sum).
+__global__ void __launch_bounds__(1024) k_scan_offsets(BuildArgs a, int nb) {
     __shared__ int wsum[2][32];
-    int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    __shared__ int carry[2];
+    __shared__ unsigned long long psum[32];
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
     if (threadIdx.x < 2) carry[threadIdx.x] = 0;
     __syncthreads();
-    for (int64_t c0 = 0; c0 < a.n_tiles; c0 += (int64_t)blockDim.x * VPT) {
-        const int64_t i0 = c0 + (int64_t)threadIdx.x * VPT;
-        int v[2][VPT], tot[2] = {0, 0};
-#pragma unroll
-        for (int k = 0; k < VPT; ++k) {
-            const bool in = i0 + k < a.n_tiles;
-            v[0][k] = in ? a.fwd_cnt[i0 + k] : 0;
-            v[1][k] = in ? a.bwd_cnt[i0 + k] : 0;
-            tot[0] += v[0][k];
-            tot[1] += v[1][k];
-        }
-        int inc[2];
+    for (int c0 = 0; c0 < nb; c0 += blockDim.x) {
+        const int i = c0 + threadIdx.x;
+        int v[2], inc[2];
         for (int q = 0; q < 2; ++q) {
-            int x = tot[q];
+            v[q] = i < nb ? a.bsum[q * nb + i] : 0;
+            int x = v[q];
 #pragma unroll
             for (int o = 1; o < 32; o <<= 1) {
-                int y = __shfl_up_sync(0xffffffffu, x, o);
+                const int y = __shfl_up_sync(0xffffffffu, x, o);
                 if (lane >= o) x += y;
             }
             inc[q] = x;
@@ -344,22 +433,15 @@ __global__ void k_scan(BuildArgs a) {
                 int x = lane < nw ? wsum[q][lane] : 0;
 #pragma unroll
                 for (int o = 1; o < 32; o <<= 1) {
-                    int y = __shfl_up_sync(0xffffffffu, x, o);
+                    const int y = __shfl_up_sync(0xffffffffu, x, o);
                     if (lane >= o) x += y;
                 }
-                if (lane < nw) wsum[q][lane] = x;  // inclusive over warps
+                if (lane < nw) wsum[q][lane] = x;   // inclusive over warps
             }
         }
         __syncthreads();
-        for (int q = 0; q < 2; ++q) {
-            int before = carry[q] + (w > 0 ? wsum[q][w - 1] : 0) + inc[q] - tot[q];
-            int32_t* ptr = q == 0 ? a.fwd_ptr : a.bwd_ptr;
-#pragma unroll
-            for (int k = 0; k < VPT; ++k) {
-                if (i0 + k < a.n_tiles) ptr[i0 + k] = before;
-                before += v[q][k];
-            }
-        }
+        for (int q = 0; q < 2; ++q)
+            if (i < nb) a.bsum[q * nb + i] = carry[q] + (w > 0 ? wsum[q][w - 1] : 0) + inc[q] - v[q];
         __syncthreads();
         if (threadIdx.x == 0) {
             carry[0] += wsum[0][nw - 1];
@@ -371,12 +453,9 @@ __global__ void k_scan(BuildArgs a) {
         a.fwd_ptr[a.n_tiles] = carry[0];
         a.bwd_ptr[a.n_tiles] = carry[1];
     }
-    // job total of the visible pairs (the trajectories' sums are complete:
-    // k_tile_stats ran before this launch)
     unsigned long long tp = 0;
     for (int b = threadIdx.x; b < a.n_traj; b += blockDim.x) tp += a.pairs[b];
     tp = warp_sum_u64(tp);
-    __shared__ unsigned long long psum[32];
     if (lane == 0) psum[w] = tp;
     __syncthreads();
     if (threadIdx.x == 0) {
@@ -386,7 +465,49 @@ __global__ void k_scan(BuildArgs a) {
     }
 }
 
-// One warp per global q-tile (fwd) or k-tile (bwd): ordered compaction.
+// Phase 3, one block per SCAN_BLOCK tiles: the block's exclusive scan plus its
+// offset.
+__global__ void __launch_bounds__(SCAN_BLOCK) k_scan_ptrs(BuildArgs a) {
+    __shared__ int wsum[2][SCAN_BLOCK / 32];
+    const int64_t i = (int64_t)blockIdx.x * SCAN_BLOCK + threadIdx.x;
+    const bool in = i < a.n_tiles;
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+    int v[2], inc[2];
+    v[0] = in ? a.fwd_cnt[i] : 0;
+    v[1] = in ? a.bwd_cnt[i] : 0;
+    for (int q = 0; q < 2; ++q) {
+        int x = v[q];
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, x, o);
+            if (lane >= o) x += y;
+        }
+        inc[q] = x;
+        if (lane == 31) wsum[q][w] = x;
+    }
+    __syncthreads();
+    if (w == 0) {
+        for (int q = 0; q < 2; ++q) {
+            int x = wsum[q][lane];   // SCAN_BLOCK / 32 = 32 warps
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int y = __shfl_up_sync(0xffffffffu, x, o);
+                if (lane >= o) x += y;
+            }
+            wsum[q][lane] = x;
+        }
+    }
+    __syncthreads();
+    if (in) {
+        a.fwd_ptr[i] = a.bsum[blockIdx.x] + (w > 0 ? wsum[0][w - 1] : 0) + inc[0] - v[0];
+        a.bwd_ptr[i] = a.bsum[gridDim.x + blockIdx.x] + (w > 0 ? wsum[1][w - 1] : 0) + inc[1] - v[1];
+    }
+}
+
+// One warp per global q-tile (fwd) or k-tile (bwd): ordered compaction. The
+// fwd list reads its row of the class triangle; the bwd list recomputes its
+// column's classes from the k-tile's statistics (the values k_classify
+// stored), which avoids reading the triangle by columns.
 __global__ void k_fill(BuildArgs a) {
     int64_t g = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
     int lane = threadIdx.x & 31;
@@ -394,9 +515,11 @@ __global__ void k_fill(BuildArgs a) {
     int b = a.tile_traj[g];
     int tb = a.traj_tile[b], nt = a.traj_tile[b + 1] - tb;
     int t = (int)(g - tb);
+    const int T = a.traj_tok[b + 1] - a.traj_tok[b];
     const uint8_t* tri = a.cls + a.traj_tri[b];
     uint32_t lt = (1u << lane) - 1u;
     int base = a.fwd_ptr[g];
+#pragma unroll 4
     for (int k0 = 0; k0 <= t; k0 += 32) {
         int kt = k0 + lane;
         int c = kt <= t ? tri[(int64_t)t * (t + 1) / 2 + kt] : MW_TILE_EMPTY;
@@ -404,26 +527,27 @@ __global__ void k_fill(BuildArgs a) {
         if (c != MW_TILE_EMPTY) a.fwd_idx[base + __popc(m & lt)] = (kt << 4) | c;
         base += __popc(m);
     }
+    // the column's non-EMPTY tiles are exactly the q-tiles t .. qend - 1
+    // (k_bwd_count), so the bwd list is written without compaction
     base = a.bwd_ptr[g];
-    for (int q0 = t; q0 < nt; q0 += 32) {
-        int qt = q0 + lane;
-        int c = qt < nt ? tri[(int64_t)qt * (qt + 1) / 2 + t] : MW_TILE_EMPTY;
-        uint32_t m = __ballot_sync(0xffffffffu, c != MW_TILE_EMPTY);
-        if (c != MW_TILE_EMPTY) a.bwd_idx[base + __popc(m & lt)] = (qt << 4) | c;
-        base += __popc(m);
-    }
+    const int4 st = tile_stat(a.tstat, g);
+    const int qend = max(t + 1, min(nt, (min(st.y, T) + MW_TILE - 1) / MW_TILE));
+    for (int qt = t + lane; qt < qend; qt += 32) a.bwd_idx[base + qt - t] = (qt << 4) | tile_class(qt, t, T, st);
 }
 
-// Compact views: one block per global segment. An exclusive prefix popcount
-// of the segment's view bits, tile by tile, gives every member key its rank in
-// view_s (cpos; -1 for non-members) and the inverse map (csrc: the key at each
-// rank); the total is |view_s|, and csrc is -1 from there to the end of the
-// last 128-entry tile. For a monotone record view_s is in physical order, so
-// the rank is the key's index in the segment's compact sequence (§4.1).
+// Compact views. An exclusive prefix popcount of the segment's view bits,
+// tile by tile, gives every member key its rank in view_s (cpos; -1 for
+// non-members) and the inverse map (csrc: the key at each rank); the total is
+// |view_s|, and csrc is -1 from there to the end of the last 128-entry tile.
+// For a monotone record view_s is in physical order, so the rank is the key's
+// index in the segment's compact sequence (§4.1). One block per (global
+// segment, chunk of 256 k-tiles): the chunk's first rank is the popcount of the
+// segment's earlier tiles; the block holding the segment's last tile writes
+// |view_s| and the tail.
+constexpr int CMAP_TILES = 256;
 __global__ void __launch_bounds__(256) k_compact_map(BuildArgs a) {
     __shared__ int tp[256];
     __shared__ int wsum[8];
-    __shared__ int carry_s;
     const int sg = blockIdx.x;
     int lo = 0, hi = a.n_traj;   // largest b with traj_seg[b] <= sg
     while (hi - lo > 1) {
@@ -433,51 +557,73 @@ __global__ void __launch_bounds__(256) k_compact_map(BuildArgs a) {
     const int b = lo;
     const int s = sg - a.traj_seg[b];
     const int nt = a.traj_tile[b + 1] - a.traj_tile[b];
+    const int c0 = blockIdx.y * CMAP_TILES;
+    if (c0 >= nt) {   // uniform over the block; an empty trajectory's segment has an empty view
+        if (blockIdx.y == 0 && threadIdx.x == 0) a.seg_len[sg] = 0;
+        return;
+    }
     const int64_t ent0 = a.traj_km[b] + (int64_t)s * nt;   // keymask entry of (s, kt = 0)
     const uint32_t* km = a.keymask + ent0 * 4;
     int32_t* pos = a.cpos + ent0 * MW_TILE;
     int32_t* src = a.csrc + ent0 * MW_TILE;
     const int t = threadIdx.x, lane = t & 31, w = t >> 5;
-    if (t == 0) carry_s = 0;
+    auto tile_cnt = [&](int kt) -> int {
+        return __popc(km[4 * kt]) + __popc(km[4 * kt + 1]) + __popc(km[4 * kt + 2]) + __popc(km[4 * kt + 3]);
+    };
+    // first rank of the chunk: members of the segment's tiles 0 .. c0 - 1
+    int before_chunk = 0;
+    for (int kt = t; kt < c0; kt += 256) before_chunk += tile_cnt(kt);
+    before_chunk = warp_sum_i(before_chunk);
+    if (lane == 0) wsum[w] = before_chunk;
     __syncthreads();
-    for (int c0 = 0; c0 < nt; c0 += 256) {
-        const int kt = c0 + t;
-        int cnt = 0;
-        if (kt < nt)
-            cnt = __popc(km[4 * kt]) + __popc(km[4 * kt + 1]) + __popc(km[4 * kt + 2]) + __popc(km[4 * kt + 3]);
-        int incl = cnt;
+    int base = 0;
 #pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const int y = __shfl_up_sync(0xffffffffu, incl, o);
-            if (lane >= o) incl += y;
-        }
-        if (lane == 31) wsum[w] = incl;
-        __syncthreads();
-        int before = carry_s;
-        for (int q = 0; q < w; ++q) before += wsum[q];
-        tp[t] = before + incl - cnt;
-        __syncthreads();
-        const int ntc = min(256, nt - c0);
-        for (int k = t; k < ntc * MW_TILE; k += 256) {
-            const int tl = k >> 7, jj = k & 127, wd = jj >> 5, bit = jj & 31;
-            const uint32_t* tw = km + 4 * (c0 + tl);
-            const uint32_t word = tw[wd];
-            int32_t r = -1;
-            if ((word >> bit) & 1u) {
-                r = tp[tl] + __popc(word & ((1u << bit) - 1u));
-                for (int q = 0; q < wd; ++q) r += __popc(tw[q]);
-                src[r] = (c0 + tl) * MW_TILE + jj;
-            }
-            pos[(int64_t)(c0 + tl) * MW_TILE + jj] = r;
-        }
-        __syncthreads();
-        if (t == 255) carry_s = tp[255] + cnt;
-        __syncthreads();
+    for (int q = 0; q < 8; ++q) base += wsum[q];
+    __syncthreads();
+    const int kt = c0 + t;
+    // this thread's tile: its four view-bit words and their exclusive prefix
+    // counts, kept in shared memory for the element loop below
+    __shared__ uint4 words[CMAP_TILES];
+    __shared__ uint4 wpre[CMAP_TILES];
+    const uint4 wv = kt < nt ? *reinterpret_cast<const uint4*>(km + 4 * kt) : make_uint4(0u, 0u, 0u, 0u);
+    const int c0w = __popc(wv.x), c1w = __popc(wv.y), c2w = __popc(wv.z), c3w = __popc(wv.w);
+    words[t] = wv;
+    wpre[t] = make_uint4(0u, (uint32_t)c0w, (uint32_t)(c0w + c1w), (uint32_t)(c0w + c1w + c2w));
+    const int cnt = c0w + c1w + c2w + c3w;
+    int incl = cnt;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
     }
-    const int len = carry_s;
-    if (t == 0) a.seg_len[sg] = len;
-    const int end = (len + MW_TILE - 1) / MW_TILE * MW_TILE;
-    for (int r = len + t; r < end; r += 256) src[r] = -1;
+    if (lane == 31) wsum[w] = incl;
+    __syncthreads();
+    int before = base;
+    for (int q = 0; q < w; ++q) before += wsum[q];
+    tp[t] = before + incl - cnt;
+    __syncthreads();
+    const int ntc = min(CMAP_TILES, nt - c0);
+    for (int k = t; k < ntc * MW_TILE; k += 256) {
+        const int tl = k >> 7, jj = k & 127, wd = jj >> 5, bit = jj & 31;
+        const uint4 w4 = words[tl], p4 = wpre[tl];
+        const uint32_t word = wd == 0 ? w4.x : wd == 1 ? w4.y : wd == 2 ? w4.z : w4.w;
+        const uint32_t pre = wd == 0 ? p4.x : wd == 1 ? p4.y : wd == 2 ? p4.z : p4.w;
+        int32_t r = -1;
+        if ((word >> bit) & 1u) {
+            r = tp[tl] + (int)pre + __popc(word & ((1u << bit) - 1u));
+            src[r] = (c0 + tl) * MW_TILE + jj;
+        }
+        pos[(int64_t)(c0 + tl) * MW_TILE + jj] = r;
+    }
+    if (c0 + CMAP_TILES >= nt) {   // the block holding the segment's last tile
+        int total = 0;
+#pragma unroll
+        for (int q = 0; q < 8; ++q) total += wsum[q];
+        const int len = base + total;
+        if (t == 0) a.seg_len[sg] = len;
+        const int end = (len + MW_TILE - 1) / MW_TILE * MW_TILE;
+        for (int r = len + t; r < end; r += 256) src[r] = -1;
+    }
 }
 
 // EVENTS records: one block per trajectory replays its events segment by
@@ -657,6 +803,7 @@ extern "C" mw_status mw_build_visibility(const mw_vis_layout* L, const int32_t* 
     if (L->n_spans > 0 && !spans) return MW_EINVAL;
     if (L->vis_bytes > 0 && !vis) return MW_EINVAL;
     if (L->ws_bytes > 0 && !ws) return MW_EINVAL;
+    if (((uintptr_t)vis | (uintptr_t)ws) % 256) return MW_EINVAL;   // arrays sit at 256-byte offsets
     if (n_junc > 0 && (span_off[0] != 0 || span_off[n_junc] != L->n_spans)) return MW_EEDITS;
     // validate junctions and spans (App. B Def. "trajectory tree")
     for (int k = 0; k < n_junc; ++k) {
@@ -720,23 +867,30 @@ extern "C" mw_status mw_build_visibility(const mw_vis_layout* L, const int32_t* 
     a.tstat = at<int32_t>(ws, L->ws_off_tstat);
     a.fwd_cnt = at<int32_t>(ws, L->ws_off_cnt);
     a.bwd_cnt = at<int32_t>(ws, L->ws_off_cnt) + n_tiles;
+    a.tpairs = reinterpret_cast<unsigned long long*>(at<int32_t>(ws, L->ws_off_cnt) + 2 * n_tiles);
+    a.bsum = at<int32_t>(ws, L->ws_off_cnt) + 4 * n_tiles;
 
-    count_launches((a.total > 0 ? 1 + (L->n_spans > 0) : 0) + (n_tiles > 0 ? 3 : 0) + 1 + 2 * (n_tiles > 0));
+    count_launches((a.total > 0 ? 1 + (L->n_spans > 0) : 0) + (n_tiles > 0 ? 3 : 0) + 1 + 4 * (n_tiles > 0));
     if (a.total > 0) {
-        int grid = (int)std::min<int64_t>(ceil_div(a.total, 256), 152 * 16);
+        int grid = (int)std::min<int64_t>(ceil_div(ceil_div(a.total, INIT_TPT), 256), 152 * 16);
         k_init_tokens<<<grid, 256, 0, stream>>>(a);
         if (L->n_spans > 0) k_scatter_spans<<<(int)std::min<int64_t>(L->n_spans, 152 * 8), 256, 0, stream>>>(a);
     }
     if (n_tiles > 0) {
-        k_tile_stats<<<(unsigned)n_tiles, MW_TILE, 0, stream>>>(a);
+        k_tile_stats<<<(unsigned)ceil_div(n_tiles * 32, 256), 256, 0, stream>>>(a);
         unsigned wgrid = (unsigned)ceil_div(n_tiles * 32, 256);
         k_classify<<<wgrid, 256, 0, stream>>>(a);
-        k_bwd_count<<<wgrid, 256, 0, stream>>>(a);
+        k_bwd_count<<<(unsigned)ceil_div(n_tiles, 256), 256, 0, stream>>>(a);
     }
-    k_scan<<<1, 1024, 0, stream>>>(a);
+    {
+        const unsigned nb = (unsigned)ceil_div(n_tiles, (int64_t)SCAN_BLOCK);
+        if (nb > 0) k_scan_sums<<<nb, SCAN_BLOCK, 0, stream>>>(a);
+        k_scan_offsets<<<1, 1024, 0, stream>>>(a, (int)nb);
+        if (nb > 0) k_scan_ptrs<<<nb, SCAN_BLOCK, 0, stream>>>(a);
+    }
     if (n_tiles > 0) {
         k_fill<<<(unsigned)ceil_div(n_tiles * 32, 256), 256, 0, stream>>>(a);
-        k_compact_map<<<(unsigned)L->n_segs, 256, 0, stream>>>(a);
+        k_compact_map<<<dim3((unsigned)L->n_segs, (unsigned)ceil_div(L->max_tiles, CMAP_TILES)), 256, 0, stream>>>(a);
     }
     return launch_status();
 }
@@ -755,6 +909,7 @@ extern "C" mw_status mw_build_views_events(const mw_vis_layout* L, const int32_t
     if (n_spans > 0 && !spans) return MW_EINVAL;
     if (L->vis_bytes > 0 && !vis) return MW_EINVAL;
     if (L->ws_bytes > 0 && !ws) return MW_EINVAL;
+    if (((uintptr_t)vis | (uintptr_t)ws) % 256) return MW_EINVAL;   // arrays sit at 256-byte offsets
     // validate: junctions ascending inside [1, T-1], spans inside [0, J), and
     // every retrieved position out of the view when its event fires (replayed
     // per trajectory on the host, one state byte per position)
@@ -842,7 +997,8 @@ extern "C" mw_status mw_build_views_events(const mw_vis_layout* L, const int32_t
     e.pairs = at<unsigned long long>(vis, L->off_pairs);
     if (a.total > 0) {
         count_launches(1);
-        k_init_tokens<<<(int)std::min<int64_t>(ceil_div(a.total, 256), 152 * 16), 256, 0, stream>>>(a);
+        k_init_tokens<<<(int)std::min<int64_t>(ceil_div(ceil_div(a.total, INIT_TPT), 256), 152 * 16), 256, 0,
+                        stream>>>(a);
     }
     if (n_traj > 0) {
         count_launches(1);

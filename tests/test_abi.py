@@ -93,8 +93,24 @@ def test_build_rejects_bad_records_before_launch(J, spans, off):
                                np.array(J, np.int32).ctypes.data_as(L._IP), jt.ctypes.data_as(L._IP),
                                np.array(off, np.int32).ctypes.data_as(L._IP),
                                sp.ctypes.data_as(L._IP) if sp.size else None,
-                               ctypes.c_void_p(16), ctypes.c_void_p(16), None)
+                               ctypes.c_void_p(256), ctypes.c_void_p(256), None)
     assert st == 2
+
+
+def test_build_rejects_unaligned_buffers_before_launch():
+    """`vis` and `ws` must be 256-byte aligned (the layout's arrays sit at
+    256-byte offsets): a valid record with an unaligned buffer is MW_EINVAL,
+    found on the host before anything could be launched."""
+    L, h = _lib()
+    cu = np.array([0, 10], np.int32)
+    J, jt, off = np.array([5], np.int32), np.zeros(1, np.int32), np.array([0, 1], np.int32)
+    sp = np.array([2, 4], np.int32)
+    lay = L.mw_visibility_layout(cu, jt, 1)
+    for vis, ws in ((16, 256), (256, 16)):
+        st = h.mw_build_visibility(ctypes.byref(lay), cu.ctypes.data_as(L._IP), 1, J.ctypes.data_as(L._IP),
+                                   jt.ctypes.data_as(L._IP), off.ctypes.data_as(L._IP), sp.ctypes.data_as(L._IP),
+                                   ctypes.c_void_p(ws), ctypes.c_void_p(vis), None)
+        assert st == 1
 
 
 def test_attention_and_lmhead_reject_bad_args_on_host():
