@@ -335,25 +335,40 @@ __device__ __forceinline__ int4 tile_stat(const int32_t* tstat, int64_t g) {
     return *reinterpret_cast<const int4*>(tstat + 4 * g);
 }
 
-// One warp per global q-tile: classes of (qt, 0..qt) and the fwd list length.
-__global__ void k_classify(BuildArgs a) {
-    int64_t g = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
-    int lane = threadIdx.x & 31;
-    if (g >= a.n_tiles) return;
-    int b = a.tile_traj[g];
-    int tb = a.traj_tile[b];
-    int qt = (int)(g - tb);
-    int T = a.traj_tok[b + 1] - a.traj_tok[b];
-    uint8_t* row = a.cls + a.traj_tri[b] + (int64_t)qt * (qt + 1) / 2;
+// One warp per q-tile, 32 consecutive q-tiles of one trajectory per block:
+// classes of (qt, 0..qt) and the fwd list length. The trajectory's k-tile
+// statistics pass through shared memory in chunks, so each is read from L2
+// once per block instead of once per q-tile.
+constexpr int CLS_CHUNK = 2048;
+__global__ void __launch_bounds__(1024) k_classify(BuildArgs a) {
+    __shared__ int4 sst[CLS_CHUNK];
+    const int b = blockIdx.x;
+    const int tb = a.traj_tile[b], nt = a.traj_tile[b + 1] - tb;
+    const int q_first = blockIdx.y * 32;
+    if (q_first >= nt) return;   // uniform over the block
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int qt = q_first + warp;
+    const bool live = qt < nt;
+    const int T = a.traj_tok[b + 1] - a.traj_tok[b];
+    const int q_last = min(nt, q_first + 32) - 1;
+    uint8_t* row = a.cls + a.traj_tri[b] + (live ? (int64_t)qt * (qt + 1) / 2 : 0);
     int cnt = 0;
-#pragma unroll 4
-    for (int kt = lane; kt <= qt; kt += 32) {
-        int c = tile_class(qt, kt, T, tile_stat(a.tstat, tb + kt));
-        row[kt] = (uint8_t)c;
-        cnt += c != MW_TILE_EMPTY;
+    for (int kc = 0; kc <= q_last; kc += CLS_CHUNK) {
+        const int kn = min(CLS_CHUNK, q_last + 1 - kc);
+        __syncthreads();   // the previous chunk is consumed
+        for (int k = threadIdx.x; k < kn; k += blockDim.x) sst[k] = tile_stat(a.tstat, tb + kc + k);
+        __syncthreads();
+        if (live) {
+            const int kend = min(qt + 1, kc + kn);
+            for (int kt = kc + lane; kt < kend; kt += 32) {
+                const int c = tile_class(qt, kt, T, sst[kt - kc]);
+                row[kt] = (uint8_t)c;
+                cnt += c != MW_TILE_EMPTY;
+            }
+        }
     }
     cnt = warp_sum_i(cnt);
-    if (lane == 0) a.fwd_cnt[g] = cnt;
+    if (live && lane == 0) a.fwd_cnt[tb + qt] = cnt;
 }
 
 // One thread per global k-tile: bwd list length, the non-EMPTY tiles of its
@@ -878,8 +893,7 @@ extern "C" mw_status mw_build_visibility(const mw_vis_layout* L, const int32_t* 
     }
     if (n_tiles > 0) {
         k_tile_stats<<<(unsigned)ceil_div(n_tiles * 32, 256), 256, 0, stream>>>(a);
-        unsigned wgrid = (unsigned)ceil_div(n_tiles * 32, 256);
-        k_classify<<<wgrid, 256, 0, stream>>>(a);
+        k_classify<<<dim3((unsigned)L->n_traj, (unsigned)ceil_div(L->max_tiles, 32)), 1024, 0, stream>>>(a);
         k_bwd_count<<<(unsigned)ceil_div(n_tiles, 256), 256, 0, stream>>>(a);
     }
     {
