@@ -23,7 +23,6 @@ mw_status attn_bwd_tc(const mw_vis_layout*, const void*, const void*, const void
                       const float* = nullptr);
 int64_t attn_fwd_tc_ws(const mw_vis_layout*, int);
 int64_t attn_bwd_tc_ws(const mw_vis_layout*, int, int);
-int64_t attn_lsd_ws(const mw_vis_layout*, int);
 mw_status attn_delta(const mw_vis_layout*, const void*, const void*, int, int, int, float*, cudaStream_t);
 mw_status attn_fwd_simt_segk(const mw_vis_layout*, const void*, const void*, const void*, const void*, void*, float*,
                              int, int, int, int, float, cudaStream_t);
@@ -38,10 +37,6 @@ mw_status rope_segments(const mw_vis_layout*, const void*, const int32_t*, const
                         int, int, int, cudaStream_t);
 mw_status rope_segments_bwd(const mw_vis_layout*, const void*, const int32_t*, const float*, int, const float*,
                             void*, int, int, int, bool, cudaStream_t);
-mw_status attn_fwd_tc_segk(const mw_vis_layout*, const void*, const void*, const void*, const void*, void*, float*,
-                           int, int, float, cudaStream_t);
-mw_status attn_bwd_tc_segk(const mw_vis_layout*, const void*, const void*, const void*, const void*, const void*,
-                           const void*, const float*, void*, float*, float*, int, int, float, float*, cudaStream_t);
 __global__ void k_loss_epilogue(int, const float*, const float*, const float*, float, float, const float*, float, float*,
                                 float*, float*);
 __global__ void k_logdiff(int, const float*, const float*, float*);
@@ -262,12 +257,13 @@ extern "C" mw_status mw_logprob_check_status(int N, int M, int d, int V, int dty
 // plain attention's.
 static bool rope_tc(int Dh, int dtype) { return dtype == MW_BF16 && Dh == 128; }
 
-// Byte offsets inside the rotary-attention workspace: rotated queries, the
-// segment key rows, then (backward only) Delta (tensor-core path: the
-// (-LSE log2 e, Delta) pair array), the float32 gradient of the segment key
-// rows and (tensor-core path) the float32 per-segment dV partials.
+// Byte offsets inside the rotary-attention workspace. Tensor-core path: the
+// rotated queries, then the compact attention's own workspace (its keys are
+// turned by rank as they are gathered). CUDA-core path: the rotated queries,
+// the segment key rows, then (backward only) Delta and the float32 gradient
+// of the segment key rows.
 struct RopeWs {
-    int64_t q, kseg, delta, dkseg, dvseg, fwd_bytes, bwd_bytes;
+    int64_t q, kseg, delta, dkseg, fwd_bytes, bwd_bytes;
 };
 static RopeWs rope_ws_layout(const mw_vis_layout* L, int Hq, int Hkv, int Dh, int dtype) {
     RopeWs w;
@@ -277,7 +273,7 @@ static RopeWs rope_ws_layout(const mw_vis_layout* L, int Hq, int Hkv, int Dh, in
     int64_t o = 0;
     if (tc) {   // rotated queries, then the compact attention's own workspace (keys rotated by rank)
         w.q = o; o = align256(o + esz * L->total_tokens * Hq * Dh);
-        w.kseg = w.delta = w.dkseg = w.dvseg = o;
+        w.kseg = w.delta = w.dkseg = o;
         w.fwd_bytes = o + attn_fwd_tc_ws(L, Hkv);
         w.bwd_bytes = o + attn_bwd_tc_ws(L, Hq, Hkv);
         return w;
@@ -285,9 +281,8 @@ static RopeWs rope_ws_layout(const mw_vis_layout* L, int Hq, int Hkv, int Dh, in
     w.q = o; o = align256(o + esz * L->total_tokens * Hq * Dh);
     w.kseg = o; o = align256(o + esz * krows * Hkv * Dh);
     w.fwd_bytes = o;
-    w.delta = o; o = align256(o + (tc ? attn_lsd_ws(L, Hq) : 4 * L->total_tokens * Hq));
+    w.delta = o; o = align256(o + 4 * L->total_tokens * Hq);
     w.dkseg = o; o = align256(o + 4 * krows * Hkv * Dh);
-    w.dvseg = o; o = align256(o + (tc ? 4 * krows * Hkv * Dh : 0));
     w.bwd_bytes = o;
     return w;
 }

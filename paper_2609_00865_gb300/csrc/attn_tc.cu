@@ -1170,9 +1170,9 @@ __global__ void __launch_bounds__(NT_BWD, 1)
 
 }  // namespace
 
-// Rows of segment key rows (keys per segment) and whether TMA's int32 row
-// coordinates and the junction-item grid reach them.
-static bool segk_fits(const mw_vis_layout* L, int Hq) {
+// Whether TMA's int32 row coordinates reach every compact K / V row (128 per
+// (segment, k-tile) entry) and the junction-item and dK/dV grids fit.
+static bool cmp_fits(const mw_vis_layout* L, int Hq) {
     return L->n_keymask * 128 <= INT32_MAX && L->n_segs * (int64_t)Hq <= INT32_MAX && L->max_segs <= 65535;
 }
 
@@ -1366,11 +1366,11 @@ __global__ void __launch_bounds__(256) k_cmp_reduce(VisView v, int Hkv, const fl
 // each segment uses its first ceil(|view_s| / 128) tiles.
 static int64_t cmp_rows(const mw_vis_layout* L) { return L->n_keymask * 128; }
 
-// The (-LSE2, Delta) pair array alone (the rotary path's backward).
-int64_t attn_lsd_ws(const mw_vis_layout* L, int Hq) { return 8 * L->n_tiles * 128 * (int64_t)Hq; }
-
+// Forward workspace: the compact K and V (bf16).
 int64_t attn_fwd_tc_ws(const mw_vis_layout* L, int Hkv) { return align256(4 * cmp_rows(L) * Hkv * DH); }
 
+// Backward workspace: the (-LSE2, Delta) pair array, the compact K and V, and
+// the float32 dK / dV partials per compact row.
 int64_t attn_bwd_tc_ws(const mw_vis_layout* L, int Hq, int Hkv) {
     return align256(8 * L->n_tiles * 128 * (int64_t)Hq) + attn_fwd_tc_ws(L, Hkv) +
            align256(8 * cmp_rows(L) * Hkv * DH);
@@ -1391,7 +1391,7 @@ static mw_status cmp_gather(const mw_vis_layout* L, const VisView& v, int Hkv, c
 mw_status attn_fwd_tc(const mw_vis_layout* L, const void* vis, const void* Q, const void* K, const void* V, void* O,
                       float* LSE, int Hq, int Hkv, float scale, void* ws, cudaStream_t s, const float* table) {
     if (L->n_tiles == 0) return MW_OK;
-    if (!segk_fits(L, Hq)) return MW_ESHAPE;
+    if (!cmp_fits(L, Hq)) return MW_ESHAPE;
     const VisView view = make_view(L, vis);
     const int64_t KR = cmp_rows(L);
     void* Kc = ws;
@@ -1433,7 +1433,7 @@ mw_status attn_bwd_tc(const mw_vis_layout* L, const void* vis, const void* Q, co
                       const void* O, const void* dO, const float* LSE, void* dQ, void* dK, void* dV, int Hq, int Hkv,
                       float scale, void* ws, cudaStream_t s, const float* table) {
     if (L->n_tiles == 0) return MW_OK;
-    if (!segk_fits(L, Hq)) return MW_ESHAPE;
+    if (!cmp_fits(L, Hq)) return MW_ESHAPE;
     const int64_t n_rows = L->n_tiles * 128;
     const int64_t KR = cmp_rows(L);
     float* lsd = reinterpret_cast<float*>(ws);
