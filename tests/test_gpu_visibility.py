@@ -95,3 +95,14 @@ def test_bad_record_raises():
     with pytest.raises(mw.MWError) as e:
         mw.build_visibility([50], [[(10, [(5, 12)])]])
     assert e.value.status == 2
+
+
+def test_many_tiles_and_long_trajectory():
+    """More tiles than one scan block (1,024) and a trajectory longer than
+    one shared-memory chunk of k-tile statistics (2,048 tiles): the
+    multi-block list-pointer scan, the chunked class pass and several
+    256-tile compact-map chunks per segment, against the oracle."""
+    c = synth.CONFIGS[5]
+    r = synth.record(4, [300_000, 70_000, 0, 140_000], 6, 0.6, c["summary"], c["prompt"], c["Lp"], c["Lo"], 7700)
+    assert sum((T + 127) // 128 for T in r.seqlens) > 3 * 1024
+    _compare(r.seqlens, r.edits)
