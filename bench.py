@@ -803,6 +803,7 @@ def run_builder(args, rank, world, local_rank):
     compact tile, which stay unspecified). The record is host data by the builder's API (the
     call packs it and uploads the span list), so the timed call includes that
     upload: ``value`` and ``e2e`` are the same measurement."""
+    import numpy as np
     import torch
 
     import paper_2609_00865_gb300 as mw
@@ -843,7 +844,31 @@ def run_builder(args, rank, world, local_rank):
     ms = reduce_max(e0.elapsed_time(e1) / args.steps, world, dev)
     if rank != 0:
         return
-    import numpy as np
+    # dense-mask export (bit-packed T x T per trajectory; T^2 / 8 bytes written)
+    # of the attention workload's record, 8 trajectories of 16,384 tokens
+    r2 = synth.config_record(2)
+    vis2 = mw.build_visibility(r2.seqlens, r2.edits)
+    masks = [torch.empty(T * ((T + 31) // 32), dtype=torch.int32, device=dev) for T in r2.seqlens]
+    cu2 = np.zeros(len(r2.seqlens) + 1, dtype=np.int32)
+    cu2[1:] = np.cumsum(r2.seqlens)
+
+    def export_all():
+        for b, m in enumerate(masks):
+            mw.mw_export_dense_mask(vis2, cu2, b, m, stream)
+
+    for _ in range(args.warmup):
+        export_all()
+    torch.cuda.synchronize()
+    m0 = torch.cuda.Event(enable_timing=True)
+    m1 = torch.cuda.Event(enable_timing=True)
+    m0.record(stream)
+    for _ in range(args.steps):
+        export_all()
+    m1.record(stream)
+    torch.cuda.synchronize()
+    mask_ms = m0.elapsed_time(m1) / args.steps
+    mask_bytes = sum(m.numel() * 4 for m in masks)
+
     n_spans = int(L.n_spans)
     # written: the whole structure except csrc past each segment's last compact
     # tile (left unspecified); read: the packed span list and the small tables
@@ -871,6 +896,10 @@ def run_builder(args, rank, world, local_rank):
                 "note": "host record in, device structure out: the timed call packs and uploads the record"},
         "gpu_launches": launches,
         "clocks": clk,
+        "dense_mask_export": {"workload": "8 x 16384-token trajectories of the attention workload",
+                              "ms": mask_ms, "bytes_written": mask_bytes,
+                              "gbs": mask_bytes / (mask_ms * 1e-3) / 1e9,
+                              "frac_of_copy_peak": mask_bytes / (mask_ms * 1e-3) / 1e9 / hbm},
     }
     print(json.dumps(line), flush=True)
 

@@ -507,6 +507,23 @@ mw_status mw_logdiff(const float* lp_train, const float* lp_rollout, int M, floa
 mw_status mw_check_status(const mw_vis_layout* layout, const void* vis, void* stream);
 
 /*
+ * Dense visibility of trajectory `traj`, bit-packed (Eq. 7's 4D mask, for
+ * checking against a dense-mask implementation on small trajectories): row i
+ * sees key j iff j is in the live view of i's segment at or before i's own
+ * place in it -- j <= i and j in view_s for an edits record, the view-order
+ * prefix for an offload / retrieve record (§4.1: the row attends to its
+ * segment's compact sequence up to itself).
+ *   cu_seqlens[n_traj+1]  host int32, the record's offsets (as for the build)
+ *   mask                  device uint32 [T][ceil(T / 32)], T = the trajectory's
+ *                         length; bit k of word w of row i is key 32 w + k
+ * T > MW_DENSE_MASK_MAX_T is MW_ESHAPE (the mask is T^2 / 8 bytes); T = 0
+ * writes nothing. Reads only `vis`; asynchronous on `stream`.
+ */
+#define MW_DENSE_MASK_MAX_T 65536
+mw_status mw_export_dense_mask(const mw_vis_layout* layout, const void* vis, const int32_t* cu_seqlens, int traj,
+                               uint32_t* mask, void* stream);
+
+/*
  * Status of the last mw_logprob_loss_fwd / mw_logprob_loss_bwd on `ws` (same
  * shape arguments): synchronises `stream`, then returns MW_ETIMEOUT if a
  * tensor-core kernel gave up a bounded wait, else MW_OK. No counterpart in the

@@ -82,6 +82,7 @@ _SIGS = {
     "mw_masked_attn_rope_bwd": (_I, [_LP, _P, _P, _P, _I, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _F,
                                      _P, _P]),
     "mw_check_status": (_I, [_LP, _P, _P]),
+    "mw_export_dense_mask": (_I, [_LP, _P, _IP, _I, _P, _P]),
     "mw_logprob_check_status": (_I, [_I, _I, _I, _I, _I, _P, _P]),
     "mw_selftest_wait_timeout": (_I, [ctypes.c_int64, _P, _P]),
 }
@@ -329,6 +330,29 @@ def build_visibility(seqlens, edits_per_traj, device="cuda", stream=None):
     ws = torch.empty(max(int(L.ws_bytes), 1), dtype=torch.uint8, device=device)
     mw_build_visibility(L, cu, J, jt, off, spans, ws, vis, stream)
     return Visibility(L, vis, ws)
+
+
+def mw_export_dense_mask(vis, cu_seqlens, traj, mask, stream=None):
+    cu, cup = _i32(cu_seqlens)
+    _check(_lib().mw_export_dense_mask(ctypes.byref(vis.layout), _ptr(vis.vis), cup, int(traj), _ptr(mask),
+                                       _stream(stream)), "mw_export_dense_mask")
+
+
+def export_dense_mask(vis, seqlens, traj, stream=None):
+    """Trajectory ``traj``'s dense visibility as a bool tensor [T, T] on the
+    device (mw_export_dense_mask, bit-packed words unpacked here). Row i sees
+    key j iff j is in the live view of i's segment at or before i's own place
+    in it; for small trajectories only."""
+    import torch
+    cu = np.zeros(len(seqlens) + 1, dtype=np.int32)
+    cu[1:] = np.cumsum(seqlens)
+    T = int(seqlens[traj])
+    words = (T + 31) // 32
+    mask = torch.zeros(max(T * words, 1), dtype=torch.int32, device=vis.vis.device)
+    mw_export_dense_mask(vis, cu, traj, mask, stream)
+    bits = torch.arange(32, dtype=torch.int32, device=mask.device)
+    dense = ((mask[: T * words].view(T, words, 1) >> bits) & 1).bool().view(T, words * 32)
+    return dense[:, :T]
 
 
 # --- branch-replicated packing (stacked layers) --------------------------------

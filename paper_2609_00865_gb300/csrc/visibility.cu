@@ -641,6 +641,42 @@ __global__ void __launch_bounds__(256) k_compact_map(BuildArgs a) {
     }
 }
 
+// Dense visibility of one trajectory, bit-packed (the 4D mask of Eq. 7 for
+// small T, for comparing with a dense-mask implementation): row i sees key j
+// iff j is in the view of i's segment at or before i's own place in it, i.e.
+// 0 <= cpos_s(j) <= cpos_s(i). That is j <= i and j in view_s for a monotone
+// record, and the view-order prefix for offload / retrieve views. One block
+// per row; a thread writes 32-key words, reading the 32 keys' ranks as eight
+// 16-byte loads.
+__global__ void __launch_bounds__(256) k_dense_mask(VisView v, int b, int T, int words, uint32_t* __restrict__ mask) {
+    const int i = blockIdx.x;
+    const int64_t tok0 = v.traj_tok[b];
+    const int nt = v.traj_tile[b + 1] - v.traj_tile[b];
+    const int s = v.seg[tok0 + i];
+    const int32_t* cp = v.cpos + (v.traj_km[b] + (int64_t)s * nt) * MW_TILE;   // key j at cp[j]
+    const int ci = cp[i];
+    for (int w = threadIdx.x; w < words; w += blockDim.x) {
+        uint32_t bits = 0u;
+        const int j0 = 32 * w;
+        if (j0 + 32 <= T) {
+            const int4* c4 = reinterpret_cast<const int4*>(cp + j0);
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                const int4 c = c4[q];
+                bits |= (uint32_t)(c.x >= 0 && c.x <= ci) << (4 * q) | (uint32_t)(c.y >= 0 && c.y <= ci) << (4 * q + 1) |
+                        (uint32_t)(c.z >= 0 && c.z <= ci) << (4 * q + 2) | (uint32_t)(c.w >= 0 && c.w <= ci) << (4 * q + 3);
+            }
+        } else {
+            for (int k = 0; j0 + k < T; ++k) {
+                const int c = cp[j0 + k];
+                bits |= (uint32_t)(c >= 0 && c <= ci) << k;
+            }
+        }
+        mask[(int64_t)i * words + w] = bits;
+    }
+}
+
+
 // EVENTS records: one block per trajectory replays its events segment by
 // segment into the compact views. view_s = (view_{s-1} without the event's
 // out-spans, order kept) + the in-spans in the given order + the segment's
@@ -1036,4 +1072,19 @@ extern "C" mw_status mw_check_status(const mw_vis_layout* L, const void* vis, vo
     if (h[ST_TIMEOUT]) return MW_ETIMEOUT;
     if (h[ST_BOUNDS]) return MW_EDEVICE;
     return MW_OK;
+}
+
+extern "C" mw_status mw_export_dense_mask(const mw_vis_layout* L, const void* vis, const int32_t* cu_seqlens,
+                                          int traj, uint32_t* mask, void* stream) {
+    if (!L || !cu_seqlens) return MW_EINVAL;
+    if (traj < 0 || traj >= L->n_traj || cu_seqlens[L->n_traj] != L->total_tokens) return MW_EINVAL;
+    const int64_t T = (int64_t)cu_seqlens[traj + 1] - cu_seqlens[traj];
+    if (T < 0) return MW_EINVAL;
+    if (T == 0) return MW_OK;
+    if (T > MW_DENSE_MASK_MAX_T) return MW_ESHAPE;
+    if (!vis || !mask) return MW_EINVAL;
+    count_launches(1);
+    k_dense_mask<<<(unsigned)T, 256, 0, (cudaStream_t)stream>>>(make_view(L, vis), traj, (int)T, (int)((T + 31) / 32),
+                                                                mask);
+    return launch_status();
 }

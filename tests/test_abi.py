@@ -266,3 +266,18 @@ def test_c_program_links_and_calls_the_abi(tmp_path):
     assert run.returncode == 0, (run.returncode, run.stderr)
     ver, n_keymask = map(int, run.stdout.split())
     assert ver >= 4 and n_keymask == (1 + 0) * 3 + (1 + 2) * 6
+
+
+def test_dense_mask_export_rejects_bad_args_on_host():
+    L, h = _lib()
+    cu = np.array([0, 10, 70000], np.int32)
+    lay = L.mw_visibility_layout(cu, np.zeros(0, np.int32), 0)
+    P = ctypes.c_void_p(256)
+    cup = cu.ctypes.data_as(L._IP)
+    assert h.mw_export_dense_mask(ctypes.byref(lay), P, cup, 1, P, None) == 3      # T > MW_DENSE_MASK_MAX_T
+    assert h.mw_export_dense_mask(ctypes.byref(lay), P, cup, -1, P, None) == 1     # no such trajectory
+    assert h.mw_export_dense_mask(ctypes.byref(lay), P, cup, 2, P, None) == 1
+    assert h.mw_export_dense_mask(ctypes.byref(lay), P, None, 0, P, None) == 1     # offsets missing
+    assert h.mw_export_dense_mask(ctypes.byref(lay), P, cup, 0, None, None) == 1   # mask missing
+    bad = np.array([0, 10, 60000], np.int32)                                       # offsets of another record
+    assert h.mw_export_dense_mask(ctypes.byref(lay), P, bad.ctypes.data_as(L._IP), 0, P, None) == 1

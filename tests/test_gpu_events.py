@@ -154,3 +154,18 @@ def test_rotary_attention_on_event_views():
     assert_grad_bf16(np64(dQ), dQr, "dQ")
     assert_grad_bf16(np64(dK), dKr, "dK")
     assert_grad_bf16(np64(dV), dVr, "dV")
+
+
+def test_dense_mask_export_on_event_views():
+    """mw_export_dense_mask on offload / retrieve views against both oracle
+    formulations of their dense mask (view order, and the per-key replay)."""
+    import paper_2609_00865_gb300 as mw
+    rng = np.random.default_rng(4100)
+    T0, ev0 = _panel()
+    seqlens = [T0] + [int(rng.integers(300, 1500)) for _ in range(2)]
+    events = [ev0] + [_memex_record(rng, T, int(rng.integers(1, 6))) for T in seqlens[1:]]
+    vis = _compare(seqlens, events)
+    for b, (T, e) in enumerate(zip(seqlens, events)):
+        got = mw.export_dense_mask(vis, seqlens, b).cpu().numpy()
+        np.testing.assert_array_equal(got, N.dense_mask(T, e), err_msg=f"trajectory {b}")
+        np.testing.assert_array_equal(got, N.replay_mask(T, e), err_msg=f"trajectory {b} (replay)")

@@ -106,3 +106,31 @@ def test_many_tiles_and_long_trajectory():
     r = synth.record(4, [300_000, 70_000, 0, 140_000], 6, 0.6, c["summary"], c["prompt"], c["Lp"], c["Lo"], 7700)
     assert sum((T + 127) // 128 for T in r.seqlens) > 3 * 1024
     _compare(r.seqlens, r.edits)
+
+
+def _mask_case(seqlens, edits):
+    import torch
+    import paper_2609_00865_gb300 as mw
+    vis = mw.build_visibility(seqlens, edits)
+    for b, (T, e) in enumerate(zip(seqlens, edits)):
+        got = mw.export_dense_mask(vis, seqlens, b)
+        torch.cuda.synchronize()
+        want = OV.dense_mask(T, e)
+        np.testing.assert_array_equal(got.cpu().numpy(), want, err_msg=f"trajectory {b}")
+
+
+def test_dense_mask_export_running_example_and_random():
+    """mw_export_dense_mask against the oracle's literal dense mask (list
+    membership of each row's live view, causal), bit for bit."""
+    g = json.load(open(os.path.join(os.path.dirname(__file__), "golden", "running_example.json")))
+    _mask_case([14], [[(J, [tuple(s) for s in sp]) for J, sp in g["edits"]]])
+    rng = np.random.default_rng(11)
+    for _ in range(4):
+        _mask_case(*_rand_record(rng, int(rng.integers(1, 5))))
+    _mask_case([300, 0, 129], [[(100, [(0, 50)])], [], [(5, [(1, 3)])]])
+
+
+def test_dense_mask_export_config2_trajectory():
+    """One 16,384-token trajectory of the attention workload (32 MB of bits)."""
+    r = synth.config_record(2)
+    _mask_case(r.seqlens[:1], r.edits[:1])
