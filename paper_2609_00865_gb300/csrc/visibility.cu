@@ -643,39 +643,57 @@ __global__ void __launch_bounds__(256) k_compact_map(BuildArgs a) {
 
 // Dense visibility of one trajectory, bit-packed (the 4D mask of Eq. 7 for
 // small T, for comparing with a dense-mask implementation): row i sees key j
-// iff j is in the view of i's segment at or before i's own place in it, i.e.
-// 0 <= cpos_s(j) <= cpos_s(i). That is j <= i and j in view_s for a monotone
-// record, and the view-order prefix for offload / retrieve views. One block
-// per row; a thread writes 32-key words, reading the 32 keys' ranks as eight
-// 16-byte loads.
-__global__ void __launch_bounds__(256) k_dense_mask(VisView v, int b, int T, int words, uint32_t* __restrict__ mask) {
-    const int i = blockIdx.x;
+// iff j is in the view of i's segment at or before i's own place in it. For an
+// edits record the view is in physical order, so that is the segment's
+// view-bit word cut at j <= i; for offload / retrieve views it is 0 <=
+// cpos_s(j) <= cpos_s(i), from the 32 keys' ranks (eight 16-byte loads).
+// DM_ROWS rows per block (their segment ids loaded up front, independently),
+// a thread per 32-key word.
+constexpr int DM_ROWS = 8;
+__global__ void __launch_bounds__(256) k_dense_mask(VisView v, int b, int T, int words, int by_rank,
+                                                    uint32_t* __restrict__ mask) {
+    const int i0 = blockIdx.x * DM_ROWS;
     const int64_t tok0 = v.traj_tok[b];
     const int nt = v.traj_tile[b + 1] - v.traj_tile[b];
-    const int s = v.seg[tok0 + i];
-    const int32_t* cp = v.cpos + (v.traj_km[b] + (int64_t)s * nt) * MW_TILE;   // key j at cp[j]
-    const int ci = cp[i];
-    for (int w = threadIdx.x; w < words; w += blockDim.x) {
-        uint32_t bits = 0u;
-        const int j0 = 32 * w;
-        if (j0 + 32 <= T) {
-            const int4* c4 = reinterpret_cast<const int4*>(cp + j0);
+    const int64_t km0 = v.traj_km[b];
+    int sr[DM_ROWS];
 #pragma unroll
-            for (int q = 0; q < 8; ++q) {
-                const int4 c = c4[q];
-                bits |= (uint32_t)(c.x >= 0 && c.x <= ci) << (4 * q) | (uint32_t)(c.y >= 0 && c.y <= ci) << (4 * q + 1) |
-                        (uint32_t)(c.z >= 0 && c.z <= ci) << (4 * q + 2) | (uint32_t)(c.w >= 0 && c.w <= ci) << (4 * q + 3);
+    for (int r = 0; r < DM_ROWS; ++r) sr[r] = i0 + r < T ? v.seg[tok0 + i0 + r] : 0;
+#pragma unroll
+    for (int r = 0; r < DM_ROWS; ++r) {
+        const int i = i0 + r;
+        if (i >= T) break;   // uniform over the block
+        const int64_t ent0 = km0 + (int64_t)sr[r] * nt;        // (segment, k-tile 0) entry
+        const int32_t* cp = v.cpos + ent0 * MW_TILE;           // key j's rank at cp[j]
+        const uint32_t* km = v.keymask + ent0 * 4;             // key j's view bit: word j / 32
+        const int ci = by_rank ? cp[i] : 0;
+        for (int w = threadIdx.x; w < words; w += blockDim.x) {
+            const int j0 = 32 * w;
+            uint32_t bits = 0u;
+            if (!by_rank) {
+                if (j0 <= i) {
+                    const int hi = i - j0;   // keys j0 .. j0 + hi are at or before i
+                    bits = km[w] & (hi >= 31 ? 0xffffffffu : ((2u << hi) - 1u));
+                }
+            } else if (j0 + 32 <= T) {
+                const int4* c4 = reinterpret_cast<const int4*>(cp + j0);
+#pragma unroll
+                for (int q = 0; q < 8; ++q) {
+                    const int4 c = c4[q];
+                    bits |= (uint32_t)(c.x >= 0 && c.x <= ci) << (4 * q) | (uint32_t)(c.y >= 0 && c.y <= ci) << (4 * q + 1) |
+                            (uint32_t)(c.z >= 0 && c.z <= ci) << (4 * q + 2) |
+                            (uint32_t)(c.w >= 0 && c.w <= ci) << (4 * q + 3);
+                }
+            } else {
+                for (int k = 0; j0 + k < T; ++k) {
+                    const int c = cp[j0 + k];
+                    bits |= (uint32_t)(c >= 0 && c <= ci) << k;
+                }
             }
-        } else {
-            for (int k = 0; j0 + k < T; ++k) {
-                const int c = cp[j0 + k];
-                bits |= (uint32_t)(c >= 0 && c <= ci) << k;
-            }
+            mask[(int64_t)i * words + w] = bits;
         }
-        mask[(int64_t)i * words + w] = bits;
     }
 }
-
 
 // EVENTS records: one block per trajectory replays its events segment by
 // segment into the compact views. view_s = (view_{s-1} without the event's
@@ -1084,7 +1102,7 @@ extern "C" mw_status mw_export_dense_mask(const mw_vis_layout* L, const void* vi
     if (T > MW_DENSE_MASK_MAX_T) return MW_ESHAPE;
     if (!vis || !mask) return MW_EINVAL;
     count_launches(1);
-    k_dense_mask<<<(unsigned)T, 256, 0, (cudaStream_t)stream>>>(make_view(L, vis), traj, (int)T, (int)((T + 31) / 32),
-                                                                mask);
+    k_dense_mask<<<(unsigned)ceil_div(T, DM_ROWS), 256, 0, (cudaStream_t)stream>>>(
+        make_view(L, vis), traj, (int)T, (int)((T + 31) / 32), L->kind != MW_VIEWS_EDITS, mask);
     return launch_status();
 }
