@@ -54,7 +54,7 @@ extern "C" const char* mw_status_str(int s) {
 }
 
 extern "C" int mw_last_cuda_error(void) { return g_last_cuda_error; }
-extern "C" int mw_abi_version(void) { return 5; }
+extern "C" int mw_abi_version(void) { return 6; }
 extern "C" uint64_t mw_kernel_launches(void) { return (uint64_t)g_launches.load(std::memory_order_relaxed); }
 
 static mw_status check_shape(int n_traj, const int32_t* cu, int n_junc, const int32_t* jt,
