@@ -73,6 +73,14 @@ const char* mw_status_str(int status);
 int mw_last_cuda_error(void);
 /* ABI version of this header (bumped on any signature or layout change). */
 int mw_abi_version(void);
+/* How this library was built: MW_BUILD_DEBUG set for libmw_debug.so, whose
+ * kernels check the indices they read from memory (a record's spans, the
+ * compact maps, segment tables, tile lists) against the arrays they address;
+ * an index out of range is not followed and the status check of the call
+ * (mw_check_status for the visibility-based calls) reports MW_EDEVICE. The
+ * arithmetic is the release library's. */
+#define MW_BUILD_DEBUG 1
+int mw_build_flags(void);
 /* Number of CUDA kernels this library has launched in this process so far
  * (all threads, all devices); lets callers count launches in a timed region. */
 uint64_t mw_kernel_launches(void);
@@ -408,8 +416,12 @@ mw_status mw_forward_kl_bwd(const void* HT, const int32_t* rows_T, const void* H
                             const void* W, int N_T, int N_S, int d, int Vocab, int dtype, float lam, float dloss,
                             int accumulate, void* ws, void* dHS, float* dW, void* stream);
 
-/* Synchronise `stream` and report a bounded device wait of the tensor-core
- * KL passes that gave up (MW_ETIMEOUT), from `ws`. */
+/* Synchronise `stream` and report, from `ws`, the last mw_forward_kl_fwd /
+ * mw_forward_kl_bwd on it: MW_ETIMEOUT if a bounded device wait of the
+ * tensor-core passes gave up, MW_EDEVICE if a pair's row index lay outside
+ * [0, N_T) (rows_T) or [0, N_S) (rows_S), else MW_OK. Such a row is never
+ * read or written (it counts as a zero row); the call's other outputs are
+ * then unspecified. */
 mw_status mw_forward_kl_check_status(int M, int d, int Vocab, int dtype, void* ws, void* stream);
 
 /*
@@ -445,6 +457,8 @@ mw_status mw_logprob_ws(int N, int M, int d, int Vocab, int dtype, size_t* ws_by
  * (App. B.4 "Pitfall A, RL view" ratio; PPO/GRPO clipping, App. F.1).
  *   H [N, d], W [Vocab, d] (dtype; W in torch Linear layout); targets[N],
  *   rows[M] distinct physical rows (int32, device); lp_old, adv [M] float32.
+ *   An index out of range (rows[m] outside [0, N), a target outside
+ *   [0, Vocab)) is not followed; mw_logprob_check_status reports it.
  *   Outputs lp, ratio, lse [M] float32, loss: one float32 (device).
  * `ws` (mw_logprob_ws bytes) keeps dL/dlp per row for the backward.
  * M = 0 is allowed: the loss is 0 (and the backward writes zero gradients).
@@ -526,8 +540,13 @@ mw_status mw_export_dense_mask(const mw_vis_layout* layout, const void* vis, con
 /*
  * Status of the last mw_logprob_loss_fwd / mw_logprob_loss_bwd on `ws` (same
  * shape arguments): synchronises `stream`, then returns MW_ETIMEOUT if a
- * tensor-core kernel gave up a bounded wait, else MW_OK. No counterpart in the
- * paper: failure detection of this implementation.
+ * tensor-core kernel gave up a bounded wait, MW_EDEVICE if some rows[m] lay
+ * outside [0, N) or its target outside [0, Vocab), else MW_OK. rows and
+ * targets are device arrays no host check sees: the kernels read each index
+ * once, never follow one out of range (that row reads as zero and its dH row
+ * is not written), and raise this flag; lp, lse, the loss and the gradients
+ * are then unspecified. No counterpart in the paper: failure detection of
+ * this implementation.
  */
 mw_status mw_logprob_check_status(int N, int M, int d, int Vocab, int dtype, const void* ws, void* stream);
 

@@ -12,7 +12,10 @@ import os
 import numpy as np
 
 HERE = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(HERE, "libmw.so")
+# MW_DEBUG=1 in the environment selects the debug library (index checks in
+# the kernels; build.build(debug=True) makes it)
+DEBUG = os.environ.get("MW_DEBUG") == "1"
+LIB_PATH = os.path.join(HERE, "libmw_debug.so" if DEBUG else "libmw.so")
 
 MW_F32, MW_BF16 = 0, 1
 TILE = 128
@@ -49,6 +52,7 @@ _SIGS = {
     "mw_status_str": (ctypes.c_char_p, [_I]),
     "mw_last_cuda_error": (_I, []),
     "mw_abi_version": (_I, []),
+    "mw_build_flags": (_I, []),
     "mw_kernel_launches": (ctypes.c_uint64, []),
     "mw_visibility_layout": (_I, [_I, _IP, _I, _IP, _I, _LP]),
     "mw_build_visibility": (_I, [_LP, _IP, _I, _IP, _IP, _IP, _IP, _P, _P, _P]),
@@ -94,7 +98,7 @@ def _lib():
     global _handle
     if _handle is None:
         if not os.path.exists(LIB_PATH):
-            raise ImportError(f"libmw.so not built at {LIB_PATH}; run __graft_entry__.build()")
+            raise ImportError(f"{os.path.basename(LIB_PATH)} not built at {LIB_PATH}; run __graft_entry__.build()")
         h = ctypes.CDLL(LIB_PATH)
         for name, (res, args) in _SIGS.items():
             fn = getattr(h, name)
@@ -107,6 +111,11 @@ def _lib():
 def kernel_launches():
     """Kernels libmw has launched in this process so far."""
     return int(_lib().mw_kernel_launches())
+
+
+def build_flags():
+    """mw_build_flags(): 1 (MW_BUILD_DEBUG) for the debug library."""
+    return int(_lib().mw_build_flags())
 
 
 def exported_names():
@@ -520,8 +529,9 @@ def forward_kl_fwd(HT, rows_T, HS, rows_S, W, lam=1.0, stream=None):
 
 
 def forward_kl_check_status(rows_T, HT, W, ws, stream=None):
-    """Synchronise and raise if a bounded device wait of the tensor-core KL
-    passes gave up (mw_forward_kl_check_status)."""
+    """Synchronise and raise MWError if a bounded device wait of the
+    tensor-core KL passes gave up (MW_ETIMEOUT) or a pair's row index was out
+    of range (MW_EDEVICE) (mw_forward_kl_check_status)."""
     _check(_lib().mw_forward_kl_check_status(int(rows_T.numel()), HT.shape[1], W.shape[0], _dtype_code(HT),
                                              _ptr(ws), _stream(stream)), "mw_forward_kl_check_status")
 
@@ -699,8 +709,9 @@ def mw_logprob_loss_bwd(H, W, targets, rows, lse, ws, dloss, dH, dW, stream=None
 
 
 def mw_logprob_check_status(H, W, rows, ws, stream=None):
-    """Raise MWError (MW_ETIMEOUT) if a tensor-core LM-head kernel that last
-    ran on ``ws`` gave up a bounded wait; synchronises the stream."""
+    """Raise MWError if an LM-head kernel that last ran on ``ws`` gave up a
+    bounded wait (MW_ETIMEOUT) or met a loss row or target out of range
+    (MW_EDEVICE); synchronises the stream."""
     N, d = H.shape
     _check(_lib().mw_logprob_check_status(N, int(rows.numel()), d, W.shape[0], _dtype_code(H), _ptr(ws),
                                           _stream(stream)), "mw_logprob_check_status")

@@ -1,7 +1,10 @@
 """Build libmw.so in-tree with nvcc for sm_103a (GB300).
 
 Each .cu file is compiled to an object in parallel, then linked into one
-shared library next to this file. Nothing is installed.
+shared library next to this file. Nothing is installed. ``debug=True`` builds
+libmw_debug.so instead: the same sources with -DMW_DEBUG, whose kernels check
+the indices they read from memory before following them (loaded by the
+binding when MW_DEBUG=1 is set in the environment).
 """
 
 import os
@@ -15,6 +18,8 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libmw.so")
+BUILD_DEBUG = os.path.join(HERE, "_build_debug")
+LIB_DEBUG = os.path.join(HERE, "libmw_debug.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 
@@ -34,14 +39,18 @@ def flags(extra=()):
                    "-I", os.path.join(ROOT, "include"), "-I", CSRC, *extra]
 
 
-def build(verbose=False, jobs=None, extra=()):
-    """Compile every kernel source and link ``libmw.so``; returns its path."""
-    os.makedirs(BUILD, exist_ok=True)
+def build(verbose=False, jobs=None, extra=(), debug=False):
+    """Compile every kernel source and link ``libmw.so`` (``libmw_debug.so``
+    with ``debug``); returns its path."""
+    bdir, lib = (BUILD_DEBUG, LIB_DEBUG) if debug else (BUILD, LIB)
+    if debug:
+        extra = ("-DMW_DEBUG", *extra)
+    os.makedirs(bdir, exist_ok=True)
     nvcc = _nvcc()
     srcs = sources()
 
     def one(src):
-        obj = os.path.join(BUILD, src[:-3] + ".o")
+        obj = os.path.join(bdir, src[:-3] + ".o")
         cmd = [nvcc, *flags(extra), "-c", os.path.join(CSRC, src), "-o", obj]
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
@@ -52,14 +61,14 @@ def build(verbose=False, jobs=None, extra=()):
 
     with ThreadPoolExecutor(max_workers=jobs or min(8, len(srcs))) as ex:
         objs = list(ex.map(one, srcs))
-    tmp = LIB + ".tmp"
+    tmp = lib + ".tmp"
     cmd = [nvcc, *ARCH, "-shared", "-Xcompiler", "-fPIC", "-o", tmp, *objs]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
-    os.replace(tmp, LIB)
-    return LIB
+    os.replace(tmp, lib)
+    return lib
 
 
 if __name__ == "__main__":
-    print(build(verbose="-v" in sys.argv))
+    print(build(verbose="-v" in sys.argv, debug="--debug" in sys.argv))

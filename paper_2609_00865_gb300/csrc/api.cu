@@ -12,10 +12,10 @@ mw_status attn_fwd_simt(const mw_vis_layout*, const void*, const void*, const vo
 mw_status attn_bwd_simt(const mw_vis_layout*, const void*, const void*, const void*, const void*, const void*,
                         const void*, const float*, void*, void*, void*, int, int, int, int, float, float*,
                         cudaStream_t);
-mw_status lm_fwd_simt(const void*, const void*, const int32_t*, const int32_t*, int, int, int, int, float*, float*,
-                      float*, cudaStream_t);
+mw_status lm_fwd_simt(const void*, const void*, const int32_t*, const int32_t*, int, int, int, int, int, float*,
+                      float*, float*, int32_t*, cudaStream_t);
 mw_status lm_bwd_simt(const void*, const void*, const int32_t*, const int32_t*, int, int, int, int, int,
-                      const float*, const float*, float, void*, float*, cudaStream_t);
+                      const float*, const float*, float, void*, float*, int32_t*, cudaStream_t);
 mw_status attn_fwd_tc(const mw_vis_layout*, const void*, const void*, const void*, const void*, void*, float*, int,
                       int, float, void*, cudaStream_t, const float* = nullptr);
 mw_status attn_bwd_tc(const mw_vis_layout*, const void*, const void*, const void*, const void*, const void*,
@@ -41,7 +41,7 @@ __global__ void k_loss_epilogue(int, const float*, const float*, const float*, f
                                 float*, float*);
 __global__ void k_logdiff(int, const float*, const float*, float*);
 
-mw_status lm_ref_tc(const void*, const void*, const int32_t*, const int32_t*, int, int, int, void*, int32_t*,
+mw_status lm_ref_tc(const void*, const void*, const int32_t*, const int32_t*, int, int, int, int, void*, int32_t*,
                     float2*, float*, float4*, int32_t*, cudaStream_t);
 
 bool lm_bwd_tc_supported(int d);
@@ -180,17 +180,18 @@ extern "C" mw_status mw_logprob_loss_fwd_kl(const void* H, const void* W, const 
     LmWs w = lm_ws_layout(N, M, d, V, dtype);
     float* g = at<float>(ws, w.g);
     float* zt = at<float>(ws, w.zt);
+    int32_t* status = at<int32_t>(ws, w.status);
+    if ((st = cuda_status(cudaMemsetAsync(status, 0, 32, s))) != MW_OK) return st;
     if (lm_tc(d, dtype)) {
-        if ((st = cuda_status(cudaMemsetAsync(at<char>(ws, w.status), 0, 32, s))) != MW_OK) return st;
         // references from the first vocabulary entries, then the fused pass
         // over the whole vocabulary (lse, lp, and E for the backward)
-        st = lm_ref_tc(H, W, targets, rows, M, d, V, at<char>(ws, w.hg), at<int32_t>(ws, w.tg),
-                       at<float2>(ws, w.part), zt, at<float4>(ws, w.bwd), at<int32_t>(ws, w.status), s);
+        st = lm_ref_tc(H, W, targets, rows, M, N, d, V, at<char>(ws, w.hg), at<int32_t>(ws, w.tg),
+                       at<float2>(ws, w.part), zt, at<float4>(ws, w.bwd), status, s);
         if (st == MW_OK)
-            st = lm_fwd_grp_tc(W, M, d, V, at<char>(ws, w.hg), at<int32_t>(ws, w.tg), zt, lse, lp,
-                               at<int32_t>(ws, w.status), at<char>(ws, w.bwd), at<char>(ws, w.fwd), s);
+            st = lm_fwd_grp_tc(W, M, d, V, at<char>(ws, w.hg), at<int32_t>(ws, w.tg), zt, lse, lp, status,
+                               at<char>(ws, w.bwd), at<char>(ws, w.fwd), s);
     } else {
-        st = lm_fwd_simt(H, W, targets, rows, M, d, V, dtype, lse, zt, lp, s);
+        st = lm_fwd_simt(H, W, targets, rows, M, N, d, V, dtype, lse, zt, lp, status, s);
     }
     if (st != MW_OK) return st;
     count_launches(1);
@@ -215,16 +216,14 @@ extern "C" mw_status mw_logprob_loss_bwd(const void* H, const void* W, const int
     if (!ws || !dW || (N > 0 && !dH)) return MW_EINVAL;
     if (M > 0 && (!H || !W || !targets || !rows || !lse)) return MW_EINVAL;
     LmWs w = lm_ws_layout(N, M, d, V, dtype);
-    if (lm_tc(d, dtype)) {
-        // the backward reads the forward's gathered rows, g, E and 1 / l; it
-        // writes the status words and the group passes' scratch
-        if ((st = cuda_status(cudaMemsetAsync(at<char>(ws, w.status), 0, 32, (cudaStream_t)stream))) != MW_OK)
-            return st;
+    // the backward reads the forward's g (and on the tensor cores its gathered
+    // rows, E and 1 / l); it adds to the status words the forward reset, so
+    // a forward that gave up a wait ends the backward's waits at once
+    int32_t* status = at<int32_t>(ws, w.status);
+    if (lm_tc(d, dtype))
         return lm_bwd_tc(W, M, N, d, V, rows, at<char>(ws, w.hg), at<int32_t>(ws, w.tg), lse, at<float>(ws, w.g),
-                         dloss, dH, dW, at<int32_t>(ws, w.status), at<char>(ws, w.bwd), at<char>(ws, w.fwd),
-                         (cudaStream_t)stream);
-    }
-    return lm_bwd_simt(H, W, targets, rows, M, N, d, V, dtype, lse, at<float>(ws, w.g), dloss, dH, dW,
+                         dloss, dH, dW, status, at<char>(ws, w.bwd), at<char>(ws, w.fwd), (cudaStream_t)stream);
+    return lm_bwd_simt(H, W, targets, rows, M, N, d, V, dtype, lse, at<float>(ws, w.g), dloss, dH, dW, status,
                        (cudaStream_t)stream);
 }
 
@@ -240,15 +239,15 @@ extern "C" mw_status mw_logprob_check_status(int N, int M, int d, int V, int dty
     mw_status st = lm_args(N, M, d, V, dtype);
     if (st != MW_OK) return st;
     if (!ws) return MW_EINVAL;
-    // only the tensor-core kernels wait on barriers; the SIMT path has no status words
-    if (!lm_tc(d, dtype)) return cuda_status(cudaStreamSynchronize((cudaStream_t)stream));
+    // timeouts come from the tensor-core kernels' barrier waits; both paths
+    // raise the bounds flag for a loss row or target out of range
     LmWs w = lm_ws_layout(N, M, d, V, dtype);
     int32_t h[8];
     if ((st = cuda_status(cudaMemcpyAsync(h, at<char>(ws, w.status), sizeof(h), cudaMemcpyDeviceToHost,
                                           (cudaStream_t)stream))) != MW_OK)
         return st;
     if ((st = cuda_status(cudaStreamSynchronize((cudaStream_t)stream))) != MW_OK) return st;
-    return h[1] ? MW_ETIMEOUT : MW_OK;
+    return h[1] ? MW_ETIMEOUT : h[0] ? MW_EDEVICE : MW_OK;
 }
 
 // --- row-wise logical positions and rotary attention (§4.2) -----------------

@@ -64,6 +64,7 @@ __global__ void __launch_bounds__(128) k_attn_fwd_simt(VisView v, int64_t total,
             const int e = v.fwd_idx[p];
             const int kt = e >> 4, cls = e & 3;
             const int jend = min(kt * MW_TILE + MW_TILE, i + 1);
+            if (!MW_DBG_IN(kt, qt + 1, v.status, 211)) continue;
             for (int j0 = kt * MW_TILE; j0 < jend; j0 += 32) {
                 const int j = j0 + lane;
                 bool vis = j < jend;
@@ -152,6 +153,7 @@ __global__ void __launch_bounds__(128) k_attn_dq_simt(VisView v, int64_t total, 
             const int e = v.fwd_idx[p];
             const int kt = e >> 4, cls = e & 3;
             const int jend = min(kt * MW_TILE + MW_TILE, i + 1);
+            if (!MW_DBG_IN(kt, qt + 1, v.status, 212)) continue;
             for (int j0 = kt * MW_TILE; j0 < jend; j0 += 32) {
                 const int j = j0 + lane;
                 bool vis = j < jend;

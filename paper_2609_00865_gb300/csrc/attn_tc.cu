@@ -503,7 +503,7 @@ __global__ void __launch_bounds__(NT_FWD, 1)
             const float inv = 1.f / l;
             __nv_bfloat16* orow = p.O + ((tok0 + ie) * p.Hq + h) * DH;
             uint32_t o[32];
-            const bool store = in_piece;
+            const bool store = in_piece && MW_DBG_IN(tok0 + i, v.total, status, 203);
 #pragma unroll
             for (int c = 0; c < 4; ++c) {
                 tmem_ld32(lane_base + TM_O + c * 32, o);
@@ -837,7 +837,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             tc_fence_after();
             __nv_bfloat16* qrow = p.dQ + ((tok0 + ie) * p.Hq + h) * DH;
             uint32_t o[32];
-            const bool store = in_piece;
+            const bool store = in_piece && MW_DBG_IN(tok0 + i, v.total, status, 204);
 #pragma unroll
             for (int cc = 0; cc < 2; ++cc) {
                 const int c = 2 * ch + cc;
@@ -1138,6 +1138,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
             // per compact row
             tc_fence_after();
             const int64_t row = ((krow0 + rl) * p.Hkv + kvh) * DH;
+            const bool kstore = kin && MW_DBG_IN(krow0 + rl, v.n_keymask * 128, status, 205);
             uint32_t o[32];
 #pragma unroll
             for (int pass = 0; pass < 2; ++pass) {
@@ -1149,7 +1150,7 @@ __global__ void __launch_bounds__(NT_BWD, 1)
                     const int c = 2 * ch + cc;
                     tmem_ld32(lane_base + col + c * 32, o);
                     tmem_wait_ld();
-                    if (kin) {
+                    if (kstore) {
 #pragma unroll
                         for (int x = 0; x < 8; ++x)
                             *reinterpret_cast<float4*>(dst + c * 32 + 4 * x) =
@@ -1242,10 +1243,12 @@ __global__ void __launch_bounds__(256) k_cmp_gather(VisView v, int n_traj, int H
     const int b = cmp_entry_traj(v, n_traj, e, s, kt, nt);
     if (kt * 128 >= v.seg_len[v.traj_seg[b] + s]) return;
     const int64_t tok0 = v.traj_tok[b];
+    const int T_b = v.traj_tok[b + 1] - (int)tok0;
     const int vec = Hkv * (DH / 8);   // 16-byte vectors per key row
     for (int x = threadIdx.x; x < 128 * vec; x += blockDim.x) {
         const int r = x / vec, k = x - r * vec;
-        const int j = v.csrc[e * 128 + r];
+        int j = v.csrc[e * 128 + r];
+        if (j >= 0 && !MW_DBG_IN(j, T_b, v.status, 201)) j = -1;
         uint4 vv = make_uint4(0u, 0u, 0u, 0u);
         if (j >= 0) vv = reinterpret_cast<const uint4*>(V + (tok0 + j) * Hkv * DH)[k];
         reinterpret_cast<uint4*>(Vc + (e * 128 + r) * Hkv * DH)[k] = vv;
@@ -1322,7 +1325,7 @@ __global__ void __launch_bounds__(256) k_cmp_reduce(VisView v, int Hkv, const fl
         for (int s = v.seg[tok0 + j]; s < nseg; ++s) {
             const int64_t base = (v.traj_km[b] + (int64_t)s * nt) * 128;
             const int c = v.cpos[base + j];
-            if (c < 0) continue;
+            if (c < 0 || !MW_DBG_IN(c, (int64_t)nt * 128, v.status, 202)) continue;
             const float4* pv = reinterpret_cast<const float4*>(dVc + (base + c) * Hkv * DH) + 2 * k;
             const float4 v0 = pv[0], v1 = pv[1];
             av[0] += v0.x; av[1] += v0.y; av[2] += v0.z; av[3] += v0.w;

@@ -51,7 +51,7 @@ __global__ void __launch_bounds__(256) k_branch_pack(VisView v, int n_traj, int 
         const int r = x / vec, k = x - r * vec;
         const int c = kt * MW_TILE + r;
         const int j = v.csrc[e * MW_TILE + r];
-        Xp[(off + c) * vec + k] = X[(tok0 + j) * vec + k];
+        if (MW_DBG_IN(j, v.traj_tok[b + 1] - tok0, v.status, 301)) Xp[(off + c) * vec + k] = X[(tok0 + j) * vec + k];
     }
 }
 
@@ -81,7 +81,7 @@ __global__ void __launch_bounds__(256) k_branch_unpack_add(VisView v, int vec, c
         for (int q = 0; q < PER; ++q) acc[q] = 0.f;
         for (int s = v.seg[tok0 + j]; s < nseg; ++s) {
             const int c = v.cpos[(v.traj_km[b] + (int64_t)s * nt) * MW_TILE + j];
-            if (c < 0) continue;
+            if (c < 0 || !MW_DBG_IN(c, v.seg_len[g0 + s], v.status, 302)) continue;
             const int64_t o = s < 64 ? off[s] : branch_off(v, g0 + s);
             const uint4 u = dXp[(o + c) * vec + k];
             const T* t = reinterpret_cast<const T*>(&u);

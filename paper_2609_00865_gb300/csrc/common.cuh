@@ -75,6 +75,7 @@ struct VisView {
     const int32_t* cpos;      // [n_keymask][128] rank of key j in view_s, -1 if absent
     const int32_t* csrc;      // [n_keymask][128] key (traj-local) at each rank of view_s
     int32_t* status;
+    int64_t total, n_keymask; // sizes for the debug library's index checks
 };
 
 inline VisView make_view(const mw_vis_layout* L, const void* vis) {
@@ -98,10 +99,44 @@ inline VisView make_view(const mw_vis_layout* L, const void* vis) {
     v.cpos = at<int32_t>(vis, L->off_cpos);
     v.csrc = at<int32_t>(vis, L->off_csrc);
     v.status = const_cast<int32_t*>(at<int32_t>(vis, L->off_status));
+    v.total = L->total_tokens;
+    v.n_keymask = L->n_keymask;
     return v;
 }
 
 // Status-word slots written by device code.
 enum { ST_BOUNDS = 0, ST_TIMEOUT = 1, ST_WHERE = 2 };
+
+// Loss rows and their targets are device arrays filled by the caller, so no
+// host check sees them. A kernel takes such an index through checked_index:
+// inside [0, n) it is returned, otherwise -1 and the row is not read or
+// written; the kernel then raises the bounds flag of its status word (the
+// status check reports MW_EDEVICE).
+__device__ __forceinline__ int checked_index(int i, int n) { return (unsigned)i < (unsigned)n ? i : -1; }
+__device__ __forceinline__ void flag_bounds(int32_t* status) {
+    if (status) atomicExch(status + ST_BOUNDS, 1);
+}
+
+// Index checks of the debug library (compiled with -DMW_DEBUG into
+// libmw_debug.so). At the accesses whose index is read from memory (a
+// record's spans, the compact maps, segment tables) or derived from one,
+// MW_DBG_IN(i, n, status, where) is false for i outside [0, n), after
+// raising the bounds flag and recording the site `where` (the first one
+// wins); the caller then skips the access. The status check reports
+// MW_EDEVICE. In the release library it is the constant true and the
+// check compiles away.
+#ifdef MW_DEBUG
+__device__ __forceinline__ bool dbg_in(long long i, long long n, int32_t* status, int where) {
+    if (i >= 0 && i < n) return true;
+    if (status) {
+        atomicExch(status + ST_BOUNDS, 1);
+        atomicCAS(status + ST_WHERE, 0, where);
+    }
+    return false;
+}
+#define MW_DBG_IN(i, n, status, where) (::mw::dbg_in((long long)(i), (long long)(n), (status), (where)))
+#else
+#define MW_DBG_IN(i, n, status, where) (true)
+#endif
 
 }  // namespace mw

@@ -646,17 +646,25 @@ __global__ void k_lm_grp_combine(int M, int M_pad, int C, const float4* __restri
 }
 
 // dH_{rows[m]} = dloss g_m (W_{tgt_m} - E_m / l_m), bf16; one block per loss
-// row (grid-stride), 16-byte vectors along d. Rows outside the loss stay 0.
-__global__ void k_lm_dh_from_e(int M, int d, const __nv_bfloat16* __restrict__ W, const int32_t* __restrict__ tg,
-                               const float* __restrict__ E, const float* __restrict__ linv,
-                               const float* __restrict__ g, float dloss, const int32_t* __restrict__ rows,
-                               __nv_bfloat16* __restrict__ dH) {
+// row (grid-stride), 16-byte vectors along d. Rows outside the loss stay 0,
+// and so does a row outside [0, N) or without a valid target (the forward's
+// gather gave it target -1; bounds flag).
+__global__ void k_lm_dh_from_e(int M, int d, int N, const __nv_bfloat16* __restrict__ W,
+                               const int32_t* __restrict__ tg, const float* __restrict__ E,
+                               const float* __restrict__ linv, const float* __restrict__ g, float dloss,
+                               const int32_t* __restrict__ rows, __nv_bfloat16* __restrict__ dH,
+                               int32_t* __restrict__ status) {
     const int nvec = d / 8;
     for (int m = blockIdx.x; m < M; m += gridDim.x) {
+        const int r = checked_index(rows[m], N), t = tg[m];
+        if (r < 0 || t < 0) {   // uniform over the block
+            if (threadIdx.x == 0) flag_bounds(status);
+            continue;
+        }
         const float a = dloss * g[m], il = linv[m];
-        const uint4* wr = reinterpret_cast<const uint4*>(W + (int64_t)tg[m] * d);
+        const uint4* wr = reinterpret_cast<const uint4*>(W + (int64_t)t * d);
         const float4* er = reinterpret_cast<const float4*>(E + (int64_t)m * d);
-        uint4* out = reinterpret_cast<uint4*>(dH + (int64_t)rows[m] * d);
+        uint4* out = reinterpret_cast<uint4*>(dH + (int64_t)r * d);
         for (int k = threadIdx.x; k < nvec; k += blockDim.x) {
             const uint4 u = __ldg(&wr[k]);
             const float4 e0 = er[2 * k], e1 = er[2 * k + 1];
@@ -707,14 +715,20 @@ __global__ void k_kl_from_e(int M, int d, const __nv_bfloat16* __restrict__ hgT,
 // dH_S of the KL: c (Ebar_S - Ebar_T) at the student row of each pair (bf16).
 // Both products are rounded before the difference (no fused multiply-add), so
 // a student equal to its teacher gets exactly 0.
-__global__ void k_kl_dh_from_e(int M, int d, const float* __restrict__ ES, const float* __restrict__ linvS,
+__global__ void k_kl_dh_from_e(int M, int d, int N_S, const float* __restrict__ ES, const float* __restrict__ linvS,
                                const float* __restrict__ ET, const float* __restrict__ linvT, float c,
-                               const int32_t* __restrict__ rowsS, int accumulate, __nv_bfloat16* __restrict__ dHS) {
+                               const int32_t* __restrict__ rowsS, int accumulate, __nv_bfloat16* __restrict__ dHS,
+                               int32_t* __restrict__ status) {
     for (int m = blockIdx.x; m < M; m += gridDim.x) {
+        const int r = checked_index(rowsS[m], N_S);
+        if (r < 0) {   // uniform over the block
+            if (threadIdx.x == 0) flag_bounds(status);
+            continue;
+        }
         const float as = c * linvS[m], at_ = c * linvT[m];
         const float4* s4 = reinterpret_cast<const float4*>(ES + (int64_t)m * d);
         const float4* t4 = reinterpret_cast<const float4*>(ET + (int64_t)m * d);
-        uint2* out = reinterpret_cast<uint2*>(dHS + (int64_t)rowsS[m] * d);
+        uint2* out = reinterpret_cast<uint2*>(dHS + (int64_t)r * d);
         for (int k = threadIdx.x; k < d / 4; k += blockDim.x) {
             const float4 x = s4[k], y = t4[k];
             float g[4] = {__fmul_rn(as, x.x) - __fmul_rn(at_, y.x), __fmul_rn(as, x.y) - __fmul_rn(at_, y.y),
@@ -916,7 +930,7 @@ mw_status lm_bwd_tc(const void* W, int M, int N, int d, int V, const int32_t* ro
     GrpArrays a = grp_arrays(fwd, M, d);
     count_launches(1);
     k_lm_dh_from_e<<<(unsigned)std::min(M, 8 * 152), 128, 0, s>>>(
-        M, d, (const __nv_bfloat16*)W, tg, a.E, a.linv, g, dloss, rows, (__nv_bfloat16*)dH);
+        M, d, N, (const __nv_bfloat16*)W, tg, a.E, a.linv, g, dloss, rows, (__nv_bfloat16*)dH, status);
     return launch_status();
 }
 
@@ -950,13 +964,13 @@ static KlWs kl_ws_layout(int M, int d) {
 
 int64_t kl_tc_ws(int M, int d) { return lm_bwd_tc_supported(d) ? kl_ws_layout(M, d).bytes : 0; }
 
-mw_status lm_ref_tc(const void*, const void*, const int32_t*, const int32_t*, int, int, int, void*, int32_t*, float2*,
-                    float*, float4*, int32_t*, cudaStream_t);
+mw_status lm_ref_tc(const void*, const void*, const int32_t*, const int32_t*, int, int, int, int, void*, int32_t*,
+                    float2*, float*, float4*, int32_t*, cudaStream_t);
 
 // Forward: for the teacher rows and then the student rows, the reference
 // prepass and the fused pass (lse, E, 1 / l); then KL per pair.
 mw_status kl_fwd_tc(const void* HT, const int32_t* rowsT, const void* HS, const int32_t* rowsS, int M, const void* W,
-                    int d, int V, float* kl, void* ws, cudaStream_t s) {
+                    int N_T, int N_S, int d, int V, float* kl, void* ws, cudaStream_t s) {
     if (!lm_bwd_tc_supported(d)) return MW_ESHAPE;
     const KlWs w = kl_ws_layout(M, d);
     mw_status st = cuda_status(cudaMemsetAsync(at<char>(ws, w.status), 0, 32, s));
@@ -965,8 +979,9 @@ mw_status kl_fwd_tc(const void* HT, const int32_t* rowsT, const void* HS, const 
         const void* H = side == 0 ? HT : HS;
         const int32_t* rows = side == 0 ? rowsT : rowsS;
         void* hg = at<char>(ws, side == 0 ? w.hgT : w.hgS);
-        st = lm_ref_tc(H, W, nullptr, rows, M, d, V, hg, at<int32_t>(ws, w.tg), at<float2>(ws, w.part),
-                       at<float>(ws, w.zt), at<float4>(ws, w.scratch), at<int32_t>(ws, w.status), s);
+        st = lm_ref_tc(H, W, nullptr, rows, M, side == 0 ? N_T : N_S, d, V, hg, at<int32_t>(ws, w.tg),
+                       at<float2>(ws, w.part), at<float>(ws, w.zt), at<float4>(ws, w.scratch),
+                       at<int32_t>(ws, w.status), s);
         if (st == MW_OK)
             st = lm_fwd_grp_tc(W, M, d, V, hg, at<int32_t>(ws, w.tg), at<float>(ws, w.zt),
                                at<float>(ws, side == 0 ? w.lseT : w.lseS), at<float>(ws, w.lp),
@@ -994,11 +1009,11 @@ mw_status kl_bwd_tc(const int32_t* rowsS, int M, const void* W, int N_S, int d, 
     if (M == 0) return accumulate ? MW_OK : cuda_status(cudaMemsetAsync(dW, 0, (size_t)V * d * 4, s));
     const KlWs w = kl_ws_layout(M, d);
     const int M_pad = (int)ceil_div(M, 128) * 128;
-    if ((st = cuda_status(cudaMemsetAsync(at<char>(ws, w.status), 0, 32, s))) != MW_OK) return st;
     const GrpArrays aT = grp_arrays(at<char>(ws, w.fwdT), M, d), aS = grp_arrays(at<char>(ws, w.fwdS), M, d);
     count_launches(1);
-    k_kl_dh_from_e<<<(unsigned)std::min(M, 8 * 152), 128, 0, s>>>(M, d, aS.E, aS.linv, aT.E, aT.linv, c, rowsS,
-                                                                  accumulate, (__nv_bfloat16*)dHS);
+    k_kl_dh_from_e<<<(unsigned)std::min(M, 8 * 152), 128, 0, s>>>(M, d, N_S, aS.E, aS.linv, aT.E, aT.linv, c, rowsS,
+                                                                  accumulate, (__nv_bfloat16*)dHS,
+                                                                  at<int32_t>(ws, w.status));
     if ((st = launch_status()) != MW_OK) return st;
     for (int side = 0; side < 2; ++side) {   // student: dz = c p_S; teacher: dz = -c p_T
         count_launches(1);

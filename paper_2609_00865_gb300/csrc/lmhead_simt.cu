@@ -80,6 +80,37 @@ __device__ __forceinline__ void lse_merge(float& m, float& l, float m2, float l2
     m = mn;
 }
 
+// Physical rows and targets of loss rows m0 .. m0 + n - 1 into shared memory:
+// -1 past M; a row outside [0, N) or a target outside [0, Vocab) also gives
+// row and target -1 and raises the bounds flag: the row then reads as zero
+// and its dH row is not written.
+__device__ __forceinline__ void stage_index(int* srow, int* stg, const int32_t* __restrict__ rows,
+                                            const int32_t* __restrict__ targets, int m0, int n, int M, int N,
+                                            int Vocab, int32_t* status) {
+    if (threadIdx.x < n) {
+        const int m = m0 + threadIdx.x;
+        int r = -1, t = -1;
+        if (m < M) {
+            r = checked_index(rows[m], N);
+            if (r >= 0) t = checked_index(targets[r], Vocab);
+            if (t < 0) {
+                flag_bounds(status);
+                r = -1;
+            }
+        }
+        srow[threadIdx.x] = r;
+        stg[threadIdx.x] = t;
+    }
+}
+
+template <typename Tin>
+__device__ __forceinline__ void stage_hidden(float* hs, const Tin* __restrict__ H, const int* srow, int n, int d) {
+    for (int x = threadIdx.x; x < n * d; x += blockDim.x) {
+        const int r = x / d, k = x % d;
+        hs[x] = srow[r] >= 0 ? ld_f(H + (int64_t)srow[r] * d + k) : 0.f;
+    }
+}
+
 template <typename Tin>
 __device__ __forceinline__ void row_logits(const float* __restrict__ hs, int d, const Tin* __restrict__ wrow,
                                            float* z) {
@@ -94,19 +125,17 @@ __device__ __forceinline__ void row_logits(const float* __restrict__ hs, int d, 
 
 // grid: ceil(M / FR); block 256. Writes lse[m] and zt[m] (target logit).
 template <typename Tin>
-__global__ void __launch_bounds__(256) k_lm_fwd_simt(int M, int d, int Vocab, const Tin* __restrict__ H,
+__global__ void __launch_bounds__(256) k_lm_fwd_simt(int M, int N, int d, int Vocab, const Tin* __restrict__ H,
                                                     const Tin* __restrict__ W, const int32_t* __restrict__ targets,
                                                     const int32_t* __restrict__ rows, float* __restrict__ lse,
-                                                    float* __restrict__ zt) {
+                                                    float* __restrict__ zt, int32_t* __restrict__ status) {
     extern __shared__ float hs[];  // [FR][d]
     __shared__ float sm[FR][8], sl[FR][8];
-    __shared__ int tg[FR];
+    __shared__ int tg[FR], srow[FR];
     const int m0 = blockIdx.x * FR;
-    for (int x = threadIdx.x; x < FR * d; x += blockDim.x) {
-        const int r = x / d, k = x % d;
-        hs[x] = (m0 + r < M) ? ld_f(H + (int64_t)rows[m0 + r] * d + k) : 0.f;
-    }
-    if (threadIdx.x < FR) tg[threadIdx.x] = (m0 + threadIdx.x < M) ? targets[rows[m0 + threadIdx.x]] : -1;
+    stage_index(srow, tg, rows, targets, m0, FR, M, N, Vocab, status);
+    __syncthreads();
+    stage_hidden(hs, H, srow, FR, d);
     __syncthreads();
     float m[FR], l[FR], z[FR];
 #pragma unroll
@@ -146,26 +175,25 @@ __global__ void k_lp_from_zt(int M, const float* __restrict__ zt, const float* _
 
 // dH: grid ceil(M / FR), block 256 (d <= 256). Vocab tiles of 256 columns.
 template <typename Tin>
-__global__ void __launch_bounds__(256) k_lm_dh_simt(int M, int d, int Vocab, const Tin* __restrict__ H,
+__global__ void __launch_bounds__(256) k_lm_dh_simt(int M, int N, int d, int Vocab, const Tin* __restrict__ H,
                                                    const Tin* __restrict__ W, const int32_t* __restrict__ targets,
                                                    const int32_t* __restrict__ rows, const float* __restrict__ lse,
-                                                   const float* __restrict__ g, float dloss, Tin* __restrict__ dH) {
+                                                   const float* __restrict__ g, float dloss, Tin* __restrict__ dH,
+                                                   int32_t* __restrict__ status) {
     extern __shared__ float sh[];
     float* hs = sh;               // [FR][d]
     float* dzs = sh + FR * d;     // [FR][256]
-    __shared__ int tg[FR];
+    __shared__ int tg[FR], srow[FR];
     __shared__ float slse[FR], sg[FR];
     const int m0 = blockIdx.x * FR;
-    for (int x = threadIdx.x; x < FR * d; x += blockDim.x) {
-        const int r = x / d, k = x % d;
-        hs[x] = (m0 + r < M) ? ld_f(H + (int64_t)rows[m0 + r] * d + k) : 0.f;
-    }
+    stage_index(srow, tg, rows, targets, m0, FR, M, N, Vocab, status);
     if (threadIdx.x < FR) {
         const bool ok = m0 + threadIdx.x < M;
-        tg[threadIdx.x] = ok ? targets[rows[m0 + threadIdx.x]] : -1;
         slse[threadIdx.x] = ok ? lse[m0 + threadIdx.x] : 0.f;
         sg[threadIdx.x] = ok ? g[m0 + threadIdx.x] * dloss : 0.f;
     }
+    __syncthreads();
+    stage_hidden(hs, H, srow, FR, d);
     __syncthreads();
     float acc[FR], z[FR];
 #pragma unroll
@@ -196,7 +224,7 @@ __global__ void __launch_bounds__(256) k_lm_dh_simt(int M, int d, int Vocab, con
     if (threadIdx.x < d) {
 #pragma unroll
         for (int r = 0; r < FR; ++r)
-            if (m0 + r < M) st_f(dH + (int64_t)rows[m0 + r] * d + threadIdx.x, acc[r]);
+            if (srow[r] >= 0) st_f(dH + (int64_t)srow[r] * d + threadIdx.x, acc[r]);
     }
 }
 
@@ -205,15 +233,16 @@ constexpr int WR = 32;  // loss rows per dW step
 
 // dW: grid ceil(Vocab / WV), block 256 (d <= 256).
 template <typename Tin>
-__global__ void __launch_bounds__(256) k_lm_dw_simt(int M, int d, int Vocab, const Tin* __restrict__ H,
+__global__ void __launch_bounds__(256) k_lm_dw_simt(int M, int N, int d, int Vocab, const Tin* __restrict__ H,
                                                    const Tin* __restrict__ W, const int32_t* __restrict__ targets,
                                                    const int32_t* __restrict__ rows, const float* __restrict__ lse,
-                                                   const float* __restrict__ g, float dloss, float* __restrict__ dW) {
+                                                   const float* __restrict__ g, float dloss, float* __restrict__ dW,
+                                                   int32_t* __restrict__ status) {
     extern __shared__ float sh[];
     float* ws = sh;                // [WV][d]
     float* hs = sh + WV * d;       // [WR][d]
     float* dzs = hs + WR * d;      // [WR][WV]
-    __shared__ int tg[WR];
+    __shared__ int tg[WR], srow[WR];
     __shared__ float slse[WR], sg[WR];
     const int v0 = blockIdx.x * WV;
     for (int x = threadIdx.x; x < WV * d; x += blockDim.x) {
@@ -225,16 +254,14 @@ __global__ void __launch_bounds__(256) k_lm_dw_simt(int M, int d, int Vocab, con
     for (int q = 0; q < WV; ++q) acc[q] = 0.f;
     for (int m0 = 0; m0 < M; m0 += WR) {
         __syncthreads();
-        for (int x = threadIdx.x; x < WR * d; x += blockDim.x) {
-            const int r = x / d, k = x % d;
-            hs[x] = (m0 + r < M) ? ld_f(H + (int64_t)rows[m0 + r] * d + k) : 0.f;
-        }
+        stage_index(srow, tg, rows, targets, m0, WR, M, N, Vocab, status);
         if (threadIdx.x < WR) {
             const bool ok = m0 + threadIdx.x < M;
-            tg[threadIdx.x] = ok ? targets[rows[m0 + threadIdx.x]] : -1;
             slse[threadIdx.x] = ok ? lse[m0 + threadIdx.x] : 0.f;
             sg[threadIdx.x] = ok ? g[m0 + threadIdx.x] * dloss : 0.f;
         }
+        __syncthreads();
+        stage_hidden(hs, H, srow, WR, d);
         __syncthreads();
         {   // 32 x 32 logits: thread -> (row r, 4 vocab columns)
             const int r = threadIdx.x >> 3, c0 = (threadIdx.x & 7) * 4;
@@ -268,50 +295,52 @@ __global__ void __launch_bounds__(256) k_lm_dw_simt(int M, int d, int Vocab, con
 }
 
 template <typename Tin>
-mw_status fwd_t(const void* H, const void* W, const int32_t* targets, const int32_t* rows, int M, int d, int Vocab,
-                float* lse, float* zt, float* lp, cudaStream_t s) {
+mw_status fwd_t(const void* H, const void* W, const int32_t* targets, const int32_t* rows, int M, int N, int d,
+                int Vocab, float* lse, float* zt, float* lp, int32_t* status, cudaStream_t s) {
     const size_t smem = sizeof(float) * FR * d;
     count_launches(2);
     cudaFuncSetAttribute(k_lm_fwd_simt<Tin>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    k_lm_fwd_simt<Tin><<<(unsigned)ceil_div(M, FR), 256, smem, s>>>(M, d, Vocab, (const Tin*)H, (const Tin*)W,
-                                                                    targets, rows, lse, zt);
+    k_lm_fwd_simt<Tin><<<(unsigned)ceil_div(M, FR), 256, smem, s>>>(M, N, d, Vocab, (const Tin*)H, (const Tin*)W,
+                                                                    targets, rows, lse, zt, status);
     k_lp_from_zt<<<(unsigned)ceil_div(M, 256), 256, 0, s>>>(M, zt, lse, lp);
     return launch_status();
 }
 
 template <typename Tin>
 mw_status bwd_t(const void* H, const void* W, const int32_t* targets, const int32_t* rows, int M, int N, int d,
-                int Vocab, const float* lse, const float* g, float dloss, void* dH, float* dW, cudaStream_t s) {
+                int Vocab, const float* lse, const float* g, float dloss, void* dH, float* dW, int32_t* status,
+                cudaStream_t s) {
     mw_status st = cuda_status(cudaMemsetAsync(dH, 0, sizeof(Tin) * (size_t)N * d, s));
     if (st != MW_OK) return st;
     if (M == 0) return cuda_status(cudaMemsetAsync(dW, 0, sizeof(float) * (size_t)Vocab * d, s));
     count_launches(2);
     const size_t smem_h = sizeof(float) * (FR * d + FR * 256);
     cudaFuncSetAttribute(k_lm_dh_simt<Tin>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_h);
-    k_lm_dh_simt<Tin><<<(unsigned)ceil_div(M, FR), 256, smem_h, s>>>(M, d, Vocab, (const Tin*)H, (const Tin*)W,
-                                                                     targets, rows, lse, g, dloss, (Tin*)dH);
+    k_lm_dh_simt<Tin><<<(unsigned)ceil_div(M, FR), 256, smem_h, s>>>(M, N, d, Vocab, (const Tin*)H, (const Tin*)W,
+                                                                     targets, rows, lse, g, dloss, (Tin*)dH, status);
     const size_t smem_w = sizeof(float) * (WV * d + WR * d + WR * WV);
     cudaFuncSetAttribute(k_lm_dw_simt<Tin>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_w);
-    k_lm_dw_simt<Tin><<<(unsigned)ceil_div(Vocab, WV), 256, smem_w, s>>>(M, d, Vocab, (const Tin*)H, (const Tin*)W,
-                                                                         targets, rows, lse, g, dloss, dW);
+    k_lm_dw_simt<Tin><<<(unsigned)ceil_div(Vocab, WV), 256, smem_w, s>>>(M, N, d, Vocab, (const Tin*)H,
+                                                                         (const Tin*)W, targets, rows, lse, g, dloss,
+                                                                         dW, status);
     return launch_status();
 }
 
 }  // namespace
 
-mw_status lm_fwd_simt(const void* H, const void* W, const int32_t* targets, const int32_t* rows, int M, int d,
-                      int Vocab, int dtype, float* lse, float* zt, float* lp, cudaStream_t s) {
+mw_status lm_fwd_simt(const void* H, const void* W, const int32_t* targets, const int32_t* rows, int M, int N, int d,
+                      int Vocab, int dtype, float* lse, float* zt, float* lp, int32_t* status, cudaStream_t s) {
     if (M == 0) return MW_OK;
-    return dtype == MW_F32 ? fwd_t<float>(H, W, targets, rows, M, d, Vocab, lse, zt, lp, s)
-                           : fwd_t<__nv_bfloat16>(H, W, targets, rows, M, d, Vocab, lse, zt, lp, s);
+    return dtype == MW_F32 ? fwd_t<float>(H, W, targets, rows, M, N, d, Vocab, lse, zt, lp, status, s)
+                           : fwd_t<__nv_bfloat16>(H, W, targets, rows, M, N, d, Vocab, lse, zt, lp, status, s);
 }
 
 mw_status lm_bwd_simt(const void* H, const void* W, const int32_t* targets, const int32_t* rows, int M, int N,
                       int d, int Vocab, int dtype, const float* lse, const float* g, float dloss, void* dH,
-                      float* dW, cudaStream_t s) {
+                      float* dW, int32_t* status, cudaStream_t s) {
     return dtype == MW_F32
-               ? bwd_t<float>(H, W, targets, rows, M, N, d, Vocab, lse, g, dloss, dH, dW, s)
-               : bwd_t<__nv_bfloat16>(H, W, targets, rows, M, N, d, Vocab, lse, g, dloss, dH, dW, s);
+               ? bwd_t<float>(H, W, targets, rows, M, N, d, Vocab, lse, g, dloss, dH, dW, status, s)
+               : bwd_t<__nv_bfloat16>(H, W, targets, rows, M, N, d, Vocab, lse, g, dloss, dH, dW, status, s);
 }
 
 }  // namespace mw

@@ -207,17 +207,26 @@ __global__ void __launch_bounds__(NT, 1)
     }
 }
 
-__global__ void k_lm_gather(int M, int M_pad, int d, const __nv_bfloat16* __restrict__ H,
+// Hg[m] = H[rows[m]], tg[m] = targets[rows[m]] (-1 without targets); padded
+// rows (m >= M) are zero with target -1. A row outside [0, N) or a target
+// outside [0, V) is neither read nor used (zero row, target -1) and raises the
+// bounds flag.
+__global__ void k_lm_gather(int M, int M_pad, int d, int N, int V, const __nv_bfloat16* __restrict__ H,
                             const int32_t* __restrict__ targets, const int32_t* __restrict__ rows,
-                            __nv_bfloat16* __restrict__ Hg, int32_t* __restrict__ tg) {
+                            __nv_bfloat16* __restrict__ Hg, int32_t* __restrict__ tg, int32_t* __restrict__ status) {
     const int vec = d / 8;   // 16-byte vectors per row
     const int64_t total = (int64_t)M_pad * vec;
     for (int64_t x = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; x < total; x += (int64_t)gridDim.x * blockDim.x) {
         const int m = (int)(x / vec), k = (int)(x % vec);
+        const int r = m < M ? checked_index(rows[m], N) : -1;
         uint4 val = make_uint4(0, 0, 0, 0);
-        if (m < M) val = reinterpret_cast<const uint4*>(H + (int64_t)rows[m] * d)[k];
+        if (r >= 0) val = reinterpret_cast<const uint4*>(H + (int64_t)r * d)[k];
         reinterpret_cast<uint4*>(Hg + (int64_t)m * d)[k] = val;
-        if (k == 0) tg[m] = m < M && targets ? targets[rows[m]] : -1;   // no targets: -1
+        if (k == 0) {
+            const int t = r >= 0 && targets ? checked_index(targets[r], V) : -1;
+            if (m < M && (r < 0 || (targets && t < 0))) flag_bounds(status);
+            tg[m] = t;
+        }
     }
 }
 
@@ -300,22 +309,23 @@ static mw_status lm_partials(const void* W, int M, int d, int V, const void* Hg,
     return launch_status();
 }
 
-static mw_status lm_gather(const void* H, const int32_t* targets, const int32_t* rows, int M, int d, void* Hg,
-                           int32_t* tg, cudaStream_t s) {
+static mw_status lm_gather(const void* H, const int32_t* targets, const int32_t* rows, int M, int N, int d, int V,
+                           void* Hg, int32_t* tg, int32_t* status, cudaStream_t s) {
     const int64_t M_pad = ceil_div(M, BM) * BM;
     const int64_t vec = M_pad * (d / 8);
     count_launches(1);
     k_lm_gather<<<(unsigned)std::min<int64_t>(ceil_div(vec, 256), 152 * 32), 256, 0, s>>>(
-        M, (int)M_pad, d, (const __nv_bfloat16*)H, targets, rows, (__nv_bfloat16*)Hg, tg);
+        M, (int)M_pad, d, N, V, (const __nv_bfloat16*)H, targets, rows, (__nv_bfloat16*)Hg, tg, status);
     return launch_status();
 }
 
 int lm_ref_vocab(int V) { return std::min(V, kRefVocab); }
 
-mw_status lm_ref_tc(const void* H, const void* W, const int32_t* targets, const int32_t* rows, int M, int d, int V,
-                    void* Hg, int32_t* tg, float2* part, float* zt, float4* par, int32_t* status, cudaStream_t s) {
+mw_status lm_ref_tc(const void* H, const void* W, const int32_t* targets, const int32_t* rows, int M, int N, int d,
+                    int V, void* Hg, int32_t* tg, float2* part, float* zt, float4* par, int32_t* status,
+                    cudaStream_t s) {
     if (M == 0) return MW_OK;
-    mw_status st = lm_gather(H, targets, rows, M, d, Hg, tg, s);
+    mw_status st = lm_gather(H, targets, rows, M, N, d, V, Hg, tg, status, s);
     LmPlan q;
     if (st == MW_OK) st = lm_partials(W, M, d, lm_ref_vocab(V), Hg, tg, part, zt, status, s, q);
     if (st != MW_OK) return st;

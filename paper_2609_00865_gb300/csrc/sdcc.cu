@@ -126,30 +126,34 @@ __device__ __forceinline__ void smerge(float& m, float& l, float m2, float l2) {
     m = mn;
 }
 
-// Stage the rows of up to n pairs (zero rows past M) into shared memory.
+// Stage the rows of up to n pairs into shared memory: zero past M, and zero
+// for a row index outside [0, N), which raises the bounds flag.
 template <typename Tin>
 __device__ __forceinline__ void stage_rows(float* dst, const Tin* __restrict__ H, const int32_t* __restrict__ rows,
-                                           int m0, int n, int M, int d) {
+                                           int m0, int n, int M, int N, int d, int32_t* status) {
     for (int x = threadIdx.x; x < n * d; x += blockDim.x) {
         const int r = x / d, k = x % d;
-        dst[x] = (m0 + r < M) ? ld_f(H + (int64_t)rows[m0 + r] * d + k) : 0.f;
+        const int t = m0 + r < M ? checked_index(rows[m0 + r], N) : 0;
+        if (t < 0 && k == 0) flag_bounds(status);
+        dst[x] = (m0 + r < M && t >= 0) ? ld_f(H + (int64_t)t * d + k) : 0.f;
     }
 }
 
 // grid ceil(M / KR), block 256; writes kl[m], lseT[m], lseS[m].
 template <typename Tin>
-__global__ void __launch_bounds__(256) k_kl_fwd_simt(int M, int d, int Vocab, const Tin* __restrict__ HT,
-                                                    const int32_t* __restrict__ rowsT, const Tin* __restrict__ HS,
-                                                    const int32_t* __restrict__ rowsS, const Tin* __restrict__ W,
-                                                    float* __restrict__ kl, float* __restrict__ lseT,
-                                                    float* __restrict__ lseS) {
+__global__ void __launch_bounds__(256) k_kl_fwd_simt(int M, int N_T, int N_S, int d, int Vocab,
+                                                    const Tin* __restrict__ HT, const int32_t* __restrict__ rowsT,
+                                                    const Tin* __restrict__ HS, const int32_t* __restrict__ rowsS,
+                                                    const Tin* __restrict__ W, float* __restrict__ kl,
+                                                    float* __restrict__ lseT, float* __restrict__ lseS,
+                                                    int32_t* __restrict__ status) {
     extern __shared__ float sh[];
     float* ht = sh;            // [KR][d]
     float* hs = sh + KR * d;   // [KR][d]
     __shared__ float red[KR][8][5];
     const int m0 = blockIdx.x * KR;
-    stage_rows(ht, HT, rowsT, m0, KR, M, d);
-    stage_rows(hs, HS, rowsS, m0, KR, M, d);
+    stage_rows(ht, HT, rowsT, m0, KR, M, N_T, d, status);
+    stage_rows(hs, HS, rowsS, m0, KR, M, N_S, d, status);
     __syncthreads();
     TStat t[KR];
     float ms[KR], ls[KR];
@@ -226,19 +230,20 @@ __global__ void k_kl_loss(int M, const float* __restrict__ kl, float lam, float*
 
 // dHS: grid ceil(M / KH), block 256 (d <= 256); vocabulary tiles of 256.
 template <typename Tin>
-__global__ void __launch_bounds__(256) k_kl_dh_simt(int M, int d, int Vocab, const Tin* __restrict__ HT,
-                                                   const int32_t* __restrict__ rowsT, const Tin* __restrict__ HS,
-                                                   const int32_t* __restrict__ rowsS, const Tin* __restrict__ W,
-                                                   const float* __restrict__ lseT, const float* __restrict__ lseS,
-                                                   float c, int accumulate, Tin* __restrict__ dHS) {
+__global__ void __launch_bounds__(256) k_kl_dh_simt(int M, int N_T, int N_S, int d, int Vocab,
+                                                   const Tin* __restrict__ HT, const int32_t* __restrict__ rowsT,
+                                                   const Tin* __restrict__ HS, const int32_t* __restrict__ rowsS,
+                                                   const Tin* __restrict__ W, const float* __restrict__ lseT,
+                                                   const float* __restrict__ lseS, float c, int accumulate,
+                                                   Tin* __restrict__ dHS, int32_t* __restrict__ status) {
     extern __shared__ float sh[];
     float* ht = sh;                // [KH][d]
     float* hs = sh + KH * d;       // [KH][d]
     float* dzs = hs + KH * d;      // [KH][256]
     __shared__ float slt[KH], sls[KH], sc[KH];
     const int m0 = blockIdx.x * KH;
-    stage_rows(ht, HT, rowsT, m0, KH, M, d);
-    stage_rows(hs, HS, rowsS, m0, KH, M, d);
+    stage_rows(ht, HT, rowsT, m0, KH, M, N_T, d, status);
+    stage_rows(hs, HS, rowsS, m0, KH, M, N_S, d, status);
     if (threadIdx.x < KH) {
         const bool ok = m0 + threadIdx.x < M;
         slt[threadIdx.x] = ok ? lseT[m0 + threadIdx.x] : 0.f;
@@ -286,7 +291,7 @@ __global__ void __launch_bounds__(256) k_kl_dh_simt(int M, int d, int Vocab, con
     if (threadIdx.x < d) {
 #pragma unroll
         for (int r = 0; r < KH; ++r)
-            if (m0 + r < M) {
+            if (m0 + r < M && checked_index(rowsS[m0 + r], N_S) >= 0) {
                 Tin* dst = dHS + (int64_t)rowsS[m0 + r] * d + threadIdx.x;
                 st_f(dst, accumulate ? ld_f(dst) + acc[r] : acc[r]);
             }
@@ -295,11 +300,12 @@ __global__ void __launch_bounds__(256) k_kl_dh_simt(int M, int d, int Vocab, con
 
 // dW: grid ceil(Vocab / KWV), block 256 (d <= 256).
 template <typename Tin>
-__global__ void __launch_bounds__(256) k_kl_dw_simt(int M, int d, int Vocab, const Tin* __restrict__ HT,
-                                                   const int32_t* __restrict__ rowsT, const Tin* __restrict__ HS,
-                                                   const int32_t* __restrict__ rowsS, const Tin* __restrict__ W,
-                                                   const float* __restrict__ lseT, const float* __restrict__ lseS,
-                                                   float c, int accumulate, float* __restrict__ dW) {
+__global__ void __launch_bounds__(256) k_kl_dw_simt(int M, int N_T, int N_S, int d, int Vocab,
+                                                   const Tin* __restrict__ HT, const int32_t* __restrict__ rowsT,
+                                                   const Tin* __restrict__ HS, const int32_t* __restrict__ rowsS,
+                                                   const Tin* __restrict__ W, const float* __restrict__ lseT,
+                                                   const float* __restrict__ lseS, float c, int accumulate,
+                                                   float* __restrict__ dW, int32_t* __restrict__ status) {
     extern __shared__ float sh[];
     float* ws = sh;                 // [KWV][d]
     float* ht = sh + KWV * d;       // [KWR][d]
@@ -316,8 +322,8 @@ __global__ void __launch_bounds__(256) k_kl_dw_simt(int M, int d, int Vocab, con
     for (int q = 0; q < KWV; ++q) acc[q] = 0.f;
     for (int m0 = 0; m0 < M; m0 += KWR) {
         __syncthreads();
-        stage_rows(ht, HT, rowsT, m0, KWR, M, d);
-        stage_rows(hs, HS, rowsS, m0, KWR, M, d);
+        stage_rows(ht, HT, rowsT, m0, KWR, M, N_T, d, status);
+        stage_rows(hs, HS, rowsS, m0, KWR, M, N_S, d, status);
         if (threadIdx.x < KWR) {
             const bool ok = m0 + threadIdx.x < M;
             slt[threadIdx.x] = ok ? lseT[m0 + threadIdx.x] : 0.f;
@@ -363,16 +369,16 @@ __global__ void __launch_bounds__(256) k_kl_dw_simt(int M, int d, int Vocab, con
 
 template <typename Tin>
 mw_status kl_fwd_t(const void* HT, const int32_t* rowsT, const void* HS, const int32_t* rowsS, int M,
-                   const void* W, int d, int Vocab, float lam, float* kl, float* loss, float* lseT, float* lseS,
-                   cudaStream_t s) {
+                   const void* W, int N_T, int N_S, int d, int Vocab, float lam, float* kl, float* loss, float* lseT,
+                   float* lseS, int32_t* status, cudaStream_t s) {
     const size_t smem = sizeof(float) * 2 * KR * d;
     mw_status st = cuda_status(
         cudaFuncSetAttribute(k_kl_fwd_simt<Tin>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
     if (st != MW_OK) return st;
     count_launches(1);
-    k_kl_fwd_simt<Tin><<<(unsigned)ceil_div(M, KR), 256, smem, s>>>(M, d, Vocab, (const Tin*)HT, rowsT,
+    k_kl_fwd_simt<Tin><<<(unsigned)ceil_div(M, KR), 256, smem, s>>>(M, N_T, N_S, d, Vocab, (const Tin*)HT, rowsT,
                                                                     (const Tin*)HS, rowsS, (const Tin*)W, kl,
-                                                                    lseT, lseS);
+                                                                    lseT, lseS, status);
     if ((st = launch_status()) != MW_OK) return st;
     count_launches(1);
     k_kl_loss<<<1, 1024, 0, s>>>(M, kl, lam, loss);
@@ -381,8 +387,8 @@ mw_status kl_fwd_t(const void* HT, const int32_t* rowsT, const void* HS, const i
 
 template <typename Tin>
 mw_status kl_bwd_t(const void* HT, const int32_t* rowsT, const void* HS, const int32_t* rowsS, int M,
-                   const void* W, int N_S, int d, int Vocab, float c, const float* lseT, const float* lseS,
-                   int accumulate, void* dHS, float* dW, cudaStream_t s) {
+                   const void* W, int N_T, int N_S, int d, int Vocab, float c, const float* lseT, const float* lseS,
+                   int accumulate, void* dHS, float* dW, int32_t* status, cudaStream_t s) {
     mw_status st = MW_OK;
     if (!accumulate && (st = cuda_status(cudaMemsetAsync(dHS, 0, sizeof(Tin) * (size_t)N_S * d, s))) != MW_OK)
         return st;
@@ -397,12 +403,13 @@ mw_status kl_bwd_t(const void* HT, const int32_t* rowsT, const void* HS, const i
                                                (int)smem_w))) != MW_OK)
         return st;
     count_launches(2);
-    k_kl_dh_simt<Tin><<<(unsigned)ceil_div(M, KH), 256, smem_h, s>>>(M, d, Vocab, (const Tin*)HT, rowsT,
+    k_kl_dh_simt<Tin><<<(unsigned)ceil_div(M, KH), 256, smem_h, s>>>(M, N_T, N_S, d, Vocab, (const Tin*)HT, rowsT,
                                                                      (const Tin*)HS, rowsS, (const Tin*)W, lseT,
-                                                                     lseS, c, accumulate, (Tin*)dHS);
-    k_kl_dw_simt<Tin><<<(unsigned)ceil_div(Vocab, KWV), 256, smem_w, s>>>(M, d, Vocab, (const Tin*)HT, rowsT,
-                                                                          (const Tin*)HS, rowsS, (const Tin*)W,
-                                                                          lseT, lseS, c, accumulate, dW);
+                                                                     lseS, c, accumulate, (Tin*)dHS, status);
+    k_kl_dw_simt<Tin><<<(unsigned)ceil_div(Vocab, KWV), 256, smem_w, s>>>(M, N_T, N_S, d, Vocab, (const Tin*)HT,
+                                                                          rowsT, (const Tin*)HS, rowsS,
+                                                                          (const Tin*)W, lseT, lseS, c, accumulate,
+                                                                          dW, status);
     return launch_status();
 }
 
@@ -426,8 +433,8 @@ extern "C" mw_status mw_final_walk(const mw_vis_layout* L, const void* vis, int3
 namespace mw {
 bool lm_bwd_tc_supported(int d);
 int64_t kl_tc_ws(int M, int d);
-mw_status kl_fwd_tc(const void*, const int32_t*, const void*, const int32_t*, int, const void*, int, int, float*,
-                    void*, cudaStream_t);
+mw_status kl_fwd_tc(const void*, const int32_t*, const void*, const int32_t*, int, const void*, int, int, int, int,
+                    float*, void*, cudaStream_t);
 mw_status kl_bwd_tc(const int32_t*, int, const void*, int, int, int, float, void*, int, void*, float*,
                     cudaStream_t);
 int32_t* kl_tc_status(int M, int d, void* ws);
@@ -446,8 +453,10 @@ static mw_status kl_args(int M, int N_T, int N_S, int d, int Vocab, int dtype) {
     return MW_OK;
 }
 
-// Workspace: CUDA cores, lse of the teacher and of the student per pair;
-// tensor cores, the fused passes' arrays (see kl_tc_ws).
+// Workspace: CUDA cores, lse of the teacher and of the student per pair and
+// the status words; tensor cores, the fused passes' arrays (see kl_tc_ws).
+static int32_t* kl_simt_status(int M, void* ws) { return at<int32_t>(ws, 2 * align256(4 * (int64_t)M)); }
+
 extern "C" mw_status mw_forward_kl_ws(int M, int d, int Vocab, int dtype, size_t* bytes) {
     if (!bytes) return MW_EINVAL;
     mw_status st = kl_args(M, M, M, d, Vocab, dtype);
@@ -460,13 +469,12 @@ extern "C" mw_status mw_forward_kl_check_status(int M, int d, int Vocab, int dty
     mw_status st = kl_args(M, M, M, d, Vocab, dtype);
     if (st != MW_OK) return st;
     if (!ws) return MW_EINVAL;
-    if (!kl_tc(d, dtype)) return cuda_status(cudaStreamSynchronize((cudaStream_t)stream));
     int32_t h[8];
-    if ((st = cuda_status(cudaMemcpyAsync(h, kl_tc_status(M, d, ws), sizeof(h), cudaMemcpyDeviceToHost,
-                                          (cudaStream_t)stream))) != MW_OK)
+    if ((st = cuda_status(cudaMemcpyAsync(h, kl_tc(d, dtype) ? kl_tc_status(M, d, ws) : kl_simt_status(M, ws),
+                                          sizeof(h), cudaMemcpyDeviceToHost, (cudaStream_t)stream))) != MW_OK)
         return st;
     if ((st = cuda_status(cudaStreamSynchronize((cudaStream_t)stream))) != MW_OK) return st;
-    return h[1] ? MW_ETIMEOUT : MW_OK;
+    return h[1] ? MW_ETIMEOUT : h[0] ? MW_EDEVICE : MW_OK;
 }
 
 extern "C" mw_status mw_forward_kl_fwd(const void* HT, const int32_t* rows_T, const void* HS, const int32_t* rows_S,
@@ -480,20 +488,23 @@ extern "C" mw_status mw_forward_kl_fwd(const void* HT, const int32_t* rows_T, co
     cudaStream_t s = (cudaStream_t)stream;
     float* lseT = at<float>(ws, 0);
     float* lseS = at<float>(ws, align256(4 * (int64_t)M));
+    int32_t* status = kl_tc(d, dtype) ? kl_tc_status(M, d, ws) : kl_simt_status(M, ws);
+    if ((st = cuda_status(cudaMemsetAsync(status, 0, 32, s))) != MW_OK) return st;
     if (M == 0) {
         count_launches(1);
         k_kl_loss<<<1, 1024, 0, s>>>(0, kl, lam, loss);
         return launch_status();
     }
     if (kl_tc(d, dtype)) {
-        if ((st = kl_fwd_tc(HT, rows_T, HS, rows_S, M, W, d, Vocab, kl, ws, s)) != MW_OK) return st;
+        if ((st = kl_fwd_tc(HT, rows_T, HS, rows_S, M, W, N_T, N_S, d, Vocab, kl, ws, s)) != MW_OK) return st;
         count_launches(1);
         k_kl_loss<<<1, 1024, 0, s>>>(M, kl, lam, loss);
         return launch_status();
     }
-    return dtype == MW_F32 ? kl_fwd_t<float>(HT, rows_T, HS, rows_S, M, W, d, Vocab, lam, kl, loss, lseT, lseS, s)
-                           : kl_fwd_t<__nv_bfloat16>(HT, rows_T, HS, rows_S, M, W, d, Vocab, lam, kl, loss, lseT,
-                                                     lseS, s);
+    return dtype == MW_F32 ? kl_fwd_t<float>(HT, rows_T, HS, rows_S, M, W, N_T, N_S, d, Vocab, lam, kl, loss, lseT,
+                                             lseS, status, s)
+                           : kl_fwd_t<__nv_bfloat16>(HT, rows_T, HS, rows_S, M, W, N_T, N_S, d, Vocab, lam, kl, loss,
+                                                     lseT, lseS, status, s);
 }
 
 extern "C" mw_status mw_forward_kl_bwd(const void* HT, const int32_t* rows_T, const void* HS, const int32_t* rows_S,
@@ -510,10 +521,12 @@ extern "C" mw_status mw_forward_kl_bwd(const void* HT, const int32_t* rows_T, co
     const float* lseS = at<float>(ws, align256(4 * (int64_t)M));
     const float c = lam * dloss;
     if (kl_tc(d, dtype)) return kl_bwd_tc(rows_S, M, W, N_S, d, Vocab, c, ws, accumulate, dHS, dW, s);
+    int32_t* status = kl_simt_status(M, ws);   // reset by the forward; the backward adds to it
     return dtype == MW_F32
-               ? kl_bwd_t<float>(HT, rows_T, HS, rows_S, M, W, N_S, d, Vocab, c, lseT, lseS, accumulate, dHS, dW, s)
-               : kl_bwd_t<__nv_bfloat16>(HT, rows_T, HS, rows_S, M, W, N_S, d, Vocab, c, lseT, lseS, accumulate,
-                                         dHS, dW, s);
+               ? kl_bwd_t<float>(HT, rows_T, HS, rows_S, M, W, N_T, N_S, d, Vocab, c, lseT, lseS, accumulate, dHS,
+                                 dW, status, s)
+               : kl_bwd_t<__nv_bfloat16>(HT, rows_T, HS, rows_S, M, W, N_T, N_S, d, Vocab, c, lseT, lseS,
+                                         accumulate, dHS, dW, status, s);
 }
 
 extern "C" mw_status mw_diverging_rows(const mw_vis_layout* L, const void* vis, uint8_t* out, void* stream) {

@@ -54,7 +54,14 @@ extern "C" const char* mw_status_str(int s) {
 }
 
 extern "C" int mw_last_cuda_error(void) { return g_last_cuda_error; }
-extern "C" int mw_abi_version(void) { return 6; }
+extern "C" int mw_abi_version(void) { return 7; }
+extern "C" int mw_build_flags(void) {
+#ifdef MW_DEBUG
+    return MW_BUILD_DEBUG;
+#else
+    return 0;
+#endif
+}
 extern "C" uint64_t mw_kernel_launches(void) { return (uint64_t)g_launches.load(std::memory_order_relaxed); }
 
 static mw_status check_shape(int n_traj, const int32_t* cu, int n_junc, const int32_t* jt,
@@ -185,6 +192,8 @@ struct BuildArgs {
     int32_t* bwd_cnt;       // [n_tiles]
     unsigned long long* tpairs;   // [n_tiles] visible pairs per k-tile
     int32_t* bsum;          // [2][n_scan_blocks] per-block count sums, then exclusive offsets
+    int32_t* status;        // device status words (debug index checks)
+    int64_t n_tri, n_keymask;
 };
 
 __device__ __forceinline__ int find_traj(const int32_t* off, int n, int64_t t) {
@@ -253,7 +262,8 @@ __global__ void k_init_tokens(BuildArgs a) {
 __global__ void k_scatter_spans(BuildArgs a) {
     for (int s = blockIdx.x; s < a.n_spans; s += gridDim.x) {
         int ga = a.spans[3 * s], gb = a.spans[3 * s + 1], J = a.spans[3 * s + 2];
-        for (int t = ga + threadIdx.x; t < gb; t += blockDim.x) atomicMin(&a.omega[t], J);
+        for (int t = ga + threadIdx.x; t < gb; t += blockDim.x)
+            if (MW_DBG_IN(t, a.total, a.status, 101)) atomicMin(&a.omega[t], J);
     }
 }
 
@@ -307,7 +317,8 @@ __global__ void __launch_bounds__(256) k_tile_stats(BuildArgs a) {
             const int j = kt * MW_TILE + 32 * q + lane;
             wd[q] = __ballot_sync(0xffffffffu, j < T && om[q] > Js && j < Jn);
         }
-        if (lane == 0) km[(int64_t)s * nt] = make_uint4(wd[0], wd[1], wd[2], wd[3]);
+        if (lane == 0 && MW_DBG_IN(a.traj_km[b] + kt + (int64_t)s * nt, a.n_keymask, a.status, 105))
+            km[(int64_t)s * nt] = make_uint4(wd[0], wd[1], wd[2], wd[3]);
     }
     if (lane == 0) {
         *reinterpret_cast<int4*>(a.tstat + 4 * g) =
@@ -539,7 +550,8 @@ __global__ void k_fill(BuildArgs a) {
         int kt = k0 + lane;
         int c = kt <= t ? tri[(int64_t)t * (t + 1) / 2 + kt] : MW_TILE_EMPTY;
         uint32_t m = __ballot_sync(0xffffffffu, c != MW_TILE_EMPTY);
-        if (c != MW_TILE_EMPTY) a.fwd_idx[base + __popc(m & lt)] = (kt << 4) | c;
+        if (c != MW_TILE_EMPTY && MW_DBG_IN(base + __popc(m & lt), a.n_tri, a.status, 102))
+            a.fwd_idx[base + __popc(m & lt)] = (kt << 4) | c;
         base += __popc(m);
     }
     // the column's non-EMPTY tiles are exactly the q-tiles t .. qend - 1
@@ -547,7 +559,8 @@ __global__ void k_fill(BuildArgs a) {
     base = a.bwd_ptr[g];
     const int4 st = tile_stat(a.tstat, g);
     const int qend = max(t + 1, min(nt, (min(st.y, T) + MW_TILE - 1) / MW_TILE));
-    for (int qt = t + lane; qt < qend; qt += 32) a.bwd_idx[base + qt - t] = (qt << 4) | tile_class(qt, t, T, st);
+    for (int qt = t + lane; qt < qend; qt += 32)
+        if (MW_DBG_IN(base + qt - t, a.n_tri, a.status, 103)) a.bwd_idx[base + qt - t] = (qt << 4) | tile_class(qt, t, T, st);
 }
 
 // Compact views. An exclusive prefix popcount of the segment's view bits,
@@ -626,7 +639,7 @@ __global__ void __launch_bounds__(256) k_compact_map(BuildArgs a) {
         int32_t r = -1;
         if ((word >> bit) & 1u) {
             r = tp[tl] + (int)pre + __popc(word & ((1u << bit) - 1u));
-            src[r] = (c0 + tl) * MW_TILE + jj;
+            if (MW_DBG_IN(r, (int64_t)nt * MW_TILE, a.status, 104)) src[r] = (c0 + tl) * MW_TILE + jj;
         }
         pos[(int64_t)(c0 + tl) * MW_TILE + jj] = r;
     }
@@ -715,6 +728,7 @@ struct EventArgs {
     int32_t* cpos;
     int32_t* csrc;
     unsigned long long* pairs;
+    int32_t* status;         // device status words (debug index checks)
 };
 
 __global__ void __launch_bounds__(1024) k_event_views(EventArgs a) {
@@ -743,14 +757,15 @@ __global__ void __launch_bounds__(1024) k_event_views(EventArgs a) {
         if (s >= 1) {
             const int32_t* jt = a.jtab + 4 * (int64_t)(g0 - b + s - 1);   // this trajectory's event s - 1
             for (int q = jt[0]; q < jt[1]; ++q)
-                for (int j = a.spans[2 * q] + t; j < a.spans[2 * q + 1]; j += blockDim.x) flag[j - tok0] = s;
+                for (int j = a.spans[2 * q] + t; j < a.spans[2 * q + 1]; j += blockDim.x)
+                    if (MW_DBG_IN(j - tok0, T, a.status, 111)) flag[j - tok0] = s;
             __syncthreads();
             // ordered compaction of view_{s-1} without the keys flagged s
             const int Lp = a.seg_len[g0 + s - 1];
             for (int c0 = 0; c0 < Lp; c0 += blockDim.x) {
                 const int c = c0 + t;
                 const int key = c < Lp ? a.csrc[prev + c] : -1;
-                const int keep = c < Lp && flag[key] != s;
+                const int keep = c < Lp && MW_DBG_IN(key, T, a.status, 112) && flag[key] != s;
                 const unsigned bal = __ballot_sync(0xffffffffu, keep);
                 if (lane == 0) wsum[w] = __popc(bal);
                 __syncthreads();
@@ -759,17 +774,22 @@ __global__ void __launch_bounds__(1024) k_event_views(EventArgs a) {
                     before += q < w ? wsum[q] : 0;
                     total += wsum[q];
                 }
-                if (keep) a.csrc[base + n + before + __popc(bal & ((1u << lane) - 1u))] = key;
+                if (keep && MW_DBG_IN(n + before + __popc(bal & ((1u << lane) - 1u)), (int64_t)nt * MW_TILE,
+                                      a.status, 113))
+                    a.csrc[base + n + before + __popc(bal & ((1u << lane) - 1u))] = key;
                 n += total;
                 __syncthreads();
             }
             for (int q = jt[2]; q < jt[3]; ++q) {
                 const int ga = a.spans[2 * q], gb = a.spans[2 * q + 1];
-                for (int j = ga + t; j < gb; j += blockDim.x) a.csrc[base + n + (j - ga)] = (int)(j - tok0);
+                for (int j = ga + t; j < gb; j += blockDim.x)
+                    if (MW_DBG_IN(n + (j - ga), (int64_t)nt * MW_TILE, a.status, 114))
+                        a.csrc[base + n + (j - ga)] = (int)(j - tok0);
                 n += gb - ga;
             }
         }
-        for (int r = lo + t; r < hi; r += blockDim.x) a.csrc[base + n + (r - lo)] = r;
+        for (int r = lo + t; r < hi; r += blockDim.x)
+            if (MW_DBG_IN(n + (r - lo), (int64_t)nt * MW_TILE, a.status, 115)) a.csrc[base + n + (r - lo)] = r;
         const int R = hi - lo;
         pairs += (unsigned long long)R * (unsigned long long)n + (unsigned long long)R * (R + 1) / 2;
         n += R;
@@ -777,7 +797,8 @@ __global__ void __launch_bounds__(1024) k_event_views(EventArgs a) {
         for (int c = n + t; c < end; c += blockDim.x) a.csrc[base + c] = -1;
         if (t == 0) a.seg_len[g0 + s] = n;
         __syncthreads();
-        for (int c = t; c < n; c += blockDim.x) a.cpos[base + a.csrc[base + c]] = c;
+        for (int c = t; c < n; c += blockDim.x)
+            if (MW_DBG_IN(a.csrc[base + c], T, a.status, 116)) a.cpos[base + a.csrc[base + c]] = c;
         __syncthreads();
     }
     if (t == 0) {
@@ -938,6 +959,9 @@ extern "C" mw_status mw_build_visibility(const mw_vis_layout* L, const int32_t* 
     a.bwd_cnt = at<int32_t>(ws, L->ws_off_cnt) + n_tiles;
     a.tpairs = reinterpret_cast<unsigned long long*>(at<int32_t>(ws, L->ws_off_cnt) + 2 * n_tiles);
     a.bsum = at<int32_t>(ws, L->ws_off_cnt) + 4 * n_tiles;
+    a.status = at<int32_t>(vis, L->off_status);
+    a.n_tri = L->n_tri;
+    a.n_keymask = L->n_keymask;
 
     count_launches((a.total > 0 ? 1 + (L->n_spans > 0) : 0) + (n_tiles > 0 ? 3 : 0) + 1 + 4 * (n_tiles > 0));
     if (a.total > 0) {
@@ -1049,8 +1073,10 @@ extern "C" mw_status mw_build_views_events(const mw_vis_layout* L, const int32_t
     a.traj_tok = at<int32_t>(vis, L->off_traj_tok);
     a.traj_seg = at<int32_t>(vis, L->off_traj_seg);
     a.seg_start = at<int32_t>(vis, L->off_seg_start);
+    a.status = at<int32_t>(vis, L->off_status);
     EventArgs e;
     e.n_traj = n_traj;
+    e.status = a.status;
     e.traj_tok = at<int32_t>(vis, L->off_traj_tok);
     e.traj_tile = at<int32_t>(vis, L->off_traj_tile);
     e.traj_seg = at<int32_t>(vis, L->off_traj_seg);

@@ -39,6 +39,20 @@ def test_header_symbols_exported():
     assert declared <= set(L.exported_names())
 
 
+def test_debug_library_exports_the_same_symbols():
+    """libmw_debug.so (-DMW_DEBUG: index checks in the kernels) carries the
+    same ABI as libmw.so and says which it is through mw_build_flags."""
+    L, h = _lib()
+    from paper_2609_00865_gb300 import build as B
+    if not os.path.exists(B.LIB_DEBUG):
+        B.build(debug=True)
+    d = ctypes.CDLL(B.LIB_DEBUG)
+    for name in _declared():
+        assert hasattr(d, name), name
+    assert (h.mw_build_flags(), d.mw_build_flags()) == (0, 1)
+    assert d.mw_abi_version() == h.mw_abi_version()
+
+
 def test_status_strings_and_version():
     L, h = _lib()
     assert h.mw_status_str(0) == b"ok"
