@@ -46,8 +46,29 @@ def _qkv(T, Hq, Hkv, Dh, seed, dtype):
 def _host(v):
     if torch.is_tensor(v):
         return v.detach().cpu()
+    if isinstance(v, (list, tuple)):   # per-trajectory arrays (the class triangles)
+        parts = [np.asarray(x, dtype=np.int64).reshape(-1) for x in v]
+        return torch.as_tensor(np.concatenate(parts) if parts else np.zeros(0, np.int64))
     a = np.asarray(v)
     return torch.as_tensor(a.astype(np.int64) if a.dtype.kind == "u" else a)
+
+
+def _views(arrs, seqlens, junctions_per_traj):
+    """The builder's arrays with csrc cut to its defined part: each segment's
+    entries up to the end of its last compact tile (the rest of its 128 nt_b
+    block is left unset by design)."""
+    out = dict(arrs)
+    csrc = np.array(arrs["csrc"], copy=True)
+    g, off = 0, 0
+    for T, K in zip(seqlens, junctions_per_traj):
+        block = (T + 127) // 128 * 128
+        for _ in range(1 + K):
+            end = (int(arrs["seg_len"][g]) + 127) // 128 * 128
+            csrc[off + end: off + block] = -2
+            g += 1
+            off += block
+    out["csrc"] = csrc
+    return out
 
 
 def _cpu(d):
@@ -61,7 +82,7 @@ def case_build():
         vis = mw.build_visibility(seqlens, edits)
         torch.cuda.synchronize()
         vis.check_status()
-        for k, v in vis.arrays().items():
+        for k, v in _views(vis.arrays(), seqlens, [len(e) for e in edits]).items():
             out[f"{name}.{k}"] = v
     return out
 
@@ -113,7 +134,8 @@ def case_events():
     dQ, dK, dV = mw.masked_attn_bwd(vis, q, k, v, O, do, LSE, 128 ** -0.5)
     torch.cuda.synchronize()
     vis.check_status()
-    out = {f"views.{k_}": v_ for k_, v_ in vis.arrays().items()}
+    arrs = _views(vis.arrays(), seqlens, [len(e) for e in events])
+    out = {f"views.{k_}": v_ for k_, v_ in arrs.items()}
     out.update(O=O, LSE=LSE, dQ=dQ, dK=dK, dV=dV)
     return out
 
