@@ -51,16 +51,16 @@ def _peaks():
 # value it had when the counters were taken.
 TRAFFIC = {
     (4, "mw_logprob_loss_bwd"): {
-        "bytes": 457216 + (81266843648 + 14094951168) + (807815424 + 247198720),   # par, dW pass, dH from E
+        "bytes": 457216 + (86640796672 + 14105479168) + (807975680 + 246783744),   # par, dW pass, dH from E
         "source": "paper_2609_00865_gb300/csrc/lmhead_bwd_tc.cu",
-        "sha256": "e37a7e91c915817da7a63c8ebadd255f857d5416446f4690c688316990724030",
+        "sha256": "e40ea9e5cf9398f20ba4c0508ee327990b45deed51f17997f7c6d5ea1739b4e8",
     },
     (4, "mw_masked_attn_bwd"): {
         # lsd, compact gather, dQ (main + junction items), dK/dV, per-key reduce
-        "bytes": (1894618880 + 28330240) + (462878976 + 700409600) + (4141256448 + 902114560) +
-                 (515859456 + 6792448) + (4016977920 + 1467208704) + (1502151680 + 262355968),
+        "bytes": (1894677760 + 28395264) + (459507712 + 700083456) + (4147593216 + 903136512) +
+                 (515563520 + 6713600) + (4001377024 + 1467339776) + (1502124032 + 262418176),
         "source": "paper_2609_00865_gb300/csrc/attn_tc.cu",
-        "sha256": "2ff43b57526d25e439966e726fc91f0d028cf69849fa1aab68c8828c6d12219f",
+        "sha256": "3cad1bdc5f9c23db994b04f0625d5e9263e4bb8f963b2293c31a0e24f726bf06",
     },
 }
 
@@ -572,7 +572,7 @@ class SdccStep(Step):
 
 # ----------------------------------------------------------------------------- reference arm (CPU oracle)
 
-def cpu_sample(w, budget_s=15.0, seed=5):
+def cpu_sample(w, budget_s=15.0, seed=5, detail=False):
     """Time the oracle on a bounded sample of loss rows of this workload
     (rows drawn by ``seed``: the cost of a row grows with its view, so every
     sample draws its own rows).
@@ -580,7 +580,8 @@ def cpu_sample(w, budget_s=15.0, seed=5):
     Per sampled row: attention fwd and the row's whole attention backward over
     all query heads (its segment's compact view: dQ and its contributions to
     dK and dV), LM-head log-prob over the full vocabulary and the dH/dW
-    contributions of that row. Returns (tokens/s, cores, description).
+    contributions of that row. Returns (tokens/s, cores, description), or
+    with ``detail`` (tokens, seconds, cores, parts).
     """
     import numpy as np
     import torch
@@ -633,6 +634,8 @@ def cpu_sample(w, budget_s=15.0, seed=5):
         parts = one_batch(np.sort(rng.choice(pool, size=batch, replace=False)))
         done += batch
     dt = time.perf_counter() - t0
+    if detail:
+        return done, dt, cores, parts
     return done / dt, cores, f"{done} sampled scored tokens ({' + '.join(parts)}), {dt:.1f} s"
 
 
@@ -641,12 +644,16 @@ def run_reference(args, rank, world):
         return
     w = make_workload(args.config, args.K, args.f, n_traj=args.n_traj, pin=False,   # the oracle runs on the host
                       rope=args.rope)
-    vals = []
+    # every step samples its own rows; the value is all timed steps' tokens
+    # over their time (whole-job throughput, as the bench's own CPU baseline)
+    tok, sec = 0, 0.0
     for i in range(args.warmup + args.steps):
-        v, cores, desc = cpu_sample(w, budget_s=args.cpu_seconds / max(1, args.steps), seed=5 + i)
+        done, dt, cores, parts = cpu_sample(w, budget_s=args.cpu_seconds / max(1, args.steps), seed=5 + i,
+                                            detail=True)
         if i >= args.warmup:
-            vals.append(v)
-    v = sorted(vals)[len(vals) // 2]
+            tok, sec = tok + done, sec + dt
+    v = tok / sec
+    desc = f"{tok} sampled scored tokens over {args.steps} steps ({' + '.join(parts)}), {sec:.1f} s"
     scored = int(w["rows"].numel()) if "rows" in w else w["record"].total
     # one whole step at the sampled rate (extrapolated: each timed step is a sample)
     line = {"impl": "reference", "metric": METRIC, "value": v, "unit": "tokens/s", "n_gpus": world,

@@ -73,3 +73,33 @@ def test_reference_arm_rank1_does_no_work(monkeypatch, capsys):
         config, K, f, n_traj, warmup, steps, cpu_seconds = 2, 8, 0.6, None, 1, 1, 1.0
     bench.run_reference(A(), rank=1, world=2)
     assert capsys.readouterr().out == ""
+
+
+def test_reference_arm_reports_whole_job_throughput(monkeypatch, capsys):
+    """The reference line's value is all timed steps' sampled tokens over
+    their total time (warm-up steps excluded), like the bench's own CPU
+    baseline, not a median of per-step rates."""
+    import json
+    samples = iter([(8, 99.0), (8, 1.0), (8, 3.0), (16, 4.0)])   # (tokens, seconds); the first is warm-up
+
+    def fake_sample(w, budget_s, seed, detail=False):
+        assert detail
+        done, dt = next(samples)
+        return done, dt, 16, ["oracle"]
+    monkeypatch.setattr(bench, "cpu_sample", fake_sample)
+    monkeypatch.setattr(bench, "make_workload", lambda *a, **k: {"rows": bench_rows(10)})
+    monkeypatch.setattr(bench, "describe", lambda w: {"workload": "test"})
+
+    class A:
+        config, K, f, n_traj, warmup, steps, cpu_seconds, rope = 4, 8, 0.6, None, 1, 3, 3.0, None
+    bench.run_reference(A(), rank=0, world=1)
+    line = json.loads(capsys.readouterr().out)
+    assert line["impl"] == "reference"
+    assert line["value"] == pytest.approx(32 / 8.0)
+    assert line["cpu_baseline"]["value"] == line["value"] == line["e2e"]["value"]
+    assert "32 sampled scored tokens over 3 steps" in line["cpu_baseline"]["sample"]
+
+
+def bench_rows(n):
+    import torch
+    return torch.arange(n, dtype=torch.int32)
