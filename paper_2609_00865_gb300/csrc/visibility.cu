@@ -13,6 +13,7 @@
 
 #include <algorithm>
 #include <atomic>
+#include <mutex>
 #include <vector>
 
 #include "common.cuh"
@@ -819,17 +820,127 @@ __global__ void k_event_keymask(int64_t n_keymask, const int32_t* __restrict__ c
     }
 }
 
+// Copy of up to four staged host arrays into device memory: part blockIdx.y,
+// 16-byte vectors (both ends are 16-byte aligned), the ragged tail by bytes.
+struct UploadArgs {
+    const char* src[4];
+    char* dst[4];
+    long long bytes[4];
+};
+__global__ void __launch_bounds__(256) k_upload(UploadArgs u) {
+    const int p = blockIdx.y;
+    const char* src = u.src[p];
+    char* dst = u.dst[p];
+    const long long n = u.bytes[p], n16 = n >> 4;
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n16; i += (long long)gridDim.x * blockDim.x)
+        reinterpret_cast<uint4*>(dst)[i] = reinterpret_cast<const uint4*>(src)[i];
+    if (blockIdx.x == 0 && threadIdx.x < (n & 15)) dst[16 * n16 + threadIdx.x] = src[16 * n16 + threadIdx.x];
+}
+
 }  // namespace
 
 // ---------------------------------------------------------------------------
+// Upload of the host-packed build inputs (the metadata image, the span table,
+// the events table). A copy from pageable memory is staged by the runtime
+// through the copy engines, in order with the caller's other uploads, so a
+// build issued while a large upload runs on another stream (a training loop
+// prefetching its next batch) waits for that upload to finish before its own
+// kernels can start. The builders instead pack into page-locked,
+// device-mapped host buffers, and k_upload on the build's stream reads them
+// over the host link into place (no copy engine). Two buffers per device
+// alternate; before a buffer is rewritten, the event recorded after its last
+// upload is waited on, so the host runs at most two builds ahead of the GPU.
+// The buffers live as long as the process. A build that may not allocate
+// (mw_build_visibility_noalloc), or a failed page-locked allocation, copies
+// from pageable memory instead.
+struct UploadPart {
+    const void* src;
+    void* dst;
+    size_t bytes;
+};
+
+namespace {
+struct StageSlot {
+    char* host = nullptr;
+    size_t cap = 0;
+    cudaEvent_t done = nullptr;
+    bool pending = false;
+};
+struct DevStage {
+    std::mutex mu;
+    StageSlot slot[2];
+    int next = 0;
+};
+constexpr int kStageDevices = 64;
+DevStage g_stage[kStageDevices];
+
+mw_status upload_pageable(const UploadPart* parts, int n, cudaStream_t s) {
+    for (int i = 0; i < n; ++i)
+        if (parts[i].bytes) {
+            mw_status st = cuda_status(
+                cudaMemcpyAsync(parts[i].dst, parts[i].src, parts[i].bytes, cudaMemcpyHostToDevice, s));
+            if (st != MW_OK) return st;
+        }
+    return MW_OK;
+}
+}  // namespace
+
+static mw_status upload_parts(const UploadPart* parts, int n, cudaStream_t s, bool staged) {
+    size_t total = 0;
+    for (int i = 0; i < n; ++i) total += (parts[i].bytes + 15) & ~size_t(15);
+    int dev = 0;
+    if (!staged || total == 0 || n > 4 || cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kStageDevices)
+        return upload_pageable(parts, n, s);
+    DevStage& d = g_stage[dev];
+    std::lock_guard<std::mutex> lock(d.mu);
+    StageSlot& slot = d.slot[d.next];
+    d.next ^= 1;
+    mw_status st = MW_OK;
+    if (slot.pending && (st = cuda_status(cudaEventSynchronize(slot.done))) != MW_OK) return st;
+    slot.pending = false;
+    if (slot.cap < total) {
+        if (slot.host) cudaFreeHost(slot.host);
+        slot.host = nullptr;
+        slot.cap = 0;
+        const size_t cap = std::max<size_t>(total + total / 4, 1 << 16);
+        void* h = nullptr;
+        if (cudaHostAlloc(&h, cap, cudaHostAllocMapped | cudaHostAllocPortable) != cudaSuccess) {
+            cudaGetLastError();   // clear the failed allocation; copy from pageable memory instead
+            return upload_pageable(parts, n, s);
+        }
+        slot.host = (char*)h;
+        slot.cap = cap;
+    }
+    if (!slot.done && (st = cuda_status(cudaEventCreateWithFlags(&slot.done, cudaEventDisableTiming))) != MW_OK)
+        return st;
+    void* dbase = nullptr;
+    if ((st = cuda_status(cudaHostGetDevicePointer(&dbase, slot.host, 0))) != MW_OK) return st;
+    UploadArgs u = {};
+    long long most = 0;
+    size_t off = 0;
+    for (int i = 0; i < n; ++i) {
+        if (parts[i].bytes) memcpy(slot.host + off, parts[i].src, parts[i].bytes);
+        u.src[i] = (const char*)dbase + off;
+        u.dst[i] = (char*)parts[i].dst;
+        u.bytes[i] = (long long)parts[i].bytes;
+        most = std::max(most, u.bytes[i]);
+        off += (parts[i].bytes + 15) & ~size_t(15);
+    }
+    const unsigned gx = (unsigned)std::min<long long>(std::max<long long>(1, ceil_div(most >> 4, 256)), 152);
+    count_launches(1);
+    k_upload<<<dim3(gx, (unsigned)n), 256, 0, s>>>(u);
+    if ((st = launch_status()) != MW_OK) return st;
+    if ((st = cuda_status(cudaEventRecord(slot.done, s))) != MW_OK) return st;
+    slot.pending = true;
+    return MW_OK;
+}
 
 // Host image of the per-trajectory tables (token, tile, segment, triangle and
-// keymask offsets, segment starts, tile owners), copied into the metadata
-// region [off_traj_tok, off_cls) of `vis` with one copy.
-static mw_status copy_meta(const mw_vis_layout* L, const int32_t* cu, int n_junc, const int32_t* J,
-                           const int32_t* jt, void* vis, cudaStream_t stream) {
+// keymask offsets, segment starts, tile owners): the bytes of the metadata
+// region [off_traj_tok, off_cls) of `vis`, uploaded as one part.
+static void pack_meta(const mw_vis_layout* L, const int32_t* cu, int n_junc, const int32_t* J, const int32_t* jt,
+                      std::vector<char>& img) {
     const int n_traj = L->n_traj;
-    mw_status st = MW_OK;
     // host-side packing of the small per-trajectory tables
     const int64_t n_tiles = L->n_tiles;
     std::vector<int32_t> traj_tile(n_traj + 1), traj_seg(n_traj + 1), seg_start(L->n_segs),
@@ -859,10 +970,8 @@ static mw_status copy_meta(const mw_vis_layout* L, const int32_t* cu, int n_junc
         traj_seg[n_traj] = segs;
     }
     // one contiguous host image of the metadata region [off_traj_tok, off_cls)
-    // (a copy from pageable memory: the runtime stages the image before the
-    // call returns)
     const int64_t meta0 = L->off_traj_tok, meta1 = L->off_cls;
-    std::vector<char> img(meta1 - meta0, 0);
+    img.assign(meta1 - meta0, 0);
     auto put = [&](int64_t off, const void* src, size_t bytes) {
         if (bytes) memcpy(img.data() + (off - meta0), src, bytes);
     };
@@ -873,16 +982,14 @@ static mw_status copy_meta(const mw_vis_layout* L, const int32_t* cu, int n_junc
     put(L->off_traj_km, traj_km.data(), 8 * traj_km.size());
     put(L->off_seg_start, seg_start.data(), 4 * seg_start.size());
     put(L->off_tile_traj, tile_traj.data(), 4 * tile_traj.size());
-    if ((st = cuda_status(cudaMemcpyAsync(at<char>(vis, meta0), img.data(), img.size(),
-                                          cudaMemcpyHostToDevice, stream))) != MW_OK)
-        return st;
-    return MW_OK;
 }
 
-extern "C" mw_status mw_build_visibility(const mw_vis_layout* L, const int32_t* cu, int n_junc,
-                                         const int32_t* J, const int32_t* jt,
-                                         const int32_t* span_off, const int32_t* spans,
-                                         void* ws, void* vis, void* stream_) {
+namespace mw {
+// mw_build_visibility; `staged` uploads the packed record through the pinned
+// staging buffers (false: from pageable memory, no allocation).
+mw_status build_visibility(const mw_vis_layout* L, const int32_t* cu, int n_junc, const int32_t* J,
+                           const int32_t* jt, const int32_t* span_off, const int32_t* spans, void* ws, void* vis,
+                           void* stream_, bool staged) {
     if (!L) return MW_EINVAL;
     if (L->kind != MW_VIEWS_EDITS || n_junc != L->n_junc) return MW_EINVAL;
     mw_status st = check_shape(L->n_traj, cu, n_junc, jt, L->n_spans);
@@ -911,7 +1018,8 @@ extern "C" mw_status mw_build_visibility(const mw_vis_layout* L, const int32_t* 
     if (L->vis_bytes == 0) return MW_OK;
 
     const int64_t n_tiles = L->n_tiles;
-    if ((st = copy_meta(L, cu, n_junc, J, jt, vis, stream)) != MW_OK) return st;
+    std::vector<char> img;
+    pack_meta(L, cu, n_junc, J, jt, img);
     std::vector<int32_t> span3(3 * (size_t)L->n_spans);
     for (int k = 0; k < n_junc; ++k)
         for (int s = span_off[k]; s < span_off[k + 1]; ++s) {
@@ -919,11 +1027,9 @@ extern "C" mw_status mw_build_visibility(const mw_vis_layout* L, const int32_t* 
             span3[3 * s + 1] = cu[jt[k]] + spans[2 * s + 1];
             span3[3 * s + 2] = J[k];
         }
-
-    if (L->n_spans > 0 &&
-        (st = cuda_status(cudaMemcpyAsync(at<char>(ws, L->ws_off_spans), span3.data(),
-                                          span3.size() * 4, cudaMemcpyHostToDevice, stream))) != MW_OK)
-        return st;
+    const UploadPart parts[2] = {{img.data(), at<char>(vis, L->off_traj_tok), img.size()},
+                                 {span3.data(), at<char>(ws, L->ws_off_spans), span3.size() * 4}};
+    if ((st = upload_parts(parts, 2, stream, staged)) != MW_OK) return st;
     if ((st = cuda_status(cudaMemsetAsync(at<char>(vis, L->off_pairs), 0, 8 * (n_traj + 1), stream))) != MW_OK)
         return st;
     if ((st = cuda_status(cudaMemsetAsync(at<char>(vis, L->off_status), 0, 32, stream))) != MW_OK)
@@ -986,6 +1092,13 @@ extern "C" mw_status mw_build_visibility(const mw_vis_layout* L, const int32_t* 
     }
     return launch_status();
 }
+}  // namespace mw
+
+extern "C" mw_status mw_build_visibility(const mw_vis_layout* L, const int32_t* cu, int n_junc, const int32_t* J,
+                                         const int32_t* jt, const int32_t* span_off, const int32_t* spans, void* ws,
+                                         void* vis, void* stream) {
+    return build_visibility(L, cu, n_junc, J, jt, span_off, spans, ws, vis, stream, true);
+}
 
 extern "C" mw_status mw_build_views_events(const mw_vis_layout* L, const int32_t* cu, int n_junc, const int32_t* J,
                                            const int32_t* jt, const int32_t* out_off, const int32_t* in_off,
@@ -1046,13 +1159,12 @@ extern "C" mw_status mw_build_views_events(const mw_vis_layout* L, const int32_t
     cudaStream_t stream = (cudaStream_t)stream_;
     if (L->vis_bytes == 0) return MW_OK;
     const int64_t n_tiles = L->n_tiles;
-    if ((st = copy_meta(L, cu, n_junc, J, jt, vis, stream)) != MW_OK) return st;
-    if (n_spans > 0 && (st = cuda_status(cudaMemcpyAsync(at<char>(ws, L->ws_off_spans), sp2.data(), sp2.size() * 4,
-                                                         cudaMemcpyHostToDevice, stream))) != MW_OK)
-        return st;
-    if (n_junc > 0 && (st = cuda_status(cudaMemcpyAsync(at<char>(ws, L->ws_off_tstat), jtab.data(), jtab.size() * 4,
-                                                        cudaMemcpyHostToDevice, stream))) != MW_OK)
-        return st;
+    std::vector<char> img;
+    pack_meta(L, cu, n_junc, J, jt, img);
+    const UploadPart parts[3] = {{img.data(), at<char>(vis, L->off_traj_tok), img.size()},
+                                 {sp2.data(), at<char>(ws, L->ws_off_spans), sp2.size() * 4},
+                                 {jtab.data(), at<char>(ws, L->ws_off_tstat), jtab.size() * 4}};
+    if ((st = upload_parts(parts, 3, stream, true)) != MW_OK) return st;
     // no tile classes or lists for these views: empty lists, zero classes
     if ((st = cuda_status(cudaMemsetAsync(at<char>(vis, L->off_cls), 0, (size_t)L->n_tri, stream))) != MW_OK ||
         (st = cuda_status(cudaMemsetAsync(at<char>(vis, L->off_fwd_ptr), 0, 4 * (size_t)(n_tiles + 1), stream))) !=

@@ -25,6 +25,11 @@
 
 #include "common.cuh"
 
+namespace mw {
+mw_status build_visibility(const mw_vis_layout*, const int32_t*, int, const int32_t*, const int32_t*, const int32_t*,
+                           const int32_t*, void*, void*, void*, bool);
+}
+
 namespace {
 
 constexpr long long kStaticWsBytes = 1ll << 20;  // 1 MiB
@@ -59,5 +64,7 @@ extern "C" mw_status mw_build_visibility_noalloc(const mw_vis_layout* L, const i
         }
         ws = g_ws_addr[dev];
     }
-    return mw_build_visibility(L, cu_seqlens, n_junc, junctions, junc_traj, junc_span_off, spans, ws, vis, stream);
+    // the record goes up from pageable memory: no page-locked staging buffer
+    return mw::build_visibility(L, cu_seqlens, n_junc, junctions, junc_traj, junc_span_off, spans, ws, vis, stream,
+                                false);
 }

@@ -22,7 +22,10 @@ def _gpu(seqlens, edits):
 
 
 def _compare(seqlens, edits):
-    got = _gpu(seqlens, edits)
+    return _check_arrays(_gpu(seqlens, edits), seqlens, edits)
+
+
+def _check_arrays(got, seqlens, edits):
     want = OV.build(seqlens, edits)
     for key in ("omega", "seg", "qtile_traj", "fwd_ptr", "fwd_idx", "bwd_ptr", "bwd_idx", "pairs", "keymask",
                 "seg_len", "cpos"):
@@ -134,3 +137,44 @@ def test_dense_mask_export_config2_trajectory():
     """One 16,384-token trajectory of the attention workload (32 MB of bits)."""
     r = synth.config_record(2)
     _mask_case(r.seqlens[:1], r.edits[:1])
+
+
+def test_builds_back_to_back_without_synchronising():
+    """Records of different sizes built one after another with no
+    synchronisation in between, on one stream and then alternating two: the
+    builder's two page-locked staging buffers are reused (and grown) while
+    earlier builds may still be in flight. Every build equals the oracle's."""
+    import torch
+    import paper_2609_00865_gb300 as mw
+    rng = np.random.default_rng(77)
+    recs = [_rand_record(rng, int(rng.integers(1, 6))) for _ in range(6)]
+    big = synth.config_record(2)
+    recs.insert(3, (big.seqlens, big.edits))          # grows the staging buffers mid-run
+    streams = [torch.cuda.current_stream(), torch.cuda.Stream()]
+    built = []
+    for i, r in enumerate(recs + recs):
+        s = streams[0] if i < len(recs) else streams[i % 2]
+        built.append((r, mw.build_visibility(*r, stream=s)))
+    torch.cuda.synchronize()
+    for r, vis in built:
+        vis.check_status()
+        _check_arrays(vis.arrays(), *r)
+
+
+def test_build_beside_a_large_upload():
+    """A build issued while a 1 GiB upload from page-locked memory runs on
+    another stream (a training loop prefetching its next batch) is correct;
+    its record goes up by a kernel, not behind that copy."""
+    import torch
+    import paper_2609_00865_gb300 as mw
+    h = torch.empty(1 << 30, dtype=torch.uint8).pin_memory()
+    d = torch.empty(1 << 30, dtype=torch.uint8, device="cuda")
+    copy = torch.cuda.Stream()
+    rec = synth.config_record(2)
+    with torch.cuda.stream(copy):
+        d.copy_(h, non_blocking=True)
+    vis = mw.build_visibility(rec.seqlens, rec.edits)
+    torch.cuda.synchronize()
+    vis.check_status()
+    _check_arrays(vis.arrays(), rec.seqlens, rec.edits)
+
