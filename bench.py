@@ -708,52 +708,73 @@ def run_gpu(args, rank, world, local_rank):
     ms = reduce_max(ms, world, dev)
     per_call = {k: sum(a.elapsed_time(b) for a, b in v) / len(v) for k, v in step.events.items()}
 
-    # e2e: pinned host inputs -> device, step, loss/metric read back. The
-    # per-step inputs are uploaded; the LM-head weight W is model state, resident
-    # on the device across steps as in a training loop.
+    # e2e: pinned host inputs -> device, step, loss/metric read back, every
+    # step. The per-step inputs are uploaded; the LM-head weight W is model
+    # state, resident on the device across steps as in a training loop.
     host = e2e_inputs(w, step.d)
     h2d = sum(v.numel() * v.element_size() for v in host.values())
     out = step.loss if hasattr(step, "loss") else step.LSE[0, :1]
     d2h = out.numel() * out.element_size()
     pinned_out = torch.empty(out.shape, dtype=out.dtype).pin_memory()
-    # Every step uploads its own inputs and reads its loss back inside the
-    # timed region. As a training loop that prefetches its next batch does,
-    # step i + 1's inputs are copied on a copy stream while step i computes,
-    # into the other of two device input sets.
-    sets = [step.d, dict(step.d)]
-    for k in host:
-        sets[1][k] = torch.empty_like(step.d[k])
-    copy = torch.cuda.Stream(dev)
-    ready = [torch.cuda.Event(), torch.cuda.Event()]
-    used = [torch.cuda.Event(), torch.cuda.Event()]
 
-    def upload(i):
-        with torch.cuda.stream(copy):
-            for k, v in host.items():
-                sets[i % 2][k].copy_(v, non_blocking=True)
-            ready[i % 2].record(copy)
+    def e2e_serial():
+        """Each step's inputs are copied on the step's stream right before it
+        (the reported schedule)."""
+        barrier()
+        torch.cuda.synchronize()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(step.stream)
+        for _ in range(args.steps):
+            step.upload(host)
+            step.run()
+            pinned_out.copy_(out, non_blocking=True)
+        e1.record(step.stream)
+        torch.cuda.synchronize()
+        return reduce_max(e0.elapsed_time(e1) / args.steps, world, dev)
 
-    barrier()
-    torch.cuda.synchronize()
-    e0 = torch.cuda.Event(enable_timing=True)
-    e1 = torch.cuda.Event(enable_timing=True)
-    e0.record(step.stream)
-    copy.wait_event(e0)
-    upload(0)
-    for i in range(args.steps):
-        if i + 1 < args.steps:
-            if i >= 1:
-                copy.wait_event(used[(i + 1) % 2])   # step i - 1 read that set
-            upload(i + 1)
-        step.stream.wait_event(ready[i % 2])
-        step.d = sets[i % 2]
-        step.run()
-        used[i % 2].record(step.stream)
-        pinned_out.copy_(out, non_blocking=True)
-    e1.record(step.stream)
-    torch.cuda.synchronize()
-    step.d = sets[0]
-    e2e_ms = reduce_max(e0.elapsed_time(e1) / args.steps, world, dev)
+    def e2e_prefetch():
+        """Step i + 1's inputs copied on a copy stream while step i computes,
+        into the other of two device input sets (reported beside, for
+        comparison: the upload's writes pass through L2 and slow the step)."""
+        base = step.d
+        sets = [base, dict(base)]
+        for k in host:
+            sets[1][k] = torch.empty_like(base[k])
+        copy = torch.cuda.Stream(dev)
+        ready = [torch.cuda.Event(), torch.cuda.Event()]
+        used = [torch.cuda.Event(), torch.cuda.Event()]
+
+        def upload(i):
+            with torch.cuda.stream(copy):
+                for k, v in host.items():
+                    sets[i % 2][k].copy_(v, non_blocking=True)
+                ready[i % 2].record(copy)
+
+        barrier()
+        torch.cuda.synchronize()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(step.stream)
+        copy.wait_event(e0)
+        upload(0)
+        for i in range(args.steps):
+            if i + 1 < args.steps:
+                if i >= 1:
+                    copy.wait_event(used[(i + 1) % 2])   # step i - 1 read that set
+                upload(i + 1)
+            step.stream.wait_event(ready[i % 2])
+            step.d = sets[i % 2]
+            step.run()
+            used[i % 2].record(step.stream)
+            pinned_out.copy_(out, non_blocking=True)
+        e1.record(step.stream)
+        torch.cuda.synchronize()
+        step.d = base
+        return reduce_max(e0.elapsed_time(e1) / args.steps, world, dev)
+
+    e2e_ms = e2e_serial()
+    e2e_prefetch_ms = e2e_prefetch()
 
     if rank != 0:
         return
@@ -784,8 +805,9 @@ def run_gpu(args, rank, world, local_rank):
         "cpu_baseline": cpu,
         "e2e": {"value": job_value(scored, world, e2e_ms), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms,
-                "upload": "pinned host -> device, every per-step input (W stays resident as model state); "
-                          "step i + 1's inputs on a copy stream during step i"},
+                "upload": "pinned host -> device, every per-step input (W stays resident as model state), "
+                          "on the step's stream before the step",
+                "prefetch_ms_per_step": e2e_prefetch_ms},
         "gpu_launches": launches,
         "clocks": clk,
     }
