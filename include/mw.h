@@ -197,11 +197,11 @@ mw_status mw_build_views_events(const mw_vis_layout* layout, const int32_t* cu_s
  * The record is validated on the host (MW_EEDITS) and packed into one of two
  * page-locked, device-mapped host buffers the library keeps per device (grown
  * as records grow, kept for the life of the process); a kernel on `stream`
- * reads it into place, so the call does not wait for the copy engines (a
- * large upload of the caller's on another stream does not hold it up). Before
- * a buffer is reused, the call waits for the build that last used it, so the
- * host runs at most two builds ahead of the GPU. Everything else runs
- * asynchronously. (mw_build_visibility_noalloc copies from pageable memory.)
+ * reads it into place over the host link (no copy engine, no host-side
+ * staging copy). Before a buffer is reused, the call waits for the build that
+ * last used it, so the host runs at most two builds ahead of the GPU.
+ * Everything else runs asynchronously. (mw_build_visibility_noalloc copies
+ * from pageable memory.)
  */
 mw_status mw_build_visibility(const mw_vis_layout* layout, const int32_t* cu_seqlens,
                               int n_junc, const int32_t* junctions, const int32_t* junc_traj,

@@ -841,18 +841,17 @@ __global__ void __launch_bounds__(256) k_upload(UploadArgs u) {
 
 // ---------------------------------------------------------------------------
 // Upload of the host-packed build inputs (the metadata image, the span table,
-// the events table). A copy from pageable memory is staged by the runtime
-// through the copy engines, in order with the caller's other uploads, so a
-// build issued while a large upload runs on another stream (a training loop
-// prefetching its next batch) waits for that upload to finish before its own
-// kernels can start. The builders instead pack into page-locked,
-// device-mapped host buffers, and k_upload on the build's stream reads them
-// over the host link into place (no copy engine). Two buffers per device
-// alternate; before a buffer is rewritten, the event recorded after its last
-// upload is waited on, so the host runs at most two builds ahead of the GPU.
-// The buffers live as long as the process. A build that may not allocate
-// (mw_build_visibility_noalloc), or a failed page-locked allocation, copies
-// from pageable memory instead.
+// the events table). A copy from pageable memory goes through the runtime's
+// staging memory and a copy engine, where it shares the engines with the
+// caller's own uploads (a training loop prefetching its next batch on another
+// stream). The builders instead pack into page-locked, device-mapped host
+// buffers, and k_upload on the build's stream reads them over the host link
+// into place: no copy engine, and the call returns without a host-side
+// staging copy. Two buffers per device alternate; before a buffer is
+// rewritten, the event recorded after its last upload is waited on, so the
+// host runs at most two builds ahead of the GPU. The buffers live as long as
+// the process. A build that may not allocate (mw_build_visibility_noalloc),
+// or a failed page-locked allocation, copies from pageable memory instead.
 struct UploadPart {
     const void* src;
     void* dst;
