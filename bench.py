@@ -155,13 +155,16 @@ def job_value(scored_per_rank, world, ms):
     return scored_per_rank * world / (ms * 1e-3)
 
 
-def make_workload(cfg, K=None, f=None, seed_offset=0, n_traj=None, pin=True, rope=None):
+def make_workload(cfg, K=None, f=None, seed_offset=0, n_traj=None, pin=True, rope=None, events=None):
     """Host-side inputs of one workload (CPU tensors, pinned unless ``pin`` is
     False, + record).
 
     ``n_traj`` keeps only the first trajectories of the record (a smaller
     case of the same kernels, for profiler captures). ``rope`` (a rotary
-    theta) runs the attention with row-wise logical rotary positions."""
+    theta) runs the attention with row-wise logical rotary positions.
+    ``events`` (a retrieve probability) turns the record into an offload /
+    retrieve record (``synth.events_record``): the compressions' evicted spans
+    are offloaded and come back at later junctions."""
     import numpy as np
     import torch
 
@@ -187,6 +190,9 @@ def make_workload(cfg, K=None, f=None, seed_offset=0, n_traj=None, pin=True, rop
         if n_traj:
             rec = synth.Record(rec.trajs[:n_traj])
         w["record"] = rec
+        if events is not None:
+            w["events"] = synth.events_record(rec, float(events), 7000 + cfg)
+            w["events_p"] = float(events)
         T = rec.total
         w["Q"] = randn(T, c["Hq"], c["Dh"])
         w["K"] = randn(T, c["Hkv"], c["Dh"])
@@ -239,6 +245,10 @@ def describe(w):
         d.update(sweep_K=w["sweep"][0], evicted_fraction=w["sweep"][1])
     if "rope" in w:
         d["rope_theta"] = w["rope"]
+    if "events" in w:
+        d["views"] = "offload / retrieve events (MemexRL): evicted spans offloaded, " \
+                     f"each brought back at a later junction with p = {w['events_p']}"
+        d["retrieved_spans"] = sum(len(i) for e in w["events"] for _, _, i in e)
     d["l2"] = "inputs larger than L2 (129 MB); no flush"
     return d
 
@@ -259,9 +269,13 @@ class Step:
         self.timing = False
         if "record" in w:
             r = w["record"]
-            self.flat = mw.flatten_record(r.seqlens, r.edits)
-            cu, J, jt, off, spans = self.flat
-            self.L = mw.mw_visibility_layout(cu, jt, len(spans))
+            if "events" in w:
+                self.flat = mw.flatten_events(r.seqlens, w["events"])
+                self.L = mw.mw_events_layout(self.flat[0], self.flat[2], len(self.flat[-1]))
+            else:
+                self.flat = mw.flatten_record(r.seqlens, r.edits)
+                cu, J, jt, off, spans = self.flat
+                self.L = mw.mw_visibility_layout(cu, jt, len(spans))
             self.vis = mw.Visibility(self.L, torch.empty(self.L.vis_bytes, dtype=torch.uint8, device=device),
                                      torch.empty(max(self.L.ws_bytes, 1), dtype=torch.uint8, device=device))
             Hq, Hkv, Dh = w["heads"]
@@ -324,9 +338,14 @@ class Step:
         self.lp_old.copy_(self.lp + self.d["noise"])
 
     def build(self):
-        cu, J, jt, off, spans = self.flat
-        self._ev("mw_build_visibility", lambda: self.mw.mw_build_visibility(
-            self.L, cu, J, jt, off, spans, self.vis.ws, self.vis.vis, self.stream))
+        if "events" in self.w:
+            cu, J, jt, oo, io, spans = self.flat
+            self._ev("mw_build_views_events", lambda: self.mw.mw_build_views_events(
+                self.L, cu, J, jt, oo, io, spans, self.vis.ws, self.vis.vis, self.stream))
+        else:
+            cu, J, jt, off, spans = self.flat
+            self._ev("mw_build_visibility", lambda: self.mw.mw_build_visibility(
+                self.L, cu, J, jt, off, spans, self.vis.ws, self.vis.vis, self.stream))
         if "rope" in self.w:
             self._ev("mw_logical_positions", lambda: self.mw.mw_logical_positions(self.vis, self.pos, self.stream))
 
@@ -389,7 +408,7 @@ class Step:
         """Attention work skipped by the visibility structure, against plain
         causal attention of the same trajectory lengths: 128x128 tiles listed
         (non-empty) vs causal tiles, visible pairs vs causal pairs."""
-        if "record" not in self.w:
+        if "record" not in self.w or "events" in self.w:   # event views have no tile lists
             return None
         import numpy as np
         L = self.vis.layout
@@ -588,6 +607,7 @@ def cpu_sample(w, budget_s=15.0, seed=5, detail=False):
 
     from oracle import attention as OA
     from oracle import logprob as OL
+    from oracle import nonmonotone as ON
     cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
     if "_f64" not in w:   # exact float64 copies of the bf16 inputs, made once
         w["_f64"] = {k: w[k].to(torch.float64).numpy() for k in ("Q", "K", "V", "dO", "H", "W") if k in w}
@@ -607,9 +627,11 @@ def cpu_sample(w, budget_s=15.0, seed=5, detail=False):
             Hq, Hkv, Dh = w["heads"]
             parts.append("attention fwd + bwd (dQ, dK, dV contributions), all heads")
             th = w.get("rope")
-            O, _ = OA.attn_fwd(r.seqlens, r.edits, x["Q"], x["K"], x["V"], Dh ** -0.5, rows=rows, rope_theta=th)
-            OA.attn_bwd_rows(r.seqlens, r.edits, x["Q"], x["K"], x["V"], x.get("dO", x["Q"]), Dh ** -0.5,
-                             rows, list(range(Hq)), rope_theta=th, with_kv=True)
+            rec, views = (w["events"], ON.live_views) if "events" in w else (r.edits, None)
+            O, _ = OA.attn_fwd(r.seqlens, rec, x["Q"], x["K"], x["V"], Dh ** -0.5, rows=rows, rope_theta=th,
+                               views=views)
+            OA.attn_bwd_rows(r.seqlens, rec, x["Q"], x["K"], x["V"], x.get("dO", x["Q"]), Dh ** -0.5,
+                             rows, list(range(Hq)), rope_theta=th, with_kv=True, views=views)
         if "rows" in w:
             parts.append("LM-head fwd over the full vocabulary + dH/dW")
             if "H" in x:
@@ -643,7 +665,7 @@ def run_reference(args, rank, world):
     if rank != 0:
         return
     w = make_workload(args.config, args.K, args.f, n_traj=args.n_traj, pin=False,   # the oracle runs on the host
-                      rope=args.rope)
+                      rope=args.rope, events=args.events)
     # every step samples its own rows; the value is all timed steps' tokens
     # over their time (whole-job throughput, as the bench's own CPU baseline)
     tok, sec = 0, 0.0
@@ -676,7 +698,8 @@ def run_gpu(args, rank, world, local_rank):
     import paper_2609_00865_gb300 as mw
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
-    w = make_workload(args.config, args.K, args.f, seed_offset=rank, n_traj=args.n_traj, rope=args.rope)
+    w = make_workload(args.config, args.K, args.f, seed_offset=rank, n_traj=args.n_traj, rope=args.rope,
+                      events=args.events)
     step = SdccStep(w, dev) if args.sdcc else Step(w, dev)
     step.prime()
     for _ in range(args.warmup):
@@ -941,9 +964,14 @@ def main():
                     help="attention with row-wise logical rotary positions (theta of the rotary table)")
     ap.add_argument("--builder", action="store_true",
                     help="time the visibility builder alone on 64 sweep trajectories (131,072 tokens, --K, --f)")
+    ap.add_argument("--events", type=float, default=None, metavar="P",
+                    help="offload / retrieve views: the record's evicted spans are offloaded and each comes "
+                         "back at a later junction with probability P (configs 2, 4, 5)")
     args = ap.parse_args()
-    if args.sdcc and (args.config != 4 or args.rope is not None):
-        ap.error("--sdcc times the 7B-shaped layer step (config 4) without rotary positions")
+    if args.sdcc and (args.config != 4 or args.rope is not None or args.events is not None):
+        ap.error("--sdcc times the 7B-shaped layer step (config 4) without rotary positions or events")
+    if args.events is not None and (args.config == 3 or args.builder or not 0.0 <= args.events <= 1.0):
+        ap.error("--events P (0 <= P <= 1) needs a record: configs 2, 4, 5")
     rank = int(os.environ.get("RANK", 0))
     world = int(os.environ.get("WORLD_SIZE", args.gpus if args.gpus == 1 else 1))
     local_rank = int(os.environ.get("LOCAL_RANK", 0))

@@ -159,6 +159,25 @@ def record(n_traj, T, K, evict, summary, prompt, Lp, Lo, seed_base, on_policy_su
                    for b in range(n_traj)])
 
 
+def events_record(rec, retrieve, seed):
+    """An offload / retrieve (MemexRL) record from a compression record: each
+    junction offloads the spans the compression evicts (its out-spans), and
+    every span offloaded at an earlier junction and still out comes back at a
+    later junction with probability ``retrieve`` (its in-spans, in the order
+    they were offloaded). Returns ``events_per_traj``: per trajectory a list
+    of (J, out_spans, in_spans)."""
+    rng = _rng(seed)
+    out = []
+    for t in rec.trajs:
+        ev, offloaded = [], []
+        for J, spans in t.edits:
+            back = [s for s in offloaded if rng.random() < retrieve]
+            offloaded = [s for s in offloaded if s not in back] + list(spans)
+            ev.append((int(J), [tuple(s) for s in spans], [tuple(s) for s in back]))
+        out.append(ev)
+    return out
+
+
 def config_record(cfg, K=None, f=None):
     """The record of workload ``cfg`` (1, 2, 4 or 5); seed = 1000*cfg + traj."""
     c = CONFIGS[cfg]

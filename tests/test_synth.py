@@ -100,3 +100,25 @@ def test_on_policy_summaries():
         for J, _ in t.edits:
             assert (t.kinds[J - 47: J + 1] == synth.POLICY).all()
             assert all(i in rows for i in range(J - 48, J))     # rows predicting the summary tokens
+
+
+def test_events_record_offloads_and_retrieves_valid_spans():
+    """The offload / retrieve stand-in keeps each compression's evicted spans
+    as out-spans and brings earlier offloaded spans back: every event is
+    valid (a retrieved span is out of the view when its event fires), some
+    spans come back, and with retrieve = 0 the views equal the compression
+    record's."""
+    from oracle import nonmonotone as N
+    rec = synth.config_record(2)
+    ev = synth.events_record(rec, 0.3, 7)
+    n_back = 0
+    for t, e in zip(rec.trajs, ev):
+        N.validate_events(t.T, e)
+        assert [(J, list(o)) for J, o, _ in e] == [(J, list(map(tuple, s))) for J, s in t.edits]
+        n_back += sum(len(i) for _, _, i in e)
+    assert n_back > 0
+    small = synth.record(2, 700, 3, 0.6, 16, 16, 20, 30, 11)
+    none = synth.events_record(small, 0.0, 7)
+    for t, e in zip(small.trajs, none):
+        assert all(not i for _, _, i in e)
+        np.testing.assert_array_equal(N.dense_mask(t.T, e), OV.dense_mask(t.T, t.edits))
