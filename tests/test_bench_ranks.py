@@ -91,7 +91,7 @@ def test_reference_arm_reports_whole_job_throughput(monkeypatch, capsys):
     monkeypatch.setattr(bench, "describe", lambda w: {"workload": "test"})
 
     class A:
-        config, K, f, n_traj, warmup, steps, cpu_seconds, rope = 4, 8, 0.6, None, 1, 3, 3.0, None
+        config, K, f, n_traj, warmup, steps, cpu_seconds, rope, events = 4, 8, 0.6, None, 1, 3, 3.0, None, None
     bench.run_reference(A(), rank=0, world=1)
     line = json.loads(capsys.readouterr().out)
     assert line["impl"] == "reference"
