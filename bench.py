@@ -442,6 +442,75 @@ class Step:
         return f
 
 
+class PackedStep(Step):
+    """One layer of the stacked-layer step (App. G's branch-replicated
+    packing, the design for more than one layer): every segment's live view
+    is packed as a branch of its own (mw_branch_pack of Q, K, V and the
+    upstream dO, through the compact maps of the record's visibility build),
+    the layer's attention runs causally over the packed branches (one build of
+    the packed record: a trajectory per branch, no junctions), and the packed
+    copies' gradients are summed back per token (mw_branch_unpack_add of dQ,
+    dK, dV). A stack of L layers repeats the attention L times between one
+    pack and one unpack. The branch lengths are structure of the record,
+    read once (untimed); both builds are timed."""
+
+    def __init__(self, w, device):
+        import torch
+        super().__init__(w, device)
+        mw = self.mw
+        Hq, Hkv, Dh = w["heads"]
+        self.build()
+        lens = mw.branch_lengths(self.vis)
+        torch.cuda.synchronize()
+        self.n = n = int(sum(lens))
+        self.flat_p = mw.flatten_record(lens, [[] for _ in lens])
+        cu, J, jt, off, spans = self.flat_p
+        self.L_p = mw.mw_visibility_layout(cu, jt, len(spans))
+        self.vis_p = mw.Visibility(self.L_p, torch.empty(self.L_p.vis_bytes, dtype=torch.uint8, device=device),
+                                   torch.empty(max(self.L_p.ws_bytes, 1), dtype=torch.uint8, device=device))
+        bf = torch.bfloat16
+        self.Qp = torch.empty(n, Hq, Dh, dtype=bf, device=device)
+        self.dOp = torch.empty_like(self.Qp)
+        self.Kp = torch.empty(n, Hkv, Dh, dtype=bf, device=device)
+        self.Vp = torch.empty_like(self.Kp)
+        self.Op = torch.empty_like(self.Qp)
+        self.LSEp = torch.empty(Hq, n, dtype=torch.float32, device=device)
+        self.dQp = torch.empty_like(self.Qp)
+        self.dKp = torch.empty_like(self.Kp)
+        self.dVp = torch.empty_like(self.Kp)
+        self.attn_fwd_ws_p = torch.empty(max(mw.mw_masked_attn_fwd_ws(self.vis_p, Hkv, Dh, mw.MW_BF16), 1),
+                                         dtype=torch.uint8, device=device)
+        self.attn_ws_p = torch.empty(max(mw.mw_masked_attn_bwd_ws(self.vis_p, Hq, Hkv, Dh, mw.MW_BF16), 1),
+                                     dtype=torch.uint8, device=device)
+        torch.cuda.synchronize()
+
+    def run(self):
+        mw = self.mw
+        self.build()
+        cu, J, jt, off, spans = self.flat_p
+        self._ev("mw_build_visibility (packed)", lambda: mw.mw_build_visibility(
+            self.L_p, cu, J, jt, off, spans, self.vis_p.ws, self.vis_p.vis, self.stream))
+        for X, Xp in ((self.d["Q"], self.Qp), (self.d["K"], self.Kp), (self.d["V"], self.Vp),
+                      (self.d["dO"], self.dOp)):
+            self._ev("mw_branch_pack", lambda: mw.mw_branch_pack(self.vis, X, Xp, self.stream))
+        self._ev("mw_masked_attn_fwd", lambda: mw.mw_masked_attn_fwd(
+            self.vis_p, self.Qp, self.Kp, self.Vp, self.Op, self.LSEp, self.scale, self.attn_fwd_ws_p, self.stream))
+        self._ev("mw_masked_attn_bwd", lambda: mw.mw_masked_attn_bwd(
+            self.vis_p, self.Qp, self.Kp, self.Vp, self.Op, self.dOp, self.LSEp, self.dQp, self.dKp, self.dVp,
+            self.scale, self.attn_ws_p, self.stream))
+        for dXp, dX in ((self.dQp, self.dQ), (self.dKp, self.dK), (self.dVp, self.dV)):
+            self._ev("mw_branch_unpack_add", lambda: mw.mw_branch_unpack_add(self.vis, dXp, dX, self.stream))
+
+    def tile_stats(self):
+        return None
+
+    def flops(self):
+        """Visible FLOPs of the layer: 14 P Dh Hq over the packed branches
+        (P counts every packed row's causal keys, trunk copies included)."""
+        Hq, _, Dh = self.w["heads"]
+        return {"attn": 14.0 * self.vis_p.pairs_total * Dh * Hq}
+
+
 class SdccStep(Step):
     """SDCC training step on the 7B-shaped layer (§5, Eq. "soft_loss"): the
     teacher is the masked attention under each row's live view (forward
@@ -700,7 +769,7 @@ def run_gpu(args, rank, world, local_rank):
     dev = torch.device("cuda", local_rank)
     w = make_workload(args.config, args.K, args.f, seed_offset=rank, n_traj=args.n_traj, rope=args.rope,
                       events=args.events)
-    step = SdccStep(w, dev) if args.sdcc else Step(w, dev)
+    step = SdccStep(w, dev) if args.sdcc else PackedStep(w, dev) if args.packed else Step(w, dev)
     step.prime()
     for _ in range(args.warmup):
         step.run()
@@ -796,7 +865,7 @@ def run_gpu(args, rank, world, local_rank):
     achieved = dom_flops / (per_call[dom] * 1e-3) / 1e12
     total_tf = sum(flops.values()) / (ms * 1e-3) / 1e12
     cpu = None
-    if world == 1 and not args.no_cpu and not args.sdcc:   # the oracle sample times the 4D-mask path
+    if world == 1 and not args.no_cpu and not args.sdcc and not args.packed:   # the oracle sample times the 4D-mask path
         v, cores, desc = cpu_sample(w, budget_s=args.cpu_seconds)
         cpu = {"value": v, "unit": "tokens/s", "cores": cores, "kind": "oracle", "sample": desc}
     line = {
@@ -824,6 +893,11 @@ def run_gpu(args, rank, world, local_rank):
         line["config"].update(method="SDCC (§5): student over the final walks + lam KL at diverging leaves",
                               walk_tokens=step.Tw, scored_leaves=step.n_leaves, kl_pairs=step.n_pairs,
                               lam=step.LAM)
+    if args.packed:
+        line["config"].update(method="one stacked layer over branch-replicated packing (App. G): pack Q, K, V, dO; "
+                                     "attention fwd + bwd over the packed branches; unpack dQ, dK, dV",
+                              packed_rows=step.n, packed_visible_pairs=int(step.vis_p.pairs_total),
+                              visible_pairs_4d_mask=int(step.vis.pairs_total))
     ts = step.tile_stats()
     if ts is not None:
         line["attention_tiles"] = ts
@@ -964,12 +1038,17 @@ def main():
                     help="attention with row-wise logical rotary positions (theta of the rotary table)")
     ap.add_argument("--builder", action="store_true",
                     help="time the visibility builder alone on 64 sweep trajectories (131,072 tokens, --K, --f)")
+    ap.add_argument("--packed", action="store_true",
+                    help="config 2: one stacked layer over branch-replicated packing (pack, attention over the "
+                         "packed branches, unpack)")
     ap.add_argument("--events", type=float, default=None, metavar="P",
                     help="offload / retrieve views: the record's evicted spans are offloaded and each comes "
                          "back at a later junction with probability P (configs 2, 4, 5)")
     args = ap.parse_args()
     if args.sdcc and (args.config != 4 or args.rope is not None or args.events is not None):
         ap.error("--sdcc times the 7B-shaped layer step (config 4) without rotary positions or events")
+    if args.packed and (args.config != 2 or args.sdcc or args.rope is not None or args.events is not None):
+        ap.error("--packed runs config 2's attention on edits views without rotary positions")
     if args.events is not None and (args.config == 3 or args.builder or not 0.0 <= args.events <= 1.0):
         ap.error("--events P (0 <= P <= 1) needs a record: configs 2, 4, 5")
     rank = int(os.environ.get("RANK", 0))

@@ -372,14 +372,24 @@ def branch_lengths(vis):
     return [int(x) for x in vis._arr(vis.layout.off_seg_len, vis.layout.n_segs, np.int32)]
 
 
+def mw_branch_pack(vis, X, Xp, stream=None):
+    row = int(np.prod(X.shape[1:]))
+    _check(_lib().mw_branch_pack(ctypes.byref(vis.layout), _ptr(vis.vis), _ptr(X), _ptr(Xp), row, _dtype_code(X),
+                                 _stream(stream)), "mw_branch_pack")
+
+
+def mw_branch_unpack_add(vis, dXp, dX, stream=None):
+    row = int(np.prod(dXp.shape[1:]))
+    _check(_lib().mw_branch_unpack_add(ctypes.byref(vis.layout), _ptr(vis.vis), _ptr(dXp), _ptr(dX), row,
+                                       _dtype_code(dXp), _stream(stream)), "mw_branch_unpack_add")
+
+
 def branch_pack(vis, X, n_packed, stream=None):
     """Packed branch copies [n_packed, ...] of the per-token rows of X
     (mw_branch_pack)."""
     import torch
     Xp = torch.empty((n_packed,) + tuple(X.shape[1:]), dtype=X.dtype, device=X.device)
-    row = int(np.prod(X.shape[1:]))
-    _check(_lib().mw_branch_pack(ctypes.byref(vis.layout), _ptr(vis.vis), _ptr(X), _ptr(Xp), row, _dtype_code(X),
-                                 _stream(stream)), "mw_branch_pack")
+    mw_branch_pack(vis, X, Xp, stream)
     return Xp
 
 
@@ -388,9 +398,7 @@ def branch_unpack_add(vis, dXp, stream=None):
     (mw_branch_unpack_add)."""
     import torch
     dX = torch.empty((int(vis.layout.total_tokens),) + tuple(dXp.shape[1:]), dtype=dXp.dtype, device=dXp.device)
-    row = int(np.prod(dXp.shape[1:]))
-    _check(_lib().mw_branch_unpack_add(ctypes.byref(vis.layout), _ptr(vis.vis), _ptr(dXp), _ptr(dX), row,
-                                       _dtype_code(dXp), _stream(stream)), "mw_branch_unpack_add")
+    mw_branch_unpack_add(vis, dXp, dX, stream)
     return dX
 
 
