@@ -904,12 +904,16 @@ __global__ void __launch_bounds__(NT_BWD, 1)
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int grp = p.Hq / p.Hkv;
-    // KV head outermost: the CTAs resident at one time share one head's Q / dO
-    // (whose working set then fits in L2)
+    // KV head outermost, then trajectory by trajectory: the CTAs resident at
+    // one time hold the key tiles of one or two trajectories under one head,
+    // and walk the same Q / dO tiles from the trajectory's end (L2 reuse
+    // across key tiles; with the trajectories interleaved instead, a record of
+    // many short trajectories spread the resident CTAs over all of them and
+    // read Q / dO from DRAM again for nearly every key tile)
     const int kvh = blockIdx.x / (p.max_tiles * p.n_traj);
     const int r = blockIdx.x % (p.max_tiles * p.n_traj);
-    const int kt = r / p.n_traj;
-    const int b = r % p.n_traj;
+    const int b = r / p.max_tiles;
+    const int kt = r % p.max_tiles;
     const VisView& v = p.v;
     const int nt = v.traj_tile[b + 1] - v.traj_tile[b];
     if (kt >= nt) return;
