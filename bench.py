@@ -51,16 +51,16 @@ def _peaks():
 # value it had when the counters were taken.
 TRAFFIC = {
     (4, "mw_logprob_loss_bwd"): {
-        "bytes": 457216 + (86640796672 + 14105479168) + (807975680 + 246783744),   # par, dW pass, dH from E
+        "bytes": 456704 + (79047485952 + 14109122048) + (807879424 + 246768896),   # par, dW pass, dH from E
         "source": "paper_2609_00865_gb300/csrc/lmhead_bwd_tc.cu",
         "sha256": "e40ea9e5cf9398f20ba4c0508ee327990b45deed51f17997f7c6d5ea1739b4e8",
     },
     (4, "mw_masked_attn_bwd"): {
         # lsd, compact gather, dQ (main + junction items), dK/dV, per-key reduce
-        "bytes": (1894677760 + 28395264) + (459507712 + 700083456) + (4147593216 + 903136512) +
-                 (515563520 + 6713600) + (4001377024 + 1467339776) + (1502124032 + 262418176),
+        "bytes": (1894792704 + 28215296) + (457391872 + 700431872) + (4153245696 + 902921984) +
+                 (515885568 + 6489344) + (2745335296 + 1457336064) + (1502192128 + 262524160),
         "source": "paper_2609_00865_gb300/csrc/attn_tc.cu",
-        "sha256": "3cad1bdc5f9c23db994b04f0625d5e9263e4bb8f963b2293c31a0e24f726bf06",
+        "sha256": "48d36168ce7bd2c054b9c265005945bbb82edcd5661adb8804942cc689e65178",
     },
 }
 
