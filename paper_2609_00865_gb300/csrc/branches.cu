@@ -93,10 +93,18 @@ __global__ void __launch_bounds__(256) k_branch_unpack_add(VisView v, int vec, c
         }
         __syncthreads();
     }
-    for (int x = threadIdx.x; x < MW_TILE * vec; x += blockDim.x) {
-        const int r = x / vec, k = x - r * vec;
+    // (key r, vector k) of x = r vec + k, advanced by the block size without a
+    // division per step
+    int r = threadIdx.x / vec, k = threadIdx.x - r * vec;
+    const int rstep = blockDim.x / vec, kstep = blockDim.x - rstep * vec;
+    for (; r < MW_TILE; r += rstep, k += kstep) {
+        if (k >= vec) {
+            k -= vec;
+            ++r;
+            if (r >= MW_TILE) break;
+        }
         const int j = kt * MW_TILE + r;
-        if (j >= T_b) continue;
+        if (j >= T_b) break;   // later keys of the tile are past the trajectory too
         float acc[PER];
 #pragma unroll
         for (int q = 0; q < PER; ++q) acc[q] = 0.f;

@@ -541,11 +541,14 @@ __global__ void k_lm_bwd_par(int M, int M_pad, const float* __restrict__ g, cons
 // Exact recomputation of a flagged row of the fused forward (some logit more
 // than kGuard above the row's reference), on CUDA cores: r = the row's largest
 // logit over the whole vocabulary (log2 units), l = sum_v 2^(z_v log2 e - r),
-// E = sum_v 2^(z_v log2 e - r) W_v, the target logit. One block per flagged
-// row (grid-stride over the rows; unflagged rows return at once); warp w takes
-// vocabulary entries w, w + 8, ...; a logit is a warp dot product over d in
-// float32. Both passes form z_v the same way, so the weights of pass 2 are
-// consistent with r and l of pass 1.
+// E = sum_v 2^(z_v log2 e - r) W_v, the target logit. A block takes 256
+// consecutive rows at a time, reads their flags in one load and then works
+// the flagged ones one after another (with none flagged, the usual case, it
+// is done after that load); warp w takes vocabulary entries w, w + 8, ...; a
+// logit is a warp dot product over d in float32. Both passes form z_v the
+// same way, so the weights of pass 2 are consistent with r and l of pass 1.
+// A row's results depend on that row alone, so the order of the flagged rows
+// within a chunk does not change them.
 constexpr int RP_WARPS = 8;
 __global__ void __launch_bounds__(RP_WARPS * 32)
     k_lm_repair(int M, int M_pad, int d, int V, int C, const __nv_bfloat16* __restrict__ Hg,
@@ -555,79 +558,89 @@ __global__ void __launch_bounds__(RP_WARPS * 32)
     float* h = rp_smem;               // [d]
     float* acc = rp_smem + d;         // [RP_WARPS][d]
     __shared__ float wm[RP_WARPS], wl[RP_WARPS];
+    __shared__ int flagged[RP_WARPS * 32];
+    __shared__ int n_flagged;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nvec = d / 8;           // 16-byte vectors of a row
-    for (int m = blockIdx.x; m < M; m += gridDim.x) {
-        if (!flag[m]) continue;       // uniform over the block
-        for (int k = threadIdx.x; k < d; k += blockDim.x) h[k] = __bfloat162float(Hg[(int64_t)m * d + k]);
-        for (int k = threadIdx.x; k < RP_WARPS * d; k += blockDim.x) acc[k] = 0.f;
+    for (int c0 = blockIdx.x * blockDim.x; c0 < M; c0 += gridDim.x * blockDim.x) {
+        if (threadIdx.x == 0) n_flagged = 0;
         __syncthreads();
-        auto logit = [&](int v) -> float {
-            const uint4* wr = reinterpret_cast<const uint4*>(W + (int64_t)v * d);
-            float a = 0.f;
-            for (int k = lane; k < nvec; k += 32) {
-                const uint4 u = __ldg(&wr[k]);
-                const uint32_t w4[4] = {u.x, u.y, u.z, u.w};
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    a = fmaf(__uint_as_float(w4[e] << 16), h[8 * k + 2 * e], a);
-                    a = fmaf(__uint_as_float(w4[e] & 0xffff0000u), h[8 * k + 2 * e + 1], a);
+        if (c0 + (int)threadIdx.x < M && flag[c0 + threadIdx.x]) flagged[atomicAdd(&n_flagged, 1)] = c0 + threadIdx.x;
+        __syncthreads();
+        const int nf = n_flagged;
+        for (int fi = 0; fi < nf; ++fi) {
+            const int m = flagged[fi];    // uniform over the block
+            for (int k = threadIdx.x; k < d; k += blockDim.x) h[k] = __bfloat162float(Hg[(int64_t)m * d + k]);
+            for (int k = threadIdx.x; k < RP_WARPS * d; k += blockDim.x) acc[k] = 0.f;
+            __syncthreads();
+            auto logit = [&](int v) -> float {
+                const uint4* wr = reinterpret_cast<const uint4*>(W + (int64_t)v * d);
+                float a = 0.f;
+                for (int k = lane; k < nvec; k += 32) {
+                    const uint4 u = __ldg(&wr[k]);
+                    const uint32_t w4[4] = {u.x, u.y, u.z, u.w};
+    #pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        a = fmaf(__uint_as_float(w4[e] << 16), h[8 * k + 2 * e], a);
+                        a = fmaf(__uint_as_float(w4[e] & 0xffff0000u), h[8 * k + 2 * e + 1], a);
+                    }
+                }
+                return warp_sum(a);
+            };
+            const int t = tg[m];
+            // pass 1: online (max, sum) per warp, log2 units
+            float mx = -INFINITY, l = 0.f;
+            for (int v = warp; v < V; v += RP_WARPS) {
+                const float z = logit(v);
+                if (v == t && lane == 0) zt[m] = z;
+                const float x = z * LOG2E_B;
+                if (x > mx) {
+                    l = l * exp2f(mx - x) + 1.f;
+                    mx = x;
+                } else {
+                    l += exp2f(x - mx);
                 }
             }
-            return warp_sum(a);
-        };
-        const int t = tg[m];
-        // pass 1: online (max, sum) per warp, log2 units
-        float mx = -INFINITY, l = 0.f;
-        for (int v = warp; v < V; v += RP_WARPS) {
-            const float z = logit(v);
-            if (v == t && lane == 0) zt[m] = z;
-            const float x = z * LOG2E_B;
-            if (x > mx) {
-                l = l * exp2f(mx - x) + 1.f;
-                mx = x;
-            } else {
-                l += exp2f(x - mx);
+            if (lane == 0) {
+                wm[warp] = mx;
+                wl[warp] = l;
             }
-        }
-        if (lane == 0) {
-            wm[warp] = mx;
-            wl[warp] = l;
-        }
-        __syncthreads();
-        float r = -INFINITY;
-        for (int w = 0; w < RP_WARPS; ++w) r = fmaxf(r, wm[w]);
-        float lt = 0.f;
-        for (int w = 0; w < RP_WARPS; ++w) lt += wl[w] > 0.f ? wl[w] * exp2f(wm[w] - r) : 0.f;
-        // pass 2: E = sum_v 2^(z_v log2 e - r) W_v, per warp into its own row of acc
-        float* aw = acc + warp * d;
-        for (int v = warp; v < V; v += RP_WARPS) {
-            const float pv = exp2f(logit(v) * LOG2E_B - r);
-            const uint4* wr = reinterpret_cast<const uint4*>(W + (int64_t)v * d);
-            for (int k = lane; k < nvec; k += 32) {
-                const uint4 u = __ldg(&wr[k]);
-                const uint32_t w4[4] = {u.x, u.y, u.z, u.w};
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    aw[8 * k + 2 * e] = fmaf(pv, __uint_as_float(w4[e] << 16), aw[8 * k + 2 * e]);
-                    aw[8 * k + 2 * e + 1] = fmaf(pv, __uint_as_float(w4[e] & 0xffff0000u), aw[8 * k + 2 * e + 1]);
+            __syncthreads();
+            float r = -INFINITY;
+            for (int w = 0; w < RP_WARPS; ++w) r = fmaxf(r, wm[w]);
+            float lt = 0.f;
+            for (int w = 0; w < RP_WARPS; ++w) lt += wl[w] > 0.f ? wl[w] * exp2f(wm[w] - r) : 0.f;
+            // pass 2: E = sum_v 2^(z_v log2 e - r) W_v, per warp into its own row of acc
+            float* aw = acc + warp * d;
+            for (int v = warp; v < V; v += RP_WARPS) {
+                const float pv = exp2f(logit(v) * LOG2E_B - r);
+                const uint4* wr = reinterpret_cast<const uint4*>(W + (int64_t)v * d);
+                for (int k = lane; k < nvec; k += 32) {
+                    const uint4 u = __ldg(&wr[k]);
+                    const uint32_t w4[4] = {u.x, u.y, u.z, u.w};
+    #pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        aw[8 * k + 2 * e] = fmaf(pv, __uint_as_float(w4[e] << 16), aw[8 * k + 2 * e]);
+                        aw[8 * k + 2 * e + 1] = fmaf(pv, __uint_as_float(w4[e] & 0xffff0000u), aw[8 * k + 2 * e + 1]);
+                    }
                 }
             }
+            __syncthreads();
+            for (int k = threadIdx.x; k < d; k += blockDim.x) {
+                float e = 0.f;
+                for (int w = 0; w < RP_WARPS; ++w) e += acc[w * d + k];
+                E[(int64_t)m * d + k] = e;
+            }
+            if (threadIdx.x == 0) {
+                float4 q = par[m];
+                q.y = r;
+                par[m] = q;
+                lpart[m] = lt;
+                for (int c = 1; c < C; ++c) lpart[(int64_t)c * M_pad + m] = 0.f;
+            }
+            __syncthreads();
         }
-        __syncthreads();
-        for (int k = threadIdx.x; k < d; k += blockDim.x) {
-            float e = 0.f;
-            for (int w = 0; w < RP_WARPS; ++w) e += acc[w * d + k];
-            E[(int64_t)m * d + k] = e;
-        }
-        if (threadIdx.x == 0) {
-            float4 q = par[m];
-            q.y = r;
-            par[m] = q;
-            lpart[m] = lt;
-            for (int c = 1; c < C; ++c) lpart[(int64_t)c * M_pad + m] = 0.f;
-        }
-        __syncthreads();
+        __syncthreads();   // every thread has read n_flagged before the next chunk resets it
     }
 }
 
@@ -900,7 +913,7 @@ mw_status lm_fwd_grp_tc(const void* W, int M, int d, int V, const void* Hg, cons
         return st;
     const int C = group_size(d);
     count_launches(2);
-    k_lm_repair<<<(unsigned)std::min(M, 4 * 152), RP_WARPS * 32, rp_smem, s>>>(
+    k_lm_repair<<<(unsigned)std::min<int64_t>(ceil_div(M, RP_WARPS * 32), 4 * 152), RP_WARPS * 32, rp_smem, s>>>(
         M, M_pad, d, V, C, (const __nv_bfloat16*)Hg, (const __nv_bfloat16*)W, tg, a.flag, (float4*)scratch, a.lpart,
         zt, a.E);
     k_lm_grp_combine<<<(unsigned)ceil_div(M, 256), 256, 0, s>>>(M, M_pad, C, (const float4*)scratch, a.lpart, zt,
