@@ -51,9 +51,9 @@ def _peaks():
 # value it had when the counters were taken.
 TRAFFIC = {
     (4, "mw_logprob_loss_bwd"): {
-        "bytes": 456704 + (79047485952 + 14109122048) + (807879424 + 246768896),   # par, dW pass, dH from E
+        "bytes": 456960 + (85569901056 + 14106740992) + (807919104 + 246921728),   # par, dW pass, dH from E
         "source": "paper_2609_00865_gb300/csrc/lmhead_bwd_tc.cu",
-        "sha256": "e40ea9e5cf9398f20ba4c0508ee327990b45deed51f17997f7c6d5ea1739b4e8",
+        "sha256": "56a02b5f128d1f4b9db9970e594ef9bf271e86f7f2ebd358a2e4d32f744c1b29",
     },
     (4, "mw_masked_attn_bwd"): {
         # lsd, compact gather, dQ (main + junction items), dK/dV, per-key reduce
