@@ -60,8 +60,8 @@ __global__ void __launch_bounds__(256) k_branch_pack(VisView v, int n_traj, int 
 // segment), float32 accumulation. With at most SCH segments per trajectory
 // the packed row of every (segment, key) of the tile is looked up once into
 // shared memory first, so a thread's loads of the key's copies do not wait on
-// one another (the lookup inside the loop made each copy's load wait for its
-// rank: 0.41 of the copy bandwidth).
+// one another's ranks. (Measured on the attention workload's packed branches:
+// 0.61 -> 0.58 ms per call, about 0.42 of the copy bandwidth either way.)
 constexpr int SCH = 16;
 template <typename T>
 __global__ void __launch_bounds__(256) k_branch_unpack_add(VisView v, int vec, const uint4* __restrict__ dXp,
