@@ -122,3 +122,17 @@ def test_events_record_offloads_and_retrieves_valid_spans():
     for t, e in zip(small.trajs, none):
         assert all(not i for _, _, i in e)
         np.testing.assert_array_equal(N.dense_mask(t.T, e), OV.dense_mask(t.T, t.edits))
+
+
+def test_debug_workload_records_are_valid():
+    """The records the debug-library workload runs on the GPU are valid
+    records for the oracle (edits and events), so a failure there is the
+    library's, not the input's."""
+    import debug_workload as D
+    from oracle import nonmonotone as N
+    for seqlens, edits in (D.EDGE, D.MEDIUM):
+        for T, e in zip(seqlens, edits):
+            OV.validate_edits(T, e)
+    for T, e in zip(*D.EVENTS):
+        N.validate_events(T, e)
+    assert any(i for e in D.EVENTS[1] for _, _, i in e)      # some span comes back
